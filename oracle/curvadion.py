@@ -1,0 +1,306 @@
+"""fp64 CPU oracle of one CurvaDion optimizer step (arXiv 2512.13728).
+
+TEST INFRASTRUCTURE ONLY.  This module is the slow, obviously-correct reference that the
+GPU path is checked against.  Only ``tests/``, ``__graft_entry__.smoke()`` and the
+``cpu_baseline`` / ``--impl reference`` legs of ``bench.py`` may import it.  It shares no
+code with the CUDA library and imports nothing from it.
+
+Everything is float64 numpy.  Inputs given in fp32 or bf16 are widened exactly.  Each
+function names the passage of the paper it follows:
+
+* Algorithm 1 (Dion baseline): buffer, power iteration, orthogonalize, error feedback,
+  column normalization, scaled low-rank parameter update.
+* Algorithm 2 (CurvaDion): per-layer RMMC with prev_norm and epsilon, max over layers,
+  strict threshold compare, sync branch = the Dion update, local branch = M <- B, X -= eta_local G.
+* Equation 1: RMMC from the momentum norms of consecutive steps (reported as a diagnostic).
+
+Readings where the paper is silent (each is also listed in the design notes):
+
+* the norm is the Frobenius norm (the proof of Theorem 1 expands ||M_t||^2 as an inner product);
+* R is computed from the orthonormalized P, after Orthogonalize (Algorithm 1 lists P and R
+  as one power-iteration output but reduces R after the orthogonalization);
+* Orthogonalize returns the Q factor of the thin QR of P whose triangular factor has a
+  positive diagonal (unique for full-rank P);
+* ColumnNormalize divides each column by (its 2-norm + eps_col);
+* sqrt(m/n) uses m = rows, n = columns of the parameter matrix X;
+* a non-finite RMMC counts as above every threshold;
+* Equation 1's ratio takes the same epsilon as Algorithm 2 in its denominator so that the
+  first step (zero momentum) is finite;
+* the local branch keeps M = B with no decay, exactly as Algorithm 2 writes it.
+
+Pins: ``tests/test_oracle_pins.py`` checks every function here against results fixed by
+the paper or by mathematics (closed forms, LAPACK, brute force on tiny cases).
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field
+from typing import List, Optional, Sequence
+
+import numpy as np
+
+# Gate modes.  ALWAYS is Algorithm 1 (every step synchronizes; RMMC only reported).
+# GLOBAL is Algorithm 2 (one decision from the max over layers).  PER_LAYER thresholds
+# each layer's own RMMC.  SCHEDULED is the Scheduled Sync Dion baseline of Section 4.3 and Appendix C:
+# synchronize on every H-th step, local updates otherwise.
+GATE_ALWAYS = 0
+GATE_GLOBAL = 1
+GATE_PER_LAYER = 2
+GATE_SCHEDULED = 3
+
+
+def as_f64(a) -> np.ndarray:
+    """Widen an fp32/bf16/fp64 array-like (numpy or torch CPU tensor) to float64 exactly."""
+    if hasattr(a, "detach"):  # torch tensor: bf16 has no numpy dtype, widen through float32
+        import torch  # local import: plain torch CPU ops only
+
+        t = a.detach().cpu()
+        if t.dtype == torch.bfloat16:
+            t = t.to(torch.float32)
+        return t.to(torch.float64).numpy().copy()
+    return np.asarray(a, dtype=np.float64).copy()
+
+
+# ---------------------------------------------------------------------------------------
+# Algorithm 1 / Algorithm 2 building blocks
+# ---------------------------------------------------------------------------------------
+
+def form_buffer(M: np.ndarray, G: np.ndarray) -> np.ndarray:
+    """B_t = M_{t-1} + G_t (Algorithm 1 and Algorithm 2, 'update buffer')."""
+    return M + G
+
+
+def frobenius_norm(A: np.ndarray) -> float:
+    """||A|| read as the Frobenius norm: the square root of the sum of squared entries."""
+    return math.sqrt(float(np.sum(A * A)))
+
+
+def rmmc_alg2(norm_b: float, prev_norm: float, eps: float) -> float:
+    """Algorithm 2's per-layer RMMC: | ||B_t|| - prev_norm | / (prev_norm + eps)."""
+    return abs(norm_b - prev_norm) / (prev_norm + eps)
+
+
+def rmmc_eq1(norm_now: float, norm_before: float, eps: float) -> float:
+    """Equation 1: | ||M(t)|| - ||M(t-1)|| | / ||M(t-1)||, with eps added to the denominator."""
+    return abs(norm_now - norm_before) / (norm_before + eps)
+
+
+def power_iter(B: np.ndarray, Q_prev: np.ndarray) -> np.ndarray:
+    """PowerIter (Algorithm 1): one multiplication of the buffer by the previous right factor, P = B Q_{t-1}."""
+    return B @ Q_prev
+
+
+def householder_qr(A: np.ndarray):
+    """Thin QR of an m x r matrix (m >= r) by Householder reflections.
+
+    Returns (Qf, Rf) with A = Qf Rf, Qf^T Qf = I_r and diag(Rf) >= 0.  This is the
+    Orthogonalize step of Algorithm 1/2 under the positive-diagonal reading.
+    Textbook algorithm: column j is reflected onto a multiple of e_j by
+    H_j = I - 2 v v^T, with v chosen to avoid cancellation; the Q factor is
+    H_0 H_1 ... H_{r-1} applied to the first r columns of the identity.
+    """
+    W = np.array(A, dtype=np.float64, copy=True)
+    m, r = W.shape
+    if r > m:
+        raise ValueError("householder_qr needs m >= r")
+    vs = []
+    for j in range(r):
+        x = W[j:, j]
+        nx = math.sqrt(float(x @ x))
+        v = x.copy()
+        if nx == 0.0:
+            vs.append(None)  # column already zero below the diagonal: H_j = I
+            continue
+        alpha = -nx if x[0] >= 0.0 else nx
+        v[0] -= alpha
+        nv = math.sqrt(float(v @ v))
+        if nv == 0.0:
+            vs.append(None)
+            continue
+        v /= nv
+        W[j:, j:] -= 2.0 * np.outer(v, v @ W[j:, j:])
+        vs.append(v)
+    Rf = np.triu(W[:r, :r])
+    Qf = np.zeros((m, r))
+    Qf[:r, :r] = np.eye(r)
+    for j in reversed(range(r)):
+        v = vs[j]
+        if v is None:
+            continue
+        Qf[j:, :] -= 2.0 * np.outer(v, v @ Qf[j:, :])
+    # Positive-diagonal convention: flip column j of Q and row j of R where R_jj < 0.
+    d = np.where(np.diag(Rf) < 0.0, -1.0, 1.0)
+    return Qf * d[None, :], Rf * d[:, None]
+
+
+def orthogonalize(P: np.ndarray) -> np.ndarray:
+    """Orthogonalize(P) (Algorithm 1/2): the orthonormal Q factor of the thin QR of P."""
+    return householder_qr(P)[0]
+
+
+def column_normalize(R: np.ndarray, eps_col: float) -> np.ndarray:
+    """ColumnNormalize(R) (Algorithm 1/2): column j divided by (||R[:, j]||_2 + eps_col)."""
+    norms = np.sqrt(np.sum(R * R, axis=0))
+    return R / (norms[None, :] + eps_col)
+
+
+@dataclass
+class SyncResult:
+    M: np.ndarray
+    Q: np.ndarray
+    X: np.ndarray
+    P: np.ndarray
+    R: np.ndarray
+
+
+def dion_sync_update(B, Q_prev, X, mu: float, eta: float, eps_col: float) -> SyncResult:
+    """The synchronized branch of Algorithm 2 (= one step of Algorithm 1 after the buffer).
+
+    With one data-parallel worker the two AllReduce_DP lines are the identity.
+      P  = PowerIter(B; Q_{t-1}) = B Q_{t-1}
+      P  = Orthogonalize(P)
+      R  = B^T P
+      M  = B - (1 - mu) P R^T
+      Q  = ColumnNormalize(R)
+      X  = X - eta sqrt(m/n) P Q^T
+    """
+    m, n = B.shape
+    P = orthogonalize(power_iter(B, Q_prev))
+    R = B.T @ P
+    M_new = B - (1.0 - mu) * (P @ R.T)
+    Q_new = column_normalize(R, eps_col)
+    X_new = X - eta * math.sqrt(m / n) * (P @ Q_new.T)
+    return SyncResult(M=M_new, Q=Q_new, X=X_new, P=P, R=R)
+
+
+def local_update(B, G, X, eta_local: float):
+    """The local branch of Algorithm 2: M = B (no decay) and X = X - eta_local G."""
+    return B.copy(), X - eta_local * G
+
+
+# ---------------------------------------------------------------------------------------
+# The gate (Algorithm 2) and a whole multi-layer step
+# ---------------------------------------------------------------------------------------
+
+def above(value: float, tau: float) -> bool:
+    """Strict threshold compare of Algorithm 2 ('> tau'); a non-finite RMMC is above every tau."""
+    return (not math.isfinite(value)) or value > tau
+
+
+def gate(rmmc: Sequence[float], taus: Sequence[float], tau_global: float, mode: int,
+         step: int, period: int):
+    """Sync decisions for one step.
+
+    Returns (flags, global_flag, active): flags[l] = RMMC_l > tau_l, global_flag = max_l RMMC_l > tau_global
+    (Algorithm 2's AllReduce_max over one worker is the max over layers), and active[l] says
+    which layers take the Dion branch under ``mode``.
+    """
+    L = len(rmmc)
+    flags = [above(rmmc[i], taus[i]) for i in range(L)]
+    gmax = -math.inf
+    for v in rmmc:
+        gmax = math.inf if not math.isfinite(v) else max(gmax, v)
+    global_flag = above(gmax, tau_global) if L > 0 else False
+    if mode == GATE_ALWAYS:
+        active = [True] * L
+    elif mode == GATE_GLOBAL:
+        active = [global_flag] * L
+    elif mode == GATE_PER_LAYER:
+        active = list(flags)
+    elif mode == GATE_SCHEDULED:
+        if period < 1:
+            raise ValueError("scheduled gate needs period >= 1")
+        active = [step % period == 0] * L
+    else:
+        raise ValueError(f"unknown gate mode {mode}")
+    return flags, global_flag, active
+
+
+@dataclass
+class LayerState:
+    X: np.ndarray  # m x n parameters
+    M: np.ndarray  # m x n momentum
+    Q: np.ndarray  # n x r right factor
+    tau: float = 0.5
+
+
+@dataclass
+class HParams:
+    mu: float = 0.95
+    eta: float = 0.01
+    eta_local: float = 0.01
+    eps_rmmc: float = 1e-8
+    eps_col: float = 1e-8
+    gate_mode: int = GATE_ALWAYS
+    tau_global: float = 0.5
+    period: int = 1
+
+
+@dataclass
+class StepOutput:
+    layers: List[LayerState]
+    prev_norm: np.ndarray
+    rmmc: np.ndarray
+    rmmc_eq1: np.ndarray
+    flags: np.ndarray
+    global_flag: bool
+    active: np.ndarray
+    norm_b: np.ndarray
+    extras: list = field(default_factory=list)
+
+
+def curvadion_step(layers: Sequence[LayerState], grads: Sequence[np.ndarray],
+                   prev_norm: Sequence[float], hp: HParams, step: int,
+                   keep_extras: bool = False) -> StepOutput:
+    """One step of Algorithm 2 over all layers (Algorithm 1 when hp.gate_mode == GATE_ALWAYS).
+
+    ``step`` is the 1-based t.  Inputs are not modified.  The returned prev_norm holds
+    ||B_t|| per layer, as Algorithm 2 assigns it.
+    """
+    L = len(layers)
+    Bs, nb, rm = [], np.zeros(L), np.zeros(L)
+    norm_m_before = np.zeros(L)
+    for i, (st, G) in enumerate(zip(layers, grads)):
+        M = as_f64(st.M)
+        norm_m_before[i] = frobenius_norm(M)
+        B = form_buffer(M, as_f64(G))
+        Bs.append(B)
+        nb[i] = frobenius_norm(B)
+        rm[i] = rmmc_alg2(nb[i], float(prev_norm[i]), hp.eps_rmmc)
+    flags, gflag, active = gate(rm, [st.tau for st in layers], hp.tau_global, hp.gate_mode,
+                                step, hp.period)
+    out_layers, eq1, extras = [], np.zeros(L), []
+    for i, st in enumerate(layers):
+        X = as_f64(st.X)
+        if active[i]:
+            res = dion_sync_update(Bs[i], as_f64(st.Q), X, hp.mu, hp.eta, hp.eps_col)
+            new = LayerState(X=res.X, M=res.M, Q=res.Q, tau=st.tau)
+            if keep_extras:
+                extras.append(res)
+        else:
+            M_new, X_new = local_update(Bs[i], as_f64(grads[i]), X, hp.eta_local)
+            new = LayerState(X=X_new, M=M_new, Q=as_f64(st.Q), tau=st.tau)
+            if keep_extras:
+                extras.append(None)
+        eq1[i] = rmmc_eq1(frobenius_norm(new.M), norm_m_before[i], hp.eps_rmmc)
+        out_layers.append(new)
+    return StepOutput(layers=out_layers, prev_norm=nb.copy(), rmmc=rm, rmmc_eq1=eq1,
+                      flags=np.array(flags, dtype=bool), global_flag=bool(gflag),
+                      active=np.array(active, dtype=bool), norm_b=nb, extras=extras)
+
+
+def run_trajectory(layers: Sequence[LayerState], grad_fn, steps: int, hp: HParams,
+                   prev_norm: Optional[Sequence[float]] = None):
+    """Run ``steps`` steps from t = 1 (Algorithm 2's loop); grad_fn(layer, t) gives G_t.
+
+    prev_norm starts at 0 for every layer (Algorithm 2's initialization).
+    Returns (final layers, list of StepOutput).
+    """
+    cur = list(layers)
+    pn = np.zeros(len(cur)) if prev_norm is None else np.asarray(prev_norm, dtype=np.float64)
+    outs = []
+    for t in range(1, steps + 1):
+        o = curvadion_step(cur, [grad_fn(i, t) for i in range(len(cur))], pn, hp, t)
+        outs.append(o)
+        cur, pn = o.layers, o.prev_norm
+    return cur, outs
