@@ -1,0 +1,405 @@
+"""Benchmark of one full-model CurvaDion optimizer step on synthetic GPT-shaped layer stacks.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload NAME] [--precision bf16|bf16x3|fp32] [--no-cpu-baseline]
+
+Prints ONE JSON line (rank 0).  A step is dion_step over every layer of the workload (all
+hot-path kernels), with inputs resident in HBM; each step moves far more than the 129 MB
+L2 (36 GB for the 1.3B-shaped stack), so no explicit L2 flush is needed between steps.
+`--impl reference` times the fp64 CPU oracle on the host cores instead (bounded sample).
+Under torchrun (N > 1) every rank runs an independent replica of the full step (the path
+has no data-path exchange on one GPU per replica) and rank 0 reports the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import csv
+import hashlib
+import io
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "ms per full-model Dion+RMMC step (160M/1.3B shapes); % of HBM roofline"
+UNIT = "ms/step"
+DEFAULT_WORKLOAD = "gpt1p3b_stack_r512"
+PREC = {"fp32": 0, "bf16": 1, "bf16x3": 2}
+DTYPE_NAME = {"fp32": "f32", "bf16": "bf16", "bf16x3": "bf16x3"}
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return dict(hbm=p["hbm_gbs"], bf16=p["bf16_tflops"], bf16_sust=p["bf16_tflops_sustained"],
+                    sm_mhz=p.get("sm_max_mhz", 2070.0), source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sust=1700.0, sm_mhz=2070.0, source="fallback")
+
+
+def csrc_hash() -> str:
+    h = hashlib.sha1()
+    d = os.path.join(ROOT, "paper_2512_13728_gb300", "csrc")
+    for name in sorted(os.listdir(d)):
+        with open(os.path.join(d, name), "rb") as f:
+            h.update(name.encode() + f.read())
+    return h.hexdigest()[:12]
+
+
+# ------------------------------------------------------------------ algorithmic work ---
+
+def kernel_work(name: str, w, prec: str):
+    """(bound, algorithmic units per launch, unit) for one kernel of the step, all layers active.
+    Bytes count each compulsory read and write once; flops count 2 per multiply-add."""
+    gsz = 2 if w.g_dtype == "bf16" else 4
+    ranks = w.ranks()
+    mn = sum(m * n for m, n in w.shapes)
+    mnr = sum(m * n * r for (m, n), r in zip(w.shapes, ranks))
+    mr2 = sum(m * r * r for (m, n), r in zip(w.shapes, ranks))
+    r3 = sum(r ** 3 for r in ranks)
+    nr = sum(n * r for (m, n), r in zip(w.shapes, ranks))
+    table = {
+        # CUDA-core path
+        "form_b": ("hbm", mn * (4 + gsz + 4), "B"),
+        "gemm_bq": ("alu", 2 * mnr, "flop"),
+        "gemm_gram": ("alu", 2 * mr2, "flop"),
+        "chol_inv": ("alu", 2 * r3 / 3, "flop"),
+        "gemm_trsm": ("alu", 2 * mr2, "flop"),
+        "gemm_btp": ("alu", 2 * mnr, "flop"),
+        "colnorm": ("hbm", nr * 8, "B"),
+        "update": ("alu", 4 * mnr, "flop") if prec == "fp32" else ("hbm", mn * 16, "B"),
+        "local": ("hbm", 0, "B"),
+        # tensor-core path
+        "tc_form_bq": ("hbm", mn * (4 + gsz + 4), "B"),
+        "tc_btp": ("hbm", mn * 4, "B"),
+        "tc_update": ("hbm", mn * 16, "B"),
+        "tc_gram": ("tensor", 2 * mr2, "flop"),
+        "tc_trsm": ("tensor", 2 * mr2, "flop"),
+    }
+    return table.get(name, ("latency", 0, ""))
+
+
+def step_bytes(w, prec):
+    """Bytes one synchronized step moves by design (the planned passes), and the compulsory floor."""
+    gsz = 2 if w.g_dtype == "bf16" else 4
+    mn = sum(m * n for m, n in w.shapes)
+    planned = mn * ((4 + gsz + 4) + 4 + 16)
+    compulsory = mn * (4 + gsz + 4 + 4 + 4)  # read M, G, X; write M, X
+    return planned, compulsory
+
+
+# ---------------------------------------------------------------------------- clocks ---
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.proc = None
+        self.gpu_id = gpu_id
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", self.gpu_id, f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (FileNotFoundError, OSError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=10)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = [r for r in csv.reader(io.StringIO(out)) if len(r) >= 7]
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[0]))
+                mx.append(float(r[1]))
+            except ValueError:
+                continue
+            for k, v in zip(names, r[3:7]):
+                if v.strip().lower() == "active":
+                    reasons.add(k)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------------- our GPU arm ---
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+
+    import paper_2512_13728_gb300 as cd
+    import workloads as wl
+    from paper_2512_13728_gb300 import build as cdbuild
+
+    if rank == 0 or world == 1:
+        cdbuild.build()
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w = wl.WORKLOADS[args.workload]
+    prec = args.precision
+    gdt = torch.bfloat16 if w.g_dtype == "bf16" else torch.float32
+
+    X, M, Q, G = [], [], [], []
+    for l in range(w.num_layers):
+        x0, m0, q0 = wl.init_layer(w, l, dev)
+        X.append(x0); M.append(m0); Q.append(q0)
+        G.append(wl.gradient(w, l, 1, dev))
+    torch.cuda.synchronize()
+    plan = cd.Plan(X, M, Q, G, [args.tau] * w.num_layers, PREC[prec])
+    gate = {"always": cd.DION_GATE_ALWAYS, "global": cd.DION_GATE_GLOBAL, "per_layer": cd.DION_GATE_PER_LAYER}[args.gate]
+    stream = torch.cuda.current_stream(dev)
+    t = 0
+
+    def one_step():
+        nonlocal t
+        t += 1
+        plan.step(cd.hparams(step=t, gate_mode=gate, tau_global=args.tau), stream=stream.cuda_stream)
+
+    for _ in range(args.warmup):
+        one_step()
+    torch.cuda.synchronize()
+    if plan.device_status() != 0:
+        raise RuntimeError("device status after warm-up: " + cd.native.dion_status_string(plan.device_status()))
+
+    # ---- timed region (device-resident inputs) ----
+    cd.native.dion_timing_enable(plan.handle, args.steps)
+    sampler = None
+    if rank == 0:
+        props = torch.cuda.get_device_properties(dev)
+        uuid = getattr(props, "uuid", None)
+        gid = f"GPU-{uuid}" if uuid is not None and not str(uuid).startswith("GPU-") else (str(uuid) if uuid else
+                                                                                           str(local_rank))
+        sampler = ClockSampler(gid)
+        sampler.start()
+        time.sleep(0.3)
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        one_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop() if sampler else None
+    ms_total = e0.elapsed_time(e1)
+    nsteps_timed, ktimes = cd.native.dion_timing_read(plan.handle)
+    cd.native.dion_timing_enable(plan.handle, 0)
+    if world > 1:
+        tt = torch.tensor([ms_total], device=dev, dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms_total = float(tt.item())
+    if plan.device_status() != 0:
+        raise RuntimeError("device status after timed steps is not OK")
+    ms_step = ms_total / args.steps
+
+    # ---- end to end: H2D of the step's gradient from pinned host memory + step + D2H of results ----
+    host_G = [g.cpu().pin_memory() for g in G]
+    host_out = torch.empty(w.num_layers * 9 + 1, dtype=torch.uint8).pin_memory()
+    h2d = sum(g.numel() * g.element_size() for g in host_G)
+    d2h = plan.rmmc[: w.num_layers].numel() * 8 + w.num_layers + 1
+    e_steps = max(1, min(args.steps, 10))
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    f0.record(stream)
+    for _ in range(e_steps):
+        for g, hg in zip(G, host_G):
+            g.copy_(hg, non_blocking=True)
+        one_step()
+        host_out[: 8 * w.num_layers].copy_(plan.rmmc[: w.num_layers].view(torch.uint8), non_blocking=True)
+        host_out[8 * w.num_layers: 9 * w.num_layers].copy_(plan.flags[: w.num_layers], non_blocking=True)
+        host_out[9 * w.num_layers:].copy_(plan.global_flag, non_blocking=True)
+    f1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = f0.elapsed_time(f1) / e_steps
+    if world > 1:
+        tt = torch.tensor([e2e_ms], device=dev, dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+    launches = plan.launches_per_step()
+    plan.close()
+    if rank != 0:
+        return None
+
+    peaks = load_peaks()
+    kern = []
+    for name, ms in ktimes:
+        bound, units, unit = kernel_work(name, w, prec)
+        kern.append(dict(name=name, ms=ms, bound=bound, units=units, unit=unit))
+    dom = max(kern, key=lambda k: k["ms"]) if kern else None
+    roofline = None
+    if dom is not None:
+        if dom["bound"] == "hbm":
+            peak, punit, achieved = peaks["hbm"], "GB/s", dom["units"] / (dom["ms"] * 1e-3) / 1e9
+        elif dom["bound"] == "tensor":
+            peak, punit, achieved = peaks["bf16_sust"], "TFLOP/s", dom["units"] / (dom["ms"] * 1e-3) / 1e12
+        else:  # fp32 FFMA on CUDA cores: 152 SMs x 128 lanes x 2 flop x max SM clock
+            peak = 152 * 128 * 2 * peaks["sm_mhz"] * 1e6 / 1e12
+            punit, achieved = "TFLOP/s", dom["units"] / (dom["ms"] * 1e-3) / 1e12
+        traffic = None
+        tpath = os.path.join(ROOT, "profiles", "traffic.json")
+        if os.path.exists(tpath):
+            with open(tpath) as f:
+                tj = json.load(f)
+            ent = tj.get(f"{args.workload}:{prec}:{dom['name']}")
+            if ent and ent.get("csrc") == csrc_hash():
+                traffic = ent["bytes_per_launch"]
+        roofline = {"kernel": dom["name"], "bound": dom["bound"], "achieved": round(achieved, 2), "peak": peak,
+                    "unit": punit, "frac": round(achieved / peak, 4), "traffic": traffic,
+                    "peak_source": f"{peaks['source']} ({'sustained bf16' if dom['bound'] == 'tensor' else 'copy' if dom['bound'] == 'hbm' else 'derived'})"}
+    planned, compulsory = step_bytes(w, prec)
+    line = {
+        "metric": METRIC, "value": round(ms_step, 4), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms_step, 4), "higher_is_better": False, "scaling": "weak",
+        "vs_baseline": None, "dtype": DTYPE_NAME[prec], "data": "synthetic",
+        "config": {"workload": args.workload, "layers": w.num_layers, "rank": w.rank, "shapes_per_block":
+                   [list(s) for s in w.shapes[:6]], "gate_mode": args.gate, "precision": prec,
+                   "l2": "no flush: each step streams far more than the 129 MB L2",
+                   "matrices_per_s": round(world * w.num_layers / (ms_step * 1e-3), 1),
+                   "step_hbm_frac_planned_bytes": round(planned / (ms_step * 1e-3) / 1e9 / peaks["hbm"], 4),
+                   "step_hbm_frac_compulsory_bytes": round(compulsory / (ms_step * 1e-3) / 1e9 / peaks["hbm"], 4),
+                   "parallelism": f"replicas x{world}"},
+        "roofline": roofline,
+        "e2e": {"value": round(e2e_ms, 4), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": launches * args.steps,
+        "clocks": clocks,
+        "kernels": [{"name": k["name"], "ms": round(k["ms"], 4)} for k in kern],
+        "timed_steps_with_kernel_events": nsteps_timed,
+    }
+    return line
+
+
+# ------------------------------------------------------------------- CPU (oracle) ---
+
+def oracle_matrix_seconds(w, layer_ids, threads):
+    """Runs the oracle step on the given layers in a child process with `threads` BLAS threads;
+    returns the per-layer seconds."""
+    env = dict(os.environ)
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        env[k] = str(threads)
+    code = ("import json,sys,time\nsys.path.insert(0,%r)\nimport oracle.curvadion as oc, workloads as wl\n"
+            "w=wl.WORKLOADS[%r]\nout=[]\n"
+            "for l in %r:\n"
+            "    X,M,Q=wl.init_layer(w,l)\n    G=wl.gradient(w,l,1)\n"
+            "    lay=oc.LayerState(X=oc.as_f64(X),M=oc.as_f64(M),Q=oc.as_f64(Q))\n    g=oc.as_f64(G)\n"
+            "    t=time.perf_counter()\n    oc.curvadion_step([lay],[g],[0.0],oc.HParams(),1)\n"
+            "    out.append(time.perf_counter()-t)\n"
+            "print(json.dumps(out))\n") % (ROOT, w.name, list(layer_ids))
+    r = subprocess.run([sys.executable, "-c", code], env=env, stdout=subprocess.PIPE, text=True, check=True)
+    return json.loads(r.stdout.strip().splitlines()[-1])
+
+
+def cpu_baseline(args):
+    import workloads as wl
+
+    w = wl.WORKLOADS[args.workload]
+    cores = os.cpu_count() or 1
+    block = list(range(min(6, w.num_layers)))
+    t0 = time.perf_counter()
+    secs = oracle_matrix_seconds(w, block, cores)
+    wall = time.perf_counter() - t0
+    per_matrix = sum(secs) / len(secs)
+    return {"value": round(per_matrix * w.num_layers * 1e3, 1), "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"fp64 numpy oracle, one step of the first {len(block)} matrices (one block) of {w.name}; "
+                      f"value = mean s/matrix x {w.num_layers} matrices; {wall:.1f} s wall"}
+
+
+def run_reference(args, rank):
+    """The oracle as the reference arm: each step runs one matrix of the first block, in rotation."""
+    if rank != 0:
+        return None
+    import workloads as wl
+
+    w = wl.WORKLOADS[args.workload]
+    cores = os.cpu_count() or 1
+    block = min(6, w.num_layers)
+    ids = [i % block for i in range(args.warmup + args.steps)]
+    secs = oracle_matrix_seconds(w, ids, cores)
+    timed = secs[args.warmup:]
+    ms = (sum(timed) / len(timed)) * w.num_layers * 1e3
+    return {"impl": "reference", "metric": METRIC, "value": round(ms, 1), "unit": UNIT, "n_gpus": 1,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 1), "higher_is_better": False,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": args.workload, "layers": w.num_layers, "rank": w.rank, "gate_mode": args.gate},
+            "cpu_baseline": {"value": round(ms, 1), "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"each step: the fp64 oracle on one matrix of the first block of {w.name} "
+                                       f"(rotating over {block} shapes); value = mean s/matrix x {w.num_layers}"},
+            "e2e": {"value": round(ms, 1), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--precision", default=None, choices=list(PREC))
+    ap.add_argument("--gate", default="always", choices=["always", "global", "per_layer"])
+    ap.add_argument("--tau", type=float, default=0.5)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.precision is None:
+        args.precision = os.environ.get("CURVADION_BENCH_PRECISION", "bf16")
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        line = run_reference(args, rank)
+        if line is not None:
+            print(json.dumps(line), flush=True)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    line = run_ours(args, rank, world, local_rank)
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+    if line is None:
+        return
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(args)
+    else:
+        line["cpu_baseline"] = None
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,162 @@
+/*
+ * curvadion.h -- C ABI of the GB300 CurvaDion optimizer-step library.
+ *
+ * One call, dion_step(), runs one optimizer step of CurvaDion (arXiv 2512.13728) over a
+ * stack of matrix layers that live in GPU memory:
+ *
+ *   for every layer l (Algorithm 2):
+ *     B      = M + G                                   buffer ("update buffer" line)
+ *     RMMC_l = | ||B|| - prev_norm_l | / (prev_norm_l + eps_rmmc),  prev_norm_l = ||B||
+ *   g = max_l RMMC_l  (the AllReduce_max over one worker)
+ *   per layer, if it synchronizes (Algorithm 1's body):
+ *     P = B Q;  P = Orthogonalize(P);  R = B^T P
+ *     M = B - (1 - mu) P R^T;  Q = ColumnNormalize(R);  X = X - eta sqrt(m/n) P Q^T
+ *   otherwise (Algorithm 2's local branch):
+ *     M = B;  X = X - eta_local G
+ *
+ * On one GPU the data-parallel AllReduce lines of Algorithms 1 and 2 are the identity and
+ * no collective is issued.  Norms are Frobenius norms.  Orthogonalize returns the Q factor
+ * of the thin QR of P with a positive-diagonal triangular factor (computed by Cholesky QR,
+ * which gives that factor for full-rank P).  ColumnNormalize divides column j of R by
+ * (||R[:, j]||_2 + eps_col).
+ *
+ * Conventions for every entry point:
+ *   - All matrices are row-major.  "ld" arguments are leading dimensions in ELEMENTS.
+ *   - Tensor pointers are DEVICE pointers owned by the caller; the library never frees them.
+ *   - A host-detectable error returns a status != DION_OK and enqueues no work.
+ *   - A device-detected error (see dion_get_device_status) leaves the affected layer's
+ *     outputs unspecified; the other layers are still updated.
+ *   - dion_step only enqueues work on the given stream: it never blocks the host and
+ *     never allocates.  One plan must not be used on two streams at the same time.
+ */
+#ifndef CURVADION_H
+#define CURVADION_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define DION_ABI_VERSION 1
+
+typedef enum {
+  DION_OK = 0,
+  DION_ERR_INVALID_ARG = 1,  /* NULL pointer, bad size, r > min(m, n), unknown enum */
+  DION_ERR_UNSUPPORTED = 2,  /* valid request outside this build's limits (e.g. r > 512) */
+  DION_ERR_ALIGNMENT = 3,    /* pointer or leading dimension breaks the 16-byte rule */
+  DION_ERR_CUDA = 4,         /* a CUDA runtime call failed (no device, launch error, OOM) */
+  DION_ERR_BREAKDOWN = 5,    /* device: Cholesky pivot <= 0 or non-finite (rank-deficient P) */
+  DION_ERR_NONFINITE = 6,    /* device: ||B|| is not finite for some layer */
+  DION_ERR_TIMEOUT = 7       /* device: a bounded wait gave up */
+} dion_status;
+
+/* Which layers run the synchronized Dion branch (Algorithm 1 body) in a step. */
+enum {
+  DION_GATE_ALWAYS = 0,     /* Algorithm 1: every layer, every step; RMMC/flags only reported */
+  DION_GATE_GLOBAL = 1,     /* Algorithm 2: all layers iff max_l RMMC_l > tau_global */
+  DION_GATE_PER_LAYER = 2,  /* layer l iff RMMC_l > tau_l */
+  DION_GATE_SCHEDULED = 3   /* Scheduled Sync Dion (Section 4.3): all layers iff step % period == 0 */
+};
+
+/* Element type of a gradient buffer G. */
+enum { DION_DTYPE_FP32 = 0, DION_DTYPE_BF16 = 1 };
+
+/* Arithmetic of the contractions (B Q, Gram, triangular solve, B^T P, P R^T, P Q^T).
+ * Every mode accumulates in fp32 and keeps M, X, Q in fp32.
+ *   DION_PREC_FP32   : fp32 operands on CUDA cores (FFMA).
+ *   DION_PREC_BF16   : bf16 operands on tcgen05 tensor cores, fp32 accumulators in TMEM.
+ *   DION_PREC_BF16X3 : tcgen05 with each fp32 operand split as hi + lo bf16 and three
+ *                      products (hi*hi + hi*lo + lo*hi): fp32-class accuracy. */
+enum { DION_PREC_FP32 = 0, DION_PREC_BF16 = 1, DION_PREC_BF16X3 = 2 };
+
+/* Largest supported rank r (one 128 x r fp32 accumulator fills the 512 TMEM columns). */
+#define DION_MAX_RANK 512
+
+/* One matrix layer.  X, M: m x n fp32; Q: n x r fp32; G: m x n of g_dtype.
+ * Pointers must be 16-byte aligned and ld * sizeof(element) a multiple of 16 bytes;
+ * ld >= number of columns.  1 <= r <= min(m, n).  The pointers are captured by
+ * dion_plan_create and must stay valid (and unchanged) for the plan's lifetime:
+ * the caller writes each step's gradient into the same G buffer. */
+typedef struct {
+  int64_t m, n, r;
+  float *X;        int64_t ldx;  /* parameters, in/out */
+  float *M;        int64_t ldm;  /* momentum, in/out; M_0 = 0 (Algorithm 2 initialization) */
+  float *Q;        int64_t ldq;  /* right factor Q_{t-1} in, Q_t out (unchanged on local steps) */
+  const void *G;   int64_t ldg;  /* gradient, read only */
+  int32_t g_dtype;               /* DION_DTYPE_* */
+  float tau;                     /* per-layer threshold for DION_GATE_PER_LAYER */
+} dion_layer;
+
+/* Per-step scalars.  Passed by value into the kernels: changing eta every step (a learning
+ * rate schedule) costs nothing. */
+typedef struct {
+  float mu;          /* momentum (paper: 0.95) */
+  float eta;         /* learning rate of the Dion update */
+  float eta_local;   /* learning rate of the local branch */
+  float eps_rmmc;    /* epsilon of Algorithm 2's RMMC denominator (and Equation 1's) */
+  float eps_col;     /* epsilon of ColumnNormalize */
+  float tau_global;  /* threshold on max_l RMMC_l */
+  int32_t gate_mode; /* DION_GATE_* */
+  int32_t period;    /* H of DION_GATE_SCHEDULED (>= 1) */
+  int64_t step;      /* 1-based step index t */
+} dion_hparams;
+
+typedef struct dion_plan dion_plan;
+
+/* Validates the layers, allocates the plan's device workspace (P, R, Gram and factor
+ * buffers, norm partials, tile lists, status word) on the current CUDA device and stores
+ * the layer pointers.  precision: DION_PREC_*.  On success *out owns the workspace until
+ * dion_plan_destroy.  Errors: INVALID_ARG, ALIGNMENT, UNSUPPORTED, CUDA (allocation). */
+dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32_t precision,
+                             dion_plan **out);
+
+/* Enqueues one step on `stream` (a cudaStream_t; NULL = legacy default stream).
+ *   prev_norm       device double[L], in/out: Algorithm 2's prev_norm_l (start at 0)
+ *   rmmc_out        device double[L], out: Algorithm 2's RMMC_l of this step
+ *   rmmc_eq1_out    device double[L] or NULL, out: Equation 1's RMMC from ||M_t||, ||M_{t-1}||
+ *                   (with eps_rmmc added to the denominator)
+ *   sync_flags_out  device uint8[L], out: 1 iff RMMC_l > tau_l (non-finite counts as above)
+ *   global_flag_out device uint8[1], out: 1 iff max_l RMMC_l > tau_global
+ * Which layers take the Dion branch follows hp->gate_mode; the decision is made on the
+ * device, so the host never waits.  Errors: INVALID_ARG, CUDA (launch failure). */
+dion_status dion_step(dion_plan *plan, const dion_hparams *hp, double *prev_norm,
+                      double *rmmc_out, double *rmmc_eq1_out, uint8_t *sync_flags_out,
+                      uint8_t *global_flag_out, void *stream);
+
+/* Reads the plan's device status word (synchronously; call after the step's stream has
+ * been synchronized) into *code_out as a dion_status, and clears it if `clear` != 0.
+ * The first device error of any step since the last clear is kept. */
+dion_status dion_get_device_status(dion_plan *plan, int32_t clear, int32_t *code_out);
+
+/* Number of kernel launches one dion_step enqueues for this plan. */
+int32_t dion_step_launch_count(const dion_plan *plan);
+
+/* Per-launch timing with CUDA events (measurement support; not part of the paper's method).
+ * dion_timing_enable(plan, max_steps): while max_steps > 0, every dion_step records one CUDA
+ * event before its first launch and one after each launch, on the step's stream, for up to
+ * max_steps steps (events are created here, so this call may allocate; dion_step does not).
+ * max_steps = 0 disables timing and frees the events.
+ * dion_timing_read(plan, cap, ms_out, names_out, count_out): synchronizes on the recorded
+ * events, writes the average duration in milliseconds of each launch position over the
+ * recorded steps (ms_out[i], names_out[i] = static kernel name) for i < min(cap, launches),
+ * sets *count_out to the number of launches per step and to 0 steps recorded afterwards.
+ * Errors: INVALID_ARG (NULL plan/outputs), CUDA. */
+dion_status dion_timing_enable(dion_plan *plan, int32_t max_steps);
+dion_status dion_timing_read(dion_plan *plan, int32_t cap, float *ms_out, const char **names_out,
+                             int32_t *count_out, int32_t *steps_out);
+
+/* Frees the plan's workspace (synchronizes the device first).  NULL is a no-op. */
+void dion_plan_destroy(dion_plan *plan);
+
+/* Static description of a status code. */
+const char *dion_status_string(dion_status status);
+
+/* DION_ABI_VERSION of the loaded library. */
+int32_t dion_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CURVADION_H */

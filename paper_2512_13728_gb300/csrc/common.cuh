@@ -1,0 +1,134 @@
+// Internal declarations shared by the kernels and the host runtime of the CurvaDion library.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+
+struct dion_plan;
+
+namespace cd {
+
+// Step-sequence timing hooks (plan.cu): no-ops unless dion_timing_enable was called.
+void tick_begin(dion_plan *p, cudaStream_t s);
+void tick(dion_plan *p, cudaStream_t s, const char *name);
+void tick_end(dion_plan *p);
+
+// Status codes mirror dion_status in include/curvadion.h.
+enum : int32_t {
+  ST_OK = 0,
+  ST_BREAKDOWN = 5,
+  ST_NONFINITE = 6,
+  ST_TIMEOUT = 7,
+};
+
+enum : int32_t { GATE_ALWAYS = 0, GATE_GLOBAL = 1, GATE_PER_LAYER = 2, GATE_SCHEDULED = 3 };
+enum : int32_t { DT_FP32 = 0, DT_BF16 = 1 };
+enum : int32_t { PREC_FP32 = 0, PREC_BF16 = 1, PREC_BF16X3 = 2 };
+
+// One layer as the kernels see it: the caller's tensors plus this layer's workspace.
+struct DevLayer {
+  int64_t m, n, r;
+  float *X;
+  int64_t ldx;
+  float *M;  // holds B = M + G between the buffer kernel and the update kernel
+  int64_t ldm;
+  float *Q;
+  int64_t ldq;
+  const void *G;
+  int64_t ldg;
+  int32_t g_dtype;
+  float tau;
+  float sqrt_m_over_n;
+  int32_t pad0;
+  // workspace (row-major, leading dimension r unless stated)
+  float *P_raw;  // m x r   P = B Q before orthogonalization
+  float *P;      // m x r   orthonormal P
+  float *R;      // n x r   R = B^T P
+  float *S;      // r x r   Gram P_raw^T P_raw; lower triangle becomes the Cholesky factor L
+  float *Linv;   // r x r   L^{-1} (lower triangular, zeros above the diagonal)
+  // tensor-core operand copies (bf16, K-major, padded leading dimensions); unused in FP32 mode
+  __nv_bfloat16 *Qt_hi, *Qt_lo;  // r x ldqt : Q_{t-1}^T split into hi + lo
+  __nv_bfloat16 *Pt_hi, *Pt_lo;  // r x ldpt : P^T
+  __nv_bfloat16 *P_hi, *P_lo;    // m x r    : P (row-major, K = r contiguous)
+  __nv_bfloat16 *R_hi, *R_lo;    // n x r    : R
+  __nv_bfloat16 *Qn_hi, *Qn_lo;  // n x r    : Q_t
+  int64_t ldqt, ldpt;
+  int32_t bpart_off, bpart_cnt;  // slots of the ||B||^2 / ||M_{t-1}||^2 partials
+  int32_t upart_off, upart_cnt;  // slots of the ||M_t||^2 partials
+};
+
+// Per-step scalars and output pointers, passed by value to the kernels.
+struct StepArgs {
+  float mu, eta, eta_local, eps_rmmc, eps_col, tau_global;
+  int32_t gate_mode, period;
+  int64_t step;
+  double *prev_norm;
+  double *rmmc;
+  double *eq1;  // may be null
+  uint8_t *flags;
+  uint8_t *gflag;
+};
+
+// Workspace shared by all kernels of a plan.
+struct Shared {
+  DevLayer *layers;
+  int32_t num_layers;
+  uint8_t *active;       // [L] 1 = layer takes the Dion branch this step
+  double *bpart;         // [2 * row tiles] per tile: sum B^2, sum M_{t-1}^2
+  double *upart;         // [update tiles]  per tile: sum M_t^2
+  double *norm_m_before; // [L]
+  double *norm_b;        // [L]
+  int32_t *status;       // [1] first device error
+};
+
+// A contraction C = op(A) op(B) for the CUDA-core path.
+// op(A)[i][k] = transA ? A[k*lda + i] : A[i*lda + k]   (i < Mrows, k < K)
+// op(B)[k][j] = transB ? B[j*ldb + k] : B[k*ldb + j]   (k < K, j < Ncols)
+struct GemmProblem {
+  const float *A;
+  const float *B;
+  float *C;
+  int64_t Mrows, Ncols, K, lda, ldb, ldc;
+  int32_t transA, transB, layer, pad;
+};
+
+__device__ __forceinline__ void set_status(int32_t *st, int32_t code) { atomicCAS(st, 0, code); }
+
+__device__ __forceinline__ float bf16_bits_to_float(uint32_t bits16) {
+  return __uint_as_float(bits16 << 16);
+}
+
+// Deterministic block sum of one double per thread (fixed shuffle tree + fixed warp order).
+template <int THREADS>
+__device__ __forceinline__ double block_sum(double v, double *red /* >= THREADS/32 */) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  double s = 0.0;
+  if (threadIdx.x == 0) {
+    for (int w = 0; w < THREADS / 32; ++w) s += red[w];
+  }
+  __syncthreads();
+  return s;  // valid in thread 0
+}
+
+// ---------------------------------------------------------------- launch wrappers ---
+// CUDA-core (fp32) kernels, kernels_simt.cu
+void launch_form_b(const Shared &sh, const int4 *tiles, int32_t ntiles, cudaStream_t s);
+void launch_gate(const Shared &sh, const StepArgs &a, cudaStream_t s);
+void launch_gemm(const Shared &sh, const GemmProblem *probs, const int4 *tiles, int32_t ntiles,
+                 cudaStream_t s);
+cudaError_t prepare_chol_inv(int32_t max_r, size_t *smem_out);
+void launch_chol_inv(const Shared &sh, size_t smem, cudaStream_t s);
+void launch_colnorm(const Shared &sh, const int4 *tiles, int32_t ntiles, float eps_col,
+                    cudaStream_t s);
+void launch_update(const Shared &sh, const int4 *tiles, int32_t ntiles, float mu, float eta,
+                   cudaStream_t s);
+void launch_local(const Shared &sh, const int4 *tiles, int32_t ntiles, float eta_local,
+                  cudaStream_t s);
+void launch_finalize(const Shared &sh, const StepArgs &a, cudaStream_t s);
+
+}  // namespace cd

@@ -1,0 +1,589 @@
+// CUDA-core kernels of the CurvaDion step (fp32 operands, fp32 FMA, fp64 partial sums).
+//
+// These kernels serve the DION_PREC_FP32 mode end to end, and the buffer, gate, Cholesky,
+// column-normalization, local-branch and finalize steps of every mode.  Every kernel reads
+// its work list (tiles) from device memory and skips layers whose `active` flag says they
+// do not take the Dion branch this step, so one fixed launch sequence serves every gate
+// decision without a host round trip.
+#include "common.cuh"
+
+#include <cmath>
+
+namespace cd {
+
+// ===================================================================== buffer + norms ===
+// B = M + G written into M (Algorithm 1/2 buffer line); per tile, sum of B^2 (Algorithm 2's
+// ||B_t||) and sum of M_{t-1}^2 (Equation 1's ||M(t-1)||) as fp64 partials in a fixed slot.
+// Tile = {layer, first row, rows, slot}.
+constexpr int kRowThreads = 256;
+
+template <int GT>
+__device__ __forceinline__ void load_g4(const void *G, int64_t off, float g[4]) {
+  if (GT == DT_BF16) {
+    const uint2 v = *reinterpret_cast<const uint2 *>(static_cast<const __nv_bfloat16 *>(G) + off);
+    g[0] = bf16_bits_to_float(v.x & 0xffffu);
+    g[1] = bf16_bits_to_float(v.x >> 16);
+    g[2] = bf16_bits_to_float(v.y & 0xffffu);
+    g[3] = bf16_bits_to_float(v.y >> 16);
+  } else {
+    const float4 v = *reinterpret_cast<const float4 *>(static_cast<const float *>(G) + off);
+    g[0] = v.x; g[1] = v.y; g[2] = v.z; g[3] = v.w;
+  }
+}
+
+template <int GT>
+__device__ __forceinline__ float load_g1(const void *G, int64_t off) {
+  if (GT == DT_BF16) return __bfloat162float(static_cast<const __nv_bfloat16 *>(G)[off]);
+  return static_cast<const float *>(G)[off];
+}
+
+template <int GT>
+__device__ void form_b_tile(const DevLayer &L, int64_t row0, int64_t nrows, float sb[4], float sm[4]) {
+  const int64_t n = L.n, n4 = n >> 2;
+  for (int64_t rr = 0; rr < nrows; ++rr) {
+    const int64_t i = row0 + rr;
+    float *Mrow = L.M + i * L.ldm;
+    const int64_t goff = i * L.ldg;
+    for (int64_t c4 = threadIdx.x; c4 < n4; c4 += kRowThreads) {
+      float4 m = *reinterpret_cast<float4 *>(Mrow + 4 * c4);
+      float g[4];
+      load_g4<GT>(L.G, goff + 4 * c4, g);
+      sm[0] = fmaf(m.x, m.x, sm[0]); sm[1] = fmaf(m.y, m.y, sm[1]);
+      sm[2] = fmaf(m.z, m.z, sm[2]); sm[3] = fmaf(m.w, m.w, sm[3]);
+      m.x += g[0]; m.y += g[1]; m.z += g[2]; m.w += g[3];
+      sb[0] = fmaf(m.x, m.x, sb[0]); sb[1] = fmaf(m.y, m.y, sb[1]);
+      sb[2] = fmaf(m.z, m.z, sb[2]); sb[3] = fmaf(m.w, m.w, sb[3]);
+      *reinterpret_cast<float4 *>(Mrow + 4 * c4) = m;
+    }
+    for (int64_t c = 4 * n4 + threadIdx.x; c < n; c += kRowThreads) {
+      const float mo = Mrow[c];
+      const float b = mo + load_g1<GT>(L.G, goff + c);
+      sm[0] = fmaf(mo, mo, sm[0]);
+      sb[0] = fmaf(b, b, sb[0]);
+      Mrow[c] = b;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kRowThreads) form_b_kernel(Shared sh, const int4 *tiles) {
+  __shared__ double red[kRowThreads / 32];
+  const int4 t = tiles[blockIdx.x];
+  const DevLayer &L = sh.layers[t.x];
+  float sb[4] = {0.f, 0.f, 0.f, 0.f}, sm[4] = {0.f, 0.f, 0.f, 0.f};
+  if (L.g_dtype == DT_BF16) form_b_tile<DT_BF16>(L, t.y, t.z, sb, sm);
+  else form_b_tile<DT_FP32>(L, t.y, t.z, sb, sm);
+  const double b = block_sum<kRowThreads>(((double)sb[0] + sb[1]) + ((double)sb[2] + sb[3]), red);
+  const double mo = block_sum<kRowThreads>(((double)sm[0] + sm[1]) + ((double)sm[2] + sm[3]), red);
+  if (threadIdx.x == 0) {
+    sh.bpart[2 * t.w] = b;
+    sh.bpart[2 * t.w + 1] = mo;
+  }
+}
+
+void launch_form_b(const Shared &sh, const int4 *tiles, int32_t ntiles, cudaStream_t s) {
+  if (ntiles > 0) form_b_kernel<<<ntiles, kRowThreads, 0, s>>>(sh, tiles);
+}
+
+// =============================================================================== gate ===
+// Algorithm 2: RMMC_l = | ||B|| - prev_l | / (prev_l + eps); prev_l = ||B||; global max over
+// layers; strict compare with tau (a non-finite RMMC counts as above every threshold); the
+// gate mode then decides which layers take the Dion branch.
+constexpr int kGateThreads = 1024;
+
+__device__ __forceinline__ bool above(double v, float tau) {
+  return !isfinite(v) || v > (double)tau;
+}
+
+__global__ void __launch_bounds__(kGateThreads) gate_kernel(Shared sh, StepArgs a) {
+  __shared__ double wmax[kGateThreads / 32];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int L = sh.num_layers;
+  double my_max = -INFINITY;
+  for (int l = warp; l < L; l += kGateThreads / 32) {
+    const DevLayer &Ly = sh.layers[l];
+    double sb = 0.0, sm = 0.0;
+    for (int k = lane; k < Ly.bpart_cnt; k += 32) {  // fixed lane/slot assignment
+      sb += sh.bpart[2 * (Ly.bpart_off + k)];
+      sm += sh.bpart[2 * (Ly.bpart_off + k) + 1];
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      sb += __shfl_xor_sync(0xffffffffu, sb, o);
+      sm += __shfl_xor_sync(0xffffffffu, sm, o);
+    }
+    if (lane == 0) {
+      const double nb = sqrt(sb);
+      const double prev = a.prev_norm[l];
+      const double rm = fabs(nb - prev) / (prev + (double)a.eps_rmmc);
+      if (!isfinite(nb)) set_status(sh.status, ST_NONFINITE);
+      a.rmmc[l] = rm;
+      a.prev_norm[l] = nb;
+      a.flags[l] = above(rm, Ly.tau) ? 1 : 0;
+      sh.norm_b[l] = nb;
+      sh.norm_m_before[l] = sqrt(sm);
+      my_max = isfinite(rm) ? fmax(my_max, rm) : INFINITY;
+    }
+  }
+  if (lane == 0) wmax[warp] = my_max;
+  __syncthreads();  // makes the per-layer global writes above visible to the whole block
+  __shared__ int gflag_s;
+  if (threadIdx.x == 0) {
+    double g = -INFINITY;
+    for (int w = 0; w < kGateThreads / 32; ++w) g = fmax(g, wmax[w]);
+    const int gf = (L > 0 && above(g, a.tau_global)) ? 1 : 0;
+    a.gflag[0] = (uint8_t)gf;
+    gflag_s = gf;
+  }
+  __syncthreads();
+  for (int l = threadIdx.x; l < L; l += kGateThreads) {
+    int act;
+    switch (a.gate_mode) {
+      case GATE_ALWAYS: act = 1; break;
+      case GATE_GLOBAL: act = gflag_s; break;
+      case GATE_PER_LAYER: act = a.flags[l]; break;
+      default: act = (a.step % a.period) == 0; break;
+    }
+    sh.active[l] = (uint8_t)act;
+  }
+}
+
+void launch_gate(const Shared &sh, const StepArgs &a, cudaStream_t s) {
+  gate_kernel<<<1, kGateThreads, 0, s>>>(sh, a);
+}
+
+// ==================================================================== grouped GEMM ===
+// C = op(A) op(B) over a list of problems; 64 x 64 output tiles, 16-deep k slices staged in
+// shared memory, 4 x 4 register tile per thread.  Tile = {problem, tile row, tile col}.
+constexpr int GBM = 64, GBN = 64, GBK = 16, kGemmThreads = 256;
+
+__global__ void __launch_bounds__(kGemmThreads) gemm_kernel(Shared sh, const GemmProblem *probs,
+                                                            const int4 *tiles) {
+  const int4 t = tiles[blockIdx.x];
+  const GemmProblem p = probs[t.x];
+  if (!sh.active[p.layer]) return;
+  __shared__ float As[GBK][GBM + 4];
+  __shared__ float Bs[GBK][GBN + 4];
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  const int64_t i0 = (int64_t)t.y * GBM, j0 = (int64_t)t.z * GBN;
+  float acc[4][4] = {};
+  for (int64_t k0 = 0; k0 < p.K; k0 += GBK) {
+#pragma unroll
+    for (int s = 0; s < (GBM * GBK) / kGemmThreads; ++s) {
+      const int idx = tid + s * kGemmThreads;
+      int ii, kk;
+      if (p.transA) { ii = idx % GBM; kk = idx / GBM; } else { kk = idx % GBK; ii = idx / GBK; }
+      const int64_t gi = i0 + ii, gk = k0 + kk;
+      float v = 0.f;
+      if (gi < p.Mrows && gk < p.K) v = p.transA ? p.A[gk * p.lda + gi] : p.A[gi * p.lda + gk];
+      As[kk][ii] = v;
+    }
+#pragma unroll
+    for (int s = 0; s < (GBN * GBK) / kGemmThreads; ++s) {
+      const int idx = tid + s * kGemmThreads;
+      int jj, kk;
+      if (p.transB) { kk = idx % GBK; jj = idx / GBK; } else { jj = idx % GBN; kk = idx / GBN; }
+      const int64_t gj = j0 + jj, gk = k0 + kk;
+      float v = 0.f;
+      if (gj < p.Ncols && gk < p.K) v = p.transB ? p.B[gj * p.ldb + gk] : p.B[gk * p.ldb + gj];
+      Bs[kk][jj] = v;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < GBK; ++kk) {
+      float av[4], bv[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) av[i] = As[kk][ty * 4 + i];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) bv[j] = Bs[kk][tx * 4 + j];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int64_t gi = i0 + ty * 4 + i;
+    if (gi >= p.Mrows) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int64_t gj = j0 + tx * 4 + j;
+      if (gj < p.Ncols) p.C[gi * p.ldc + gj] = acc[i][j];
+    }
+  }
+}
+
+void launch_gemm(const Shared &sh, const GemmProblem *probs, const int4 *tiles, int32_t ntiles,
+                 cudaStream_t s) {
+  if (ntiles > 0) gemm_kernel<<<ntiles, kGemmThreads, 0, s>>>(sh, probs, tiles);
+}
+
+// =========================================================== Cholesky + L^{-1} ===
+// Orthogonalize by Cholesky QR: S = P^T P = L L^T, P_orth = P L^{-T}.  For full-rank P this
+// is the Q factor of the thin QR with a positive-diagonal triangular factor.  One CTA per
+// layer factors S (r <= 512) by right-looking blocked Cholesky with 32-wide block columns,
+// then inverts L block row by block row.  S and L^{-1} stay in global memory (L2-resident);
+// diagonal blocks, panels and partial products are staged in shared memory.
+// A pivot <= 0 or non-finite sets DION_ERR_BREAKDOWN and makes L^{-1} = 0 for that layer,
+// so the layer's P, R and Q become 0, M becomes B and X is unchanged (no NaN is written).
+constexpr int CB = 32, CBP = CB + 1, kCholThreads = 512;
+
+__device__ __forceinline__ int64_t tri_row(int64_t p) {
+  // largest b with b (b + 1) / 2 <= p
+  int64_t b = (int64_t)((sqrt(8.0 * (double)p + 1.0) - 1.0) * 0.5);
+  while ((b + 1) * (b + 2) / 2 <= p) ++b;
+  while (b * (b + 1) / 2 > p) --b;
+  return b;
+}
+
+__global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh) {
+  const int l = blockIdx.x;
+  if (!sh.active[l]) return;
+  const DevLayer &Ly = sh.layers[l];
+  const int r = (int)Ly.r;
+  float *S = Ly.S;
+  float *Li = Ly.Linv;
+  extern __shared__ float smem[];
+  float *D = smem;            // CB x CBP: diagonal block / its inverse
+  float *DI = D + CB * CBP;   // CB x CBP
+  float *Pn = DI + CB * CBP;  // panel (r x CBP) or partial products (CB x r)
+  __shared__ int bad;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (tid == 0) bad = 0;
+  __syncthreads();
+
+  // ---------------- Cholesky: S lower triangle <- L ----------------
+  for (int k0 = 0; k0 < r; k0 += CB) {
+    const int nb = min(CB, r - k0);
+    for (int e = tid; e < CB * CB; e += kCholThreads) {
+      const int i = e / CB, j = e % CB;
+      float v;
+      if (i < nb && j < nb) v = (j <= i) ? S[(int64_t)(k0 + i) * r + k0 + j] : 0.f;
+      else v = (i == j) ? 1.f : 0.f;  // identity padding of a short last block
+      D[i * CBP + j] = v;
+    }
+    __syncthreads();
+    if (warp == 0) {
+      for (int j = 0; j < CB; ++j) {
+        const float djj = D[j * CBP + j];
+        if (!(djj > 0.f) || !isfinite(djj)) {
+          if (lane == 0) bad = 1;
+          break;  // uniform across the warp: every lane read the same djj
+        }
+        const float s = sqrtf(djj);
+        __syncwarp();
+        if (lane == j) D[j * CBP + j] = s;
+        if (lane > j) D[lane * CBP + j] /= s;
+        __syncwarp();
+        if (lane > j) {
+          const float lij = D[lane * CBP + j];
+          for (int k = j + 1; k <= lane; ++k) D[lane * CBP + k] -= lij * D[k * CBP + j];
+        }
+        __syncwarp();
+      }
+    }
+    __syncthreads();
+    if (bad) break;
+    for (int e = tid; e < nb * nb; e += kCholThreads) {
+      const int i = e / nb, j = e % nb;
+      if (j <= i) S[(int64_t)(k0 + i) * r + k0 + j] = D[i * CBP + j];
+    }
+    // panel: rows below the block solve x L11^T = s
+    const int t = r - k0 - nb;
+    for (int ii = tid; ii < t; ii += kCholThreads) {
+      const int64_t row = (int64_t)(k0 + nb + ii) * r + k0;
+      float x[CB];
+#pragma unroll
+      for (int j = 0; j < CB; ++j) x[j] = (j < nb) ? S[row + j] : 0.f;
+#pragma unroll
+      for (int j = 0; j < CB; ++j) {
+        float v = x[j];
+#pragma unroll
+        for (int k = 0; k < j; ++k) v -= x[k] * D[j * CBP + k];
+        x[j] = v / D[j * CBP + j];
+      }
+#pragma unroll
+      for (int j = 0; j < CB; ++j) {
+        Pn[ii * CBP + j] = x[j];
+        if (j < nb) S[row + j] = x[j];
+      }
+    }
+    __syncthreads();
+    // trailing update of the lower triangle: S22 -= L21 L21^T, in 4 x 4 micro tiles
+    const int64_t nbt = (t + 3) / 4, pairs = nbt * (nbt + 1) / 2;
+    for (int64_t pidx = tid; pidx < pairs; pidx += kCholThreads) {
+      const int64_t bi = tri_row(pidx), bj = pidx - bi * (bi + 1) / 2;
+      float acc[4][4] = {};
+#pragma unroll 8
+      for (int k = 0; k < CB; ++k) {
+        float a[4], b[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int64_t ri = bi * 4 + u, rj = bj * 4 + u;
+          a[u] = (ri < t) ? Pn[ri * CBP + k] : 0.f;
+          b[u] = (rj < t) ? Pn[rj * CBP + k] : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(a[u], b[v], acc[u][v]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int64_t ri = bi * 4 + u;
+        if (ri >= t) continue;
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          const int64_t rj = bj * 4 + v;
+          if (rj < t && rj <= ri) S[(k0 + nb + ri) * r + k0 + nb + rj] -= acc[u][v];
+        }
+      }
+    }
+    __syncthreads();
+  }
+
+  if (bad) {
+    if (tid == 0) set_status(sh.status, ST_BREAKDOWN);
+    for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) Li[e] = 0.f;
+    return;
+  }
+
+  // ---------------- L^{-1}, block row by block row ----------------
+  // Linv[I,I] = L[I,I]^{-1};  Linv[I,J] = -L[I,I]^{-1} sum_{K=J..I-1} L[I,K] Linv[K,J]  (J < I)
+  for (int I0 = 0; I0 < r; I0 += CB) {
+    const int nb = min(CB, r - I0);
+    for (int e = tid; e < CB * CB; e += kCholThreads) {
+      const int i = e / CB, j = e % CB;
+      float v;
+      if (i < nb && j < nb) v = (j <= i) ? S[(int64_t)(I0 + i) * r + I0 + j] : 0.f;
+      else v = (i == j) ? 1.f : 0.f;
+      D[i * CBP + j] = v;
+    }
+    __syncthreads();
+    if (warp == 0) {  // lane c solves L_II x = e_c
+      float x[CB];
+#pragma unroll
+      for (int i = 0; i < CB; ++i) {
+        float v = (i == lane) ? 1.f : 0.f;
+#pragma unroll
+        for (int k = 0; k < i; ++k) v -= D[i * CBP + k] * x[k];
+        x[i] = v / D[i * CBP + i];
+      }
+#pragma unroll
+      for (int i = 0; i < CB; ++i) DI[i * CBP + lane] = x[i];
+    }
+    // T[i][c] = sum_{k=c}^{I0-1} L[I0+i][k] Linv[k][c]   for c < I0
+    for (int e = tid; e < CB * I0; e += kCholThreads) {
+      const int i = e / I0, c = e % I0;
+      float v = 0.f;
+      if (i < nb) {
+        const float *Lrow = S + (int64_t)(I0 + i) * r;
+        for (int k = c; k < I0; ++k) v = fmaf(Lrow[k], Li[(int64_t)k * r + c], v);
+      }
+      Pn[i * r + c] = v;
+    }
+    __syncthreads();
+    // Linv row block I: -DI T for c < I0, DI on the diagonal block, 0 to the right
+    for (int e = tid; e < nb * r; e += kCholThreads) {
+      const int i = e / r, c = e % r;
+      float v = 0.f;
+      if (c < I0) {
+        for (int j = 0; j <= i; ++j) v -= DI[i * CBP + j] * Pn[j * r + c];
+      } else if (c < I0 + nb) {
+        const int j = c - I0;
+        v = (j <= i) ? DI[i * CBP + j] : 0.f;
+      }
+      Li[(int64_t)(I0 + i) * r + c] = v;
+    }
+    __syncthreads();
+  }
+}
+
+cudaError_t prepare_chol_inv(int32_t max_r, size_t *smem_out) {
+  const int64_t big = (int64_t)max_r * CBP > (int64_t)CB * max_r ? (int64_t)max_r * CBP : (int64_t)CB * max_r;
+  const size_t smem = sizeof(float) * (2 * CB * CBP + big);
+  *smem_out = smem;
+  return cudaFuncSetAttribute(chol_inv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+}
+
+void launch_chol_inv(const Shared &sh, size_t smem, cudaStream_t s) {
+  if (sh.num_layers > 0) chol_inv_kernel<<<sh.num_layers, kCholThreads, smem, s>>>(sh);
+}
+
+// ===================================================================== ColumnNormalize ===
+// Q_t[:, j] = R[:, j] / (||R[:, j]||_2 + eps_col).  Tile = {layer, 32-column group}; lane =
+// column, warps stride over rows; fp32 sums of 16 rows folded into fp64 in a fixed order.
+constexpr int kColThreads = 256;
+
+__global__ void __launch_bounds__(kColThreads) colnorm_kernel(Shared sh, const int4 *tiles, float eps_col) {
+  const int4 t = tiles[blockIdx.x];
+  if (!sh.active[t.x]) return;
+  const DevLayer &L = sh.layers[t.x];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t j = (int64_t)t.y * 32 + lane, n = L.n, r = L.r;
+  __shared__ double part[kColThreads / 32][32];
+  __shared__ float inv[32];
+  double acc = 0.0;
+  if (j < r) {
+    float f = 0.f;
+    int cnt = 0;
+    for (int64_t i = warp; i < n; i += kColThreads / 32) {
+      const float v = L.R[i * r + j];
+      f = fmaf(v, v, f);
+      if (++cnt == 16) { acc += f; f = 0.f; cnt = 0; }
+    }
+    acc += f;
+  }
+  part[warp][lane] = acc;
+  __syncthreads();
+  if (warp == 0) {
+    double s = 0.0;
+    for (int w = 0; w < kColThreads / 32; ++w) s += part[w][lane];
+    inv[lane] = (float)(1.0 / (sqrt(s) + (double)eps_col));
+  }
+  __syncthreads();
+  if (j < r) {
+    const float c = inv[lane];
+    for (int64_t i = warp; i < n; i += kColThreads / 32) L.Q[i * L.ldq + j] = L.R[i * r + j] * c;
+  }
+}
+
+void launch_colnorm(const Shared &sh, const int4 *tiles, int32_t ntiles, float eps_col, cudaStream_t s) {
+  if (ntiles > 0) colnorm_kernel<<<ntiles, kColThreads, 0, s>>>(sh, tiles, eps_col);
+}
+
+// =============================================================== error feedback + update ===
+// M = B - (1 - mu) P R^T and X = X - eta sqrt(m/n) P Q_t^T in one pass over the tile, plus the
+// fp64 partial of ||M_t||^2 for Equation 1.  Tile = {layer, tile row, tile col, slot}.
+constexpr int UBM = 64, UBN = 64, UBK = 16, kUpdThreads = 256;
+
+__global__ void __launch_bounds__(kUpdThreads) update_kernel(Shared sh, const int4 *tiles, float mu, float eta) {
+  __shared__ float As[UBK][UBM + 4];
+  __shared__ float Rs[UBK][UBN + 4];
+  __shared__ float Qs[UBK][UBN + 4];
+  __shared__ double red[kUpdThreads / 32];
+  const int4 t = tiles[blockIdx.x];
+  if (!sh.active[t.x]) return;
+  const DevLayer &L = sh.layers[t.x];
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  const int64_t i0 = (int64_t)t.y * UBM, j0 = (int64_t)t.z * UBN, r = L.r;
+  float u1[4][4] = {}, u2[4][4] = {};
+  for (int64_t k0 = 0; k0 < r; k0 += UBK) {
+#pragma unroll
+    for (int s = 0; s < (UBM * UBK) / kUpdThreads; ++s) {
+      const int idx = tid + s * kUpdThreads;
+      const int kk = idx % UBK, ii = idx / UBK;
+      const int64_t gk = k0 + kk, gi = i0 + ii, gj = j0 + ii;
+      As[kk][ii] = (gi < L.m && gk < r) ? L.P[gi * r + gk] : 0.f;
+      Rs[kk][ii] = (gj < L.n && gk < r) ? L.R[gj * r + gk] : 0.f;
+      Qs[kk][ii] = (gj < L.n && gk < r) ? L.Q[gj * L.ldq + gk] : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < UBK; ++kk) {
+      float a[4], b[4], q[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) a[i] = As[kk][ty * 4 + i];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) { b[j] = Rs[kk][tx * 4 + j]; q[j] = Qs[kk][tx * 4 + j]; }
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          u1[i][j] = fmaf(a[i], b[j], u1[i][j]);
+          u2[i][j] = fmaf(a[i], q[j], u2[i][j]);
+        }
+    }
+    __syncthreads();
+  }
+  const float dec = 1.f - mu, c = eta * L.sqrt_m_over_n;
+  float ss = 0.f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int64_t gi = i0 + ty * 4 + i;
+    if (gi >= L.m) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int64_t gj = j0 + tx * 4 + j;
+      if (gj >= L.n) continue;
+      float *mp = L.M + gi * L.ldm + gj;
+      const float mn = fmaf(-dec, u1[i][j], *mp);
+      *mp = mn;
+      float *xp = L.X + gi * L.ldx + gj;
+      *xp = fmaf(-c, u2[i][j], *xp);
+      ss = fmaf(mn, mn, ss);
+    }
+  }
+  const double tot = block_sum<kUpdThreads>((double)ss, red);
+  if (tid == 0) sh.upart[t.w] = tot;
+}
+
+void launch_update(const Shared &sh, const int4 *tiles, int32_t ntiles, float mu, float eta, cudaStream_t s) {
+  if (ntiles > 0) update_kernel<<<ntiles, kUpdThreads, 0, s>>>(sh, tiles, mu, eta);
+}
+
+// ======================================================================== local branch ===
+// Algorithm 2's else-branch: M = B is already in place; X = X - eta_local G.
+template <int GT>
+__device__ void local_tile(const DevLayer &L, int64_t row0, int64_t nrows, float eta_local) {
+  const int64_t n = L.n, n4 = n >> 2;
+  for (int64_t rr = 0; rr < nrows; ++rr) {
+    const int64_t i = row0 + rr;
+    float *Xrow = L.X + i * L.ldx;
+    const int64_t goff = i * L.ldg;
+    for (int64_t c4 = threadIdx.x; c4 < n4; c4 += kRowThreads) {
+      float4 x = *reinterpret_cast<float4 *>(Xrow + 4 * c4);
+      float g[4];
+      load_g4<GT>(L.G, goff + 4 * c4, g);
+      x.x = fmaf(-eta_local, g[0], x.x); x.y = fmaf(-eta_local, g[1], x.y);
+      x.z = fmaf(-eta_local, g[2], x.z); x.w = fmaf(-eta_local, g[3], x.w);
+      *reinterpret_cast<float4 *>(Xrow + 4 * c4) = x;
+    }
+    for (int64_t c = 4 * n4 + threadIdx.x; c < n; c += kRowThreads)
+      Xrow[c] = fmaf(-eta_local, load_g1<GT>(L.G, goff + c), Xrow[c]);
+  }
+}
+
+__global__ void __launch_bounds__(kRowThreads) local_kernel(Shared sh, const int4 *tiles, float eta_local) {
+  const int4 t = tiles[blockIdx.x];
+  if (sh.active[t.x]) return;
+  const DevLayer &L = sh.layers[t.x];
+  if (L.g_dtype == DT_BF16) local_tile<DT_BF16>(L, t.y, t.z, eta_local);
+  else local_tile<DT_FP32>(L, t.y, t.z, eta_local);
+}
+
+void launch_local(const Shared &sh, const int4 *tiles, int32_t ntiles, float eta_local, cudaStream_t s) {
+  if (ntiles > 0) local_kernel<<<ntiles, kRowThreads, 0, s>>>(sh, tiles, eta_local);
+}
+
+// ============================================================================ finalize ===
+// Equation 1: | ||M_t|| - ||M_{t-1}|| | / (||M_{t-1}|| + eps).  ||M_t|| comes from the update
+// kernel's partials on synchronized layers and equals ||B_t|| on local layers (M = B).
+__global__ void __launch_bounds__(kGateThreads) finalize_kernel(Shared sh, StepArgs a) {
+  if (a.eq1 == nullptr) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int l = warp; l < sh.num_layers; l += kGateThreads / 32) {
+    const DevLayer &Ly = sh.layers[l];
+    double nm;
+    if (sh.active[l]) {
+      double s = 0.0;
+      for (int k = lane; k < Ly.upart_cnt; k += 32) s += sh.upart[Ly.upart_off + k];
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+      nm = sqrt(s);
+    } else {
+      nm = sh.norm_b[l];
+    }
+    if (lane == 0) {
+      const double before = sh.norm_m_before[l];
+      a.eq1[l] = fabs(nm - before) / (before + (double)a.eps_rmmc);
+    }
+  }
+}
+
+void launch_finalize(const Shared &sh, const StepArgs &a, cudaStream_t s) {
+  if (a.eq1 != nullptr) finalize_kernel<<<1, kGateThreads, 0, s>>>(sh, a);
+}
+
+}  // namespace cd

@@ -1,0 +1,421 @@
+// Host runtime and C ABI of the CurvaDion library: plan creation (validation, workspace,
+// tile lists), the per-step launch sequence, device status and teardown.
+#include "../../include/curvadion.h"
+#include "common.cuh"
+#include "tc.cuh"
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <new>
+#include <vector>
+
+using namespace cd;
+
+struct dion_plan {
+  int device = 0;
+  int32_t L = 0;
+  int32_t precision = PREC_FP32;
+  int32_t max_r = 0;
+  int num_sms = 0;
+  void *ws = nullptr;  // one device allocation holding everything below
+  Shared sh{};
+  // tile lists (device)
+  int4 *btiles = nullptr;
+  int32_t n_btiles = 0;  // buffer / local row tiles
+  int4 *utiles = nullptr;
+  int32_t n_utiles = 0;  // update tiles
+  int4 *ctiles = nullptr;
+  int32_t n_ctiles = 0;  // column-normalization tiles
+  GemmProblem *probs[4] = {nullptr, nullptr, nullptr, nullptr};
+  int4 *gtiles[4] = {nullptr, nullptr, nullptr, nullptr};
+  int32_t n_gtiles[4] = {0, 0, 0, 0};
+  size_t chol_smem = 0;
+  tc::TcPlan tcp{};  // tensor-core path (BF16 / BF16X3)
+  int32_t launches_per_step = 0;
+  // per-launch timing (dion_timing_enable)
+  std::vector<cudaEvent_t> ev;  // [max_steps][launches + 1]
+  std::vector<const char *> names;
+  int32_t timing_steps = 0, recorded = 0, cursor = 0;
+};
+
+namespace cd {
+// Called by the step sequences: records the event that closes launch `cursor` when timing is on.
+void tick(dion_plan *p, cudaStream_t s, const char *name) {
+  if (p->timing_steps <= 0 || p->recorded >= p->timing_steps) return;
+  const int32_t per = p->launches_per_step + 1;
+  if (p->cursor < p->launches_per_step) {
+    if ((int32_t)p->names.size() < p->launches_per_step) p->names.resize(p->launches_per_step, "");
+    p->names[p->cursor] = name;
+    cudaEventRecord(p->ev[(size_t)p->recorded * per + p->cursor + 1], s);
+  }
+  ++p->cursor;
+}
+void tick_begin(dion_plan *p, cudaStream_t s) {
+  p->cursor = 0;
+  if (p->timing_steps <= 0 || p->recorded >= p->timing_steps) return;
+  cudaEventRecord(p->ev[(size_t)p->recorded * (p->launches_per_step + 1)], s);
+}
+void tick_end(dion_plan *p) {
+  if (p->timing_steps <= 0 || p->recorded >= p->timing_steps) return;
+  ++p->recorded;
+}
+}  // namespace cd
+
+namespace {
+
+constexpr size_t kAlign = 256;
+
+struct Carver {
+  size_t off = 0;
+  template <class T>
+  size_t take(size_t count) {
+    off = (off + kAlign - 1) / kAlign * kAlign;
+    const size_t at = off;
+    off += count * sizeof(T);
+    return at;
+  }
+};
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+dion_status validate_layer(const dion_layer &ly) {
+  if (ly.m < 1 || ly.n < 1 || ly.r < 1) return DION_ERR_INVALID_ARG;
+  if (ly.r > std::min(ly.m, ly.n)) return DION_ERR_INVALID_ARG;
+  if (ly.r > DION_MAX_RANK) return DION_ERR_UNSUPPORTED;
+  if (ly.m > (int64_t(1) << 31) - 1 || ly.n > (int64_t(1) << 31) - 1) return DION_ERR_UNSUPPORTED;
+  if (!ly.X || !ly.M || !ly.Q || !ly.G) return DION_ERR_INVALID_ARG;
+  if (ly.g_dtype != DION_DTYPE_FP32 && ly.g_dtype != DION_DTYPE_BF16) return DION_ERR_INVALID_ARG;
+  if (ly.ldx < ly.n || ly.ldm < ly.n || ly.ldg < ly.n || ly.ldq < ly.r) return DION_ERR_INVALID_ARG;
+  if (!std::isfinite(ly.tau)) {
+    if (!(ly.tau > 0)) return DION_ERR_INVALID_ARG;  // +inf allowed (never above), NaN/-inf not
+  }
+  const int64_t gsz = ly.g_dtype == DION_DTYPE_BF16 ? 2 : 4;
+  if (!aligned16(ly.X) || !aligned16(ly.M) || !aligned16(ly.Q) || !aligned16(ly.G))
+    return DION_ERR_ALIGNMENT;
+  if ((ly.ldx * 4) % 16 || (ly.ldm * 4) % 16 || (ly.ldq * 4) % 16 || (ly.ldg * gsz) % 16)
+    return DION_ERR_ALIGNMENT;
+  return DION_OK;
+}
+
+template <class T>
+cudaError_t upload(T *dst, const std::vector<T> &src) {
+  if (src.empty()) return cudaSuccess;
+  return cudaMemcpy(dst, src.data(), src.size() * sizeof(T), cudaMemcpyHostToDevice);
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t dion_abi_version(void) { return DION_ABI_VERSION; }
+
+const char *dion_status_string(dion_status s) {
+  switch (s) {
+    case DION_OK: return "DION_OK";
+    case DION_ERR_INVALID_ARG: return "DION_ERR_INVALID_ARG: invalid argument";
+    case DION_ERR_UNSUPPORTED: return "DION_ERR_UNSUPPORTED: outside this build's limits";
+    case DION_ERR_ALIGNMENT: return "DION_ERR_ALIGNMENT: pointer or leading dimension not 16-byte aligned";
+    case DION_ERR_CUDA: return "DION_ERR_CUDA: CUDA runtime error";
+    case DION_ERR_BREAKDOWN: return "DION_ERR_BREAKDOWN: Cholesky breakdown (rank-deficient P)";
+    case DION_ERR_NONFINITE: return "DION_ERR_NONFINITE: non-finite buffer norm";
+    case DION_ERR_TIMEOUT: return "DION_ERR_TIMEOUT: bounded device wait gave up";
+  }
+  return "unknown dion_status";
+}
+
+dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32_t precision,
+                             dion_plan **out) {
+  if (out == nullptr) return DION_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (num_layers < 0 || (num_layers > 0 && layers == nullptr)) return DION_ERR_INVALID_ARG;
+  if (precision != DION_PREC_FP32 && precision != DION_PREC_BF16 && precision != DION_PREC_BF16X3)
+    return DION_ERR_INVALID_ARG;
+  for (int32_t l = 0; l < num_layers; ++l) {
+    const dion_status st = validate_layer(layers[l]);
+    if (st != DION_OK) return st;
+  }
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return DION_ERR_CUDA;
+  int sms = 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return DION_ERR_CUDA;
+
+  dion_plan *p = new (std::nothrow) dion_plan();
+  if (!p) return DION_ERR_CUDA;
+  p->device = dev;
+  p->L = num_layers;
+  p->precision = precision;
+  p->num_sms = sms;
+
+  // ---- host-side layout of the workspace ----
+  Carver cv;
+  std::vector<DevLayer> dl(num_layers);
+  std::vector<size_t> o_Praw(num_layers), o_P(num_layers), o_R(num_layers), o_S(num_layers), o_Li(num_layers);
+  std::vector<int4> bt, ut, ct;
+  for (int32_t l = 0; l < num_layers; ++l) {
+    const dion_layer &ly = layers[l];
+    DevLayer &d = dl[l];
+    std::memset(&d, 0, sizeof(d));
+    d.m = ly.m; d.n = ly.n; d.r = ly.r;
+    d.X = ly.X; d.ldx = ly.ldx;
+    d.M = ly.M; d.ldm = ly.ldm;
+    d.Q = ly.Q; d.ldq = ly.ldq;
+    d.G = ly.G; d.ldg = ly.ldg; d.g_dtype = ly.g_dtype;
+    d.tau = ly.tau;
+    d.sqrt_m_over_n = (float)std::sqrt((double)ly.m / (double)ly.n);
+    p->max_r = std::max<int32_t>(p->max_r, (int32_t)ly.r);
+    o_Praw[l] = cv.take<float>(ly.m * ly.r);
+    o_P[l] = cv.take<float>(ly.m * ly.r);
+    o_R[l] = cv.take<float>(ly.n * ly.r);
+    o_S[l] = cv.take<float>(ly.r * ly.r);
+    o_Li[l] = cv.take<float>(ly.r * ly.r);
+    // row tiles of about 64K elements for the buffer and local kernels
+    const int64_t rows = std::max<int64_t>(1, std::min<int64_t>(ly.m, 65536 / ly.n));
+    d.bpart_off = (int32_t)bt.size();
+    for (int64_t r0 = 0; r0 < ly.m; r0 += rows)
+      bt.push_back(make_int4(l, (int)r0, (int)std::min(rows, ly.m - r0), (int)bt.size()));
+    d.bpart_cnt = (int32_t)bt.size() - d.bpart_off;
+    // 64 x 64 update tiles
+    d.upart_off = (int32_t)ut.size();
+    for (int64_t ti = 0; ti < (ly.m + 63) / 64; ++ti)
+      for (int64_t tj = 0; tj < (ly.n + 63) / 64; ++tj)
+        ut.push_back(make_int4(l, (int)ti, (int)tj, (int)ut.size()));
+    d.upart_cnt = (int32_t)ut.size() - d.upart_off;
+    for (int64_t cg = 0; cg < (ly.r + 31) / 32; ++cg) ct.push_back(make_int4(l, (int)cg, 0, 0));
+  }
+  // GEMM problems of the CUDA-core path: 0 P_raw = B Q, 1 S = P_raw^T P_raw,
+  // 2 P = P_raw L^{-T}, 3 R = B^T P.
+  std::vector<GemmProblem> gp[4];
+  std::vector<int4> gt[4];
+  const size_t o_layers = cv.take<DevLayer>(std::max(num_layers, 1));
+  const size_t o_active = cv.take<uint8_t>(std::max(num_layers, 1));
+  const size_t o_bpart = cv.take<double>(2 * std::max<size_t>(bt.size(), 1));
+  const size_t o_upart = cv.take<double>(std::max<size_t>(ut.size(), 1));
+  const size_t o_nmb = cv.take<double>(std::max(num_layers, 1));
+  const size_t o_nb = cv.take<double>(std::max(num_layers, 1));
+  const size_t o_status = cv.take<int32_t>(1);
+  const size_t o_bt = cv.take<int4>(std::max<size_t>(bt.size(), 1));
+  const size_t o_ut = cv.take<int4>(std::max<size_t>(ut.size(), 1));
+  const size_t o_ct = cv.take<int4>(std::max<size_t>(ct.size(), 1));
+  // tensor-core workspace (operand copies, tile lists); sized by the tc module
+  tc::TcLayout tcl{};
+  if (precision != DION_PREC_FP32) {
+    const dion_status st = tc::layout(layers, num_layers, precision, sms, cv.off, &tcl);
+    if (st != DION_OK) {
+      delete p;
+      return st;
+    }
+    cv.off = tcl.end;
+  }
+  // GEMM problem/tile arrays are sized after the problem lists are known; reserve below.
+  size_t o_gp[4], o_gt[4];
+  for (int k = 0; k < 4; ++k) {
+    for (int32_t l = 0; l < num_layers; ++l) {
+      const dion_layer &ly = layers[l];
+      GemmProblem q{};
+      q.layer = l;
+      switch (k) {
+        case 0: q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.n; q.lda = ly.ldm; q.ldb = ly.ldq; q.ldc = ly.r; break;
+        case 1: q.Mrows = ly.r; q.Ncols = ly.r; q.K = ly.m; q.lda = ly.r; q.ldb = ly.r; q.ldc = ly.r; q.transA = 1; break;
+        case 2: q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.r; q.lda = ly.r; q.ldb = ly.r; q.ldc = ly.r; q.transB = 1; break;
+        default: q.Mrows = ly.n; q.Ncols = ly.r; q.K = ly.m; q.lda = ly.ldm; q.ldb = ly.r; q.ldc = ly.r; q.transA = 1; break;
+      }
+      const int32_t pi = (int32_t)gp[k].size();
+      gp[k].push_back(q);
+      for (int64_t ti = 0; ti < (q.Mrows + 63) / 64; ++ti)
+        for (int64_t tj = 0; tj < (q.Ncols + 63) / 64; ++tj) gt[k].push_back(make_int4(pi, (int)ti, (int)tj, 0));
+    }
+    o_gp[k] = cv.take<GemmProblem>(std::max<size_t>(gp[k].size(), 1));
+    o_gt[k] = cv.take<int4>(std::max<size_t>(gt[k].size(), 1));
+  }
+
+  if (cudaMalloc(&p->ws, cv.off) != cudaSuccess) {
+    delete p;
+    return DION_ERR_CUDA;
+  }
+  char *base = static_cast<char *>(p->ws);
+  for (int32_t l = 0; l < num_layers; ++l) {
+    dl[l].P_raw = reinterpret_cast<float *>(base + o_Praw[l]);
+    dl[l].P = reinterpret_cast<float *>(base + o_P[l]);
+    dl[l].R = reinterpret_cast<float *>(base + o_R[l]);
+    dl[l].S = reinterpret_cast<float *>(base + o_S[l]);
+    dl[l].Linv = reinterpret_cast<float *>(base + o_Li[l]);
+  }
+  if (precision != DION_PREC_FP32) tc::bind(tcl, base, dl.data(), num_layers, &p->tcp);
+  for (int k = 0; k < 4; ++k) {
+    for (auto &q : gp[k]) {
+      const DevLayer &d = dl[q.layer];
+      switch (k) {
+        case 0: q.A = d.M; q.B = d.Q; q.C = d.P_raw; break;
+        case 1: q.A = d.P_raw; q.B = d.P_raw; q.C = d.S; break;
+        case 2: q.A = d.P_raw; q.B = d.Linv; q.C = d.P; break;
+        default: q.A = d.M; q.B = d.P; q.C = d.R; break;
+      }
+    }
+    p->probs[k] = reinterpret_cast<GemmProblem *>(base + o_gp[k]);
+    p->gtiles[k] = reinterpret_cast<int4 *>(base + o_gt[k]);
+    p->n_gtiles[k] = (int32_t)gt[k].size();
+  }
+  p->sh.layers = reinterpret_cast<DevLayer *>(base + o_layers);
+  p->sh.num_layers = num_layers;
+  p->sh.active = reinterpret_cast<uint8_t *>(base + o_active);
+  p->sh.bpart = reinterpret_cast<double *>(base + o_bpart);
+  p->sh.upart = reinterpret_cast<double *>(base + o_upart);
+  p->sh.norm_m_before = reinterpret_cast<double *>(base + o_nmb);
+  p->sh.norm_b = reinterpret_cast<double *>(base + o_nb);
+  p->sh.status = reinterpret_cast<int32_t *>(base + o_status);
+  p->btiles = reinterpret_cast<int4 *>(base + o_bt);
+  p->n_btiles = (int32_t)bt.size();
+  p->utiles = reinterpret_cast<int4 *>(base + o_ut);
+  p->n_utiles = (int32_t)ut.size();
+  p->ctiles = reinterpret_cast<int4 *>(base + o_ct);
+  p->n_ctiles = (int32_t)ct.size();
+
+  cudaError_t e = cudaSuccess;
+  if (e == cudaSuccess) e = upload(p->sh.layers, dl);
+  if (e == cudaSuccess) e = upload(p->btiles, bt);
+  if (e == cudaSuccess) e = upload(p->utiles, ut);
+  if (e == cudaSuccess) e = upload(p->ctiles, ct);
+  for (int k = 0; k < 4 && e == cudaSuccess; ++k) {
+    e = upload(p->probs[k], gp[k]);
+    if (e == cudaSuccess) e = upload(p->gtiles[k], gt[k]);
+  }
+  if (e == cudaSuccess) e = cudaMemset(p->sh.status, 0, sizeof(int32_t));
+  if (e == cudaSuccess && num_layers > 0) e = prepare_chol_inv(p->max_r, &p->chol_smem);
+  if (e == cudaSuccess && precision != DION_PREC_FP32) e = tc::init(tcl, dl.data(), num_layers, &p->tcp);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    cudaFree(p->ws);
+    delete p;
+    return DION_ERR_CUDA;
+  }
+  p->launches_per_step = (precision == DION_PREC_FP32) ? 11 : tc::launches_per_step(p->tcp);
+  *out = p;
+  return DION_OK;
+}
+
+dion_status dion_step(dion_plan *p, const dion_hparams *hp, double *prev_norm, double *rmmc_out,
+                      double *rmmc_eq1_out, uint8_t *sync_flags_out, uint8_t *global_flag_out,
+                      void *stream) {
+  if (!p || !hp || !prev_norm || !rmmc_out || !sync_flags_out || !global_flag_out) return DION_ERR_INVALID_ARG;
+  if (hp->gate_mode < DION_GATE_ALWAYS || hp->gate_mode > DION_GATE_SCHEDULED) return DION_ERR_INVALID_ARG;
+  if (hp->gate_mode == DION_GATE_SCHEDULED && hp->period < 1) return DION_ERR_INVALID_ARG;
+  if (hp->step < 1) return DION_ERR_INVALID_ARG;
+  if (!std::isfinite(hp->mu) || !std::isfinite(hp->eta) || !std::isfinite(hp->eta_local) ||
+      !std::isfinite(hp->eps_rmmc) || !std::isfinite(hp->eps_col) || std::isnan(hp->tau_global))
+    return DION_ERR_INVALID_ARG;
+  if (hp->eps_rmmc < 0.f || hp->eps_col < 0.f) return DION_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  StepArgs a{};
+  a.mu = hp->mu; a.eta = hp->eta; a.eta_local = hp->eta_local;
+  a.eps_rmmc = hp->eps_rmmc; a.eps_col = hp->eps_col; a.tau_global = hp->tau_global;
+  a.gate_mode = hp->gate_mode; a.period = hp->period < 1 ? 1 : hp->period; a.step = hp->step;
+  a.prev_norm = prev_norm; a.rmmc = rmmc_out; a.eq1 = rmmc_eq1_out;
+  a.flags = sync_flags_out; a.gflag = global_flag_out;
+  const Shared &sh = p->sh;
+  int cur = -1;
+  if (cudaGetDevice(&cur) != cudaSuccess || cur != p->device) {
+    if (cudaSetDevice(p->device) != cudaSuccess) return DION_ERR_CUDA;
+  }
+  tick_begin(p, s);
+  if (p->precision == DION_PREC_FP32) {
+    launch_form_b(sh, p->btiles, p->n_btiles, s);
+    tick(p, s, "form_b");
+    launch_gate(sh, a, s);
+    tick(p, s, "gate");
+    launch_gemm(sh, p->probs[0], p->gtiles[0], p->n_gtiles[0], s);  // P = B Q
+    tick(p, s, "gemm_bq");
+    launch_gemm(sh, p->probs[1], p->gtiles[1], p->n_gtiles[1], s);  // S = P^T P
+    tick(p, s, "gemm_gram");
+    launch_chol_inv(sh, p->chol_smem, s);                           // L, L^{-1}
+    tick(p, s, "chol_inv");
+    launch_gemm(sh, p->probs[2], p->gtiles[2], p->n_gtiles[2], s);  // P = P L^{-T}
+    tick(p, s, "gemm_trsm");
+    launch_gemm(sh, p->probs[3], p->gtiles[3], p->n_gtiles[3], s);  // R = B^T P
+    tick(p, s, "gemm_btp");
+    launch_colnorm(sh, p->ctiles, p->n_ctiles, a.eps_col, s);       // Q = ColumnNormalize(R)
+    tick(p, s, "colnorm");
+    launch_update(sh, p->utiles, p->n_utiles, a.mu, a.eta, s);      // M, X
+    tick(p, s, "update");
+    launch_local(sh, p->btiles, p->n_btiles, a.eta_local, s);       // local branch
+    tick(p, s, "local");
+    launch_finalize(sh, a, s);                                      // Equation 1
+    tick(p, s, "finalize");
+  } else {
+    tc::step(p, p->tcp, sh, a, p->btiles, p->n_btiles, p->ctiles, p->n_ctiles, p->chol_smem, s);
+  }
+  tick_end(p);
+  if (cudaGetLastError() != cudaSuccess) return DION_ERR_CUDA;
+  if (cur >= 0 && cur != p->device) cudaSetDevice(cur);
+  return DION_OK;
+}
+
+dion_status dion_get_device_status(dion_plan *p, int32_t clear, int32_t *code_out) {
+  if (!p || !code_out) return DION_ERR_INVALID_ARG;
+  int32_t v = 0;
+  if (cudaMemcpy(&v, p->sh.status, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return DION_ERR_CUDA;
+  if (clear && cudaMemset(p->sh.status, 0, sizeof(int32_t)) != cudaSuccess) return DION_ERR_CUDA;
+  *code_out = v;
+  return DION_OK;
+}
+
+int32_t dion_step_launch_count(const dion_plan *p) { return p ? p->launches_per_step : 0; }
+
+static void free_events(dion_plan *p) {
+  for (cudaEvent_t e : p->ev) cudaEventDestroy(e);
+  p->ev.clear();
+  p->timing_steps = p->recorded = 0;
+}
+
+dion_status dion_timing_enable(dion_plan *p, int32_t max_steps) {
+  if (!p || max_steps < 0) return DION_ERR_INVALID_ARG;
+  if (cudaDeviceSynchronize() != cudaSuccess) return DION_ERR_CUDA;
+  free_events(p);
+  if (max_steps == 0) return DION_OK;
+  const size_t count = (size_t)max_steps * (p->launches_per_step + 1);
+  p->ev.resize(count);
+  for (size_t i = 0; i < count; ++i) {
+    if (cudaEventCreate(&p->ev[i]) != cudaSuccess) {
+      p->ev.resize(i);
+      free_events(p);
+      return DION_ERR_CUDA;
+    }
+  }
+  p->timing_steps = max_steps;
+  p->recorded = 0;
+  return DION_OK;
+}
+
+dion_status dion_timing_read(dion_plan *p, int32_t cap, float *ms_out, const char **names_out, int32_t *count_out,
+                             int32_t *steps_out) {
+  if (!p || !count_out || !steps_out || (cap > 0 && (!ms_out || !names_out))) return DION_ERR_INVALID_ARG;
+  const int32_t per = p->launches_per_step + 1;
+  const int32_t n = std::min(cap, p->launches_per_step);
+  for (int32_t i = 0; i < n; ++i) {
+    double tot = 0.0;
+    for (int32_t st = 0; st < p->recorded; ++st) {
+      float ms = 0.f;
+      if (cudaEventSynchronize(p->ev[(size_t)st * per + i + 1]) != cudaSuccess) return DION_ERR_CUDA;
+      if (cudaEventElapsedTime(&ms, p->ev[(size_t)st * per + i], p->ev[(size_t)st * per + i + 1]) != cudaSuccess)
+        return DION_ERR_CUDA;
+      tot += ms;
+    }
+    ms_out[i] = p->recorded ? (float)(tot / p->recorded) : 0.f;
+    names_out[i] = i < (int32_t)p->names.size() ? p->names[i] : "";
+  }
+  *count_out = p->launches_per_step;
+  *steps_out = p->recorded;
+  p->recorded = 0;
+  return DION_OK;
+}
+
+void dion_plan_destroy(dion_plan *p) {
+  if (!p) return;
+  cudaDeviceSynchronize();
+  free_events(p);
+  tc::destroy(&p->tcp);
+  cudaFree(p->ws);
+  delete p;
+}
+
+}  // extern "C"

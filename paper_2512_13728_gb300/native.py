@@ -1,0 +1,165 @@
+"""ctypes binding of include/curvadion.h: the same entry points, argument marshalling only.
+
+Every computation happens inside libcurvadion.so.  Loading fails loudly when the library
+has not been built; there is no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "libcurvadion.so")
+
+DION_OK = 0
+DION_ERR_INVALID_ARG = 1
+DION_ERR_UNSUPPORTED = 2
+DION_ERR_ALIGNMENT = 3
+DION_ERR_CUDA = 4
+DION_ERR_BREAKDOWN = 5
+DION_ERR_NONFINITE = 6
+DION_ERR_TIMEOUT = 7
+
+DION_GATE_ALWAYS = 0
+DION_GATE_GLOBAL = 1
+DION_GATE_PER_LAYER = 2
+DION_GATE_SCHEDULED = 3
+
+DION_DTYPE_FP32 = 0
+DION_DTYPE_BF16 = 1
+
+DION_PREC_FP32 = 0
+DION_PREC_BF16 = 1
+DION_PREC_BF16X3 = 2
+
+DION_MAX_RANK = 512
+
+# Every function declared in include/curvadion.h.
+EXPORTED = ("dion_plan_create", "dion_step", "dion_get_device_status", "dion_step_launch_count",
+            "dion_timing_enable", "dion_timing_read", "dion_plan_destroy", "dion_status_string",
+            "dion_abi_version")
+
+
+class dion_layer(C.Structure):
+    _fields_ = [
+        ("m", C.c_int64), ("n", C.c_int64), ("r", C.c_int64),
+        ("X", C.c_void_p), ("ldx", C.c_int64),
+        ("M", C.c_void_p), ("ldm", C.c_int64),
+        ("Q", C.c_void_p), ("ldq", C.c_int64),
+        ("G", C.c_void_p), ("ldg", C.c_int64),
+        ("g_dtype", C.c_int32),
+        ("tau", C.c_float),
+    ]
+
+
+class dion_hparams(C.Structure):
+    _fields_ = [
+        ("mu", C.c_float), ("eta", C.c_float), ("eta_local", C.c_float),
+        ("eps_rmmc", C.c_float), ("eps_col", C.c_float), ("tau_global", C.c_float),
+        ("gate_mode", C.c_int32), ("period", C.c_int32), ("step", C.c_int64),
+    ]
+
+
+class DionError(RuntimeError):
+    def __init__(self, code: int, what: str = ""):
+        self.code = code
+        super().__init__(f"{what}: {dion_status_string(code)} ({code})")
+
+
+_lib = None
+
+
+def load(path: str = LIB_PATH) -> C.CDLL:
+    """Loads libcurvadion.so (built by paper_2512_13728_gb300.build) and declares its signatures."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise ImportError(f"{path} is missing: build it with `python -m paper_2512_13728_gb300.build`")
+    lib = C.CDLL(path)
+    P = C.c_void_p
+    lib.dion_plan_create.argtypes = [C.POINTER(dion_layer), C.c_int32, C.c_int32, C.POINTER(P)]
+    lib.dion_plan_create.restype = C.c_int
+    lib.dion_step.argtypes = [P, C.POINTER(dion_hparams), P, P, P, P, P, P]
+    lib.dion_step.restype = C.c_int
+    lib.dion_get_device_status.argtypes = [P, C.c_int32, C.POINTER(C.c_int32)]
+    lib.dion_get_device_status.restype = C.c_int
+    lib.dion_step_launch_count.argtypes = [P]
+    lib.dion_step_launch_count.restype = C.c_int32
+    lib.dion_timing_enable.argtypes = [P, C.c_int32]
+    lib.dion_timing_enable.restype = C.c_int
+    lib.dion_timing_read.argtypes = [P, C.c_int32, C.POINTER(C.c_float), C.POINTER(C.c_char_p),
+                                     C.POINTER(C.c_int32), C.POINTER(C.c_int32)]
+    lib.dion_timing_read.restype = C.c_int
+    lib.dion_plan_destroy.argtypes = [P]
+    lib.dion_plan_destroy.restype = None
+    lib.dion_status_string.argtypes = [C.c_int]
+    lib.dion_status_string.restype = C.c_char_p
+    lib.dion_abi_version.argtypes = []
+    lib.dion_abi_version.restype = C.c_int32
+    _lib = lib
+    return lib
+
+
+def dion_status_string(code: int) -> str:
+    return load().dion_status_string(int(code)).decode()
+
+
+def dion_abi_version() -> int:
+    return int(load().dion_abi_version())
+
+
+def dion_plan_create(layers, precision: int) -> int:
+    """layers: sequence of dion_layer; returns the opaque plan handle (an int)."""
+    arr = (dion_layer * max(len(layers), 1))(*layers)
+    out = C.c_void_p()
+    st = load().dion_plan_create(arr, len(layers), int(precision), C.byref(out))
+    if st != DION_OK:
+        raise DionError(st, "dion_plan_create")
+    return out.value
+
+
+def dion_step(plan: int, hp: dion_hparams, prev_norm: int, rmmc_out: int, rmmc_eq1_out, sync_flags_out: int,
+              global_flag_out: int, stream: int) -> None:
+    """All pointers are device addresses (ints); rmmc_eq1_out may be None."""
+    st = load().dion_step(C.c_void_p(plan), C.byref(hp), C.c_void_p(prev_norm), C.c_void_p(rmmc_out),
+                          C.c_void_p(rmmc_eq1_out) if rmmc_eq1_out else None, C.c_void_p(sync_flags_out),
+                          C.c_void_p(global_flag_out), C.c_void_p(stream) if stream else None)
+    if st != DION_OK:
+        raise DionError(st, "dion_step")
+
+
+def dion_get_device_status(plan: int, clear: bool = True) -> int:
+    code = C.c_int32(0)
+    st = load().dion_get_device_status(C.c_void_p(plan), 1 if clear else 0, C.byref(code))
+    if st != DION_OK:
+        raise DionError(st, "dion_get_device_status")
+    return int(code.value)
+
+
+def dion_step_launch_count(plan: int) -> int:
+    return int(load().dion_step_launch_count(C.c_void_p(plan)))
+
+
+def dion_timing_enable(plan: int, max_steps: int) -> None:
+    st = load().dion_timing_enable(C.c_void_p(plan), int(max_steps))
+    if st != DION_OK:
+        raise DionError(st, "dion_timing_enable")
+
+
+def dion_timing_read(plan: int):
+    """Returns (steps recorded, [(kernel name, average ms per launch), ...]) in launch order."""
+    cap = 64
+    ms = (C.c_float * cap)()
+    names = (C.c_char_p * cap)()
+    count, steps = C.c_int32(0), C.c_int32(0)
+    st = load().dion_timing_read(C.c_void_p(plan), cap, ms, names, C.byref(count), C.byref(steps))
+    if st != DION_OK:
+        raise DionError(st, "dion_timing_read")
+    n = min(cap, count.value)
+    return steps.value, [((names[i] or b"").decode(), float(ms[i])) for i in range(n)]
+
+
+def dion_plan_destroy(plan: int) -> None:
+    if plan:
+        load().dion_plan_destroy(C.c_void_p(plan))

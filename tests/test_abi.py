@@ -1,0 +1,99 @@
+"""The C-ABI library loads, exports every function include/curvadion.h declares, and rejects
+bad arguments on the host (CPU only: no kernel is launched; device pointers are fake and
+never dereferenced because validation fails first)."""
+import ctypes as C
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "curvadion.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2512_13728_gb300 import build, native
+
+    build.build()
+    return native.load()
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(dion_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_header_declares_expected_api():
+    from paper_2512_13728_gb300 import native
+
+    assert declared_functions() == sorted(native.EXPORTED)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_exported_symbols_via_nm(lib):
+    out = os.popen(f"nm -D --defined-only {lib._name}").read()
+    for name in declared_functions():
+        assert re.search(rf"\bT {name}$", out, flags=re.M), name
+
+
+def test_abi_version_and_status_strings(lib):
+    from paper_2512_13728_gb300 import native
+
+    assert native.dion_abi_version() == 1
+    for code in range(8):
+        assert native.dion_status_string(code).startswith("DION_")
+    assert "unknown" in native.dion_status_string(99)
+
+
+def fake_layer(**kw):
+    from paper_2512_13728_gb300 import native
+
+    base = dict(m=64, n=48, r=8, X=0x10000, ldx=48, M=0x20000, ldm=48, Q=0x30000, ldq=8, G=0x40000, ldg=48,
+                g_dtype=native.DION_DTYPE_BF16, tau=0.5)
+    base.update(kw)
+    return native.dion_layer(**base)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(r=0), 1), (dict(r=49), 1), (dict(m=0), 1), (dict(n=-1), 1),
+    (dict(r=513, m=1024, n=1024, ldx=1024, ldm=1024, ldg=1024, ldq=516), 2),
+    (dict(X=0), 1), (dict(G=0), 1), (dict(g_dtype=7), 1), (dict(ldx=40), 1), (dict(ldq=4), 1),
+    (dict(X=0x10004), 3), (dict(ldm=50), 3), (dict(ldg=52), 3), (dict(ldq=10), 3),
+    (dict(tau=float("nan")), 1),
+])
+def test_plan_create_rejects_bad_layers(lib, kw, code):
+    from paper_2512_13728_gb300 import native
+
+    layers = (native.dion_layer * 1)(fake_layer(**kw))
+    out = C.c_void_p(123)
+    st = lib.dion_plan_create(layers, 1, native.DION_PREC_FP32, C.byref(out))
+    assert st == code
+    assert out.value is None  # *out cleared on failure
+
+
+def test_plan_create_rejects_bad_precision_and_counts(lib):
+    from paper_2512_13728_gb300 import native
+
+    layers = (native.dion_layer * 1)(fake_layer())
+    out = C.c_void_p()
+    assert lib.dion_plan_create(layers, 1, 9, C.byref(out)) == 1
+    assert lib.dion_plan_create(layers, -1, 0, C.byref(out)) == 1
+    assert lib.dion_plan_create(None, 2, 0, C.byref(out)) == 1
+    assert lib.dion_plan_create(layers, 1, 0, None) == 1
+
+
+def test_step_rejects_null_plan(lib):
+    from paper_2512_13728_gb300 import hparams
+
+    hp = hparams()
+    assert lib.dion_step(None, C.byref(hp), None, None, None, None, None, None) == 1
+    code = C.c_int32()
+    assert lib.dion_get_device_status(None, 0, C.byref(code)) == 1
+    assert lib.dion_step_launch_count(None) == 0
+    lib.dion_plan_destroy(None)  # no-op

@@ -1,0 +1,216 @@
+"""Parity of the CUDA library (through the C ABI) with the fp64 oracle on seeded inputs.
+
+Per-step parity: before each step the device state is copied to the host, the oracle runs one
+step of Algorithm 2 from that exact state with the same gradient, and the library's outputs
+are compared: sync flags and the global flag bit-exact, RMMC to fp32-accumulation accuracy,
+M, X, Q by relative Frobenius error (1e-4 for fp32 arithmetic; 2e-2 where bf16 operands
+are used, the tolerances the design states for fp32 and bf16 inputs).
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle.curvadion as oc
+import workloads as wl
+from tests import gpu_util as gu
+
+pytestmark = pytest.mark.gpu
+
+TOL_FP32 = 1e-4
+TOL_BF16 = 2e-2
+RMMC_RTOL = 1e-5  # fp32 per-thread sums folded into fp64
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2512_13728_gb300 import build
+
+    build.build()
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+
+
+def run_per_step(w, precision, hp_kw, steps, tol, taus=None, pad=0, min_margin=1e-4, layer_ids=None,
+                 check_gate=True):
+    import paper_2512_13728_gb300 as cd
+
+    st = gu.make_state(w, taus=taus, pad=pad)
+    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, precision)
+    hpo = gu.oracle_hp(**hp_kw)
+    worst = dict(M=0.0, X=0.0, Q=0.0, rmmc=0.0, eq1=0.0)
+    flag_seq = []
+    try:
+        for t in range(1, steps + 1):
+            gu.write_gradients(st, t)
+            layers, grads, prev = gu.snapshot(st, plan)
+            plan.step(cd.hparams(step=t, **hp_kw))
+            torch.cuda.synchronize()
+            assert plan.device_status() == 0
+            c = gu.compare_step(st, plan, layers, grads, prev, hpo, t, layer_ids)
+            flag_seq.append(c.want.flags.copy())
+            worst = {k: max(worst[k], v) for k, v in
+                     dict(M=c.err_M, X=c.err_X, Q=c.err_Q, rmmc=c.err_rmmc, eq1=c.err_eq1).items()}
+            if check_gate:
+                if c.margin > min_margin:
+                    assert c.flags_equal, f"step {t}: flags differ (margin {c.margin:.2e})"
+                    assert c.gflag_equal, f"step {t}: global flag differs"
+            assert c.err_M <= tol and c.err_X <= tol and c.err_Q <= tol, (t, c.err_M, c.err_X, c.err_Q)
+            assert c.err_rmmc <= RMMC_RTOL and c.err_eq1 <= RMMC_RTOL, (t, c.err_rmmc, c.err_eq1)
+    finally:
+        plan.close()
+    return worst, flag_seq
+
+
+# ------------------------------------------------------------- fp32 single matrix ---
+
+@pytest.mark.parametrize("mode", [oc.GATE_ALWAYS, oc.GATE_GLOBAL, oc.GATE_PER_LAYER, oc.GATE_SCHEDULED])
+def test_fp32_256x512_r16_all_modes(mode):
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.WORKLOADS["fp32_256x512_r16"]
+    run_per_step(w, cd.DION_PREC_FP32, dict(gate_mode=mode, period=3, mu=0.95, eta=0.01), w.steps, TOL_FP32)
+
+
+# ------------------------------------------------- ragged shapes, several tiles ---
+
+RAGGED = wl.scaled(wl.WORKLOADS["gpt160m_block_r192"], "ragged", [(200, 136), (136, 200), (264, 264), (67, 33),
+                                                                  (1, 5), (5, 1)], rank=24, steps=4)
+
+
+@pytest.mark.parametrize("pad", [0, 3])
+def test_ragged_shapes_fp32(pad):
+    import paper_2512_13728_gb300 as cd
+
+    run_per_step(RAGGED, cd.DION_PREC_FP32, dict(gate_mode=oc.GATE_ALWAYS), RAGGED.steps, TOL_FP32, pad=pad)
+
+
+def test_full_rank_and_max_rank_fp32():
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.scaled(wl.WORKLOADS["gpt160m_block_r192"], "maxrank", [(512, 600), (40, 40), (520, 512)], rank=512,
+                  steps=3)
+    run_per_step(w, cd.DION_PREC_FP32, dict(gate_mode=oc.GATE_ALWAYS), w.steps, TOL_FP32)
+
+
+def test_gpt160m_block_r192_fp32():
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.scaled(wl.WORKLOADS["gpt160m_block_r192"], "block", wl.WORKLOADS["gpt160m_block_r192"].shapes,
+                  steps=4)
+    run_per_step(w, cd.DION_PREC_FP32, dict(gate_mode=oc.GATE_ALWAYS), w.steps, TOL_FP32)
+
+
+# ------------------------------------------------------------------ gate sequences ---
+
+def test_gate_stress_flag_sequences_fp32():
+    """Flat/spiky phases (5 steps each) on a reduced 350M-shaped block: per-layer flags and
+    the global flag bit-exact every step in both gated modes."""
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.scaled(wl.WORKLOADS["gpt350m_gate_stress_r256"], "stress", [(128, 128), (128, 512), (512, 128)],
+                  rank=16, steps=20, phase_len=5)
+    for mode in (oc.GATE_PER_LAYER, oc.GATE_GLOBAL):
+        _, seq = run_per_step(w, cd.DION_PREC_FP32, dict(gate_mode=mode, tau_global=0.5), w.steps, TOL_FP32,
+                              taus=[0.5, 0.3, 0.9])
+        seq = np.array(seq)
+        assert seq.any() and not seq.all()  # the workload exercises both branches
+
+
+def test_empty_plan_step():
+    import paper_2512_13728_gb300 as cd
+
+    plan = cd.Plan([], [], [], [], [], cd.DION_PREC_FP32)
+    plan.global_flag.fill_(7)
+    plan.step(cd.hparams(step=1, gate_mode=cd.DION_GATE_GLOBAL))
+    torch.cuda.synchronize()
+    assert plan.global_flag.item() == 0
+    plan.close()
+
+
+# ------------------------------------------------------------- device-side errors ---
+
+def test_breakdown_on_zero_buffer_sets_status_and_no_nan():
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.scaled(RAGGED, "zero", [(64, 48)], rank=4, steps=1)
+    st = gu.make_state(w)
+    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_FP32)
+    x0 = st.X[0].clone()
+    plan.step(cd.hparams(step=1))  # G = 0 and M = 0: B = 0, P = 0, Gram = 0
+    torch.cuda.synchronize()
+    assert plan.device_status() == cd.native.DION_ERR_BREAKDOWN
+    assert torch.isfinite(st.X[0]).all() and torch.isfinite(st.M[0]).all() and torch.isfinite(st.Q[0]).all()
+    assert torch.equal(st.X[0], x0)
+    assert plan.device_status() == 0  # cleared by the previous read
+    plan.close()
+
+
+def test_nonfinite_gradient_sets_status_and_flags():
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.scaled(RAGGED, "nan", [(64, 48), (32, 32)], rank=4, steps=1)
+    st = gu.make_state(w, taus=[1e9, 1e9])
+    gu.write_gradients(st, 1)
+    st.G[0][3, 5] = float("nan")
+    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_FP32)
+    plan.step(cd.hparams(step=1, gate_mode=cd.DION_GATE_PER_LAYER, tau_global=1e9))
+    torch.cuda.synchronize()
+    assert plan.device_status() == cd.native.DION_ERR_NONFINITE
+    assert plan.flags[0].item() == 1 and plan.global_flag.item() == 1
+    plan.close()
+
+
+def test_deterministic_bitwise():
+    import paper_2512_13728_gb300 as cd
+
+    outs = []
+    for _ in range(2):
+        st = gu.make_state(RAGGED)
+        plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_FP32)
+        for t in range(1, 4):
+            gu.write_gradients(st, t)
+            plan.step(cd.hparams(step=t))
+        torch.cuda.synchronize()
+        outs.append([x.clone() for x in st.X + st.M + st.Q] + [plan.rmmc.clone()])
+        plan.close()
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
+
+
+def test_checkpoint_resume_bitwise():
+    """10 steps == 5 steps, copy all state out and into fresh buffers and a fresh plan, 5 steps."""
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.scaled(RAGGED, "ckpt", [(96, 80), (80, 96)], rank=8, steps=10)
+    st = gu.make_state(w)
+    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_FP32)
+    for t in range(1, 11):
+        gu.write_gradients(st, t)
+        plan.step(cd.hparams(step=t, gate_mode=cd.DION_GATE_PER_LAYER))
+    torch.cuda.synchronize()
+    ref = [x.clone() for x in st.X + st.M + st.Q] + [plan.prev_norm.clone()]
+    plan.close()
+
+    st = gu.make_state(w)
+    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_FP32)
+    for t in range(1, 6):
+        gu.write_gradients(st, t)
+        plan.step(cd.hparams(step=t, gate_mode=cd.DION_GATE_PER_LAYER))
+    torch.cuda.synchronize()
+    saved = [x.cpu() for x in st.X + st.M + st.Q] + [plan.prev_norm.cpu()]
+    plan.close()
+    st2 = gu.make_state(w)
+    L = w.num_layers
+    for i, t in enumerate(st2.X + st2.M + st2.Q):
+        t.copy_(saved[i])
+    plan2 = cd.Plan(st2.X, st2.M, st2.Q, st2.G, st2.taus, cd.DION_PREC_FP32)
+    plan2.prev_norm.copy_(saved[3 * L])
+    for t in range(6, 11):
+        gu.write_gradients(st2, t)
+        plan2.step(cd.hparams(step=t, gate_mode=cd.DION_GATE_PER_LAYER))
+    torch.cuda.synchronize()
+    got = [x for x in st2.X + st2.M + st2.Q] + [plan2.prev_norm]
+    for a, b in zip(got, ref):
+        assert torch.equal(a, b)
+    plan2.close()
