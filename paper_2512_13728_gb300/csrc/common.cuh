@@ -80,17 +80,21 @@ struct Shared {
   double *norm_m_before; // [L]
   double *norm_b;        // [L]
   int32_t *status;       // [1] first device error
+  uint8_t *orth_shifted; // [L] 1 = a Cholesky pass of this step needed the shift (third pass runs)
 };
 
 // A contraction C = op(A) op(B) for the CUDA-core path.
 // op(A)[i][k] = transA ? A[k*lda + i] : A[i*lda + k]   (i < Mrows, k < K)
 // op(B)[k][j] = transB ? B[j*ldb + k] : B[k*ldb + j]   (k < K, j < Ncols)
+// mode: GEMM_ACTIVE runs on active layers; GEMM_SHIFTED only where orth_shifted is set;
+// GEMM_SHIFTED_OR_COPY multiplies where orth_shifted is set and copies A to C elsewhere.
+enum : int32_t { GEMM_ACTIVE = 0, GEMM_SHIFTED = 1, GEMM_SHIFTED_OR_COPY = 2 };
 struct GemmProblem {
   const float *A;
   const float *B;
   float *C;
   int64_t Mrows, Ncols, K, lda, ldb, ldc;
-  int32_t transA, transB, layer, pad;
+  int32_t transA, transB, layer, mode;
 };
 
 __device__ __forceinline__ void set_status(int32_t *st, int32_t code) { atomicCAS(st, 0, code); }
@@ -122,7 +126,7 @@ void launch_gate(const Shared &sh, const StepArgs &a, cudaStream_t s);
 void launch_gemm(const Shared &sh, const GemmProblem *probs, const int4 *tiles, int32_t ntiles,
                  cudaStream_t s);
 cudaError_t prepare_chol_inv(int32_t max_r, size_t *smem_out);
-void launch_chol_inv(const Shared &sh, size_t smem, cudaStream_t s);
+void launch_chol_inv(const Shared &sh, size_t smem, int32_t pass, cudaStream_t s);
 void launch_colnorm(const Shared &sh, const int4 *tiles, int32_t ntiles, float eps_col,
                     cudaStream_t s);
 void launch_update(const Shared &sh, const int4 *tiles, int32_t ntiles, float mu, float eta,

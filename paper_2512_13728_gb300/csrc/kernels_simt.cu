@@ -161,10 +161,19 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_kernel(Shared sh, const Gem
   const int4 t = tiles[blockIdx.x];
   const GemmProblem p = probs[t.x];
   if (!sh.active[p.layer]) return;
-  __shared__ float As[GBK][GBM + 4];
-  __shared__ float Bs[GBK][GBN + 4];
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
   const int64_t i0 = (int64_t)t.y * GBM, j0 = (int64_t)t.z * GBN;
+  if (p.mode != GEMM_ACTIVE && !sh.orth_shifted[p.layer]) {
+    if (p.mode == GEMM_SHIFTED_OR_COPY) {  // C = A (same shape, A not transposed)
+      for (int e = tid; e < GBM * GBN; e += kGemmThreads) {
+        const int64_t gi = i0 + e / GBN, gj = j0 + e % GBN;
+        if (gi < p.Mrows && gj < p.Ncols) p.C[gi * p.ldc + gj] = p.A[gi * p.lda + gj];
+      }
+    }
+    return;
+  }
+  __shared__ float As[GBK][GBM + 4];
+  __shared__ float Bs[GBK][GBN + 4];
   float acc[4][4] = {};
   for (int64_t k0 = 0; k0 < p.K; k0 += GBK) {
 #pragma unroll
@@ -220,14 +229,21 @@ void launch_gemm(const Shared &sh, const GemmProblem *probs, const int4 *tiles, 
 }
 
 // =========================================================== Cholesky + L^{-1} ===
-// Orthogonalize by Cholesky QR: S = P^T P = L L^T, P_orth = P L^{-T}.  For full-rank P this
-// is the Q factor of the thin QR with a positive-diagonal triangular factor.  One CTA per
-// layer factors S (r <= 512) by right-looking blocked Cholesky with 32-wide block columns,
-// then inverts L block row by block row.  S and L^{-1} stay in global memory (L2-resident);
-// diagonal blocks, panels and partial products are staged in shared memory.
-// A pivot <= 0 or non-finite sets DION_ERR_BREAKDOWN and makes L^{-1} = 0 for that layer,
-// so the layer's P, R and Q become 0, M becomes B and X is unchanged (no NaN is written).
+// Orthogonalize by Cholesky QR: S = P^T P = L L^T, P <- P L^{-T}.  The step runs it twice
+// (CholeskyQR2) so that P is orthonormal to fp32 roundoff.  When a pivot is <= 0 or not
+// finite, the pass is retried on S + s I with the shift of shifted CholeskyQR (Fukaya,
+// Kannan, Nakatsukasa, Yamamoto, Yanagisawa 2020): s = 11 (m r + r (r + 1)) u trace(S),
+// u = 2^-24; the layer is then marked and a third pass runs.  Every pass multiplies P by an
+// upper-triangular matrix with positive diagonal, so the final P is the Q factor of the
+// thin QR of the original P with a positive-diagonal triangular factor.
+// One CTA per layer (r <= 512): right-looking blocked Cholesky with 32-wide block columns,
+// then L^{-1} block row by block row.  S and L^{-1} live in global memory (L2-resident);
+// diagonal blocks, panels and partial products are staged in shared memory.  Only the lower
+// triangle of S is overwritten, so a retry rebuilds S from its upper triangle and the saved
+// diagonal.  If the shifted retry also fails, DION_ERR_BREAKDOWN is set and L^{-1} = 0 for
+// the layer, so its P, R and Q become 0, M becomes B and X is unchanged (no NaN written).
 constexpr int CB = 32, CBP = CB + 1, kCholThreads = 512;
+constexpr int DION_MAX_RANK_PAD = 512;  // diag0 slot: r <= 512
 
 __device__ __forceinline__ int64_t tri_row(int64_t p) {
   // largest b with b (b + 1) / 2 <= p
@@ -237,23 +253,12 @@ __device__ __forceinline__ int64_t tri_row(int64_t p) {
   return b;
 }
 
-__global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh) {
-  const int l = blockIdx.x;
-  if (!sh.active[l]) return;
-  const DevLayer &Ly = sh.layers[l];
-  const int r = (int)Ly.r;
-  float *S = Ly.S;
-  float *Li = Ly.Linv;
-  extern __shared__ float smem[];
-  float *D = smem;            // CB x CBP: diagonal block / its inverse
-  float *DI = D + CB * CBP;   // CB x CBP
-  float *Pn = DI + CB * CBP;  // panel (r x CBP) or partial products (CB x r)
-  __shared__ int bad;
+// Factors the lower triangle of S (r x r, row-major) in place.  Returns false (uniformly over
+// the block) on a pivot <= 0 or non-finite.  Smem: D (CB x CBP), Pn (r x CBP).
+__device__ bool cholesky_blocked(float *S, int r, float *D, float *Pn, int *bad) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (tid == 0) bad = 0;
+  if (tid == 0) *bad = 0;
   __syncthreads();
-
-  // ---------------- Cholesky: S lower triangle <- L ----------------
   for (int k0 = 0; k0 < r; k0 += CB) {
     const int nb = min(CB, r - k0);
     for (int e = tid; e < CB * CB; e += kCholThreads) {
@@ -268,13 +273,13 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh) {
       for (int j = 0; j < CB; ++j) {
         const float djj = D[j * CBP + j];
         if (!(djj > 0.f) || !isfinite(djj)) {
-          if (lane == 0) bad = 1;
+          if (lane == 0) *bad = 1;
           break;  // uniform across the warp: every lane read the same djj
         }
-        const float s = sqrtf(djj);
+        const float sq = sqrtf(djj);
         __syncwarp();
-        if (lane == j) D[j * CBP + j] = s;
-        if (lane > j) D[lane * CBP + j] /= s;
+        if (lane == j) D[j * CBP + j] = sq;
+        if (lane > j) D[lane * CBP + j] /= sq;
         __syncwarp();
         if (lane > j) {
           const float lij = D[lane * CBP + j];
@@ -284,7 +289,7 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh) {
       }
     }
     __syncthreads();
-    if (bad) break;
+    if (*bad) return false;
     for (int e = tid; e < nb * nb; e += kCholThreads) {
       const int i = e / nb, j = e % nb;
       if (j <= i) S[(int64_t)(k0 + i) * r + k0 + j] = D[i * CBP + j];
@@ -342,8 +347,54 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh) {
     }
     __syncthreads();
   }
+  return true;
+}
 
-  if (bad) {
+// pass 0 and 1: every active layer; pass 2: only layers marked by a shifted retry.
+__global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int pass) {
+  const int l = blockIdx.x;
+  if (!sh.active[l]) return;
+  if (pass == 2 && !sh.orth_shifted[l]) return;
+  const DevLayer &Ly = sh.layers[l];
+  const int r = (int)Ly.r;
+  float *S = Ly.S;
+  float *Li = Ly.Linv;
+  extern __shared__ float smem[];
+  float *D = smem;            // CB x CBP: diagonal block
+  float *DI = D + CB * CBP;   // CB x CBP: its inverse
+  float *diag0 = DI + CB * CBP;  // r: the diagonal of S before factorization
+  float *Pn = diag0 + DION_MAX_RANK_PAD;  // panel (r x CBP) or partial products (CB x r)
+  __shared__ int bad;
+  __shared__ double trace_s;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int i = tid; i < r; i += kCholThreads) diag0[i] = S[(int64_t)i * r + i];
+  __syncthreads();
+
+  bool ok = cholesky_blocked(S, r, D, Pn, &bad);
+  bool shifted = false;
+  if (!ok) {  // shifted retry: lower triangle from the untouched upper triangle, shifted diagonal
+    if (tid == 0) {
+      double tr = 0.0;
+      for (int i = 0; i < r; ++i) tr += (double)diag0[i];
+      trace_s = tr;
+    }
+    __syncthreads();
+    const double u = 5.9604644775390625e-8;  // 2^-24
+    const double shift = 11.0 * ((double)Ly.m * r + (double)r * (r + 1)) * u * trace_s;
+    for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) {
+      const int64_t i = e / r, j = e % r;
+      if (j < i) S[e] = S[j * r + i];
+      else if (j == i) S[e] = (float)((double)diag0[i] + shift);
+    }
+    __syncthreads();
+    shifted = true;
+    ok = (trace_s > 0.0) && isfinite(trace_s) && cholesky_blocked(S, r, D, Pn, &bad);
+  }
+  if (tid == 0) {
+    if (pass == 0) sh.orth_shifted[l] = shifted ? 1 : 0;
+    else if (shifted) sh.orth_shifted[l] = 1;
+  }
+  if (!ok) {
     if (tid == 0) set_status(sh.status, ST_BREAKDOWN);
     for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) Li[e] = 0.f;
     return;
@@ -402,13 +453,13 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh) {
 
 cudaError_t prepare_chol_inv(int32_t max_r, size_t *smem_out) {
   const int64_t big = (int64_t)max_r * CBP > (int64_t)CB * max_r ? (int64_t)max_r * CBP : (int64_t)CB * max_r;
-  const size_t smem = sizeof(float) * (2 * CB * CBP + big);
+  const size_t smem = sizeof(float) * (2 * CB * CBP + DION_MAX_RANK_PAD + big);
   *smem_out = smem;
   return cudaFuncSetAttribute(chol_inv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
 }
 
-void launch_chol_inv(const Shared &sh, size_t smem, cudaStream_t s) {
-  if (sh.num_layers > 0) chol_inv_kernel<<<sh.num_layers, kCholThreads, smem, s>>>(sh);
+void launch_chol_inv(const Shared &sh, size_t smem, int32_t pass, cudaStream_t s) {
+  if (sh.num_layers > 0) chol_inv_kernel<<<sh.num_layers, kCholThreads, smem, s>>>(sh, pass);
 }
 
 // ===================================================================== ColumnNormalize ===

@@ -27,9 +27,10 @@ struct dion_plan {
   int32_t n_utiles = 0;  // update tiles
   int4 *ctiles = nullptr;
   int32_t n_ctiles = 0;  // column-normalization tiles
-  GemmProblem *probs[4] = {nullptr, nullptr, nullptr, nullptr};
-  int4 *gtiles[4] = {nullptr, nullptr, nullptr, nullptr};
-  int32_t n_gtiles[4] = {0, 0, 0, 0};
+  static constexpr int kSets = 8;
+  GemmProblem *probs[kSets] = {};
+  int4 *gtiles[kSets] = {};
+  int32_t n_gtiles[kSets] = {};
   size_t chol_smem = 0;
   tc::TcPlan tcp{};  // tensor-core path (BF16 / BF16X3)
   int32_t launches_per_step = 0;
@@ -183,10 +184,14 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
     d.upart_cnt = (int32_t)ut.size() - d.upart_off;
     for (int64_t cg = 0; cg < (ly.r + 31) / 32; ++cg) ct.push_back(make_int4(l, (int)cg, 0, 0));
   }
-  // GEMM problems of the CUDA-core path: 0 P_raw = B Q, 1 S = P_raw^T P_raw,
-  // 2 P = P_raw L^{-T}, 3 R = B^T P.
-  std::vector<GemmProblem> gp[4];
-  std::vector<int4> gt[4];
+  // GEMM problem sets of the CUDA-core path:
+  //   0     P_raw = B Q
+  //   1..3  Gram of pass j:  S = X_j^T X_j        (X_0 = P_raw, X_1 = P, X_2 = P_raw)
+  //   4..6  TRSM of pass j:  X_{j+1} = X_j L^{-T}  (X_3 = P); pass 2 only where a shift was needed
+  //   7     R = B^T P
+  constexpr int kSets = dion_plan::kSets;
+  std::vector<GemmProblem> gp[kSets];
+  std::vector<int4> gt[kSets];
   const size_t o_layers = cv.take<DevLayer>(std::max(num_layers, 1));
   const size_t o_active = cv.take<uint8_t>(std::max(num_layers, 1));
   const size_t o_bpart = cv.take<double>(2 * std::max<size_t>(bt.size(), 1));
@@ -207,18 +212,23 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
     }
     cv.off = tcl.end;
   }
-  // GEMM problem/tile arrays are sized after the problem lists are known; reserve below.
-  size_t o_gp[4], o_gt[4];
-  for (int k = 0; k < 4; ++k) {
+  const size_t o_shift = cv.take<uint8_t>(std::max(num_layers, 1));
+  size_t o_gp[kSets], o_gt[kSets];
+  for (int k = 0; k < kSets; ++k) {
     for (int32_t l = 0; l < num_layers; ++l) {
       const dion_layer &ly = layers[l];
       GemmProblem q{};
       q.layer = l;
-      switch (k) {
-        case 0: q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.n; q.lda = ly.ldm; q.ldb = ly.ldq; q.ldc = ly.r; break;
-        case 1: q.Mrows = ly.r; q.Ncols = ly.r; q.K = ly.m; q.lda = ly.r; q.ldb = ly.r; q.ldc = ly.r; q.transA = 1; break;
-        case 2: q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.r; q.lda = ly.r; q.ldb = ly.r; q.ldc = ly.r; q.transB = 1; break;
-        default: q.Mrows = ly.n; q.Ncols = ly.r; q.K = ly.m; q.lda = ly.ldm; q.ldb = ly.r; q.ldc = ly.r; q.transA = 1; break;
+      if (k == 0) {
+        q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.n; q.lda = ly.ldm; q.ldb = ly.ldq; q.ldc = ly.r;
+      } else if (k <= 3) {
+        q.Mrows = ly.r; q.Ncols = ly.r; q.K = ly.m; q.lda = ly.r; q.ldb = ly.r; q.ldc = ly.r; q.transA = 1;
+        q.mode = (k == 3) ? GEMM_SHIFTED : GEMM_ACTIVE;
+      } else if (k <= 6) {
+        q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.r; q.lda = ly.r; q.ldb = ly.r; q.ldc = ly.r; q.transB = 1;
+        q.mode = (k == 6) ? GEMM_SHIFTED_OR_COPY : GEMM_ACTIVE;
+      } else {
+        q.Mrows = ly.n; q.Ncols = ly.r; q.K = ly.m; q.lda = ly.ldm; q.ldb = ly.r; q.ldc = ly.r; q.transA = 1;
       }
       const int32_t pi = (int32_t)gp[k].size();
       gp[k].push_back(q);
@@ -242,15 +252,14 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
     dl[l].Linv = reinterpret_cast<float *>(base + o_Li[l]);
   }
   if (precision != DION_PREC_FP32) tc::bind(tcl, base, dl.data(), num_layers, &p->tcp);
-  for (int k = 0; k < 4; ++k) {
+  for (int k = 0; k < kSets; ++k) {
     for (auto &q : gp[k]) {
       const DevLayer &d = dl[q.layer];
-      switch (k) {
-        case 0: q.A = d.M; q.B = d.Q; q.C = d.P_raw; break;
-        case 1: q.A = d.P_raw; q.B = d.P_raw; q.C = d.S; break;
-        case 2: q.A = d.P_raw; q.B = d.Linv; q.C = d.P; break;
-        default: q.A = d.M; q.B = d.P; q.C = d.R; break;
-      }
+      float *Xs[4] = {d.P_raw, d.P, d.P_raw, d.P};
+      if (k == 0) { q.A = d.M; q.B = d.Q; q.C = d.P_raw; }
+      else if (k <= 3) { q.A = Xs[k - 1]; q.B = Xs[k - 1]; q.C = d.S; }
+      else if (k <= 6) { q.A = Xs[k - 4]; q.B = d.Linv; q.C = Xs[k - 3]; }
+      else { q.A = d.M; q.B = d.P; q.C = d.R; }
     }
     p->probs[k] = reinterpret_cast<GemmProblem *>(base + o_gp[k]);
     p->gtiles[k] = reinterpret_cast<int4 *>(base + o_gt[k]);
@@ -264,6 +273,7 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
   p->sh.norm_m_before = reinterpret_cast<double *>(base + o_nmb);
   p->sh.norm_b = reinterpret_cast<double *>(base + o_nb);
   p->sh.status = reinterpret_cast<int32_t *>(base + o_status);
+  p->sh.orth_shifted = reinterpret_cast<uint8_t *>(base + o_shift);
   p->btiles = reinterpret_cast<int4 *>(base + o_bt);
   p->n_btiles = (int32_t)bt.size();
   p->utiles = reinterpret_cast<int4 *>(base + o_ut);
@@ -276,7 +286,7 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
   if (e == cudaSuccess) e = upload(p->btiles, bt);
   if (e == cudaSuccess) e = upload(p->utiles, ut);
   if (e == cudaSuccess) e = upload(p->ctiles, ct);
-  for (int k = 0; k < 4 && e == cudaSuccess; ++k) {
+  for (int k = 0; k < kSets && e == cudaSuccess; ++k) {
     e = upload(p->probs[k], gp[k]);
     if (e == cudaSuccess) e = upload(p->gtiles[k], gt[k]);
   }
@@ -289,7 +299,7 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
     delete p;
     return DION_ERR_CUDA;
   }
-  p->launches_per_step = (precision == DION_PREC_FP32) ? 11 : tc::launches_per_step(p->tcp);
+  p->launches_per_step = (precision == DION_PREC_FP32) ? 17 : tc::launches_per_step(p->tcp);
   *out = p;
   return DION_OK;
 }
@@ -325,13 +335,18 @@ dion_status dion_step(dion_plan *p, const dion_hparams *hp, double *prev_norm, d
     tick(p, s, "gate");
     launch_gemm(sh, p->probs[0], p->gtiles[0], p->n_gtiles[0], s);  // P = B Q
     tick(p, s, "gemm_bq");
-    launch_gemm(sh, p->probs[1], p->gtiles[1], p->n_gtiles[1], s);  // S = P^T P
-    tick(p, s, "gemm_gram");
-    launch_chol_inv(sh, p->chol_smem, s);                           // L, L^{-1}
-    tick(p, s, "chol_inv");
-    launch_gemm(sh, p->probs[2], p->gtiles[2], p->n_gtiles[2], s);  // P = P L^{-T}
-    tick(p, s, "gemm_trsm");
-    launch_gemm(sh, p->probs[3], p->gtiles[3], p->n_gtiles[3], s);  // R = B^T P
+    static const char *kGram[3] = {"gemm_gram0", "gemm_gram1", "gemm_gram2"};
+    static const char *kChol[3] = {"chol_inv0", "chol_inv1", "chol_inv2"};
+    static const char *kTrsm[3] = {"gemm_trsm0", "gemm_trsm1", "gemm_trsm2"};
+    for (int pass = 0; pass < 3; ++pass) {  // CholeskyQR2, third pass only after a shifted retry
+      launch_gemm(sh, p->probs[1 + pass], p->gtiles[1 + pass], p->n_gtiles[1 + pass], s);  // S = X^T X
+      tick(p, s, kGram[pass]);
+      launch_chol_inv(sh, p->chol_smem, pass, s);  // L, L^{-1}
+      tick(p, s, kChol[pass]);
+      launch_gemm(sh, p->probs[4 + pass], p->gtiles[4 + pass], p->n_gtiles[4 + pass], s);  // X L^{-T}
+      tick(p, s, kTrsm[pass]);
+    }
+    launch_gemm(sh, p->probs[7], p->gtiles[7], p->n_gtiles[7], s);  // R = B^T P
     tick(p, s, "gemm_btp");
     launch_colnorm(sh, p->ctiles, p->n_ctiles, a.eps_col, s);       // Q = ColumnNormalize(R)
     tick(p, s, "colnorm");
