@@ -40,20 +40,17 @@ struct DevLayer {
   int32_t g_dtype;
   float tau;
   float sqrt_m_over_n;
-  int32_t pad0;
-  // workspace (row-major, leading dimension r unless stated)
-  float *P_raw;  // m x r   P = B Q before orthogonalization
-  float *P;      // m x r   orthonormal P
-  float *R;      // n x r   R = B^T P
+  int32_t ldp;  // leading dimension of P_raw, P, R (r rounded up to a multiple of 8)
+  // workspace (row-major)
+  float *P_raw;  // m x r (ld ldp)  P = B Q before orthogonalization
+  float *P;      // m x r (ld ldp)  orthonormal P
+  float *R;      // n x r (ld ldp)  R = B^T P
   float *S;      // r x r   Gram P_raw^T P_raw; lower triangle becomes the Cholesky factor L
   float *Linv;   // r x r   L^{-1} (lower triangular, zeros above the diagonal)
-  // tensor-core operand copies (bf16, K-major, padded leading dimensions); unused in FP32 mode
-  __nv_bfloat16 *Qt_hi, *Qt_lo;  // r x ldqt : Q_{t-1}^T split into hi + lo
-  __nv_bfloat16 *Pt_hi, *Pt_lo;  // r x ldpt : P^T
-  __nv_bfloat16 *P_hi, *P_lo;    // m x r    : P (row-major, K = r contiguous)
-  __nv_bfloat16 *R_hi, *R_lo;    // n x r    : R
-  __nv_bfloat16 *Qn_hi, *Qn_lo;  // n x r    : Q_t
-  int64_t ldqt, ldpt;
+  // tensor-core operand copies (bf16, K-major rows, pitch ldp); null in FP32 mode
+  __nv_bfloat16 *P_hi;   // m x r : P
+  __nv_bfloat16 *R_hi;   // n x r : R
+  __nv_bfloat16 *Qn_hi;  // n x r : Q_t
   int32_t bpart_off, bpart_cnt;  // slots of the ||B||^2 / ||M_{t-1}||^2 partials
   int32_t upart_off, upart_cnt;  // slots of the ||M_t||^2 partials
 };

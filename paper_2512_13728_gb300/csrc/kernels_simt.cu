@@ -472,7 +472,7 @@ __global__ void __launch_bounds__(kColThreads) colnorm_kernel(Shared sh, const i
   if (!sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int64_t j = (int64_t)t.y * 32 + lane, n = L.n, r = L.r;
+  const int64_t j = (int64_t)t.y * 32 + lane, n = L.n, r = L.r, ldp = L.ldp;
   __shared__ double part[kColThreads / 32][32];
   __shared__ float inv[32];
   double acc = 0.0;
@@ -480,7 +480,7 @@ __global__ void __launch_bounds__(kColThreads) colnorm_kernel(Shared sh, const i
     float f = 0.f;
     int cnt = 0;
     for (int64_t i = warp; i < n; i += kColThreads / 32) {
-      const float v = L.R[i * r + j];
+      const float v = L.R[i * ldp + j];
       f = fmaf(v, v, f);
       if (++cnt == 16) { acc += f; f = 0.f; cnt = 0; }
     }
@@ -496,7 +496,14 @@ __global__ void __launch_bounds__(kColThreads) colnorm_kernel(Shared sh, const i
   __syncthreads();
   if (j < r) {
     const float c = inv[lane];
-    for (int64_t i = warp; i < n; i += kColThreads / 32) L.Q[i * L.ldq + j] = L.R[i * r + j] * c;
+    for (int64_t i = warp; i < n; i += kColThreads / 32) {
+      const float rv = L.R[i * ldp + j], q = rv * c;
+      L.Q[i * L.ldq + j] = q;
+      if (L.R_hi != nullptr) {  // bf16 operands of the tensor-core update (rounded to nearest)
+        L.R_hi[i * ldp + j] = __float2bfloat16_rn(rv);
+        L.Qn_hi[i * ldp + j] = __float2bfloat16_rn(q);
+      }
+    }
   }
 }
 
@@ -510,6 +517,7 @@ void launch_colnorm(const Shared &sh, const int4 *tiles, int32_t ntiles, float e
 constexpr int UBM = 64, UBN = 64, UBK = 16, kUpdThreads = 256;
 
 __global__ void __launch_bounds__(kUpdThreads) update_kernel(Shared sh, const int4 *tiles, float mu, float eta) {
+  // P, R: ld ldp; Q: ld ldq
   __shared__ float As[UBK][UBM + 4];
   __shared__ float Rs[UBK][UBN + 4];
   __shared__ float Qs[UBK][UBN + 4];
@@ -518,7 +526,7 @@ __global__ void __launch_bounds__(kUpdThreads) update_kernel(Shared sh, const in
   if (!sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
-  const int64_t i0 = (int64_t)t.y * UBM, j0 = (int64_t)t.z * UBN, r = L.r;
+  const int64_t i0 = (int64_t)t.y * UBM, j0 = (int64_t)t.z * UBN, r = L.r, ldp = L.ldp;
   float u1[4][4] = {}, u2[4][4] = {};
   for (int64_t k0 = 0; k0 < r; k0 += UBK) {
 #pragma unroll
@@ -526,8 +534,8 @@ __global__ void __launch_bounds__(kUpdThreads) update_kernel(Shared sh, const in
       const int idx = tid + s * kUpdThreads;
       const int kk = idx % UBK, ii = idx / UBK;
       const int64_t gk = k0 + kk, gi = i0 + ii, gj = j0 + ii;
-      As[kk][ii] = (gi < L.m && gk < r) ? L.P[gi * r + gk] : 0.f;
-      Rs[kk][ii] = (gj < L.n && gk < r) ? L.R[gj * r + gk] : 0.f;
+      As[kk][ii] = (gi < L.m && gk < r) ? L.P[gi * ldp + gk] : 0.f;
+      Rs[kk][ii] = (gj < L.n && gk < r) ? L.R[gj * ldp + gk] : 0.f;
       Qs[kk][ii] = (gj < L.n && gk < r) ? L.Q[gj * L.ldq + gk] : 0.f;
     }
     __syncthreads();

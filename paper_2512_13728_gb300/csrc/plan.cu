@@ -164,10 +164,11 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
     d.G = ly.G; d.ldg = ly.ldg; d.g_dtype = ly.g_dtype;
     d.tau = ly.tau;
     d.sqrt_m_over_n = (float)std::sqrt((double)ly.m / (double)ly.n);
+    d.ldp = (int32_t)((ly.r + 7) / 8 * 8);
     p->max_r = std::max<int32_t>(p->max_r, (int32_t)ly.r);
-    o_Praw[l] = cv.take<float>(ly.m * ly.r);
-    o_P[l] = cv.take<float>(ly.m * ly.r);
-    o_R[l] = cv.take<float>(ly.n * ly.r);
+    o_Praw[l] = cv.take<float>(ly.m * d.ldp);
+    o_P[l] = cv.take<float>(ly.m * d.ldp);
+    o_R[l] = cv.take<float>(ly.n * d.ldp);
     o_S[l] = cv.take<float>(ly.r * ly.r);
     o_Li[l] = cv.take<float>(ly.r * ly.r);
     // row tiles of about 64K elements for the buffer and local kernels
@@ -217,18 +218,19 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
   for (int k = 0; k < kSets; ++k) {
     for (int32_t l = 0; l < num_layers; ++l) {
       const dion_layer &ly = layers[l];
+      const int64_t ldp = dl[l].ldp;
       GemmProblem q{};
       q.layer = l;
       if (k == 0) {
-        q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.n; q.lda = ly.ldm; q.ldb = ly.ldq; q.ldc = ly.r;
+        q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.n; q.lda = ly.ldm; q.ldb = ly.ldq; q.ldc = ldp;
       } else if (k <= 3) {
-        q.Mrows = ly.r; q.Ncols = ly.r; q.K = ly.m; q.lda = ly.r; q.ldb = ly.r; q.ldc = ly.r; q.transA = 1;
+        q.Mrows = ly.r; q.Ncols = ly.r; q.K = ly.m; q.lda = ldp; q.ldb = ldp; q.ldc = ly.r; q.transA = 1;
         q.mode = (k == 3) ? GEMM_SHIFTED : GEMM_ACTIVE;
       } else if (k <= 6) {
-        q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.r; q.lda = ly.r; q.ldb = ly.r; q.ldc = ly.r; q.transB = 1;
+        q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.r; q.lda = ldp; q.ldb = ly.r; q.ldc = ldp; q.transB = 1;
         q.mode = (k == 6) ? GEMM_SHIFTED_OR_COPY : GEMM_ACTIVE;
       } else {
-        q.Mrows = ly.n; q.Ncols = ly.r; q.K = ly.m; q.lda = ly.ldm; q.ldb = ly.r; q.ldc = ly.r; q.transA = 1;
+        q.Mrows = ly.n; q.Ncols = ly.r; q.K = ly.m; q.lda = ly.ldm; q.ldb = ldp; q.ldc = ldp; q.transA = 1;
       }
       const int32_t pi = (int32_t)gp[k].size();
       gp[k].push_back(q);
@@ -292,7 +294,12 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
   }
   if (e == cudaSuccess) e = cudaMemset(p->sh.status, 0, sizeof(int32_t));
   if (e == cudaSuccess && num_layers > 0) e = prepare_chol_inv(p->max_r, &p->chol_smem);
-  if (e == cudaSuccess && precision != DION_PREC_FP32) e = tc::init(tcl, dl.data(), num_layers, &p->tcp);
+  if (e == cudaSuccess && precision != DION_PREC_FP32) {
+    p->tcp.probs = p->probs;
+    p->tcp.gtiles = p->gtiles;
+    p->tcp.n_gtiles = p->n_gtiles;
+    e = tc::init(tcl, base, dl.data(), num_layers, &p->tcp);
+  }
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
   if (e != cudaSuccess) {
     cudaFree(p->ws);

@@ -1,0 +1,398 @@
+// Tensor-core path of the CurvaDion step (DION_PREC_BF16): plan layout, tensor maps, and the
+// tcgen05 kernels.
+//
+// Error feedback + parameter update (Algorithm 1/2, sync branch):
+//   M = B - (1 - mu) P R^T,   X = X - eta sqrt(m/n) P Q_t^T
+// run as one persistent, warp-specialized kernel over 128 x 128 output tiles:
+//   warp 0      TMA producer: bf16 K-major chunks of P (A), R and Q_t (two B operands) into a
+//               3-stage shared-memory ring;
+//   warp 1      MMA issuer: two 128x128x16 tcgen05.mma per k-step into a double-buffered
+//               pair of TMEM accumulators (U1 = P R^T, U2 = P Q_t^T; 4 x 128 = 512 columns);
+//   warps 2..5  epilogue: TMA-load 128 x 32 fp32 boxes of B (in the M buffer) and X, read
+//               U1/U2 from TMEM (thread = tile row), compute M_t and X_t in shared memory,
+//               TMA-store both; per-tile fp64 partial of ||M_t||^2 for Equation 1.
+// Every HBM byte of the pass (read B, X; write M, X) moves by TMA in 128-byte rows.
+#include "tc.cuh"
+#include "tc_common.cuh"
+
+#include <algorithm>
+#include <cstring>
+
+namespace cd {
+
+void tick_begin(dion_plan *p, cudaStream_t s);
+void tick(dion_plan *p, cudaStream_t s, const char *name);
+
+namespace tc {
+
+// ================================================================== P -> bf16 copy ===
+// P (fp32, ld ldp) -> P_hi (bf16, same pitch) for the update's A operand; active layers only.
+constexpr int kCvtThreads = 256;
+
+__global__ void __launch_bounds__(kCvtThreads) cvt_p_kernel(Shared sh, const int4 *tiles) {
+  const int4 t = tiles[blockIdx.x];  // {layer, first row, rows, 0}
+  if (!sh.active[t.x]) return;
+  const DevLayer &L = sh.layers[t.x];
+  const int64_t r = L.r, ldp = L.ldp;
+  const int64_t total = (int64_t)t.z * r;
+  for (int64_t e = threadIdx.x; e < total; e += kCvtThreads) {
+    const int64_t i = t.y + e / r, j = e % r;
+    L.P_hi[i * ldp + j] = __float2bfloat16_rn(L.P[i * ldp + j]);
+  }
+}
+
+// ============================================================ update (tcgen05) kernel ===
+constexpr int U_STAGES = 3;
+constexpr uint32_t U_OPB = 128u * 64u * 2u;           // one 128 x 64 bf16 operand box
+constexpr uint32_t U_STAGE = 3u * U_OPB;              // P, R, Q_t
+constexpr uint32_t U_EPI = 128u * 32u * 4u;           // one 128 x 32 fp32 box
+constexpr uint32_t U_SMEM = 1024u + U_STAGES * U_STAGE + 4u * U_EPI + 256u;
+constexpr int U_THREADS = 192;
+constexpr uint32_t U_IDESC = idesc_bf16(128, 128, false, false);
+
+struct Abort {
+  int *flag;
+  __device__ bool wait(uint64_t *bar, uint32_t parity, int32_t *status) const {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t i = 1;; ++i) {
+      if (mbar_try_wait(bar, parity)) return true;
+      if ((i & 255u) == 0) {
+        if (*(volatile int *)flag) return false;
+        if (globaltimer_ns() - t0 > kWaitLimitNs) {
+          set_status(status, ST_TIMEOUT);
+          *(volatile int *)flag = 1;
+          return false;
+        }
+      }
+    }
+  }
+};
+
+__device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
+  return reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+
+__global__ void __launch_bounds__(U_THREADS, 1)
+    tc_update_kernel(Shared sh, const int4 *__restrict__ tiles, int ntiles, const LayerMaps *__restrict__ maps,
+                     float mu, float eta) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = align1024(smem_raw);
+  uint8_t *stage = smem;
+  uint8_t *epi = smem + U_STAGES * U_STAGE;
+  uint64_t *bars = reinterpret_cast<uint64_t *>(epi + 4 * U_EPI);
+  uint64_t *full = bars, *empty = bars + U_STAGES;
+  uint64_t *acc_full = bars + 2 * U_STAGES, *acc_empty = acc_full + 2, *epi_full = acc_empty + 2;
+  uint64_t *drain = epi_full + 2;
+  __shared__ uint32_t tmem_base_s;
+  __shared__ int abort_s;
+  __shared__ double red_s[4];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const Abort ab{&abort_s};
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < U_STAGES; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 128);
+      mbar_init(&epi_full[b], 1);
+    }
+    mbar_init(drain, 1);
+    abort_s = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&tmem_base_s, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_s;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+        const int4 t = tiles[ti];
+        if (!sh.active[t.x]) continue;
+        const LayerMaps *mp = maps + t.x;
+        const int kch = (int)((sh.layers[t.x].r + 63) / 64);
+        for (int kc = 0; kc < kch; ++kc, ++it) {
+          const uint32_t s = it % U_STAGES, ph = (it / U_STAGES) & 1u;
+          if (!ab.wait(&empty[s], ph ^ 1u, sh.status)) { ok = false; break; }
+          uint8_t *sp = stage + s * U_STAGE;
+          mbar_expect_tx(&full[s], U_STAGE);
+          tma_load_2d(sp, &mp->P_hi, &full[s], kc * 64, t.y * 128);
+          tma_load_2d(sp + U_OPB, &mp->R_hi, &full[s], kc * 64, t.z * 128);
+          tma_load_2d(sp + 2 * U_OPB, &mp->Qn_hi, &full[s], kc * 64, t.z * 128);
+        }
+      }
+      // drain: every issued load has landed before the CTA may exit
+      for (uint32_t k = (it > U_STAGES ? it - U_STAGES : 0); k < it; ++k)
+        mbar_wait(&full[k % U_STAGES], (k / U_STAGES) & 1u, sh.status);
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      uint32_t it = 0, tcount = 0;
+      bool ok = true;
+      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+        const int4 t = tiles[ti];
+        if (!sh.active[t.x]) continue;
+        const int kch = (int)((sh.layers[t.x].r + 63) / 64);
+        const uint32_t b = tcount & 1u, aph = (tcount >> 1) & 1u;
+        if (!ab.wait(&acc_empty[b], aph ^ 1u, sh.status)) break;
+        tc_fence_after();
+        const uint32_t d1 = tmem + b * 256u, d2 = d1 + 128u;
+        for (int kc = 0; kc < kch; ++kc, ++it) {
+          const uint32_t s = it % U_STAGES, ph = (it / U_STAGES) & 1u;
+          if (!ab.wait(&full[s], ph, sh.status)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t base = smem_u32(stage + s * U_STAGE);
+#pragma unroll
+          for (int k16 = 0; k16 < 4; ++k16) {
+            const uint64_t ad = smem_desc_sw128(base + k16 * 32, 0, 1024);
+            const uint64_t rd = smem_desc_sw128(base + U_OPB + k16 * 32, 0, 1024);
+            const uint64_t qd = smem_desc_sw128(base + 2 * U_OPB + k16 * 32, 0, 1024);
+            const uint32_t acc = (kc | k16) ? 1u : 0u;
+            umma_bf16(d1, ad, rd, U_IDESC, acc);
+            umma_bf16(d2, ad, qd, U_IDESC, acc);
+          }
+          umma_commit(&empty[s]);
+        }
+        if (!ok) break;
+        umma_commit(&acc_full[b]);
+        ++tcount;
+      }
+      umma_commit(drain);  // every MMA of this CTA has completed before TMEM is freed
+      mbar_wait(drain, 0, sh.status);
+    }
+  } else {
+    // ---------------------------------------------------------------- epilogue (128 threads)
+    const int et = threadIdx.x - 64;
+    const uint32_t row = 32u * (warp & 3) + lane;  // TMEM lane = tile row
+    const bool leader = (et == 0);
+    uint32_t tcount = 0, ecount = 0, issued = 0;
+    bool ok = true;
+    for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+      const int4 t = tiles[ti];
+      if (!sh.active[t.x]) continue;
+      const DevLayer &L = sh.layers[t.x];
+      const LayerMaps *mp = maps + t.x;
+      const float dec = 1.f - mu, c = eta * L.sqrt_m_over_n;
+      const int r0 = t.y * 128, c0 = t.z * 128;
+      const uint32_t b = tcount & 1u, aph = (tcount >> 1) & 1u;
+      auto issue = [&](int j) {  // TMA-load chunk j of this tile into its epilogue buffer
+        const uint32_t eb = (ecount + j) & 1u;
+        uint8_t *bs = epi + eb * 2 * U_EPI;
+        bulk_wait_read<0>();  // the store that last used this buffer has read it
+        mbar_expect_tx(&epi_full[eb], 2 * U_EPI);
+        tma_load_2d(bs, &mp->Mf, &epi_full[eb], c0 + j * 32, r0);
+        tma_load_2d(bs + U_EPI, &mp->Xf, &epi_full[eb], c0 + j * 32, r0);
+        ++issued;
+      };
+      if (leader) issue(0);
+      if (!ab.wait(&acc_full[b], aph, sh.status)) break;
+      tc_fence_after();
+      float ss = 0.f;
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t eb = (ecount + j) & 1u, eph = ((ecount + j) >> 1) & 1u;
+        if (leader && j + 1 < 4) issue(j + 1);
+        uint32_t u1[32], u2[32];
+        tmem_ld32(tmem + ((32u * (warp & 3)) << 16) + b * 256u + j * 32, u1);
+        tmem_ld32(tmem + ((32u * (warp & 3)) << 16) + b * 256u + 128u + j * 32, u2);
+        tmem_ld_wait();
+        if (!ab.wait(&epi_full[eb], eph, sh.status)) { ok = false; break; }
+        uint8_t *bs = epi + eb * 2 * U_EPI;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const uint32_t off = sw128_f32(row, q);
+          float4 bv = *reinterpret_cast<float4 *>(bs + off);
+          float4 xv = *reinterpret_cast<float4 *>(bs + U_EPI + off);
+          bv.x = fmaf(-dec, __uint_as_float(u1[4 * q + 0]), bv.x);
+          bv.y = fmaf(-dec, __uint_as_float(u1[4 * q + 1]), bv.y);
+          bv.z = fmaf(-dec, __uint_as_float(u1[4 * q + 2]), bv.z);
+          bv.w = fmaf(-dec, __uint_as_float(u1[4 * q + 3]), bv.w);
+          xv.x = fmaf(-c, __uint_as_float(u2[4 * q + 0]), xv.x);
+          xv.y = fmaf(-c, __uint_as_float(u2[4 * q + 1]), xv.y);
+          xv.z = fmaf(-c, __uint_as_float(u2[4 * q + 2]), xv.z);
+          xv.w = fmaf(-c, __uint_as_float(u2[4 * q + 3]), xv.w);
+          ss = fmaf(bv.x, bv.x, ss); ss = fmaf(bv.y, bv.y, ss);
+          ss = fmaf(bv.z, bv.z, ss); ss = fmaf(bv.w, bv.w, ss);
+          *reinterpret_cast<float4 *>(bs + off) = bv;
+          *reinterpret_cast<float4 *>(bs + U_EPI + off) = xv;
+        }
+        fence_async_smem();
+        named_sync(1, 128);
+        if (leader) {  // out-of-range rows/columns of a ragged tile are clipped by the store
+          tma_store_2d(&mp->Mf, bs, c0 + j * 32, r0);
+          tma_store_2d(&mp->Xf, bs + U_EPI, c0 + j * 32, r0);
+          bulk_commit();
+        }
+      }
+      ecount += 4;
+      tc_fence_before();
+      mbar_arrive(&acc_empty[b]);
+      if (!ok) break;
+      // per-tile ||M_t||^2 (rows/columns outside the matrix hold 0), fixed reduction order
+      double v = (double)ss;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+      if (lane == 0) red_s[warp - 2] = v;
+      named_sync(1, 128);
+      if (leader) sh.upart[t.w] = (red_s[0] + red_s[1]) + (red_s[2] + red_s[3]);
+      ++tcount;
+    }
+    if (leader) {
+      bulk_wait<0>();
+      // loads issued but not consumed (only after an abort)
+      for (uint32_t k = ecount; k < issued; ++k) mbar_wait(&epi_full[k & 1u], (k >> 1) & 1u, sh.status);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 512);
+}
+
+// ========================================================================= host side ===
+dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int num_sms, size_t start,
+                   TcLayout *out) {
+  if (precision != DION_PREC_BF16) return DION_ERR_UNSUPPORTED;
+  TcLayout &lo = *out;
+  lo.precision = precision;
+  size_t off = start;
+  auto take = [&](size_t bytes, size_t align = 256) {
+    off = (off + align - 1) / align * align;
+    const size_t at = off;
+    off += bytes;
+    return at;
+  };
+  lo.o_phi.resize(L);
+  lo.o_rhi.resize(L);
+  lo.o_qnhi.resize(L);
+  for (int32_t l = 0; l < L; ++l) {
+    const dion_layer &ly = layers[l];
+    const int64_t ldp = (ly.r + 7) / 8 * 8;
+    lo.o_phi[l] = take(ly.m * ldp * 2);
+    lo.o_rhi[l] = take(ly.n * ldp * 2);
+    lo.o_qnhi[l] = take(ly.n * ldp * 2);
+    for (int64_t mb = 0; mb < (ly.m + 127) / 128; ++mb)
+      for (int64_t nb = 0; nb < (ly.n + 127) / 128; ++nb)
+        lo.utiles.push_back(make_int4(l, (int)mb, (int)nb, (int)lo.utiles.size()));
+    const int64_t prow = std::max<int64_t>(1, std::min<int64_t>(ly.m, 16384 / ly.r));
+    for (int64_t r0 = 0; r0 < ly.m; r0 += prow)
+      lo.ptiles.push_back(make_int4(l, (int)r0, (int)std::min(prow, ly.m - r0), 0));
+  }
+  lo.o_maps = take(sizeof(LayerMaps) * std::max(L, 1), 128);
+  lo.o_utiles = take(sizeof(int4) * std::max<size_t>(lo.utiles.size(), 1));
+  lo.o_ptiles = take(sizeof(int4) * std::max<size_t>(lo.ptiles.size(), 1));
+  lo.end = off;
+  (void)num_sms;
+  return DION_OK;
+}
+
+void bind(const TcLayout &lo, char *base, DevLayer *dl, int32_t L, TcPlan *tp) {
+  for (int32_t l = 0; l < L; ++l) {
+    dl[l].P_hi = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_phi[l]);
+    dl[l].R_hi = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_rhi[l]);
+    dl[l].Qn_hi = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_qnhi[l]);
+    // the update tiles replace the CUDA-core update's partial slots
+    dl[l].upart_off = -1;
+  }
+  int32_t cur = -1;
+  for (size_t i = 0; i < lo.utiles.size(); ++i) {
+    const int l = lo.utiles[i].x;
+    if (l != cur) {
+      dl[l].upart_off = (int32_t)i;
+      dl[l].upart_cnt = 0;
+      cur = l;
+    }
+    ++dl[l].upart_cnt;
+  }
+  tp->maps = reinterpret_cast<LayerMaps *>(base + lo.o_maps);
+  tp->utiles = reinterpret_cast<int4 *>(base + lo.o_utiles);
+  tp->n_utiles = (int32_t)lo.utiles.size();
+  tp->ptiles = reinterpret_cast<int4 *>(base + lo.o_ptiles);
+  tp->n_ptiles = (int32_t)lo.ptiles.size();
+  tp->precision = lo.precision;
+}
+
+cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, TcPlan *tp) {
+  (void)base;
+  std::vector<LayerMaps> maps(std::max(L, 1));
+  std::memset(maps.data(), 0, sizeof(LayerMaps) * maps.size());
+  for (int32_t l = 0; l < L; ++l) {
+    const DevLayer &d = dl[l];
+    LayerMaps &m = maps[l];
+    const uint64_t pitch16 = (uint64_t)d.ldp * 2;
+    bool ok = encode_bf16_2d(&m.P_hi, d.P_hi, d.r, d.m, pitch16, 64, 128) &&
+              encode_bf16_2d(&m.R_hi, d.R_hi, d.r, d.n, pitch16, 64, 128) &&
+              encode_bf16_2d(&m.Qn_hi, d.Qn_hi, d.r, d.n, pitch16, 64, 128) &&
+              encode_f32_2d(&m.Mf, d.M, d.n, d.m, (uint64_t)d.ldm * 4, 32, 128) &&
+              encode_f32_2d(&m.Xf, d.X, d.n, d.m, (uint64_t)d.ldx * 4, 32, 128);
+    if (!ok) return cudaErrorInvalidValue;
+  }
+  cudaError_t e = cudaMemcpy(tp->maps, maps.data(), sizeof(LayerMaps) * maps.size(), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && !lo.utiles.empty())
+    e = cudaMemcpy(tp->utiles, lo.utiles.data(), sizeof(int4) * lo.utiles.size(), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && !lo.ptiles.empty())
+    e = cudaMemcpy(tp->ptiles, lo.ptiles.data(), sizeof(int4) * lo.ptiles.size(), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(tc_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)U_SMEM);
+  int dev = 0, sms = 0;
+  if (e == cudaSuccess) e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  tp->num_sms = sms;
+  tp->launches = 18;
+  return e;
+}
+
+int32_t launches_per_step(const TcPlan &tp) { return tp.launches; }
+
+void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, const int4 *btiles,
+          int32_t n_btiles, const int4 *ctiles, int32_t n_ctiles, size_t chol_smem, cudaStream_t s) {
+  launch_form_b(sh, btiles, n_btiles, s);
+  tick(p, s, "form_b");
+  launch_gate(sh, a, s);
+  tick(p, s, "gate");
+  launch_gemm(sh, tp.probs[0], tp.gtiles[0], tp.n_gtiles[0], s);  // P = B Q
+  tick(p, s, "gemm_bq");
+  static const char *kGram[3] = {"gemm_gram0", "gemm_gram1", "gemm_gram2"};
+  static const char *kChol[3] = {"chol_inv0", "chol_inv1", "chol_inv2"};
+  static const char *kTrsm[3] = {"gemm_trsm0", "gemm_trsm1", "gemm_trsm2"};
+  for (int pass = 0; pass < 3; ++pass) {
+    launch_gemm(sh, tp.probs[1 + pass], tp.gtiles[1 + pass], tp.n_gtiles[1 + pass], s);
+    tick(p, s, kGram[pass]);
+    launch_chol_inv(sh, chol_smem, pass, s);
+    tick(p, s, kChol[pass]);
+    launch_gemm(sh, tp.probs[4 + pass], tp.gtiles[4 + pass], tp.n_gtiles[4 + pass], s);
+    tick(p, s, kTrsm[pass]);
+  }
+  launch_gemm(sh, tp.probs[7], tp.gtiles[7], tp.n_gtiles[7], s);  // R = B^T P
+  tick(p, s, "gemm_btp");
+  launch_colnorm(sh, ctiles, n_ctiles, a.eps_col, s);  // Q_t, and bf16 R, Q_t
+  tick(p, s, "colnorm");
+  if (tp.n_ptiles > 0) cvt_p_kernel<<<tp.n_ptiles, kCvtThreads, 0, s>>>(sh, tp.ptiles);
+  tick(p, s, "cvt_p");
+  if (tp.n_utiles > 0) {
+    const int grid = std::min(tp.n_utiles, std::max(tp.num_sms, 1));
+    tc_update_kernel<<<grid, U_THREADS, U_SMEM, s>>>(sh, tp.utiles, tp.n_utiles, tp.maps, a.mu, a.eta);
+  }
+  tick(p, s, "tc_update");
+  launch_local(sh, btiles, n_btiles, a.eta_local, s);
+  tick(p, s, "local");
+  launch_finalize(sh, a, s);
+  tick(p, s, "finalize");
+}
+
+void destroy(TcPlan *tp) { (void)tp; }
+
+}  // namespace tc
+}  // namespace cd

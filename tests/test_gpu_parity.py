@@ -160,6 +160,34 @@ def test_gpt160m_block_r192_fp32():
     run_per_step(w, cd.DION_PREC_FP32, dict(gate_mode=oc.GATE_ALWAYS), w.steps, TOL_FP32)
 
 
+# ------------------------------------------------------- tensor-core (bf16) path ---
+
+@pytest.mark.parametrize("pad", [0, 1])
+def test_ragged_shapes_bf16(pad):
+    import paper_2512_13728_gb300 as cd
+
+    run_per_step(RAGGED, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_ALWAYS), RAGGED.steps, TOL_BF16, pad=pad)
+
+
+def test_gpt160m_block_r192_bf16():
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.scaled(wl.WORKLOADS["gpt160m_block_r192"], "block", wl.WORKLOADS["gpt160m_block_r192"].shapes,
+                  steps=4)
+    worst, _ = run_per_step(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_ALWAYS), w.steps, TOL_BF16)
+    print("bf16 block worst", worst)
+
+
+def test_gate_modes_bf16():
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.scaled(wl.WORKLOADS["gpt350m_gate_stress_r256"], "stress", [(128, 128), (128, 512), (512, 128)],
+                  rank=16, steps=12, phase_len=4)
+    for mode in (oc.GATE_PER_LAYER, oc.GATE_GLOBAL, oc.GATE_SCHEDULED):
+        run_per_step(w, cd.DION_PREC_BF16, dict(gate_mode=mode, tau_global=0.5, period=3), w.steps, TOL_BF16,
+                     taus=[0.5, 0.3, 0.9])
+
+
 # ------------------------------------------------------------------ gate sequences ---
 
 def test_gate_stress_flag_sequences_fp32():
