@@ -187,6 +187,8 @@ __global__ void __launch_bounds__(U_THREADS, 1)
       const LayerMaps *mp = maps + t.x;
       const float dec = 1.f - mu, c = eta * L.sqrt_m_over_n;
       const int r0 = t.y * 128, c0 = t.z * 128;
+      // 32-column chunks that start inside the matrix (a ragged last tile has fewer)
+      const int nj = (int)std::min<int64_t>(4, (L.n - c0 + 31) / 32);
       const uint32_t b = tcount & 1u, aph = (tcount >> 1) & 1u;
       auto issue = [&](int j) {  // TMA-load chunk j of this tile into its epilogue buffer
         const uint32_t eb = (ecount + j) & 1u;
@@ -201,9 +203,9 @@ __global__ void __launch_bounds__(U_THREADS, 1)
       if (!ab.wait(&acc_full[b], aph, sh.status)) break;
       tc_fence_after();
       float ss = 0.f;
-      for (int j = 0; j < 4; ++j) {
+      for (int j = 0; j < nj; ++j) {
         const uint32_t eb = (ecount + j) & 1u, eph = ((ecount + j) >> 1) & 1u;
-        if (leader && j + 1 < 4) issue(j + 1);
+        if (leader && j + 1 < nj) issue(j + 1);
         uint32_t u1[32], u2[32];
         tmem_ld32(tmem + ((32u * (warp & 3)) << 16) + b * 256u + j * 32, u1);
         tmem_ld32(tmem + ((32u * (warp & 3)) << 16) + b * 256u + 128u + j * 32, u2);
@@ -236,7 +238,7 @@ __global__ void __launch_bounds__(U_THREADS, 1)
           bulk_commit();
         }
       }
-      ecount += 4;
+      ecount += nj;
       tc_fence_before();
       mbar_arrive(&acc_empty[b]);
       if (!ok) break;

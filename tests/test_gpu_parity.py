@@ -56,7 +56,9 @@ def run_per_step(w, precision, hp_kw, steps, tol, taus=None, pad=0, min_margin=1
                     assert c.flags_equal, f"step {t}: flags differ (margin {c.margin:.2e})"
                     assert c.gflag_equal, f"step {t}: global flag differs"
             assert c.err_M <= tol and c.err_X <= tol and c.err_Q <= tol, (t, c.err_M, c.err_X, c.err_Q)
-            assert c.err_rmmc <= RMMC_RTOL and c.err_eq1 <= RMMC_RTOL, (t, c.err_rmmc, c.err_eq1)
+            # Algorithm 2's RMMC comes from ||B|| (an exact fp32 add in every mode); Equation 1's
+            # from ||M_t||, which carries the mode's error on M
+            assert c.err_rmmc <= RMMC_RTOL and c.err_eq1 <= max(RMMC_RTOL, tol), (t, c.err_rmmc, c.err_eq1)
     finally:
         plan.close()
     return worst, flag_seq
