@@ -129,6 +129,13 @@ dion_status dion_step(dion_plan *plan, const dion_hparams *hp, double *prev_norm
  * The first device error of any step since the last clear is kept. */
 dion_status dion_get_device_status(dion_plan *plan, int32_t clear, int32_t *code_out);
 
+/* The tensor-core modes keep a bf16 copy of every layer's Q (made by dion_plan_create and
+ * updated by each step that writes Q).  A caller that writes Q itself between steps (for
+ * example when restoring a checkpoint) calls dion_plan_refresh before the next dion_step;
+ * it enqueues the re-copy on `stream` and allocates nothing.  No-op in DION_PREC_FP32.
+ * Errors: INVALID_ARG (NULL plan), CUDA. */
+dion_status dion_plan_refresh(dion_plan *plan, void *stream);
+
 /* Number of kernel launches one dion_step enqueues for this plan. */
 int32_t dion_step_launch_count(const dion_plan *plan);
 

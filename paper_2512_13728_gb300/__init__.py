@@ -72,6 +72,13 @@ class Plan:
                          self.rmmc_eq1.data_ptr() if eq1 else None, self.flags.data_ptr(),
                          self.global_flag.data_ptr(), s)
 
+    def refresh(self, stream: Optional[int] = None) -> None:
+        """Call after writing Q from outside dion_step (e.g. a checkpoint restore)."""
+        import torch
+
+        s = torch.cuda.current_stream(self.device).cuda_stream if stream is None else stream
+        native.dion_plan_refresh(self.handle, s)
+
     def device_status(self, clear: bool = True) -> int:
         return native.dion_get_device_status(self.handle, clear)
 

@@ -47,10 +47,12 @@ struct DevLayer {
   float *R;      // n x r (ld ldp)  R = B^T P
   float *S;      // r x r   Gram P_raw^T P_raw; lower triangle becomes the Cholesky factor L
   float *Linv;   // r x r   L^{-1} (lower triangular, zeros above the diagonal)
-  // tensor-core operand copies (bf16, K-major rows, pitch ldp); null in FP32 mode
+  // tensor-core operand copies (bf16, rows of pitch ldp unless stated); null in FP32 mode
   __nv_bfloat16 *P_hi;   // m x r : P
   __nv_bfloat16 *R_hi;   // n x r : R
-  __nv_bfloat16 *Qn_hi;  // n x r : Q_t
+  __nv_bfloat16 *Qn_hi;  // n x r : Q (Q_{t-1} when a step starts, Q_t after a sync step)
+  __nv_bfloat16 *Bh;     // m x n, pitch ldbh : B rounded to bf16
+  int64_t ldbh;
   int32_t bpart_off, bpart_cnt;  // slots of the ||B||^2 / ||M_{t-1}||^2 partials
   int32_t upart_off, upart_cnt;  // slots of the ||M_t||^2 partials
 };

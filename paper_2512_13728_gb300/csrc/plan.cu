@@ -195,7 +195,8 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
   std::vector<int4> gt[kSets];
   const size_t o_layers = cv.take<DevLayer>(std::max(num_layers, 1));
   const size_t o_active = cv.take<uint8_t>(std::max(num_layers, 1));
-  const size_t o_bpart = cv.take<double>(2 * std::max<size_t>(bt.size(), 1));
+  const size_t nslots = std::max<size_t>(bt.size(), precision == DION_PREC_FP32 ? 0 : tc::norm_slots(layers, num_layers));
+  const size_t o_bpart = cv.take<double>(2 * std::max<size_t>(nslots, 1));
   const size_t o_upart = cv.take<double>(std::max<size_t>(ut.size(), 1));
   const size_t o_nmb = cv.take<double>(std::max(num_layers, 1));
   const size_t o_nb = cv.take<double>(std::max(num_layers, 1));
@@ -299,6 +300,10 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
     p->tcp.gtiles = p->gtiles;
     p->tcp.n_gtiles = p->n_gtiles;
     e = tc::init(tcl, base, dl.data(), num_layers, &p->tcp);
+    if (e == cudaSuccess) {  // the tensor-core path works from a bf16 copy of Q
+      tc::refresh(p->tcp, p->sh, nullptr);
+      e = cudaGetLastError();
+    }
   }
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
   if (e != cudaSuccess) {
@@ -382,6 +387,13 @@ dion_status dion_get_device_status(dion_plan *p, int32_t clear, int32_t *code_ou
 }
 
 int32_t dion_step_launch_count(const dion_plan *p) { return p ? p->launches_per_step : 0; }
+
+dion_status dion_plan_refresh(dion_plan *p, void *stream) {
+  if (!p) return DION_ERR_INVALID_ARG;
+  if (p->precision == DION_PREC_FP32) return DION_OK;
+  tc::refresh(p->tcp, p->sh, static_cast<cudaStream_t>(stream));
+  return cudaGetLastError() == cudaSuccess ? DION_OK : DION_ERR_CUDA;
+}
 
 static void free_events(dion_plan *p) {
   for (cudaEvent_t e : p->ev) cudaEventDestroy(e);

@@ -14,6 +14,7 @@
 // Every HBM byte of the pass (read B, X; write M, X) moves by TMA in 128-byte rows.
 #include "tc.cuh"
 #include "tc_common.cuh"
+#include "tc_kernels.cuh"
 
 #include <algorithm>
 #include <cstring>
@@ -49,29 +50,6 @@ constexpr uint32_t U_EPI = 128u * 32u * 4u;           // one 128 x 32 fp32 box
 constexpr uint32_t U_SMEM = 1024u + U_STAGES * U_STAGE + 4u * U_EPI + 256u;
 constexpr int U_THREADS = 192;
 constexpr uint32_t U_IDESC = idesc_bf16(128, 128, false, false);
-
-struct Abort {
-  int *flag;
-  __device__ bool wait(uint64_t *bar, uint32_t parity, int32_t *status) const {
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = globaltimer_ns();
-    for (uint32_t i = 1;; ++i) {
-      if (mbar_try_wait(bar, parity)) return true;
-      if ((i & 255u) == 0) {
-        if (*(volatile int *)flag) return false;
-        if (globaltimer_ns() - t0 > kWaitLimitNs) {
-          set_status(status, ST_TIMEOUT);
-          *(volatile int *)flag = 1;
-          return false;
-        }
-      }
-    }
-  }
-};
-
-__device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
-  return reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
-}
 
 __global__ void __launch_bounds__(U_THREADS, 1)
     tc_update_kernel(Shared sh, const int4 *__restrict__ tiles, int ntiles, const LayerMaps *__restrict__ maps,
@@ -200,7 +178,7 @@ __global__ void __launch_bounds__(U_THREADS, 1)
         ++issued;
       };
       if (leader) issue(0);
-      if (!ab.wait(&acc_full[b], aph, sh.status)) break;
+      if (!named_and(1, 128, ab.wait(&acc_full[b], aph, sh.status))) break;
       tc_fence_after();
       float ss = 0.f;
       for (int j = 0; j < nj; ++j) {
@@ -210,7 +188,7 @@ __global__ void __launch_bounds__(U_THREADS, 1)
         tmem_ld32(tmem + ((32u * (warp & 3)) << 16) + b * 256u + j * 32, u1);
         tmem_ld32(tmem + ((32u * (warp & 3)) << 16) + b * 256u + 128u + j * 32, u2);
         tmem_ld_wait();
-        if (!ab.wait(&epi_full[eb], eph, sh.status)) { ok = false; break; }
+        if (!named_and(1, 128, ab.wait(&epi_full[eb], eph, sh.status))) { ok = false; break; }
         uint8_t *bs = epi + eb * 2 * U_EPI;
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
@@ -264,6 +242,16 @@ __global__ void __launch_bounds__(U_THREADS, 1)
 }
 
 // ========================================================================= host side ===
+namespace {
+size_t bq_tiles(int64_t m) { return (size_t)((m + 127) / 128); }
+}  // namespace
+
+size_t norm_slots(const dion_layer *layers, int32_t L) {
+  size_t n = 0;
+  for (int32_t l = 0; l < L; ++l) n += 8 * bq_tiles(layers[l].m);
+  return n;
+}
+
 dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int num_sms, size_t start,
                    TcLayout *out) {
   if (precision != DION_PREC_BF16) return DION_ERR_UNSUPPORTED;
@@ -279,33 +267,57 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
   lo.o_phi.resize(L);
   lo.o_rhi.resize(L);
   lo.o_qnhi.resize(L);
+  lo.o_bh.resize(L);
+  int32_t fslot = 0;
   for (int32_t l = 0; l < L; ++l) {
     const dion_layer &ly = layers[l];
-    const int64_t ldp = (ly.r + 7) / 8 * 8;
+    const int64_t ldp = (ly.r + 7) / 8 * 8, ldbh = (ly.n + 7) / 8 * 8;
+    lo.max_r = std::max<int32_t>(lo.max_r, (int32_t)ly.r);
     lo.o_phi[l] = take(ly.m * ldp * 2);
     lo.o_rhi[l] = take(ly.n * ldp * 2);
     lo.o_qnhi[l] = take(ly.n * ldp * 2);
+    lo.o_bh[l] = take(ly.m * ldbh * 2);
     for (int64_t mb = 0; mb < (ly.m + 127) / 128; ++mb)
       for (int64_t nb = 0; nb < (ly.n + 127) / 128; ++nb)
         lo.utiles.push_back(make_int4(l, (int)mb, (int)nb, (int)lo.utiles.size()));
     const int64_t prow = std::max<int64_t>(1, std::min<int64_t>(ly.m, 16384 / ly.r));
     for (int64_t r0 = 0; r0 < ly.m; r0 += prow)
       lo.ptiles.push_back(make_int4(l, (int)r0, (int)std::min(prow, ly.m - r0), 0));
+    const int64_t qrow = std::max<int64_t>(1, std::min<int64_t>(ly.n, 16384 / ly.r));
+    for (int64_t r0 = 0; r0 < ly.n; r0 += qrow)
+      lo.qtiles.push_back(make_int4(l, (int)r0, (int)std::min(qrow, ly.n - r0), 0));
+    for (int64_t mb = 0; mb < (ly.m + 127) / 128; ++mb) lo.ftiles.push_back(make_int4(l, (int)mb, 0, fslot++));
+    for (int64_t nb = 0; nb < (ly.n + 127) / 128; ++nb) lo.rtiles.push_back(make_int4(l, (int)nb, 0, 0));
   }
+  // longest K loops first (static round-robin over the SMs then balances well)
+  std::stable_sort(lo.ftiles.begin(), lo.ftiles.end(),
+                   [&](const int4 &a, const int4 &b) { return layers[a.x].n > layers[b.x].n; });
+  std::stable_sort(lo.rtiles.begin(), lo.rtiles.end(),
+                   [&](const int4 &a, const int4 &b) { return layers[a.x].m > layers[b.x].m; });
   lo.o_maps = take(sizeof(LayerMaps) * std::max(L, 1), 128);
   lo.o_utiles = take(sizeof(int4) * std::max<size_t>(lo.utiles.size(), 1));
   lo.o_ptiles = take(sizeof(int4) * std::max<size_t>(lo.ptiles.size(), 1));
+  lo.o_ftiles = take(sizeof(int4) * std::max<size_t>(lo.ftiles.size(), 1));
+  lo.o_rtiles = take(sizeof(int4) * std::max<size_t>(lo.rtiles.size(), 1));
+  lo.o_qtiles = take(sizeof(int4) * std::max<size_t>(lo.qtiles.size(), 1));
   lo.end = off;
   (void)num_sms;
   return DION_OK;
 }
 
 void bind(const TcLayout &lo, char *base, DevLayer *dl, int32_t L, TcPlan *tp) {
+  int32_t fslot = 0;
   for (int32_t l = 0; l < L; ++l) {
     dl[l].P_hi = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_phi[l]);
     dl[l].R_hi = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_rhi[l]);
     dl[l].Qn_hi = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_qnhi[l]);
-    // the update tiles replace the CUDA-core update's partial slots
+    dl[l].Bh = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_bh[l]);
+    dl[l].ldbh = (dl[l].n + 7) / 8 * 8;
+    // norm partials: 8 slots (one per producer warp) per 128-row tile of the fused B Q kernel
+    const int32_t tiles = (int32_t)bq_tiles(dl[l].m);
+    dl[l].bpart_off = 8 * fslot;
+    dl[l].bpart_cnt = 8 * tiles;
+    fslot += tiles;
     dl[l].upart_off = -1;
   }
   int32_t cur = -1;
@@ -323,7 +335,14 @@ void bind(const TcLayout &lo, char *base, DevLayer *dl, int32_t L, TcPlan *tp) {
   tp->n_utiles = (int32_t)lo.utiles.size();
   tp->ptiles = reinterpret_cast<int4 *>(base + lo.o_ptiles);
   tp->n_ptiles = (int32_t)lo.ptiles.size();
+  tp->ftiles = reinterpret_cast<int4 *>(base + lo.o_ftiles);
+  tp->n_ftiles = (int32_t)lo.ftiles.size();
+  tp->rtiles = reinterpret_cast<int4 *>(base + lo.o_rtiles);
+  tp->n_rtiles = (int32_t)lo.rtiles.size();
+  tp->qtiles = reinterpret_cast<int4 *>(base + lo.o_qtiles);
+  tp->n_qtiles = (int32_t)lo.qtiles.size();
   tp->precision = lo.precision;
+  tp->max_r = lo.max_r;
 }
 
 cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, TcPlan *tp) {
@@ -333,39 +352,62 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   for (int32_t l = 0; l < L; ++l) {
     const DevLayer &d = dl[l];
     LayerMaps &m = maps[l];
-    const uint64_t pitch16 = (uint64_t)d.ldp * 2;
-    bool ok = encode_bf16_2d(&m.P_hi, d.P_hi, d.r, d.m, pitch16, 64, 128) &&
-              encode_bf16_2d(&m.R_hi, d.R_hi, d.r, d.n, pitch16, 64, 128) &&
-              encode_bf16_2d(&m.Qn_hi, d.Qn_hi, d.r, d.n, pitch16, 64, 128) &&
-              encode_f32_2d(&m.Mf, d.M, d.n, d.m, (uint64_t)d.ldm * 4, 32, 128) &&
-              encode_f32_2d(&m.Xf, d.X, d.n, d.m, (uint64_t)d.ldx * 4, 32, 128);
+    const uint64_t p16 = (uint64_t)d.ldp * 2, p32 = (uint64_t)d.ldp * 4;
+    const bool ok = encode_bf16_2d(&m.P_hi, d.P_hi, d.r, d.m, p16, 64, 128) &&
+                    encode_bf16_2d(&m.R_hi, d.R_hi, d.r, d.n, p16, 64, 128) &&
+                    encode_bf16_2d(&m.Qn_hi, d.Qn_hi, d.r, d.n, p16, 64, 128) &&
+                    encode_f32_2d(&m.Mf, d.M, d.n, d.m, (uint64_t)d.ldm * 4, 32, 128) &&
+                    encode_f32_2d(&m.Xf, d.X, d.n, d.m, (uint64_t)d.ldx * 4, 32, 128) &&
+                    encode_bf16_2d(&m.Qn_mn, d.Qn_hi, d.r, d.n, p16, 64, 64) &&
+                    encode_bf16_2d(&m.P_mn, d.P_hi, d.r, d.m, p16, 64, 64) &&
+                    encode_bf16_2d(&m.Bh_mn, d.Bh, d.n, d.m, (uint64_t)d.ldbh * 2, 64, 64) &&
+                    encode_f32_2d(&m.Praw, d.P_raw, d.r, d.m, p32, 32, 128) &&
+                    encode_f32_2d(&m.Rst, d.R, d.r, d.n, p32, 32, 128);
     if (!ok) return cudaErrorInvalidValue;
   }
+  auto up = [&](int4 *dst, const std::vector<int4> &v) {
+    return v.empty() ? cudaSuccess : cudaMemcpy(dst, v.data(), sizeof(int4) * v.size(), cudaMemcpyHostToDevice);
+  };
   cudaError_t e = cudaMemcpy(tp->maps, maps.data(), sizeof(LayerMaps) * maps.size(), cudaMemcpyHostToDevice);
-  if (e == cudaSuccess && !lo.utiles.empty())
-    e = cudaMemcpy(tp->utiles, lo.utiles.data(), sizeof(int4) * lo.utiles.size(), cudaMemcpyHostToDevice);
-  if (e == cudaSuccess && !lo.ptiles.empty())
-    e = cudaMemcpy(tp->ptiles, lo.ptiles.data(), sizeof(int4) * lo.ptiles.size(), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = up(tp->utiles, lo.utiles);
+  if (e == cudaSuccess) e = up(tp->ptiles, lo.ptiles);
+  if (e == cudaSuccess) e = up(tp->ftiles, lo.ftiles);
+  if (e == cudaSuccess) e = up(tp->rtiles, lo.rtiles);
+  if (e == cudaSuccess) e = up(tp->qtiles, lo.qtiles);
+  // shared-memory budget: stages of (128 x 64 A tile + r/64 boxes of 64 x 64) + 2 output boxes
+  const uint32_t nb64 = (uint32_t)std::max(1, (lo.max_r + 63) / 64);
+  const uint32_t stage = 128u * 64u * 2u + nb64 * 64u * 64u * 2u;
+  const uint32_t budget = 227u * 1024u - 1024u - 2u * 128u * 32u * 4u - 512u - 256u;
+  const int stages = (int)std::min<uint32_t>(4u, budget / stage);
+  if (stages < 2) return cudaErrorInvalidValue;
+  tp->nb64 = nb64;
+  tp->f_stages = tp->r_stages = stages;
+  tp->f_smem = form_bq_smem(stages, stage);
+  tp->r_smem = btp_smem(stages, stage);
+  uint32_t cols = 32;
+  while (cols < (uint32_t)((lo.max_r + 15) / 16 * 16)) cols <<= 1;
+  tp->tmem_cols = cols;
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(tc_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)U_SMEM);
+  if (e == cudaSuccess) e = setup_bq_kernels(tp->f_smem, tp->r_smem);
   int dev = 0, sms = 0;
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   tp->num_sms = sms;
-  tp->launches = 18;
+  tp->launches = 17;
   return e;
 }
 
 int32_t launches_per_step(const TcPlan &tp) { return tp.launches; }
 
+void refresh(const TcPlan &tp, const Shared &sh, cudaStream_t s) { launch_qn_refresh(sh, tp, s); }
+
 void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, const int4 *btiles,
           int32_t n_btiles, const int4 *ctiles, int32_t n_ctiles, size_t chol_smem, cudaStream_t s) {
-  launch_form_b(sh, btiles, n_btiles, s);
-  tick(p, s, "form_b");
+  launch_form_bq(sh, tp, s);  // B = M + G, ||B||, ||M_{t-1}||, P = B Q_{t-1}
+  tick(p, s, "tc_form_bq");
   launch_gate(sh, a, s);
   tick(p, s, "gate");
-  launch_gemm(sh, tp.probs[0], tp.gtiles[0], tp.n_gtiles[0], s);  // P = B Q
-  tick(p, s, "gemm_bq");
   static const char *kGram[3] = {"gemm_gram0", "gemm_gram1", "gemm_gram2"};
   static const char *kChol[3] = {"chol_inv0", "chol_inv1", "chol_inv2"};
   static const char *kTrsm[3] = {"gemm_trsm0", "gemm_trsm1", "gemm_trsm2"};
@@ -377,12 +419,12 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, c
     launch_gemm(sh, tp.probs[4 + pass], tp.gtiles[4 + pass], tp.n_gtiles[4 + pass], s);
     tick(p, s, kTrsm[pass]);
   }
-  launch_gemm(sh, tp.probs[7], tp.gtiles[7], tp.n_gtiles[7], s);  // R = B^T P
-  tick(p, s, "gemm_btp");
-  launch_colnorm(sh, ctiles, n_ctiles, a.eps_col, s);  // Q_t, and bf16 R, Q_t
-  tick(p, s, "colnorm");
   if (tp.n_ptiles > 0) cvt_p_kernel<<<tp.n_ptiles, kCvtThreads, 0, s>>>(sh, tp.ptiles);
   tick(p, s, "cvt_p");
+  launch_btp(sh, tp, s);  // R = B^T P
+  tick(p, s, "tc_btp");
+  launch_colnorm(sh, ctiles, n_ctiles, a.eps_col, s);  // Q_t, and bf16 R, Q_t
+  tick(p, s, "colnorm");
   if (tp.n_utiles > 0) {
     const int grid = std::min(tp.n_utiles, std::max(tp.num_sms, 1));
     tc_update_kernel<<<grid, U_THREADS, U_SMEM, s>>>(sh, tp.utiles, tp.n_utiles, tp.maps, a.mu, a.eta);

@@ -14,20 +14,28 @@ namespace tc {
 // Per-layer TMA descriptors (device memory, 64-byte aligned).  bf16 maps use a 128-byte
 // swizzle with 64-element inner boxes; fp32 maps use 32-element (128-byte) inner boxes.
 struct LayerMaps {
-  CUtensorMap P_hi;   // m x r bf16 (pitch rp):   box {64, 128}  A operand of the update
-  CUtensorMap R_hi;   // n x r bf16 (pitch rp):   box {64, 128}  B operand (P R^T)
-  CUtensorMap Qn_hi;  // n x r bf16 (pitch rp):   box {64, 128}  B operand (P Q_t^T)
-  CUtensorMap Mf;     // m x n fp32 (caller M):  box {32, 128}  B in / M_t out
-  CUtensorMap Xf;     // m x n fp32 (caller X):  box {32, 128}  X in / out
+  CUtensorMap P_hi;   // m x r bf16:  box {64, 128}  update: A operand (K = r)
+  CUtensorMap R_hi;   // n x r bf16:  box {64, 128}  update: B operand of P R^T
+  CUtensorMap Qn_hi;  // n x r bf16:  box {64, 128}  update: B operand of P Q_t^T
+  CUtensorMap Mf;     // m x n fp32 (caller M): box {32, 128}  update: B in / M_t out
+  CUtensorMap Xf;     // m x n fp32 (caller X): box {32, 128}  update: X in / out
+  CUtensorMap Qn_mn;  // n x r bf16:  box {64, 64}   B Q: MN-major B operand (K = n)
+  CUtensorMap P_mn;   // m x r bf16:  box {64, 64}   B^T P: MN-major B operand (K = m)
+  CUtensorMap Bh_mn;  // m x n bf16:  box {64, 64}   B^T P: MN-major A operand (K = m)
+  CUtensorMap Praw;   // m x r fp32:  box {32, 128}  B Q: output store
+  CUtensorMap Rst;    // n x r fp32:  box {32, 128}  B^T P: output store
 };
 
 struct TcLayout {
   size_t end = 0;
   size_t o_maps = 0;
-  size_t o_utiles = 0, o_ptiles = 0;
-  std::vector<size_t> o_phi, o_rhi, o_qnhi;
-  std::vector<int4> utiles, ptiles;  // update tiles {layer, m-block, n-block, slot}; P-convert tiles
+  size_t o_utiles = 0, o_ptiles = 0, o_ftiles = 0, o_rtiles = 0, o_qtiles = 0;
+  std::vector<size_t> o_phi, o_rhi, o_qnhi, o_bh;
+  // update tiles {layer, m-block, n-block, slot}; P-convert tiles {layer, row0, rows, 0};
+  // B Q tiles {layer, m-block, 0, slot}; B^T P tiles {layer, n-block, 0, 0}; Q-copy tiles
+  std::vector<int4> utiles, ptiles, ftiles, rtiles, qtiles;
   int32_t precision = 0;
+  int32_t max_r = 0;
 };
 
 struct TcPlan {
@@ -36,6 +44,15 @@ struct TcPlan {
   int32_t n_utiles = 0;
   int4 *ptiles = nullptr;
   int32_t n_ptiles = 0;
+  int4 *ftiles = nullptr;
+  int32_t n_ftiles = 0;
+  int4 *rtiles = nullptr;
+  int32_t n_rtiles = 0;
+  int4 *qtiles = nullptr;
+  int32_t n_qtiles = 0;
+  int32_t max_r = 0;
+  int32_t f_stages = 0, r_stages = 0;
+  uint32_t f_smem = 0, r_smem = 0, nb64 = 0, tmem_cols = 0;
   int32_t num_sms = 0;
   int32_t precision = 0;
   int32_t launches = 0;
@@ -59,6 +76,11 @@ int32_t launches_per_step(const TcPlan &tp);
 void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, const int4 *btiles,
           int32_t n_btiles, const int4 *ctiles, int32_t n_ctiles, size_t chol_smem, cudaStream_t s);
 void destroy(TcPlan *tp);
+// Re-derives the bf16 copy of every layer's Q from the caller's fp32 Q (plan creation and
+// dion_plan_refresh).
+void refresh(const TcPlan &tp, const Shared &sh, cudaStream_t s);
+// Number of B Q tiles (one norm-partial slot each) the layout needs for these layers.
+size_t norm_slots(const dion_layer *layers, int32_t L);
 
 }  // namespace tc
 }  // namespace cd

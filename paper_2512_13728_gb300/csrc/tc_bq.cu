@@ -1,0 +1,447 @@
+// tcgen05 kernels of the power iteration and of R (DION_PREC_BF16):
+//
+//   tc_form_bq   B = M + G written back into M (Algorithm 1/2 buffer line), its bf16 copy
+//                Bh, the fp64 per-tile partials of ||B||^2 and ||M_{t-1}||^2 (Algorithm 2's
+//                RMMC and Equation 1), and P = B Q_{t-1} (PowerIter) -- one pass over M and G.
+//                Tile = 128 rows of one layer; K loop over n in 64-column chunks.
+//                  warps 0..7   producers: coalesced loads of M and G, B in registers, stores of
+//                               B and Bh, bf16 B into the K-major 128-byte-swizzled A operand;
+//                  warp 8       TMA: the bf16 copy of Q (n x r) as an MN-major B operand;
+//                  warp 9       MMA: 128 x N x 16 tcgen05.mma (N <= 256 per instruction) into a
+//                               128 x r fp32 TMEM accumulator;
+//                  warps 10..13 epilogue: TMEM -> swizzled shared boxes -> TMA store of P (fp32).
+//   tc_btp       R = B^T P (after Orthogonalize).  Tile = 128 columns of B (rows of R); K loop
+//                over m.  A = Bh^T and B = P are both read as MN-major operands straight from
+//                the row-major bf16 copies Bh (m x n) and P_hi (m x r), so no transpose is made.
+//                  warp 0 TMA, warp 1 MMA, warps 2..5 epilogue (TMA store of R, fp32).
+//   qn_refresh   the bf16 copy of the caller's Q (plan creation, dion_plan_refresh).
+#include "tc.cuh"
+#include "tc_common.cuh"
+#include "tc_kernels.cuh"
+
+namespace cd {
+namespace tc {
+
+constexpr uint32_t OPB_A = 128u * 64u * 2u;   // 128 x 64 bf16 A-operand tile (16 KB)
+constexpr uint32_t BOX64 = 64u * 64u * 2u;    // 64 x 64 bf16 MN-major box (8 KB)
+constexpr uint32_t EPI_BOX = 128u * 32u * 4u; // 128 x 32 fp32 output box (16 KB)
+
+__device__ __forceinline__ uint32_t rpad16(int64_t r) { return (uint32_t)((r + 15) / 16 * 16); }
+
+// ---------------------------------------------------------------------------------------
+// Epilogue shared by tc_form_bq and tc_btp: the 128 x r fp32 accumulator in TMEM is written
+// to global memory through two 16 KB swizzled staging boxes and TMA stores (rows/columns
+// outside the matrix are clipped by the store).  Called by 128 threads (4 warps covering the
+// 4 TMEM lane groups); `leader` issues the stores.
+__device__ __forceinline__ void store_accumulator(uint32_t tmem, int warp, int lane, bool leader, uint8_t *stg,
+                                                  const CUtensorMap *map, int64_t r, int32_t row0,
+                                                  uint32_t &ecount, uint32_t bar_id) {
+  const uint32_t lg = (uint32_t)(warp & 3), row = 32u * lg + lane;
+  const int nch = (int)((r + 31) / 32);
+  for (int j = 0; j < nch; ++j) {
+    const uint32_t eb = ecount & 1u;
+    uint8_t *box = stg + eb * EPI_BOX;
+    if (leader) bulk_wait_read<1>();  // the store issued two boxes ago has read this buffer
+    named_sync(bar_id, 128);
+    uint32_t v[32];
+    tmem_ld32(tmem + (lg * 32u << 16) + j * 32, v);
+    tmem_ld_wait();
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      float4 f = make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]), __uint_as_float(v[4 * q + 2]),
+                             __uint_as_float(v[4 * q + 3]));
+      *reinterpret_cast<float4 *>(box + sw128_f32(row, q)) = f;
+    }
+    fence_async_smem();
+    named_sync(bar_id, 128);
+    if (leader) {
+      tma_store_2d(map, box, j * 32, row0);
+      bulk_commit();
+    }
+    ++ecount;
+  }
+}
+
+// =============================================================== B = M + G, P = B Q ===
+constexpr int F_THREADS = 14 * 32;
+
+template <int GT>
+__device__ __forceinline__ void load_group(const DevLayer &L, int64_t gi, int64_t gc, float m[4], float g[4]) {
+  const bool full = gi < L.m && gc + 4 <= L.n;
+  if (full) {
+    const float4 mv = *reinterpret_cast<const float4 *>(L.M + gi * L.ldm + gc);
+    m[0] = mv.x; m[1] = mv.y; m[2] = mv.z; m[3] = mv.w;
+    if (GT == DT_BF16) {
+      const uint2 gv = *reinterpret_cast<const uint2 *>(static_cast<const __nv_bfloat16 *>(L.G) + gi * L.ldg + gc);
+      g[0] = bf16_bits_to_float(gv.x & 0xffffu); g[1] = bf16_bits_to_float(gv.x >> 16);
+      g[2] = bf16_bits_to_float(gv.y & 0xffffu); g[3] = bf16_bits_to_float(gv.y >> 16);
+    } else {
+      const float4 gv = *reinterpret_cast<const float4 *>(static_cast<const float *>(L.G) + gi * L.ldg + gc);
+      g[0] = gv.x; g[1] = gv.y; g[2] = gv.z; g[3] = gv.w;
+    }
+  } else {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const bool in = gi < L.m && gc + e < L.n;
+      m[e] = in ? L.M[gi * L.ldm + gc + e] : 0.f;
+      if (GT == DT_BF16) g[e] = in ? __bfloat162float(static_cast<const __nv_bfloat16 *>(L.G)[gi * L.ldg + gc + e]) : 0.f;
+      else g[e] = in ? static_cast<const float *>(L.G)[gi * L.ldg + gc + e] : 0.f;
+    }
+  }
+}
+
+// One 128 x 64 chunk: 256 producer threads, 8 groups of 4 columns each
+// (row = u * 16 + warp * 2 + lane / 16, columns 4 * (lane % 16) ..).
+template <int GT>
+__device__ __forceinline__ void produce_chunk(const DevLayer &L, int64_t r0, int64_t c0, uint8_t *sA, int warp,
+                                              int lane, float &sb, float &sm, const Abort &ab, uint64_t *empty_bar,
+                                              uint32_t parity, int32_t *status, bool &ok) {
+  const int prow = warp * 2 + (lane >> 4), pcol = (lane & 15) * 4;
+  float mv[8][4], gv[8][4];
+#pragma unroll
+  for (int u = 0; u < 8; ++u) load_group<GT>(L, r0 + u * 16 + prow, c0 + pcol, mv[u], gv[u]);
+  if (!__all_sync(0xffffffffu, ab.wait(empty_bar, parity, status))) {  // warp-uniform decision
+    ok = false;
+    return;
+  }
+#pragma unroll
+  for (int u = 0; u < 8; ++u) {
+    const int64_t row = u * 16 + prow, gi = r0 + row, gc = c0 + pcol;
+    float b[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      sm = fmaf(mv[u][e], mv[u][e], sm);
+      b[e] = mv[u][e] + gv[u][e];
+      sb = fmaf(b[e], b[e], sb);
+    }
+    const __nv_bfloat162 h01 = __floats2bfloat162_rn(b[0], b[1]), h23 = __floats2bfloat162_rn(b[2], b[3]);
+    uint2 hv;
+    hv.x = *reinterpret_cast<const uint32_t *>(&h01);
+    hv.y = *reinterpret_cast<const uint32_t *>(&h23);
+    if (gi < L.m && gc + 4 <= L.n) {
+      *reinterpret_cast<float4 *>(L.M + gi * L.ldm + gc) = make_float4(b[0], b[1], b[2], b[3]);
+      *reinterpret_cast<uint2 *>(L.Bh + gi * L.ldbh + gc) = hv;
+    } else if (gi < L.m) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        if (gc + e < L.n) {
+          L.M[gi * L.ldm + gc + e] = b[e];
+          L.Bh[gi * L.ldbh + gc + e] = __float2bfloat16_rn(b[e]);
+        }
+    }
+    // K-major 128-byte-swizzled A operand; out-of-range elements are 0
+    *reinterpret_cast<uint2 *>(sA + sw128_offset((uint32_t)row, (uint32_t)(pcol >> 3)) + (pcol & 7) * 2) = hv;
+  }
+}
+
+__global__ void __launch_bounds__(F_THREADS, 1)
+    tc_form_bq_kernel(Shared sh, const int4 *__restrict__ tiles, int ntiles, const LayerMaps *__restrict__ maps,
+                      int nstages, uint32_t stage_bytes, uint32_t tmem_cols) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = align1024(smem_raw);
+  uint8_t *stg = smem + nstages * stage_bytes;  // 2 output boxes
+  uint64_t *bars = reinterpret_cast<uint64_t *>(stg + 2 * EPI_BOX);
+  uint64_t *a_full = bars, *q_full = bars + nstages, *empty = bars + 2 * nstages;
+  uint64_t *acc_full = bars + 3 * nstages, *acc_empty = acc_full + 1, *drain = acc_full + 2;
+  __shared__ uint32_t tmem_base_s;
+  __shared__ int abort_s;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const Abort ab{&abort_s};
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < nstages; ++i) {
+      mbar_init(&a_full[i], 8);  // one arrive per producer warp
+      mbar_init(&q_full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    mbar_init(acc_full, 1);
+    mbar_init(acc_empty, 128);
+    mbar_init(drain, 1);
+    abort_s = 0;
+    fence_mbar_init();
+  }
+  if (warp == 9) {
+    tmem_alloc(&tmem_base_s, tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_s;
+
+  if (warp < 8) {
+    // ------------------------------------------------------------------ producers
+    uint32_t it = 0;
+    bool ok = true;
+    for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+      const int4 t = tiles[ti];
+      const DevLayer &L = sh.layers[t.x];
+      const int64_t r0 = (int64_t)t.y * 128;
+      const int kch = (int)((L.n + 63) / 64);
+      double vb = 0.0, vm = 0.0;  // fp32 sums of 32 squares per chunk, folded into fp64
+      for (int kc = 0; kc < kch && ok; ++kc, ++it) {
+        const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
+        uint8_t *sA = smem + s * stage_bytes;
+        float sb = 0.f, sm = 0.f;
+        if (L.g_dtype == DT_BF16)
+          produce_chunk<DT_BF16>(L, r0, (int64_t)kc * 64, sA, warp, lane, sb, sm, ab, &empty[s], ph ^ 1u, sh.status, ok);
+        else
+          produce_chunk<DT_FP32>(L, r0, (int64_t)kc * 64, sA, warp, lane, sb, sm, ab, &empty[s], ph ^ 1u, sh.status, ok);
+        if (!ok) break;
+        vb += (double)sb;
+        vm += (double)sm;
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&a_full[s]);
+      }
+      if (!ok) break;
+      // each producer warp owns norm-partial slot 8 * tile + warp (fixed-order sum in the gate)
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        vb += __shfl_xor_sync(0xffffffffu, vb, o);
+        vm += __shfl_xor_sync(0xffffffffu, vm, o);
+      }
+      if (lane == 0) {
+        sh.bpart[2 * (8 * t.w + warp)] = vb;
+        sh.bpart[2 * (8 * t.w + warp) + 1] = vm;
+      }
+    }
+  } else if (warp == 8) {
+    // ------------------------------------------------------------------ TMA (Q operand)
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+        const int4 t = tiles[ti];
+        const DevLayer &L = sh.layers[t.x];
+        const LayerMaps *mp = maps + t.x;
+        const int kch = (int)((L.n + 63) / 64);
+        const int nb = (int)((L.r + 63) / 64);
+        for (int kc = 0; kc < kch; ++kc, ++it) {
+          const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
+          if (!ab.wait(&empty[s], ph ^ 1u, sh.status)) { ok = false; break; }
+          uint8_t *sQ = smem + s * stage_bytes + OPB_A;
+          mbar_expect_tx(&q_full[s], (uint32_t)nb * BOX64);
+          for (int j = 0; j < nb; ++j) tma_load_2d(sQ + j * BOX64, &mp->Qn_mn, &q_full[s], j * 64, kc * 64);
+        }
+      }
+      for (uint32_t k = (it > (uint32_t)nstages ? it - nstages : 0); k < it; ++k)
+        mbar_wait(&q_full[k % nstages], (k / nstages) & 1u, sh.status);
+    }
+  } else if (warp == 9) {
+    // ------------------------------------------------------------------ MMA
+    if (lane == 0) {
+      uint32_t it = 0, tcount = 0;
+      bool ok = true;
+      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x, ++tcount) {
+        const int4 t = tiles[ti];
+        const DevLayer &L = sh.layers[t.x];
+        const int kch = (int)((L.n + 63) / 64);
+        const uint32_t np = rpad16(L.r), nparts = (np + 255) / 256;
+        if (!ab.wait(acc_empty, (tcount & 1u) ^ 1u, sh.status)) break;
+        tc_fence_after();
+        for (int kc = 0; kc < kch; ++kc, ++it) {
+          const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
+          if (!ab.wait(&a_full[s], ph, sh.status) || !ab.wait(&q_full[s], ph, sh.status)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t aB = smem_u32(smem + s * stage_bytes), qB = aB + OPB_A;
+#pragma unroll
+          for (int k16 = 0; k16 < 4; ++k16) {
+            const uint64_t ad = smem_desc_sw128(aB + k16 * 32, 0, 1024);
+            for (uint32_t part = 0; part < nparts; ++part) {
+              const uint32_t n_here = min(256u, np - part * 256u);
+              const uint64_t bd = smem_desc_sw128(qB + part * 4u * BOX64 + k16 * 2048, BOX64, 1024);
+              umma_bf16(tmem + part * 256u, ad, bd, idesc_bf16(128, n_here, false, true), (kc | k16) ? 1u : 0u);
+            }
+          }
+          umma_commit(&empty[s]);
+        }
+        if (!ok) break;
+        umma_commit(acc_full);
+      }
+      umma_commit(drain);
+      mbar_wait(drain, 0, sh.status);
+    }
+  } else {
+    // ------------------------------------------------------------------ epilogue (warps 10..13)
+    const bool leader = (warp == 10 && lane == 0);
+    uint32_t tcount = 0, ecount = 0;
+    for (int ti = blockIdx.x; ti < ntiles; ti += gridDim.x, ++tcount) {
+      const int4 t = tiles[ti];
+      const DevLayer &L = sh.layers[t.x];
+      if (!named_and(3, 128, ab.wait(acc_full, tcount & 1u, sh.status))) break;
+      tc_fence_after();
+      store_accumulator(tmem, warp, lane, leader, stg, &maps[t.x].Praw, L.r, t.y * 128, ecount, 3);
+      tc_fence_before();
+      mbar_arrive(acc_empty);
+    }
+    if (leader) bulk_wait<0>();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 9) tmem_dealloc(tmem, tmem_cols);
+}
+
+// ========================================================================= R = B^T P ===
+constexpr int R_THREADS = 6 * 32;
+
+__global__ void __launch_bounds__(R_THREADS, 1)
+    tc_btp_kernel(Shared sh, const int4 *__restrict__ tiles, int ntiles, const LayerMaps *__restrict__ maps,
+                  int nstages, uint32_t stage_bytes, uint32_t tmem_cols) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = align1024(smem_raw);
+  uint8_t *stg = smem + nstages * stage_bytes;
+  uint64_t *bars = reinterpret_cast<uint64_t *>(stg + 2 * EPI_BOX);
+  uint64_t *full = bars, *empty = bars + nstages;
+  uint64_t *acc_full = bars + 2 * nstages, *acc_empty = acc_full + 1, *drain = acc_full + 2;
+  __shared__ uint32_t tmem_base_s;
+  __shared__ int abort_s;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const Abort ab{&abort_s};
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < nstages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    mbar_init(acc_full, 1);
+    mbar_init(acc_empty, 128);
+    mbar_init(drain, 1);
+    abort_s = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&tmem_base_s, tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_s;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+        const int4 t = tiles[ti];
+        if (!sh.active[t.x]) continue;
+        const DevLayer &L = sh.layers[t.x];
+        const LayerMaps *mp = maps + t.x;
+        const int kch = (int)((L.m + 63) / 64);
+        const int nb = (int)((L.r + 63) / 64);
+        for (int kc = 0; kc < kch; ++kc, ++it) {
+          const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
+          if (!ab.wait(&empty[s], ph ^ 1u, sh.status)) { ok = false; break; }
+          uint8_t *sA = smem + s * stage_bytes, *sB = sA + OPB_A;
+          mbar_expect_tx(&full[s], OPB_A + (uint32_t)nb * BOX64);
+          tma_load_2d(sA, &mp->Bh_mn, &full[s], t.y * 128, kc * 64);
+          tma_load_2d(sA + BOX64, &mp->Bh_mn, &full[s], t.y * 128 + 64, kc * 64);
+          for (int j = 0; j < nb; ++j) tma_load_2d(sB + j * BOX64, &mp->P_mn, &full[s], j * 64, kc * 64);
+        }
+      }
+      for (uint32_t k = (it > (uint32_t)nstages ? it - nstages : 0); k < it; ++k)
+        mbar_wait(&full[k % nstages], (k / nstages) & 1u, sh.status);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      uint32_t it = 0, tcount = 0;
+      bool ok = true;
+      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+        const int4 t = tiles[ti];
+        if (!sh.active[t.x]) continue;
+        const DevLayer &L = sh.layers[t.x];
+        const int kch = (int)((L.m + 63) / 64);
+        const uint32_t np = rpad16(L.r), nparts = (np + 255) / 256;
+        if (!ab.wait(acc_empty, (tcount & 1u) ^ 1u, sh.status)) break;
+        tc_fence_after();
+        for (int kc = 0; kc < kch; ++kc, ++it) {
+          const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
+          if (!ab.wait(&full[s], ph, sh.status)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t aB = smem_u32(smem + s * stage_bytes), bB = aB + OPB_A;
+#pragma unroll
+          for (int k16 = 0; k16 < 4; ++k16) {
+            const uint64_t ad = smem_desc_sw128(aB + k16 * 2048, BOX64, 1024);
+            for (uint32_t part = 0; part < nparts; ++part) {
+              const uint32_t n_here = min(256u, np - part * 256u);
+              const uint64_t bd = smem_desc_sw128(bB + part * 4u * BOX64 + k16 * 2048, BOX64, 1024);
+              umma_bf16(tmem + part * 256u, ad, bd, idesc_bf16(128, n_here, true, true), (kc | k16) ? 1u : 0u);
+            }
+          }
+          umma_commit(&empty[s]);
+        }
+        if (!ok) break;
+        umma_commit(acc_full);
+        ++tcount;
+      }
+      umma_commit(drain);
+      mbar_wait(drain, 0, sh.status);
+    }
+  } else {
+    const bool leader = (warp == 2 && lane == 0);
+    uint32_t tcount = 0, ecount = 0;
+    for (int ti = blockIdx.x; ti < ntiles; ti += gridDim.x) {
+      const int4 t = tiles[ti];
+      if (!sh.active[t.x]) continue;
+      const DevLayer &L = sh.layers[t.x];
+      if (!named_and(1, 128, ab.wait(acc_full, tcount & 1u, sh.status))) break;
+      tc_fence_after();
+      store_accumulator(tmem, warp, lane, leader, stg, &maps[t.x].Rst, L.r, t.y * 128, ecount, 1);
+      tc_fence_before();
+      mbar_arrive(acc_empty);
+      ++tcount;
+    }
+    if (leader) bulk_wait<0>();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, tmem_cols);
+}
+
+// ================================================================== Q -> bf16 copy ===
+__global__ void __launch_bounds__(256) qn_refresh_kernel(Shared sh, const int4 *tiles) {
+  const int4 t = tiles[blockIdx.x];  // {layer, first row, rows, 0}
+  const DevLayer &L = sh.layers[t.x];
+  const int64_t r = L.r, total = (int64_t)t.z * r;
+  for (int64_t e = threadIdx.x; e < total; e += 256) {
+    const int64_t i = t.y + e / r, j = e % r;
+    L.Qn_hi[i * L.ldp + j] = __float2bfloat16_rn(L.Q[i * L.ldq + j]);
+  }
+}
+
+// ======================================================================= launchers ===
+uint32_t form_bq_smem(int nstages, uint32_t stage_bytes) {
+  return 1024u + nstages * stage_bytes + 2 * EPI_BOX + 512u;  // + barriers
+}
+uint32_t btp_smem(int nstages, uint32_t stage_bytes) { return form_bq_smem(nstages, stage_bytes); }
+
+cudaError_t setup_bq_kernels(uint32_t f_smem, uint32_t r_smem) {
+  cudaError_t e = cudaFuncSetAttribute(tc_form_bq_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)f_smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(tc_btp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)r_smem);
+  return e;
+}
+
+void launch_form_bq(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
+  if (tp.n_ftiles <= 0) return;
+  const int grid = std::min(tp.n_ftiles, std::max(tp.num_sms, 1));
+  const uint32_t stage = OPB_A + tp.nb64 * BOX64;
+  tc_form_bq_kernel<<<grid, F_THREADS, tp.f_smem, s>>>(sh, tp.ftiles, tp.n_ftiles, tp.maps, tp.f_stages, stage,
+                                                        tp.tmem_cols);
+}
+
+void launch_btp(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
+  if (tp.n_rtiles <= 0) return;
+  const int grid = std::min(tp.n_rtiles, std::max(tp.num_sms, 1));
+  const uint32_t stage = OPB_A + tp.nb64 * BOX64;
+  tc_btp_kernel<<<grid, R_THREADS, tp.r_smem, s>>>(sh, tp.rtiles, tp.n_rtiles, tp.maps, tp.r_stages, stage,
+                                                    tp.tmem_cols);
+}
+
+void launch_qn_refresh(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
+  if (tp.n_qtiles > 0) qn_refresh_kernel<<<tp.n_qtiles, 256, 0, s>>>(sh, tp.qtiles);
+}
+
+}  // namespace tc
+}  // namespace cd

@@ -182,6 +182,17 @@ __device__ __forceinline__ void bulk_wait() {
 __device__ __forceinline__ void named_sync(uint32_t id, uint32_t count) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
+// named barrier that also ANDs a predicate over the `count` threads: every thread of a role
+// reaches it exactly once per bounded wait, so an abort decision is the same for all of them
+__device__ __forceinline__ bool named_and(uint32_t id, uint32_t count, bool v) {
+  uint32_t out;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\tbar.red.and.pred q, %2, %3, p;\n\tselp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(out)
+      : "r"((uint32_t)v), "r"(id), "r"(count)
+      : "memory");
+  return out != 0;
+}
 
 // fp32 (row, 16-byte chunk) offset inside a SW128 tile of 32-float (128-byte) rows
 __device__ __forceinline__ uint32_t sw128_f32(uint32_t row, uint32_t chunk) {
@@ -190,6 +201,32 @@ __device__ __forceinline__ uint32_t sw128_f32(uint32_t row, uint32_t chunk) {
 
 bool encode_f32_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
                    uint32_t box_inner, uint32_t box_outer);
+
+// Bounded mbarrier wait shared by the roles of one CTA: a role that times out sets
+// DION_ERR_TIMEOUT and the CTA's abort flag, and every other role's wait then returns false
+// promptly so the CTA can drain its in-flight copies, free TMEM and exit.
+struct Abort {
+  int *flag;
+  __device__ bool wait(uint64_t *bar, uint32_t parity, int32_t *status) const {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t i = 1;; ++i) {
+      if (mbar_try_wait(bar, parity)) return true;
+      if ((i & 255u) == 0) {
+        if (*(volatile int *)flag) return false;
+        if (globaltimer_ns() - t0 > kWaitLimitNs) {
+          set_status(status, ST_TIMEOUT);
+          *(volatile int *)flag = 1;
+          return false;
+        }
+      }
+    }
+  }
+};
+
+__device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
+  return reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
 
 }  // namespace tc
 }  // namespace cd

@@ -1,0 +1,18 @@
+// Launch wrappers of the tcgen05 kernels (tc_bq.cu, tc.cu).
+#pragma once
+
+#include "common.cuh"
+#include "tc.cuh"
+
+namespace cd {
+namespace tc {
+
+uint32_t form_bq_smem(int nstages, uint32_t stage_bytes);
+uint32_t btp_smem(int nstages, uint32_t stage_bytes);
+cudaError_t setup_bq_kernels(uint32_t f_smem, uint32_t r_smem);
+void launch_form_bq(const Shared &sh, const TcPlan &tp, cudaStream_t s);
+void launch_btp(const Shared &sh, const TcPlan &tp, cudaStream_t s);
+void launch_qn_refresh(const Shared &sh, const TcPlan &tp, cudaStream_t s);
+
+}  // namespace tc
+}  // namespace cd

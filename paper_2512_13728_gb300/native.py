@@ -35,7 +35,7 @@ DION_PREC_BF16X3 = 2
 DION_MAX_RANK = 512
 
 # Every function declared in include/curvadion.h.
-EXPORTED = ("dion_plan_create", "dion_step", "dion_get_device_status", "dion_step_launch_count",
+EXPORTED = ("dion_plan_create", "dion_step", "dion_get_device_status", "dion_plan_refresh", "dion_step_launch_count",
             "dion_timing_enable", "dion_timing_read", "dion_plan_destroy", "dion_status_string",
             "dion_abi_version")
 
@@ -84,6 +84,8 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     lib.dion_step.restype = C.c_int
     lib.dion_get_device_status.argtypes = [P, C.c_int32, C.POINTER(C.c_int32)]
     lib.dion_get_device_status.restype = C.c_int
+    lib.dion_plan_refresh.argtypes = [P, P]
+    lib.dion_plan_refresh.restype = C.c_int
     lib.dion_step_launch_count.argtypes = [P]
     lib.dion_step_launch_count.restype = C.c_int32
     lib.dion_timing_enable.argtypes = [P, C.c_int32]
@@ -135,6 +137,12 @@ def dion_get_device_status(plan: int, clear: bool = True) -> int:
     if st != DION_OK:
         raise DionError(st, "dion_get_device_status")
     return int(code.value)
+
+
+def dion_plan_refresh(plan: int, stream: int = 0) -> None:
+    st = load().dion_plan_refresh(C.c_void_p(plan), C.c_void_p(stream) if stream else None)
+    if st != DION_OK:
+        raise DionError(st, "dion_plan_refresh")
 
 
 def dion_step_launch_count(plan: int) -> int:
