@@ -53,6 +53,8 @@ struct DevLayer {
   __nv_bfloat16 *Qn_hi;  // n x r : Q (Q_{t-1} when a step starts, Q_t after a sync step)
   __nv_bfloat16 *Bh;     // m x n, pitch ldbh : B rounded to bf16
   int64_t ldbh;
+  float *PT_raw, *PT;    // r x m, pitch ldmt : transposed copies of P_raw and P (tensor-core Gram)
+  int64_t ldmt;
   int32_t bpart_off, bpart_cnt;  // slots of the ||B||^2 / ||M_{t-1}||^2 partials
   int32_t upart_off, upart_cnt;  // slots of the ||M_t||^2 partials
 };

@@ -367,6 +367,12 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int p
   __shared__ int bad;
   __shared__ double trace_s;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  // The Gram producers may write only the lower triangle: mirror it into the upper one, which
+  // the factorization never touches and the shifted retry restores the lower triangle from.
+  for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) {
+    const int64_t i = e / r, j = e % r;
+    if (j > i) S[e] = S[j * r + i];
+  }
   for (int i = tid; i < r; i += kCholThreads) diag0[i] = S[(int64_t)i * r + i];
   __syncthreads();
 
@@ -424,24 +430,52 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int p
 #pragma unroll
       for (int i = 0; i < CB; ++i) DI[i * CBP + lane] = x[i];
     }
-    // T[i][c] = sum_{k=c}^{I0-1} L[I0+i][k] Linv[k][c]   for c < I0
+    // Row block I of L staged in shared memory: Lb[i][k] = L[I0+i][k], k < I0.
     for (int e = tid; e < CB * I0; e += kCholThreads) {
-      const int i = e / I0, c = e % I0;
-      float v = 0.f;
-      if (i < nb) {
-        const float *Lrow = S + (int64_t)(I0 + i) * r;
-        for (int k = c; k < I0; ++k) v = fmaf(Lrow[k], Li[(int64_t)k * r + c], v);
-      }
-      Pn[i * r + c] = v;
+      const int i = e / I0, k = e % I0;
+      Pn[i * I0 + k] = (i < nb) ? S[(int64_t)(I0 + i) * r + k] : 0.f;
     }
     __syncthreads();
-    // Linv row block I: -DI T for c < I0, DI on the diagonal block, 0 to the right
-    for (int e = tid; e < nb * r; e += kCholThreads) {
-      const int i = e / r, c = e % r;
+    // Thread c < I0 owns column c: T[i] = sum_{k=c}^{I0-1} Lb[i][k] Linv[k][c] for the 32 rows
+    // i of the block (one load of Linv[k][c] feeds 32 FMAs), then Linv[I0+i][c] = -(DI T)[i].
+    for (int c = tid; c < I0; c += kCholThreads) {
+      float acc[CB];
+#pragma unroll
+      for (int i = 0; i < CB; ++i) acc[i] = 0.f;
+      // Linv[k][c] = 0 for k < c (upper triangle, stored as zeros), so every lane of a warp can
+      // start at the warp's first column: uniform trip counts, 8 independent loads in flight.
+      const int kbeg = c & ~31;
+      int k = kbeg;
+      for (; k + 8 <= I0; k += 8) {
+        float lk[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) lk[u] = Li[(int64_t)(k + u) * r + c];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+#pragma unroll
+          for (int i = 0; i < CB; ++i) acc[i] = fmaf(Pn[i * I0 + k + u], lk[u], acc[i]);
+      }
+      for (; k < I0; ++k) {
+        const float lk = Li[(int64_t)k * r + c];
+#pragma unroll
+        for (int i = 0; i < CB; ++i) acc[i] = fmaf(Pn[i * I0 + k], lk, acc[i]);
+      }
+#pragma unroll
+      for (int i = CB - 1; i >= 0; --i) {  // in place: row i needs acc[j] for j <= i only
+        float v = 0.f;
+#pragma unroll
+        for (int j = 0; j <= i; ++j) v = fmaf(DI[i * CBP + j], acc[j], v);
+        acc[i] = -v;
+      }
+#pragma unroll
+      for (int i = 0; i < CB; ++i)
+        if (i < nb) Li[(int64_t)(I0 + i) * r + c] = acc[i];
+    }
+    // diagonal block DI and zeros to its right
+    for (int e = tid; e < nb * (r - I0); e += kCholThreads) {
+      const int i = e / (r - I0), c = I0 + e % (r - I0);
       float v = 0.f;
-      if (c < I0) {
-        for (int j = 0; j <= i; ++j) v -= DI[i * CBP + j] * Pn[j * r + c];
-      } else if (c < I0 + nb) {
+      if (c < I0 + nb) {
         const int j = c - I0;
         v = (j <= i) ? DI[i * CBP + j] : 0.f;
       }

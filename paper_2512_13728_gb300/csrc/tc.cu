@@ -30,15 +30,17 @@ namespace tc {
 // P (fp32, ld ldp) -> P_hi (bf16, same pitch) for the update's A operand; active layers only.
 constexpr int kCvtThreads = 256;
 
+// The orthogonalization ends in P after a shifted third pass and in P_raw otherwise.
 __global__ void __launch_bounds__(kCvtThreads) cvt_p_kernel(Shared sh, const int4 *tiles) {
   const int4 t = tiles[blockIdx.x];  // {layer, first row, rows, 0}
   if (!sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
   const int64_t r = L.r, ldp = L.ldp;
+  const float *src = sh.orth_shifted[t.x] ? L.P : L.P_raw;
   const int64_t total = (int64_t)t.z * r;
   for (int64_t e = threadIdx.x; e < total; e += kCvtThreads) {
     const int64_t i = t.y + e / r, j = e % r;
-    L.P_hi[i * ldp + j] = __float2bfloat16_rn(L.P[i * ldp + j]);
+    L.P_hi[i * ldp + j] = __float2bfloat16_rn(src[i * ldp + j]);
   }
 }
 
@@ -268,6 +270,8 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
   lo.o_rhi.resize(L);
   lo.o_qnhi.resize(L);
   lo.o_bh.resize(L);
+  lo.o_ptraw.resize(L);
+  lo.o_pt.resize(L);
   int32_t fslot = 0;
   for (int32_t l = 0; l < L; ++l) {
     const dion_layer &ly = layers[l];
@@ -277,6 +281,11 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
     lo.o_rhi[l] = take(ly.n * ldp * 2);
     lo.o_qnhi[l] = take(ly.n * ldp * 2);
     lo.o_bh[l] = take(ly.m * ldbh * 2);
+    const int64_t ldmt = (ly.m + 7) / 8 * 8;
+    lo.o_ptraw[l] = take(ly.r * ldmt * 4);
+    lo.o_pt[l] = take(ly.r * ldmt * 4);
+    for (int64_t rb = 0; rb < (ly.r + 127) / 128; ++rb) lo.gram_tiles.push_back(make_int4(l, (int)rb, 0, 0));
+    for (int64_t mb = 0; mb < (ly.m + 127) / 128; ++mb) lo.trsm_tiles.push_back(make_int4(l, (int)mb, 0, 0));
     for (int64_t mb = 0; mb < (ly.m + 127) / 128; ++mb)
       for (int64_t nb = 0; nb < (ly.n + 127) / 128; ++nb)
         lo.utiles.push_back(make_int4(l, (int)mb, (int)nb, (int)lo.utiles.size()));
@@ -294,12 +303,16 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
                    [&](const int4 &a, const int4 &b) { return layers[a.x].n > layers[b.x].n; });
   std::stable_sort(lo.rtiles.begin(), lo.rtiles.end(),
                    [&](const int4 &a, const int4 &b) { return layers[a.x].m > layers[b.x].m; });
+  std::stable_sort(lo.gram_tiles.begin(), lo.gram_tiles.end(),
+                   [&](const int4 &a, const int4 &b) { return layers[a.x].m > layers[b.x].m; });
   lo.o_maps = take(sizeof(LayerMaps) * std::max(L, 1), 128);
   lo.o_utiles = take(sizeof(int4) * std::max<size_t>(lo.utiles.size(), 1));
   lo.o_ptiles = take(sizeof(int4) * std::max<size_t>(lo.ptiles.size(), 1));
   lo.o_ftiles = take(sizeof(int4) * std::max<size_t>(lo.ftiles.size(), 1));
   lo.o_rtiles = take(sizeof(int4) * std::max<size_t>(lo.rtiles.size(), 1));
   lo.o_qtiles = take(sizeof(int4) * std::max<size_t>(lo.qtiles.size(), 1));
+  lo.o_gtiles = take(sizeof(int4) * std::max<size_t>(lo.gram_tiles.size(), 1));
+  lo.o_ttiles = take(sizeof(int4) * std::max<size_t>(lo.trsm_tiles.size(), 1));
   lo.end = off;
   (void)num_sms;
   return DION_OK;
@@ -313,6 +326,9 @@ void bind(const TcLayout &lo, char *base, DevLayer *dl, int32_t L, TcPlan *tp) {
     dl[l].Qn_hi = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_qnhi[l]);
     dl[l].Bh = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_bh[l]);
     dl[l].ldbh = (dl[l].n + 7) / 8 * 8;
+    dl[l].PT_raw = reinterpret_cast<float *>(base + lo.o_ptraw[l]);
+    dl[l].PT = reinterpret_cast<float *>(base + lo.o_pt[l]);
+    dl[l].ldmt = (dl[l].m + 7) / 8 * 8;
     // norm partials: 8 slots (one per producer warp) per 128-row tile of the fused B Q kernel
     const int32_t tiles = (int32_t)bq_tiles(dl[l].m);
     dl[l].bpart_off = 8 * fslot;
@@ -341,6 +357,10 @@ void bind(const TcLayout &lo, char *base, DevLayer *dl, int32_t L, TcPlan *tp) {
   tp->n_rtiles = (int32_t)lo.rtiles.size();
   tp->qtiles = reinterpret_cast<int4 *>(base + lo.o_qtiles);
   tp->n_qtiles = (int32_t)lo.qtiles.size();
+  tp->gram_tiles = reinterpret_cast<int4 *>(base + lo.o_gtiles);
+  tp->n_gram_tiles = (int32_t)lo.gram_tiles.size();
+  tp->trsm_tiles = reinterpret_cast<int4 *>(base + lo.o_ttiles);
+  tp->n_trsm_tiles = (int32_t)lo.trsm_tiles.size();
   tp->precision = lo.precision;
   tp->max_r = lo.max_r;
 }
@@ -362,7 +382,14 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
                     encode_bf16_2d(&m.P_mn, d.P_hi, d.r, d.m, p16, 64, 64) &&
                     encode_bf16_2d(&m.Bh_mn, d.Bh, d.n, d.m, (uint64_t)d.ldbh * 2, 64, 64) &&
                     encode_f32_2d(&m.Praw, d.P_raw, d.r, d.m, p32, 32, 128) &&
-                    encode_f32_2d(&m.Rst, d.R, d.r, d.n, p32, 32, 128);
+                    encode_f32_2d(&m.Rst, d.R, d.r, d.n, p32, 32, 128) &&
+                    encode_f32_2d(&m.Pf, d.P, d.r, d.m, p32, 32, 128) &&
+                    encode_f32_2d(&m.PTraw, d.PT_raw, d.m, d.r, (uint64_t)d.ldmt * 4, 32, 128) &&
+                    encode_f32_2d(&m.PT, d.PT, d.m, d.r, (uint64_t)d.ldmt * 4, 32, 128) &&
+                    encode_f32_2d(&m.PTraw_t, d.PT_raw, d.m, d.r, (uint64_t)d.ldmt * 4, 32, 32) &&
+                    encode_f32_2d(&m.PT_t, d.PT, d.m, d.r, (uint64_t)d.ldmt * 4, 32, 32) &&
+                    encode_f32_2d(&m.Sst, d.S, d.r, d.r, (uint64_t)d.r * 4, 32, 128) &&
+                    encode_f32_2d(&m.Linv, d.Linv, d.r, d.r, (uint64_t)d.r * 4, 32, 128);
     if (!ok) return cudaErrorInvalidValue;
   }
   auto up = [&](int4 *dst, const std::vector<int4> &v) {
@@ -374,22 +401,31 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   if (e == cudaSuccess) e = up(tp->ftiles, lo.ftiles);
   if (e == cudaSuccess) e = up(tp->rtiles, lo.rtiles);
   if (e == cudaSuccess) e = up(tp->qtiles, lo.qtiles);
-  // shared-memory budget: stages of (128 x 64 A tile + r/64 boxes of 64 x 64) + 2 output boxes
+  if (e == cudaSuccess) e = up(tp->gram_tiles, lo.gram_tiles);
+  if (e == cudaSuccess) e = up(tp->trsm_tiles, lo.trsm_tiles);
+  // shared-memory budget: operand stages + 2 staging buffers of (128 x 32 + 4 x 32 x 32) fp32
+  const uint32_t budget = 227u * 1024u - 1024u - 4u * 128u * 32u * 4u - 512u - 256u;
   const uint32_t nb64 = (uint32_t)std::max(1, (lo.max_r + 63) / 64);
-  const uint32_t stage = 128u * 64u * 2u + nb64 * 64u * 64u * 2u;
-  const uint32_t budget = 227u * 1024u - 1024u - 2u * 128u * 32u * 4u - 512u - 256u;
+  const uint32_t stage = 128u * 64u * 2u + nb64 * 64u * 64u * 2u;  // bf16: A tile + r/64 boxes
   const int stages = (int)std::min<uint32_t>(4u, budget / stage);
-  if (stages < 2) return cudaErrorInvalidValue;
+  const uint32_t nb128 = (uint32_t)std::max(1, (lo.max_r + 127) / 128);
+  const uint32_t ostage = 128u * 32u * 4u * (1u + nb128);  // fp32: A box + r/128 B boxes
+  const int ostages = (int)std::min<uint32_t>(4u, budget / ostage);
+  if (stages < 2 || ostages < 2) return cudaErrorInvalidValue;
   tp->nb64 = nb64;
+  tp->nb128 = nb128;
   tp->f_stages = tp->r_stages = stages;
+  tp->o_stages = ostages;
   tp->f_smem = form_bq_smem(stages, stage);
   tp->r_smem = btp_smem(stages, stage);
+  tp->o_smem = orth_smem(ostages, ostage);
   uint32_t cols = 32;
   while (cols < (uint32_t)((lo.max_r + 15) / 16 * 16)) cols <<= 1;
   tp->tmem_cols = cols;
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(tc_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)U_SMEM);
   if (e == cudaSuccess) e = setup_bq_kernels(tp->f_smem, tp->r_smem);
+  if (e == cudaSuccess) e = setup_orth_kernels(tp->o_smem);
   int dev = 0, sms = 0;
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -408,15 +444,15 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, c
   tick(p, s, "tc_form_bq");
   launch_gate(sh, a, s);
   tick(p, s, "gate");
-  static const char *kGram[3] = {"gemm_gram0", "gemm_gram1", "gemm_gram2"};
+  static const char *kGram[3] = {"tc_gram0", "tc_gram1", "tc_gram2"};
   static const char *kChol[3] = {"chol_inv0", "chol_inv1", "chol_inv2"};
-  static const char *kTrsm[3] = {"gemm_trsm0", "gemm_trsm1", "gemm_trsm2"};
-  for (int pass = 0; pass < 3; ++pass) {
-    launch_gemm(sh, tp.probs[1 + pass], tp.gtiles[1 + pass], tp.n_gtiles[1 + pass], s);
+  static const char *kTrsm[3] = {"tc_trsm0", "tc_trsm1", "tc_trsm2"};
+  for (int pass = 0; pass < 3; ++pass) {  // CholeskyQR2; the third pass only after a shifted retry
+    launch_orth(sh, tp, true, pass, s);  // S = X^T X
     tick(p, s, kGram[pass]);
-    launch_chol_inv(sh, chol_smem, pass, s);
+    launch_chol_inv(sh, chol_smem, pass, s);  // L, L^{-1}
     tick(p, s, kChol[pass]);
-    launch_gemm(sh, tp.probs[4 + pass], tp.gtiles[4 + pass], tp.n_gtiles[4 + pass], s);
+    launch_orth(sh, tp, false, pass, s);  // X L^{-T} and its transpose
     tick(p, s, kTrsm[pass]);
   }
   if (tp.n_ptiles > 0) cvt_p_kernel<<<tp.n_ptiles, kCvtThreads, 0, s>>>(sh, tp.ptiles);

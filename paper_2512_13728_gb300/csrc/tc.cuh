@@ -22,15 +22,23 @@ struct LayerMaps {
   CUtensorMap Qn_mn;  // n x r bf16:  box {64, 64}   B Q: MN-major B operand (K = n)
   CUtensorMap P_mn;   // m x r bf16:  box {64, 64}   B^T P: MN-major B operand (K = m)
   CUtensorMap Bh_mn;  // m x n bf16:  box {64, 64}   B^T P: MN-major A operand (K = m)
-  CUtensorMap Praw;   // m x r fp32:  box {32, 128}  B Q: output store
+  CUtensorMap Praw;   // m x r fp32:  box {32, 128}  B Q output; TRSM A operand / output
   CUtensorMap Rst;    // n x r fp32:  box {32, 128}  B^T P: output store
+  CUtensorMap Pf;     // m x r fp32 (P):      box {32, 128}  TRSM A operand / output
+  CUtensorMap PTraw;  // r x m fp32 (P_raw^T): box {32, 128}  Gram operands
+  CUtensorMap PT;     // r x m fp32 (P^T):    box {32, 128}  Gram operands
+  CUtensorMap PTraw_t;  // r x m fp32: box {32, 32}  transposed output store
+  CUtensorMap PT_t;     // r x m fp32: box {32, 32}  transposed output store
+  CUtensorMap Sst;    // r x r fp32:  box {32, 128}  Gram output
+  CUtensorMap Linv;   // r x r fp32:  box {32, 128}  TRSM B operand (rows of L^{-1})
 };
 
 struct TcLayout {
   size_t end = 0;
   size_t o_maps = 0;
-  size_t o_utiles = 0, o_ptiles = 0, o_ftiles = 0, o_rtiles = 0, o_qtiles = 0;
-  std::vector<size_t> o_phi, o_rhi, o_qnhi, o_bh;
+  size_t o_utiles = 0, o_ptiles = 0, o_ftiles = 0, o_rtiles = 0, o_qtiles = 0, o_gtiles = 0, o_ttiles = 0;
+  std::vector<size_t> o_phi, o_rhi, o_qnhi, o_bh, o_ptraw, o_pt;
+  std::vector<int4> gram_tiles, trsm_tiles;
   // update tiles {layer, m-block, n-block, slot}; P-convert tiles {layer, row0, rows, 0};
   // B Q tiles {layer, m-block, 0, slot}; B^T P tiles {layer, n-block, 0, 0}; Q-copy tiles
   std::vector<int4> utiles, ptiles, ftiles, rtiles, qtiles;
@@ -50,9 +58,13 @@ struct TcPlan {
   int32_t n_rtiles = 0;
   int4 *qtiles = nullptr;
   int32_t n_qtiles = 0;
+  int4 *gram_tiles = nullptr;
+  int32_t n_gram_tiles = 0;
+  int4 *trsm_tiles = nullptr;
+  int32_t n_trsm_tiles = 0;
   int32_t max_r = 0;
-  int32_t f_stages = 0, r_stages = 0;
-  uint32_t f_smem = 0, r_smem = 0, nb64 = 0, tmem_cols = 0;
+  int32_t f_stages = 0, r_stages = 0, o_stages = 0;
+  uint32_t f_smem = 0, r_smem = 0, o_smem = 0, nb64 = 0, nb128 = 0, tmem_cols = 0;
   int32_t num_sms = 0;
   int32_t precision = 0;
   int32_t launches = 0;

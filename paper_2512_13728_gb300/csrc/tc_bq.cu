@@ -34,14 +34,15 @@ __device__ __forceinline__ uint32_t rpad16(int64_t r) { return (uint32_t)((r + 1
 // outside the matrix are clipped by the store).  Called by 128 threads (4 warps covering the
 // 4 TMEM lane groups); `leader` issues the stores.
 __device__ __forceinline__ void store_accumulator(uint32_t tmem, int warp, int lane, bool leader, uint8_t *stg,
-                                                  const CUtensorMap *map, int64_t r, int32_t row0,
-                                                  uint32_t &ecount, uint32_t bar_id) {
+                                                  const CUtensorMap *map, const CUtensorMap *map_t, int64_t r,
+                                                  int64_t rows, int32_t row0, uint32_t &ecount, uint32_t bar_id) {
+  // staging buffer eb: [row-major 128 x 32 box | 4 transposed 32 x 32 boxes (one per warp)]
   const uint32_t lg = (uint32_t)(warp & 3), row = 32u * lg + lane;
   const int nch = (int)((r + 31) / 32);
   for (int j = 0; j < nch; ++j) {
     const uint32_t eb = ecount & 1u;
-    uint8_t *box = stg + eb * EPI_BOX;
-    if (leader) bulk_wait_read<1>();  // the store issued two boxes ago has read this buffer
+    uint8_t *box = stg + eb * 2 * EPI_BOX, *tbox = box + EPI_BOX + lg * (EPI_BOX / 4);
+    if (leader) bulk_wait_read<1>();  // the stores issued two chunks ago have read this buffer
     named_sync(bar_id, 128);
     uint32_t v[32];
     tmem_ld32(tmem + (lg * 32u << 16) + j * 32, v);
@@ -52,10 +53,20 @@ __device__ __forceinline__ void store_accumulator(uint32_t tmem, int warp, int l
                              __uint_as_float(v[4 * q + 3]));
       *reinterpret_cast<float4 *>(box + sw128_f32(row, q)) = f;
     }
+    if (map_t != nullptr) {
+#pragma unroll
+      for (int c = 0; c < 32; ++c)
+        *reinterpret_cast<float *>(tbox + c * 128 + ((((uint32_t)lane >> 2) ^ (c & 7)) << 4) + (lane & 3) * 4) =
+            __uint_as_float(v[c]);
+    }
     fence_async_smem();
     named_sync(bar_id, 128);
     if (leader) {
       tma_store_2d(map, box, j * 32, row0);
+      if (map_t != nullptr)
+        for (int w4 = 0; w4 < 4; ++w4)
+          if ((int64_t)row0 + w4 * 32 < rows)
+            tma_store_2d(map_t, box + EPI_BOX + w4 * (EPI_BOX / 4), row0 + w4 * 32, j * 32);
       bulk_commit();
     }
     ++ecount;
@@ -139,8 +150,8 @@ __global__ void __launch_bounds__(F_THREADS, 1)
                       int nstages, uint32_t stage_bytes, uint32_t tmem_cols) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = align1024(smem_raw);
-  uint8_t *stg = smem + nstages * stage_bytes;  // 2 output boxes
-  uint64_t *bars = reinterpret_cast<uint64_t *>(stg + 2 * EPI_BOX);
+  uint8_t *stg = smem + nstages * stage_bytes;  // 2 staging buffers of 2 output boxes
+  uint64_t *bars = reinterpret_cast<uint64_t *>(stg + 4 * EPI_BOX);
   uint64_t *a_full = bars, *q_full = bars + nstages, *empty = bars + 2 * nstages;
   uint64_t *acc_full = bars + 3 * nstages, *acc_empty = acc_full + 1, *drain = acc_full + 2;
   __shared__ uint32_t tmem_base_s;
@@ -270,7 +281,8 @@ __global__ void __launch_bounds__(F_THREADS, 1)
       const DevLayer &L = sh.layers[t.x];
       if (!named_and(3, 128, ab.wait(acc_full, tcount & 1u, sh.status))) break;
       tc_fence_after();
-      store_accumulator(tmem, warp, lane, leader, stg, &maps[t.x].Praw, L.r, t.y * 128, ecount, 3);
+      store_accumulator(tmem, warp, lane, leader, stg, &maps[t.x].Praw, &maps[t.x].PTraw_t, L.r, L.m, t.y * 128,
+                        ecount, 3);
       tc_fence_before();
       mbar_arrive(acc_empty);
     }
@@ -291,7 +303,7 @@ __global__ void __launch_bounds__(R_THREADS, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = align1024(smem_raw);
   uint8_t *stg = smem + nstages * stage_bytes;
-  uint64_t *bars = reinterpret_cast<uint64_t *>(stg + 2 * EPI_BOX);
+  uint64_t *bars = reinterpret_cast<uint64_t *>(stg + 4 * EPI_BOX);
   uint64_t *full = bars, *empty = bars + nstages;
   uint64_t *acc_full = bars + 2 * nstages, *acc_empty = acc_full + 1, *drain = acc_full + 2;
   __shared__ uint32_t tmem_base_s;
@@ -386,7 +398,7 @@ __global__ void __launch_bounds__(R_THREADS, 1)
       const DevLayer &L = sh.layers[t.x];
       if (!named_and(1, 128, ab.wait(acc_full, tcount & 1u, sh.status))) break;
       tc_fence_after();
-      store_accumulator(tmem, warp, lane, leader, stg, &maps[t.x].Rst, L.r, t.y * 128, ecount, 1);
+      store_accumulator(tmem, warp, lane, leader, stg, &maps[t.x].Rst, nullptr, L.r, L.n, t.y * 128, ecount, 1);
       tc_fence_before();
       mbar_arrive(acc_empty);
       ++tcount;
@@ -412,7 +424,7 @@ __global__ void __launch_bounds__(256) qn_refresh_kernel(Shared sh, const int4 *
 
 // ======================================================================= launchers ===
 uint32_t form_bq_smem(int nstages, uint32_t stage_bytes) {
-  return 1024u + nstages * stage_bytes + 2 * EPI_BOX + 512u;  // + barriers
+  return 1024u + nstages * stage_bytes + 4 * EPI_BOX + 512u;  // + barriers
 }
 uint32_t btp_smem(int nstages, uint32_t stage_bytes) { return form_bq_smem(nstages, stage_bytes); }
 

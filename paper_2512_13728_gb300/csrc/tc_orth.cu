@@ -1,0 +1,261 @@
+// Orthogonalize on tensor cores for DION_PREC_BF16: the Gram matrix and the triangular
+// solve of each CholeskyQR pass as kind::tf32 tcgen05 GEMMs on fp32 operands loaded by TMA.
+//
+//   Gram   S = X^T X (r x r, lower triangle).  Tile = 128 rows of S; K loop over m.  Both
+//          operands are K-major rows of the transposed copy X^T (r x m), which the producing
+//          kernel (the B Q epilogue or the previous TRSM) writes next to X.
+//   TRSM   Y = X L^{-T} (m x r).  Tile = 128 rows of X; K loop over r.  A = rows of X
+//          (K-major), B = rows of L^{-1} (K-major, lower triangular: K chunks above a column
+//          part are skipped).  Epilogue stores Y (row-major) and Y^T (transposed boxes).
+//
+// Accuracy: tf32 products (10-bit mantissa) with fp32 accumulation give ~5e-4 relative
+// error in S and Y; the second CholeskyQR pass (on an already nearly orthonormal X) brings
+// P back to orthonormal to that level, below the bf16 rounding the following kernels apply.
+// Roles: warp 0 TMA, warp 1 MMA (+ TMEM), warps 2..5 epilogue.
+#include "tc.cuh"
+#include "tc_common.cuh"
+#include "tc_kernels.cuh"
+
+namespace cd {
+namespace tc {
+
+constexpr uint32_t O_BOX = 128u * 32u * 4u;  // one fp32 box: 128 rows x 32 (K) = 16 KB
+constexpr uint32_t O_TBOX = 32u * 32u * 4u;  // one transposed output box: 32 x 32 fp32 = 4 KB
+constexpr int O_THREADS = 6 * 32;
+
+enum : int32_t { ORTH_GRAM = 0, ORTH_TRSM = 1 };
+
+__device__ __forceinline__ uint32_t pad16(int64_t v) { return (uint32_t)((v + 15) / 16 * 16); }
+
+struct OrthMaps {
+  const CUtensorMap *A, *B, *out, *out_t;  // out_t null for the Gram
+};
+
+template <int KIND>
+__device__ __forceinline__ OrthMaps orth_maps(const LayerMaps &mp, int pass) {
+  // X_0 = P_raw, X_1 = P, X_2 = P_raw, X_3 = P (ping-pong between the two buffers)
+  const bool raw_in = (pass != 1);
+  OrthMaps o;
+  if (KIND == ORTH_GRAM) {
+    o.A = raw_in ? &mp.PTraw : &mp.PT;
+    o.B = o.A;
+    o.out = &mp.Sst;
+    o.out_t = nullptr;
+  } else {
+    o.A = raw_in ? &mp.Praw : &mp.Pf;
+    o.B = &mp.Linv;
+    o.out = raw_in ? &mp.Pf : &mp.Praw;
+    o.out_t = raw_in ? &mp.PT_t : &mp.PTraw_t;
+  }
+  return o;
+}
+
+// Per tile: M-dim rows [row0, row0 + 128), N columns, K extent, and whether K chunk kc
+// feeds N part p (TRSM: L^{-1} is lower triangular, so column part p needs k < 256 (p + 1)).
+template <int KIND>
+__device__ __forceinline__ void orth_dims(const DevLayer &L, int blk, uint32_t &N, int64_t &K) {
+  if (KIND == ORTH_GRAM) {
+    N = min(pad16(L.r), (uint32_t)(blk + 1) * 128u);  // lower triangle of S only
+    K = L.m;
+  } else {
+    N = pad16(L.r);
+    K = L.r;
+  }
+}
+
+template <int KIND>
+__device__ __forceinline__ bool part_needs(int kc, uint32_t part) {
+  return KIND == ORTH_GRAM || (uint32_t)kc * 32u < 256u * (part + 1u);
+}
+
+template <int KIND>
+__global__ void __launch_bounds__(O_THREADS, 1)
+    tc_orth_kernel(Shared sh, const int4 *__restrict__ tiles, int ntiles, const LayerMaps *__restrict__ maps,
+                   int pass, int nstages, uint32_t stage_bytes, uint32_t tmem_cols) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = align1024(smem_raw);
+  uint8_t *stg = smem + nstages * stage_bytes;  // 2 x (row box 16 KB + 4 transposed boxes 16 KB)
+  uint64_t *bars = reinterpret_cast<uint64_t *>(stg + 4 * O_BOX);
+  uint64_t *full = bars, *empty = bars + nstages;
+  uint64_t *acc_full = bars + 2 * nstages, *acc_empty = acc_full + 1, *drain = acc_full + 2;
+  __shared__ uint32_t tmem_base_s;
+  __shared__ int abort_s;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const Abort ab{&abort_s};
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < nstages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    mbar_init(acc_full, 1);
+    mbar_init(acc_empty, 128);
+    mbar_init(drain, 1);
+    abort_s = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&tmem_base_s, tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_s;
+  auto skip = [&](int layer) { return !sh.active[layer] || (pass == 2 && !sh.orth_shifted[layer]); };
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+        const int4 t = tiles[ti];
+        if (skip(t.x)) continue;
+        const DevLayer &L = sh.layers[t.x];
+        const OrthMaps om = orth_maps<KIND>(maps[t.x], pass);
+        uint32_t N;
+        int64_t K;
+        orth_dims<KIND>(L, t.y, N, K);
+        const int kch = (int)((K + 31) / 32);
+        const uint32_t nboxes = (N + 127) / 128;
+        for (int kc = 0; kc < kch; ++kc, ++it) {
+          const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
+          if (!ab.wait(&empty[s], ph ^ 1u, sh.status)) { ok = false; break; }
+          uint8_t *sA = smem + s * stage_bytes, *sB = sA + O_BOX;
+          uint32_t nb = 0;  // B boxes this chunk feeds (all, or only the lower-triangular parts)
+          for (uint32_t b = 0; b < nboxes; ++b)
+            if (part_needs<KIND>(kc, b / 2)) ++nb;
+          mbar_expect_tx(&full[s], O_BOX * (1 + nb));
+          tma_load_2d(sA, om.A, &full[s], kc * 32, t.y * 128);
+          for (uint32_t b = 0; b < nboxes; ++b)
+            if (part_needs<KIND>(kc, b / 2)) tma_load_2d(sB + b * O_BOX, om.B, &full[s], kc * 32, b * 128);
+        }
+      }
+      for (uint32_t k = (it > (uint32_t)nstages ? it - nstages : 0); k < it; ++k)
+        mbar_wait(&full[k % nstages], (k / nstages) & 1u, sh.status);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      uint32_t it = 0, tcount = 0;
+      bool ok = true;
+      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+        const int4 t = tiles[ti];
+        if (skip(t.x)) continue;
+        const DevLayer &L = sh.layers[t.x];
+        uint32_t N;
+        int64_t K;
+        orth_dims<KIND>(L, t.y, N, K);
+        const int kch = (int)((K + 31) / 32);
+        const uint32_t nparts = (N + 255) / 256;
+        if (!ab.wait(acc_empty, (tcount & 1u) ^ 1u, sh.status)) break;
+        tc_fence_after();
+        for (int kc = 0; kc < kch; ++kc, ++it) {
+          const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
+          if (!ab.wait(&full[s], ph, sh.status)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t aB = smem_u32(smem + s * stage_bytes), bB = aB + O_BOX;
+#pragma unroll
+          for (int k8 = 0; k8 < 4; ++k8) {
+            const uint64_t ad = smem_desc_sw128(aB + k8 * 32, 0, 1024);
+            for (uint32_t part = 0; part < nparts; ++part) {
+              if (!part_needs<KIND>(kc, part)) continue;
+              const uint32_t n_here = min(256u, N - part * 256u);
+              const uint64_t bd = smem_desc_sw128(bB + part * 2u * O_BOX + k8 * 32, 0, 1024);
+              // the first chunk that feeds a part starts its accumulation
+              umma_tf32(tmem + part * 256u, ad, bd, idesc_tf32(128, n_here, false, false), (kc | k8) ? 1u : 0u);
+            }
+          }
+          umma_commit(&empty[s]);
+        }
+        if (!ok) break;
+        umma_commit(acc_full);
+        ++tcount;
+      }
+      umma_commit(drain);
+      mbar_wait(drain, 0, sh.status);
+    }
+  } else {
+    // epilogue: 128 threads, thread = output row (TMEM lane)
+    const bool leader = (warp == 2 && lane == 0);
+    const uint32_t lg = (uint32_t)(warp & 3), row = 32u * lg + lane;
+    uint32_t tcount = 0, ecount = 0;
+    for (int ti = blockIdx.x; ti < ntiles; ti += gridDim.x) {
+      const int4 t = tiles[ti];
+      if (skip(t.x)) continue;
+      const DevLayer &L = sh.layers[t.x];
+      const OrthMaps om = orth_maps<KIND>(maps[t.x], pass);
+      uint32_t N;
+      int64_t K;
+      orth_dims<KIND>(L, t.y, N, K);
+      if (!named_and(1, 128, ab.wait(acc_full, tcount & 1u, sh.status))) break;
+      tc_fence_after();
+      const int nch = (int)((min((int64_t)N, L.r) + 31) / 32);
+      for (int j = 0; j < nch; ++j) {
+        const uint32_t eb = ecount & 1u;
+        uint8_t *box = stg + eb * 2 * O_BOX, *tbox = box + O_BOX + lg * O_TBOX;
+        if (leader) bulk_wait_read<1>();
+        named_sync(1, 128);
+        uint32_t v[32];
+        tmem_ld32(tmem + (lg * 32u << 16) + j * 32, v);
+        tmem_ld_wait();
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          *reinterpret_cast<float4 *>(box + sw128_f32(row, q)) =
+              make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]), __uint_as_float(v[4 * q + 2]),
+                          __uint_as_float(v[4 * q + 3]));
+        if (KIND == ORTH_TRSM) {
+          // transposed 32 x 32 box of this warp's rows: box row c = output column j*32 + c
+#pragma unroll
+          for (int c = 0; c < 32; ++c)
+            *reinterpret_cast<float *>(tbox + c * 128 + ((((uint32_t)lane >> 2) ^ (c & 7)) << 4) + (lane & 3) * 4) =
+                __uint_as_float(v[c]);
+        }
+        fence_async_smem();
+        named_sync(1, 128);
+        if (leader) {
+          tma_store_2d(om.out, box, j * 32, t.y * 128);
+          if (KIND == ORTH_TRSM)
+            for (int w4 = 0; w4 < 4; ++w4)
+              if ((int64_t)t.y * 128 + w4 * 32 < L.m)
+                tma_store_2d(om.out_t, stg + eb * 2 * O_BOX + O_BOX + w4 * O_TBOX, t.y * 128 + w4 * 32, j * 32);
+          bulk_commit();
+        }
+        ++ecount;
+      }
+      tc_fence_before();
+      mbar_arrive(acc_empty);
+      ++tcount;
+    }
+    if (leader) bulk_wait<0>();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, tmem_cols);
+}
+
+uint32_t orth_smem(int nstages, uint32_t stage_bytes) { return 1024u + nstages * stage_bytes + 4u * O_BOX + 512u; }
+
+cudaError_t setup_orth_kernels(uint32_t smem) {
+  cudaError_t e =
+      cudaFuncSetAttribute(tc_orth_kernel<ORTH_GRAM>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(tc_orth_kernel<ORTH_TRSM>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  return e;
+}
+
+void launch_orth(const Shared &sh, const TcPlan &tp, bool gram, int pass, cudaStream_t s) {
+  const int4 *tiles = gram ? tp.gram_tiles : tp.trsm_tiles;
+  const int n = gram ? tp.n_gram_tiles : tp.n_trsm_tiles;
+  if (n <= 0) return;
+  const int grid = std::min(n, std::max(tp.num_sms, 1));
+  const uint32_t stage = O_BOX * (1 + tp.nb128);
+  if (gram)
+    tc_orth_kernel<ORTH_GRAM><<<grid, O_THREADS, tp.o_smem, s>>>(sh, tiles, n, tp.maps, pass, tp.o_stages, stage,
+                                                                   tp.tmem_cols);
+  else
+    tc_orth_kernel<ORTH_TRSM><<<grid, O_THREADS, tp.o_smem, s>>>(sh, tiles, n, tp.maps, pass, tp.o_stages, stage,
+                                                                   tp.tmem_cols);
+}
+
+}  // namespace tc
+}  // namespace cd
