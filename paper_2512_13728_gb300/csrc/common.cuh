@@ -45,8 +45,8 @@ struct DevLayer {
   float *P_raw;  // m x r (ld ldp)  P = B Q before orthogonalization
   float *P;      // m x r (ld ldp)  orthonormal P
   float *R;      // n x r (ld ldp)  R = B^T P
-  float *S;      // r x r   Gram P_raw^T P_raw; lower triangle becomes the Cholesky factor L
-  float *Linv;   // r x r   L^{-1} (lower triangular, zeros above the diagonal)
+  float *S;      // r x r (ld ldp)  Gram X^T X; lower triangle becomes the Cholesky factor L
+  float *Linv;   // r x r (ld ldp)  L^{-1} (lower triangular, zeros above the diagonal)
   // tensor-core operand copies (bf16, rows of pitch ldp unless stated); null in FP32 mode
   __nv_bfloat16 *P_hi;   // m x r : P
   __nv_bfloat16 *R_hi;   // n x r : R

@@ -255,7 +255,7 @@ __device__ __forceinline__ int64_t tri_row(int64_t p) {
 
 // Factors the lower triangle of S (r x r, row-major) in place.  Returns false (uniformly over
 // the block) on a pivot <= 0 or non-finite.  Smem: D (CB x CBP), Pn (r x CBP).
-__device__ bool cholesky_blocked(float *S, int r, float *D, float *Pn, int *bad) {
+__device__ bool cholesky_blocked(float *S, int r, int64_t ls, float *D, float *Pn, int *bad) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (tid == 0) *bad = 0;
   __syncthreads();
@@ -264,7 +264,7 @@ __device__ bool cholesky_blocked(float *S, int r, float *D, float *Pn, int *bad)
     for (int e = tid; e < CB * CB; e += kCholThreads) {
       const int i = e / CB, j = e % CB;
       float v;
-      if (i < nb && j < nb) v = (j <= i) ? S[(int64_t)(k0 + i) * r + k0 + j] : 0.f;
+      if (i < nb && j < nb) v = (j <= i) ? S[(int64_t)(k0 + i) * ls + k0 + j] : 0.f;
       else v = (i == j) ? 1.f : 0.f;  // identity padding of a short last block
       D[i * CBP + j] = v;
     }
@@ -292,12 +292,12 @@ __device__ bool cholesky_blocked(float *S, int r, float *D, float *Pn, int *bad)
     if (*bad) return false;
     for (int e = tid; e < nb * nb; e += kCholThreads) {
       const int i = e / nb, j = e % nb;
-      if (j <= i) S[(int64_t)(k0 + i) * r + k0 + j] = D[i * CBP + j];
+      if (j <= i) S[(int64_t)(k0 + i) * ls + k0 + j] = D[i * CBP + j];
     }
     // panel: rows below the block solve x L11^T = s
     const int t = r - k0 - nb;
     for (int ii = tid; ii < t; ii += kCholThreads) {
-      const int64_t row = (int64_t)(k0 + nb + ii) * r + k0;
+      const int64_t row = (int64_t)(k0 + nb + ii) * ls + k0;
       float x[CB];
 #pragma unroll
       for (int j = 0; j < CB; ++j) x[j] = (j < nb) ? S[row + j] : 0.f;
@@ -341,7 +341,7 @@ __device__ bool cholesky_blocked(float *S, int r, float *D, float *Pn, int *bad)
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
           const int64_t rj = bj * 4 + v;
-          if (rj < t && rj <= ri) S[(k0 + nb + ri) * r + k0 + nb + rj] -= acc[u][v];
+          if (rj < t && rj <= ri) S[(k0 + nb + ri) * ls + k0 + nb + rj] -= acc[u][v];
         }
       }
     }
@@ -357,6 +357,7 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int p
   if (pass == 2 && !sh.orth_shifted[l]) return;
   const DevLayer &Ly = sh.layers[l];
   const int r = (int)Ly.r;
+  const int64_t ls = Ly.ldp;  // leading dimension of S and L^{-1}
   float *S = Ly.S;
   float *Li = Ly.Linv;
   extern __shared__ float smem[];
@@ -371,12 +372,12 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int p
   // the factorization never touches and the shifted retry restores the lower triangle from.
   for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) {
     const int64_t i = e / r, j = e % r;
-    if (j > i) S[e] = S[j * r + i];
+    if (j > i) S[i * ls + j] = S[j * ls + i];
   }
-  for (int i = tid; i < r; i += kCholThreads) diag0[i] = S[(int64_t)i * r + i];
+  for (int i = tid; i < r; i += kCholThreads) diag0[i] = S[(int64_t)i * ls + i];
   __syncthreads();
 
-  bool ok = cholesky_blocked(S, r, D, Pn, &bad);
+  bool ok = cholesky_blocked(S, r, ls, D, Pn, &bad);
   bool shifted = false;
   if (!ok) {  // shifted retry: lower triangle from the untouched upper triangle, shifted diagonal
     if (tid == 0) {
@@ -389,12 +390,12 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int p
     const double shift = 11.0 * ((double)Ly.m * r + (double)r * (r + 1)) * u * trace_s;
     for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) {
       const int64_t i = e / r, j = e % r;
-      if (j < i) S[e] = S[j * r + i];
-      else if (j == i) S[e] = (float)((double)diag0[i] + shift);
+      if (j < i) S[i * ls + j] = S[j * ls + i];
+      else if (j == i) S[i * ls + j] = (float)((double)diag0[i] + shift);
     }
     __syncthreads();
     shifted = true;
-    ok = (trace_s > 0.0) && isfinite(trace_s) && cholesky_blocked(S, r, D, Pn, &bad);
+    ok = (trace_s > 0.0) && isfinite(trace_s) && cholesky_blocked(S, r, ls, D, Pn, &bad);
   }
   if (tid == 0) {
     if (pass == 0) sh.orth_shifted[l] = shifted ? 1 : 0;
@@ -402,7 +403,7 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int p
   }
   if (!ok) {
     if (tid == 0) set_status(sh.status, ST_BREAKDOWN);
-    for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) Li[e] = 0.f;
+    for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) Li[(e / r) * ls + e % r] = 0.f;
     return;
   }
 
@@ -413,7 +414,7 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int p
     for (int e = tid; e < CB * CB; e += kCholThreads) {
       const int i = e / CB, j = e % CB;
       float v;
-      if (i < nb && j < nb) v = (j <= i) ? S[(int64_t)(I0 + i) * r + I0 + j] : 0.f;
+      if (i < nb && j < nb) v = (j <= i) ? S[(int64_t)(I0 + i) * ls + I0 + j] : 0.f;
       else v = (i == j) ? 1.f : 0.f;
       D[i * CBP + j] = v;
     }
@@ -433,7 +434,7 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int p
     // Row block I of L staged in shared memory: Lb[i][k] = L[I0+i][k], k < I0.
     for (int e = tid; e < CB * I0; e += kCholThreads) {
       const int i = e / I0, k = e % I0;
-      Pn[i * I0 + k] = (i < nb) ? S[(int64_t)(I0 + i) * r + k] : 0.f;
+      Pn[i * I0 + k] = (i < nb) ? S[(int64_t)(I0 + i) * ls + k] : 0.f;
     }
     __syncthreads();
     // Thread c < I0 owns column c: T[i] = sum_{k=c}^{I0-1} Lb[i][k] Linv[k][c] for the 32 rows
@@ -449,14 +450,14 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int p
       for (; k + 8 <= I0; k += 8) {
         float lk[8];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) lk[u] = Li[(int64_t)(k + u) * r + c];
+        for (int u = 0; u < 8; ++u) lk[u] = Li[(int64_t)(k + u) * ls + c];
 #pragma unroll
         for (int u = 0; u < 8; ++u)
 #pragma unroll
           for (int i = 0; i < CB; ++i) acc[i] = fmaf(Pn[i * I0 + k + u], lk[u], acc[i]);
       }
       for (; k < I0; ++k) {
-        const float lk = Li[(int64_t)k * r + c];
+        const float lk = Li[(int64_t)k * ls + c];
 #pragma unroll
         for (int i = 0; i < CB; ++i) acc[i] = fmaf(Pn[i * I0 + k], lk, acc[i]);
       }
@@ -469,7 +470,7 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int p
       }
 #pragma unroll
       for (int i = 0; i < CB; ++i)
-        if (i < nb) Li[(int64_t)(I0 + i) * r + c] = acc[i];
+        if (i < nb) Li[(int64_t)(I0 + i) * ls + c] = acc[i];
     }
     // diagonal block DI and zeros to its right
     for (int e = tid; e < nb * (r - I0); e += kCholThreads) {
@@ -479,7 +480,7 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int p
         const int j = c - I0;
         v = (j <= i) ? DI[i * CBP + j] : 0.f;
       }
-      Li[(int64_t)(I0 + i) * r + c] = v;
+      Li[(int64_t)(I0 + i) * ls + c] = v;
     }
     __syncthreads();
   }

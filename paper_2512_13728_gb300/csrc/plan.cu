@@ -169,8 +169,8 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
     o_Praw[l] = cv.take<float>(ly.m * d.ldp);
     o_P[l] = cv.take<float>(ly.m * d.ldp);
     o_R[l] = cv.take<float>(ly.n * d.ldp);
-    o_S[l] = cv.take<float>(ly.r * ly.r);
-    o_Li[l] = cv.take<float>(ly.r * ly.r);
+    o_S[l] = cv.take<float>(ly.r * d.ldp);
+    o_Li[l] = cv.take<float>(ly.r * d.ldp);
     // row tiles of about 64K elements for the buffer and local kernels
     const int64_t rows = std::max<int64_t>(1, std::min<int64_t>(ly.m, 65536 / ly.n));
     d.bpart_off = (int32_t)bt.size();
@@ -225,10 +225,10 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
       if (k == 0) {
         q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.n; q.lda = ly.ldm; q.ldb = ly.ldq; q.ldc = ldp;
       } else if (k <= 3) {
-        q.Mrows = ly.r; q.Ncols = ly.r; q.K = ly.m; q.lda = ldp; q.ldb = ldp; q.ldc = ly.r; q.transA = 1;
+        q.Mrows = ly.r; q.Ncols = ly.r; q.K = ly.m; q.lda = ldp; q.ldb = ldp; q.ldc = ldp; q.transA = 1;
         q.mode = (k == 3) ? GEMM_SHIFTED : GEMM_ACTIVE;
       } else if (k <= 6) {
-        q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.r; q.lda = ldp; q.ldb = ly.r; q.ldc = ldp; q.transB = 1;
+        q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.r; q.lda = ldp; q.ldb = ldp; q.ldc = ldp; q.transB = 1;
         q.mode = (k == 6) ? GEMM_SHIFTED_OR_COPY : GEMM_ACTIVE;
       } else {
         q.Mrows = ly.n; q.Ncols = ly.r; q.K = ly.m; q.lda = ly.ldm; q.ldb = ldp; q.ldc = ldp; q.transA = 1;

@@ -388,8 +388,8 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
                     encode_f32_2d(&m.PT, d.PT, d.m, d.r, (uint64_t)d.ldmt * 4, 32, 128) &&
                     encode_f32_2d(&m.PTraw_t, d.PT_raw, d.m, d.r, (uint64_t)d.ldmt * 4, 32, 32) &&
                     encode_f32_2d(&m.PT_t, d.PT, d.m, d.r, (uint64_t)d.ldmt * 4, 32, 32) &&
-                    encode_f32_2d(&m.Sst, d.S, d.r, d.r, (uint64_t)d.r * 4, 32, 128) &&
-                    encode_f32_2d(&m.Linv, d.Linv, d.r, d.r, (uint64_t)d.r * 4, 32, 128);
+                    encode_f32_2d(&m.Sst, d.S, d.r, d.r, p32, 32, 128) &&
+                    encode_f32_2d(&m.Linv, d.Linv, d.r, d.r, p32, 32, 128);
     if (!ok) return cudaErrorInvalidValue;
   }
   auto up = [&](int4 *dst, const std::vector<int4> &v) {
