@@ -54,7 +54,7 @@ constexpr int U_THREADS = 192;
 constexpr uint32_t U_IDESC = idesc_bf16(128, 128, false, false);
 
 __global__ void __launch_bounds__(U_THREADS, 1)
-    tc_update_kernel(Shared sh, const int4 *__restrict__ tiles, int ntiles, const LayerMaps *__restrict__ maps,
+    tc_update_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off, const LayerMaps *__restrict__ maps,
                      float mu, float eta) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = align1024(smem_raw);
@@ -98,7 +98,7 @@ __global__ void __launch_bounds__(U_THREADS, 1)
     if (lane == 0) {
       uint32_t it = 0;
       bool ok = true;
-      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+      for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
         if (!sh.active[t.x]) continue;
         const LayerMaps *mp = maps + t.x;
@@ -122,7 +122,7 @@ __global__ void __launch_bounds__(U_THREADS, 1)
     if (lane == 0) {
       uint32_t it = 0, tcount = 0;
       bool ok = true;
-      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+      for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
         if (!sh.active[t.x]) continue;
         const int kch = (int)((sh.layers[t.x].r + 63) / 64);
@@ -160,7 +160,7 @@ __global__ void __launch_bounds__(U_THREADS, 1)
     const bool leader = (et == 0);
     uint32_t tcount = 0, ecount = 0, issued = 0;
     bool ok = true;
-    for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+    for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
       const int4 t = tiles[ti];
       if (!sh.active[t.x]) continue;
       const DevLayer &L = sh.layers[t.x];
@@ -246,6 +246,35 @@ __global__ void __launch_bounds__(U_THREADS, 1)
 // ========================================================================= host side ===
 namespace {
 size_t bq_tiles(int64_t m) { return (size_t)((m + 127) / 128); }
+
+// Longest-processing-time-first assignment of tiles to at most `max_grid` persistent CTAs.
+Schedule lpt(const std::vector<int4> &tiles, const std::vector<double> &cost, int max_grid) {
+  Schedule sc;
+  const int n = (int)tiles.size();
+  sc.grid = std::max(0, std::min(n, max_grid));
+  if (n == 0) {
+    sc.off.assign(1, 0);
+    return sc;
+  }
+  std::vector<int> order(n);
+  for (int i = 0; i < n; ++i) order[i] = i;
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return cost[a] > cost[b]; });
+  std::vector<double> load(sc.grid, 0.0);
+  std::vector<std::vector<int>> per(sc.grid);
+  for (int i : order) {
+    int best = 0;
+    for (int c = 1; c < sc.grid; ++c)
+      if (load[c] < load[best]) best = c;
+    load[best] += cost[i];
+    per[best].push_back(i);
+  }
+  sc.off.push_back(0);
+  for (int c = 0; c < sc.grid; ++c) {
+    for (int i : per[c]) sc.tiles.push_back(tiles[i]);
+    sc.off.push_back((int)sc.tiles.size());
+  }
+  return sc;
+}
 }  // namespace
 
 size_t norm_slots(const dion_layer *layers, int32_t L) {
@@ -298,13 +327,23 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
     for (int64_t mb = 0; mb < (ly.m + 127) / 128; ++mb) lo.ftiles.push_back(make_int4(l, (int)mb, 0, fslot++));
     for (int64_t nb = 0; nb < (ly.n + 127) / 128; ++nb) lo.rtiles.push_back(make_int4(l, (int)nb, 0, 0));
   }
-  // longest K loops first (static round-robin over the SMs then balances well)
-  std::stable_sort(lo.ftiles.begin(), lo.ftiles.end(),
-                   [&](const int4 &a, const int4 &b) { return layers[a.x].n > layers[b.x].n; });
-  std::stable_sort(lo.rtiles.begin(), lo.rtiles.end(),
-                   [&](const int4 &a, const int4 &b) { return layers[a.x].m > layers[b.x].m; });
-  std::stable_sort(lo.gram_tiles.begin(), lo.gram_tiles.end(),
-                   [&](const int4 &a, const int4 &b) { return layers[a.x].m > layers[b.x].m; });
+  // per-tile cost ~ K-loop length (+ a constant for the epilogue), LPT over the SMs
+  auto sched = [&](const std::vector<int4> &tl, auto costf) {
+    std::vector<double> c(tl.size());
+    for (size_t i = 0; i < tl.size(); ++i) c[i] = costf(tl[i]);
+    return lpt(tl, c, std::max(num_sms, 1));
+  };
+  lo.s_update = sched(lo.utiles, [&](const int4 &t) { return (double)layers[t.x].r + 64.0; });
+  lo.s_bq = sched(lo.ftiles, [&](const int4 &t) { return (double)layers[t.x].n + 2.0 * layers[t.x].r; });
+  lo.s_btp = sched(lo.rtiles, [&](const int4 &t) { return (double)layers[t.x].m + 2.0 * layers[t.x].r; });
+  lo.s_gram = sched(lo.gram_tiles, [&](const int4 &t) {
+    return (double)layers[t.x].m * std::min<double>(layers[t.x].r, 128.0 * (t.y + 1)) / 128.0;
+  });
+  lo.s_trsm = sched(lo.trsm_tiles, [&](const int4 &t) { return 3.0 * layers[t.x].r + 64.0; });
+  for (Schedule *sc : {&lo.s_update, &lo.s_bq, &lo.s_btp, &lo.s_gram, &lo.s_trsm}) {
+    sc->o_tiles = take(sizeof(int4) * std::max<size_t>(sc->tiles.size(), 1));
+    sc->o_off = take(sizeof(int) * sc->off.size());
+  }
   lo.o_maps = take(sizeof(LayerMaps) * std::max(L, 1), 128);
   lo.o_utiles = take(sizeof(int4) * std::max<size_t>(lo.utiles.size(), 1));
   lo.o_ptiles = take(sizeof(int4) * std::max<size_t>(lo.ptiles.size(), 1));
@@ -363,10 +402,19 @@ void bind(const TcLayout &lo, char *base, DevLayer *dl, int32_t L, TcPlan *tp) {
   tp->n_trsm_tiles = (int32_t)lo.trsm_tiles.size();
   tp->precision = lo.precision;
   tp->max_r = lo.max_r;
+  auto bind_sched = [&](const Schedule &sc, DevSchedule &d) {
+    d.tiles = reinterpret_cast<const int4 *>(base + sc.o_tiles);
+    d.off = reinterpret_cast<const int *>(base + sc.o_off);
+    d.grid = sc.grid;
+  };
+  bind_sched(lo.s_update, tp->d_update);
+  bind_sched(lo.s_bq, tp->d_bq);
+  bind_sched(lo.s_btp, tp->d_btp);
+  bind_sched(lo.s_gram, tp->d_gram);
+  bind_sched(lo.s_trsm, tp->d_trsm);
 }
 
 cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, TcPlan *tp) {
-  (void)base;
   std::vector<LayerMaps> maps(std::max(L, 1));
   std::memset(maps.data(), 0, sizeof(LayerMaps) * maps.size());
   for (int32_t l = 0; l < L; ++l) {
@@ -403,6 +451,12 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   if (e == cudaSuccess) e = up(tp->qtiles, lo.qtiles);
   if (e == cudaSuccess) e = up(tp->gram_tiles, lo.gram_tiles);
   if (e == cudaSuccess) e = up(tp->trsm_tiles, lo.trsm_tiles);
+  for (const Schedule *sc : {&lo.s_update, &lo.s_bq, &lo.s_btp, &lo.s_gram, &lo.s_trsm}) {
+    if (e == cudaSuccess && !sc->tiles.empty())
+      e = cudaMemcpy(base + sc->o_tiles, sc->tiles.data(), sizeof(int4) * sc->tiles.size(), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess)
+      e = cudaMemcpy(base + sc->o_off, sc->off.data(), sizeof(int) * sc->off.size(), cudaMemcpyHostToDevice);
+  }
   // shared-memory budget: operand stages + 2 staging buffers of (128 x 32 + 4 x 32 x 32) fp32
   const uint32_t budget = 227u * 1024u - 1024u - 4u * 128u * 32u * 4u - 512u - 256u;
   const uint32_t nb64 = (uint32_t)std::max(1, (lo.max_r + 63) / 64);
@@ -461,10 +515,9 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, c
   tick(p, s, "tc_btp");
   launch_colnorm(sh, ctiles, n_ctiles, a.eps_col, s);  // Q_t, and bf16 R, Q_t
   tick(p, s, "colnorm");
-  if (tp.n_utiles > 0) {
-    const int grid = std::min(tp.n_utiles, std::max(tp.num_sms, 1));
-    tc_update_kernel<<<grid, U_THREADS, U_SMEM, s>>>(sh, tp.utiles, tp.n_utiles, tp.maps, a.mu, a.eta);
-  }
+  if (tp.d_update.grid > 0)
+    tc_update_kernel<<<tp.d_update.grid, U_THREADS, U_SMEM, s>>>(sh, tp.d_update.tiles, tp.d_update.off, tp.maps,
+                                                                  a.mu, a.eta);
   tick(p, s, "tc_update");
   launch_local(sh, btiles, n_btiles, a.eta_local, s);
   tick(p, s, "local");

@@ -33,7 +33,16 @@ struct LayerMaps {
   CUtensorMap Linv;   // r x r fp32:  box {32, 128}  TRSM B operand (rows of L^{-1})
 };
 
+// Tiles of one persistent kernel, reordered so that CTA b processes tiles [off[b], off[b+1]).
+struct Schedule {
+  std::vector<int4> tiles;
+  std::vector<int> off;
+  int grid = 0;
+  size_t o_tiles = 0, o_off = 0;  // workspace offsets
+};
+
 struct TcLayout {
+  Schedule s_update, s_bq, s_btp, s_gram, s_trsm;
   size_t end = 0;
   size_t o_maps = 0;
   size_t o_utiles = 0, o_ptiles = 0, o_ftiles = 0, o_rtiles = 0, o_qtiles = 0, o_gtiles = 0, o_ttiles = 0;
@@ -46,7 +55,14 @@ struct TcLayout {
   int32_t max_r = 0;
 };
 
+struct DevSchedule {
+  const int4 *tiles = nullptr;
+  const int *off = nullptr;
+  int grid = 0;
+};
+
 struct TcPlan {
+  DevSchedule d_update, d_bq, d_btp, d_gram, d_trsm;
   LayerMaps *maps = nullptr;
   int4 *utiles = nullptr;
   int32_t n_utiles = 0;

@@ -19,6 +19,8 @@
 #include "tc_common.cuh"
 #include "tc_kernels.cuh"
 
+#include <type_traits>
+
 namespace cd {
 namespace tc {
 
@@ -35,14 +37,20 @@ __device__ __forceinline__ uint32_t rpad16(int64_t r) { return (uint32_t)((r + 1
 // 4 TMEM lane groups); `leader` issues the stores.
 __device__ __forceinline__ void store_accumulator(uint32_t tmem, int warp, int lane, bool leader, uint8_t *stg,
                                                   const CUtensorMap *map, const CUtensorMap *map_t, int64_t r,
-                                                  int64_t rows, int32_t row0, uint32_t &ecount, uint32_t bar_id) {
-  // staging buffer eb: [row-major 128 x 32 box | 4 transposed 32 x 32 boxes (one per warp)]
+                                                  int64_t rows, int32_t row0, uint32_t &ecount, uint32_t bar_id,
+                                                  int group, int ngroups) {
+  // ngroups 128-thread groups (4 warps each, covering the 4 TMEM lane quarters) split the
+  // 32-column chunks; each staging buffer is [row-major 128 x 32 box | 4 transposed 32 x 32
+  // boxes].  With one group the two buffers alternate; with two, group g owns buffer g.
   const uint32_t lg = (uint32_t)(warp & 3), row = 32u * lg + lane;
   const int nch = (int)((r + 31) / 32);
-  for (int j = 0; j < nch; ++j) {
-    const uint32_t eb = ecount & 1u;
+  for (int j = group; j < nch; j += ngroups) {
+    const uint32_t eb = (ngroups == 1) ? (ecount & 1u) : (uint32_t)group;
     uint8_t *box = stg + eb * 2 * EPI_BOX, *tbox = box + EPI_BOX + lg * (EPI_BOX / 4);
-    if (leader) bulk_wait_read<1>();  // the stores issued two chunks ago have read this buffer
+    if (leader) {  // the stores that last used this buffer have read it
+      if (ngroups == 1) bulk_wait_read<1>();
+      else bulk_wait_read<0>();
+    }
     named_sync(bar_id, 128);
     uint32_t v[32];
     tmem_ld32(tmem + (lg * 32u << 16) + j * 32, v);
@@ -74,55 +82,79 @@ __device__ __forceinline__ void store_accumulator(uint32_t tmem, int warp, int l
 }
 
 // =============================================================== B = M + G, P = B Q ===
-constexpr int F_THREADS = 14 * 32;
+constexpr int F_THREADS = 10 * 32;  // 8 producer/epilogue warps, TMA warp, MMA warp
+
+// A chunk (128 rows x 64 columns of B) is produced in two halves of 64 rows.  Each producer
+// thread owns 4 groups of 4 columns per half (row = h * 64 + u * 16 + warp * 2 + lane / 16,
+// columns 4 * (lane % 16) ..).  All loads of a half are issued before any is used, and the next
+// half's loads are in flight while the current half is processed.
+template <int GT>
+struct RawHalf {
+  float4 m[4];
+  typename std::conditional<GT == DT_BF16, uint2, float4>::type g[4];
+};
 
 template <int GT>
-__device__ __forceinline__ void load_group(const DevLayer &L, int64_t gi, int64_t gc, float m[4], float g[4]) {
-  const bool full = gi < L.m && gc + 4 <= L.n;
-  if (full) {
-    const float4 mv = *reinterpret_cast<const float4 *>(L.M + gi * L.ldm + gc);
-    m[0] = mv.x; m[1] = mv.y; m[2] = mv.z; m[3] = mv.w;
-    if (GT == DT_BF16) {
-      const uint2 gv = *reinterpret_cast<const uint2 *>(static_cast<const __nv_bfloat16 *>(L.G) + gi * L.ldg + gc);
-      g[0] = bf16_bits_to_float(gv.x & 0xffffu); g[1] = bf16_bits_to_float(gv.x >> 16);
-      g[2] = bf16_bits_to_float(gv.y & 0xffffu); g[3] = bf16_bits_to_float(gv.y >> 16);
-    } else {
-      const float4 gv = *reinterpret_cast<const float4 *>(static_cast<const float *>(L.G) + gi * L.ldg + gc);
-      g[0] = gv.x; g[1] = gv.y; g[2] = gv.z; g[3] = gv.w;
-    }
-  } else {
+__device__ __forceinline__ void load_half(const DevLayer &L, int64_t r0, int64_t c0, int warp, int lane,
+                                          RawHalf<GT> &raw) {
+  const int prow = warp * 2 + (lane >> 4), pcol = (lane & 15) * 4;
+  const int64_t gc = c0 + pcol;
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const bool in = gi < L.m && gc + e < L.n;
-      m[e] = in ? L.M[gi * L.ldm + gc + e] : 0.f;
-      if (GT == DT_BF16) g[e] = in ? __bfloat162float(static_cast<const __nv_bfloat16 *>(L.G)[gi * L.ldg + gc + e]) : 0.f;
-      else g[e] = in ? static_cast<const float *>(L.G)[gi * L.ldg + gc + e] : 0.f;
+  for (int u = 0; u < 4; ++u) {
+    const int64_t gi = r0 + u * 16 + prow;
+    if (gi < L.m && gc + 4 <= L.n) {
+      raw.m[u] = __ldg(reinterpret_cast<const float4 *>(L.M + gi * L.ldm + gc));
+      if constexpr (GT == DT_BF16)
+        raw.g[u] = __ldg(reinterpret_cast<const uint2 *>(static_cast<const __nv_bfloat16 *>(L.G) + gi * L.ldg + gc));
+      else
+        raw.g[u] = __ldg(reinterpret_cast<const float4 *>(static_cast<const float *>(L.G) + gi * L.ldg + gc));
+    } else {  // ragged edge: element-wise, zeros outside the matrix
+      float mm[4];
+      uint32_t gb[4];
+      float gf[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const bool in = gi < L.m && gc + e < L.n;
+        mm[e] = in ? L.M[gi * L.ldm + gc + e] : 0.f;
+        if constexpr (GT == DT_BF16)
+          gb[e] = in ? (uint32_t)reinterpret_cast<const uint16_t *>(L.G)[gi * L.ldg + gc + e] : 0u;
+        else
+          gf[e] = in ? static_cast<const float *>(L.G)[gi * L.ldg + gc + e] : 0.f;
+      }
+      raw.m[u] = make_float4(mm[0], mm[1], mm[2], mm[3]);
+      if constexpr (GT == DT_BF16)
+        raw.g[u] = make_uint2(gb[0] | (gb[1] << 16), gb[2] | (gb[3] << 16));
+      else
+        raw.g[u] = make_float4(gf[0], gf[1], gf[2], gf[3]);
     }
   }
 }
 
-// One 128 x 64 chunk: 256 producer threads, 8 groups of 4 columns each
-// (row = u * 16 + warp * 2 + lane / 16, columns 4 * (lane % 16) ..).
+// B = M + G for one half: stores of B and Bh, bf16 B into the K-major 128-byte-swizzled A
+// operand (zeros outside the matrix), squared-norm sums.  r0 is the half's first row and
+// trow its first row inside the 128-row tile.
 template <int GT>
-__device__ __forceinline__ void produce_chunk(const DevLayer &L, int64_t r0, int64_t c0, uint8_t *sA, int warp,
-                                              int lane, float &sb, float &sm, const Abort &ab, uint64_t *empty_bar,
-                                              uint32_t parity, int32_t *status, bool &ok) {
+__device__ __forceinline__ void process_half(const DevLayer &L, int64_t r0, int trow, int64_t c0, uint8_t *sA,
+                                             int warp, int lane, const RawHalf<GT> &raw, float &sb, float &sm) {
   const int prow = warp * 2 + (lane >> 4), pcol = (lane & 15) * 4;
-  float mv[8][4], gv[8][4];
+  const int64_t gc = c0 + pcol;
 #pragma unroll
-  for (int u = 0; u < 8; ++u) load_group<GT>(L, r0 + u * 16 + prow, c0 + pcol, mv[u], gv[u]);
-  if (!__all_sync(0xffffffffu, ab.wait(empty_bar, parity, status))) {  // warp-uniform decision
-    ok = false;
-    return;
-  }
-#pragma unroll
-  for (int u = 0; u < 8; ++u) {
-    const int64_t row = u * 16 + prow, gi = r0 + row, gc = c0 + pcol;
+  for (int u = 0; u < 4; ++u) {
+    const int row = trow + u * 16 + prow;
+    const int64_t gi = r0 + u * 16 + prow;
+    const float mv[4] = {raw.m[u].x, raw.m[u].y, raw.m[u].z, raw.m[u].w};
+    float gv[4];
+    if constexpr (GT == DT_BF16) {
+      gv[0] = bf16_bits_to_float(raw.g[u].x & 0xffffu); gv[1] = bf16_bits_to_float(raw.g[u].x >> 16);
+      gv[2] = bf16_bits_to_float(raw.g[u].y & 0xffffu); gv[3] = bf16_bits_to_float(raw.g[u].y >> 16);
+    } else {
+      gv[0] = raw.g[u].x; gv[1] = raw.g[u].y; gv[2] = raw.g[u].z; gv[3] = raw.g[u].w;
+    }
     float b[4];
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
-      sm = fmaf(mv[u][e], mv[u][e], sm);
-      b[e] = mv[u][e] + gv[u][e];
+      sm = fmaf(mv[e], mv[e], sm);
+      b[e] = mv[e] + gv[e];
       sb = fmaf(b[e], b[e], sb);
     }
     const __nv_bfloat162 h01 = __floats2bfloat162_rn(b[0], b[1]), h23 = __floats2bfloat162_rn(b[2], b[3]);
@@ -140,13 +172,47 @@ __device__ __forceinline__ void produce_chunk(const DevLayer &L, int64_t r0, int
           L.Bh[gi * L.ldbh + gc + e] = __float2bfloat16_rn(b[e]);
         }
     }
-    // K-major 128-byte-swizzled A operand; out-of-range elements are 0
     *reinterpret_cast<uint2 *>(sA + sw128_offset((uint32_t)row, (uint32_t)(pcol >> 3)) + (pcol & 7) * 2) = hv;
   }
 }
 
-__global__ void __launch_bounds__(F_THREADS, 1)
-    tc_form_bq_kernel(Shared sh, const int4 *__restrict__ tiles, int ntiles, const LayerMaps *__restrict__ maps,
+// The producer loop of one tile, in half-chunk steps h = 2 kc + half.
+template <int GT>
+__device__ __forceinline__ bool produce_tile(const DevLayer &L, int64_t r0, uint8_t *smem, uint32_t stage_bytes,
+                                             int nstages, uint64_t *a_full, uint64_t *empty, uint32_t &it, int warp,
+                                             int lane, const Abort &ab, int32_t *status, double &vb, double &vm) {
+  const int kch = (int)((L.n + 63) / 64), nh = 2 * kch;
+  RawHalf<GT> cur, nxt;
+  load_half<GT>(L, r0, 0, warp, lane, cur);
+  float sb = 0.f, sm = 0.f;
+  for (int h = 0; h < nh; ++h) {
+    const int kc = h >> 1, half = h & 1;
+    if (h + 1 < nh)
+      load_half<GT>(L, r0 + ((h + 1) & 1) * 64, (int64_t)((h + 1) >> 1) * 64, warp, lane, nxt);
+    const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
+    if (half == 0) {
+      if (!__all_sync(0xffffffffu, ab.wait(&empty[s], ph ^ 1u, status))) return false;  // warp-uniform
+      sb = 0.f;
+      sm = 0.f;
+    }
+    process_half<GT>(L, r0 + half * 64, half * 64, (int64_t)kc * 64, smem + s * stage_bytes, warp, lane, cur, sb, sm);
+    if (half == 1) {  // fp32 sums of 32 squares per chunk, folded into fp64
+      vb += (double)sb;
+      vm += (double)sm;
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&a_full[s]);
+      ++it;
+    }
+    if (h + 1 < nh) cur = nxt;
+  }
+  return true;
+}
+
+// 10 warps: at most 3 per SM sub-partition, so up to 168 registers per thread fit the
+// 16K-register file of each sub-partition (room for the producers' prefetch).
+__global__ void __maxnreg__(168)
+    tc_form_bq_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off, const LayerMaps *__restrict__ maps,
                       int nstages, uint32_t stage_bytes, uint32_t tmem_cols) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = align1024(smem_raw);
@@ -165,7 +231,7 @@ __global__ void __launch_bounds__(F_THREADS, 1)
       mbar_init(&empty[i], 1);
     }
     mbar_init(acc_full, 1);
-    mbar_init(acc_empty, 128);
+    mbar_init(acc_empty, 256);  // all 8 producer/epilogue warps
     mbar_init(drain, 1);
     abort_s = 0;
     fence_mbar_init();
@@ -180,30 +246,19 @@ __global__ void __launch_bounds__(F_THREADS, 1)
   const uint32_t tmem = tmem_base_s;
 
   if (warp < 8) {
-    // ------------------------------------------------------------------ producers
-    uint32_t it = 0;
+    // ------------------------------------------------------- producers, then the tile's epilogue
+    const int grp = warp >> 2;  // warps 0..3 and 4..7 each cover the 4 TMEM lane quarters
+    const bool leader = (lane == 0 && (warp & 3) == 0);
+    uint32_t it = 0, tcount = 0, ecount = 0;
     bool ok = true;
-    for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+    for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
       const int4 t = tiles[ti];
       const DevLayer &L = sh.layers[t.x];
       const int64_t r0 = (int64_t)t.y * 128;
-      const int kch = (int)((L.n + 63) / 64);
-      double vb = 0.0, vm = 0.0;  // fp32 sums of 32 squares per chunk, folded into fp64
-      for (int kc = 0; kc < kch && ok; ++kc, ++it) {
-        const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
-        uint8_t *sA = smem + s * stage_bytes;
-        float sb = 0.f, sm = 0.f;
-        if (L.g_dtype == DT_BF16)
-          produce_chunk<DT_BF16>(L, r0, (int64_t)kc * 64, sA, warp, lane, sb, sm, ab, &empty[s], ph ^ 1u, sh.status, ok);
-        else
-          produce_chunk<DT_FP32>(L, r0, (int64_t)kc * 64, sA, warp, lane, sb, sm, ab, &empty[s], ph ^ 1u, sh.status, ok);
-        if (!ok) break;
-        vb += (double)sb;
-        vm += (double)sm;
-        fence_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&a_full[s]);
-      }
+      double vb = 0.0, vm = 0.0;
+      ok = (L.g_dtype == DT_BF16)
+               ? produce_tile<DT_BF16>(L, r0, smem, stage_bytes, nstages, a_full, empty, it, warp, lane, ab, sh.status, vb, vm)
+               : produce_tile<DT_FP32>(L, r0, smem, stage_bytes, nstages, a_full, empty, it, warp, lane, ab, sh.status, vb, vm);
       if (!ok) break;
       // each producer warp owns norm-partial slot 8 * tile + warp (fixed-order sum in the gate)
 #pragma unroll
@@ -215,13 +270,22 @@ __global__ void __launch_bounds__(F_THREADS, 1)
         sh.bpart[2 * (8 * t.w + warp)] = vb;
         sh.bpart[2 * (8 * t.w + warp) + 1] = vm;
       }
+      // epilogue: P (row-major) and P^T of this tile from TMEM
+      if (!named_and(3 + grp, 128, ab.wait(acc_full, tcount & 1u, sh.status))) { ok = false; break; }
+      tc_fence_after();
+      store_accumulator(tmem, warp, lane, leader, stg, &maps[t.x].Praw, &maps[t.x].PTraw_t, L.r, L.m, t.y * 128,
+                        ecount, 3 + grp, grp, 2);
+      tc_fence_before();
+      mbar_arrive(acc_empty);
+      ++tcount;
     }
+    if (leader) bulk_wait<0>();
   } else if (warp == 8) {
     // ------------------------------------------------------------------ TMA (Q operand)
     if (lane == 0) {
       uint32_t it = 0;
       bool ok = true;
-      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+      for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
         const DevLayer &L = sh.layers[t.x];
         const LayerMaps *mp = maps + t.x;
@@ -243,7 +307,7 @@ __global__ void __launch_bounds__(F_THREADS, 1)
     if (lane == 0) {
       uint32_t it = 0, tcount = 0;
       bool ok = true;
-      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x, ++tcount) {
+      for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti, ++tcount) {
         const int4 t = tiles[ti];
         const DevLayer &L = sh.layers[t.x];
         const int kch = (int)((L.n + 63) / 64);
@@ -272,21 +336,6 @@ __global__ void __launch_bounds__(F_THREADS, 1)
       umma_commit(drain);
       mbar_wait(drain, 0, sh.status);
     }
-  } else {
-    // ------------------------------------------------------------------ epilogue (warps 10..13)
-    const bool leader = (warp == 10 && lane == 0);
-    uint32_t tcount = 0, ecount = 0;
-    for (int ti = blockIdx.x; ti < ntiles; ti += gridDim.x, ++tcount) {
-      const int4 t = tiles[ti];
-      const DevLayer &L = sh.layers[t.x];
-      if (!named_and(3, 128, ab.wait(acc_full, tcount & 1u, sh.status))) break;
-      tc_fence_after();
-      store_accumulator(tmem, warp, lane, leader, stg, &maps[t.x].Praw, &maps[t.x].PTraw_t, L.r, L.m, t.y * 128,
-                        ecount, 3);
-      tc_fence_before();
-      mbar_arrive(acc_empty);
-    }
-    if (leader) bulk_wait<0>();
   }
   tc_fence_before();
   __syncthreads();
@@ -298,7 +347,7 @@ __global__ void __launch_bounds__(F_THREADS, 1)
 constexpr int R_THREADS = 6 * 32;
 
 __global__ void __launch_bounds__(R_THREADS, 1)
-    tc_btp_kernel(Shared sh, const int4 *__restrict__ tiles, int ntiles, const LayerMaps *__restrict__ maps,
+    tc_btp_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off, const LayerMaps *__restrict__ maps,
                   int nstages, uint32_t stage_bytes, uint32_t tmem_cols) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = align1024(smem_raw);
@@ -334,7 +383,7 @@ __global__ void __launch_bounds__(R_THREADS, 1)
     if (lane == 0) {
       uint32_t it = 0;
       bool ok = true;
-      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+      for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
         if (!sh.active[t.x]) continue;
         const DevLayer &L = sh.layers[t.x];
@@ -358,7 +407,7 @@ __global__ void __launch_bounds__(R_THREADS, 1)
     if (lane == 0) {
       uint32_t it = 0, tcount = 0;
       bool ok = true;
-      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+      for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
         if (!sh.active[t.x]) continue;
         const DevLayer &L = sh.layers[t.x];
@@ -392,13 +441,13 @@ __global__ void __launch_bounds__(R_THREADS, 1)
   } else {
     const bool leader = (warp == 2 && lane == 0);
     uint32_t tcount = 0, ecount = 0;
-    for (int ti = blockIdx.x; ti < ntiles; ti += gridDim.x) {
+    for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1]; ++ti) {
       const int4 t = tiles[ti];
       if (!sh.active[t.x]) continue;
       const DevLayer &L = sh.layers[t.x];
       if (!named_and(1, 128, ab.wait(acc_full, tcount & 1u, sh.status))) break;
       tc_fence_after();
-      store_accumulator(tmem, warp, lane, leader, stg, &maps[t.x].Rst, nullptr, L.r, L.n, t.y * 128, ecount, 1);
+      store_accumulator(tmem, warp, lane, leader, stg, &maps[t.x].Rst, nullptr, L.r, L.n, t.y * 128, ecount, 1, 0, 1);
       tc_fence_before();
       mbar_arrive(acc_empty);
       ++tcount;
@@ -436,19 +485,17 @@ cudaError_t setup_bq_kernels(uint32_t f_smem, uint32_t r_smem) {
 }
 
 void launch_form_bq(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
-  if (tp.n_ftiles <= 0) return;
-  const int grid = std::min(tp.n_ftiles, std::max(tp.num_sms, 1));
+  if (tp.d_bq.grid <= 0) return;
   const uint32_t stage = OPB_A + tp.nb64 * BOX64;
-  tc_form_bq_kernel<<<grid, F_THREADS, tp.f_smem, s>>>(sh, tp.ftiles, tp.n_ftiles, tp.maps, tp.f_stages, stage,
-                                                        tp.tmem_cols);
+  tc_form_bq_kernel<<<tp.d_bq.grid, F_THREADS, tp.f_smem, s>>>(sh, tp.d_bq.tiles, tp.d_bq.off, tp.maps,
+                                                               tp.f_stages, stage, tp.tmem_cols);
 }
 
 void launch_btp(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
-  if (tp.n_rtiles <= 0) return;
-  const int grid = std::min(tp.n_rtiles, std::max(tp.num_sms, 1));
+  if (tp.d_btp.grid <= 0) return;
   const uint32_t stage = OPB_A + tp.nb64 * BOX64;
-  tc_btp_kernel<<<grid, R_THREADS, tp.r_smem, s>>>(sh, tp.rtiles, tp.n_rtiles, tp.maps, tp.r_stages, stage,
-                                                    tp.tmem_cols);
+  tc_btp_kernel<<<tp.d_btp.grid, R_THREADS, tp.r_smem, s>>>(sh, tp.d_btp.tiles, tp.d_btp.off, tp.maps,
+                                                            tp.r_stages, stage, tp.tmem_cols);
 }
 
 void launch_qn_refresh(const Shared &sh, const TcPlan &tp, cudaStream_t s) {

@@ -70,7 +70,7 @@ __device__ __forceinline__ bool part_needs(int kc, uint32_t part) {
 
 template <int KIND>
 __global__ void __launch_bounds__(O_THREADS, 1)
-    tc_orth_kernel(Shared sh, const int4 *__restrict__ tiles, int ntiles, const LayerMaps *__restrict__ maps,
+    tc_orth_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off, const LayerMaps *__restrict__ maps,
                    int pass, int nstages, uint32_t stage_bytes, uint32_t tmem_cols) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = align1024(smem_raw);
@@ -107,7 +107,7 @@ __global__ void __launch_bounds__(O_THREADS, 1)
     if (lane == 0) {
       uint32_t it = 0;
       bool ok = true;
-      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+      for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
         if (skip(t.x)) continue;
         const DevLayer &L = sh.layers[t.x];
@@ -137,7 +137,7 @@ __global__ void __launch_bounds__(O_THREADS, 1)
     if (lane == 0) {
       uint32_t it = 0, tcount = 0;
       bool ok = true;
-      for (int ti = blockIdx.x; ti < ntiles && ok; ti += gridDim.x) {
+      for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
         if (skip(t.x)) continue;
         const DevLayer &L = sh.layers[t.x];
@@ -178,7 +178,7 @@ __global__ void __launch_bounds__(O_THREADS, 1)
     const bool leader = (warp == 2 && lane == 0);
     const uint32_t lg = (uint32_t)(warp & 3), row = 32u * lg + lane;
     uint32_t tcount = 0, ecount = 0;
-    for (int ti = blockIdx.x; ti < ntiles; ti += gridDim.x) {
+    for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1]; ++ti) {
       const int4 t = tiles[ti];
       if (skip(t.x)) continue;
       const DevLayer &L = sh.layers[t.x];
@@ -244,17 +244,15 @@ cudaError_t setup_orth_kernels(uint32_t smem) {
 }
 
 void launch_orth(const Shared &sh, const TcPlan &tp, bool gram, int pass, cudaStream_t s) {
-  const int4 *tiles = gram ? tp.gram_tiles : tp.trsm_tiles;
-  const int n = gram ? tp.n_gram_tiles : tp.n_trsm_tiles;
-  if (n <= 0) return;
-  const int grid = std::min(n, std::max(tp.num_sms, 1));
+  const DevSchedule &d = gram ? tp.d_gram : tp.d_trsm;
+  if (d.grid <= 0) return;
   const uint32_t stage = O_BOX * (1 + tp.nb128);
   if (gram)
-    tc_orth_kernel<ORTH_GRAM><<<grid, O_THREADS, tp.o_smem, s>>>(sh, tiles, n, tp.maps, pass, tp.o_stages, stage,
-                                                                   tp.tmem_cols);
+    tc_orth_kernel<ORTH_GRAM><<<d.grid, O_THREADS, tp.o_smem, s>>>(sh, d.tiles, d.off, tp.maps, pass, tp.o_stages,
+                                                                     stage, tp.tmem_cols);
   else
-    tc_orth_kernel<ORTH_TRSM><<<grid, O_THREADS, tp.o_smem, s>>>(sh, tiles, n, tp.maps, pass, tp.o_stages, stage,
-                                                                   tp.tmem_cols);
+    tc_orth_kernel<ORTH_TRSM><<<d.grid, O_THREADS, tp.o_smem, s>>>(sh, d.tiles, d.off, tp.maps, pass, tp.o_stages,
+                                                                     stage, tp.tmem_cols);
 }
 
 }  // namespace tc
