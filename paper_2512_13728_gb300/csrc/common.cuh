@@ -55,6 +55,9 @@ struct DevLayer {
   int64_t ldbh;
   float *PT_raw, *PT;    // r x m, pitch ldmt : transposed copies of P_raw and P (tensor-core Gram)
   int64_t ldmt;
+  double *colsq;         // [row tiles of R][ldp]: per-tile column sums of squares of R
+  float *colinv;         // [ldp]: 1 / (||R[:, j]|| + eps_col)
+  int32_t rtile_cnt, pad1;
   int32_t bpart_off, bpart_cnt;  // slots of the ||B||^2 / ||M_{t-1}||^2 partials
   int32_t upart_off, upart_cnt;  // slots of the ||M_t||^2 partials
 };
@@ -127,7 +130,8 @@ void launch_gate(const Shared &sh, const StepArgs &a, cudaStream_t s);
 void launch_gemm(const Shared &sh, const GemmProblem *probs, const int4 *tiles, int32_t ntiles,
                  cudaStream_t s);
 cudaError_t prepare_chol_inv(int32_t max_r, size_t *smem_out);
-void launch_chol_inv(const Shared &sh, size_t smem, int32_t pass, cudaStream_t s);
+// near_identity: Frobenius bound on S - I below which passes 1 and 2 use the first-order factor
+void launch_chol_inv(const Shared &sh, size_t smem, int32_t pass, float near_identity, cudaStream_t s);
 void launch_colnorm(const Shared &sh, const int4 *tiles, int32_t ntiles, float eps_col,
                     cudaStream_t s);
 void launch_update(const Shared &sh, const int4 *tiles, int32_t ntiles, float mu, float eta,

@@ -351,7 +351,11 @@ __device__ bool cholesky_blocked(float *S, int r, int64_t ls, float *D, float *P
 }
 
 // pass 0 and 1: every active layer; pass 2: only layers marked by a shifted retry.
-__global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int pass) {
+// Passes 1 and 2 factor the Gram matrix of an already nearly orthonormal X: when 1.5 times a
+// power-iteration estimate of ||S - I||_2 is below near_identity, the factor of S = I + E is
+// taken to first order, L = I + F with F = strictly-lower(E) + diag(E) / 2 and
+// L^{-1} = I - F; the resulting X L^{-T} is then orthonormal up to O(||E||_2^2).
+__global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int pass, float near_identity) {
   const int l = blockIdx.x;
   if (!sh.active[l]) return;
   if (pass == 2 && !sh.orth_shifted[l]) return;
@@ -370,11 +374,93 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int p
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   // The Gram producers may write only the lower triangle: mirror it into the upper one, which
   // the factorization never touches and the shifted retry restores the lower triangle from.
-  for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) {
-    const int64_t i = e / r, j = e % r;
-    if (j > i) S[i * ls + j] = S[j * ls + i];
+  // 32 x 32 tiles transposed through a per-warp shared scratch (Pn holds 33 r floats, so r / 32
+  // warps have room), coalesced on both sides.
+  {
+    const int nt = (r + 31) / 32, nwm = min(kCholThreads / 32, r / 32);
+    if (nwm == 0) {
+      for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) {
+        const int64_t i = e / r, j = e % r;
+        if (j > i) S[i * ls + j] = S[j * ls + i];
+      }
+    } else if (warp < nwm) {
+      float *tb = Pn + warp * (32 * 33);
+      const int npairs = nt * (nt - 1) / 2;
+      for (int u = warp; u < npairs + nt; u += nwm) {
+        int bi, bj;  // upper tile (bi, bj), bj >= bi; u < npairs: off-diagonal, else the diagonal tile
+        if (u < npairs) {
+          bj = (int)tri_row(u) + 1;
+          bi = u - (bj - 1) * bj / 2;
+        } else {
+          bi = bj = u - npairs;
+        }
+        for (int y = 0; y < 32; ++y) {  // lower tile (bj, bi) -> scratch
+          const int gi = bj * 32 + y, gj = bi * 32 + lane;
+          tb[y * 33 + lane] = (gi < r && gj < r) ? S[(int64_t)gi * ls + gj] : 0.f;
+        }
+        __syncwarp();
+        for (int y = 0; y < 32; ++y) {  // upper tile (bi, bj) = transpose
+          const int gi = bi * 32 + y, gj = bj * 32 + lane;
+          if (gi < r && gj < r && gj > gi) S[(int64_t)gi * ls + gj] = tb[lane * 33 + y];
+        }
+        __syncwarp();
+      }
+    }
+    __syncthreads();
   }
   for (int i = tid; i < r; i += kCholThreads) diag0[i] = S[(int64_t)i * ls + i];
+  if (pass >= 1) {
+    // ||E||_2 of E = S - I by 8 power iterations (one warp per row, coalesced row reads)
+    float *v = Pn, *wv = Pn + r;  // Pn holds at least 33 * r floats
+    __shared__ float wn[kCholThreads / 32];
+    __shared__ float lam_s;
+    for (int i = tid; i < r; i += kCholThreads) v[i] = 1.f + 0.25f * __sinf(0.7f * (float)i);  // fixed start
+    __syncthreads();
+    float lam = 0.f;
+    for (int itp = 0; itp < 8; ++itp) {
+      for (int i = warp; i < r; i += kCholThreads / 32) {
+        float acc0 = 0.f, acc1 = 0.f;
+        int j = lane;
+        for (; j + 32 < r; j += 64) {
+          acc0 = fmaf(S[(int64_t)i * ls + j] - (i == j ? 1.f : 0.f), v[j], acc0);
+          acc1 = fmaf(S[(int64_t)i * ls + j + 32] - (i == j + 32 ? 1.f : 0.f), v[j + 32], acc1);
+        }
+        if (j < r) acc0 = fmaf(S[(int64_t)i * ls + j] - (i == j ? 1.f : 0.f), v[j], acc0);
+        float acc = acc0 + acc1;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        if (lane == 0) wv[i] = acc;
+      }
+      __syncthreads();
+      float pn = 0.f;
+      for (int i = tid; i < r; i += kCholThreads) pn = fmaf(wv[i], wv[i], pn);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) pn += __shfl_xor_sync(0xffffffffu, pn, o);
+      if (lane == 0) wn[warp] = pn;
+      __syncthreads();
+      if (tid == 0) {
+        float a = 0.f;
+        for (int w = 0; w < kCholThreads / 32; ++w) a += wn[w];
+        lam_s = a;  // ||E v||^2
+      }
+      __syncthreads();
+      const float nrm = sqrtf(lam_s);
+      // ||E v|| / ||v||: v has unit norm from the second iteration on
+      lam = nrm;
+      const float inv = (nrm > 0.f && isfinite(nrm)) ? 1.f / nrm : 0.f;
+      for (int i = tid; i < r; i += kCholThreads) v[i] = wv[i] * inv;
+      __syncthreads();
+      if (itp == 0) lam = INFINITY;  // the first product uses an unnormalized start vector
+    }
+    if (isfinite(lam) && 1.5f * lam < near_identity) {
+      for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) {
+        const int64_t i = e / r, j = e % r;
+        const float sij = S[i * ls + j];
+        Li[i * ls + j] = (j < i) ? -sij : (j == i ? 1.f - 0.5f * (sij - 1.f) : 0.f);
+      }
+      return;
+    }
+  }
   __syncthreads();
 
   bool ok = cholesky_blocked(S, r, ls, D, Pn, &bad);
@@ -493,8 +579,8 @@ cudaError_t prepare_chol_inv(int32_t max_r, size_t *smem_out) {
   return cudaFuncSetAttribute(chol_inv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
 }
 
-void launch_chol_inv(const Shared &sh, size_t smem, int32_t pass, cudaStream_t s) {
-  if (sh.num_layers > 0) chol_inv_kernel<<<sh.num_layers, kCholThreads, smem, s>>>(sh, pass);
+void launch_chol_inv(const Shared &sh, size_t smem, int32_t pass, float near_identity, cudaStream_t s) {
+  if (sh.num_layers > 0) chol_inv_kernel<<<sh.num_layers, kCholThreads, smem, s>>>(sh, pass, near_identity);
 }
 
 // ===================================================================== ColumnNormalize ===

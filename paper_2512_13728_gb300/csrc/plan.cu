@@ -353,7 +353,7 @@ dion_status dion_step(dion_plan *p, const dion_hparams *hp, double *prev_norm, d
     for (int pass = 0; pass < 3; ++pass) {  // CholeskyQR2, third pass only after a shifted retry
       launch_gemm(sh, p->probs[1 + pass], p->gtiles[1 + pass], p->n_gtiles[1 + pass], s);  // S = X^T X
       tick(p, s, kGram[pass]);
-      launch_chol_inv(sh, p->chol_smem, pass, s);  // L, L^{-1}
+      launch_chol_inv(sh, p->chol_smem, pass, 1e-3f, s);  // L, L^{-1}
       tick(p, s, kChol[pass]);
       launch_gemm(sh, p->probs[4 + pass], p->gtiles[4 + pass], p->n_gtiles[4 + pass], s);  // X L^{-T}
       tick(p, s, kTrsm[pass]);

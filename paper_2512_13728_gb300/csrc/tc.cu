@@ -301,6 +301,8 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
   lo.o_bh.resize(L);
   lo.o_ptraw.resize(L);
   lo.o_pt.resize(L);
+  lo.o_colsq.resize(L);
+  lo.o_colinv.resize(L);
   int32_t fslot = 0;
   for (int32_t l = 0; l < L; ++l) {
     const dion_layer &ly = layers[l];
@@ -313,6 +315,8 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
     const int64_t ldmt = (ly.m + 7) / 8 * 8;
     lo.o_ptraw[l] = take(ly.r * ldmt * 4);
     lo.o_pt[l] = take(ly.r * ldmt * 4);
+    lo.o_colsq[l] = take((size_t)((ly.n + 127) / 128) * ldp * 8);
+    lo.o_colinv[l] = take(ldp * 4);
     for (int64_t rb = 0; rb < (ly.r + 127) / 128; ++rb) lo.gram_tiles.push_back(make_int4(l, (int)rb, 0, 0));
     for (int64_t mb = 0; mb < (ly.m + 127) / 128; ++mb) lo.trsm_tiles.push_back(make_int4(l, (int)mb, 0, 0));
     for (int64_t mb = 0; mb < (ly.m + 127) / 128; ++mb)
@@ -368,6 +372,9 @@ void bind(const TcLayout &lo, char *base, DevLayer *dl, int32_t L, TcPlan *tp) {
     dl[l].PT_raw = reinterpret_cast<float *>(base + lo.o_ptraw[l]);
     dl[l].PT = reinterpret_cast<float *>(base + lo.o_pt[l]);
     dl[l].ldmt = (dl[l].m + 7) / 8 * 8;
+    dl[l].colsq = reinterpret_cast<double *>(base + lo.o_colsq[l]);
+    dl[l].colinv = reinterpret_cast<float *>(base + lo.o_colinv[l]);
+    dl[l].rtile_cnt = (int32_t)((dl[l].n + 127) / 128);
     // norm partials: 8 slots (one per producer warp) per 128-row tile of the fused B Q kernel
     const int32_t tiles = (int32_t)bq_tiles(dl[l].m);
     dl[l].bpart_off = 8 * fslot;
@@ -484,7 +491,7 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   tp->num_sms = sms;
-  tp->launches = 17;
+  tp->launches = 18;
   return e;
 }
 
@@ -504,7 +511,7 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, c
   for (int pass = 0; pass < 3; ++pass) {  // CholeskyQR2; the third pass only after a shifted retry
     launch_orth(sh, tp, true, pass, s);  // S = X^T X
     tick(p, s, kGram[pass]);
-    launch_chol_inv(sh, chol_smem, pass, s);  // L, L^{-1}
+    launch_chol_inv(sh, chol_smem, pass, 6e-2f, s);  // L, L^{-1}
     tick(p, s, kChol[pass]);
     launch_orth(sh, tp, false, pass, s);  // X L^{-T} and its transpose
     tick(p, s, kTrsm[pass]);
@@ -513,8 +520,10 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, c
   tick(p, s, "cvt_p");
   launch_btp(sh, tp, s);  // R = B^T P
   tick(p, s, "tc_btp");
-  launch_colnorm(sh, ctiles, n_ctiles, a.eps_col, s);  // Q_t, and bf16 R, Q_t
-  tick(p, s, "colnorm");
+  launch_colnorm_reduce(sh, ctiles, n_ctiles, a.eps_col, s);  // 1 / (||R_j|| + eps) from tile partials
+  tick(p, s, "colnorm_reduce");
+  launch_colnorm_scale(sh, tp, s);  // Q_t = R diag(...), its bf16 copy
+  tick(p, s, "colnorm_scale");
   if (tp.d_update.grid > 0)
     tc_update_kernel<<<tp.d_update.grid, U_THREADS, U_SMEM, s>>>(sh, tp.d_update.tiles, tp.d_update.off, tp.maps,
                                                                   a.mu, a.eta);

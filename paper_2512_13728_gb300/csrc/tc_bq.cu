@@ -81,6 +81,80 @@ __device__ __forceinline__ void store_accumulator(uint32_t tmem, int warp, int l
   }
 }
 
+// Epilogue of R = B^T P for one 128-row tile of R: the fp32 rows of R and their bf16 copy
+// (TMA stores) and, per column, the tile's fp64 sum of squares for ColumnNormalize.
+// Two 32-column chunks are handled together so the bf16 box is one 64-column SW128 box.
+__device__ __forceinline__ void store_r_tile(uint32_t tmem, int warp, int lane, bool leader, uint8_t *stg,
+                                             const LayerMaps &mp, const DevLayer &L, int tile, uint32_t &ecount) {
+  const uint32_t lg = (uint32_t)(warp & 3), row = 32u * lg + lane;
+  const int et = (warp - 2) * 32 + lane;  // 0..127 within the epilogue warps (warps 2..5)
+  const int nch = (int)((L.r + 31) / 32), row0 = tile * 128;
+  // staging: [fp32 box 16 KB][fp32 box 16 KB][bf16 box 16 KB] + column-partial scratch 4 x 64 floats
+  uint8_t *f0 = stg, *f1 = stg + EPI_BOX, *hb = stg + 2 * EPI_BOX;
+  float *red = reinterpret_cast<float *>(stg + 3 * EPI_BOX);
+  for (int j = 0; j < nch; j += 2) {
+    const bool two = (j + 1 < nch);
+    if (leader) bulk_wait_read<0>();
+    named_sync(1, 128);
+    uint32_t v[32];
+#pragma unroll 1
+    for (int h = 0; h < (two ? 2 : 1); ++h) {
+      tmem_ld32(tmem + (lg * 32u << 16) + (j + h) * 32, v);
+      tmem_ld_wait();
+      uint8_t *fb = h ? f1 : f0;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        *reinterpret_cast<float4 *>(fb + sw128_f32(row, q)) =
+            make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]), __uint_as_float(v[4 * q + 2]),
+                        __uint_as_float(v[4 * q + 3]));
+        const __nv_bfloat162 a = __floats2bfloat162_rn(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]));
+        const __nv_bfloat162 b = __floats2bfloat162_rn(__uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+        uint2 hv;
+        hv.x = *reinterpret_cast<const uint32_t *>(&a);
+        hv.y = *reinterpret_cast<const uint32_t *>(&b);
+        // bf16 64-column box: columns h*32 + 4q .. live in 16-byte chunk (h*4 + q/2)
+        *reinterpret_cast<uint2 *>(hb + sw128_offset(row, (uint32_t)(h * 4 + (q >> 1))) + (q & 1) * 8) = hv;
+      }
+    }
+    if (!two) {  // a lone last chunk: zero the unused half of the bf16 box (clipped by the store anyway)
+#pragma unroll
+      for (int q = 4; q < 8; ++q) *reinterpret_cast<uint4 *>(hb + sw128_offset(row, q)) = make_uint4(0, 0, 0, 0);
+    }
+    fence_async_smem();
+    named_sync(1, 128);
+    if (leader) {
+      tma_store_2d(&mp.Rst, f0, j * 32, row0);
+      if (two) tma_store_2d(&mp.Rst, f1, (j + 1) * 32, row0);
+      tma_store_2d(&mp.R_hi, hb, j * 32, row0);
+      bulk_commit();
+    }
+    // column sums of squares: thread et sums column (et % 32) of chunk j + h over rows (et / 32) * 32 ..
+    const int c = et & 31, quarter = et >> 5;
+#pragma unroll 1
+    for (int h = 0; h < (two ? 2 : 1); ++h) {
+      const uint8_t *fb = h ? f1 : f0;
+      float ssq = 0.f;
+      for (int rr = 0; rr < 32; ++rr) {
+        const uint32_t rw = (uint32_t)(quarter * 32 + rr);
+        const float x = *reinterpret_cast<const float *>(fb + rw * 128u + ((((uint32_t)c >> 2) ^ (rw & 7u)) << 4) +
+                                                         (c & 3) * 4);
+        ssq = fmaf(x, x, ssq);
+      }
+      red[h * 128 + quarter * 32 + c] = ssq;
+    }
+    named_sync(1, 128);
+    if (et < 64) {
+      const int h = et >> 5, cc = et & 31, col = (j + h) * 32 + cc;
+      if (h == 0 || two) {
+        const double tot = ((double)red[h * 128 + cc] + red[h * 128 + 32 + cc]) +
+                           ((double)red[h * 128 + 64 + cc] + red[h * 128 + 96 + cc]);
+        if (col < L.r) L.colsq[(int64_t)tile * L.ldp + col] = tot;  // rows outside R held zeros
+      }
+    }
+    ecount += two ? 2 : 1;
+  }
+}
+
 // =============================================================== B = M + G, P = B Q ===
 constexpr int F_THREADS = 10 * 32;  // 8 producer/epilogue warps, TMA warp, MMA warp
 
@@ -447,7 +521,7 @@ __global__ void __launch_bounds__(R_THREADS, 1)
       const DevLayer &L = sh.layers[t.x];
       if (!named_and(1, 128, ab.wait(acc_full, tcount & 1u, sh.status))) break;
       tc_fence_after();
-      store_accumulator(tmem, warp, lane, leader, stg, &maps[t.x].Rst, nullptr, L.r, L.n, t.y * 128, ecount, 1, 0, 1);
+      store_r_tile(tmem, warp, lane, leader, stg, maps[t.x], L, t.y, ecount);
       tc_fence_before();
       mbar_arrive(acc_empty);
       ++tcount;
@@ -500,6 +574,48 @@ void launch_btp(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
 
 void launch_qn_refresh(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
   if (tp.n_qtiles > 0) qn_refresh_kernel<<<tp.n_qtiles, 256, 0, s>>>(sh, tp.qtiles);
+}
+
+// ColumnNormalize from the per-tile column sums of squares: colinv[j] = 1 / (||R_j|| + eps),
+// fixed-order fp64 sum over the R tiles of the layer.  Grid: one block per (layer, 32 columns).
+__global__ void __launch_bounds__(256) colnorm_reduce_kernel(Shared sh, const int4 *ctiles, float eps_col) {
+  const int4 t = ctiles[blockIdx.x];  // {layer, 32-column group, 0, 0}
+  if (!sh.active[t.x]) return;
+  const DevLayer &L = sh.layers[t.x];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t j = (int64_t)t.y * 32 + lane;
+  __shared__ double part[8][32];
+  double acc = 0.0;
+  if (j < L.r)
+    for (int k = warp; k < L.rtile_cnt; k += 8) acc += L.colsq[(int64_t)k * L.ldp + j];
+  part[warp][lane] = acc;
+  __syncthreads();
+  if (warp == 0 && j < L.r) {
+    double s2 = 0.0;
+    for (int w = 0; w < 8; ++w) s2 += part[w][lane];
+    L.colinv[j] = (float)(1.0 / (sqrt(s2) + (double)eps_col));
+  }
+}
+
+// Q_t = R diag(colinv) (fp32, caller's buffer) and its bf16 copy; tiles of rows of R.
+__global__ void __launch_bounds__(256) colnorm_scale_kernel(Shared sh, const int4 *tiles) {
+  const int4 t = tiles[blockIdx.x];  // {layer, first row, rows, 0}
+  if (!sh.active[t.x]) return;
+  const DevLayer &L = sh.layers[t.x];
+  const int64_t r = L.r, total = (int64_t)t.z * r;
+  for (int64_t e = threadIdx.x; e < total; e += 256) {
+    const int64_t i = t.y + e / r, j = e % r;
+    const float q = L.R[i * L.ldp + j] * L.colinv[j];
+    L.Q[i * L.ldq + j] = q;
+    L.Qn_hi[i * L.ldp + j] = __float2bfloat16_rn(q);
+  }
+}
+
+void launch_colnorm_reduce(const Shared &sh, const int4 *ctiles, int32_t n_ctiles, float eps_col, cudaStream_t s) {
+  if (n_ctiles > 0) colnorm_reduce_kernel<<<n_ctiles, 256, 0, s>>>(sh, ctiles, eps_col);
+}
+void launch_colnorm_scale(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
+  if (tp.n_qtiles > 0) colnorm_scale_kernel<<<tp.n_qtiles, 256, 0, s>>>(sh, tp.qtiles);
 }
 
 }  // namespace tc

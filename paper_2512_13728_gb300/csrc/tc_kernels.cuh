@@ -13,6 +13,8 @@ cudaError_t setup_bq_kernels(uint32_t f_smem, uint32_t r_smem);
 void launch_form_bq(const Shared &sh, const TcPlan &tp, cudaStream_t s);
 void launch_btp(const Shared &sh, const TcPlan &tp, cudaStream_t s);
 void launch_qn_refresh(const Shared &sh, const TcPlan &tp, cudaStream_t s);
+void launch_colnorm_reduce(const Shared &sh, const int4 *ctiles, int32_t n_ctiles, float eps_col, cudaStream_t s);
+void launch_colnorm_scale(const Shared &sh, const TcPlan &tp, cudaStream_t s);
 uint32_t orth_smem(int nstages, uint32_t stage_bytes);
 cudaError_t setup_orth_kernels(uint32_t smem);
 void launch_orth(const Shared &sh, const TcPlan &tp, bool gram, int pass, cudaStream_t s);
