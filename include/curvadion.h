@@ -153,6 +153,28 @@ dion_status dion_timing_enable(dion_plan *plan, int32_t max_steps);
 dion_status dion_timing_read(dion_plan *plan, int32_t cap, float *ms_out, const char **names_out,
                              int32_t *count_out, int32_t *steps_out);
 
+/* Limits of dion_buffer_norms_noalloc (its fixed device scratch is ~1 MB per GPU). */
+#define DION_NOALLOC_MAX_LAYERS 256
+#define DION_NOALLOC_MAX_TILES 65536
+
+/* Buffer step without any allocation, for callers that cannot call cudaMalloc (a framework
+ * whose allocator has reserved the device memory up front, or a latency-critical loop where
+ * cudaMalloc/cudaFree would synchronize the device).  The paper has no counterpart: it is the
+ * buffer line B = M + G (written back into M, as dion_step does) plus ||B|| and ||M_{t-1}||
+ * per layer -- the inputs of Algorithm 2's RMMC -- without a plan.
+ * Only m, n, M, ldm, G, ldg and g_dtype of each layer are used (same rules as dion_layer).
+ * norm_b_out, norm_m_out: device double[num_layers], written.  Enqueued on `stream`.
+ * Scratch: a fixed device array inside this library (layer table + per-tile partial sums),
+ * held by every GPU that loads the library until the process exits.  Every call overwrites
+ * what it reads, so nothing needs clearing, but calls that overlap on the GPU (two streams,
+ * or two host threads) share that array and race: serialize them.  The first call on each
+ * device looks up the array's device address (cudaGetSymbolAddress); make that first call
+ * before any stream capture.  Allocates no device or host memory.
+ * Errors: INVALID_ARG, ALIGNMENT, UNSUPPORTED (num_layers > DION_NOALLOC_MAX_LAYERS, or the
+ * layers need more than DION_NOALLOC_MAX_TILES tiles of ~64K elements), CUDA. */
+dion_status dion_buffer_norms_noalloc(const dion_layer *layers, int32_t num_layers, double *norm_b_out,
+                                      double *norm_m_out, void *stream);
+
 /* Frees the plan's workspace (synchronizes the device first).  NULL is a no-op. */
 void dion_plan_destroy(dion_plan *plan);
 

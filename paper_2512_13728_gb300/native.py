@@ -36,8 +36,11 @@ DION_MAX_RANK = 512
 
 # Every function declared in include/curvadion.h.
 EXPORTED = ("dion_plan_create", "dion_step", "dion_get_device_status", "dion_plan_refresh", "dion_step_launch_count",
-            "dion_timing_enable", "dion_timing_read", "dion_plan_destroy", "dion_status_string",
-            "dion_abi_version")
+            "dion_timing_enable", "dion_timing_read", "dion_buffer_norms_noalloc", "dion_plan_destroy",
+            "dion_status_string", "dion_abi_version")
+
+DION_NOALLOC_MAX_LAYERS = 256
+DION_NOALLOC_MAX_TILES = 65536
 
 
 class dion_layer(C.Structure):
@@ -93,6 +96,8 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     lib.dion_timing_read.argtypes = [P, C.c_int32, C.POINTER(C.c_float), C.POINTER(C.c_char_p),
                                      C.POINTER(C.c_int32), C.POINTER(C.c_int32)]
     lib.dion_timing_read.restype = C.c_int
+    lib.dion_buffer_norms_noalloc.argtypes = [C.POINTER(dion_layer), C.c_int32, P, P, P]
+    lib.dion_buffer_norms_noalloc.restype = C.c_int
     lib.dion_plan_destroy.argtypes = [P]
     lib.dion_plan_destroy.restype = None
     lib.dion_status_string.argtypes = [C.c_int]
@@ -166,6 +171,15 @@ def dion_timing_read(plan: int):
         raise DionError(st, "dion_timing_read")
     n = min(cap, count.value)
     return steps.value, [((names[i] or b"").decode(), float(ms[i])) for i in range(n)]
+
+
+def dion_buffer_norms_noalloc(layers, norm_b_out: int, norm_m_out: int, stream: int = 0) -> None:
+    """B = M + G in place and ||B||, ||M_{t-1}|| per layer, without allocating (see the header)."""
+    arr = (dion_layer * max(len(layers), 1))(*layers)
+    st = load().dion_buffer_norms_noalloc(arr, len(layers), C.c_void_p(norm_b_out), C.c_void_p(norm_m_out),
+                                          C.c_void_p(stream) if stream else None)
+    if st != DION_OK:
+        raise DionError(st, "dion_buffer_norms_noalloc")
 
 
 def dion_plan_destroy(plan: int) -> None:
