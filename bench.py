@@ -65,9 +65,11 @@ def kernel_work(name: str, w, prec: str):
     mr2 = sum(m * r * r for (m, n), r in zip(w.shapes, ranks))
     r3 = sum(r ** 3 for r in ranks)
     nr = sum(n * r for (m, n), r in zip(w.shapes, ranks))
+    mr = sum(m * r for (m, n), r in zip(w.shapes, ranks))
+    bh = 2 if prec == "bf16" else 0  # the bf16 copy of B the tensor-core contractions read
     table = {
         # CUDA-core path
-        "form_b": ("hbm", mn * (4 + gsz + 4), "B"),
+        "form_b": ("hbm", mn * (4 + gsz + 4 + bh), "B"),
         "gemm_bq": ("alu", 2 * mnr, "flop"),
         "gemm_gram": ("alu", 2 * mr2, "flop"),
         "chol_inv": ("alu", 2 * r3 / 3, "flop"),
@@ -77,8 +79,8 @@ def kernel_work(name: str, w, prec: str):
         "update": ("alu", 4 * mnr, "flop") if prec == "fp32" else ("hbm", mn * 16, "B"),
         "local": ("hbm", 0, "B"),
         # tensor-core path
-        "tc_form_bq": ("hbm", mn * (4 + gsz + 4), "B"),
-        "tc_btp": ("hbm", mn * 4, "B"),
+        "tc_bq": ("hbm", mn * 2 + nr * 2 + mr * 8, "B"),  # Bh, bf16 Q; P and P^T fp32
+        "tc_btp": ("hbm", mn * 2 + mr * 2 + nr * 6, "B"),  # Bh, bf16 P; R fp32 and bf16
         "tc_update": ("hbm", mn * 16, "B"),
         "tc_gram": ("tensor", 2 * mr2, "flop"),
         "tc_trsm": ("tensor", 2 * mr2, "flop"),
@@ -90,7 +92,7 @@ def step_bytes(w, prec):
     """Bytes one synchronized step moves by design (the planned passes), and the compulsory floor."""
     gsz = 2 if w.g_dtype == "bf16" else 4
     mn = sum(m * n for m, n in w.shapes)
-    planned = mn * ((4 + gsz + 4) + 4 + 16)
+    planned = mn * ((4 + gsz + 4) + 4 + 4 + 16) if prec == "fp32" else mn * ((4 + gsz + 4 + 2) + 2 + 2 + 16)
     compulsory = mn * (4 + gsz + 4 + 4 + 4)  # read M, G, X; write M, X
     return planned, compulsory
 

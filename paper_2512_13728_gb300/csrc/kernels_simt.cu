@@ -37,7 +37,7 @@ __device__ __forceinline__ float load_g1(const void *G, int64_t off) {
   return static_cast<const float *>(G)[off];
 }
 
-template <int GT>
+template <int GT, bool HAS_BH>
 __device__ void form_b_tile(const DevLayer &L, int64_t row0, int64_t nrows, float sb[4], float sm[4]) {
   const int64_t n = L.n, n4 = n >> 2;
   for (int64_t rr = 0; rr < nrows; ++rr) {
@@ -54,6 +54,13 @@ __device__ void form_b_tile(const DevLayer &L, int64_t row0, int64_t nrows, floa
       sb[0] = fmaf(m.x, m.x, sb[0]); sb[1] = fmaf(m.y, m.y, sb[1]);
       sb[2] = fmaf(m.z, m.z, sb[2]); sb[3] = fmaf(m.w, m.w, sb[3]);
       *reinterpret_cast<float4 *>(Mrow + 4 * c4) = m;
+      if (HAS_BH) {  // bf16 copy of B (operand of the tensor-core contractions)
+        const __nv_bfloat162 h01 = __floats2bfloat162_rn(m.x, m.y), h23 = __floats2bfloat162_rn(m.z, m.w);
+        uint2 hv;
+        hv.x = *reinterpret_cast<const uint32_t *>(&h01);
+        hv.y = *reinterpret_cast<const uint32_t *>(&h23);
+        *reinterpret_cast<uint2 *>(L.Bh + i * L.ldbh + 4 * c4) = hv;
+      }
     }
     for (int64_t c = 4 * n4 + threadIdx.x; c < n; c += kRowThreads) {
       const float mo = Mrow[c];
@@ -61,6 +68,7 @@ __device__ void form_b_tile(const DevLayer &L, int64_t row0, int64_t nrows, floa
       sm[0] = fmaf(mo, mo, sm[0]);
       sb[0] = fmaf(b, b, sb[0]);
       Mrow[c] = b;
+      if (HAS_BH) L.Bh[i * L.ldbh + c] = __float2bfloat16_rn(b);
     }
   }
 }
@@ -70,8 +78,13 @@ __global__ void __launch_bounds__(kRowThreads) form_b_kernel(Shared sh, const in
   const int4 t = tiles[blockIdx.x];
   const DevLayer &L = sh.layers[t.x];
   float sb[4] = {0.f, 0.f, 0.f, 0.f}, sm[4] = {0.f, 0.f, 0.f, 0.f};
-  if (L.g_dtype == DT_BF16) form_b_tile<DT_BF16>(L, t.y, t.z, sb, sm);
-  else form_b_tile<DT_FP32>(L, t.y, t.z, sb, sm);
+  if (L.Bh != nullptr) {
+    if (L.g_dtype == DT_BF16) form_b_tile<DT_BF16, true>(L, t.y, t.z, sb, sm);
+    else form_b_tile<DT_FP32, true>(L, t.y, t.z, sb, sm);
+  } else {
+    if (L.g_dtype == DT_BF16) form_b_tile<DT_BF16, false>(L, t.y, t.z, sb, sm);
+    else form_b_tile<DT_FP32, false>(L, t.y, t.z, sb, sm);
+  }
   const double b = block_sum<kRowThreads>(((double)sb[0] + sb[1]) + ((double)sb[2] + sb[3]), red);
   const double mo = block_sum<kRowThreads>(((double)sm[0] + sm[1]) + ((double)sm[2] + sm[3]), red);
   if (threadIdx.x == 0) {

@@ -195,8 +195,7 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
   std::vector<int4> gt[kSets];
   const size_t o_layers = cv.take<DevLayer>(std::max(num_layers, 1));
   const size_t o_active = cv.take<uint8_t>(std::max(num_layers, 1));
-  const size_t nslots = std::max<size_t>(bt.size(), precision == DION_PREC_FP32 ? 0 : tc::norm_slots(layers, num_layers));
-  const size_t o_bpart = cv.take<double>(2 * std::max<size_t>(nslots, 1));
+  const size_t o_bpart = cv.take<double>(2 * std::max<size_t>(bt.size(), 1));
   const size_t o_upart = cv.take<double>(std::max<size_t>(ut.size(), 1));
   const size_t o_nmb = cv.take<double>(std::max(num_layers, 1));
   const size_t o_nb = cv.take<double>(std::max(num_layers, 1));

@@ -245,7 +245,6 @@ __global__ void __launch_bounds__(U_THREADS, 1)
 
 // ========================================================================= host side ===
 namespace {
-size_t bq_tiles(int64_t m) { return (size_t)((m + 127) / 128); }
 
 // Longest-processing-time-first assignment of tiles to at most `max_grid` persistent CTAs.
 Schedule lpt(const std::vector<int4> &tiles, const std::vector<double> &cost, int max_grid) {
@@ -277,12 +276,6 @@ Schedule lpt(const std::vector<int4> &tiles, const std::vector<double> &cost, in
 }
 }  // namespace
 
-size_t norm_slots(const dion_layer *layers, int32_t L) {
-  size_t n = 0;
-  for (int32_t l = 0; l < L; ++l) n += 8 * bq_tiles(layers[l].m);
-  return n;
-}
-
 dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int num_sms, size_t start,
                    TcLayout *out) {
   if (precision != DION_PREC_BF16) return DION_ERR_UNSUPPORTED;
@@ -303,7 +296,6 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
   lo.o_pt.resize(L);
   lo.o_colsq.resize(L);
   lo.o_colinv.resize(L);
-  int32_t fslot = 0;
   for (int32_t l = 0; l < L; ++l) {
     const dion_layer &ly = layers[l];
     const int64_t ldp = (ly.r + 7) / 8 * 8, ldbh = (ly.n + 7) / 8 * 8;
@@ -328,7 +320,7 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
     const int64_t qrow = std::max<int64_t>(1, std::min<int64_t>(ly.n, 16384 / ly.r));
     for (int64_t r0 = 0; r0 < ly.n; r0 += qrow)
       lo.qtiles.push_back(make_int4(l, (int)r0, (int)std::min(qrow, ly.n - r0), 0));
-    for (int64_t mb = 0; mb < (ly.m + 127) / 128; ++mb) lo.ftiles.push_back(make_int4(l, (int)mb, 0, fslot++));
+    for (int64_t mb = 0; mb < (ly.m + 127) / 128; ++mb) lo.ftiles.push_back(make_int4(l, (int)mb, 0, 0));
     for (int64_t nb = 0; nb < (ly.n + 127) / 128; ++nb) lo.rtiles.push_back(make_int4(l, (int)nb, 0, 0));
   }
   // per-tile cost ~ K-loop length (+ a constant for the epilogue), LPT over the SMs
@@ -362,7 +354,6 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
 }
 
 void bind(const TcLayout &lo, char *base, DevLayer *dl, int32_t L, TcPlan *tp) {
-  int32_t fslot = 0;
   for (int32_t l = 0; l < L; ++l) {
     dl[l].P_hi = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_phi[l]);
     dl[l].R_hi = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_rhi[l]);
@@ -375,11 +366,6 @@ void bind(const TcLayout &lo, char *base, DevLayer *dl, int32_t L, TcPlan *tp) {
     dl[l].colsq = reinterpret_cast<double *>(base + lo.o_colsq[l]);
     dl[l].colinv = reinterpret_cast<float *>(base + lo.o_colinv[l]);
     dl[l].rtile_cnt = (int32_t)((dl[l].n + 127) / 128);
-    // norm partials: 8 slots (one per producer warp) per 128-row tile of the fused B Q kernel
-    const int32_t tiles = (int32_t)bq_tiles(dl[l].m);
-    dl[l].bpart_off = 8 * fslot;
-    dl[l].bpart_cnt = 8 * tiles;
-    fslot += tiles;
     dl[l].upart_off = -1;
   }
   int32_t cur = -1;
@@ -436,6 +422,7 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
                     encode_bf16_2d(&m.Qn_mn, d.Qn_hi, d.r, d.n, p16, 64, 64) &&
                     encode_bf16_2d(&m.P_mn, d.P_hi, d.r, d.m, p16, 64, 64) &&
                     encode_bf16_2d(&m.Bh_mn, d.Bh, d.n, d.m, (uint64_t)d.ldbh * 2, 64, 64) &&
+                    encode_bf16_2d(&m.Bh_k, d.Bh, d.n, d.m, (uint64_t)d.ldbh * 2, 64, 128) &&
                     encode_f32_2d(&m.Praw, d.P_raw, d.r, d.m, p32, 32, 128) &&
                     encode_f32_2d(&m.Rst, d.R, d.r, d.n, p32, 32, 128) &&
                     encode_f32_2d(&m.Pf, d.P, d.r, d.m, p32, 32, 128) &&
@@ -491,7 +478,7 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   tp->num_sms = sms;
-  tp->launches = 18;
+  tp->launches = 19;
   return e;
 }
 
@@ -501,10 +488,12 @@ void refresh(const TcPlan &tp, const Shared &sh, cudaStream_t s) { launch_qn_ref
 
 void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, const int4 *btiles,
           int32_t n_btiles, const int4 *ctiles, int32_t n_ctiles, size_t chol_smem, cudaStream_t s) {
-  launch_form_bq(sh, tp, s);  // B = M + G, ||B||, ||M_{t-1}||, P = B Q_{t-1}
-  tick(p, s, "tc_form_bq");
+  launch_form_b(sh, btiles, n_btiles, s);  // B = M + G (and its bf16 copy), ||B||, ||M_{t-1}||
+  tick(p, s, "form_b");
   launch_gate(sh, a, s);
   tick(p, s, "gate");
+  launch_form_bq(sh, tp, s);  // P = B Q_{t-1} on the layers that take the Dion branch
+  tick(p, s, "tc_bq");
   static const char *kGram[3] = {"tc_gram0", "tc_gram1", "tc_gram2"};
   static const char *kChol[3] = {"chol_inv0", "chol_inv1", "chol_inv2"};
   static const char *kTrsm[3] = {"tc_trsm0", "tc_trsm1", "tc_trsm2"};

@@ -22,6 +22,7 @@ struct LayerMaps {
   CUtensorMap Qn_mn;  // n x r bf16:  box {64, 64}   B Q: MN-major B operand (K = n)
   CUtensorMap P_mn;   // m x r bf16:  box {64, 64}   B^T P: MN-major B operand (K = m)
   CUtensorMap Bh_mn;  // m x n bf16:  box {64, 64}   B^T P: MN-major A operand (K = m)
+  CUtensorMap Bh_k;   // m x n bf16:  box {64, 128}  B Q: K-major A operand (K = n)
   CUtensorMap Praw;   // m x r fp32:  box {32, 128}  B Q output; TRSM A operand / output
   CUtensorMap Rst;    // n x r fp32:  box {32, 128}  B^T P: output store
   CUtensorMap Pf;     // m x r fp32 (P):      box {32, 128}  TRSM A operand / output
@@ -108,7 +109,6 @@ void destroy(TcPlan *tp);
 // dion_plan_refresh).
 void refresh(const TcPlan &tp, const Shared &sh, cudaStream_t s);
 // Number of B Q tiles (one norm-partial slot each) the layout needs for these layers.
-size_t norm_slots(const dion_layer *layers, int32_t L);
 
 }  // namespace tc
 }  // namespace cd
