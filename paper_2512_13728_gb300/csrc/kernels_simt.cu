@@ -7,6 +7,7 @@
 // decision without a host round trip.
 #include "common.cuh"
 
+#include <algorithm>
 #include <cmath>
 
 namespace cd {
@@ -249,113 +250,219 @@ void launch_gemm(const Shared &sh, const GemmProblem *probs, const int4 *tiles, 
 // u = 2^-24; the layer is then marked and a third pass runs.  Every pass multiplies P by an
 // upper-triangular matrix with positive diagonal, so the final P is the Q factor of the
 // thin QR of the original P with a positive-diagonal triangular factor.
-// One CTA per layer (r <= 512): right-looking blocked Cholesky with 32-wide block columns,
-// then L^{-1} block row by block row.  S and L^{-1} live in global memory (L2-resident);
-// diagonal blocks, panels and partial products are staged in shared memory.  Only the lower
-// triangle of S is overwritten, so a retry rebuilds S from its upper triangle and the saved
-// diagonal.  If the shifted retry also fails, DION_ERR_BREAKDOWN is set and L^{-1} = 0 for
-// the layer, so its P, R and Q become 0, M becomes B and X is unchanged (no NaN written).
+//
+// One CTA per layer (r <= 512), 16 warps.  S (full, symmetric) is only read; the factor and
+// its inverse are built in place in the L^{-1} buffer W by one right-looking sweep over
+// 32-wide block columns k (k0 = 32 k).  Before step k, for rows i >= k0:
+//   W[i][j], j >= k0 : the Schur complement S - L[:, :k0] L[:, :k0]^T (lower triangle),
+//   W[i][j], j <  k0 : U[i][j] = -sum_{K < k} L[i, K] L^{-1}[K, j],
+// and rows above k0 hold their final L^{-1}.  Step k:
+//   warp 0     factors the 32 x 32 diagonal block in registers (shuffles) and inverts it
+//              (D_k = L_kk^{-1}), while warps 1..15 load the rest of block row k's U and the
+//              panel rows below the block;
+//   warps 1..  finish block row k: L^{-1}[k, :k0] = D_k U[k, :k0], and form the panel
+//              L[i, k] = A[i, k] D_k^T of every row below;
+//   all        with Y = [L^{-1}[k, :k0 + 32] | L[k0 + 32 :, k]^T] (32 x r, shared memory),
+//              apply W[i][j] -= sum_c Y[c][i] Y[c][j] to every row i below the block and every
+//              j <= i: for j >= k0 + 32 this is the trailing Cholesky update, for j < k0 + 32
+//              the accumulation of U (whose columns k0 .. k0 + 31 start from zero here).
+// The update is a rank-32 outer product over a lower trapezoid, 8 x 8 register tiles fed by
+// 128-bit shared loads, so the factorization and the inverse (r^3 / 3 multiply-adds in all)
+// run at the FMA rate instead of being serialized behind per-column solves.  A retry starts
+// again from S with its diagonal shifted.  If the shifted retry also fails, DION_ERR_BREAKDOWN
+// is set and L^{-1} = 0 for the layer, so its P, R and Q become 0, M becomes B and X is
+// unchanged (no NaN written).
 constexpr int CB = 32, CBP = CB + 1, kCholThreads = 512;
-constexpr int DION_MAX_RANK_PAD = 512;  // diag0 slot: r <= 512
 
-__device__ __forceinline__ int64_t tri_row(int64_t p) {
-  // largest b with b (b + 1) / 2 <= p
-  int64_t b = (int64_t)((sqrt(8.0 * (double)p + 1.0) - 1.0) * 0.5);
-  while ((b + 1) * (b + 2) / 2 <= p) ++b;
-  while (b * (b + 1) / 2 > p) --b;
+// Row-tile index of tile p in a lower trapezoid whose row tile b holds c1 + b tiles: the
+// largest b with b c1 + b (b - 1) / 2 <= p.
+// fp32 estimate (p < 2^21 here), corrected exactly in integers.
+__device__ __forceinline__ int trap_row(int p, int c1) {
+  const float bq = 2.f * (float)c1 - 1.f;
+  int b = (int)((sqrtf(bq * bq + 8.f * (float)p) - bq) * 0.5f);
+  if (b < 0) b = 0;
+  while ((b + 1) * c1 + (b + 1) * b / 2 <= p) ++b;
+  while (b > 0 && b * c1 + b * (b - 1) / 2 > p) --b;
   return b;
 }
 
-// Factors the lower triangle of S (r x r, row-major) in place.  Returns false (uniformly over
-// the block) on a pivot <= 0 or non-finite.  Smem: D (CB x CBP), Pn (r x CBP).
-__device__ bool cholesky_blocked(float *S, int r, int64_t ls, float *D, float *Pn, int *bad) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (tid == 0) *bad = 0;
-  __syncthreads();
-  for (int k0 = 0; k0 < r; k0 += CB) {
-    const int nb = min(CB, r - k0);
-    for (int e = tid; e < CB * CB; e += kCholThreads) {
-      const int i = e / CB, j = e % CB;
-      float v;
-      if (i < nb && j < nb) v = (j <= i) ? S[(int64_t)(k0 + i) * ls + k0 + j] : 0.f;
-      else v = (i == j) ? 1.f : 0.f;  // identity padding of a short last block
-      D[i * CBP + j] = v;
+// Column c of Y lives at ysw(c): bit 2 flips when bit 5 is set, so the two 16-byte halves of
+// an 8-column group swap in every other 32-column stretch.  Eight consecutive groups read by
+// one quarter-warp then fall on distinct banks.
+__device__ __forceinline__ int ysw(int c) { return c ^ ((c >> 3) & 4); }
+__device__ __forceinline__ void load8y(const float *row, int c0, float w[8]) {  // c0 % 8 == 0
+  const int s = (c0 >> 3) & 4;
+  const float4 a = *reinterpret_cast<const float4 *>(row + c0 + s), b = *reinterpret_cast<const float4 *>(row + c0 + (s ^ 4));
+  w[0] = a.x; w[1] = a.y; w[2] = a.z; w[3] = a.w; w[4] = b.x; w[5] = b.y; w[6] = b.z; w[7] = b.w;
+}
+
+__device__ __forceinline__ void load8(const float *p, float w[8]) {
+  const float4 a = *reinterpret_cast<const float4 *>(p), b = *reinterpret_cast<const float4 *>(p + 4);
+  w[0] = a.x; w[1] = a.y; w[2] = a.z; w[3] = a.w; w[4] = b.x; w[5] = b.y; w[6] = b.z; w[7] = b.w;
+}
+__device__ __forceinline__ void store8(float *p, const float w[8]) {
+  *reinterpret_cast<float4 *>(p) = make_float4(w[0], w[1], w[2], w[3]);
+  *reinterpret_cast<float4 *>(p + 4) = make_float4(w[4], w[5], w[6], w[7]);
+}
+
+// The 32 x 32 diagonal-block kernels below are unrolled through template recursion so that
+// every register array is indexed by constants (no local-memory copies).
+// Column J of the Cholesky factor of a 32 x 32 block held one row per lane.
+template <int J>
+__device__ __forceinline__ void chol32_col(float (&v)[CB], float *rd, int lane, bool &ok) {
+  if constexpr (J < CB) {
+    const float piv = __shfl_sync(0xffffffffu, v[J], J);
+    ok = ok && (piv > 0.f) && (piv < INFINITY);  // uniform: every lane sees the same pivot
+    const float rs = rsqrtf(piv), sq = piv * rs;
+    v[J] = (lane == J) ? sq : (lane > J ? v[J] * rs : 0.f);
+    if (lane == 0) rd[J] = rs;
+#pragma unroll
+    for (int k = J + 1; k < CB; ++k) {
+      const float lkj = __shfl_sync(0xffffffffu, v[J], k);
+      if (lane >= k) v[k] = fmaf(-v[J], lkj, v[k]);
     }
-    __syncthreads();
+    chol32_col<J + 1>(v, rd, lane, ok);
+  }
+}
+
+// Row I of the forward substitution L x = e_lane (lane c computes column c of L^{-1}).
+template <int I>
+__device__ __forceinline__ void trinv32_row(float (&x)[CB], const float *D, const float *rd, int lane) {
+  if constexpr (I < CB) {
+    float a = (I == lane) ? 1.f : 0.f;
+#pragma unroll
+    for (int k = 0; k < I; ++k) a = fmaf(-D[I * CBP + k], x[k], a);
+    x[I] = a * rd[I];
+    trinv32_row<I + 1>(x, D, rd, lane);
+  }
+}
+
+// v <- T v for a lower-triangular 32 x 32 T (row-major, stride CB), in place from the bottom.
+template <int C>
+__device__ __forceinline__ void trmv32(float (&v)[CB], const float *T) {
+  if constexpr (C >= 0) {
+    float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+    for (int c2 = 0; c2 <= C; c2 += 2) {
+      a0 = fmaf(T[C * CB + c2], v[c2], a0);
+      if (c2 + 1 <= C) a1 = fmaf(T[C * CB + c2 + 1], v[c2 + 1], a1);
+    }
+    v[C] = a0 + a1;
+    trmv32<C - 1>(v, T);
+  }
+}
+
+// W <- L^{-1} with L L^T = S + shift I (lower triangle of S read).  Returns false, uniformly
+// over the block, on a pivot that is not positive and finite.  Shared memory: D (CB x CBP),
+// DI (CB x CB), rd (CB reciprocal pivots), Y (CB x ldy, ldy >= r rounded up to 8, columns
+// >= r zero).
+__device__ bool chol_inverse(const float *__restrict__ S, float *__restrict__ W, int r, int64_t ls, float shift,
+                             float *D, float *DI, float *rd, float *Y, int ldy, int *bad) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, q = tid - 32;
+  for (int k0 = 0; k0 < r; k0 += CB) {
+    const int nb = min(CB, r - k0), R0 = k0 + nb, t = r - R0;
+    const float *src = (k0 == 0) ? S : W;
+    const float dshift = (k0 == 0) ? shift : 0.f;
+    float v[CB];
     if (warp == 0) {
-      for (int j = 0; j < CB; ++j) {
-        const float djj = D[j * CBP + j];
-        if (!(djj > 0.f) || !isfinite(djj)) {
-          if (lane == 0) *bad = 1;
-          break;  // uniform across the warp: every lane read the same djj
-        }
-        const float sq = sqrtf(djj);
-        __syncwarp();
-        if (lane == j) D[j * CBP + j] = sq;
-        if (lane > j) D[lane * CBP + j] /= sq;
-        __syncwarp();
-        if (lane > j) {
-          const float lij = D[lane * CBP + j];
-          for (int k = j + 1; k <= lane; ++k) D[lane * CBP + k] -= lij * D[k * CBP + j];
-        }
-        __syncwarp();
+      // ---- diagonal block: lane i holds row k0 + i (identity padding below a short block)
+      const int64_t row = k0 + lane;
+      if (nb == CB) {
+        load8(src + row * ls + k0, v);
+        load8(src + row * ls + k0 + 8, v + 8);
+        load8(src + row * ls + k0 + 16, v + 16);
+        load8(src + row * ls + k0 + 24, v + 24);
+      } else {
+#pragma unroll
+        for (int j = 0; j < CB; ++j) v[j] = (lane < nb && j < nb) ? src[row * ls + k0 + j] : 0.f;
       }
+#pragma unroll
+      for (int j = 0; j < CB; ++j) {
+        if (j > lane) v[j] = 0.f;
+        if (j == lane) v[j] = (lane < nb) ? v[j] + dshift : 1.f;
+      }
+      bool ok = true;
+      chol32_col<0>(v, rd, lane, ok);
+#pragma unroll
+      for (int j = 0; j < CB; ++j) D[lane * CBP + j] = v[j];
+      __syncwarp();
+      // lane c: column c of D_k = L_kk^{-1} by forward substitution on e_c
+      trinv32_row<0>(v, D, rd, lane);
+#pragma unroll
+      for (int i = 0; i < CB; ++i) DI[i * CB + lane] = v[i];
+      if (lane == 0) *bad = ok ? 0 : 1;
+    } else if (q < k0) {
+      // ---- column q of U[k, :k0]
+#pragma unroll
+      for (int c = 0; c < CB; ++c) v[c] = (c < nb) ? W[(int64_t)(k0 + c) * ls + q] : 0.f;
+    } else if (q < k0 + t) {
+      // ---- panel row R0 + q - k0 (a full block: nb = 32 whenever rows remain below it)
+      const float *p = src + (int64_t)(R0 + q - k0) * ls + k0;
+      load8(p, v);
+      load8(p + 8, v + 8);
+      load8(p + 16, v + 16);
+      load8(p + 24, v + 24);
     }
     __syncthreads();
     if (*bad) return false;
-    for (int e = tid; e < nb * nb; e += kCholThreads) {
-      const int i = e / nb, j = e % nb;
-      if (j <= i) S[(int64_t)(k0 + i) * ls + k0 + j] = D[i * CBP + j];
-    }
-    // panel: rows below the block solve x L11^T = s
-    const int t = r - k0 - nb;
-    for (int ii = tid; ii < t; ii += kCholThreads) {
-      const int64_t row = (int64_t)(k0 + nb + ii) * ls + k0;
-      float x[CB];
+    if (warp > 0 && q < k0 + t) {
+      // v <- D_k v (lower triangular, in place from the bottom): the finished L^{-1}[k, q]
+      // for a U column, the panel entries L[row, k0 ..] = A[row, k0 ..] D_k^T for a panel row
+      trmv32<CB - 1>(v, DI);
+      if (q < k0) {
 #pragma unroll
-      for (int j = 0; j < CB; ++j) x[j] = (j < nb) ? S[row + j] : 0.f;
+        for (int c = 0; c < CB; ++c) {
+          if (c < nb) W[(int64_t)(k0 + c) * ls + q] = v[c];
+          Y[c * ldy + ysw(q)] = v[c];
+        }
+      } else {
 #pragma unroll
-      for (int j = 0; j < CB; ++j) {
-        float v = x[j];
-#pragma unroll
-        for (int k = 0; k < j; ++k) v -= x[k] * D[j * CBP + k];
-        x[j] = v / D[j * CBP + j];
-      }
-#pragma unroll
-      for (int j = 0; j < CB; ++j) {
-        Pn[ii * CBP + j] = x[j];
-        if (j < nb) S[row + j] = x[j];
+        for (int c = 0; c < CB; ++c) Y[c * ldy + ysw(R0 + q - k0)] = v[c];
       }
     }
+    // block row k right of k0: D_k on the diagonal block, zeros beyond
+    for (int i = warp; i < nb; i += kCholThreads / 32)
+      for (int c = lane; c < r - k0; c += 32) W[(int64_t)(k0 + i) * ls + k0 + c] = (c <= i) ? DI[i * CB + c] : 0.f;
+    if (t > 0)
+      for (int e = tid; e < CB * CB; e += kCholThreads) Y[(e >> 5) * ldy + ysw(k0 + (e & 31))] = DI[e];
     __syncthreads();
-    // trailing update of the lower triangle: S22 -= L21 L21^T, in 4 x 4 micro tiles
-    const int64_t nbt = (t + 3) / 4, pairs = nbt * (nbt + 1) / 2;
-    for (int64_t pidx = tid; pidx < pairs; pidx += kCholThreads) {
-      const int64_t bi = tri_row(pidx), bj = pidx - bi * (bi + 1) / 2;
-      float acc[4][4] = {};
-#pragma unroll 8
-      for (int k = 0; k < CB; ++k) {
-        float a[4], b[4];
+    if (t > 0) {
+      // ---- rank-32 update of rows R0 .. r - 1, columns 0 .. i, in 8 x 8 tiles
+      const int c1 = R0 / 8 + 1, nbt = (t + 7) / 8;
+      const int ntiles = nbt * c1 + nbt * (nbt - 1) / 2;
+      for (int p = tid; p < ntiles; p += kCholThreads) {
+        const int bi = trap_row(p, c1), bj = p - (bi * c1 + bi * (bi - 1) / 2);
+        const int i0 = R0 + 8 * bi, j0 = 8 * bj;
+        // the tile starts from the current W (one load latency per tile), or from zero for
+        // the U columns of block k, which start here
+        const bool fresh = (j0 >= k0 && j0 < R0);
+        float acc[8][8];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int64_t ri = bi * 4 + u, rj = bj * 4 + u;
-          a[u] = (ri < t) ? Pn[ri * CBP + k] : 0.f;
-          b[u] = (rj < t) ? Pn[rj * CBP + k] : 0.f;
+        for (int u = 0; u < 8; ++u) {
+          const int row = i0 + u;
+          if (fresh || row >= r) {
+#pragma unroll
+            for (int w = 0; w < 8; ++w) acc[u][w] = 0.f;
+          } else {
+            load8(src + (int64_t)row * ls + j0, acc[u]);
+#pragma unroll
+            for (int w = 0; w < 8; ++w)
+              if (j0 + w == row) acc[u][w] += dshift;
+          }
+        }
+#pragma unroll 1
+        for (int c = 0; c < CB; ++c) {
+          float a[8], b[8];
+          load8y(Y + c * ldy, i0, a);
+          load8y(Y + c * ldy, j0, b);
+#pragma unroll
+          for (int u = 0; u < 8; ++u)
+#pragma unroll
+            for (int w = 0; w < 8; ++w) acc[u][w] = fmaf(-a[u], b[w], acc[u][w]);
         }
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
-#pragma unroll
-          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(a[u], b[v], acc[u][v]);
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int64_t ri = bi * 4 + u;
-        if (ri >= t) continue;
-#pragma unroll
-        for (int v = 0; v < 4; ++v) {
-          const int64_t rj = bj * 4 + v;
-          if (rj < t && rj <= ri) S[(k0 + nb + ri) * ls + k0 + nb + rj] -= acc[u][v];
-        }
+        for (int u = 0; u < 8; ++u)
+          if (i0 + u < r) store8(W + (int64_t)(i0 + u) * ls + j0, acc[u]);
       }
     }
     __syncthreads();
@@ -364,137 +471,114 @@ __device__ bool cholesky_blocked(float *S, int r, int64_t ls, float *D, float *P
 }
 
 // pass 0 and 1: every active layer; pass 2: only layers marked by a shifted retry.
-// Passes 1 and 2 factor the Gram matrix of an already nearly orthonormal X: when 1.5 times a
-// power-iteration estimate of ||S - I||_2 is below near_identity, the factor of S = I + E is
-// taken to first order, L = I + F with F = strictly-lower(E) + diag(E) / 2 and
-// L^{-1} = I - F; the resulting X L^{-T} is then orthonormal up to O(||E||_2^2).
-__global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int pass, float near_identity) {
+// Passes 1 and 2 factor the Gram matrix of an already nearly orthonormal X.  With E = S - I,
+// when 1.5 times a bound on ||E||_2 is below near_identity, the factor of S = I + E is taken
+// to first order, L = I + F with F = strictly-lower(E) + diag(E) / 2 and L^{-1} = I - F; the
+// resulting X L^{-T} is then orthonormal up to O(||E||_2^2).  The bound is ||E||_F when that
+// is small enough, else a power-iteration estimate of ||E||_2.
+__global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, int pass, float near_identity) {
   const int l = blockIdx.x;
   if (!sh.active[l]) return;
   if (pass == 2 && !sh.orth_shifted[l]) return;
   const DevLayer &Ly = sh.layers[l];
   const int r = (int)Ly.r;
-  const int64_t ls = Ly.ldp;  // leading dimension of S and L^{-1}
-  float *S = Ly.S;
+  const int64_t ls = Ly.ldp;  // leading dimension of S and L^{-1} (a multiple of 8)
+  const float *S = Ly.S;
   float *Li = Ly.Linv;
-  extern __shared__ float smem[];
-  float *D = smem;            // CB x CBP: diagonal block
-  float *DI = D + CB * CBP;   // CB x CBP: its inverse
-  float *diag0 = DI + CB * CBP;  // r: the diagonal of S before factorization
-  float *Pn = diag0 + DION_MAX_RANK_PAD;  // panel (r x CBP) or partial products (CB x r)
+  extern __shared__ __align__(16) float smem[];
+  float *D = smem;                 // CB x CBP
+  float *rd = D + CB * CBP;        // CB
+  float *DI = rd + 32;             // CB x CB (16-byte aligned)
+  float *Y = DI + CB * CB;         // CB x ldy
+  const int ldy = (r + 7) / 8 * 8;
   __shared__ int bad;
-  __shared__ double trace_s;
+  __shared__ double red[kCholThreads / 32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  // The Gram producers may write only the lower triangle: mirror it into the upper one, which
-  // the factorization never touches and the shifted retry restores the lower triangle from.
-  // 32 x 32 tiles transposed through a per-warp shared scratch (Pn holds 33 r floats, so r / 32
-  // warps have room), coalesced on both sides.
-  {
-    const int nt = (r + 31) / 32, nwm = min(kCholThreads / 32, r / 32);
-    if (nwm == 0) {
-      for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) {
-        const int64_t i = e / r, j = e % r;
-        if (j > i) S[i * ls + j] = S[j * ls + i];
-      }
-    } else if (warp < nwm) {
-      float *tb = Pn + warp * (32 * 33);
-      const int npairs = nt * (nt - 1) / 2;
-      for (int u = warp; u < npairs + nt; u += nwm) {
-        int bi, bj;  // upper tile (bi, bj), bj >= bi; u < npairs: off-diagonal, else the diagonal tile
-        if (u < npairs) {
-          bj = (int)tri_row(u) + 1;
-          bi = u - (bj - 1) * bj / 2;
-        } else {
-          bi = bj = u - npairs;
-        }
-        for (int y = 0; y < 32; ++y) {  // lower tile (bj, bi) -> scratch
-          const int gi = bj * 32 + y, gj = bi * 32 + lane;
-          tb[y * 33 + lane] = (gi < r && gj < r) ? S[(int64_t)gi * ls + gj] : 0.f;
-        }
-        __syncwarp();
-        for (int y = 0; y < 32; ++y) {  // upper tile (bi, bj) = transpose
-          const int gi = bi * 32 + y, gj = bj * 32 + lane;
-          if (gi < r && gj < r && gj > gi) S[(int64_t)gi * ls + gj] = tb[lane * 33 + y];
-        }
-        __syncwarp();
-      }
-    }
-    __syncthreads();
-  }
-  for (int i = tid; i < r; i += kCholThreads) diag0[i] = S[(int64_t)i * ls + i];
+
   if (pass >= 1) {
-    // ||E||_2 of E = S - I by 8 power iterations (one warp per row, coalesced row reads)
-    float *v = Pn, *wv = Pn + r;  // Pn holds at least 33 * r floats
-    __shared__ float wn[kCholThreads / 32];
+    // ||E||_F^2 from the lower triangle (E symmetric), fixed-order reduction
+    double fs = 0.0;
+    for (int i = warp; i < r; i += kCholThreads / 32) {
+      float a = 0.f;
+      for (int j = lane; j <= i; j += 32) {
+        const float e = S[(int64_t)i * ls + j] - (i == j ? 1.f : 0.f);
+        a = fmaf((j < i ? 2.f : 1.f) * e, e, a);
+      }
+      fs += (double)a;
+    }
+    fs = block_sum<kCholThreads>(fs, red);
     __shared__ float lam_s;
-    for (int i = tid; i < r; i += kCholThreads) v[i] = 1.f + 0.25f * __sinf(0.7f * (float)i);  // fixed start
+    if (tid == 0) lam_s = (float)sqrt(fs);
     __syncthreads();
-    float lam = 0.f;
-    for (int itp = 0; itp < 8; ++itp) {
-      for (int i = warp; i < r; i += kCholThreads / 32) {
-        float acc0 = 0.f, acc1 = 0.f;
-        int j = lane;
-        for (; j + 32 < r; j += 64) {
-          acc0 = fmaf(S[(int64_t)i * ls + j] - (i == j ? 1.f : 0.f), v[j], acc0);
-          acc1 = fmaf(S[(int64_t)i * ls + j + 32] - (i == j + 32 ? 1.f : 0.f), v[j + 32], acc1);
+    float lam = lam_s;
+    if (!(isfinite(lam) && 1.5f * lam < near_identity)) {
+      // ||E||_2 by 8 power iterations (one warp per row, coalesced row reads of the full S)
+      float *pv = Y, *wv = Y + ldy;
+      __shared__ float wn[kCholThreads / 32];
+      for (int i = tid; i < r; i += kCholThreads) pv[i] = 1.f + 0.25f * __sinf(0.7f * (float)i);  // fixed start
+      __syncthreads();
+      for (int itp = 0; itp < 8; ++itp) {
+        for (int i = warp; i < r; i += kCholThreads / 32) {
+          float acc0 = 0.f, acc1 = 0.f;
+          int j = lane;
+          for (; j + 32 < r; j += 64) {
+            acc0 = fmaf(S[(int64_t)i * ls + j] - (i == j ? 1.f : 0.f), pv[j], acc0);
+            acc1 = fmaf(S[(int64_t)i * ls + j + 32] - (i == j + 32 ? 1.f : 0.f), pv[j + 32], acc1);
+          }
+          if (j < r) acc0 = fmaf(S[(int64_t)i * ls + j] - (i == j ? 1.f : 0.f), pv[j], acc0);
+          float acc = acc0 + acc1;
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+          if (lane == 0) wv[i] = acc;
         }
-        if (j < r) acc0 = fmaf(S[(int64_t)i * ls + j] - (i == j ? 1.f : 0.f), v[j], acc0);
-        float acc = acc0 + acc1;
+        __syncthreads();
+        float pn = 0.f;
+        for (int i = tid; i < r; i += kCholThreads) pn = fmaf(wv[i], wv[i], pn);
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-        if (lane == 0) wv[i] = acc;
+        for (int o = 16; o > 0; o >>= 1) pn += __shfl_xor_sync(0xffffffffu, pn, o);
+        if (lane == 0) wn[warp] = pn;
+        __syncthreads();
+        if (tid == 0) {
+          float a = 0.f;
+          for (int w = 0; w < kCholThreads / 32; ++w) a += wn[w];
+          lam_s = a;  // ||E v||^2
+        }
+        __syncthreads();
+        const float nrm = sqrtf(lam_s);
+        lam = nrm;  // ||E v|| / ||v||: v has unit norm from the second iteration on
+        const float inv = (nrm > 0.f && isfinite(nrm)) ? 1.f / nrm : 0.f;
+        for (int i = tid; i < r; i += kCholThreads) pv[i] = wv[i] * inv;
+        __syncthreads();
+        if (itp == 0) lam = INFINITY;  // the first product uses an unnormalized start vector
       }
-      __syncthreads();
-      float pn = 0.f;
-      for (int i = tid; i < r; i += kCholThreads) pn = fmaf(wv[i], wv[i], pn);
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) pn += __shfl_xor_sync(0xffffffffu, pn, o);
-      if (lane == 0) wn[warp] = pn;
-      __syncthreads();
-      if (tid == 0) {
-        float a = 0.f;
-        for (int w = 0; w < kCholThreads / 32; ++w) a += wn[w];
-        lam_s = a;  // ||E v||^2
-      }
-      __syncthreads();
-      const float nrm = sqrtf(lam_s);
-      // ||E v|| / ||v||: v has unit norm from the second iteration on
-      lam = nrm;
-      const float inv = (nrm > 0.f && isfinite(nrm)) ? 1.f / nrm : 0.f;
-      for (int i = tid; i < r; i += kCholThreads) v[i] = wv[i] * inv;
-      __syncthreads();
-      if (itp == 0) lam = INFINITY;  // the first product uses an unnormalized start vector
     }
     if (isfinite(lam) && 1.5f * lam < near_identity) {
       for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) {
         const int64_t i = e / r, j = e % r;
-        const float sij = S[i * ls + j];
+        const float sij = (j <= i) ? S[i * ls + j] : 0.f;
         Li[i * ls + j] = (j < i) ? -sij : (j == i ? 1.f - 0.5f * (sij - 1.f) : 0.f);
       }
       return;
     }
   }
+  // Y: zero the columns past r once (the update's tiles read up to the next multiple of 8)
+  for (int e = tid; e < CB * ldy; e += kCholThreads)
+    if (ysw(e % ldy) >= r) Y[e] = 0.f;
   __syncthreads();
 
-  bool ok = cholesky_blocked(S, r, ls, D, Pn, &bad);
+  bool ok = chol_inverse(S, Li, r, ls, 0.f, D, DI, rd, Y, ldy, &bad);
   bool shifted = false;
-  if (!ok) {  // shifted retry: lower triangle from the untouched upper triangle, shifted diagonal
-    if (tid == 0) {
-      double tr = 0.0;
-      for (int i = 0; i < r; ++i) tr += (double)diag0[i];
-      trace_s = tr;
-    }
+  if (!ok) {  // shifted retry from S + s I
+    double tr = 0.0;
+    for (int i = tid; i < r; i += kCholThreads) tr += (double)S[(int64_t)i * ls + i];
+    tr = block_sum<kCholThreads>(tr, red);
+    __shared__ double trace_s;
+    if (tid == 0) trace_s = tr;
     __syncthreads();
     const double u = 5.9604644775390625e-8;  // 2^-24
     const double shift = 11.0 * ((double)Ly.m * r + (double)r * (r + 1)) * u * trace_s;
-    for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) {
-      const int64_t i = e / r, j = e % r;
-      if (j < i) S[i * ls + j] = S[j * ls + i];
-      else if (j == i) S[i * ls + j] = (float)((double)diag0[i] + shift);
-    }
-    __syncthreads();
     shifted = true;
-    ok = (trace_s > 0.0) && isfinite(trace_s) && cholesky_blocked(S, r, ls, D, Pn, &bad);
+    ok = (trace_s > 0.0) && isfinite(trace_s) && chol_inverse(S, Li, r, ls, (float)shift, D, DI, rd, Y, ldy, &bad);
   }
   if (tid == 0) {
     if (pass == 0) sh.orth_shifted[l] = shifted ? 1 : 0;
@@ -502,92 +586,14 @@ __global__ void __launch_bounds__(kCholThreads) chol_inv_kernel(Shared sh, int p
   }
   if (!ok) {
     if (tid == 0) set_status(sh.status, ST_BREAKDOWN);
+    __syncthreads();
     for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) Li[(e / r) * ls + e % r] = 0.f;
-    return;
-  }
-
-  // ---------------- L^{-1}, block row by block row ----------------
-  // Linv[I,I] = L[I,I]^{-1};  Linv[I,J] = -L[I,I]^{-1} sum_{K=J..I-1} L[I,K] Linv[K,J]  (J < I)
-  for (int I0 = 0; I0 < r; I0 += CB) {
-    const int nb = min(CB, r - I0);
-    for (int e = tid; e < CB * CB; e += kCholThreads) {
-      const int i = e / CB, j = e % CB;
-      float v;
-      if (i < nb && j < nb) v = (j <= i) ? S[(int64_t)(I0 + i) * ls + I0 + j] : 0.f;
-      else v = (i == j) ? 1.f : 0.f;
-      D[i * CBP + j] = v;
-    }
-    __syncthreads();
-    if (warp == 0) {  // lane c solves L_II x = e_c
-      float x[CB];
-#pragma unroll
-      for (int i = 0; i < CB; ++i) {
-        float v = (i == lane) ? 1.f : 0.f;
-#pragma unroll
-        for (int k = 0; k < i; ++k) v -= D[i * CBP + k] * x[k];
-        x[i] = v / D[i * CBP + i];
-      }
-#pragma unroll
-      for (int i = 0; i < CB; ++i) DI[i * CBP + lane] = x[i];
-    }
-    // Row block I of L staged in shared memory: Lb[i][k] = L[I0+i][k], k < I0.
-    for (int e = tid; e < CB * I0; e += kCholThreads) {
-      const int i = e / I0, k = e % I0;
-      Pn[i * I0 + k] = (i < nb) ? S[(int64_t)(I0 + i) * ls + k] : 0.f;
-    }
-    __syncthreads();
-    // Thread c < I0 owns column c: T[i] = sum_{k=c}^{I0-1} Lb[i][k] Linv[k][c] for the 32 rows
-    // i of the block (one load of Linv[k][c] feeds 32 FMAs), then Linv[I0+i][c] = -(DI T)[i].
-    for (int c = tid; c < I0; c += kCholThreads) {
-      float acc[CB];
-#pragma unroll
-      for (int i = 0; i < CB; ++i) acc[i] = 0.f;
-      // Linv[k][c] = 0 for k < c (upper triangle, stored as zeros), so every lane of a warp can
-      // start at the warp's first column: uniform trip counts, 8 independent loads in flight.
-      const int kbeg = c & ~31;
-      int k = kbeg;
-      for (; k + 8 <= I0; k += 8) {
-        float lk[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) lk[u] = Li[(int64_t)(k + u) * ls + c];
-#pragma unroll
-        for (int u = 0; u < 8; ++u)
-#pragma unroll
-          for (int i = 0; i < CB; ++i) acc[i] = fmaf(Pn[i * I0 + k + u], lk[u], acc[i]);
-      }
-      for (; k < I0; ++k) {
-        const float lk = Li[(int64_t)k * ls + c];
-#pragma unroll
-        for (int i = 0; i < CB; ++i) acc[i] = fmaf(Pn[i * I0 + k], lk, acc[i]);
-      }
-#pragma unroll
-      for (int i = CB - 1; i >= 0; --i) {  // in place: row i needs acc[j] for j <= i only
-        float v = 0.f;
-#pragma unroll
-        for (int j = 0; j <= i; ++j) v = fmaf(DI[i * CBP + j], acc[j], v);
-        acc[i] = -v;
-      }
-#pragma unroll
-      for (int i = 0; i < CB; ++i)
-        if (i < nb) Li[(int64_t)(I0 + i) * ls + c] = acc[i];
-    }
-    // diagonal block DI and zeros to its right
-    for (int e = tid; e < nb * (r - I0); e += kCholThreads) {
-      const int i = e / (r - I0), c = I0 + e % (r - I0);
-      float v = 0.f;
-      if (c < I0 + nb) {
-        const int j = c - I0;
-        v = (j <= i) ? DI[i * CBP + j] : 0.f;
-      }
-      Li[(int64_t)(I0 + i) * ls + c] = v;
-    }
-    __syncthreads();
   }
 }
 
 cudaError_t prepare_chol_inv(int32_t max_r, size_t *smem_out) {
-  const int64_t big = (int64_t)max_r * CBP > (int64_t)CB * max_r ? (int64_t)max_r * CBP : (int64_t)CB * max_r;
-  const size_t smem = sizeof(float) * (2 * CB * CBP + DION_MAX_RANK_PAD + big);
+  const int ldy = (max_r + 7) / 8 * 8;
+  const size_t smem = sizeof(float) * (CB * CBP + 32 + CB * CB + (size_t)CB * std::max(ldy, 8));
   *smem_out = smem;
   return cudaFuncSetAttribute(chol_inv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
 }

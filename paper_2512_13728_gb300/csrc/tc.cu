@@ -26,24 +26,6 @@ void tick(dion_plan *p, cudaStream_t s, const char *name);
 
 namespace tc {
 
-// ================================================================== P -> bf16 copy ===
-// P (fp32, ld ldp) -> P_hi (bf16, same pitch) for the update's A operand; active layers only.
-constexpr int kCvtThreads = 256;
-
-// The orthogonalization ends in P after a shifted third pass and in P_raw otherwise.
-__global__ void __launch_bounds__(kCvtThreads) cvt_p_kernel(Shared sh, const int4 *tiles) {
-  const int4 t = tiles[blockIdx.x];  // {layer, first row, rows, 0}
-  if (!sh.active[t.x]) return;
-  const DevLayer &L = sh.layers[t.x];
-  const int64_t r = L.r, ldp = L.ldp;
-  const float *src = sh.orth_shifted[t.x] ? L.P : L.P_raw;
-  const int64_t total = (int64_t)t.z * r;
-  for (int64_t e = threadIdx.x; e < total; e += kCvtThreads) {
-    const int64_t i = t.y + e / r, j = e % r;
-    L.P_hi[i * ldp + j] = __float2bfloat16_rn(src[i * ldp + j]);
-  }
-}
-
 // ============================================================ update (tcgen05) kernel ===
 constexpr int U_STAGES = 3;
 constexpr uint32_t U_OPB = 128u * 64u * 2u;           // one 128 x 64 bf16 operand box
@@ -314,9 +296,6 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
     for (int64_t mb = 0; mb < (ly.m + 127) / 128; ++mb)
       for (int64_t nb = 0; nb < (ly.n + 127) / 128; ++nb)
         lo.utiles.push_back(make_int4(l, (int)mb, (int)nb, (int)lo.utiles.size()));
-    const int64_t prow = std::max<int64_t>(1, std::min<int64_t>(ly.m, 16384 / ly.r));
-    for (int64_t r0 = 0; r0 < ly.m; r0 += prow)
-      lo.ptiles.push_back(make_int4(l, (int)r0, (int)std::min(prow, ly.m - r0), 0));
     const int64_t qrow = std::max<int64_t>(1, std::min<int64_t>(ly.n, 16384 / ly.r));
     for (int64_t r0 = 0; r0 < ly.n; r0 += qrow)
       lo.qtiles.push_back(make_int4(l, (int)r0, (int)std::min(qrow, ly.n - r0), 0));
@@ -342,7 +321,6 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
   }
   lo.o_maps = take(sizeof(LayerMaps) * std::max(L, 1), 128);
   lo.o_utiles = take(sizeof(int4) * std::max<size_t>(lo.utiles.size(), 1));
-  lo.o_ptiles = take(sizeof(int4) * std::max<size_t>(lo.ptiles.size(), 1));
   lo.o_ftiles = take(sizeof(int4) * std::max<size_t>(lo.ftiles.size(), 1));
   lo.o_rtiles = take(sizeof(int4) * std::max<size_t>(lo.rtiles.size(), 1));
   lo.o_qtiles = take(sizeof(int4) * std::max<size_t>(lo.qtiles.size(), 1));
@@ -381,8 +359,6 @@ void bind(const TcLayout &lo, char *base, DevLayer *dl, int32_t L, TcPlan *tp) {
   tp->maps = reinterpret_cast<LayerMaps *>(base + lo.o_maps);
   tp->utiles = reinterpret_cast<int4 *>(base + lo.o_utiles);
   tp->n_utiles = (int32_t)lo.utiles.size();
-  tp->ptiles = reinterpret_cast<int4 *>(base + lo.o_ptiles);
-  tp->n_ptiles = (int32_t)lo.ptiles.size();
   tp->ftiles = reinterpret_cast<int4 *>(base + lo.o_ftiles);
   tp->n_ftiles = (int32_t)lo.ftiles.size();
   tp->rtiles = reinterpret_cast<int4 *>(base + lo.o_rtiles);
@@ -431,6 +407,7 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
                     encode_f32_2d(&m.PTraw_t, d.PT_raw, d.m, d.r, (uint64_t)d.ldmt * 4, 32, 32) &&
                     encode_f32_2d(&m.PT_t, d.PT, d.m, d.r, (uint64_t)d.ldmt * 4, 32, 32) &&
                     encode_f32_2d(&m.Sst, d.S, d.r, d.r, p32, 32, 128) &&
+                    encode_f32_2d(&m.Sst_t, d.S, d.r, d.r, p32, 32, 32) &&
                     encode_f32_2d(&m.Linv, d.Linv, d.r, d.r, p32, 32, 128);
     if (!ok) return cudaErrorInvalidValue;
   }
@@ -439,7 +416,6 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   };
   cudaError_t e = cudaMemcpy(tp->maps, maps.data(), sizeof(LayerMaps) * maps.size(), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = up(tp->utiles, lo.utiles);
-  if (e == cudaSuccess) e = up(tp->ptiles, lo.ptiles);
   if (e == cudaSuccess) e = up(tp->ftiles, lo.ftiles);
   if (e == cudaSuccess) e = up(tp->rtiles, lo.rtiles);
   if (e == cudaSuccess) e = up(tp->qtiles, lo.qtiles);
@@ -478,7 +454,7 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   tp->num_sms = sms;
-  tp->launches = 19;
+  tp->launches = 18;
   return e;
 }
 
@@ -502,11 +478,9 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, c
     tick(p, s, kGram[pass]);
     launch_chol_inv(sh, chol_smem, pass, 6e-2f, s);  // L, L^{-1}
     tick(p, s, kChol[pass]);
-    launch_orth(sh, tp, false, pass, s);  // X L^{-T} and its transpose
+    launch_orth(sh, tp, false, pass, s);  // X L^{-T} and its transpose, or its bf16 copy at the end
     tick(p, s, kTrsm[pass]);
   }
-  if (tp.n_ptiles > 0) cvt_p_kernel<<<tp.n_ptiles, kCvtThreads, 0, s>>>(sh, tp.ptiles);
-  tick(p, s, "cvt_p");
   launch_btp(sh, tp, s);  // R = B^T P
   tick(p, s, "tc_btp");
   launch_colnorm_reduce(sh, ctiles, n_ctiles, a.eps_col, s);  // 1 / (||R_j|| + eps) from tile partials

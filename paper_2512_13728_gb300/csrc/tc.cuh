@@ -31,6 +31,7 @@ struct LayerMaps {
   CUtensorMap PTraw_t;  // r x m fp32: box {32, 32}  transposed output store
   CUtensorMap PT_t;     // r x m fp32: box {32, 32}  transposed output store
   CUtensorMap Sst;    // r x r fp32:  box {32, 128}  Gram output
+  CUtensorMap Sst_t;  // r x r fp32:  box {32, 32}   Gram output, transposed boxes (upper triangle)
   CUtensorMap Linv;   // r x r fp32:  box {32, 128}  TRSM B operand (rows of L^{-1})
 };
 
@@ -46,12 +47,12 @@ struct TcLayout {
   Schedule s_update, s_bq, s_btp, s_gram, s_trsm;
   size_t end = 0;
   size_t o_maps = 0;
-  size_t o_utiles = 0, o_ptiles = 0, o_ftiles = 0, o_rtiles = 0, o_qtiles = 0, o_gtiles = 0, o_ttiles = 0;
+  size_t o_utiles = 0, o_ftiles = 0, o_rtiles = 0, o_qtiles = 0, o_gtiles = 0, o_ttiles = 0;
   std::vector<size_t> o_phi, o_rhi, o_qnhi, o_bh, o_ptraw, o_pt, o_colsq, o_colinv;
   std::vector<int4> gram_tiles, trsm_tiles;
   // update tiles {layer, m-block, n-block, slot}; P-convert tiles {layer, row0, rows, 0};
   // B Q tiles {layer, m-block, 0, slot}; B^T P tiles {layer, n-block, 0, 0}; Q-copy tiles
-  std::vector<int4> utiles, ptiles, ftiles, rtiles, qtiles;
+  std::vector<int4> utiles, ftiles, rtiles, qtiles;
   int32_t precision = 0;
   int32_t max_r = 0;
 };
@@ -67,8 +68,6 @@ struct TcPlan {
   LayerMaps *maps = nullptr;
   int4 *utiles = nullptr;
   int32_t n_utiles = 0;
-  int4 *ptiles = nullptr;
-  int32_t n_ptiles = 0;
   int4 *ftiles = nullptr;
   int32_t n_ftiles = 0;
   int4 *rtiles = nullptr;

@@ -1,12 +1,16 @@
 // Orthogonalize on tensor cores for DION_PREC_BF16: the Gram matrix and the triangular
 // solve of each CholeskyQR pass as kind::tf32 tcgen05 GEMMs on fp32 operands loaded by TMA.
 //
-//   Gram   S = X^T X (r x r, lower triangle).  Tile = 128 rows of S; K loop over m.  Both
-//          operands are K-major rows of the transposed copy X^T (r x m), which the producing
-//          kernel (the B Q epilogue or the previous TRSM) writes next to X.
+//   Gram   S = X^T X (r x r).  Tile = 128 rows of S; K loop over m; only the columns up to
+//          the end of the tile's diagonal 128-block are computed, and the chunks strictly left
+//          of that block are also stored transposed, so the whole symmetric S is written with
+//          every entry written once.  Both operands are K-major rows of the transposed copy
+//          X^T (r x m), which the producing kernel (the B Q epilogue or the previous TRSM)
+//          writes next to X.
 //   TRSM   Y = X L^{-T} (m x r).  Tile = 128 rows of X; K loop over r.  A = rows of X
 //          (K-major), B = rows of L^{-1} (K-major, lower triangular: K chunks above a column
-//          part are skipped).  Epilogue stores Y (row-major) and Y^T (transposed boxes).
+//          part are skipped).  Epilogue stores Y (row-major) and Y^T (transposed boxes) for
+//          the next pass, or, in the pass that ends Orthogonalize, only the bf16 copy of Y.
 //
 // Accuracy: tf32 products (10-bit mantissa) with fp32 accumulation give ~5e-4 relative
 // error in S and Y; the second CholeskyQR pass (on an already nearly orthonormal X) brings
@@ -28,7 +32,7 @@ enum : int32_t { ORTH_GRAM = 0, ORTH_TRSM = 1 };
 __device__ __forceinline__ uint32_t pad16(int64_t v) { return (uint32_t)((v + 15) / 16 * 16); }
 
 struct OrthMaps {
-  const CUtensorMap *A, *B, *out, *out_t;  // out_t null for the Gram
+  const CUtensorMap *A, *B, *out, *out_t;
 };
 
 template <int KIND>
@@ -40,7 +44,7 @@ __device__ __forceinline__ OrthMaps orth_maps(const LayerMaps &mp, int pass) {
     o.A = raw_in ? &mp.PTraw : &mp.PT;
     o.B = o.A;
     o.out = &mp.Sst;
-    o.out_t = nullptr;
+    o.out_t = &mp.Sst_t;
   } else {
     o.A = raw_in ? &mp.Praw : &mp.Pf;
     o.B = &mp.Linv;
@@ -189,37 +193,80 @@ __global__ void __launch_bounds__(O_THREADS, 1)
       if (!named_and(1, 128, ab.wait(acc_full, tcount & 1u, sh.status))) break;
       tc_fence_after();
       const int nch = (int)((min((int64_t)N, L.r) + 31) / 32);
-      for (int j = 0; j < nch; ++j) {
-        const uint32_t eb = ecount & 1u;
-        uint8_t *box = stg + eb * 2 * O_BOX, *tbox = box + O_BOX + lg * O_TBOX;
-        if (leader) bulk_wait_read<1>();
-        named_sync(1, 128);
-        uint32_t v[32];
-        tmem_ld32(tmem + (lg * 32u << 16) + j * 32, v);
-        tmem_ld_wait();
+      // The solve that ends Orthogonalize writes only the bf16 copy of P that R = B^T P and the
+      // update read: pass 1 unless a shifted retry asked for pass 2, and pass 2 itself.
+      const bool final_pass = (KIND == ORTH_TRSM) && (pass == 2 || (pass == 1 && !sh.orth_shifted[t.x]));
+      if (final_pass) {
+        for (int j = 0; j < nch; j += 2) {  // two 32-column chunks per 64-column bf16 box
+          const uint32_t eb = ecount & 1u;
+          uint8_t *hb = stg + eb * 2 * O_BOX;
+          if (leader) bulk_wait_read<1>();
+          named_sync(1, 128);
+#pragma unroll 1
+          for (int h = 0; h < 2; ++h) {
+            if (j + h < nch) {
+              uint32_t v[32];
+              tmem_ld32(tmem + (lg * 32u << 16) + (j + h) * 32, v);
+              tmem_ld_wait();
 #pragma unroll
-        for (int q = 0; q < 8; ++q)
-          *reinterpret_cast<float4 *>(box + sw128_f32(row, q)) =
-              make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]), __uint_as_float(v[4 * q + 2]),
-                          __uint_as_float(v[4 * q + 3]));
-        if (KIND == ORTH_TRSM) {
-          // transposed 32 x 32 box of this warp's rows: box row c = output column j*32 + c
+              for (int q = 0; q < 8; ++q) {
+                const __nv_bfloat162 a = __floats2bfloat162_rn(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]));
+                const __nv_bfloat162 b =
+                    __floats2bfloat162_rn(__uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+                uint2 hv;
+                hv.x = *reinterpret_cast<const uint32_t *>(&a);
+                hv.y = *reinterpret_cast<const uint32_t *>(&b);
+                *reinterpret_cast<uint2 *>(hb + sw128_offset(row, (uint32_t)(h * 4 + (q >> 1))) + (q & 1) * 8) = hv;
+              }
+            } else {  // a lone last chunk: the other half of the box (clipped by the store)
 #pragma unroll
-          for (int c = 0; c < 32; ++c)
-            *reinterpret_cast<float *>(tbox + c * 128 + ((((uint32_t)lane >> 2) ^ (c & 7)) << 4) + (lane & 3) * 4) =
-                __uint_as_float(v[c]);
+              for (int q = 4; q < 8; ++q) *reinterpret_cast<uint4 *>(hb + sw128_offset(row, q)) = make_uint4(0, 0, 0, 0);
+            }
+          }
+          fence_async_smem();
+          named_sync(1, 128);
+          if (leader) {
+            tma_store_2d(&maps[t.x].P_hi, hb, j * 32, t.y * 128);
+            bulk_commit();
+          }
+          ++ecount;
         }
-        fence_async_smem();
-        named_sync(1, 128);
-        if (leader) {
-          tma_store_2d(om.out, box, j * 32, t.y * 128);
-          if (KIND == ORTH_TRSM)
-            for (int w4 = 0; w4 < 4; ++w4)
-              if ((int64_t)t.y * 128 + w4 * 32 < L.m)
-                tma_store_2d(om.out_t, stg + eb * 2 * O_BOX + O_BOX + w4 * O_TBOX, t.y * 128 + w4 * 32, j * 32);
-          bulk_commit();
+      } else {
+        const int64_t trows = (KIND == ORTH_GRAM) ? L.r : L.m;  // rows of the transposed output
+        for (int j = 0; j < nch; ++j) {
+          // Gram: chunks left of the diagonal 128-block are mirrored into the upper triangle
+          const bool store_t = (KIND == ORTH_TRSM) || (j * 32 + 32 <= t.y * 128);
+          const uint32_t eb = ecount & 1u;
+          uint8_t *box = stg + eb * 2 * O_BOX, *tbox = box + O_BOX + lg * O_TBOX;
+          if (leader) bulk_wait_read<1>();
+          named_sync(1, 128);
+          uint32_t v[32];
+          tmem_ld32(tmem + (lg * 32u << 16) + j * 32, v);
+          tmem_ld_wait();
+  #pragma unroll
+          for (int q = 0; q < 8; ++q)
+            *reinterpret_cast<float4 *>(box + sw128_f32(row, q)) =
+                make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]), __uint_as_float(v[4 * q + 2]),
+                            __uint_as_float(v[4 * q + 3]));
+          if (store_t) {
+            // transposed 32 x 32 box of this warp's rows: box row c = output column j*32 + c
+  #pragma unroll
+            for (int c = 0; c < 32; ++c)
+              *reinterpret_cast<float *>(tbox + c * 128 + ((((uint32_t)lane >> 2) ^ (c & 7)) << 4) + (lane & 3) * 4) =
+                  __uint_as_float(v[c]);
+          }
+          fence_async_smem();
+          named_sync(1, 128);
+          if (leader) {
+            tma_store_2d(om.out, box, j * 32, t.y * 128);
+            if (store_t)
+              for (int w4 = 0; w4 < 4; ++w4)
+                if ((int64_t)t.y * 128 + w4 * 32 < trows)
+                  tma_store_2d(om.out_t, stg + eb * 2 * O_BOX + O_BOX + w4 * O_TBOX, t.y * 128 + w4 * 32, j * 32);
+            bulk_commit();
+          }
+          ++ecount;
         }
-        ++ecount;
       }
       tc_fence_before();
       mbar_arrive(acc_empty);

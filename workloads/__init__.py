@@ -72,6 +72,8 @@ WORKLOADS = {
     # 1.3B-shaped stack: 24 blocks, d = 2048, 144 matrices
     "gpt1p3b_stack_r512": Workload("gpt1p3b_stack_r512", gpt_block(2048, 8192) * 24, 512, 50, "bf16",
                                    1e-3, seed=15),
+    # one block of the 1.3B-shaped stack (the profiling case: same shapes and rank, 6 matrices)
+    "gpt1p3b_block_r512": Workload("gpt1p3b_block_r512", gpt_block(2048, 8192), 512, 50, "bf16", 1e-3, seed=15),
     # 350M-shaped gate stress stack: 24 blocks, d = 1024, flat/spiky phases every 50 steps
     "gpt350m_gate_stress_r256": Workload("gpt350m_gate_stress_r256", gpt_block(1024, 4096) * 24, 256,
                                          300, "bf16", 1e-3, kind="spiky", seed=16),
