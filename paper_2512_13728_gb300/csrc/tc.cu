@@ -311,9 +311,7 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
   lo.s_update = sched(lo.utiles, [&](const int4 &t) { return (double)layers[t.x].r + 64.0; });
   lo.s_bq = sched(lo.ftiles, [&](const int4 &t) { return (double)layers[t.x].n + 2.0 * layers[t.x].r; });
   lo.s_btp = sched(lo.rtiles, [&](const int4 &t) { return (double)layers[t.x].m + 2.0 * layers[t.x].r; });
-  lo.s_gram = sched(lo.gram_tiles, [&](const int4 &t) {
-    return (double)layers[t.x].m * std::min<double>(layers[t.x].r, 128.0 * (t.y + 1)) / 128.0;
-  });
+  lo.s_gram = sched(lo.gram_tiles, [&](const int4 &t) { return (double)layers[t.x].m * layers[t.x].r; });
   lo.s_trsm = sched(lo.trsm_tiles, [&](const int4 &t) { return 3.0 * layers[t.x].r + 64.0; });
   for (Schedule *sc : {&lo.s_update, &lo.s_bq, &lo.s_btp, &lo.s_gram, &lo.s_trsm}) {
     sc->o_tiles = take(sizeof(int4) * std::max<size_t>(sc->tiles.size(), 1));
@@ -407,7 +405,6 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
                     encode_f32_2d(&m.PTraw_t, d.PT_raw, d.m, d.r, (uint64_t)d.ldmt * 4, 32, 32) &&
                     encode_f32_2d(&m.PT_t, d.PT, d.m, d.r, (uint64_t)d.ldmt * 4, 32, 32) &&
                     encode_f32_2d(&m.Sst, d.S, d.r, d.r, p32, 32, 128) &&
-                    encode_f32_2d(&m.Sst_t, d.S, d.r, d.r, p32, 32, 32) &&
                     encode_f32_2d(&m.Linv, d.Linv, d.r, d.r, p32, 32, 128);
     if (!ok) return cudaErrorInvalidValue;
   }

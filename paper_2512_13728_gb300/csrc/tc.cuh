@@ -31,7 +31,6 @@ struct LayerMaps {
   CUtensorMap PTraw_t;  // r x m fp32: box {32, 32}  transposed output store
   CUtensorMap PT_t;     // r x m fp32: box {32, 32}  transposed output store
   CUtensorMap Sst;    // r x r fp32:  box {32, 128}  Gram output
-  CUtensorMap Sst_t;  // r x r fp32:  box {32, 32}   Gram output, transposed boxes (upper triangle)
   CUtensorMap Linv;   // r x r fp32:  box {32, 128}  TRSM B operand (rows of L^{-1})
 };
 

@@ -352,17 +352,47 @@ __global__ void __launch_bounds__(256) colnorm_reduce_kernel(Shared sh, const in
   }
 }
 
-// Q_t = R diag(colinv) (fp32, caller's buffer) and its bf16 copy; tiles of rows of R.
-__global__ void __launch_bounds__(256) colnorm_scale_kernel(Shared sh, const int4 *tiles) {
+// Q_t = R diag(colinv) (fp32, caller's buffer) and its bf16 copy; tiles of rows of R.  One
+// warp per row, 16-byte loads of R (rows padded to a multiple of 8 floats), the scale factors
+// of the lane's columns kept in registers; the caller's Q is written only inside its r columns.
+constexpr int kScaleThreads = 256;
+__global__ void __launch_bounds__(kScaleThreads) colnorm_scale_kernel(Shared sh, const int4 *tiles) {
   const int4 t = tiles[blockIdx.x];  // {layer, first row, rows, 0}
   if (!sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
-  const int64_t r = L.r, total = (int64_t)t.z * r;
-  for (int64_t e = threadIdx.x; e < total; e += 256) {
-    const int64_t i = t.y + e / r, j = e % r;
-    const float q = L.R[i * L.ldp + j] * L.colinv[j];
-    L.Q[i * L.ldq + j] = q;
-    L.Qn_hi[i * L.ldp + j] = __float2bfloat16_rn(q);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int r = (int)L.r, r4 = (r + 3) / 4;  // r <= 512: at most 4 chunks per lane
+  float4 cs[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int c = 4 * (lane + 32 * k);
+    cs[k] = make_float4(c < r ? L.colinv[c] : 0.f, c + 1 < r ? L.colinv[c + 1] : 0.f,
+                        c + 2 < r ? L.colinv[c + 2] : 0.f, c + 3 < r ? L.colinv[c + 3] : 0.f);
+  }
+  for (int64_t i = t.y + warp; i < (int64_t)t.y + t.z; i += kScaleThreads / 32) {
+    const float *Rrow = L.R + i * L.ldp;
+    float4 rv[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (lane + 32 * k < r4) rv[k] = *reinterpret_cast<const float4 *>(Rrow + 4 * (lane + 32 * k));
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int c4 = lane + 32 * k;
+      if (c4 >= r4) continue;
+      const float4 q = make_float4(rv[k].x * cs[k].x, rv[k].y * cs[k].y, rv[k].z * cs[k].z, rv[k].w * cs[k].w);
+      const __nv_bfloat162 h01 = __floats2bfloat162_rn(q.x, q.y), h23 = __floats2bfloat162_rn(q.z, q.w);
+      uint2 hv;
+      hv.x = *reinterpret_cast<const uint32_t *>(&h01);
+      hv.y = *reinterpret_cast<const uint32_t *>(&h23);
+      *reinterpret_cast<uint2 *>(L.Qn_hi + i * L.ldp + 4 * c4) = hv;  // workspace rows: padded
+      float *Qrow = L.Q + i * L.ldq + 4 * c4;
+      if (4 * c4 + 4 <= r) {
+        *reinterpret_cast<float4 *>(Qrow) = q;
+      } else {
+        const float qq[4] = {q.x, q.y, q.z, q.w};
+        for (int e = 0; e < r - 4 * c4; ++e) Qrow[e] = qq[e];
+      }
+    }
   }
 }
 
@@ -370,7 +400,7 @@ void launch_colnorm_reduce(const Shared &sh, const int4 *ctiles, int32_t n_ctile
   if (n_ctiles > 0) colnorm_reduce_kernel<<<n_ctiles, 256, 0, s>>>(sh, ctiles, eps_col);
 }
 void launch_colnorm_scale(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
-  if (tp.n_qtiles > 0) colnorm_scale_kernel<<<tp.n_qtiles, 256, 0, s>>>(sh, tp.qtiles);
+  if (tp.n_qtiles > 0) colnorm_scale_kernel<<<tp.n_qtiles, kScaleThreads, 0, s>>>(sh, tp.qtiles);
 }
 
 }  // namespace tc

@@ -1,12 +1,11 @@
 // Orthogonalize on tensor cores for DION_PREC_BF16: the Gram matrix and the triangular
 // solve of each CholeskyQR pass as kind::tf32 tcgen05 GEMMs on fp32 operands loaded by TMA.
 //
-//   Gram   S = X^T X (r x r).  Tile = 128 rows of S; K loop over m; only the columns up to
-//          the end of the tile's diagonal 128-block are computed, and the chunks strictly left
-//          of that block are also stored transposed, so the whole symmetric S is written with
-//          every entry written once.  Both operands are K-major rows of the transposed copy
-//          X^T (r x m), which the producing kernel (the B Q epilogue or the previous TRSM)
-//          writes next to X.
+//   Gram   S = X^T X (r x r).  Tile = 128 full rows of S; K loop over m.  B = all r rows of
+//          the transposed copy X^T (r x m, K-major), which the producing kernel (the B Q
+//          epilogue or the previous TRSM) writes next to X; A = the tile's own 128 rows, read
+//          in place from B's boxes.  Every tile of a layer costs the same and streams the same
+//          X^T, so the layer's tiles run side by side and read X^T from DRAM about once.
 //   TRSM   Y = X L^{-T} (m x r).  Tile = 128 rows of X; K loop over r.  A = rows of X
 //          (K-major), B = rows of L^{-1} (K-major, lower triangular: K chunks above a column
 //          part are skipped).  Epilogue stores Y (row-major) and Y^T (transposed boxes) for
@@ -44,7 +43,7 @@ __device__ __forceinline__ OrthMaps orth_maps(const LayerMaps &mp, int pass) {
     o.A = raw_in ? &mp.PTraw : &mp.PT;
     o.B = o.A;
     o.out = &mp.Sst;
-    o.out_t = &mp.Sst_t;
+    o.out_t = nullptr;
   } else {
     o.A = raw_in ? &mp.Praw : &mp.Pf;
     o.B = &mp.Linv;
@@ -59,7 +58,7 @@ __device__ __forceinline__ OrthMaps orth_maps(const LayerMaps &mp, int pass) {
 template <int KIND>
 __device__ __forceinline__ void orth_dims(const DevLayer &L, int blk, uint32_t &N, int64_t &K) {
   if (KIND == ORTH_GRAM) {
-    N = min(pad16(L.r), (uint32_t)(blk + 1) * 128u);  // lower triangle of S only
+    N = pad16(L.r);
     K = L.m;
   } else {
     N = pad16(L.r);
@@ -128,8 +127,8 @@ __global__ void __launch_bounds__(O_THREADS, 1)
           uint32_t nb = 0;  // B boxes this chunk feeds (all, or only the lower-triangular parts)
           for (uint32_t b = 0; b < nboxes; ++b)
             if (part_needs<KIND>(kc, b / 2)) ++nb;
-          mbar_expect_tx(&full[s], O_BOX * (1 + nb));
-          tma_load_2d(sA, om.A, &full[s], kc * 32, t.y * 128);
+          mbar_expect_tx(&full[s], O_BOX * ((KIND == ORTH_GRAM ? 0 : 1) + nb));
+          if (KIND != ORTH_GRAM) tma_load_2d(sA, om.A, &full[s], kc * 32, t.y * 128);
           for (uint32_t b = 0; b < nboxes; ++b)
             if (part_needs<KIND>(kc, b / 2)) tma_load_2d(sB + b * O_BOX, om.B, &full[s], kc * 32, b * 128);
         }
@@ -159,7 +158,8 @@ __global__ void __launch_bounds__(O_THREADS, 1)
           const uint32_t aB = smem_u32(smem + s * stage_bytes), bB = aB + O_BOX;
 #pragma unroll
           for (int k8 = 0; k8 < 4; ++k8) {
-            const uint64_t ad = smem_desc_sw128(aB + k8 * 32, 0, 1024);
+            // Gram: the tile's rows are B box t.y of the same stage
+            const uint64_t ad = smem_desc_sw128((KIND == ORTH_GRAM ? bB + (uint32_t)t.y * O_BOX : aB) + k8 * 32, 0, 1024);
             for (uint32_t part = 0; part < nparts; ++part) {
               if (!part_needs<KIND>(kc, part)) continue;
               const uint32_t n_here = min(256u, N - part * 256u);
@@ -232,10 +232,8 @@ __global__ void __launch_bounds__(O_THREADS, 1)
           ++ecount;
         }
       } else {
-        const int64_t trows = (KIND == ORTH_GRAM) ? L.r : L.m;  // rows of the transposed output
         for (int j = 0; j < nch; ++j) {
-          // Gram: chunks left of the diagonal 128-block are mirrored into the upper triangle
-          const bool store_t = (KIND == ORTH_TRSM) || (j * 32 + 32 <= t.y * 128);
+          const bool store_t = (KIND == ORTH_TRSM);  // transposed copy: the next Gram's operand
           const uint32_t eb = ecount & 1u;
           uint8_t *box = stg + eb * 2 * O_BOX, *tbox = box + O_BOX + lg * O_TBOX;
           if (leader) bulk_wait_read<1>();
@@ -243,14 +241,14 @@ __global__ void __launch_bounds__(O_THREADS, 1)
           uint32_t v[32];
           tmem_ld32(tmem + (lg * 32u << 16) + j * 32, v);
           tmem_ld_wait();
-  #pragma unroll
+#pragma unroll
           for (int q = 0; q < 8; ++q)
             *reinterpret_cast<float4 *>(box + sw128_f32(row, q)) =
                 make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]), __uint_as_float(v[4 * q + 2]),
                             __uint_as_float(v[4 * q + 3]));
           if (store_t) {
             // transposed 32 x 32 box of this warp's rows: box row c = output column j*32 + c
-  #pragma unroll
+#pragma unroll
             for (int c = 0; c < 32; ++c)
               *reinterpret_cast<float *>(tbox + c * 128 + ((((uint32_t)lane >> 2) ^ (c & 7)) << 4) + (lane & 3) * 4) =
                   __uint_as_float(v[c]);
@@ -261,7 +259,7 @@ __global__ void __launch_bounds__(O_THREADS, 1)
             tma_store_2d(om.out, box, j * 32, t.y * 128);
             if (store_t)
               for (int w4 = 0; w4 < 4; ++w4)
-                if ((int64_t)t.y * 128 + w4 * 32 < trows)
+                if ((int64_t)t.y * 128 + w4 * 32 < L.m)
                   tma_store_2d(om.out_t, stg + eb * 2 * O_BOX + O_BOX + w4 * O_TBOX, t.y * 128 + w4 * 32, j * 32);
             bulk_commit();
           }
