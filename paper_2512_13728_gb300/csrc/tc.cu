@@ -3,15 +3,15 @@
 //
 // Error feedback + parameter update (Algorithm 1/2, sync branch):
 //   M = B - (1 - mu) P R^T,   X = X - eta sqrt(m/n) P Q_t^T
-// run as one persistent, warp-specialized kernel over 128 x 128 output tiles:
+// run as one persistent, warp-specialized kernel over 128 x 128 output tiles, in clusters of
+// two CTAs that share the R and Q_t chunks by multicast:
 //   warp 0      TMA producer: bf16 K-major chunks of P (A), R and Q_t (two B operands) into a
 //               3-stage shared-memory ring;
 //   warp 1      MMA issuer: two 128x128x16 tcgen05.mma per k-step into a double-buffered
 //               pair of TMEM accumulators (U1 = P R^T, U2 = P Q_t^T; 4 x 128 = 512 columns);
-//   warps 2..5  epilogue: TMA-load 128 x 32 fp32 boxes of B (in the M buffer) and X, read
-//               U1/U2 from TMEM (thread = tile row), compute M_t and X_t in shared memory,
-//               TMA-store both; per-tile fp64 partial of ||M_t||^2 for Equation 1.
-// Every HBM byte of the pass (read B, X; write M, X) moves by TMA in 128-byte rows.
+//   warps 2..5  epilogue (both CTAs): TMA-load 128 x 16 fp32 boxes of B (in the M buffer) and X,
+//               read U1/U2 from TMEM (thread = tile row), compute M_t and X_t in shared
+//               memory, TMA-store both; per-tile fp64 partial of ||M_t||^2 for Equation 1.
 #include "tc.cuh"
 #include "tc_common.cuh"
 #include "tc_kernels.cuh"
@@ -27,41 +27,50 @@ void tick(dion_plan *p, cudaStream_t s, const char *name);
 namespace tc {
 
 // ============================================================ update (tcgen05) kernel ===
+// Clusters of two CTAs (one per SM) take row tiles 2 p and 2 p + 1 of the same column block:
+// the R and Q_t chunks are the same for both, so CTA 0 loads the R chunk and CTA 1 the Q_t
+// chunk and each multicasts it to the pair (half the L2 reads of those operands); each CTA's
+// MMA completion frees the stage in both CTAs.
 constexpr int U_STAGES = 3;
-constexpr uint32_t U_OPB = 128u * 64u * 2u;           // one 128 x 64 bf16 operand box
+constexpr uint32_t U_OPB = 128u * 64u * 2u;           // 128 x 64 bf16 operand box
 constexpr uint32_t U_STAGE = 3u * U_OPB;              // P, R, Q_t
-constexpr uint32_t U_EPI = 128u * 32u * 4u;           // one 128 x 32 fp32 box
-constexpr uint32_t U_SMEM = 1024u + U_STAGES * U_STAGE + 4u * U_EPI + 256u;
+constexpr uint32_t U_EBOX = 128u * 16u * 4u;          // one 128 x 16 fp32 box (64-byte swizzle)
+constexpr uint32_t U_EBUF2 = 2u * U_EBOX;             // B and X of one 16-column sub-chunk
+constexpr int U_EBUF = 5;                             // sub-chunk buffers of the epilogue
+constexpr uint32_t U_SMEM = 1024u + U_STAGES * U_STAGE + U_EBUF * U_EBUF2 + 256u;
 constexpr int U_THREADS = 192;
 constexpr uint32_t U_IDESC = idesc_bf16(128, 128, false, false);
 
-__global__ void __launch_bounds__(U_THREADS, 1)
+// Tile = {layer, row-tile pair p, column tile, ||M_t|| slot of row tile 2 p}.
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
     tc_update_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off, const LayerMaps *__restrict__ maps,
                      float mu, float eta) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = align1024(smem_raw);
   uint8_t *stage = smem;
   uint8_t *epi = smem + U_STAGES * U_STAGE;
-  uint64_t *bars = reinterpret_cast<uint64_t *>(epi + 4 * U_EPI);
+  uint64_t *bars = reinterpret_cast<uint64_t *>(epi + U_EBUF * U_EBUF2);
   uint64_t *full = bars, *empty = bars + U_STAGES;
   uint64_t *acc_full = bars + 2 * U_STAGES, *acc_empty = acc_full + 2, *epi_full = acc_empty + 2;
-  uint64_t *drain = epi_full + 2;
+  uint64_t *drain = epi_full + U_EBUF;
   __shared__ uint32_t tmem_base_s;
   __shared__ int abort_s;
   __shared__ double red_s[4];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const Abort ab{&abort_s};
+  const uint32_t rank = cluster_ctarank();
+  const int seg = blockIdx.x >> 1;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < U_STAGES; ++i) {
       mbar_init(&full[i], 1);
-      mbar_init(&empty[i], 1);
+      mbar_init(&empty[i], 2);  // the MMA commits of both CTAs of the pair
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
-      mbar_init(&acc_empty[b], 128);
-      mbar_init(&epi_full[b], 1);
+      mbar_init(&acc_empty[b], 1);  // the epilogue leader, after its warps have read TMEM
     }
+    for (int b = 0; b < U_EBUF; ++b) mbar_init(&epi_full[b], 1);
     mbar_init(drain, 1);
     abort_s = 0;
     fence_mbar_init();
@@ -73,38 +82,40 @@ __global__ void __launch_bounds__(U_THREADS, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  cluster_sync();  // the peer's barriers are initialized before anything is multicast to them
   const uint32_t tmem = tmem_base_s;
 
   if (warp == 0) {
-    // ---------------------------------------------------------------- TMA producer
+    // ---------------------------------------------------------------- TMA producer (both CTAs)
     if (lane == 0) {
       uint32_t it = 0;
       bool ok = true;
-      for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
+      for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
         if (!sh.active[t.x]) continue;
         const LayerMaps *mp = maps + t.x;
         const int kch = (int)((sh.layers[t.x].r + 63) / 64);
+        const int mb = 2 * t.y + (int)rank;  // past the last row tile: zero-filled, not stored
         for (int kc = 0; kc < kch; ++kc, ++it) {
           const uint32_t s = it % U_STAGES, ph = (it / U_STAGES) & 1u;
           if (!ab.wait(&empty[s], ph ^ 1u, sh.status)) { ok = false; break; }
           uint8_t *sp = stage + s * U_STAGE;
           mbar_expect_tx(&full[s], U_STAGE);
-          tma_load_2d(sp, &mp->P_hi, &full[s], kc * 64, t.y * 128);
-          tma_load_2d(sp + U_OPB, &mp->R_hi, &full[s], kc * 64, t.z * 128);
-          tma_load_2d(sp + 2 * U_OPB, &mp->Qn_hi, &full[s], kc * 64, t.z * 128);
+          tma_load_2d(sp, &mp->P_hi, &full[s], kc * 64, mb * 128);
+          if (rank == 0) tma_load_2d_mc(sp + U_OPB, &mp->R_hi, &full[s], kc * 64, t.z * 128, 0x3);
+          else tma_load_2d_mc(sp + 2 * U_OPB, &mp->Qn_hi, &full[s], kc * 64, t.z * 128, 0x3);
         }
       }
-      // drain: every issued load has landed before the CTA may exit
+      // drain: every load into this CTA (its own and the peer's multicasts) has landed
       for (uint32_t k = (it > U_STAGES ? it - U_STAGES : 0); k < it; ++k)
         mbar_wait(&full[k % U_STAGES], (k / U_STAGES) & 1u, sh.status);
     }
   } else if (warp == 1) {
-    // ---------------------------------------------------------------- MMA issuer
+    // ---------------------------------------------------------------- MMA issuer (each CTA)
     if (lane == 0) {
       uint32_t it = 0, tcount = 0;
       bool ok = true;
-      for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
+      for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
         if (!sh.active[t.x]) continue;
         const int kch = (int)((sh.layers[t.x].r + 63) / 64);
@@ -126,7 +137,7 @@ __global__ void __launch_bounds__(U_THREADS, 1)
             umma_bf16(d1, ad, rd, U_IDESC, acc);
             umma_bf16(d2, ad, qd, U_IDESC, acc);
           }
-          umma_commit(&empty[s]);
+          umma_commit_mc(&empty[s], 0x3);  // the stage is free in both CTAs
         }
         if (!ok) break;
         umma_commit(&acc_full[b]);
@@ -137,92 +148,135 @@ __global__ void __launch_bounds__(U_THREADS, 1)
     }
   } else {
     // ---------------------------------------------------------------- epilogue (128 threads)
+    // B and X stream in 16-column sub-chunks through U_EBUF buffers.  The leader keeps the
+    // loads U_EBUF - 1 sub-chunks ahead of the one being written back, across tile boundaries
+    // (they do not depend on the MMAs), so HBM latency is covered without taking shared memory
+    // from the operand ring.
     const int et = threadIdx.x - 64;
     const uint32_t row = 32u * (warp & 3) + lane;  // TMEM lane = tile row
     const bool leader = (et == 0);
-    uint32_t tcount = 0, ecount = 0, issued = 0;
+    const int tend = off[seg + 1];
+    // 16-column sub-chunks of a tile that start inside the matrix; 0 for the pair's second tile
+    // when it lies past the last row tile
+    auto subs_of = [&](const int4 &t) -> int {
+      const DevLayer &L = sh.layers[t.x];
+      if ((int64_t)(2 * t.y + (int)rank) * 128 >= L.m) return 0;
+      return (int)std::min<int64_t>(8, (L.n - (int64_t)t.z * 128 + 15) / 16);
+    };
+    int lt = off[seg], lj = 0;  // load cursor: tile, sub-chunk
+    auto skip_empty = [&]() {
+      while (lt < tend && (!sh.active[tiles[lt].x] || subs_of(tiles[lt]) == 0)) ++lt;
+    };
+    skip_empty();
+    uint32_t ecount = 0, issued = 0;
+    auto issue_upto = [&](uint32_t target) {  // leader: loads of sub-chunks [issued, target)
+      while (issued < target && lt < tend) {
+        const int4 t = tiles[lt];
+        const LayerMaps *mp = maps + t.x;
+        const uint32_t eb = issued % U_EBUF;
+        // the buffer's previous sub-chunk (issued - U_EBUF) was stored at least one sub-chunk
+        // ago: at most the latest store group may still be reading shared memory
+        if (issued >= U_EBUF) bulk_wait_read<1>();
+        uint8_t *bs = epi + eb * U_EBUF2;
+        const int r0 = (2 * t.y + (int)rank) * 128, x0 = t.z * 128 + lj * 16;
+        mbar_expect_tx(&epi_full[eb], U_EBUF2);
+        tma_load_2d(bs, &mp->Mf16, &epi_full[eb], x0, r0);
+        tma_load_2d(bs + U_EBOX, &mp->Xf16, &epi_full[eb], x0, r0);
+        ++issued;
+        if (++lj == subs_of(t)) {
+          lj = 0;
+          ++lt;
+          skip_empty();
+        }
+      }
+    };
+    if (leader) issue_upto(U_EBUF - 1);
+    uint32_t tcount = 0;
     bool ok = true;
-    for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
+    for (int ti = off[seg]; ti < tend && ok; ++ti) {
       const int4 t = tiles[ti];
       if (!sh.active[t.x]) continue;
       const DevLayer &L = sh.layers[t.x];
       const LayerMaps *mp = maps + t.x;
       const float dec = 1.f - mu, c = eta * L.sqrt_m_over_n;
-      const int r0 = t.y * 128, c0 = t.z * 128;
-      // 32-column chunks that start inside the matrix (a ragged last tile has fewer)
-      const int nj = (int)std::min<int64_t>(4, (L.n - c0 + 31) / 32);
+      const int mb = 2 * t.y + (int)rank, r0 = mb * 128, c0 = t.z * 128;
+      const int ntc = (int)((L.n + 127) / 128);
+      const int ns = subs_of(t);
       const uint32_t b = tcount & 1u, aph = (tcount >> 1) & 1u;
-      auto issue = [&](int j) {  // TMA-load chunk j of this tile into its epilogue buffer
-        const uint32_t eb = (ecount + j) & 1u;
-        uint8_t *bs = epi + eb * 2 * U_EPI;
-        bulk_wait_read<0>();  // the store that last used this buffer has read it
-        mbar_expect_tx(&epi_full[eb], 2 * U_EPI);
-        tma_load_2d(bs, &mp->Mf, &epi_full[eb], c0 + j * 32, r0);
-        tma_load_2d(bs + U_EPI, &mp->Xf, &epi_full[eb], c0 + j * 32, r0);
-        ++issued;
-      };
-      if (leader) issue(0);
       if (!named_and(1, 128, ab.wait(&acc_full[b], aph, sh.status))) break;
       tc_fence_after();
       float ss = 0.f;
-      for (int j = 0; j < nj; ++j) {
-        const uint32_t eb = (ecount + j) & 1u, eph = ((ecount + j) >> 1) & 1u;
-        if (leader && j + 1 < nj) issue(j + 1);
+      for (int j = 0; j < (ns + 1) / 2 && ok; ++j) {  // 32-column TMEM chunk j = sub-chunks 2j, 2j + 1
         uint32_t u1[32], u2[32];
         tmem_ld32(tmem + ((32u * (warp & 3)) << 16) + b * 256u + j * 32, u1);
         tmem_ld32(tmem + ((32u * (warp & 3)) << 16) + b * 256u + 128u + j * 32, u2);
         tmem_ld_wait();
-        if (!named_and(1, 128, ab.wait(&epi_full[eb], eph, sh.status))) { ok = false; break; }
-        uint8_t *bs = epi + eb * 2 * U_EPI;
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          const uint32_t off = sw128_f32(row, q);
-          float4 bv = *reinterpret_cast<float4 *>(bs + off);
-          float4 xv = *reinterpret_cast<float4 *>(bs + U_EPI + off);
-          bv.x = fmaf(-dec, __uint_as_float(u1[4 * q + 0]), bv.x);
-          bv.y = fmaf(-dec, __uint_as_float(u1[4 * q + 1]), bv.y);
-          bv.z = fmaf(-dec, __uint_as_float(u1[4 * q + 2]), bv.z);
-          bv.w = fmaf(-dec, __uint_as_float(u1[4 * q + 3]), bv.w);
-          xv.x = fmaf(-c, __uint_as_float(u2[4 * q + 0]), xv.x);
-          xv.y = fmaf(-c, __uint_as_float(u2[4 * q + 1]), xv.y);
-          xv.z = fmaf(-c, __uint_as_float(u2[4 * q + 2]), xv.z);
-          xv.w = fmaf(-c, __uint_as_float(u2[4 * q + 3]), xv.w);
-          ss = fmaf(bv.x, bv.x, ss); ss = fmaf(bv.y, bv.y, ss);
-          ss = fmaf(bv.z, bv.z, ss); ss = fmaf(bv.w, bv.w, ss);
-          *reinterpret_cast<float4 *>(bs + off) = bv;
-          *reinterpret_cast<float4 *>(bs + U_EPI + off) = xv;
-        }
-        fence_async_smem();
-        named_sync(1, 128);
-        if (leader) {  // out-of-range rows/columns of a ragged tile are clipped by the store
-          tma_store_2d(&mp->Mf, bs, c0 + j * 32, r0);
-          tma_store_2d(&mp->Xf, bs + U_EPI, c0 + j * 32, r0);
-          bulk_commit();
+        for (int h = 0; h < 2; ++h) {
+          const int sub = 2 * j + h;
+          if (sub >= ns) break;
+          const uint32_t k = ecount + sub, eb = k % U_EBUF, eph = (k / U_EBUF) & 1u;
+          if (!named_and(1, 128, ab.wait(&epi_full[eb], eph, sh.status))) {
+            ok = false;
+            break;
+          }
+          uint8_t *bs = epi + eb * U_EBUF2;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const uint32_t o = sw64_f32(row, q);
+            const int cc = h * 16 + q * 4;
+            float4 bv = *reinterpret_cast<float4 *>(bs + o);
+            float4 xv = *reinterpret_cast<float4 *>(bs + U_EBOX + o);
+            bv.x = fmaf(-dec, __uint_as_float(u1[cc + 0]), bv.x);
+            bv.y = fmaf(-dec, __uint_as_float(u1[cc + 1]), bv.y);
+            bv.z = fmaf(-dec, __uint_as_float(u1[cc + 2]), bv.z);
+            bv.w = fmaf(-dec, __uint_as_float(u1[cc + 3]), bv.w);
+            xv.x = fmaf(-c, __uint_as_float(u2[cc + 0]), xv.x);
+            xv.y = fmaf(-c, __uint_as_float(u2[cc + 1]), xv.y);
+            xv.z = fmaf(-c, __uint_as_float(u2[cc + 2]), xv.z);
+            xv.w = fmaf(-c, __uint_as_float(u2[cc + 3]), xv.w);
+            ss = fmaf(bv.x, bv.x, ss); ss = fmaf(bv.y, bv.y, ss);
+            ss = fmaf(bv.z, bv.z, ss); ss = fmaf(bv.w, bv.w, ss);
+            *reinterpret_cast<float4 *>(bs + o) = bv;
+            *reinterpret_cast<float4 *>(bs + U_EBOX + o) = xv;
+          }
+          fence_async_smem();
+          named_sync(1, 128);
+          if (leader) {  // out-of-range rows/columns of a ragged tile are clipped by the store
+            tma_store_2d(&mp->Mf16, bs, c0 + sub * 16, r0);
+            tma_store_2d(&mp->Xf16, bs + U_EBOX, c0 + sub * 16, r0);
+            bulk_commit();
+            issue_upto(k + U_EBUF);  // sub-chunk k + U_EBUF - 1 reuses the buffer of k - 1
+          }
         }
       }
-      ecount += nj;
-      tc_fence_before();
-      mbar_arrive(&acc_empty[b]);
       if (!ok) break;
-      // per-tile ||M_t||^2 (rows/columns outside the matrix hold 0), fixed reduction order
+      ecount += ns;
+      // per-tile ||M_t||^2 (rows/columns outside the matrix hold 0), fixed reduction order;
+      // the barrier also ends every thread's TMEM reads of this accumulator
       double v = (double)ss;
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
       if (lane == 0) red_s[warp - 2] = v;
+      tc_fence_before();
       named_sync(1, 128);
-      if (leader) sh.upart[t.w] = (red_s[0] + red_s[1]) + (red_s[2] + red_s[3]);
+      if (leader) {
+        mbar_arrive(&acc_empty[b]);  // every thread has read accumulator buffer b
+        if (ns > 0) sh.upart[t.w + (int)rank * ntc] = (red_s[0] + red_s[1]) + (red_s[2] + red_s[3]);
+      }
       ++tcount;
     }
     if (leader) {
       bulk_wait<0>();
       // loads issued but not consumed (only after an abort)
-      for (uint32_t k = ecount; k < issued; ++k) mbar_wait(&epi_full[k & 1u], (k >> 1) & 1u, sh.status);
+      for (uint32_t k = ecount; k < issued; ++k) mbar_wait(&epi_full[k % U_EBUF], (k / U_EBUF) & 1u, sh.status);
     }
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem, 512);
+  cluster_sync();  // nothing more is multicast to, or arrives at, a CTA that has exited
 }
 
 // ========================================================================= host side ===
@@ -308,7 +362,13 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
     for (size_t i = 0; i < tl.size(); ++i) c[i] = costf(tl[i]);
     return lpt(tl, c, std::max(num_sms, 1));
   };
-  lo.s_update = sched(lo.utiles, [&](const int4 &t) { return (double)layers[t.x].r + 64.0; });
+  // update: row-tile pairs (one per cluster of two CTAs); w = ||M_t|| slot of the pair's first tile
+  std::vector<int4> upairs;
+  for (size_t i = 0; i < lo.utiles.size(); ++i) {
+    const int4 &u = lo.utiles[i];
+    if (u.y % 2 == 0) upairs.push_back(make_int4(u.x, u.y / 2, u.z, u.w));
+  }
+  lo.s_update = lpt(upairs, std::vector<double>(upairs.size(), 1.0), std::max(num_sms / 2, 1));
   lo.s_bq = sched(lo.ftiles, [&](const int4 &t) { return (double)layers[t.x].n + 2.0 * layers[t.x].r; });
   lo.s_btp = sched(lo.rtiles, [&](const int4 &t) { return (double)layers[t.x].m + 2.0 * layers[t.x].r; });
   lo.s_gram = sched(lo.gram_tiles, [&](const int4 &t) { return (double)layers[t.x].m * layers[t.x].r; });
@@ -393,6 +453,8 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
                     encode_bf16_2d(&m.Qn_hi, d.Qn_hi, d.r, d.n, p16, 64, 128) &&
                     encode_f32_2d(&m.Mf, d.M, d.n, d.m, (uint64_t)d.ldm * 4, 32, 128) &&
                     encode_f32_2d(&m.Xf, d.X, d.n, d.m, (uint64_t)d.ldx * 4, 32, 128) &&
+                    encode_f32_2d(&m.Mf16, d.M, d.n, d.m, (uint64_t)d.ldm * 4, 16, 128) &&
+                    encode_f32_2d(&m.Xf16, d.X, d.n, d.m, (uint64_t)d.ldx * 4, 16, 128) &&
                     encode_bf16_2d(&m.Qn_mn, d.Qn_hi, d.r, d.n, p16, 64, 64) &&
                     encode_bf16_2d(&m.P_mn, d.P_hi, d.r, d.m, p16, 64, 64) &&
                     encode_bf16_2d(&m.Bh_mn, d.Bh, d.n, d.m, (uint64_t)d.ldbh * 2, 64, 64) &&
@@ -485,8 +547,8 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, c
   launch_colnorm_scale(sh, tp, s);  // Q_t = R diag(...), its bf16 copy
   tick(p, s, "colnorm_scale");
   if (tp.d_update.grid > 0)
-    tc_update_kernel<<<tp.d_update.grid, U_THREADS, U_SMEM, s>>>(sh, tp.d_update.tiles, tp.d_update.off, tp.maps,
-                                                                  a.mu, a.eta);
+    tc_update_kernel<<<2 * tp.d_update.grid, U_THREADS, U_SMEM, s>>>(sh, tp.d_update.tiles, tp.d_update.off, tp.maps,
+                                                                      a.mu, a.eta);
   tick(p, s, "tc_update");
   launch_local(sh, btiles, n_btiles, a.eta_local, s);
   tick(p, s, "local");
