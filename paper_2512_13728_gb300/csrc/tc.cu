@@ -369,8 +369,20 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
     if (u.y % 2 == 0) upairs.push_back(make_int4(u.x, u.y / 2, u.z, u.w));
   }
   lo.s_update = lpt(upairs, std::vector<double>(upairs.size(), 1.0), std::max(num_sms / 2, 1));
-  lo.s_bq = sched(lo.ftiles, [&](const int4 &t) { return (double)layers[t.x].n + 2.0 * layers[t.x].r; });
-  lo.s_btp = sched(lo.rtiles, [&](const int4 &t) { return (double)layers[t.x].m + 2.0 * layers[t.x].r; });
+  // B Q and B^T P run in CTA pairs over two consecutive 128-row tiles: tile {layer, pair}
+  auto pairs_of = [](const std::vector<int4> &tl) {
+    std::vector<int4> pr;
+    for (const int4 &t : tl)
+      if (t.y % 2 == 0) pr.push_back(make_int4(t.x, t.y / 2, 0, 0));
+    return pr;
+  };
+  auto pair_sched = [&](const std::vector<int4> &tl, auto costf) {
+    std::vector<double> c(tl.size());
+    for (size_t i = 0; i < tl.size(); ++i) c[i] = costf(tl[i]);
+    return lpt(tl, c, std::max(num_sms / 2, 1));
+  };
+  lo.s_bq = pair_sched(pairs_of(lo.ftiles), [&](const int4 &t) { return (double)layers[t.x].n + 2.0 * layers[t.x].r; });
+  lo.s_btp = pair_sched(pairs_of(lo.rtiles), [&](const int4 &t) { return (double)layers[t.x].m + 2.0 * layers[t.x].r; });
   lo.s_gram = sched(lo.gram_tiles, [&](const int4 &t) { return (double)layers[t.x].m * layers[t.x].r; });
   lo.s_trsm = sched(lo.trsm_tiles, [&](const int4 &t) { return 3.0 * layers[t.x].r + 64.0; });
   for (Schedule *sc : {&lo.s_update, &lo.s_bq, &lo.s_btp, &lo.s_gram, &lo.s_trsm}) {
@@ -489,13 +501,16 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   // shared-memory budget: operand stages + 2 staging buffers of (128 x 32 + 4 x 32 x 32) fp32
   const uint32_t budget = 227u * 1024u - 1024u - 4u * 128u * 32u * 4u - 512u - 256u;
   const uint32_t nb64 = (uint32_t)std::max(1, (lo.max_r + 63) / 64);
-  const uint32_t stage = 128u * 64u * 2u + nb64 * 64u * 64u * 2u;  // bf16: A tile + r/64 boxes
+  // B Q / B^T P (CTA pairs): A tile + per 256-column part of N, this CTA's half (two 64-column boxes)
+  const uint32_t bq_boxes = 2u * (uint32_t)std::max(1, ((lo.max_r + 15) / 16 * 16 + 255) / 256);
+  const uint32_t stage = 128u * 64u * 2u + bq_boxes * 64u * 64u * 2u;
   const int stages = (int)std::min<uint32_t>(4u, budget / stage);
   const uint32_t nb128 = (uint32_t)std::max(1, (lo.max_r + 127) / 128);
   const uint32_t ostage = 128u * 32u * 4u * (1u + nb128);  // fp32: A box + r/128 B boxes
   const int ostages = (int)std::min<uint32_t>(4u, budget / ostage);
   if (stages < 2 || ostages < 2) return cudaErrorInvalidValue;
   tp->nb64 = nb64;
+  tp->bq_boxes = bq_boxes;
   tp->nb128 = nb128;
   tp->f_stages = tp->r_stages = stages;
   tp->o_stages = ostages;

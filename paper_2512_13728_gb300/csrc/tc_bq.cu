@@ -161,8 +161,13 @@ enum : int { GEMM_BQ = 0, GEMM_BTP = 1 };
 //                  both MN-major boxes of the row-major copies.  Epilogue: R, bf16 R, column
 //                  sums of squares.
 // Both run on layers that take the Dion branch only.
+// Run in clusters of two CTAs that compute 256-row blocks with pair MMAs (cta_group::2): CTA c
+// of the pair owns 128-row tile 2 p + c, holds that tile's A chunk and, of every N part of up
+// to 256 columns, the half c of its B columns, and receives its 128 rows of the accumulator
+// in its own TMEM.  Per SM and k-chunk that is 16 KB of A and 32 KB of B (r = 512) instead of
+// 16 + 64 KB.  Tile = {layer, pair p}.
 template <int KIND>
-__global__ void __launch_bounds__(R_THREADS, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(R_THREADS, 1)
     tc_tma_gemm_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off,
                        const LayerMaps *__restrict__ maps, int nstages, uint32_t stage_bytes, uint32_t tmem_cols) {
   extern __shared__ uint8_t smem_raw[];
@@ -175,60 +180,75 @@ __global__ void __launch_bounds__(R_THREADS, 1)
   __shared__ int abort_s;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const Abort ab{&abort_s};
+  const uint32_t rank = cluster_ctarank();
+  const int seg = blockIdx.x >> 1;
   if (threadIdx.x == 0) {
     for (int i = 0; i < nstages; ++i) {
-      mbar_init(&full[i], 1);
-      mbar_init(&empty[i], 1);
+      mbar_init(&full[i], 1);   // used in CTA 0: its arm, both CTAs' bytes
+      mbar_init(&empty[i], 1);  // pair commit after the stage's MMAs
     }
-    mbar_init(acc_full, 1);
-    mbar_init(acc_empty, 128);
+    mbar_init(acc_full, 1);   // pair commit after the tile's MMAs
+    mbar_init(acc_empty, 2);  // used in CTA 0: one arrival per CTA's epilogue
     mbar_init(drain, 1);
     abort_s = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc(&tmem_base_s, tmem_cols);
-    tmem_relinquish();
+    tmem_alloc_pair(&tmem_base_s, tmem_cols);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  cluster_sync();  // both CTAs' barriers and TMEM exist before anything crosses the pair
   const uint32_t tmem = tmem_base_s;
+  // N parts of up to 256 columns; each CTA holds half of a part's columns (64-column boxes)
+  auto half_cols = [](uint32_t np, uint32_t part) { return min(256u, np - part * 256u) / 2u; };
 
   if (warp == 0) {
     if (lane == 0) {
       uint32_t it = 0;
       bool ok = true;
-      for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
+      for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
         if (!sh.active[t.x]) continue;
         const DevLayer &L = sh.layers[t.x];
         const LayerMaps *mp = maps + t.x;
         const int kch = (int)(((KIND == GEMM_BQ ? L.n : L.m) + 63) / 64);
-        const int nb = (int)((L.r + 63) / 64);
+        const int tr = 2 * t.y + (int)rank;  // past the last tile: zero-filled, not stored
+        const uint32_t np = rpad16(L.r), nparts = (np + 255) / 256;
+        uint32_t nbox = 0;  // 64-column B boxes per CTA and k-chunk
+        for (uint32_t part = 0; part < nparts; ++part) nbox += (half_cols(np, part) + 63) / 64;
         for (int kc = 0; kc < kch; ++kc, ++it) {
           const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
           if (!ab.wait(&empty[s], ph ^ 1u, sh.status)) { ok = false; break; }
           uint8_t *sA = smem + s * stage_bytes, *sB = sA + OPB_A;
-          mbar_expect_tx(&full[s], OPB_A + (uint32_t)nb * BOX64);
+          const uint32_t fb = cluster_addr(&full[s], 0);
+          if (rank == 0) mbar_expect_tx(&full[s], 2u * (OPB_A + nbox * BOX64));
           if (KIND == GEMM_BQ) {
-            tma_load_2d(sA, &mp->Bh_k, &full[s], kc * 64, t.y * 128);
-            for (int j = 0; j < nb; ++j) tma_load_2d(sB + j * BOX64, &mp->Qn_mn, &full[s], j * 64, kc * 64);
+            tma_load_2d_pair(sA, &mp->Bh_k, fb, kc * 64, tr * 128);
           } else {
-            tma_load_2d(sA, &mp->Bh_mn, &full[s], t.y * 128, kc * 64);
-            tma_load_2d(sA + BOX64, &mp->Bh_mn, &full[s], t.y * 128 + 64, kc * 64);
-            for (int j = 0; j < nb; ++j) tma_load_2d(sB + j * BOX64, &mp->P_mn, &full[s], j * 64, kc * 64);
+            tma_load_2d_pair(sA, &mp->Bh_mn, fb, tr * 128, kc * 64);
+            tma_load_2d_pair(sA + BOX64, &mp->Bh_mn, fb, tr * 128 + 64, kc * 64);
+          }
+          const CUtensorMap *bmap = (KIND == GEMM_BQ) ? &mp->Qn_mn : &mp->P_mn;
+          for (uint32_t part = 0; part < nparts; ++part) {
+            const uint32_t hc = half_cols(np, part);
+            const int x0 = (int)(part * 256u + rank * hc);
+            for (uint32_t j = 0; j < (hc + 63) / 64; ++j)
+              tma_load_2d_pair(sB + (part * 2u + j) * BOX64, bmap, fb, x0 + (int)j * 64, kc * 64);
           }
         }
       }
+      // drain: the last stages' loads have landed and been consumed (their stage was freed)
       for (uint32_t k = (it > (uint32_t)nstages ? it - nstages : 0); k < it; ++k)
-        mbar_wait(&full[k % nstages], (k / nstages) & 1u, sh.status);
+        mbar_wait(&empty[k % nstages], (k / nstages) & 1u, sh.status);
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && rank == 0) {
       uint32_t it = 0, tcount = 0;
       bool ok = true;
-      for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
+      for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
         if (!sh.active[t.x]) continue;
         const DevLayer &L = sh.layers[t.x];
@@ -247,45 +267,50 @@ __global__ void __launch_bounds__(R_THREADS, 1)
             const uint64_t ad = (KIND == GEMM_BQ) ? smem_desc_sw128(aB + k16 * 32, 0, 1024)
                                                   : smem_desc_sw128(aB + k16 * 2048, BOX64, 1024);
             for (uint32_t part = 0; part < nparts; ++part) {
-              const uint32_t n_here = min(256u, np - part * 256u);
-              const uint64_t bd = smem_desc_sw128(bB + part * 4u * BOX64 + k16 * 2048, BOX64, 1024);
-              umma_bf16(tmem + part * 256u, ad, bd, idesc_bf16(128, n_here, KIND == GEMM_BTP, true),
-                        (kc | k16) ? 1u : 0u);
+              const uint32_t n_here = 2u * half_cols(np, part);
+              const uint64_t bd = smem_desc_sw128(bB + part * 2u * BOX64 + k16 * 2048, BOX64, 1024);
+              umma_pair_bf16(tmem + part * 256u, ad, bd, idesc_bf16(256, n_here, KIND == GEMM_BTP, true),
+                             (kc | k16) ? 1u : 0u);
             }
           }
-          umma_commit(&empty[s]);
+          umma_pair_commit_mc(&empty[s], 0x3);  // the stage is free in both CTAs
         }
         if (!ok) break;
-        umma_commit(acc_full);
+        umma_pair_commit_mc(acc_full, 0x3);
         ++tcount;
       }
-      umma_commit(drain);
+      umma_pair_commit(drain);  // every MMA of the pair has completed before TMEM is freed
       mbar_wait(drain, 0, sh.status);
     }
   } else {
     const bool leader = (warp == 2 && lane == 0);
     uint32_t tcount = 0, ecount = 0;
-    for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1]; ++ti) {
+    for (int ti = off[seg]; ti < off[seg + 1]; ++ti) {
       const int4 t = tiles[ti];
       if (!sh.active[t.x]) continue;
       const DevLayer &L = sh.layers[t.x];
+      const int tr = 2 * t.y + (int)rank;
       if (!named_and(1, 128, ab.wait(acc_full, tcount & 1u, sh.status))) break;
       tc_fence_after();
-      if (KIND == GEMM_BQ)
-        store_accumulator(tmem, warp, lane, leader, stg, &maps[t.x].Praw, &maps[t.x].PTraw_t, L.r, L.m, t.y * 128,
-                          ecount, 1, 0, 1);
-      else
-        store_r_tile(tmem, warp, lane, leader, stg, maps[t.x], L, t.y, ecount);
+      if ((int64_t)tr * 128 < (KIND == GEMM_BQ ? L.m : L.n)) {  // not the pair's empty second tile
+        if (KIND == GEMM_BQ)
+          store_accumulator(tmem, warp, lane, leader, stg, &maps[t.x].Praw, &maps[t.x].PTraw_t, L.r, L.m, tr * 128,
+                            ecount, 1, 0, 1);
+        else
+          store_r_tile(tmem, warp, lane, leader, stg, maps[t.x], L, tr, ecount);
+      }
       tc_fence_before();
-      mbar_arrive(acc_empty);
+      named_sync(1, 128);  // every thread's TMEM reads of this accumulator are done
+      if (leader) mbar_arrive_cluster(cluster_addr(acc_empty, 0));
       ++tcount;
     }
     if (leader) bulk_wait<0>();
   }
   tc_fence_before();
   __syncthreads();
+  cluster_sync();  // both CTAs are done with the pair's TMEM and barriers
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem, tmem_cols);
+  if (warp == 1) tmem_dealloc_pair(tmem, tmem_cols);
 }
 
 // ================================================================== Q -> bf16 copy ===
@@ -315,16 +340,16 @@ cudaError_t setup_bq_kernels(uint32_t f_smem, uint32_t r_smem) {
 
 void launch_form_bq(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
   if (tp.d_bq.grid <= 0) return;
-  const uint32_t stage = OPB_A + tp.nb64 * BOX64;
-  tc_tma_gemm_kernel<GEMM_BQ><<<tp.d_bq.grid, R_THREADS, tp.f_smem, s>>>(sh, tp.d_bq.tiles, tp.d_bq.off, tp.maps,
-                                                                         tp.f_stages, stage, tp.tmem_cols);
+  const uint32_t stage = OPB_A + tp.bq_boxes * BOX64;
+  tc_tma_gemm_kernel<GEMM_BQ><<<2 * tp.d_bq.grid, R_THREADS, tp.f_smem, s>>>(sh, tp.d_bq.tiles, tp.d_bq.off,
+                                                                             tp.maps, tp.f_stages, stage, tp.tmem_cols);
 }
 
 void launch_btp(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
   if (tp.d_btp.grid <= 0) return;
-  const uint32_t stage = OPB_A + tp.nb64 * BOX64;
-  tc_tma_gemm_kernel<GEMM_BTP><<<tp.d_btp.grid, R_THREADS, tp.r_smem, s>>>(sh, tp.d_btp.tiles, tp.d_btp.off, tp.maps,
-                                                                           tp.r_stages, stage, tp.tmem_cols);
+  const uint32_t stage = OPB_A + tp.bq_boxes * BOX64;
+  tc_tma_gemm_kernel<GEMM_BTP><<<2 * tp.d_btp.grid, R_THREADS, tp.r_smem, s>>>(sh, tp.d_btp.tiles, tp.d_btp.off,
+                                                                               tp.maps, tp.r_stages, stage, tp.tmem_cols);
 }
 
 void launch_qn_refresh(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
