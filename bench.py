@@ -145,6 +145,19 @@ class ClockSampler:
 
 # --------------------------------------------------------------------- our GPU arm ---
 
+def max_over_ranks(value: float, world: int, device) -> float:
+    """The slowest replica's time: every rank contributes its own, every rank gets the max
+    (NCCL on the GPU in the bench; any backend whose tensors live on `device`)."""
+    if world <= 1:
+        return float(value)
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([float(value)], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
 
@@ -214,10 +227,7 @@ def run_ours(args, rank, world, local_rank):
     ms_total = e0.elapsed_time(e1)
     nsteps_timed, ktimes = cd.native.dion_timing_read(plan.handle)
     cd.native.dion_timing_enable(plan.handle, 0)
-    if world > 1:
-        tt = torch.tensor([ms_total], device=dev, dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms_total = float(tt.item())
+    ms_total = max_over_ranks(ms_total, world, dev)
     if plan.device_status() != 0:
         raise RuntimeError("device status after timed steps is not OK")
     ms_step = ms_total / args.steps
@@ -243,10 +253,7 @@ def run_ours(args, rank, world, local_rank):
     f1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = f0.elapsed_time(f1) / e_steps
-    if world > 1:
-        tt = torch.tensor([e2e_ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
+    e2e_ms = max_over_ranks(e2e_ms, world, dev)
     launches = plan.launches_per_step()
     plan.close()
     if rank != 0:
