@@ -470,6 +470,83 @@ __device__ bool chol_inverse(const float *__restrict__ S, float *__restrict__ W,
   return true;
 }
 
+// ||S - I||_2 estimated by 8 power iterations.  S - I is symmetric, so each product reads only
+// the 32 x 32 tiles on and below the diagonal (half of S, which stays in L2 across the
+// iterations): warp w takes tiles w, w + 16, ... and adds each tile's row sums (a
+// reduce-scatter over the lanes) and, off the diagonal, its column sums into its own partial
+// vector; the partials are then summed in warp order, so the estimate is deterministic.
+// Shared memory: Y (at least 18 rows of ldy floats).  Called by the whole block.
+__device__ __noinline__ float power_norm_sym(const float *__restrict__ S, int r, int64_t ls, float *Y, int ldy) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  __shared__ float wn[kCholThreads / 32];
+  __shared__ float lam_s;
+  float lam = INFINITY;
+  float *part = Y;                  // 16 rows of ldy: one partial vector per warp
+  float *pv = Y + 16 * ldy, *wv = Y + 17 * ldy;
+  for (int i = tid; i < r; i += kCholThreads) pv[i] = 1.f + 0.25f * __sinf(0.7f * (float)i);  // fixed start
+  const int nt = (r + 31) / 32, ntiles = nt * (nt + 1) / 2;
+  __syncthreads();
+  for (int itp = 0; itp < 8; ++itp) {
+    float *mine = part + warp * ldy;
+    for (int i = lane; i < r; i += 32) mine[i] = 0.f;
+    __syncwarp();
+    for (int p = warp; p < ntiles; p += kCholThreads / 32) {
+      const int bi = trap_row(p, 1), bj = p - bi * (bi + 1) / 2;  // tile row bi >= tile column bj
+      const int c = bj * 32 + lane;
+      const float vc = (c < r) ? pv[c] : 0.f;
+      float a[32], colsum = 0.f;
+#pragma unroll
+      for (int y = 0; y < 32; ++y) {
+        const int row = bi * 32 + y;
+        float e = 0.f;
+        if (row < r && c < r) e = S[(int64_t)row * ls + c] - (row == c ? 1.f : 0.f);
+        a[y] = e * vc;
+        if (bi != bj) colsum = fmaf(e, (row < r) ? pv[row] : 0.f, colsum);
+      }
+      // reduce-scatter: lane y ends with sum over the lanes of a[y] (row y of the tile)
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const bool upper = (lane & o) != 0;
+#pragma unroll
+        for (int k = 0; k < o; ++k) {
+          const float send = upper ? a[k] : a[k + o];
+          const float keep = upper ? a[k + o] : a[k];
+          a[k] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+      }
+      if (bi * 32 + lane < r) mine[bi * 32 + lane] += a[0];
+      __syncwarp();
+      if (bi != bj && c < r) mine[c] += colsum;
+      __syncwarp();
+    }
+    __syncthreads();
+    float pn = 0.f;
+    for (int i = tid; i < r; i += kCholThreads) {
+      float yv = 0.f;
+      for (int w = 0; w < kCholThreads / 32; ++w) yv += part[w * ldy + i];
+      wv[i] = yv;
+      pn = fmaf(yv, yv, pn);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) pn += __shfl_xor_sync(0xffffffffu, pn, o);
+    if (lane == 0) wn[warp] = pn;
+    __syncthreads();
+    if (tid == 0) {
+      float a = 0.f;
+      for (int w = 0; w < kCholThreads / 32; ++w) a += wn[w];
+      lam_s = a;  // ||E v||^2
+    }
+    __syncthreads();
+    const float nrm = sqrtf(lam_s);
+    lam = nrm;  // ||E v|| / ||v||: v has unit norm from the second iteration on
+    const float inv = (nrm > 0.f && isfinite(nrm)) ? 1.f / nrm : 0.f;
+    for (int i = tid; i < r; i += kCholThreads) pv[i] = wv[i] * inv;
+    __syncthreads();
+    if (itp == 0) lam = INFINITY;  // the first product uses an unnormalized start vector
+  }
+  return lam;
+}
+
 // pass 0 and 1: every active layer; pass 2: only layers marked by a shifted retry.
 // Passes 1 and 2 factor the Gram matrix of an already nearly orthonormal X.  With E = S - I,
 // when 1.5 times a bound on ||E||_2 is below near_identity, the factor of S = I + E is taken
@@ -512,52 +589,14 @@ __global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, in
     __syncthreads();
     float lam = lam_s;
     if (!(isfinite(lam) && 1.5f * lam < near_identity)) {
-      // ||E||_2 by 8 power iterations (one warp per row, coalesced row reads of the full S)
-      float *pv = Y, *wv = Y + ldy;
-      __shared__ float wn[kCholThreads / 32];
-      for (int i = tid; i < r; i += kCholThreads) pv[i] = 1.f + 0.25f * __sinf(0.7f * (float)i);  // fixed start
-      __syncthreads();
-      for (int itp = 0; itp < 8; ++itp) {
-        for (int i = warp; i < r; i += kCholThreads / 32) {
-          float acc0 = 0.f, acc1 = 0.f;
-          int j = lane;
-          for (; j + 32 < r; j += 64) {
-            acc0 = fmaf(S[(int64_t)i * ls + j] - (i == j ? 1.f : 0.f), pv[j], acc0);
-            acc1 = fmaf(S[(int64_t)i * ls + j + 32] - (i == j + 32 ? 1.f : 0.f), pv[j + 32], acc1);
-          }
-          if (j < r) acc0 = fmaf(S[(int64_t)i * ls + j] - (i == j ? 1.f : 0.f), pv[j], acc0);
-          float acc = acc0 + acc1;
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-          if (lane == 0) wv[i] = acc;
-        }
-        __syncthreads();
-        float pn = 0.f;
-        for (int i = tid; i < r; i += kCholThreads) pn = fmaf(wv[i], wv[i], pn);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) pn += __shfl_xor_sync(0xffffffffu, pn, o);
-        if (lane == 0) wn[warp] = pn;
-        __syncthreads();
-        if (tid == 0) {
-          float a = 0.f;
-          for (int w = 0; w < kCholThreads / 32; ++w) a += wn[w];
-          lam_s = a;  // ||E v||^2
-        }
-        __syncthreads();
-        const float nrm = sqrtf(lam_s);
-        lam = nrm;  // ||E v|| / ||v||: v has unit norm from the second iteration on
-        const float inv = (nrm > 0.f && isfinite(nrm)) ? 1.f / nrm : 0.f;
-        for (int i = tid; i < r; i += kCholThreads) pv[i] = wv[i] * inv;
-        __syncthreads();
-        if (itp == 0) lam = INFINITY;  // the first product uses an unnormalized start vector
-      }
+      lam = power_norm_sym(S, r, ls, Y, ldy);
     }
     if (isfinite(lam) && 1.5f * lam < near_identity) {
-      for (int64_t e = tid; e < (int64_t)r * r; e += kCholThreads) {
-        const int64_t i = e / r, j = e % r;
-        const float sij = (j <= i) ? S[i * ls + j] : 0.f;
-        Li[i * ls + j] = (j < i) ? -sij : (j == i ? 1.f - 0.5f * (sij - 1.f) : 0.f);
-      }
+      for (int i = warp; i < r; i += kCholThreads / 32)
+        for (int j = lane; j < r; j += 32) {
+          const float sij = (j <= i) ? S[(int64_t)i * ls + j] : 0.f;
+          Li[(int64_t)i * ls + j] = (j < i) ? -sij : (j == i ? 1.f - 0.5f * (sij - 1.f) : 0.f);
+        }
       return;
     }
   }
