@@ -383,8 +383,8 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
   };
   lo.s_bq = pair_sched(pairs_of(lo.ftiles), [&](const int4 &t) { return (double)layers[t.x].n + 2.0 * layers[t.x].r; });
   lo.s_btp = pair_sched(pairs_of(lo.rtiles), [&](const int4 &t) { return (double)layers[t.x].m + 2.0 * layers[t.x].r; });
-  lo.s_gram = sched(lo.gram_tiles, [&](const int4 &t) { return (double)layers[t.x].m * layers[t.x].r; });
-  lo.s_trsm = sched(lo.trsm_tiles, [&](const int4 &t) { return 3.0 * layers[t.x].r + 64.0; });
+  lo.s_gram = pair_sched(pairs_of(lo.gram_tiles), [&](const int4 &t) { return (double)layers[t.x].m * layers[t.x].r; });
+  lo.s_trsm = pair_sched(pairs_of(lo.trsm_tiles), [&](const int4 &t) { return 3.0 * layers[t.x].r + 64.0; });
   for (Schedule *sc : {&lo.s_update, &lo.s_bq, &lo.s_btp, &lo.s_gram, &lo.s_trsm}) {
     sc->o_tiles = take(sizeof(int4) * std::max<size_t>(sc->tiles.size(), 1));
     sc->o_off = take(sizeof(int) * sc->off.size());
@@ -506,12 +506,15 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   const uint32_t stage = 128u * 64u * 2u + bq_boxes * 64u * 64u * 2u;
   const int stages = (int)std::min<uint32_t>(4u, budget / stage);
   const uint32_t nb128 = (uint32_t)std::max(1, (lo.max_r + 127) / 128);
-  const uint32_t ostage = 128u * 32u * 4u * (1u + nb128);  // fp32: A box + r/128 B boxes
+  // Gram / TRSM (CTA pairs): A box + per 256-column part of N, this CTA's half (one 128-row box)
+  const uint32_t o_parts = (uint32_t)std::max(1, ((lo.max_r + 15) / 16 * 16 + 255) / 256);
+  const uint32_t ostage = 128u * 32u * 4u * (1u + o_parts);
   const int ostages = (int)std::min<uint32_t>(4u, budget / ostage);
   if (stages < 2 || ostages < 2) return cudaErrorInvalidValue;
   tp->nb64 = nb64;
   tp->bq_boxes = bq_boxes;
   tp->nb128 = nb128;
+  tp->o_parts = o_parts;
   tp->f_stages = tp->r_stages = stages;
   tp->o_stages = ostages;
   tp->f_smem = form_bq_smem(stages, stage);

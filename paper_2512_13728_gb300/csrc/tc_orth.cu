@@ -14,7 +14,8 @@
 // Accuracy: tf32 products (10-bit mantissa) with fp32 accumulation give ~5e-4 relative
 // error in S and Y; the second CholeskyQR pass (on an already nearly orthonormal X) brings
 // P back to orthonormal to that level, below the bf16 rounding the following kernels apply.
-// Roles: warp 0 TMA, warp 1 MMA (+ TMEM), warps 2..5 epilogue.
+// Both run as pair MMAs over 256-row blocks (two CTAs on two SMs, cta_group::2), so each SM
+// receives half of the B operand.  Roles: warp 0 TMA, warp 1 MMA (even CTA), warps 2..5 epilogue.
 #include "tc.cuh"
 #include "tc_common.cuh"
 #include "tc_kernels.cuh"
@@ -71,8 +72,14 @@ __device__ __forceinline__ bool part_needs(int kc, uint32_t part) {
   return KIND == ORTH_GRAM || (uint32_t)kc * 32u < 256u * (part + 1u);
 }
 
+// Run in clusters of two CTAs with pair MMAs (cta_group::2, M = 256): CTA c of the pair owns
+// 128-row tile 2 p + c (rows of S for the Gram, rows of X for the TRSM), its A chunk, and of
+// every N part of up to 256 columns the half c of the B rows; the even CTA issues the MMAs and
+// each CTA receives its 128 rows of the accumulator in its own TMEM.  For the Gram with a
+// full 256-column part the tile's own rows of X^T are exactly the CTA's B half of part p,
+// so A is read in place.  Tile = {layer, pair p}.
 template <int KIND>
-__global__ void __launch_bounds__(O_THREADS, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
     tc_orth_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off, const LayerMaps *__restrict__ maps,
                    int pass, int nstages, uint32_t stage_bytes, uint32_t tmem_cols) {
   extern __shared__ uint8_t smem_raw[];
@@ -85,32 +92,37 @@ __global__ void __launch_bounds__(O_THREADS, 1)
   __shared__ int abort_s;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const Abort ab{&abort_s};
+  const uint32_t rank = cluster_ctarank();
+  const int seg = blockIdx.x >> 1;
   if (threadIdx.x == 0) {
     for (int i = 0; i < nstages; ++i) {
-      mbar_init(&full[i], 1);
-      mbar_init(&empty[i], 1);
+      mbar_init(&full[i], 1);   // used in CTA 0: its arm, both CTAs' bytes
+      mbar_init(&empty[i], 1);  // pair commit after the stage's MMAs
     }
-    mbar_init(acc_full, 1);
-    mbar_init(acc_empty, 128);
+    mbar_init(acc_full, 1);   // pair commit after the tile's MMAs
+    mbar_init(acc_empty, 2);  // used in CTA 0: one arrival per CTA's epilogue
     mbar_init(drain, 1);
     abort_s = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc(&tmem_base_s, tmem_cols);
-    tmem_relinquish();
+    tmem_alloc_pair(&tmem_base_s, tmem_cols);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  cluster_sync();  // both CTAs' barriers and TMEM exist before anything crosses the pair
   const uint32_t tmem = tmem_base_s;
   auto skip = [&](int layer) { return !sh.active[layer] || (pass == 2 && !sh.orth_shifted[layer]); };
+  // half of N part q held by each CTA (rows of the B operand)
+  auto half_rows = [](uint32_t N, uint32_t q) { return min(256u, N - q * 256u) / 2u; };
 
   if (warp == 0) {
     if (lane == 0) {
       uint32_t it = 0;
       bool ok = true;
-      for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
+      for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
         if (skip(t.x)) continue;
         const DevLayer &L = sh.layers[t.x];
@@ -119,28 +131,33 @@ __global__ void __launch_bounds__(O_THREADS, 1)
         int64_t K;
         orth_dims<KIND>(L, t.y, N, K);
         const int kch = (int)((K + 31) / 32);
-        const uint32_t nboxes = (N + 127) / 128;
+        const uint32_t nparts = (N + 255) / 256;
+        const int tr = 2 * t.y + (int)rank;  // past the last tile: zero-filled, not stored
+        const bool a_in_b = (KIND == ORTH_GRAM) && (uint32_t)t.y < nparts && half_rows(N, (uint32_t)t.y) == 128u;
         for (int kc = 0; kc < kch; ++kc, ++it) {
           const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
           if (!ab.wait(&empty[s], ph ^ 1u, sh.status)) { ok = false; break; }
           uint8_t *sA = smem + s * stage_bytes, *sB = sA + O_BOX;
+          const uint32_t fb = cluster_addr(&full[s], 0);
           uint32_t nb = 0;  // B boxes this chunk feeds (all, or only the lower-triangular parts)
-          for (uint32_t b = 0; b < nboxes; ++b)
-            if (part_needs<KIND>(kc, b / 2)) ++nb;
-          mbar_expect_tx(&full[s], O_BOX * ((KIND == ORTH_GRAM ? 0 : 1) + nb));
-          if (KIND != ORTH_GRAM) tma_load_2d(sA, om.A, &full[s], kc * 32, t.y * 128);
-          for (uint32_t b = 0; b < nboxes; ++b)
-            if (part_needs<KIND>(kc, b / 2)) tma_load_2d(sB + b * O_BOX, om.B, &full[s], kc * 32, b * 128);
+          for (uint32_t q = 0; q < nparts; ++q)
+            if (part_needs<KIND>(kc, q)) ++nb;
+          if (rank == 0) mbar_expect_tx(&full[s], 2u * O_BOX * ((a_in_b ? 0u : 1u) + nb));
+          if (!a_in_b) tma_load_2d_pair(sA, om.A, fb, kc * 32, tr * 128);
+          for (uint32_t q = 0; q < nparts; ++q)
+            if (part_needs<KIND>(kc, q))
+              tma_load_2d_pair(sB + q * O_BOX, om.B, fb, kc * 32, (int)(q * 256u + rank * half_rows(N, q)));
         }
       }
+      // drain: the last stages' loads have landed and been consumed (their stage was freed)
       for (uint32_t k = (it > (uint32_t)nstages ? it - nstages : 0); k < it; ++k)
-        mbar_wait(&full[k % nstages], (k / nstages) & 1u, sh.status);
+        mbar_wait(&empty[k % nstages], (k / nstages) & 1u, sh.status);
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && rank == 0) {
       uint32_t it = 0, tcount = 0;
       bool ok = true;
-      for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1] && ok; ++ti) {
+      for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
         if (skip(t.x)) continue;
         const DevLayer &L = sh.layers[t.x];
@@ -149,6 +166,7 @@ __global__ void __launch_bounds__(O_THREADS, 1)
         orth_dims<KIND>(L, t.y, N, K);
         const int kch = (int)((K + 31) / 32);
         const uint32_t nparts = (N + 255) / 256;
+        const bool a_in_b = (KIND == ORTH_GRAM) && (uint32_t)t.y < nparts && half_rows(N, (uint32_t)t.y) == 128u;
         if (!ab.wait(acc_empty, (tcount & 1u) ^ 1u, sh.status)) break;
         tc_fence_after();
         for (int kc = 0; kc < kch; ++kc, ++it) {
@@ -156,25 +174,25 @@ __global__ void __launch_bounds__(O_THREADS, 1)
           if (!ab.wait(&full[s], ph, sh.status)) { ok = false; break; }
           tc_fence_after();
           const uint32_t aB = smem_u32(smem + s * stage_bytes), bB = aB + O_BOX;
+          const uint32_t aSrc = a_in_b ? bB + (uint32_t)t.y * O_BOX : aB;
 #pragma unroll
           for (int k8 = 0; k8 < 4; ++k8) {
-            // Gram: the tile's rows are B box t.y of the same stage
-            const uint64_t ad = smem_desc_sw128((KIND == ORTH_GRAM ? bB + (uint32_t)t.y * O_BOX : aB) + k8 * 32, 0, 1024);
-            for (uint32_t part = 0; part < nparts; ++part) {
-              if (!part_needs<KIND>(kc, part)) continue;
-              const uint32_t n_here = min(256u, N - part * 256u);
-              const uint64_t bd = smem_desc_sw128(bB + part * 2u * O_BOX + k8 * 32, 0, 1024);
+            const uint64_t ad = smem_desc_sw128(aSrc + k8 * 32, 0, 1024);
+            for (uint32_t q = 0; q < nparts; ++q) {
+              if (!part_needs<KIND>(kc, q)) continue;
+              const uint64_t bd = smem_desc_sw128(bB + q * O_BOX + k8 * 32, 0, 1024);
               // the first chunk that feeds a part starts its accumulation
-              umma_tf32(tmem + part * 256u, ad, bd, idesc_tf32(128, n_here, false, false), (kc | k8) ? 1u : 0u);
+              umma_pair_tf32(tmem + q * 256u, ad, bd, idesc_tf32(256, 2u * half_rows(N, q), false, false),
+                             (kc | k8) ? 1u : 0u);
             }
           }
-          umma_commit(&empty[s]);
+          umma_pair_commit_mc(&empty[s], 0x3);  // the stage is free in both CTAs
         }
         if (!ok) break;
-        umma_commit(acc_full);
+        umma_pair_commit_mc(acc_full, 0x3);
         ++tcount;
       }
-      umma_commit(drain);
+      umma_pair_commit(drain);  // every MMA of the pair has completed before TMEM is freed
       mbar_wait(drain, 0, sh.status);
     }
   } else {
@@ -182,7 +200,7 @@ __global__ void __launch_bounds__(O_THREADS, 1)
     const bool leader = (warp == 2 && lane == 0);
     const uint32_t lg = (uint32_t)(warp & 3), row = 32u * lg + lane;
     uint32_t tcount = 0, ecount = 0;
-    for (int ti = off[blockIdx.x]; ti < off[blockIdx.x + 1]; ++ti) {
+    for (int ti = off[seg]; ti < off[seg + 1]; ++ti) {
       const int4 t = tiles[ti];
       if (skip(t.x)) continue;
       const DevLayer &L = sh.layers[t.x];
@@ -190,9 +208,11 @@ __global__ void __launch_bounds__(O_THREADS, 1)
       uint32_t N;
       int64_t K;
       orth_dims<KIND>(L, t.y, N, K);
+      const int tr = 2 * t.y + (int)rank;
       if (!named_and(1, 128, ab.wait(acc_full, tcount & 1u, sh.status))) break;
       tc_fence_after();
-      const int nch = (int)((min((int64_t)N, L.r) + 31) / 32);
+      const bool real = (int64_t)tr * 128 < (KIND == ORTH_GRAM ? L.r : L.m);  // not the pair's empty second tile
+      const int nch = real ? (int)((min((int64_t)N, L.r) + 31) / 32) : 0;
       // The solve that ends Orthogonalize writes only the bf16 copy of P that R = B^T P and the
       // update read: pass 1 unless a shifted retry asked for pass 2, and pass 2 itself.
       const bool final_pass = (KIND == ORTH_TRSM) && (pass == 2 || (pass == 1 && !sh.orth_shifted[t.x]));
@@ -226,7 +246,7 @@ __global__ void __launch_bounds__(O_THREADS, 1)
           fence_async_smem();
           named_sync(1, 128);
           if (leader) {
-            tma_store_2d(&maps[t.x].P_hi, hb, j * 32, t.y * 128);
+            tma_store_2d(&maps[t.x].P_hi, hb, j * 32, tr * 128);
             bulk_commit();
           }
           ++ecount;
@@ -256,26 +276,28 @@ __global__ void __launch_bounds__(O_THREADS, 1)
           fence_async_smem();
           named_sync(1, 128);
           if (leader) {
-            tma_store_2d(om.out, box, j * 32, t.y * 128);
+            tma_store_2d(om.out, box, j * 32, tr * 128);
             if (store_t)
               for (int w4 = 0; w4 < 4; ++w4)
-                if ((int64_t)t.y * 128 + w4 * 32 < L.m)
-                  tma_store_2d(om.out_t, stg + eb * 2 * O_BOX + O_BOX + w4 * O_TBOX, t.y * 128 + w4 * 32, j * 32);
+                if ((int64_t)tr * 128 + w4 * 32 < L.m)
+                  tma_store_2d(om.out_t, stg + eb * 2 * O_BOX + O_BOX + w4 * O_TBOX, tr * 128 + w4 * 32, j * 32);
             bulk_commit();
           }
           ++ecount;
         }
       }
       tc_fence_before();
-      mbar_arrive(acc_empty);
+      named_sync(1, 128);  // every thread's TMEM reads of this accumulator are done
+      if (leader) mbar_arrive_cluster(cluster_addr(acc_empty, 0));
       ++tcount;
     }
     if (leader) bulk_wait<0>();
   }
   tc_fence_before();
   __syncthreads();
+  cluster_sync();  // both CTAs are done with the pair's TMEM and barriers
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem, tmem_cols);
+  if (warp == 1) tmem_dealloc_pair(tmem, tmem_cols);
 }
 
 uint32_t orth_smem(int nstages, uint32_t stage_bytes) { return 1024u + nstages * stage_bytes + 4u * O_BOX + 512u; }
@@ -291,13 +313,13 @@ cudaError_t setup_orth_kernels(uint32_t smem) {
 void launch_orth(const Shared &sh, const TcPlan &tp, bool gram, int pass, cudaStream_t s) {
   const DevSchedule &d = gram ? tp.d_gram : tp.d_trsm;
   if (d.grid <= 0) return;
-  const uint32_t stage = O_BOX * (1 + tp.nb128);
+  const uint32_t stage = O_BOX * (1 + tp.o_parts);
   if (gram)
-    tc_orth_kernel<ORTH_GRAM><<<d.grid, O_THREADS, tp.o_smem, s>>>(sh, d.tiles, d.off, tp.maps, pass, tp.o_stages,
-                                                                     stage, tp.tmem_cols);
+    tc_orth_kernel<ORTH_GRAM><<<2 * d.grid, O_THREADS, tp.o_smem, s>>>(sh, d.tiles, d.off, tp.maps, pass,
+                                                                         tp.o_stages, stage, tp.tmem_cols);
   else
-    tc_orth_kernel<ORTH_TRSM><<<d.grid, O_THREADS, tp.o_smem, s>>>(sh, d.tiles, d.off, tp.maps, pass, tp.o_stages,
-                                                                     stage, tp.tmem_cols);
+    tc_orth_kernel<ORTH_TRSM><<<2 * d.grid, O_THREADS, tp.o_smem, s>>>(sh, d.tiles, d.off, tp.maps, pass,
+                                                                         tp.o_stages, stage, tp.tmem_cols);
 }
 
 }  // namespace tc
