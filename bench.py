@@ -294,8 +294,12 @@ def run_ours(args, rank, world, local_rank):
                    [list(s) for s in w.shapes[:6]], "gate_mode": args.gate, "precision": prec,
                    "l2": "no flush: each step streams far more than the 129 MB L2",
                    "matrices_per_s": round(world * w.num_layers / (ms_step * 1e-3), 1),
-                   "step_hbm_frac_planned_bytes": round(planned / (ms_step * 1e-3) / 1e9 / peaks["hbm"], 4),
-                   "step_hbm_frac_compulsory_bytes": round(compulsory / (ms_step * 1e-3) / 1e9 / peaks["hbm"], 4),
+                   # byte models of a step in which every layer syncs; a gated run takes the cheaper
+                   # local branch on most layers, so they are reported for --gate always only
+                   "step_hbm_frac_planned_bytes": round(planned / (ms_step * 1e-3) / 1e9 / peaks["hbm"], 4)
+                   if args.gate == "always" else None,
+                   "step_hbm_frac_compulsory_bytes": round(compulsory / (ms_step * 1e-3) / 1e9 / peaks["hbm"], 4)
+                   if args.gate == "always" else None,
                    "parallelism": f"replicas x{world}"},
         "roofline": roofline,
         "e2e": {"value": round(e2e_ms, 4), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
