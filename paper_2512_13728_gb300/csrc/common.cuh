@@ -85,6 +85,7 @@ struct Shared {
   double *norm_b;        // [L]
   int32_t *status;       // [1] first device error
   uint8_t *orth_shifted; // [L] 1 = a Cholesky pass of this step needed the shift (third pass runs)
+  unsigned long long *gate_scratch;  // [2] the gate's running max of RMMC (ordered key), finished-block count
 };
 
 // A contraction C = op(A) op(B) for the CUDA-core path.

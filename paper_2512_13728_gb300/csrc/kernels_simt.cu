@@ -102,18 +102,31 @@ void launch_form_b(const Shared &sh, const int4 *tiles, int32_t ntiles, cudaStre
 // Algorithm 2: RMMC_l = | ||B|| - prev_l | / (prev_l + eps); prev_l = ||B||; global max over
 // layers; strict compare with tau (a non-finite RMMC counts as above every threshold); the
 // gate mode then decides which layers take the Dion branch.
-constexpr int kGateThreads = 1024;
 
 __device__ __forceinline__ bool above(double v, float tau) {
   return !isfinite(v) || v > (double)tau;
 }
 
-__global__ void __launch_bounds__(kGateThreads) gate_kernel(Shared sh, StepArgs a) {
-  __shared__ double wmax[kGateThreads / 32];
+// Monotone map of a non-negative double (or +inf) to an unsigned key, so that the maximum can
+// be taken with an integer atomic: for x >= 0 the IEEE bit pattern already orders correctly.
+__device__ __forceinline__ unsigned long long max_key(double x) {
+  return (unsigned long long)__double_as_longlong(x) | (1ull << 63);
+}
+__device__ __forceinline__ double from_max_key(unsigned long long k) {
+  return __longlong_as_double((long long)(k & ~(1ull << 63)));
+}
+
+// One warp per layer: ||B|| and ||M_{t-1}|| from the buffer pass's tile partials (fixed-order
+// fp64 sums), Algorithm 2's RMMC, prev_norm <- ||B||, the per-layer flag; the running maximum
+// of RMMC goes to an atomic max (order-independent, so deterministic).  The last block to
+// finish sets the global flag and the branch mask of every layer and resets the scratch.
+constexpr int kGateWarps = 8;
+__global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(Shared sh, StepArgs a) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int L = sh.num_layers;
-  double my_max = -INFINITY;
-  for (int l = warp; l < L; l += kGateThreads / 32) {
+  const int l = blockIdx.x * kGateWarps + warp;
+  __shared__ int last_s, gflag_s;
+  if (l < L) {
     const DevLayer &Ly = sh.layers[l];
     double sb = 0.0, sm = 0.0;
     for (int k = lane; k < Ly.bpart_cnt; k += 32) {  // fixed lane/slot assignment
@@ -135,34 +148,40 @@ __global__ void __launch_bounds__(kGateThreads) gate_kernel(Shared sh, StepArgs 
       a.flags[l] = above(rm, Ly.tau) ? 1 : 0;
       sh.norm_b[l] = nb;
       sh.norm_m_before[l] = sqrt(sm);
-      my_max = isfinite(rm) ? fmax(my_max, rm) : INFINITY;
+      atomicMax(&sh.gate_scratch[0], max_key(isfinite(rm) ? rm : INFINITY));
     }
   }
-  if (lane == 0) wmax[warp] = my_max;
-  __syncthreads();  // makes the per-layer global writes above visible to the whole block
-  __shared__ int gflag_s;
+  __syncthreads();
   if (threadIdx.x == 0) {
-    double g = -INFINITY;
-    for (int w = 0; w < kGateThreads / 32; ++w) g = fmax(g, wmax[w]);
-    const int gf = (L > 0 && above(g, a.tau_global)) ? 1 : 0;
-    a.gflag[0] = (uint8_t)gf;
-    gflag_s = gf;
+    __threadfence();  // this block's writes are visible before it is counted
+    last_s = atomicAdd(&sh.gate_scratch[1], 1ull) == (unsigned long long)(gridDim.x - 1);
   }
   __syncthreads();
-  for (int l = threadIdx.x; l < L; l += kGateThreads) {
+  if (!last_s) return;
+  if (threadIdx.x == 0) {
+    __threadfence();
+    const unsigned long long key = atomicAdd(&sh.gate_scratch[0], 0ull);
+    const int gf = (L > 0 && above(from_max_key(key), a.tau_global)) ? 1 : 0;
+    a.gflag[0] = (uint8_t)gf;
+    gflag_s = gf;
+    sh.gate_scratch[0] = 0ull;  // for the next step (kernel boundary orders it)
+    sh.gate_scratch[1] = 0ull;
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < L; i += kGateWarps * 32) {
     int act;
     switch (a.gate_mode) {
       case GATE_ALWAYS: act = 1; break;
       case GATE_GLOBAL: act = gflag_s; break;
-      case GATE_PER_LAYER: act = a.flags[l]; break;
+      case GATE_PER_LAYER: act = *reinterpret_cast<const volatile uint8_t *>(&a.flags[i]); break;  // other blocks'
       default: act = (a.step % a.period) == 0; break;
     }
-    sh.active[l] = (uint8_t)act;
+    sh.active[i] = (uint8_t)act;
   }
 }
 
 void launch_gate(const Shared &sh, const StepArgs &a, cudaStream_t s) {
-  gate_kernel<<<1, kGateThreads, 0, s>>>(sh, a);
+  gate_kernel<<<std::max(1, (sh.num_layers + kGateWarps - 1) / kGateWarps), kGateWarps * 32, 0, s>>>(sh, a);
 }
 
 // ==================================================================== grouped GEMM ===
@@ -798,10 +817,11 @@ void launch_local(const Shared &sh, const int4 *tiles, int32_t ntiles, float eta
 // ============================================================================ finalize ===
 // Equation 1: | ||M_t|| - ||M_{t-1}|| | / (||M_{t-1}|| + eps).  ||M_t|| comes from the update
 // kernel's partials on synchronized layers and equals ||B_t|| on local layers (M = B).
-__global__ void __launch_bounds__(kGateThreads) finalize_kernel(Shared sh, StepArgs a) {
+// One warp per layer: Equation 1 from the update's tile partials of ||M_t||^2.
+__global__ void __launch_bounds__(kGateWarps * 32) finalize_kernel(Shared sh, StepArgs a) {
   if (a.eq1 == nullptr) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int l = warp; l < sh.num_layers; l += kGateThreads / 32) {
+  for (int l = blockIdx.x * kGateWarps + warp; l < sh.num_layers; l += gridDim.x * kGateWarps) {
     const DevLayer &Ly = sh.layers[l];
     double nm;
     if (sh.active[l]) {
@@ -821,7 +841,8 @@ __global__ void __launch_bounds__(kGateThreads) finalize_kernel(Shared sh, StepA
 }
 
 void launch_finalize(const Shared &sh, const StepArgs &a, cudaStream_t s) {
-  if (a.eq1 != nullptr) finalize_kernel<<<1, kGateThreads, 0, s>>>(sh, a);
+  if (a.eq1 != nullptr)
+    finalize_kernel<<<std::max(1, (sh.num_layers + kGateWarps - 1) / kGateWarps), kGateWarps * 32, 0, s>>>(sh, a);
 }
 
 }  // namespace cd

@@ -357,11 +357,7 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
     for (int64_t nb = 0; nb < (ly.n + 127) / 128; ++nb) lo.rtiles.push_back(make_int4(l, (int)nb, 0, 0));
   }
   // per-tile cost ~ K-loop length (+ a constant for the epilogue), LPT over the SMs
-  auto sched = [&](const std::vector<int4> &tl, auto costf) {
-    std::vector<double> c(tl.size());
-    for (size_t i = 0; i < tl.size(); ++i) c[i] = costf(tl[i]);
-    return lpt(tl, c, std::max(num_sms, 1));
-  };
+
   // update: row-tile pairs (one per cluster of two CTAs); w = ||M_t|| slot of the pair's first tile
   std::vector<int4> upairs;
   for (size_t i = 0; i < lo.utiles.size(); ++i) {
