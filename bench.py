@@ -241,11 +241,21 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
+    # the gradients go up on several side streams (one copy engine each), joined before the step
+    up = [torch.cuda.Stream(dev) for _ in range(4)]
     f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     f0.record(stream)
     for _ in range(e_steps):
-        for g, hg in zip(G, host_G):
-            g.copy_(hg, non_blocking=True)
+        start = torch.cuda.Event()
+        start.record(stream)
+        for i, (g, hg) in enumerate(zip(G, host_G)):
+            us = up[i % len(up)]
+            if i < len(up):
+                us.wait_event(start)  # after the previous step's kernels have read G
+            with torch.cuda.stream(us):
+                g.copy_(hg, non_blocking=True)
+        for us in up:
+            stream.wait_stream(us)
         one_step()
         host_out[: 8 * w.num_layers].copy_(plan.rmmc[: w.num_layers].view(torch.uint8), non_blocking=True)
         host_out[8 * w.num_layers: 9 * w.num_layers].copy_(plan.flags[: w.num_layers], non_blocking=True)
