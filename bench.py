@@ -67,9 +67,12 @@ def kernel_work(name: str, w, prec: str):
     nr = sum(n * r for (m, n), r in zip(w.shapes, ranks))
     mr = sum(m * r for (m, n), r in zip(w.shapes, ranks))
     bh = 2 if prec == "bf16" else 0  # the bf16 copy of B the tensor-core contractions read
+    # tensor-core mode with bf16 G: the buffer pass leaves M_{t-1} in place and the update
+    # forms B = M + G itself (it reads G, the buffer pass does not write M)
+    deferred = prec == "bf16" and w.g_dtype == "bf16"
     table = {
         # CUDA-core path
-        "form_b": ("hbm", mn * (4 + gsz + 4 + bh), "B"),
+        "form_b": ("hbm", mn * (4 + gsz + (0 if deferred else 4) + bh), "B"),
         "gemm_bq": ("alu", 2 * mnr, "flop"),
         "gemm_gram": ("alu", 2 * mr2, "flop"),
         "chol_inv": ("alu", 2 * r3 / 3, "flop"),
@@ -81,7 +84,7 @@ def kernel_work(name: str, w, prec: str):
         # tensor-core path
         "tc_bq": ("hbm", mn * 2 + nr * 2 + mr * 8, "B"),  # Bh, bf16 Q; P and P^T fp32
         "tc_btp": ("hbm", mn * 2 + mr * 2 + nr * 6, "B"),  # Bh, bf16 P; R fp32 and bf16
-        "tc_update": ("hbm", mn * 16, "B"),
+        "tc_update": ("hbm", mn * (16 + (gsz if deferred else 0)), "B"),
         "tc_gram": ("tensor", 2 * mr2, "flop"),
         "tc_trsm": ("tensor", 2 * mr2, "flop"),
     }
@@ -92,7 +95,12 @@ def step_bytes(w, prec):
     """Bytes one synchronized step moves by design (the planned passes), and the compulsory floor."""
     gsz = 2 if w.g_dtype == "bf16" else 4
     mn = sum(m * n for m, n in w.shapes)
-    planned = mn * ((4 + gsz + 4) + 4 + 4 + 16) if prec == "fp32" else mn * ((4 + gsz + 4 + 2) + 2 + 2 + 16)
+    if prec == "fp32":
+        planned = mn * ((4 + gsz + 4) + 4 + 4 + 16)
+    elif w.g_dtype == "bf16":  # buffer pass 8, two Bh reads 2 + 2, update 18
+        planned = mn * ((4 + gsz + 2) + 2 + 2 + (16 + gsz))
+    else:
+        planned = mn * ((4 + gsz + 4 + 2) + 2 + 2 + 16)
     compulsory = mn * (4 + gsz + 4 + 4 + 4)  # read M, G, X; write M, X
     return planned, compulsory
 

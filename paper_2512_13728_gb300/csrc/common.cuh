@@ -31,7 +31,7 @@ struct DevLayer {
   int64_t m, n, r;
   float *X;
   int64_t ldx;
-  float *M;  // holds B = M + G between the buffer kernel and the update kernel
+  float *M;  // holds B = M + G between the buffer kernel and the update kernel (unless b_deferred)
   int64_t ldm;
   float *Q;
   int64_t ldq;
@@ -57,7 +57,10 @@ struct DevLayer {
   int64_t ldmt;
   double *colsq;         // [row tiles of R][ldp]: per-tile column sums of squares of R
   float *colinv;         // [ldp]: 1 / (||R[:, j]|| + eps_col)
-  int32_t rtile_cnt, pad1;
+  int32_t rtile_cnt;
+  // 1: the buffer pass leaves M_{t-1} in place (it writes only the norms and the bf16 copy of B),
+  // and the update or the local branch forms B = M + G itself (tensor-core mode, bf16 G)
+  int32_t b_deferred;
   int32_t bpart_off, bpart_cnt;  // slots of the ||B||^2 / ||M_{t-1}||^2 partials
   int32_t upart_off, upart_cnt;  // slots of the ||M_t||^2 partials
 };

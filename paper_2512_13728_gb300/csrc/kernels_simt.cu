@@ -54,7 +54,7 @@ __device__ void form_b_tile(const DevLayer &L, int64_t row0, int64_t nrows, floa
       m.x += g[0]; m.y += g[1]; m.z += g[2]; m.w += g[3];
       sb[0] = fmaf(m.x, m.x, sb[0]); sb[1] = fmaf(m.y, m.y, sb[1]);
       sb[2] = fmaf(m.z, m.z, sb[2]); sb[3] = fmaf(m.w, m.w, sb[3]);
-      *reinterpret_cast<float4 *>(Mrow + 4 * c4) = m;
+      if (!HAS_BH || !L.b_deferred) *reinterpret_cast<float4 *>(Mrow + 4 * c4) = m;
       if (HAS_BH) {  // bf16 copy of B (operand of the tensor-core contractions)
         const __nv_bfloat162 h01 = __floats2bfloat162_rn(m.x, m.y), h23 = __floats2bfloat162_rn(m.z, m.w);
         uint2 hv;
@@ -68,7 +68,7 @@ __device__ void form_b_tile(const DevLayer &L, int64_t row0, int64_t nrows, floa
       const float b = mo + load_g1<GT>(L.G, goff + c);
       sm[0] = fmaf(mo, mo, sm[0]);
       sb[0] = fmaf(b, b, sb[0]);
-      Mrow[c] = b;
+      if (!HAS_BH || !L.b_deferred) Mrow[c] = b;
       if (HAS_BH) L.Bh[i * L.ldbh + c] = __float2bfloat16_rn(b);
     }
   }
@@ -781,13 +781,15 @@ void launch_update(const Shared &sh, const int4 *tiles, int32_t ntiles, float mu
 }
 
 // ======================================================================== local branch ===
-// Algorithm 2's else-branch: M = B is already in place; X = X - eta_local G.
+// Algorithm 2's else-branch: X = X - eta_local G, and M = B = M + G (already in place unless
+// the layer defers B to the update).
 template <int GT>
 __device__ void local_tile(const DevLayer &L, int64_t row0, int64_t nrows, float eta_local) {
   const int64_t n = L.n, n4 = n >> 2;
+  const bool form_m = L.b_deferred != 0;
   for (int64_t rr = 0; rr < nrows; ++rr) {
     const int64_t i = row0 + rr;
-    float *Xrow = L.X + i * L.ldx;
+    float *Xrow = L.X + i * L.ldx, *Mrow = L.M + i * L.ldm;
     const int64_t goff = i * L.ldg;
     for (int64_t c4 = threadIdx.x; c4 < n4; c4 += kRowThreads) {
       float4 x = *reinterpret_cast<float4 *>(Xrow + 4 * c4);
@@ -796,9 +798,17 @@ __device__ void local_tile(const DevLayer &L, int64_t row0, int64_t nrows, float
       x.x = fmaf(-eta_local, g[0], x.x); x.y = fmaf(-eta_local, g[1], x.y);
       x.z = fmaf(-eta_local, g[2], x.z); x.w = fmaf(-eta_local, g[3], x.w);
       *reinterpret_cast<float4 *>(Xrow + 4 * c4) = x;
+      if (form_m) {
+        float4 m = *reinterpret_cast<float4 *>(Mrow + 4 * c4);
+        m.x += g[0]; m.y += g[1]; m.z += g[2]; m.w += g[3];
+        *reinterpret_cast<float4 *>(Mrow + 4 * c4) = m;
+      }
     }
-    for (int64_t c = 4 * n4 + threadIdx.x; c < n; c += kRowThreads)
-      Xrow[c] = fmaf(-eta_local, load_g1<GT>(L.G, goff + c), Xrow[c]);
+    for (int64_t c = 4 * n4 + threadIdx.x; c < n; c += kRowThreads) {
+      const float g = load_g1<GT>(L.G, goff + c);
+      Xrow[c] = fmaf(-eta_local, g, Xrow[c]);
+      if (form_m) Mrow[c] += g;
+    }
   }
 }
 

@@ -35,8 +35,10 @@ constexpr int U_STAGES = 3;
 constexpr uint32_t U_OPB = 128u * 64u * 2u;           // 128 x 64 bf16 operand box
 constexpr uint32_t U_STAGE = 3u * U_OPB;              // P, R, Q_t
 constexpr uint32_t U_EBOX = 128u * 16u * 4u;          // one 128 x 16 fp32 box (64-byte swizzle)
-constexpr uint32_t U_EBUF2 = 2u * U_EBOX;             // B and X of one 16-column sub-chunk
-constexpr int U_EBUF = 5;                             // sub-chunk buffers of the epilogue
+constexpr uint32_t U_GBOX = 128u * 16u * 2u;          // one 128 x 16 bf16 box of G (32-byte swizzle)
+constexpr uint32_t U_EBUF2 = 2u * U_EBOX + U_GBOX;     // M, X and G of one 16-column sub-chunk (20 KB)
+constexpr int U_EBUF = 4;                             // sub-chunk buffers of the epilogue
+static_assert(U_EBUF2 % 1024u == 0, "every box of a sub-chunk buffer stays 1024-byte aligned");
 constexpr uint32_t U_SMEM = 1024u + U_STAGES * U_STAGE + U_EBUF * U_EBUF2 + 256u;
 constexpr int U_THREADS = 192;
 constexpr uint32_t U_IDESC = idesc_bf16(128, 128, false, false);
@@ -179,9 +181,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
         if (issued >= U_EBUF) bulk_wait_read<1>();
         uint8_t *bs = epi + eb * U_EBUF2;
         const int r0 = (2 * t.y + (int)rank) * 128, x0 = t.z * 128 + lj * 16;
-        mbar_expect_tx(&epi_full[eb], U_EBUF2);
+        const bool defer = sh.layers[t.x].b_deferred != 0;  // B = M + G is formed here
+        mbar_expect_tx(&epi_full[eb], 2u * U_EBOX + (defer ? U_GBOX : 0u));
         tma_load_2d(bs, &mp->Mf16, &epi_full[eb], x0, r0);
         tma_load_2d(bs + U_EBOX, &mp->Xf16, &epi_full[eb], x0, r0);
+        if (defer) tma_load_2d(bs + 2 * U_EBOX, &mp->Gh16, &epi_full[eb], x0, r0);
         ++issued;
         if (++lj == subs_of(t)) {
           lj = 0;
@@ -202,6 +206,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
       const int mb = 2 * t.y + (int)rank, r0 = mb * 128, c0 = t.z * 128;
       const int ntc = (int)((L.n + 127) / 128);
       const int ns = subs_of(t);
+      const bool defer = L.b_deferred != 0;
       const uint32_t b = tcount & 1u, aph = (tcount >> 1) & 1u;
       if (!named_and(1, 128, ab.wait(&acc_full[b], aph, sh.status))) break;
       tc_fence_after();
@@ -227,6 +232,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
             const int cc = h * 16 + q * 4;
             float4 bv = *reinterpret_cast<float4 *>(bs + o);
             float4 xv = *reinterpret_cast<float4 *>(bs + U_EBOX + o);
+            if (defer) {  // B = M_{t-1} + G, the same fp32 additions as the buffer pass
+              const uint2 gv = *reinterpret_cast<const uint2 *>(bs + 2 * U_EBOX + sw32_offset(row, (uint32_t)q >> 1) +
+                                                                (q & 1) * 8);
+              bv.x += __uint_as_float(gv.x << 16);
+              bv.y += __uint_as_float(gv.x & 0xffff0000u);
+              bv.z += __uint_as_float(gv.y << 16);
+              bv.w += __uint_as_float(gv.y & 0xffff0000u);
+            }
             bv.x = fmaf(-dec, __uint_as_float(u1[cc + 0]), bv.x);
             bv.y = fmaf(-dec, __uint_as_float(u1[cc + 1]), bv.y);
             bv.z = fmaf(-dec, __uint_as_float(u1[cc + 2]), bv.z);
@@ -410,6 +423,7 @@ void bind(const TcLayout &lo, char *base, DevLayer *dl, int32_t L, TcPlan *tp) {
     dl[l].colsq = reinterpret_cast<double *>(base + lo.o_colsq[l]);
     dl[l].colinv = reinterpret_cast<float *>(base + lo.o_colinv[l]);
     dl[l].rtile_cnt = (int32_t)((dl[l].n + 127) / 128);
+    dl[l].b_deferred = (dl[l].g_dtype == DT_BF16) ? 1 : 0;  // the update forms B = M + G itself
     dl[l].upart_off = -1;
   }
   int32_t cur = -1;
@@ -463,6 +477,7 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
                     encode_f32_2d(&m.Xf, d.X, d.n, d.m, (uint64_t)d.ldx * 4, 32, 128) &&
                     encode_f32_2d(&m.Mf16, d.M, d.n, d.m, (uint64_t)d.ldm * 4, 16, 128) &&
                     encode_f32_2d(&m.Xf16, d.X, d.n, d.m, (uint64_t)d.ldx * 4, 16, 128) &&
+                    (d.g_dtype != DT_BF16 || encode_bf16_2d(&m.Gh16, d.G, d.n, d.m, (uint64_t)d.ldg * 2, 16, 128)) &&
                     encode_bf16_2d(&m.Qn_mn, d.Qn_hi, d.r, d.n, p16, 64, 64) &&
                     encode_bf16_2d(&m.P_mn, d.P_hi, d.r, d.m, p16, 64, 64) &&
                     encode_bf16_2d(&m.Bh_mn, d.Bh, d.n, d.m, (uint64_t)d.ldbh * 2, 64, 64) &&

@@ -20,6 +20,7 @@ struct LayerMaps {
   CUtensorMap Mf;     // m x n fp32 (caller M): box {32, 128}  update: B in / M_t out
   CUtensorMap Xf;     // m x n fp32 (caller X): box {32, 128}  update: X in / out
   CUtensorMap Mf16, Xf16;  // m x n fp32: box {16, 128}, 64-byte swizzle (update epilogue)
+  CUtensorMap Gh16;        // m x n bf16 G: box {16, 128}, 32-byte swizzle (update epilogue)
   CUtensorMap Qn_mn;  // n x r bf16:  box {64, 64}   B Q: MN-major B operand (K = n)
   CUtensorMap P_mn;   // m x r bf16:  box {64, 64}   B^T P: MN-major B operand (K = m)
   CUtensorMap Bh_mn;  // m x n bf16:  box {64, 64}   B^T P: MN-major A operand (K = m)

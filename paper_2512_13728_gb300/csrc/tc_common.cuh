@@ -307,6 +307,11 @@ __device__ __forceinline__ bool named_and(uint32_t id, uint32_t count, bool v) {
 __device__ __forceinline__ uint32_t sw128_f32(uint32_t row, uint32_t chunk) {
   return row * 128u + ((chunk ^ (row & 7u)) << 4);
 }
+// Byte offset of 16-byte chunk `chunk` (0..1) of row `row` in a 32-byte-swizzled box of
+// 32-byte rows (16 bf16): the chunk index is XORed with bit 2 of the row.
+__device__ __forceinline__ uint32_t sw32_offset(uint32_t row, uint32_t chunk) {
+  return row * 32u + ((chunk ^ ((row >> 2) & 1u)) << 4);
+}
 // Byte offset of 16-byte chunk `chunk` (0..3) of row `row` in a 64-byte-swizzled box of
 // 64-byte rows (16 fp32): the chunk index is XORed with bits 1..2 of the row.
 __device__ __forceinline__ uint32_t sw64_f32(uint32_t row, uint32_t chunk) {

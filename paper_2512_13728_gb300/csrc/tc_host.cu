@@ -29,15 +29,19 @@ EncodeTiledFn encoder() {
 bool encode_bf16_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
                     uint32_t box_inner, uint32_t box_outer) {
   EncodeTiledFn fn = encoder();
-  if (!fn || (reinterpret_cast<uintptr_t>(base) & 15u) || (pitch_bytes & 15u) || box_inner * 2 > 128 ||
-      box_outer > 256 || box_inner == 0 || box_outer == 0)
+  if (!fn || (reinterpret_cast<uintptr_t>(base) & 15u) || (pitch_bytes & 15u) ||
+      (box_inner * 2 != 128 && box_inner * 2 != 64 && box_inner * 2 != 32) || box_outer > 256 || box_outer == 0)
     return false;
   cuuint64_t dims[2] = {inner, outer};
   cuuint64_t strides[1] = {pitch_bytes};
   cuuint32_t box[2] = {box_inner, box_outer};
   cuuint32_t estr[2] = {1, 1};
+  // the swizzle spans the box's row (128, 64 or 32 bytes)
+  const CUtensorMapSwizzle sw = box_inner * 2 == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+                                : box_inner * 2 == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                      : CU_TENSOR_MAP_SWIZZLE_32B;
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
