@@ -83,6 +83,8 @@ def kernel_work(name: str, w, prec: str):
         "local": ("hbm", 0, "B"),
         # tensor-core path
         "tc_bq": ("hbm", mn * 2 + nr * 2 + mr * 8, "B"),  # Bh, bf16 Q; P and P^T fp32
+        # buffer pass fused into B Q (bf16 G): read M, G; write Bh, P and P^T fp32
+        "tc_form_bq": ("hbm", mn * (4 + gsz + 2) + mr * 8, "B"),
         "tc_btp": ("hbm", mn * 2 + mr * 2 + nr * 6, "B"),  # Bh, bf16 P; R fp32 and bf16
         "tc_update": ("hbm", mn * (16 + (gsz if deferred else 0)), "B"),
         "tc_gram": ("tensor", 2 * mr2, "flop"),
@@ -97,8 +99,8 @@ def step_bytes(w, prec):
     mn = sum(m * n for m, n in w.shapes)
     if prec == "fp32":
         planned = mn * ((4 + gsz + 4) + 4 + 4 + 16)
-    elif w.g_dtype == "bf16":  # buffer pass 8, two Bh reads 2 + 2, update 18
-        planned = mn * ((4 + gsz + 2) + 2 + 2 + (16 + gsz))
+    elif w.g_dtype == "bf16":  # buffer pass fused with B Q 8, the Bh read of B^T P 2, update 18
+        planned = mn * ((4 + gsz + 2) + 2 + (16 + gsz))
     else:
         planned = mn * ((4 + gsz + 4 + 2) + 2 + 2 + 16)
     compulsory = mn * (4 + gsz + 4 + 4 + 4)  # read M, G, X; write M, X

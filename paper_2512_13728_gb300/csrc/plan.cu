@@ -195,7 +195,11 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
   std::vector<int4> gt[kSets];
   const size_t o_layers = cv.take<DevLayer>(std::max(num_layers, 1));
   const size_t o_active = cv.take<uint8_t>(std::max(num_layers, 1));
-  const size_t o_bpart = cv.take<double>(2 * std::max<size_t>(bt.size(), 1));
+  // norm-partial slots: one per buffer row tile, or one per 128-row tile when the tensor-core
+  // path fuses the buffer pass into B Q
+  size_t tile128 = 0;
+  for (int32_t l = 0; l < num_layers; ++l) tile128 += (size_t)((layers[l].m + 127) / 128);
+  const size_t o_bpart = cv.take<double>(2 * std::max<size_t>(std::max(bt.size(), tile128), 1));
   const size_t o_upart = cv.take<double>(std::max<size_t>(ut.size(), 1));
   const size_t o_nmb = cv.take<double>(std::max(num_layers, 1));
   const size_t o_nb = cv.take<double>(std::max(num_layers, 1));

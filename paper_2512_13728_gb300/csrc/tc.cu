@@ -405,6 +405,8 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
   lo.o_qtiles = take(sizeof(int4) * std::max<size_t>(lo.qtiles.size(), 1));
   lo.o_gtiles = take(sizeof(int4) * std::max<size_t>(lo.gram_tiles.size(), 1));
   lo.o_ttiles = take(sizeof(int4) * std::max<size_t>(lo.trsm_tiles.size(), 1));
+  lo.fuse_buffer = L > 0;
+  for (int32_t l = 0; l < L; ++l) lo.fuse_buffer = lo.fuse_buffer && layers[l].g_dtype == DION_DTYPE_BF16;
   lo.end = off;
   (void)num_sms;
   return DION_OK;
@@ -426,6 +428,15 @@ void bind(const TcLayout &lo, char *base, DevLayer *dl, int32_t L, TcPlan *tp) {
     dl[l].b_deferred = (dl[l].g_dtype == DT_BF16) ? 1 : 0;  // the update forms B = M + G itself
     dl[l].upart_off = -1;
   }
+  if (lo.fuse_buffer) {  // the fused kernel writes one ||B||^2 / ||M_{t-1}||^2 slot per 128-row tile
+    int32_t slot = 0;
+    for (int32_t l = 0; l < L; ++l) {
+      dl[l].bpart_off = slot;
+      dl[l].bpart_cnt = (int32_t)((dl[l].m + 127) / 128);
+      slot += dl[l].bpart_cnt;
+    }
+  }
+  tp->fuse_buffer = lo.fuse_buffer;
   int32_t cur = -1;
   for (size_t i = 0; i < lo.utiles.size(); ++i) {
     const int l = lo.utiles[i].x;
@@ -478,6 +489,7 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
                     encode_f32_2d(&m.Mf16, d.M, d.n, d.m, (uint64_t)d.ldm * 4, 16, 128) &&
                     encode_f32_2d(&m.Xf16, d.X, d.n, d.m, (uint64_t)d.ldx * 4, 16, 128) &&
                     (d.g_dtype != DT_BF16 || encode_bf16_2d(&m.Gh16, d.G, d.n, d.m, (uint64_t)d.ldg * 2, 16, 128)) &&
+                    (d.g_dtype != DT_BF16 || encode_bf16_2d(&m.Gh64, d.G, d.n, d.m, (uint64_t)d.ldg * 2, 64, 128)) &&
                     encode_bf16_2d(&m.Qn_mn, d.Qn_hi, d.r, d.n, p16, 64, 64) &&
                     encode_bf16_2d(&m.P_mn, d.P_hi, d.r, d.m, p16, 64, 64) &&
                     encode_bf16_2d(&m.Bh_mn, d.Bh, d.n, d.m, (uint64_t)d.ldbh * 2, 64, 64) &&
@@ -537,12 +549,15 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(tc_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)U_SMEM);
   if (e == cudaSuccess) e = setup_bq_kernels(tp->f_smem, tp->r_smem);
+  tp->fb_smem = fused_bq_smem(bq_boxes);
+  if (tp->fuse_buffer && tp->fb_smem > 227u * 1024u) return cudaErrorInvalidValue;
+  if (e == cudaSuccess && tp->fuse_buffer) e = setup_fused_bq_kernel(tp->fb_smem);
   if (e == cudaSuccess) e = setup_orth_kernels(tp->o_smem);
   int dev = 0, sms = 0;
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   tp->num_sms = sms;
-  tp->launches = 18;
+  tp->launches = tp->fuse_buffer ? 17 : 18;
   return e;
 }
 
@@ -552,12 +567,19 @@ void refresh(const TcPlan &tp, const Shared &sh, cudaStream_t s) { launch_qn_ref
 
 void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, const int4 *btiles,
           int32_t n_btiles, const int4 *ctiles, int32_t n_ctiles, size_t chol_smem, cudaStream_t s) {
-  launch_form_b(sh, btiles, n_btiles, s);  // B = M + G (and its bf16 copy), ||B||, ||M_{t-1}||
-  tick(p, s, "form_b");
-  launch_gate(sh, a, s);
-  tick(p, s, "gate");
-  launch_form_bq(sh, tp, s);  // P = B Q_{t-1} on the layers that take the Dion branch
-  tick(p, s, "tc_bq");
+  if (tp.fuse_buffer) {
+    launch_fused_bq(sh, tp, s);  // B = M + G, Bh, ||B||, ||M_{t-1}||, P = B Q_{t-1} (every layer)
+    tick(p, s, "tc_form_bq");
+    launch_gate(sh, a, s);
+    tick(p, s, "gate");
+  } else {
+    launch_form_b(sh, btiles, n_btiles, s);  // B = M + G (and its bf16 copy), ||B||, ||M_{t-1}||
+    tick(p, s, "form_b");
+    launch_gate(sh, a, s);
+    tick(p, s, "gate");
+    launch_form_bq(sh, tp, s);  // P = B Q_{t-1} on the layers that take the Dion branch
+    tick(p, s, "tc_bq");
+  }
   static const char *kGram[3] = {"tc_gram0", "tc_gram1", "tc_gram2"};
   static const char *kChol[3] = {"chol_inv0", "chol_inv1", "chol_inv2"};
   static const char *kTrsm[3] = {"tc_trsm0", "tc_trsm1", "tc_trsm2"};

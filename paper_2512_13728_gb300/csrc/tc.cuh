@@ -21,6 +21,7 @@ struct LayerMaps {
   CUtensorMap Xf;     // m x n fp32 (caller X): box {32, 128}  update: X in / out
   CUtensorMap Mf16, Xf16;  // m x n fp32: box {16, 128}, 64-byte swizzle (update epilogue)
   CUtensorMap Gh16;        // m x n bf16 G: box {16, 128}, 32-byte swizzle (update epilogue)
+  CUtensorMap Gh64;        // m x n bf16 G: box {64, 128}  fused buffer pass + B Q
   CUtensorMap Qn_mn;  // n x r bf16:  box {64, 64}   B Q: MN-major B operand (K = n)
   CUtensorMap P_mn;   // m x r bf16:  box {64, 64}   B^T P: MN-major B operand (K = m)
   CUtensorMap Bh_mn;  // m x n bf16:  box {64, 64}   B^T P: MN-major A operand (K = m)
@@ -56,6 +57,8 @@ struct TcLayout {
   std::vector<int4> utiles, ftiles, rtiles, qtiles;
   int32_t precision = 0;
   int32_t max_r = 0;
+  // every layer has bf16 G: the buffer pass is fused into B Q (norm slots = 128-row tiles)
+  bool fuse_buffer = false;
 };
 
 struct DevSchedule {
@@ -85,6 +88,8 @@ struct TcPlan {
   int32_t num_sms = 0;
   int32_t precision = 0;
   int32_t launches = 0;
+  bool fuse_buffer = false;
+  uint32_t fb_smem = 0;
   // CUDA-core pieces reused by this path (set by the plan)
   const GemmProblem *const *probs = nullptr;
   const int4 *const *gtiles = nullptr;

@@ -14,6 +14,7 @@
 #include "tc_common.cuh"
 #include "tc_kernels.cuh"
 
+#include <algorithm>
 #include <type_traits>
 
 namespace cd {
@@ -313,6 +314,314 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(R_THREADS, 1)
   if (warp == 1) tmem_dealloc_pair(tmem, tmem_cols);
 }
 
+// ============================================== buffer pass fused with P = B Q_{t-1} ===
+// Algorithm 1/2 with bf16 gradients: B = M_{t-1} + G is formed on the fly from TMA tiles of M
+// (fp32) and G (bf16) and fed to the pair MMA of P = B Q_{t-1}, so B is read from HBM once.
+// Per {layer, pair p} (CTA c owns 128-row tile 2 p + c) and 64-column k-chunk:
+//   warp 0      TMA: M as two 128 x 32 fp32 SW128 boxes into the M ring, G as one 128 x 64 bf16
+//               SW128 box into the A ring;
+//   warps 6..9  B = M + G in fp32, rounded to bf16 and written in place over the G box, which
+//               has the layout of the K-major A operand; the per-tile sums of B^2 and M_{t-1}^2
+//               (Algorithm 2's ||B|| and Equation 1's ||M_{t-1}||).  The M stage is free again
+//               as soon as it is converted;
+//   warp 11     TMA store of each converted box to Bh (the operand of B^T P); the A slot is
+//               refilled once that store has read it and the chunk's MMAs have completed;
+//   warp 10     TMA: this CTA's half of the Q_{t-1} chunk (MN-major boxes, bytes counted on
+//               CTA 0's barrier) into the Q ring;
+//   warp 1      (CTA 0) the pair MMAs of the chunk once both CTAs' A boxes and Q halves are in;
+//   warps 2..5  drain the 128 x r accumulator into P_raw and its transpose (as in B Q), staged
+//               through the Q ring: the next tile's MMAs wait for TMEM anyway, so its Q loads
+//               wait until the staged stores have been read.
+// Separate rings keep each slot's turnaround short: an M slot waits for one load and one
+// conversion, an A slot for the load, conversion, MMA and store.
+constexpr int FB_MSTAGES = 3;  // M ring (2 x 16 KB per slot)
+constexpr int FB_ASTAGES = 4;  // G / A ring (16 KB per slot)
+constexpr int FB_QSTAGES = 2;  // Q ring (also the epilogue's staging)
+constexpr int FB_THREADS = 12 * 32;
+constexpr uint32_t FB_MBOX = 128u * 32u * 4u;  // 128 x 32 fp32 box of M (16 KB)
+constexpr uint32_t FB_GBOX = 128u * 64u * 2u;  // 128 x 64 bf16 box of G, then of B (16 KB)
+constexpr uint32_t FB_MSLOT = 2u * FB_MBOX;
+constexpr uint32_t FB_A_OFF = FB_MSTAGES * FB_MSLOT;
+constexpr uint32_t FB_Q_OFF = FB_A_OFF + FB_ASTAGES * FB_GBOX;
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
+    tc_form_bq_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off,
+                      const LayerMaps *__restrict__ maps, uint32_t qstage_bytes, uint32_t qring_bytes,
+                      uint32_t tmem_cols) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = align1024(smem_raw);
+  uint8_t *aring = smem + FB_A_OFF;
+  uint8_t *qring = smem + FB_Q_OFF;  // Q stages; the epilogue's staging between tiles
+  uint64_t *bars = reinterpret_cast<uint64_t *>(qring + qring_bytes);
+  uint64_t *mfull = bars, *mempty = mfull + FB_MSTAGES;
+  uint64_t *gfull = mempty + FB_MSTAGES, *gempty = gfull + FB_ASTAGES, *afull = gempty + FB_ASTAGES,
+           *cvt = afull + FB_ASTAGES;
+  uint64_t *qfull = cvt + FB_ASTAGES, *qempty = qfull + FB_QSTAGES;
+  uint64_t *acc_full = qempty + FB_QSTAGES, *acc_empty = acc_full + 1, *epi_free = acc_full + 2,
+           *drain = acc_full + 3;
+  __shared__ uint32_t tmem_base_s;
+  __shared__ int abort_s;
+  __shared__ double red_s[2][4];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const Abort ab{&abort_s};
+  const uint32_t rank = cluster_ctarank();
+  const int seg = blockIdx.x >> 1;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < FB_MSTAGES; ++i) {
+      mbar_init(&mfull[i], 1);   // this CTA's M boxes
+      mbar_init(&mempty[i], 1);  // converted
+    }
+    for (int i = 0; i < FB_ASTAGES; ++i) {
+      mbar_init(&gfull[i], 1);   // this CTA's G box
+      mbar_init(&gempty[i], 2);  // pair commit after the chunk's MMAs + this CTA's Bh store read
+      mbar_init(&afull[i], 2);   // used in CTA 0: one arrival per CTA's converted A box
+      mbar_init(&cvt[i], 1);     // this CTA's box is converted (for the Bh store)
+    }
+    for (int i = 0; i < FB_QSTAGES; ++i) {
+      mbar_init(&qfull[i], 1);   // used in CTA 0: its arm, both CTAs' Q bytes
+      mbar_init(&qempty[i], 1);  // pair commit after the chunk's MMAs
+    }
+    mbar_init(acc_full, 1);
+    mbar_init(acc_empty, 2);  // used in CTA 0: one arrival per CTA's epilogue
+    mbar_init(epi_free, 1);   // this CTA's staged epilogue stores have been read
+    mbar_init(drain, 1);
+    abort_s = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(&tmem_base_s, tmem_cols);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  cluster_sync();
+  const uint32_t tmem = tmem_base_s;
+  auto half_cols = [](uint32_t np, uint32_t part) { return min(256u, np - part * 256u) / 2u; };
+
+  if (warp == 0) {  // M and G loads
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
+        const int4 t = tiles[ti];
+        const DevLayer &L = sh.layers[t.x];
+        const LayerMaps *mp = maps + t.x;
+        const int kch = (int)((L.n + 63) / 64);
+        const int tr = 2 * t.y + (int)rank;  // past the last tile: zero-filled, not stored
+        for (int kc = 0; kc < kch; ++kc, ++it) {
+          const uint32_t sm = it % FB_MSTAGES, pm = (it / FB_MSTAGES) & 1u;
+          const uint32_t sg = it % FB_ASTAGES, pg = (it / FB_ASTAGES) & 1u;
+          if (!ab.wait(&mempty[sm], pm ^ 1u, sh.status)) { ok = false; break; }
+          uint8_t *sM = smem + sm * FB_MSLOT;
+          mbar_expect_tx(&mfull[sm], FB_MSLOT);
+          tma_load_2d(sM, &mp->Mf, &mfull[sm], kc * 64, tr * 128);
+          tma_load_2d(sM + FB_MBOX, &mp->Mf, &mfull[sm], kc * 64 + 32, tr * 128);
+          if (!ab.wait(&gempty[sg], pg ^ 1u, sh.status)) { ok = false; break; }
+          mbar_expect_tx(&gfull[sg], FB_GBOX);
+          tma_load_2d(aring + sg * FB_GBOX, &mp->Gh64, &gfull[sg], kc * 64, tr * 128);
+        }
+      }
+      for (uint32_t k = (it > (uint32_t)FB_MSTAGES ? it - FB_MSTAGES : 0); k < it; ++k)
+        mbar_wait(&mempty[k % FB_MSTAGES], (k / FB_MSTAGES) & 1u, sh.status);
+      for (uint32_t k = (it > (uint32_t)FB_ASTAGES ? it - FB_ASTAGES : 0); k < it; ++k)
+        mbar_wait(&gempty[k % FB_ASTAGES], (k / FB_ASTAGES) & 1u, sh.status);
+    }
+  } else if (warp == 10) {  // Q loads
+    if (lane == 0) {
+      uint32_t it = 0, tcount = 0;
+      bool ok = true;
+      for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti, ++tcount) {
+        const int4 t = tiles[ti];
+        const DevLayer &L = sh.layers[t.x];
+        const LayerMaps *mp = maps + t.x;
+        const int kch = (int)((L.n + 63) / 64);
+        const uint32_t np = rpad16(L.r), nparts = (np + 255) / 256;
+        uint32_t nbox = 0;
+        for (uint32_t part = 0; part < nparts; ++part) nbox += (half_cols(np, part) + 63) / 64;
+        // the ring holds the previous tile's staged accumulator until its stores have read it
+        if (tcount > 0 && !ab.wait(epi_free, (tcount - 1) & 1u, sh.status)) break;
+        for (int kc = 0; kc < kch; ++kc, ++it) {
+          const uint32_t s = it % FB_QSTAGES, ph = (it / FB_QSTAGES) & 1u;
+          if (!ab.wait(&qempty[s], ph ^ 1u, sh.status)) { ok = false; break; }
+          uint8_t *sQ = qring + s * qstage_bytes;
+          const uint32_t qb = cluster_addr(&qfull[s], 0);
+          if (rank == 0) mbar_expect_tx(&qfull[s], 2u * nbox * BOX64);
+          for (uint32_t part = 0; part < nparts; ++part) {
+            const uint32_t hc = half_cols(np, part);
+            const int x0 = (int)(part * 256u + rank * hc);
+            for (uint32_t j = 0; j < (hc + 63) / 64; ++j)
+              tma_load_2d_pair(sQ + (part * 2u + j) * BOX64, &mp->Qn_mn, qb, x0 + (int)j * 64, kc * 64);
+          }
+        }
+      }
+      for (uint32_t k = (it > (uint32_t)FB_QSTAGES ? it - FB_QSTAGES : 0); k < it; ++k)
+        mbar_wait(&qempty[k % FB_QSTAGES], (k / FB_QSTAGES) & 1u, sh.status);
+    }
+  } else if (warp == 11) {  // Bh stores
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
+        const int4 t = tiles[ti];
+        const DevLayer &L = sh.layers[t.x];
+        const int kch = (int)((L.n + 63) / 64);
+        const int tr = 2 * t.y + (int)rank;
+        const bool real = (int64_t)tr * 128 < L.m;
+        for (int kc = 0; kc < kch; ++kc, ++it) {
+          const uint32_t sg = it % FB_ASTAGES, pg = (it / FB_ASTAGES) & 1u;
+          if (!ab.wait(&cvt[sg], pg, sh.status)) { ok = false; break; }
+          if (real) {
+            tma_store_2d(&maps[t.x].Bh_k, aring + sg * FB_GBOX, kc * 64, tr * 128);
+            bulk_commit();
+            bulk_wait_read<0>();
+          }
+          mbar_arrive(&gempty[sg]);
+        }
+      }
+      bulk_wait<0>();
+    }
+  } else if (warp == 1) {  // MMA issue (CTA 0)
+    if (lane == 0 && rank == 0) {
+      uint32_t it = 0, tcount = 0;
+      bool ok = true;
+      for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
+        const int4 t = tiles[ti];
+        const DevLayer &L = sh.layers[t.x];
+        const int kch = (int)((L.n + 63) / 64);
+        const uint32_t np = rpad16(L.r), nparts = (np + 255) / 256;
+        if (!ab.wait(acc_empty, (tcount & 1u) ^ 1u, sh.status)) break;
+        tc_fence_after();
+        for (int kc = 0; kc < kch; ++kc, ++it) {
+          const uint32_t sg = it % FB_ASTAGES, pg = (it / FB_ASTAGES) & 1u;
+          const uint32_t q = it % FB_QSTAGES, qph = (it / FB_QSTAGES) & 1u;
+          if (!ab.wait(&qfull[q], qph, sh.status) || !ab.wait(&afull[sg], pg, sh.status)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t aB = smem_u32(aring + sg * FB_GBOX), bB = smem_u32(qring + q * qstage_bytes);
+#pragma unroll
+          for (int k16 = 0; k16 < 4; ++k16) {
+            const uint64_t ad = smem_desc_sw128(aB + k16 * 32, 0, 1024);
+            for (uint32_t part = 0; part < nparts; ++part) {
+              const uint32_t n_here = 2u * half_cols(np, part);
+              const uint64_t bd = smem_desc_sw128(bB + part * 2u * BOX64 + k16 * 2048, BOX64, 1024);
+              umma_pair_bf16(tmem + part * 256u, ad, bd, idesc_bf16(256, n_here, false, true), (kc | k16) ? 1u : 0u);
+            }
+          }
+          umma_pair_commit_mc(&gempty[sg], 0x3);
+          umma_pair_commit_mc(&qempty[q], 0x3);
+        }
+        if (!ok) break;
+        umma_pair_commit_mc(acc_full, 0x3);
+        ++tcount;
+      }
+      umma_pair_commit(drain);
+      mbar_wait(drain, 0, sh.status);
+    }
+  } else if (warp <= 5) {  // epilogue
+    const bool leader = (warp == 2 && lane == 0);
+    uint32_t tcount = 0, ecount = 0;
+    for (int ti = off[seg]; ti < off[seg + 1]; ++ti) {
+      const int4 t = tiles[ti];
+      const DevLayer &L = sh.layers[t.x];
+      const int tr = 2 * t.y + (int)rank;
+      if (!named_and(1, 128, ab.wait(acc_full, tcount & 1u, sh.status))) break;
+      tc_fence_after();
+      if ((int64_t)tr * 128 < L.m)
+        store_accumulator(tmem, warp, lane, leader, qring, &maps[t.x].Praw, &maps[t.x].PTraw_t, L.r, L.m, tr * 128,
+                          ecount, 1, 0, 1);
+      tc_fence_before();
+      named_sync(1, 128);
+      if (leader) {
+        mbar_arrive_cluster(cluster_addr(acc_empty, 0));
+        bulk_wait_read<0>();
+        mbar_arrive(epi_free);
+      }
+      ++tcount;
+    }
+    if (leader) bulk_wait<0>();
+  } else {  // warps 6..9: B = M + G
+    const int ct = threadIdx.x - 6 * 32, cw = warp - 6;  // 0..127, 0..3
+    uint32_t it = 0;
+    for (int ti = off[seg]; ti < off[seg + 1]; ++ti) {
+      const int4 t = tiles[ti];
+      const DevLayer &L = sh.layers[t.x];
+      const int tr = 2 * t.y + (int)rank;
+      const int kch = (int)((L.n + 63) / 64);
+      double accb = 0.0, accm = 0.0;
+      bool ok = true;
+      for (int kc = 0; kc < kch; ++kc, ++it) {
+        const uint32_t sm = it % FB_MSTAGES, pm = (it / FB_MSTAGES) & 1u;
+        const uint32_t sg = it % FB_ASTAGES, pg = (it / FB_ASTAGES) & 1u;
+        const bool in = ab.wait(&mfull[sm], pm, sh.status) && ab.wait(&gfull[sg], pg, sh.status);
+        if (in) {
+          const uint8_t *sM = smem + sm * FB_MSLOT;
+          uint8_t *sG = aring + sg * FB_GBOX;
+          float fb = 0.f, fm = 0.f;
+#pragma unroll 4
+          for (int i = 0; i < 8; ++i) {
+            // element group e: rows 8 (e >> 6) + (e & 7), 16-byte chunk (e >> 3) & 7 (8 columns);
+            // the 8 threads of a shared-memory phase take 8 rows of one chunk (distinct banks)
+            const uint32_t e = (uint32_t)(i * 128 + ct);
+            const uint32_t row = (e & 7u) + 8u * (e >> 6), c = (e >> 3) & 7u, sw = row & 7u;
+            uint4 *ga = reinterpret_cast<uint4 *>(sG + row * 128u + ((c ^ sw) << 4));
+            const uint4 g = *ga;
+            const uint8_t *mrow = sM + (c >> 2) * FB_MBOX + row * 128u;
+            const uint32_t mc = 2u * (c & 3u);
+            const float4 m0 = *reinterpret_cast<const float4 *>(mrow + ((mc ^ sw) << 4));
+            const float4 m1 = *reinterpret_cast<const float4 *>(mrow + (((mc + 1u) ^ sw) << 4));
+            const float mv[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
+            const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
+            uint32_t hw[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const float b0 = mv[2 * q] + __uint_as_float(gw[q] << 16);
+              const float b1 = mv[2 * q + 1] + __uint_as_float(gw[q] & 0xffff0000u);
+              fm = fmaf(mv[2 * q], mv[2 * q], fm);
+              fm = fmaf(mv[2 * q + 1], mv[2 * q + 1], fm);
+              fb = fmaf(b0, b0, fb);
+              fb = fmaf(b1, b1, fb);
+              const __nv_bfloat162 h = __floats2bfloat162_rn(b0, b1);
+              hw[q] = *reinterpret_cast<const uint32_t *>(&h);
+            }
+            *ga = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+          }
+          accb += (double)fb;
+          accm += (double)fm;
+          fence_async_smem();  // the A box is read by the MMA and the Bh store (async proxy)
+        }
+        if (!named_and(2, 128, in)) { ok = false; break; }
+        if (ct == 0) {
+          mbar_arrive(&mempty[sm]);
+          mbar_arrive_cluster(cluster_addr(&afull[sg], 0));
+          mbar_arrive(&cvt[sg]);
+        }
+      }
+      if (!ok) break;
+      // the row tile's sums of B^2 and M_{t-1}^2: fixed-order fp64 reduction
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        accb += __shfl_xor_sync(0xffffffffu, accb, o);
+        accm += __shfl_xor_sync(0xffffffffu, accm, o);
+      }
+      if (lane == 0) {
+        red_s[0][cw] = accb;
+        red_s[1][cw] = accm;
+      }
+      named_sync(2, 128);
+      if (ct == 0 && (int64_t)tr * 128 < L.m) {
+        const int slot = L.bpart_off + tr;
+        sh.bpart[2 * slot] = (red_s[0][0] + red_s[0][1]) + (red_s[0][2] + red_s[0][3]);
+        sh.bpart[2 * slot + 1] = (red_s[1][0] + red_s[1][1]) + (red_s[1][2] + red_s[1][3]);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc_pair(tmem, tmem_cols);
+}
+
 // ================================================================== Q -> bf16 copy ===
 __global__ void __launch_bounds__(256) qn_refresh_kernel(Shared sh, const int4 *tiles) {
   const int4 t = tiles[blockIdx.x];  // {layer, first row, rows, 0}
@@ -329,6 +638,9 @@ uint32_t form_bq_smem(int nstages, uint32_t stage_bytes) {
   return 1024u + nstages * stage_bytes + 4 * EPI_BOX + 512u;  // + barriers
 }
 uint32_t btp_smem(int nstages, uint32_t stage_bytes) { return form_bq_smem(nstages, stage_bytes); }
+// Q ring of the fused kernel: FB_QSTAGES Q chunks, at least the epilogue's 4 staging boxes
+uint32_t fused_bq_qring(uint32_t bq_boxes) { return std::max(FB_QSTAGES * bq_boxes * BOX64, 4u * EPI_BOX); }
+uint32_t fused_bq_smem(uint32_t bq_boxes) { return 1024u + FB_Q_OFF + fused_bq_qring(bq_boxes) + 512u; }
 
 cudaError_t setup_bq_kernels(uint32_t f_smem, uint32_t r_smem) {
   cudaError_t e =
@@ -336,6 +648,16 @@ cudaError_t setup_bq_kernels(uint32_t f_smem, uint32_t r_smem) {
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(tc_tma_gemm_kernel<GEMM_BTP>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)r_smem);
   return e;
+}
+
+cudaError_t setup_fused_bq_kernel(uint32_t smem) {
+  return cudaFuncSetAttribute(tc_form_bq_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+}
+
+void launch_fused_bq(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
+  if (tp.d_bq.grid <= 0) return;
+  tc_form_bq_kernel<<<2 * tp.d_bq.grid, FB_THREADS, tp.fb_smem, s>>>(
+      sh, tp.d_bq.tiles, tp.d_bq.off, tp.maps, tp.bq_boxes * BOX64, fused_bq_qring(tp.bq_boxes), tp.tmem_cols);
 }
 
 void launch_form_bq(const Shared &sh, const TcPlan &tp, cudaStream_t s) {

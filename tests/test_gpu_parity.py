@@ -171,6 +171,15 @@ def test_ragged_shapes_bf16(pad):
     run_per_step(RAGGED, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_ALWAYS), RAGGED.steps, TOL_BF16, pad=pad)
 
 
+def test_ragged_shapes_bf16_fp32_gradients():
+    """fp32 gradients in the tensor-core mode take the separate buffer pass (B written back to
+    M) and the unfused B Q kernel; bf16 gradients take the fused buffer + B Q kernel."""
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.scaled(RAGGED, "ragged_fp32g", RAGGED.shapes, g_dtype="fp32")
+    run_per_step(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_ALWAYS), w.steps, TOL_BF16, pad=1)
+
+
 def test_gpt160m_block_r192_bf16():
     import paper_2512_13728_gb300 as cd
 
@@ -264,6 +273,27 @@ def test_deterministic_bitwise():
             plan.step(cd.hparams(step=t))
         torch.cuda.synchronize()
         outs.append([x.clone() for x in st.X + st.M + st.Q] + [plan.rmmc.clone()])
+        plan.close()
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("g_dtype", ["bf16", "fp32"])
+def test_deterministic_bitwise_bf16_mode(g_dtype):
+    """The tensor-core mode repeats bit for bit (fixed-order norm and column reductions)."""
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.scaled(RAGGED, "ragged_det", RAGGED.shapes, g_dtype=g_dtype)
+    outs = []
+    for _ in range(2):
+        st = gu.make_state(w)
+        plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_BF16)
+        for t in range(1, 4):
+            gu.write_gradients(st, t)
+            plan.step(cd.hparams(step=t))
+        torch.cuda.synchronize()
+        assert plan.device_status() == 0
+        outs.append([x.clone() for x in st.X + st.M + st.Q] + [plan.rmmc.clone(), plan.rmmc_eq1.clone()])
         plan.close()
     for a, b in zip(*outs):
         assert torch.equal(a, b)
