@@ -243,33 +243,34 @@ def run_ours(args, rank, world, local_rank):
     ms_step = ms_total / args.steps
 
     # ---- end to end: H2D of the step's gradient from pinned host memory + step + D2H of results ----
+    # Through the C ABI's host-gradient entry point: each step copies every layer's G_t from
+    # pinned host memory into one of the plan's two device buffers (on the plan's copy stream,
+    # overlapping the previous step's kernels), runs the step behind the copies, and reads the
+    # step's RMMC values and flags back into pinned host memory.
     host_G = [g.cpu().pin_memory() for g in G]
     host_out = torch.empty(w.num_layers * 9 + 1, dtype=torch.uint8).pin_memory()
     h2d = sum(g.numel() * g.element_size() for g in host_G)
     d2h = plan.rmmc[: w.num_layers].numel() * 8 + w.num_layers + 1
     e_steps = max(1, min(args.steps, 10))
-    torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
-    # the gradients go up on several side streams (one copy engine each), joined before the step
-    up = [torch.cuda.Stream(dev) for _ in range(4)]
-    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    f0.record(stream)
-    for _ in range(e_steps):
-        start = torch.cuda.Event()
-        start.record(stream)
-        for i, (g, hg) in enumerate(zip(G, host_G)):
-            us = up[i % len(up)]
-            if i < len(up):
-                us.wait_event(start)  # after the previous step's kernels have read G
-            with torch.cuda.stream(us):
-                g.copy_(hg, non_blocking=True)
-        for us in up:
-            stream.wait_stream(us)
-        one_step()
+    plan.enable_host_gradients()
+
+    def e2e_step():
+        nonlocal t
+        t += 1
+        plan.step_host(cd.hparams(step=t, gate_mode=gate, tau_global=args.tau), host_G, stream=stream.cuda_stream)
         host_out[: 8 * w.num_layers].copy_(plan.rmmc[: w.num_layers].view(torch.uint8), non_blocking=True)
         host_out[8 * w.num_layers: 9 * w.num_layers].copy_(plan.flags[: w.num_layers], non_blocking=True)
         host_out[9 * w.num_layers:].copy_(plan.global_flag, non_blocking=True)
+
+    for _ in range(max(2, args.warmup)):  # first use of the pinned pages and buffers stays untimed
+        e2e_step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    f0.record(stream)
+    for _ in range(e_steps):
+        e2e_step()
     f1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = f0.elapsed_time(f1) / e_steps

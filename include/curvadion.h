@@ -124,6 +124,30 @@ dion_status dion_step(dion_plan *plan, const dion_hparams *hp, double *prev_norm
                       double *rmmc_out, double *rmmc_eq1_out, uint8_t *sync_flags_out,
                       uint8_t *global_flag_out, void *stream);
 
+/* Gradients from host memory (no counterpart in the paper: it moves Algorithm 1's input G_t
+ * onto the device).  dion_plan_enable_host_gradients allocates, once, two device gradient
+ * buffers per layer (the layer's g_dtype, rows padded to 16 bytes: 2 x sum m n x 2 or 4
+ * bytes), a copy stream and four events; the G pointers given to dion_plan_create are no
+ * longer read by dion_step_host (dion_step still reads them).  Calling it again is a no-op.
+ * Errors: INVALID_ARG (NULL plan), CUDA (allocation).
+ *
+ * dion_step_host is dion_step with layer l's G_t read from host memory: host_G[l] points to
+ * m x n elements of the layer's g_dtype, row-major with leading dimension host_ldg[l] >= n
+ * (elements).  Consecutive calls alternate between the two device buffers.  The copies of
+ * this call go on the plan's copy stream, which waits only for the step two calls back (the
+ * last reader of the same buffer), so they overlap the previous step's kernels; the step is
+ * then enqueued on `stream` behind the copies.  Outputs and errors as dion_step.  The host
+ * memory should be page-locked (cudaHostAlloc / cudaHostRegister) for the copies to run
+ * asynchronously, and must not change until they have executed, i.e. until `stream` has
+ * passed this step's first kernel (synchronizing `stream` after the call is enough).
+ * Errors also: INVALID_ARG when host gradients were not enabled or a pointer or leading
+ * dimension is invalid. */
+dion_status dion_plan_enable_host_gradients(dion_plan *plan);
+dion_status dion_step_host(dion_plan *plan, const dion_hparams *hp, const void *const *host_G,
+                           const int64_t *host_ldg, double *prev_norm, double *rmmc_out,
+                           double *rmmc_eq1_out, uint8_t *sync_flags_out, uint8_t *global_flag_out,
+                           void *stream);
+
 /* Reads the plan's device status word (synchronously; call after the step's stream has
  * been synchronized) into *code_out as a dion_status, and clears it if `clear` != 0.
  * The first device error of any step since the last clear is kept. */

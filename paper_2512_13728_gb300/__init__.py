@@ -72,6 +72,29 @@ class Plan:
                          self.rmmc_eq1.data_ptr() if eq1 else None, self.flags.data_ptr(),
                          self.global_flag.data_ptr(), s)
 
+    def enable_host_gradients(self) -> None:
+        """Lets step_host read each step's gradients from host memory (two device buffers per
+        layer, filled in turn on the plan's copy stream)."""
+        native.dion_plan_enable_host_gradients(self.handle)
+
+    def step_host(self, hp: dion_hparams, host_G: Sequence, stream: Optional[int] = None, eq1: bool = True) -> None:
+        """One step with the gradients read from host tensors (row-major 2-D CPU tensors of each
+        layer's gradient dtype and shape; pinned memory lets the copies overlap the previous
+        step).  The tensors must not change until the step's stream has passed its start."""
+        import torch
+
+        if len(host_G) != self.num_layers:
+            raise ValueError("one host gradient per layer")
+        for g, ly in zip(host_G, self.layers):
+            want = torch.bfloat16 if ly.g_dtype == DION_DTYPE_BF16 else torch.float32
+            if g.is_cuda or g.dtype != want or g.dim() != 2 or tuple(g.shape) != (ly.m, ly.n) or g.stride(1) != 1:
+                raise ValueError("host gradients must be row-major CPU tensors of the layer's shape and dtype")
+        s = torch.cuda.current_stream(self.device).cuda_stream if stream is None else stream
+        native.dion_step_host(self.handle, hp, [g.data_ptr() for g in host_G], [g.stride(0) for g in host_G],
+                              self.prev_norm.data_ptr(), self.rmmc.data_ptr(),
+                              self.rmmc_eq1.data_ptr() if eq1 else None, self.flags.data_ptr(),
+                              self.global_flag.data_ptr(), s)
+
     def refresh(self, stream: Optional[int] = None) -> None:
         """Call after writing Q from outside dion_step (e.g. a checkpoint restore)."""
         import torch

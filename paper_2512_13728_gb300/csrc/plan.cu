@@ -38,6 +38,19 @@ struct dion_plan {
   std::vector<cudaEvent_t> ev;  // [max_steps][launches + 1]
   std::vector<const char *> names;
   int32_t timing_steps = 0, recorded = 0, cursor = 0;
+  // host gradients (dion_step_host): two device gradient buffers per layer, filled in turn
+  std::vector<DevLayer> dl_host;  // the layer records as uploaded at creation
+  struct HostGrad {
+    bool on = false;
+    void *mem = nullptr;  // both buffers' gradients, both layer tables, both map tables
+    DevLayer *layers[2] = {};
+    tc::LayerMaps *maps[2] = {};
+    std::vector<char *> g[2];     // per layer device gradient of each buffer
+    std::vector<int64_t> ldg;     // their leading dimension (elements)
+    cudaStream_t copy = nullptr;
+    cudaEvent_t up[2] = {}, used[2] = {};
+    int parity = 0;
+  } hg;
 };
 
 namespace cd {
@@ -291,6 +304,7 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
 
   cudaError_t e = cudaSuccess;
   if (e == cudaSuccess) e = upload(p->sh.layers, dl);
+  p->dl_host = dl;
   if (e == cudaSuccess) e = upload(p->btiles, bt);
   if (e == cudaSuccess) e = upload(p->utiles, ut);
   if (e == cudaSuccess) e = upload(p->ctiles, ct);
@@ -322,9 +336,12 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
   return DION_OK;
 }
 
-dion_status dion_step(dion_plan *p, const dion_hparams *hp, double *prev_norm, double *rmmc_out,
-                      double *rmmc_eq1_out, uint8_t *sync_flags_out, uint8_t *global_flag_out,
-                      void *stream) {
+}  // extern "C"
+
+namespace {
+
+dion_status check_step_args(const dion_plan *p, const dion_hparams *hp, const double *prev_norm,
+                            const double *rmmc_out, const uint8_t *sync_flags_out, const uint8_t *global_flag_out) {
   if (!p || !hp || !prev_norm || !rmmc_out || !sync_flags_out || !global_flag_out) return DION_ERR_INVALID_ARG;
   if (hp->gate_mode < DION_GATE_ALWAYS || hp->gate_mode > DION_GATE_SCHEDULED) return DION_ERR_INVALID_ARG;
   if (hp->gate_mode == DION_GATE_SCHEDULED && hp->period < 1) return DION_ERR_INVALID_ARG;
@@ -333,18 +350,21 @@ dion_status dion_step(dion_plan *p, const dion_hparams *hp, double *prev_norm, d
       !std::isfinite(hp->eps_rmmc) || !std::isfinite(hp->eps_col) || std::isnan(hp->tau_global))
     return DION_ERR_INVALID_ARG;
   if (hp->eps_rmmc < 0.f || hp->eps_col < 0.f) return DION_ERR_INVALID_ARG;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  return DION_OK;
+}
+
+// Enqueues the step's launch sequence on s with the given layer table and tensor maps (the
+// plan's own, or those of a host-gradient buffer).  The caller has checked the arguments and
+// made the plan's device current.
+void enqueue_step(dion_plan *p, const Shared &sh, const tc::TcPlan &tcp, const dion_hparams *hp, double *prev_norm,
+                  double *rmmc_out, double *rmmc_eq1_out, uint8_t *sync_flags_out, uint8_t *global_flag_out,
+                  cudaStream_t s) {
   StepArgs a{};
   a.mu = hp->mu; a.eta = hp->eta; a.eta_local = hp->eta_local;
   a.eps_rmmc = hp->eps_rmmc; a.eps_col = hp->eps_col; a.tau_global = hp->tau_global;
   a.gate_mode = hp->gate_mode; a.period = hp->period < 1 ? 1 : hp->period; a.step = hp->step;
   a.prev_norm = prev_norm; a.rmmc = rmmc_out; a.eq1 = rmmc_eq1_out;
   a.flags = sync_flags_out; a.gflag = global_flag_out;
-  const Shared &sh = p->sh;
-  int cur = -1;
-  if (cudaGetDevice(&cur) != cudaSuccess || cur != p->device) {
-    if (cudaSetDevice(p->device) != cudaSuccess) return DION_ERR_CUDA;
-  }
   tick_begin(p, s);
   if (p->precision == DION_PREC_FP32) {
     launch_form_b(sh, p->btiles, p->n_btiles, s);
@@ -375,12 +395,145 @@ dion_status dion_step(dion_plan *p, const dion_hparams *hp, double *prev_norm, d
     launch_finalize(sh, a, s);                                      // Equation 1
     tick(p, s, "finalize");
   } else {
-    tc::step(p, p->tcp, sh, a, p->btiles, p->n_btiles, p->ctiles, p->n_ctiles, p->chol_smem, s);
+    tc::step(p, tcp, sh, a, p->btiles, p->n_btiles, p->ctiles, p->n_ctiles, p->chol_smem, s);
   }
   tick_end(p);
-  if (cudaGetLastError() != cudaSuccess) return DION_ERR_CUDA;
-  if (cur >= 0 && cur != p->device) cudaSetDevice(cur);
+}
+
+// Makes the plan's device current for the duration of a call.
+struct DeviceGuard {
+  int prev = -1;
+  bool ok = true;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) != cudaSuccess || prev != dev) ok = cudaSetDevice(dev) == cudaSuccess;
+  }
+  ~DeviceGuard() {
+    if (prev >= 0 && ok) cudaSetDevice(prev);
+  }
+};
+
+}  // namespace
+
+extern "C" {
+
+dion_status dion_step(dion_plan *p, const dion_hparams *hp, double *prev_norm, double *rmmc_out,
+                      double *rmmc_eq1_out, uint8_t *sync_flags_out, uint8_t *global_flag_out,
+                      void *stream) {
+  const dion_status st = check_step_args(p, hp, prev_norm, rmmc_out, sync_flags_out, global_flag_out);
+  if (st != DION_OK) return st;
+  DeviceGuard g(p->device);
+  if (!g.ok) return DION_ERR_CUDA;
+  enqueue_step(p, p->sh, p->tcp, hp, prev_norm, rmmc_out, rmmc_eq1_out, sync_flags_out, global_flag_out,
+               static_cast<cudaStream_t>(stream));
+  return cudaGetLastError() == cudaSuccess ? DION_OK : DION_ERR_CUDA;
+}
+
+dion_status dion_plan_enable_host_gradients(dion_plan *p) {
+  if (!p) return DION_ERR_INVALID_ARG;
+  if (p->hg.on) return DION_OK;
+  DeviceGuard g(p->device);
+  if (!g.ok) return DION_ERR_CUDA;
+  auto &hg = p->hg;
+  const int32_t L = p->L;
+  Carver cv;
+  std::vector<size_t> off[2];
+  hg.ldg.resize(L);
+  for (int b = 0; b < 2; ++b) {
+    off[b].resize(L);
+    for (int32_t l = 0; l < L; ++l) {
+      const DevLayer &d = p->dl_host[l];
+      const int64_t esz = d.g_dtype == DT_BF16 ? 2 : 4, ld = (d.n * esz + 15) / 16 * 16 / esz;
+      hg.ldg[l] = ld;
+      off[b][l] = cv.take<char>((size_t)(d.m * ld * esz));
+    }
+  }
+  const size_t o_layers[2] = {cv.take<DevLayer>(std::max(L, 1)), cv.take<DevLayer>(std::max(L, 1))};
+  const bool tcm = p->precision != DION_PREC_FP32;
+  size_t o_maps[2] = {0, 0};
+  if (tcm) {
+    cv.off = (cv.off + 127) / 128 * 128;
+    o_maps[0] = cv.take<tc::LayerMaps>(std::max(L, 1));
+    o_maps[1] = cv.take<tc::LayerMaps>(std::max(L, 1));
+  }
+  if (cudaMalloc(&hg.mem, cv.off) != cudaSuccess) {
+    hg.mem = nullptr;
+    return DION_ERR_CUDA;
+  }
+  char *base = static_cast<char *>(hg.mem);
+  cudaError_t e = cudaSuccess;
+  for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
+    std::vector<DevLayer> dl = p->dl_host;
+    hg.g[b].resize(L);
+    for (int32_t l = 0; l < L; ++l) {
+      hg.g[b][l] = base + off[b][l];
+      dl[l].G = hg.g[b][l];
+      dl[l].ldg = hg.ldg[l];
+    }
+    hg.layers[b] = reinterpret_cast<DevLayer *>(base + o_layers[b]);
+    e = upload(hg.layers[b], dl);
+    if (e == cudaSuccess && tcm) {
+      hg.maps[b] = reinterpret_cast<tc::LayerMaps *>(base + o_maps[b]);
+      e = tc::encode_maps(dl.data(), L, hg.maps[b]);
+    }
+  }
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&hg.copy, cudaStreamNonBlocking);
+  for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
+    e = cudaEventCreateWithFlags(&hg.up[b], cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&hg.used[b], cudaEventDisableTiming);
+  }
+  if (e != cudaSuccess) {
+    for (int b = 0; b < 2; ++b) {
+      if (hg.up[b]) cudaEventDestroy(hg.up[b]);
+      if (hg.used[b]) cudaEventDestroy(hg.used[b]);
+      hg.up[b] = hg.used[b] = nullptr;
+    }
+    if (hg.copy) cudaStreamDestroy(hg.copy);
+    hg.copy = nullptr;
+    cudaFree(hg.mem);
+    hg.mem = nullptr;
+    return DION_ERR_CUDA;
+  }
+  hg.parity = 0;
+  hg.on = true;
   return DION_OK;
+}
+
+dion_status dion_step_host(dion_plan *p, const dion_hparams *hp, const void *const *host_G, const int64_t *host_ldg,
+                           double *prev_norm, double *rmmc_out, double *rmmc_eq1_out, uint8_t *sync_flags_out,
+                           uint8_t *global_flag_out, void *stream) {
+  const dion_status st = check_step_args(p, hp, prev_norm, rmmc_out, sync_flags_out, global_flag_out);
+  if (st != DION_OK) return st;
+  if (!p->hg.on || (p->L > 0 && (!host_G || !host_ldg))) return DION_ERR_INVALID_ARG;
+  for (int32_t l = 0; l < p->L; ++l)
+    if (!host_G[l] || host_ldg[l] < p->dl_host[l].n) return DION_ERR_INVALID_ARG;
+  DeviceGuard g(p->device);
+  if (!g.ok) return DION_ERR_CUDA;
+  auto &hg = p->hg;
+  const int b = hg.parity;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // buffer b was last read by the step two calls back
+  if (cudaStreamWaitEvent(hg.copy, hg.used[b], 0) != cudaSuccess) return DION_ERR_CUDA;
+  for (int32_t l = 0; l < p->L; ++l) {
+    const DevLayer &d = p->dl_host[l];
+    const size_t esz = d.g_dtype == DT_BF16 ? 2 : 4;
+    cudaError_t e;
+    if (host_ldg[l] == hg.ldg[l])
+      e = cudaMemcpyAsync(hg.g[b][l], host_G[l], (size_t)(d.m * hg.ldg[l]) * esz, cudaMemcpyHostToDevice, hg.copy);
+    else
+      e = cudaMemcpy2DAsync(hg.g[b][l], (size_t)hg.ldg[l] * esz, host_G[l], (size_t)host_ldg[l] * esz,
+                            (size_t)d.n * esz, (size_t)d.m, cudaMemcpyHostToDevice, hg.copy);
+    if (e != cudaSuccess) return DION_ERR_CUDA;
+  }
+  if (cudaEventRecord(hg.up[b], hg.copy) != cudaSuccess || cudaStreamWaitEvent(s, hg.up[b], 0) != cudaSuccess)
+    return DION_ERR_CUDA;
+  Shared sh = p->sh;
+  sh.layers = hg.layers[b];
+  tc::TcPlan tcp = p->tcp;
+  if (p->precision != DION_PREC_FP32) tcp.maps = hg.maps[b];
+  enqueue_step(p, sh, tcp, hp, prev_norm, rmmc_out, rmmc_eq1_out, sync_flags_out, global_flag_out, s);
+  if (cudaEventRecord(hg.used[b], s) != cudaSuccess) return DION_ERR_CUDA;
+  hg.parity ^= 1;
+  return cudaGetLastError() == cudaSuccess ? DION_OK : DION_ERR_CUDA;
 }
 
 dion_status dion_get_device_status(dion_plan *p, int32_t clear, int32_t *code_out) {
@@ -453,6 +606,12 @@ void dion_plan_destroy(dion_plan *p) {
   if (!p) return;
   cudaDeviceSynchronize();
   free_events(p);
+  for (int b = 0; b < 2; ++b) {
+    if (p->hg.up[b]) cudaEventDestroy(p->hg.up[b]);
+    if (p->hg.used[b]) cudaEventDestroy(p->hg.used[b]);
+  }
+  if (p->hg.copy) cudaStreamDestroy(p->hg.copy);
+  cudaFree(p->hg.mem);
   tc::destroy(&p->tcp);
   cudaFree(p->ws);
   delete p;

@@ -474,7 +474,7 @@ void bind(const TcLayout &lo, char *base, DevLayer *dl, int32_t L, TcPlan *tp) {
   bind_sched(lo.s_trsm, tp->d_trsm);
 }
 
-cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, TcPlan *tp) {
+cudaError_t encode_maps(const DevLayer *dl, int32_t L, LayerMaps *dst) {
   std::vector<LayerMaps> maps(std::max(L, 1));
   std::memset(maps.data(), 0, sizeof(LayerMaps) * maps.size());
   for (int32_t l = 0; l < L; ++l) {
@@ -505,10 +505,14 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
                     encode_f32_2d(&m.Linv, d.Linv, d.r, d.r, p32, 32, 128);
     if (!ok) return cudaErrorInvalidValue;
   }
+  return cudaMemcpy(dst, maps.data(), sizeof(LayerMaps) * maps.size(), cudaMemcpyHostToDevice);
+}
+
+cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, TcPlan *tp) {
+  cudaError_t e = encode_maps(dl, L, tp->maps);
   auto up = [&](int4 *dst, const std::vector<int4> &v) {
     return v.empty() ? cudaSuccess : cudaMemcpy(dst, v.data(), sizeof(int4) * v.size(), cudaMemcpyHostToDevice);
   };
-  cudaError_t e = cudaMemcpy(tp->maps, maps.data(), sizeof(LayerMaps) * maps.size(), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = up(tp->utiles, lo.utiles);
   if (e == cudaSuccess) e = up(tp->ftiles, lo.ftiles);
   if (e == cudaSuccess) e = up(tp->rtiles, lo.rtiles);

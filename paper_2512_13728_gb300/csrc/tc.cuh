@@ -103,6 +103,8 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
                    TcLayout *out);
 // Stores the workspace pointers of this path into the layer records.
 void bind(const TcLayout &lay, char *base, DevLayer *dl, int32_t L, TcPlan *tp);
+// Encodes the per-layer tensor maps of these layer records into dst (device, L entries).
+cudaError_t encode_maps(const DevLayer *dl, int32_t L, LayerMaps *dst);
 // Encodes the tensor maps, uploads tile lists, sets kernel attributes.
 cudaError_t init(const TcLayout &lay, char *base, const DevLayer *dl, int32_t L, TcPlan *tp);
 int32_t launches_per_step(const TcPlan &tp);

@@ -37,7 +37,7 @@ DION_MAX_RANK = 512
 # Every function declared in include/curvadion.h.
 EXPORTED = ("dion_plan_create", "dion_step", "dion_get_device_status", "dion_plan_refresh", "dion_step_launch_count",
             "dion_timing_enable", "dion_timing_read", "dion_buffer_norms_noalloc", "dion_plan_destroy",
-            "dion_status_string", "dion_abi_version")
+            "dion_status_string", "dion_abi_version", "dion_plan_enable_host_gradients", "dion_step_host")
 
 DION_NOALLOC_MAX_LAYERS = 256
 DION_NOALLOC_MAX_TILES = 65536
@@ -85,6 +85,10 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     lib.dion_plan_create.restype = C.c_int
     lib.dion_step.argtypes = [P, C.POINTER(dion_hparams), P, P, P, P, P, P]
     lib.dion_step.restype = C.c_int
+    lib.dion_plan_enable_host_gradients.argtypes = [P]
+    lib.dion_plan_enable_host_gradients.restype = C.c_int
+    lib.dion_step_host.argtypes = [P, C.POINTER(dion_hparams), C.POINTER(P), C.POINTER(C.c_int64), P, P, P, P, P, P]
+    lib.dion_step_host.restype = C.c_int
     lib.dion_get_device_status.argtypes = [P, C.c_int32, C.POINTER(C.c_int32)]
     lib.dion_get_device_status.restype = C.c_int
     lib.dion_plan_refresh.argtypes = [P, P]
@@ -134,6 +138,26 @@ def dion_step(plan: int, hp: dion_hparams, prev_norm: int, rmmc_out: int, rmmc_e
                           C.c_void_p(global_flag_out), C.c_void_p(stream) if stream else None)
     if st != DION_OK:
         raise DionError(st, "dion_step")
+
+
+def dion_plan_enable_host_gradients(plan: int) -> None:
+    st = load().dion_plan_enable_host_gradients(C.c_void_p(plan))
+    if st != DION_OK:
+        raise DionError(st, "dion_plan_enable_host_gradients")
+
+
+def dion_step_host(plan: int, hp: dion_hparams, host_G, host_ldg, prev_norm: int, rmmc_out: int, rmmc_eq1_out,
+                   sync_flags_out: int, global_flag_out: int, stream: int) -> None:
+    """host_G: host addresses (ints) of the layers' gradients, host_ldg: their leading dimensions
+    (elements); the other pointers are device addresses as in dion_step."""
+    n = max(len(host_G), 1)
+    gp = (C.c_void_p * n)(*[C.c_void_p(int(a)) for a in host_G])
+    ld = (C.c_int64 * n)(*[int(v) for v in host_ldg])
+    st = load().dion_step_host(C.c_void_p(plan), C.byref(hp), gp, ld, C.c_void_p(prev_norm), C.c_void_p(rmmc_out),
+                               C.c_void_p(rmmc_eq1_out) if rmmc_eq1_out else None, C.c_void_p(sync_flags_out),
+                               C.c_void_p(global_flag_out), C.c_void_p(stream) if stream else None)
+    if st != DION_OK:
+        raise DionError(st, "dion_step_host")
 
 
 def dion_get_device_status(plan: int, clear: bool = True) -> int:

@@ -96,4 +96,6 @@ def test_step_rejects_null_plan(lib):
     code = C.c_int32()
     assert lib.dion_get_device_status(None, 0, C.byref(code)) == 1
     assert lib.dion_step_launch_count(None) == 0
+    assert lib.dion_plan_enable_host_gradients(None) == 1
+    assert lib.dion_step_host(None, C.byref(hp), None, None, None, None, None, None, None, None) == 1
     lib.dion_plan_destroy(None)  # no-op

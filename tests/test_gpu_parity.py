@@ -299,6 +299,47 @@ def test_deterministic_bitwise_bf16_mode(g_dtype):
         assert torch.equal(a, b)
 
 
+@pytest.mark.parametrize("prec,g_dtype", [("bf16", "bf16"), ("bf16", "fp32"), ("fp32", "bf16")])
+def test_step_host_matches_device_gradients(prec, g_dtype):
+    """dion_step_host (gradients copied from pinned host tensors into the plan's two alternating
+    buffers) gives bit for bit the results of dion_step on the same gradients in device memory;
+    the host tensors of odd steps have a padded leading dimension (2-D copy)."""
+    import paper_2512_13728_gb300 as cd
+
+    p = cd.DION_PREC_BF16 if prec == "bf16" else cd.DION_PREC_FP32
+    w = wl.scaled(RAGGED, "ragged_host", RAGGED.shapes, g_dtype=g_dtype, steps=5)
+    outs = []
+    for host in (False, True):
+        st = gu.make_state(w)
+        plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, p)
+        if host:
+            plan.enable_host_gradients()
+            plan.enable_host_gradients()  # a second call is a no-op
+        seq = []
+        for t in range(1, w.steps + 1):
+            gu.write_gradients(st, t)
+            if host:
+                hg = []
+                for g in st.G:
+                    m, n = g.shape
+                    pad = 8 if t % 2 else 0
+                    buf = torch.full((m, n + pad), float("nan"), dtype=g.dtype).pin_memory()
+                    buf[:, :n].copy_(g.cpu())
+                    hg.append(buf[:, :n])
+                    g.fill_(float("nan"))  # the device copies given at creation are not read
+                plan.step_host(cd.hparams(step=t), hg)
+                torch.cuda.synchronize()
+            else:
+                plan.step(cd.hparams(step=t))
+            seq.append((plan.rmmc.clone(), plan.flags.clone(), plan.global_flag.clone()))
+        torch.cuda.synchronize()
+        assert plan.device_status() == 0
+        outs.append([x.clone() for x in st.X + st.M + st.Q] + [v for tup in seq for v in tup])
+        plan.close()
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
+
+
 def test_checkpoint_resume_bitwise():
     """10 steps == 5 steps, copy all state out and into fresh buffers and a fresh plan, 5 steps."""
     import paper_2512_13728_gb300 as cd
