@@ -38,7 +38,7 @@
 extern "C" {
 #endif
 
-#define DION_ABI_VERSION 1
+#define DION_ABI_VERSION 2
 
 typedef enum {
   DION_OK = 0,
@@ -100,6 +100,10 @@ typedef struct {
   int32_t gate_mode; /* DION_GATE_* */
   int32_t period;    /* H of DION_GATE_SCHEDULED (>= 1) */
   int64_t step;      /* 1-based step index t */
+  float weight_decay; /* decoupled weight decay (Section 4 trains with 0.01; 0 = Algorithms 1/2 as
+                       * printed): X is multiplied by (1 - lr * weight_decay) before the branch's
+                       * update, lr = eta in the Dion branch and eta_local in the local branch.
+                       * Must be finite and >= 0. */
 } dion_hparams;
 
 typedef struct dion_plan dion_plan;
@@ -147,6 +151,17 @@ dion_status dion_step_host(dion_plan *plan, const dion_hparams *hp, const void *
                            const int64_t *host_ldg, double *prev_norm, double *rmmc_out,
                            double *rmmc_eq1_out, uint8_t *sync_flags_out, uint8_t *global_flag_out,
                            void *stream);
+
+/* Host helpers for the training loop of Section 4 (no device work, callable without a GPU).
+ * dion_lr_schedule: learning rate at 1-based `step` of a `total_steps` run with linear warmup
+ * and warmdown (Section 4: 1% warmup, 10% or 20% warmdown): with W = warmup_frac T and
+ * D = warmdown_frac T rounded half up, base_lr * step / W for step <= W, base_lr * (T - step) / D for
+ * step > T - D (0 at the last step), base_lr otherwise; step is clamped to [1, T].  Returns
+ * NaN for total_steps < 1, fractions outside [0, 1] or warmup + warmdown steps > T.
+ * dion_rank_for: Dion rank for a rank fraction (Section 4: 0.125): ceil(fraction min(m, n)),
+ * clamped to [1, min(m, n)]; returns 0 for m < 1, n < 1 or fraction outside (0, 1]. */
+float dion_lr_schedule(int64_t step, int64_t total_steps, float base_lr, float warmup_frac, float warmdown_frac);
+int64_t dion_rank_for(int64_t m, int64_t n, double fraction);
 
 /* Reads the plan's device status word (synchronously; call after the step's stream has
  * been synchronized) into *code_out as a dion_status, and clears it if `clear` != 0.

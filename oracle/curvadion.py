@@ -27,6 +27,14 @@ Readings where the paper is silent (each is also listed in the design notes):
 * Equation 1's ratio takes the same epsilon as Algorithm 2 in its denominator so that the
   first step (zero momentum) is finite;
 * the local branch keeps M = B with no decay, exactly as Algorithm 2 writes it.
+* weight decay (Section 4 trains with 0.01 but Algorithms 1/2 have no such line) is decoupled:
+  X is multiplied by (1 - lr * weight_decay) before the branch's update, lr being the branch's
+  learning rate (eta for the Dion update, eta_local for the local one); weight_decay = 0 is the
+  algorithm as printed;
+* the learning-rate schedule (Section 4: 1% warmup, 10% or 20% warmdown) is linear: it rises
+  from base/W at step 1 to base at step W, stays at base, and falls linearly to 0 at the last
+  step over the final D steps (W, D = warmup_frac * T, warmdown_frac * T rounded half up);
+* the Dion rank for a rank fraction f (Section 4: f = 0.125) is ceil(f * min(m, n)), at least 1.
 
 Pins: ``tests/test_oracle_pins.py`` checks every function here against results fixed by
 the paper or by mathematics (closed forms, LAPACK, brute force on tiny cases).
@@ -153,7 +161,38 @@ class SyncResult:
     R: np.ndarray
 
 
-def dion_sync_update(B, Q_prev, X, mu: float, eta: float, eps_col: float) -> SyncResult:
+def decay_parameters(X, lr: float, weight_decay: float):
+    """Decoupled weight decay applied before a branch's update: (1 - lr * weight_decay) X."""
+    return (1.0 - lr * weight_decay) * X
+
+
+def lr_schedule(step: int, total_steps: int, base_lr: float, warmup_frac: float, warmdown_frac: float) -> float:
+    """Learning rate at 1-based ``step`` of a ``total_steps`` run (Section 4's warmup/warmdown).
+
+    W = warmup_frac * T and D = warmdown_frac * T, each rounded half up, must fit in T.
+    W warmup steps: base * step / W for step <= W.  D warmdown steps: base * (T - step) / D for
+    step > T - D (ending at 0 on the last step).  Otherwise base.  Steps outside [1, T] clamp.
+    """
+    T = int(total_steps)
+    t = min(max(int(step), 1), T)
+    W = int(math.floor(warmup_frac * T + 0.5))
+    D = int(math.floor(warmdown_frac * T + 0.5))
+    if T < 1 or W + D > T:
+        raise ValueError("warmup and warmdown do not fit in the run")
+    if W > 0 and t <= W:
+        return base_lr * t / W
+    if D > 0 and t > T - D:
+        return base_lr * (T - t) / D
+    return base_lr
+
+
+def rank_for(m: int, n: int, fraction: float) -> int:
+    """Dion rank from a rank fraction (Section 4: r = 0.125): ceil(fraction * min(m, n)), >= 1."""
+    k = min(m, n)
+    return max(1, min(k, int(math.ceil(fraction * k - 1e-12))))
+
+
+def dion_sync_update(B, Q_prev, X, mu: float, eta: float, eps_col: float, weight_decay: float = 0.0) -> SyncResult:
     """The synchronized branch of Algorithm 2 (= one step of Algorithm 1 after the buffer).
 
     With one data-parallel worker the two AllReduce_DP lines are the identity.
@@ -162,20 +201,21 @@ def dion_sync_update(B, Q_prev, X, mu: float, eta: float, eps_col: float) -> Syn
       R  = B^T P
       M  = B - (1 - mu) P R^T
       Q  = ColumnNormalize(R)
-      X  = X - eta sqrt(m/n) P Q^T
+      X  = X - eta sqrt(m/n) P Q^T      (after decoupled weight decay of X, if any)
     """
     m, n = B.shape
     P = orthogonalize(power_iter(B, Q_prev))
     R = B.T @ P
     M_new = B - (1.0 - mu) * (P @ R.T)
     Q_new = column_normalize(R, eps_col)
-    X_new = X - eta * math.sqrt(m / n) * (P @ Q_new.T)
+    X_new = decay_parameters(X, eta, weight_decay) - eta * math.sqrt(m / n) * (P @ Q_new.T)
     return SyncResult(M=M_new, Q=Q_new, X=X_new, P=P, R=R)
 
 
-def local_update(B, G, X, eta_local: float):
-    """The local branch of Algorithm 2: M = B (no decay) and X = X - eta_local G."""
-    return B.copy(), X - eta_local * G
+def local_update(B, G, X, eta_local: float, weight_decay: float = 0.0):
+    """The local branch of Algorithm 2: M = B (no decay) and X = X - eta_local G (after
+    decoupled weight decay of X, if any)."""
+    return B.copy(), decay_parameters(X, eta_local, weight_decay) - eta_local * G
 
 
 # ---------------------------------------------------------------------------------------
@@ -234,6 +274,7 @@ class HParams:
     gate_mode: int = GATE_ALWAYS
     tau_global: float = 0.5
     period: int = 1
+    weight_decay: float = 0.0
 
 
 @dataclass
@@ -273,12 +314,12 @@ def curvadion_step(layers: Sequence[LayerState], grads: Sequence[np.ndarray],
     for i, st in enumerate(layers):
         X = as_f64(st.X)
         if active[i]:
-            res = dion_sync_update(Bs[i], as_f64(st.Q), X, hp.mu, hp.eta, hp.eps_col)
+            res = dion_sync_update(Bs[i], as_f64(st.Q), X, hp.mu, hp.eta, hp.eps_col, hp.weight_decay)
             new = LayerState(X=res.X, M=res.M, Q=res.Q, tau=st.tau)
             if keep_extras:
                 extras.append(res)
         else:
-            M_new, X_new = local_update(Bs[i], as_f64(grads[i]), X, hp.eta_local)
+            M_new, X_new = local_update(Bs[i], as_f64(grads[i]), X, hp.eta_local, hp.weight_decay)
             new = LayerState(X=X_new, M=M_new, Q=as_f64(st.Q), tau=st.tau)
             if keep_extras:
                 extras.append(None)

@@ -33,9 +33,21 @@ def _layer(X, M, Q, G, tau: float) -> dion_layer:
 
 
 def hparams(mu=0.95, eta=0.01, eta_local=None, eps_rmmc=1e-8, eps_col=1e-8, tau_global=0.5,
-            gate_mode=DION_GATE_ALWAYS, period=1, step=1) -> dion_hparams:
+            gate_mode=DION_GATE_ALWAYS, period=1, step=1, weight_decay=0.0) -> dion_hparams:
     return dion_hparams(mu=mu, eta=eta, eta_local=eta if eta_local is None else eta_local, eps_rmmc=eps_rmmc,
-                        eps_col=eps_col, tau_global=tau_global, gate_mode=gate_mode, period=period, step=step)
+                        eps_col=eps_col, tau_global=tau_global, gate_mode=gate_mode, period=period, step=step,
+                        weight_decay=weight_decay)
+
+
+def lr_schedule(step: int, total_steps: int, base_lr: float, warmup_frac: float = 0.01,
+                warmdown_frac: float = 0.1) -> float:
+    """Section 4's learning-rate schedule (the library's dion_lr_schedule)."""
+    return native.dion_lr_schedule(step, total_steps, base_lr, warmup_frac, warmdown_frac)
+
+
+def rank_for(m: int, n: int, fraction: float = 0.125) -> int:
+    """Dion rank for a rank fraction (the library's dion_rank_for)."""
+    return native.dion_rank_for(m, n, fraction)
 
 
 class Plan:

@@ -68,6 +68,7 @@ struct DevLayer {
 // Per-step scalars and output pointers, passed by value to the kernels.
 struct StepArgs {
   float mu, eta, eta_local, eps_rmmc, eps_col, tau_global;
+  float keep_sync, keep_local;  // decoupled weight decay: X scaled by 1 - lr * weight_decay
   int32_t gate_mode, period;
   int64_t step;
   double *prev_norm;
@@ -138,9 +139,9 @@ cudaError_t prepare_chol_inv(int32_t max_r, size_t *smem_out);
 void launch_chol_inv(const Shared &sh, size_t smem, int32_t pass, float near_identity, cudaStream_t s);
 void launch_colnorm(const Shared &sh, const int4 *tiles, int32_t ntiles, float eps_col,
                     cudaStream_t s);
-void launch_update(const Shared &sh, const int4 *tiles, int32_t ntiles, float mu, float eta,
+void launch_update(const Shared &sh, const int4 *tiles, int32_t ntiles, float mu, float eta, float keep,
                    cudaStream_t s);
-void launch_local(const Shared &sh, const int4 *tiles, int32_t ntiles, float eta_local,
+void launch_local(const Shared &sh, const int4 *tiles, int32_t ntiles, float eta_local, float keep,
                   cudaStream_t s);
 void launch_finalize(const Shared &sh, const StepArgs &a, cudaStream_t s);
 

@@ -714,7 +714,8 @@ void launch_colnorm(const Shared &sh, const int4 *tiles, int32_t ntiles, float e
 // fp64 partial of ||M_t||^2 for Equation 1.  Tile = {layer, tile row, tile col, slot}.
 constexpr int UBM = 64, UBN = 64, UBK = 16, kUpdThreads = 256;
 
-__global__ void __launch_bounds__(kUpdThreads) update_kernel(Shared sh, const int4 *tiles, float mu, float eta) {
+__global__ void __launch_bounds__(kUpdThreads) update_kernel(Shared sh, const int4 *tiles, float mu, float eta,
+                                                             float keep) {
   // P, R: ld ldp; Q: ld ldq
   __shared__ float As[UBK][UBM + 4];
   __shared__ float Rs[UBK][UBN + 4];
@@ -768,7 +769,7 @@ __global__ void __launch_bounds__(kUpdThreads) update_kernel(Shared sh, const in
       const float mn = fmaf(-dec, u1[i][j], *mp);
       *mp = mn;
       float *xp = L.X + gi * L.ldx + gj;
-      *xp = fmaf(-c, u2[i][j], *xp);
+      *xp = fmaf(-c, u2[i][j], *xp * keep);
       ss = fmaf(mn, mn, ss);
     }
   }
@@ -776,15 +777,17 @@ __global__ void __launch_bounds__(kUpdThreads) update_kernel(Shared sh, const in
   if (tid == 0) sh.upart[t.w] = tot;
 }
 
-void launch_update(const Shared &sh, const int4 *tiles, int32_t ntiles, float mu, float eta, cudaStream_t s) {
-  if (ntiles > 0) update_kernel<<<ntiles, kUpdThreads, 0, s>>>(sh, tiles, mu, eta);
+void launch_update(const Shared &sh, const int4 *tiles, int32_t ntiles, float mu, float eta, float keep,
+                   cudaStream_t s) {
+  if (ntiles > 0) update_kernel<<<ntiles, kUpdThreads, 0, s>>>(sh, tiles, mu, eta, keep);
 }
 
 // ======================================================================== local branch ===
-// Algorithm 2's else-branch: X = X - eta_local G, and M = B = M + G (already in place unless
-// the layer defers B to the update).
+// Algorithm 2's else-branch: X = X - eta_local G (after decoupled weight decay: X scaled by
+// keep = 1 - eta_local * weight_decay), and M = B = M + G (already in place unless the layer
+// defers B to the update).
 template <int GT>
-__device__ void local_tile(const DevLayer &L, int64_t row0, int64_t nrows, float eta_local) {
+__device__ void local_tile(const DevLayer &L, int64_t row0, int64_t nrows, float eta_local, float keep) {
   const int64_t n = L.n, n4 = n >> 2;
   const bool form_m = L.b_deferred != 0;
   for (int64_t rr = 0; rr < nrows; ++rr) {
@@ -795,8 +798,8 @@ __device__ void local_tile(const DevLayer &L, int64_t row0, int64_t nrows, float
       float4 x = *reinterpret_cast<float4 *>(Xrow + 4 * c4);
       float g[4];
       load_g4<GT>(L.G, goff + 4 * c4, g);
-      x.x = fmaf(-eta_local, g[0], x.x); x.y = fmaf(-eta_local, g[1], x.y);
-      x.z = fmaf(-eta_local, g[2], x.z); x.w = fmaf(-eta_local, g[3], x.w);
+      x.x = fmaf(-eta_local, g[0], x.x * keep); x.y = fmaf(-eta_local, g[1], x.y * keep);
+      x.z = fmaf(-eta_local, g[2], x.z * keep); x.w = fmaf(-eta_local, g[3], x.w * keep);
       *reinterpret_cast<float4 *>(Xrow + 4 * c4) = x;
       if (form_m) {
         float4 m = *reinterpret_cast<float4 *>(Mrow + 4 * c4);
@@ -806,22 +809,22 @@ __device__ void local_tile(const DevLayer &L, int64_t row0, int64_t nrows, float
     }
     for (int64_t c = 4 * n4 + threadIdx.x; c < n; c += kRowThreads) {
       const float g = load_g1<GT>(L.G, goff + c);
-      Xrow[c] = fmaf(-eta_local, g, Xrow[c]);
+      Xrow[c] = fmaf(-eta_local, g, Xrow[c] * keep);
       if (form_m) Mrow[c] += g;
     }
   }
 }
 
-__global__ void __launch_bounds__(kRowThreads) local_kernel(Shared sh, const int4 *tiles, float eta_local) {
+__global__ void __launch_bounds__(kRowThreads) local_kernel(Shared sh, const int4 *tiles, float eta_local, float keep) {
   const int4 t = tiles[blockIdx.x];
   if (sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
-  if (L.g_dtype == DT_BF16) local_tile<DT_BF16>(L, t.y, t.z, eta_local);
-  else local_tile<DT_FP32>(L, t.y, t.z, eta_local);
+  if (L.g_dtype == DT_BF16) local_tile<DT_BF16>(L, t.y, t.z, eta_local, keep);
+  else local_tile<DT_FP32>(L, t.y, t.z, eta_local, keep);
 }
 
-void launch_local(const Shared &sh, const int4 *tiles, int32_t ntiles, float eta_local, cudaStream_t s) {
-  if (ntiles > 0) local_kernel<<<ntiles, kRowThreads, 0, s>>>(sh, tiles, eta_local);
+void launch_local(const Shared &sh, const int4 *tiles, int32_t ntiles, float eta_local, float keep, cudaStream_t s) {
+  if (ntiles > 0) local_kernel<<<ntiles, kRowThreads, 0, s>>>(sh, tiles, eta_local, keep);
 }
 
 // ============================================================================ finalize ===

@@ -350,6 +350,7 @@ dion_status check_step_args(const dion_plan *p, const dion_hparams *hp, const do
       !std::isfinite(hp->eps_rmmc) || !std::isfinite(hp->eps_col) || std::isnan(hp->tau_global))
     return DION_ERR_INVALID_ARG;
   if (hp->eps_rmmc < 0.f || hp->eps_col < 0.f) return DION_ERR_INVALID_ARG;
+  if (!std::isfinite(hp->weight_decay) || hp->weight_decay < 0.f) return DION_ERR_INVALID_ARG;
   return DION_OK;
 }
 
@@ -362,6 +363,8 @@ void enqueue_step(dion_plan *p, const Shared &sh, const tc::TcPlan &tcp, const d
   StepArgs a{};
   a.mu = hp->mu; a.eta = hp->eta; a.eta_local = hp->eta_local;
   a.eps_rmmc = hp->eps_rmmc; a.eps_col = hp->eps_col; a.tau_global = hp->tau_global;
+  a.keep_sync = (float)(1.0 - (double)hp->eta * (double)hp->weight_decay);
+  a.keep_local = (float)(1.0 - (double)hp->eta_local * (double)hp->weight_decay);
   a.gate_mode = hp->gate_mode; a.period = hp->period < 1 ? 1 : hp->period; a.step = hp->step;
   a.prev_norm = prev_norm; a.rmmc = rmmc_out; a.eq1 = rmmc_eq1_out;
   a.flags = sync_flags_out; a.gflag = global_flag_out;
@@ -388,9 +391,9 @@ void enqueue_step(dion_plan *p, const Shared &sh, const tc::TcPlan &tcp, const d
     tick(p, s, "gemm_btp");
     launch_colnorm(sh, p->ctiles, p->n_ctiles, a.eps_col, s);       // Q = ColumnNormalize(R)
     tick(p, s, "colnorm");
-    launch_update(sh, p->utiles, p->n_utiles, a.mu, a.eta, s);      // M, X
+    launch_update(sh, p->utiles, p->n_utiles, a.mu, a.eta, a.keep_sync, s);  // M, X
     tick(p, s, "update");
-    launch_local(sh, p->btiles, p->n_btiles, a.eta_local, s);       // local branch
+    launch_local(sh, p->btiles, p->n_btiles, a.eta_local, a.keep_local, s);  // local branch
     tick(p, s, "local");
     launch_finalize(sh, a, s);                                      // Equation 1
     tick(p, s, "finalize");
@@ -534,6 +537,26 @@ dion_status dion_step_host(dion_plan *p, const dion_hparams *hp, const void *con
   if (cudaEventRecord(hg.used[b], s) != cudaSuccess) return DION_ERR_CUDA;
   hg.parity ^= 1;
   return cudaGetLastError() == cudaSuccess ? DION_OK : DION_ERR_CUDA;
+}
+
+float dion_lr_schedule(int64_t step, int64_t total_steps, float base_lr, float warmup_frac, float warmdown_frac) {
+  if (total_steps < 1 || !(warmup_frac >= 0.f && warmup_frac <= 1.f) || !(warmdown_frac >= 0.f && warmdown_frac <= 1.f))
+    return NAN;
+  const int64_t T = total_steps;
+  const int64_t W = (int64_t)std::floor((double)warmup_frac * (double)T + 0.5);  // rounded half up
+  const int64_t D = (int64_t)std::floor((double)warmdown_frac * (double)T + 0.5);
+  if (W + D > T) return NAN;
+  const int64_t t = std::min(std::max<int64_t>(step, 1), T);
+  if (W > 0 && t <= W) return (float)((double)base_lr * (double)t / (double)W);
+  if (D > 0 && t > T - D) return (float)((double)base_lr * (double)(T - t) / (double)D);
+  return base_lr;
+}
+
+int64_t dion_rank_for(int64_t m, int64_t n, double fraction) {
+  if (m < 1 || n < 1 || !(fraction > 0.0 && fraction <= 1.0)) return 0;
+  const int64_t k = std::min(m, n);
+  const int64_t r = (int64_t)std::ceil(fraction * (double)k - 1e-12);
+  return std::min(k, std::max<int64_t>(1, r));
 }
 
 dion_status dion_get_device_status(dion_plan *p, int32_t clear, int32_t *code_out) {

@@ -46,7 +46,7 @@ constexpr uint32_t U_IDESC = idesc_bf16(128, 128, false, false);
 // Tile = {layer, row-tile pair p, column tile, ||M_t|| slot of row tile 2 p}.
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
     tc_update_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off, const LayerMaps *__restrict__ maps,
-                     float mu, float eta) {
+                     float mu, float eta, float keep) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = align1024(smem_raw);
   uint8_t *stage = smem;
@@ -244,10 +244,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
             bv.y = fmaf(-dec, __uint_as_float(u1[cc + 1]), bv.y);
             bv.z = fmaf(-dec, __uint_as_float(u1[cc + 2]), bv.z);
             bv.w = fmaf(-dec, __uint_as_float(u1[cc + 3]), bv.w);
-            xv.x = fmaf(-c, __uint_as_float(u2[cc + 0]), xv.x);
-            xv.y = fmaf(-c, __uint_as_float(u2[cc + 1]), xv.y);
-            xv.z = fmaf(-c, __uint_as_float(u2[cc + 2]), xv.z);
-            xv.w = fmaf(-c, __uint_as_float(u2[cc + 3]), xv.w);
+            xv.x = fmaf(-c, __uint_as_float(u2[cc + 0]), xv.x * keep);  // keep: decoupled weight decay
+            xv.y = fmaf(-c, __uint_as_float(u2[cc + 1]), xv.y * keep);
+            xv.z = fmaf(-c, __uint_as_float(u2[cc + 2]), xv.z * keep);
+            xv.w = fmaf(-c, __uint_as_float(u2[cc + 3]), xv.w * keep);
             ss = fmaf(bv.x, bv.x, ss); ss = fmaf(bv.y, bv.y, ss);
             ss = fmaf(bv.z, bv.z, ss); ss = fmaf(bv.w, bv.w, ss);
             *reinterpret_cast<float4 *>(bs + o) = bv;
@@ -603,9 +603,9 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, c
   tick(p, s, "colnorm_scale");
   if (tp.d_update.grid > 0)
     tc_update_kernel<<<2 * tp.d_update.grid, U_THREADS, U_SMEM, s>>>(sh, tp.d_update.tiles, tp.d_update.off, tp.maps,
-                                                                      a.mu, a.eta);
+                                                                      a.mu, a.eta, a.keep_sync);
   tick(p, s, "tc_update");
-  launch_local(sh, btiles, n_btiles, a.eta_local, s);
+  launch_local(sh, btiles, n_btiles, a.eta_local, a.keep_local, s);
   tick(p, s, "local");
   launch_finalize(sh, a, s);
   tick(p, s, "finalize");

@@ -37,8 +37,10 @@ DION_MAX_RANK = 512
 # Every function declared in include/curvadion.h.
 EXPORTED = ("dion_plan_create", "dion_step", "dion_get_device_status", "dion_plan_refresh", "dion_step_launch_count",
             "dion_timing_enable", "dion_timing_read", "dion_buffer_norms_noalloc", "dion_plan_destroy",
-            "dion_status_string", "dion_abi_version", "dion_plan_enable_host_gradients", "dion_step_host")
+            "dion_status_string", "dion_abi_version", "dion_plan_enable_host_gradients", "dion_step_host",
+            "dion_lr_schedule", "dion_rank_for")
 
+DION_ABI_VERSION = 2
 DION_NOALLOC_MAX_LAYERS = 256
 DION_NOALLOC_MAX_TILES = 65536
 
@@ -60,6 +62,7 @@ class dion_hparams(C.Structure):
         ("mu", C.c_float), ("eta", C.c_float), ("eta_local", C.c_float),
         ("eps_rmmc", C.c_float), ("eps_col", C.c_float), ("tau_global", C.c_float),
         ("gate_mode", C.c_int32), ("period", C.c_int32), ("step", C.c_int64),
+        ("weight_decay", C.c_float),
     ]
 
 
@@ -89,6 +92,10 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     lib.dion_plan_enable_host_gradients.restype = C.c_int
     lib.dion_step_host.argtypes = [P, C.POINTER(dion_hparams), C.POINTER(P), C.POINTER(C.c_int64), P, P, P, P, P, P]
     lib.dion_step_host.restype = C.c_int
+    lib.dion_lr_schedule.argtypes = [C.c_int64, C.c_int64, C.c_float, C.c_float, C.c_float]
+    lib.dion_lr_schedule.restype = C.c_float
+    lib.dion_rank_for.argtypes = [C.c_int64, C.c_int64, C.c_double]
+    lib.dion_rank_for.restype = C.c_int64
     lib.dion_get_device_status.argtypes = [P, C.c_int32, C.POINTER(C.c_int32)]
     lib.dion_get_device_status.restype = C.c_int
     lib.dion_plan_refresh.argtypes = [P, P]
@@ -108,6 +115,9 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     lib.dion_status_string.restype = C.c_char_p
     lib.dion_abi_version.argtypes = []
     lib.dion_abi_version.restype = C.c_int32
+    if lib.dion_abi_version() != DION_ABI_VERSION:  # the structs above follow this version's header
+        raise ImportError(f"{path} has ABI version {lib.dion_abi_version()}, this binding expects {DION_ABI_VERSION}: "
+                          "rebuild it with `python -m paper_2512_13728_gb300.build --force`")
     _lib = lib
     return lib
 
@@ -138,6 +148,15 @@ def dion_step(plan: int, hp: dion_hparams, prev_norm: int, rmmc_out: int, rmmc_e
                           C.c_void_p(global_flag_out), C.c_void_p(stream) if stream else None)
     if st != DION_OK:
         raise DionError(st, "dion_step")
+
+
+def dion_lr_schedule(step: int, total_steps: int, base_lr: float, warmup_frac: float, warmdown_frac: float) -> float:
+    return float(load().dion_lr_schedule(int(step), int(total_steps), float(base_lr), float(warmup_frac),
+                                         float(warmdown_frac)))
+
+
+def dion_rank_for(m: int, n: int, fraction: float) -> int:
+    return int(load().dion_rank_for(int(m), int(n), float(fraction)))
 
 
 def dion_plan_enable_host_gradients(plan: int) -> None:

@@ -77,10 +77,10 @@ def snapshot(st: DevState, plan=None):
 
 
 def oracle_hp(mu=0.95, eta=0.01, eta_local=None, eps_rmmc=1e-8, eps_col=1e-8, tau_global=0.5, gate_mode=0,
-              period=1) -> oc.HParams:
+              period=1, weight_decay=0.0) -> oc.HParams:
     return oc.HParams(mu=f32(mu), eta=f32(eta), eta_local=f32(eta if eta_local is None else eta_local),
                       eps_rmmc=f32(eps_rmmc), eps_col=f32(eps_col), gate_mode=gate_mode, tau_global=f32(tau_global),
-                      period=period)
+                      period=period, weight_decay=f32(weight_decay))
 
 
 @dataclass

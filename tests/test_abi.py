@@ -45,7 +45,7 @@ def test_exported_symbols_via_nm(lib):
 def test_abi_version_and_status_strings(lib):
     from paper_2512_13728_gb300 import native
 
-    assert native.dion_abi_version() == 1
+    assert native.dion_abi_version() == native.DION_ABI_VERSION == 2
     for code in range(8):
         assert native.dion_status_string(code).startswith("DION_")
     assert "unknown" in native.dion_status_string(99)
@@ -99,3 +99,52 @@ def test_step_rejects_null_plan(lib):
     assert lib.dion_plan_enable_host_gradients(None) == 1
     assert lib.dion_step_host(None, C.byref(hp), None, None, None, None, None, None, None, None) == 1
     lib.dion_plan_destroy(None)  # no-op
+
+
+def test_hparams_struct_layout():
+    from paper_2512_13728_gb300 import native
+
+    assert C.sizeof(native.dion_hparams) == 48
+    assert native.dion_hparams.weight_decay.offset == 40
+
+
+@pytest.mark.parametrize("T,wu,wd", [(3000, 0.01, 0.2), (3000, 0.01, 0.1), (100, 0.0, 0.5), (50, 0.01, 0.0),
+                                     (8, 0.5, 0.5), (1, 0.0, 1.0), (50, 0.1, 0.1)])
+def test_lr_schedule_matches_oracle(lib, T, wu, wd):
+    """The library's host-side schedule (fp32 result) against the oracle's definition."""
+    import numpy as np
+
+    import oracle.curvadion as oc
+    from paper_2512_13728_gb300 import native
+
+    for t in list(range(-1, min(T, 60) + 2)) + list(range(max(1, T - 60), T + 3)):
+        want = np.float32(oc.lr_schedule(t, T, float(np.float32(0.02)), float(np.float32(wu)), float(np.float32(wd))))
+        assert native.dion_lr_schedule(t, T, 0.02, wu, wd) == pytest.approx(float(want), rel=2e-7, abs=0.0), t
+
+
+def test_lr_schedule_rejects_bad_arguments(lib):
+    import math
+
+    from paper_2512_13728_gb300 import native
+
+    assert math.isnan(native.dion_lr_schedule(1, 0, 0.02, 0.01, 0.1))
+    assert math.isnan(native.dion_lr_schedule(1, 100, 0.02, -0.1, 0.1))
+    assert math.isnan(native.dion_lr_schedule(1, 100, 0.02, 0.6, 0.6))
+    assert math.isnan(native.dion_lr_schedule(1, 100, 0.02, 0.01, float("nan")))
+
+
+@pytest.mark.parametrize("m,n,f", [(768, 3072, 0.125), (2048, 8192, 0.125), (100, 100, 0.125), (1, 5, 0.125),
+                                   (64, 64, 1.0), (4096, 1024, 1 / 16), (768, 768, 0.25), (3, 1000, 0.3)])
+def test_rank_for_matches_oracle(lib, m, n, f):
+    import oracle.curvadion as oc
+    from paper_2512_13728_gb300 import native
+
+    assert native.dion_rank_for(m, n, f) == oc.rank_for(m, n, f)
+
+
+def test_rank_for_rejects_bad_arguments(lib):
+    from paper_2512_13728_gb300 import native
+
+    assert native.dion_rank_for(0, 5, 0.1) == 0
+    assert native.dion_rank_for(5, 5, 0.0) == 0
+    assert native.dion_rank_for(5, 5, 1.5) == 0

@@ -201,6 +201,22 @@ def test_gate_modes_bf16():
                      taus=[0.5, 0.3, 0.9])
 
 
+@pytest.mark.parametrize("prec", ["bf16", "fp32"])
+def test_weight_decay_both_branches(prec):
+    """Decoupled weight decay (Section 4's 0.01, here 0.5 so that it is visible against the
+    tolerance) in the Dion branch and the local branch: a per-layer gate with one layer that
+    syncs only at step 1 (tau 1e6), one that always syncs (tau 1e-6) and one in between,
+    against the oracle step by step."""
+    import paper_2512_13728_gb300 as cd
+
+    p = cd.DION_PREC_BF16 if prec == "bf16" else cd.DION_PREC_FP32
+    w = wl.scaled(wl.WORKLOADS["gpt350m_gate_stress_r256"], "wd", [(128, 192), (192, 128), (64, 64)],
+                  rank=16, steps=6, kind="gaussian")
+    run_per_step(w, p, dict(gate_mode=oc.GATE_PER_LAYER, tau_global=0.5, eta=0.05, eta_local=0.03,
+                            weight_decay=0.5), w.steps, TOL_BF16 if prec == "bf16" else TOL_FP32,
+                 taus=[1e6, 1e-6, 0.5])
+
+
 # ------------------------------------------------------------------ gate sequences ---
 
 def test_gate_stress_flag_sequences_fp32():

@@ -290,8 +290,8 @@ def _pins_fail(monkeypatch, name, fake, pins):
 def test_mutation_wrong_decay_is_caught(monkeypatch):
     real = oc.dion_sync_update
 
-    def mutated(B, Qp, X, mu, eta, eps_col):  # (1 - mu) replaced by mu
-        return real(B, Qp, X, 1.0 - mu, eta, eps_col)
+    def mutated(B, Qp, X, mu, eta, eps_col, weight_decay=0.0):  # (1 - mu) replaced by mu
+        return real(B, Qp, X, 1.0 - mu, eta, eps_col, weight_decay)
 
     assert _pins_fail(monkeypatch, "dion_sync_update", mutated,
                       [lambda: test_full_rank_recovers_buffer(12, 8)]) == 1
@@ -307,7 +307,7 @@ def test_mutation_missing_sign_fix_is_caught(monkeypatch):
 
 
 def test_mutation_transposed_scale_is_caught(monkeypatch):
-    def mutated(B, Qp, X, mu, eta, eps_col):  # sqrt(n/m) instead of sqrt(m/n)
+    def mutated(B, Qp, X, mu, eta, eps_col, weight_decay=0.0):  # sqrt(n/m) instead of sqrt(m/n)
         m, n = B.shape
         P = oc.orthogonalize(B @ Qp)
         R = B.T @ P
@@ -319,7 +319,7 @@ def test_mutation_transposed_scale_is_caught(monkeypatch):
 
 
 def test_mutation_stale_q_in_update_is_caught(monkeypatch):
-    def mutated(B, Qp, X, mu, eta, eps_col):  # parameter update with Q_{t-1} instead of Q_t
+    def mutated(B, Qp, X, mu, eta, eps_col, weight_decay=0.0):  # parameter update with Q_{t-1} instead of Q_t
         m, n = B.shape
         P = oc.orthogonalize(B @ Qp)
         R = B.T @ P
@@ -345,3 +345,87 @@ def test_mutation_rmmc_without_abs_is_caught(monkeypatch):
 
     pin_decreasing()
     assert _pins_fail(monkeypatch, "rmmc_alg2", mutated, [pin_decreasing]) == 1
+
+
+# ------------------------------------------- training-loop fidelity (Section 4 settings) ---
+
+@pytest.mark.parametrize("m,n,r", [(6, 9, 3), (12, 5, 5)])
+def test_weight_decay_is_decoupled(m, n, r):
+    """Decoupled decay changes only X, and by exactly -lr * wd * X in both branches; M, Q, P, R
+    are those of the undecayed step (the decay never enters the momentum)."""
+    B = RNG.standard_normal((m, n))
+    Qp = RNG.standard_normal((n, r))
+    X = RNG.standard_normal((m, n))
+    G = RNG.standard_normal((m, n))
+    a = oc.dion_sync_update(B, Qp, X, 0.9, 0.05, 1e-8, 0.0)
+    b = oc.dion_sync_update(B, Qp, X, 0.9, 0.05, 1e-8, 0.3)
+    assert np.array_equal(a.M, b.M) and np.array_equal(a.Q, b.Q) and np.array_equal(a.P, b.P)
+    assert np.allclose(b.X - a.X, -0.05 * 0.3 * X, rtol=0, atol=1e-14)
+    M0, X0 = oc.local_update(B, G, X, 0.07, 0.0)
+    M1, X1 = oc.local_update(B, G, X, 0.07, 0.3)
+    assert np.array_equal(M0, M1)
+    assert np.allclose(X1 - X0, -0.07 * 0.3 * X, rtol=0, atol=1e-14)
+
+
+def test_weight_decay_local_steps_closed_form():
+    """With zero gradients every local step only decays: X_t = (1 - eta_local wd)^t X_0 (scalar
+    loop check), and M stays 0."""
+    m, n = 3, 4
+    X0 = RNG.standard_normal((m, n))
+    layer = oc.LayerState(X=X0.copy(), M=np.zeros((m, n)), Q=np.eye(n)[:, :2], tau=math.inf)
+    hp = oc.HParams(eta_local=0.1, weight_decay=0.5, gate_mode=oc.GATE_PER_LAYER)
+    cur, prev = [layer], [0.0]
+    for t in range(1, 6):
+        o = oc.curvadion_step(cur, [np.zeros((m, n))], prev, hp, t)
+        cur, prev = o.layers, o.prev_norm
+    for i in range(m):
+        for j in range(n):
+            v = X0[i, j]
+            for _ in range(5):
+                v = v * (1.0 - 0.1 * 0.5)
+            assert cur[0].X[i, j] == pytest.approx(v, rel=1e-14, abs=1e-300)
+    assert not np.any(cur[0].M)
+
+
+@pytest.mark.parametrize("T,wu,wd", [(3000, 0.01, 0.2), (3000, 0.01, 0.1), (100, 0.0, 0.5), (50, 0.1, 0.0)])
+def test_lr_schedule_shape(T, wu, wd):
+    """Section 4's schedule: linear rise to the base rate over round(wu T) steps, flat, linear fall
+    to exactly 0 at the last step over round(wd T) steps; every piece is affine in the step."""
+    base = 0.02
+    lr = np.array([oc.lr_schedule(t, T, base, wu, wd) for t in range(1, T + 1)])
+    W, D = int(math.floor(wu * T + 0.5)), int(math.floor(wd * T + 0.5))
+    assert np.all(lr >= 0) and np.all(lr <= base)
+    if D > 0:
+        assert lr[-1] == 0.0
+        assert lr[T - D - 1] == base  # last flat step
+        fall = lr[T - D - 1:]
+        assert np.allclose(np.diff(fall, 2), 0.0, atol=1e-15) and np.all(np.diff(fall) < 0)
+    else:
+        assert lr[-1] == base
+    if W > 0:
+        rise = np.concatenate([[0.0], lr[:W]])
+        assert lr[W - 1] == base and np.allclose(np.diff(rise, 2), 0.0, atol=1e-15)
+        assert lr[0] == pytest.approx(base / W)
+    flat = lr[W:T - D]
+    assert np.all(flat == base)
+    # outside [1, T] the schedule clamps
+    assert oc.lr_schedule(0, T, base, wu, wd) == lr[0] and oc.lr_schedule(T + 5, T, base, wu, wd) == lr[-1]
+
+
+@pytest.mark.parametrize("m,n,f,r", [(768, 3072, 0.125, 96), (2048, 8192, 0.125, 256), (100, 100, 0.125, 13),
+                                     (1, 5, 0.125, 1), (64, 64, 1.0, 64), (4096, 1024, 1 / 16, 64),
+                                     (768, 768, 0.25, 192)])
+def test_rank_for(m, n, f, r):
+    assert oc.rank_for(m, n, f) == r
+
+
+def test_mutation_decay_after_update_is_caught(monkeypatch):
+    real = oc.dion_sync_update
+
+    def mutated(B, Qp, X, mu, eta, eps_col, weight_decay=0.0):  # decays the updated X instead of X
+        res = real(B, Qp, X, mu, eta, eps_col, 0.0)
+        res.X = (1.0 - eta * weight_decay) * res.X
+        return res
+
+    assert _pins_fail(monkeypatch, "dion_sync_update", mutated,
+                      [lambda: test_weight_decay_is_decoupled(6, 9, 3)]) == 1
