@@ -345,3 +345,53 @@ def run_trajectory(layers: Sequence[LayerState], grad_fn, steps: int, hp: HParam
         outs.append(o)
         cur, pn = o.layers, o.prev_norm
     return cur, outs
+
+
+# ---------------------------------------------------------------------------------------
+# Theorem 1 (RMMC and directional curvature) on a quadratic objective
+# ---------------------------------------------------------------------------------------
+# For a 1 x n parameter the Dion branch is heavy-ball momentum with a normalized step: r = 1,
+# P = sign(B Q_{t-1}) (1 x 1), R = B^T P, Q_t = R / (||R|| + eps_col), so
+#   X_t = X_{t-1} - eta sqrt(1/n) B / (||B|| + eps_col)   and   M_t = mu B,
+# i.e. B_t = mu B_{t-1} + G_t is the theorem's momentum M_t and the step is x_t = x_{t-1} -
+# eta_eff M_{t-1} with eta_eff = eta / (sqrt(n) (||B_{t-1}|| + eps_col)).  On F(x) = x^T H x / 2
+# the gradient expansion of the proof is exact, so with v = B_{t-1} / ||B_{t-1}||,
+# kappa = v^T H v, B_t = (1 - mu) - v^T grad F(x_{t-1}) / ||B_{t-1}||, and rho = the part of
+# grad F(x_t) perpendicular to v divided by ||B_{t-1}||:
+#   ||B_t|| / ||B_{t-1}|| = sqrt((1 - B_t - eta_eff kappa)^2 + rho^2),
+# which is Theorem 1's |eta kappa + B_t| when rho = 0 (exactly so for n = 1); otherwise the
+# two differ by at most rho^2 / (2 (1 - B_t - eta_eff kappa)) (sqrt(a^2 + c) - a <= c / (2a)).
+
+def rank1_step_size(eta: float, n: int, b_prev: np.ndarray, eps_col: float) -> float:
+    """eta_eff of a 1 x n layer's Dion step: eta / (sqrt(n) (||B_{t-1}|| + eps_col))."""
+    return eta / (math.sqrt(n) * (frobenius_norm(b_prev) + eps_col))
+
+
+@dataclass
+class Theorem1Terms:
+    kappa: float        # v^T H v, v = B_{t-1} / ||B_{t-1}||
+    bias: float         # B_t = (1 - mu) - v^T grad F(x_{t-1}) / ||B_{t-1}||
+    eta_eff: float
+    prediction: float   # |eta_eff kappa + B_t|
+    rho: float          # |grad F(x_t) perpendicular to v| / ||B_{t-1}||
+    exact: float        # |sqrt((1 - B_t - eta_eff kappa)^2 + rho^2) - 1|
+
+
+def theorem1_terms(H: np.ndarray, x_prev: np.ndarray, b_prev: np.ndarray, mu: float, eta_eff: float) -> Theorem1Terms:
+    """Theorem 1's quantities for the step from x_{t-1} (1 x n) with momentum B_{t-1} on
+    F(x) = x^T H x / 2 (H symmetric), and the exact ratio of the momentum norms."""
+    H = as_f64(H)
+    x_prev = as_f64(x_prev).reshape(-1)
+    b_prev = as_f64(b_prev).reshape(-1)
+    m_prev = float(np.linalg.norm(b_prev))
+    v = b_prev / m_prev
+    g_prev = H @ x_prev
+    kappa = float(v @ H @ v)
+    bias = (1.0 - mu) - float(v @ g_prev) / m_prev
+    x_now = x_prev - eta_eff * b_prev
+    g_now = H @ x_now
+    g_perp = g_now - float(v @ g_now) * v
+    rho = float(np.linalg.norm(g_perp)) / m_prev
+    a = 1.0 - bias - eta_eff * kappa
+    return Theorem1Terms(kappa=kappa, bias=bias, eta_eff=eta_eff, prediction=abs(eta_eff * kappa + bias),
+                         rho=rho, exact=abs(math.sqrt(a * a + rho * rho) - 1.0))

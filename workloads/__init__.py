@@ -162,3 +162,34 @@ def scaled(w: Workload, name: str, shapes, rank: int | None = None, steps: int |
         fields["steps"] = steps
     fields.update(kw)
     return Workload(**fields)
+
+
+# ----------------------------------------------------------- quadratic objective (Theorem 1) ---
+# Vector parameters (1 x n layers, rank 1) on F(x) = x^T H x / 2 with a symmetric positive
+# definite H per layer whose eigenvalues are log-spaced in [lam_min, lam_max] and whose
+# eigenvectors are a seeded random rotation.  The gradient H x is the test's input: it is
+# computed from the parameters each step (a closed loop), with the same formula on both sides.
+
+QUADRATIC_SHAPES = ((1, 1), (1, 64), (1, 512), (1, 2048))
+
+
+def quadratic_hessian(n: int, seed: int, lam_min: float = 0.1, lam_max: float = 10.0, device="cpu") -> torch.Tensor:
+    g = torch.Generator(device="cpu")
+    g.manual_seed(seed)
+    a = torch.randn((n, n), generator=g, dtype=torch.float64)
+    u, _ = torch.linalg.qr(a)
+    lam = torch.logspace(math.log10(lam_min), math.log10(lam_max), n, dtype=torch.float64)
+    h = (u * lam[None, :]) @ u.T
+    h = 0.5 * (h + h.T)
+    return h.to(torch.float32).to(device)
+
+
+def quadratic_start(n: int, seed: int, device="cpu") -> torch.Tensor:
+    g = torch.Generator(device="cpu")
+    g.manual_seed(seed)
+    return torch.randn((1, n), generator=g, dtype=torch.float32).to(device)
+
+
+def quadratic_gradient(H: torch.Tensor, X: torch.Tensor) -> torch.Tensor:
+    """grad F = H x for a 1 x n row x (H symmetric): x H."""
+    return X @ H
