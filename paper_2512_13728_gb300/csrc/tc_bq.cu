@@ -318,8 +318,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(R_THREADS, 1)
 // Algorithm 1/2 with bf16 gradients: B = M_{t-1} + G is formed on the fly from TMA tiles of M
 // (fp32) and G (bf16) and fed to the pair MMA of P = B Q_{t-1}, so B is read from HBM once.
 // Per {layer, pair p} (CTA c owns 128-row tile 2 p + c) and 64-column k-chunk:
-//   warp 0      TMA: M as two 128 x 32 fp32 SW128 boxes into the M ring, G as one 128 x 64 bf16
-//               SW128 box into the A ring;
+//   warps 12..15 M through the load/store path: 16-byte cp.async copies written in the same
+//               swizzled layout as two 128 x 32 fp32 SW128 boxes, into the M ring (zero-filled
+//               past the matrix); their landing completes the slot's barrier.  (Each SM's TMA
+//               unit already carries G, Q, Bh and P: M, the largest stream, goes around it);
+//   warp 0      TMA: G as one 128 x 64 bf16 SW128 box into the A ring;
 //   warps 6..9  B = M + G in fp32, rounded to bf16 and written in place over the G box, which
 //               has the layout of the K-major A operand; the per-tile sums of B^2 and M_{t-1}^2
 //               (Algorithm 2's ||B|| and Equation 1's ||M_{t-1}||).  The M stage is free again
@@ -337,7 +340,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(R_THREADS, 1)
 constexpr int FB_MSTAGES = 3;  // M ring (2 x 16 KB per slot)
 constexpr int FB_ASTAGES = 4;  // G / A ring (16 KB per slot)
 constexpr int FB_QSTAGES = 2;  // Q ring (also the epilogue's staging)
-constexpr int FB_THREADS = 12 * 32;
+constexpr int FB_THREADS = 16 * 32;
+constexpr int FB_LOADERS = 128;  // threads of warps 12..15
 constexpr uint32_t FB_MBOX = 128u * 32u * 4u;  // 128 x 32 fp32 box of M (16 KB)
 constexpr uint32_t FB_GBOX = 128u * 64u * 2u;  // 128 x 64 bf16 box of G, then of B (16 KB)
 constexpr uint32_t FB_MSLOT = 2u * FB_MBOX;
@@ -368,7 +372,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
   const int seg = blockIdx.x >> 1;
   if (threadIdx.x == 0) {
     for (int i = 0; i < FB_MSTAGES; ++i) {
-      mbar_init(&mfull[i], 1);   // this CTA's M boxes
+      mbar_init(&mfull[i], FB_LOADERS);  // every loader thread's copies of this CTA's M chunk
       mbar_init(&mempty[i], 1);  // converted
     }
     for (int i = 0; i < FB_ASTAGES; ++i) {
@@ -399,7 +403,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
   const uint32_t tmem = tmem_base_s;
   auto half_cols = [](uint32_t np, uint32_t part) { return min(256u, np - part * 256u) / 2u; };
 
-  if (warp == 0) {  // M and G loads
+  if (warp == 0) {  // G loads
     if (lane == 0) {
       uint32_t it = 0;
       bool ok = true;
@@ -410,23 +414,45 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
         const int kch = (int)((L.n + 63) / 64);
         const int tr = 2 * t.y + (int)rank;  // past the last tile: zero-filled, not stored
         for (int kc = 0; kc < kch; ++kc, ++it) {
-          const uint32_t sm = it % FB_MSTAGES, pm = (it / FB_MSTAGES) & 1u;
           const uint32_t sg = it % FB_ASTAGES, pg = (it / FB_ASTAGES) & 1u;
-          if (!ab.wait(&mempty[sm], pm ^ 1u, sh.status)) { ok = false; break; }
-          uint8_t *sM = smem + sm * FB_MSLOT;
-          mbar_expect_tx(&mfull[sm], FB_MSLOT);
-          tma_load_2d(sM, &mp->Mf, &mfull[sm], kc * 64, tr * 128);
-          tma_load_2d(sM + FB_MBOX, &mp->Mf, &mfull[sm], kc * 64 + 32, tr * 128);
           if (!ab.wait(&gempty[sg], pg ^ 1u, sh.status)) { ok = false; break; }
           mbar_expect_tx(&gfull[sg], FB_GBOX);
           tma_load_2d(aring + sg * FB_GBOX, &mp->Gh64, &gfull[sg], kc * 64, tr * 128);
         }
       }
-      for (uint32_t k = (it > (uint32_t)FB_MSTAGES ? it - FB_MSTAGES : 0); k < it; ++k)
-        mbar_wait(&mempty[k % FB_MSTAGES], (k / FB_MSTAGES) & 1u, sh.status);
       for (uint32_t k = (it > (uint32_t)FB_ASTAGES ? it - FB_ASTAGES : 0); k < it; ++k)
         mbar_wait(&gempty[k % FB_ASTAGES], (k / FB_ASTAGES) & 1u, sh.status);
     }
+  } else if (warp >= 12) {  // M loads (cp.async)
+    const int lt = threadIdx.x - 12 * 32;  // 0..127
+    uint32_t it = 0;
+    for (int ti = off[seg]; ti < off[seg + 1]; ++ti) {
+      const int4 t = tiles[ti];
+      const DevLayer &L = sh.layers[t.x];
+      const int kch = (int)((L.n + 63) / 64);
+      const int64_t row0 = (int64_t)(2 * t.y + (int)rank) * 128;
+      bool ok = true;
+      for (int kc = 0; kc < kch; ++kc, ++it) {
+        const uint32_t sm = it % FB_MSTAGES, pm = (it / FB_MSTAGES) & 1u;
+        if (!named_and(3, FB_LOADERS, ab.wait(&mempty[sm], pm ^ 1u, sh.status))) { ok = false; break; }
+        uint8_t *sM = smem + sm * FB_MSLOT;
+#pragma unroll 4
+        for (int i = 0; i < 16; ++i) {
+          // copy e: row e >> 4, 16-byte chunk e & 15 of the row's 64 columns (a warp covers two
+          // whole 256-byte row segments); box = chunk >> 3, swizzled chunk within the box
+          const uint32_t e = (uint32_t)(i * FB_LOADERS + lt), row = e >> 4, c16 = e & 15u;
+          const uint32_t box = c16 >> 3, ch = c16 & 7u;
+          uint8_t *dst = sM + box * FB_MBOX + row * 128u + ((ch ^ (row & 7u)) << 4);
+          const int64_t gr = row0 + row, gc = (int64_t)kc * 64 + 4 * c16;
+          const bool in = gr < L.m && gc < L.n;
+          const uint32_t bytes = in ? (uint32_t)((L.n - gc < 4 ? L.n - gc : 4) * 4) : 0u;
+          cp_async16(dst, in ? (const void *)(L.M + gr * L.ldm + gc) : (const void *)L.M, bytes);
+        }
+        cp_async_arrive(&mfull[sm]);
+      }
+      if (!ok) break;
+    }
+    cp_async_wait_all();
   } else if (warp == 10) {  // Q loads
     if (lane == 0) {
       uint32_t it = 0, tcount = 0;

@@ -59,7 +59,9 @@ __device__ __forceinline__ OrthMaps orth_maps(const LayerMaps &mp, int pass) {
 template <int KIND>
 __device__ __forceinline__ void orth_dims(const DevLayer &L, int blk, uint32_t &N, int64_t &K) {
   if (KIND == ORTH_GRAM) {
-    N = pad16(L.r);
+    // rows 256 blk .. 256 blk + 255 of S: only columns below 256 (blk + 1) are read (the
+    // Cholesky and the orthogonality bound use the lower triangle of S)
+    N = min(pad16(L.r), 256u * (uint32_t)(blk + 1));
     K = L.m;
   } else {
     N = pad16(L.r);
