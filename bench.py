@@ -267,13 +267,18 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
-    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    f0.record(stream)
-    for _ in range(e_steps):
-        e2e_step()
-    f1.record(stream)
-    torch.cuda.synchronize()
-    e2e_ms = f0.elapsed_time(f1) / e_steps
+    # three repetitions of e_steps steps, the median reported: the host side of the copies is
+    # shared with whatever else the machine runs
+    reps = []
+    for _ in range(3):
+        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        f0.record(stream)
+        for _ in range(e_steps):
+            e2e_step()
+        f1.record(stream)
+        torch.cuda.synchronize()
+        reps.append(f0.elapsed_time(f1) / e_steps)
+    e2e_ms = sorted(reps)[1]
     e2e_ms = max_over_ranks(e2e_ms, world, dev)
     launches = plan.launches_per_step()
     plan.close()
