@@ -246,30 +246,35 @@ def test_empty_plan_step():
 
 # ------------------------------------------------------------- device-side errors ---
 
-def test_breakdown_on_zero_buffer_sets_status_and_no_nan():
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_breakdown_on_zero_buffer_sets_status_and_no_nan(prec):
+    """B = 0 (rank-deficient P): DION_ERR_BREAKDOWN, L^{-1} = 0, so X is unchanged and nothing
+    non-finite is written, in both the CUDA-core and the tensor-core path (fused buffer + B Q)."""
     import paper_2512_13728_gb300 as cd
 
-    w = wl.scaled(RAGGED, "zero", [(64, 48)], rank=4, steps=1)
+    w = wl.scaled(RAGGED, "zero", [(64, 48), (256, 136)], rank=4, steps=1)
     st = gu.make_state(w)
-    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_FP32)
-    x0 = st.X[0].clone()
+    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_FP32 if prec == "fp32" else cd.DION_PREC_BF16)
+    x0 = [x.clone() for x in st.X]
     plan.step(cd.hparams(step=1))  # G = 0 and M = 0: B = 0, P = 0, Gram = 0
     torch.cuda.synchronize()
     assert plan.device_status() == cd.native.DION_ERR_BREAKDOWN
-    assert torch.isfinite(st.X[0]).all() and torch.isfinite(st.M[0]).all() and torch.isfinite(st.Q[0]).all()
-    assert torch.equal(st.X[0], x0)
+    for l in range(w.num_layers):
+        assert torch.isfinite(st.X[l]).all() and torch.isfinite(st.M[l]).all() and torch.isfinite(st.Q[l]).all()
+        assert torch.equal(st.X[l], x0[l])
     assert plan.device_status() == 0  # cleared by the previous read
     plan.close()
 
 
-def test_nonfinite_gradient_sets_status_and_flags():
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_nonfinite_gradient_sets_status_and_flags(prec):
     import paper_2512_13728_gb300 as cd
 
     w = wl.scaled(RAGGED, "nan", [(64, 48), (32, 32)], rank=4, steps=1)
     st = gu.make_state(w, taus=[1e9, 1e9])
     gu.write_gradients(st, 1)
     st.G[0][3, 5] = float("nan")
-    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_FP32)
+    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_FP32 if prec == "fp32" else cd.DION_PREC_BF16)
     plan.step(cd.hparams(step=1, gate_mode=cd.DION_GATE_PER_LAYER, tau_global=1e9))
     torch.cuda.synchronize()
     assert plan.device_status() == cd.native.DION_ERR_NONFINITE
