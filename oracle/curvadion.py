@@ -395,3 +395,60 @@ def theorem1_terms(H: np.ndarray, x_prev: np.ndarray, b_prev: np.ndarray, mu: fl
     a = 1.0 - bias - eta_eff * kappa
     return Theorem1Terms(kappa=kappa, bias=bias, eta_eff=eta_eff, prediction=abs(eta_eff * kappa + bias),
                          rho=rho, exact=abs(math.sqrt(a * a + rho * rho) - 1.0))
+
+
+# ---------------------------------------------------------------------------------------
+# Data-parallel semantics of Algorithm 2 (W workers emulated on one host)
+# ---------------------------------------------------------------------------------------
+# Worker w holds its own X^w, M^w, Q^w and prev_norm^w and computes its own gradient.  Each
+# step: B^w = M^w + G^w and RMMC^w_l per layer (local); AllReduce_max of RMMC over workers (and
+# over layers for the global flag); on a sync, P = AllReduce_DP(B^w Q^w), Orthogonalize(P),
+# R = AllReduce_DP(B^w^T P), then each worker applies the same P, R, Q_t to its own M^w, X^w;
+# otherwise each worker takes its local step.  AllReduce_DP is read as the mean over workers
+# (the data-parallel average of Dion's reference implementation); with one worker it is the
+# identity and this is curvadion_step.
+
+@dataclass
+class DPStepOutput:
+    workers: List[List[LayerState]]
+    prev_norm: List[np.ndarray]
+    rmmc: List[np.ndarray]          # per worker, per layer (local)
+    rmmc_max: np.ndarray            # per layer, max over workers (the AllReduce_max)
+    flags: np.ndarray
+    global_flag: bool
+    active: np.ndarray
+
+
+def curvadion_step_dp(workers: Sequence[Sequence[LayerState]], grads: Sequence[Sequence[np.ndarray]],
+                      prev_norm: Sequence[Sequence[float]], hp: HParams, step: int) -> DPStepOutput:
+    """One step of Algorithm 2 over W data-parallel workers (lists indexed [worker][layer])."""
+    W = len(workers)
+    L = len(workers[0]) if W else 0
+    Bs = [[form_buffer(as_f64(workers[w][l].M), as_f64(grads[w][l])) for l in range(L)] for w in range(W)]
+    nb = [np.array([frobenius_norm(Bs[w][l]) for l in range(L)]) for w in range(W)]
+    rm = [np.array([rmmc_alg2(nb[w][l], float(prev_norm[w][l]), hp.eps_rmmc) for l in range(L)])
+          for w in range(W)]
+    rmax = np.array([max((rm[w][l] if math.isfinite(rm[w][l]) else math.inf) for w in range(W))
+                     for l in range(L)])
+    flags, gflag, active = gate(rmax, [workers[0][l].tau for l in range(L)], hp.tau_global, hp.gate_mode,
+                                step, hp.period)
+    out = [[None] * L for _ in range(W)]
+    for l in range(L):
+        if active[l]:
+            P = sum(power_iter(Bs[w][l], as_f64(workers[w][l].Q)) for w in range(W)) / W
+            P = orthogonalize(P)
+            R = sum(Bs[w][l].T @ P for w in range(W)) / W
+            Q_new = column_normalize(R, hp.eps_col)
+            for w in range(W):
+                st = workers[w][l]
+                m, n = Bs[w][l].shape
+                M_new = Bs[w][l] - (1.0 - hp.mu) * (P @ R.T)
+                X_new = decay_parameters(as_f64(st.X), hp.eta, hp.weight_decay) - hp.eta * math.sqrt(m / n) * (P @ Q_new.T)
+                out[w][l] = LayerState(X=X_new, M=M_new, Q=Q_new.copy(), tau=st.tau)
+        else:
+            for w in range(W):
+                st = workers[w][l]
+                M_new, X_new = local_update(Bs[w][l], as_f64(grads[w][l]), as_f64(st.X), hp.eta_local, hp.weight_decay)
+                out[w][l] = LayerState(X=X_new, M=M_new, Q=as_f64(st.Q), tau=st.tau)
+    return DPStepOutput(workers=out, prev_norm=[x.copy() for x in nb], rmmc=rm, rmmc_max=rmax,
+                        flags=np.array(flags, dtype=bool), global_flag=bool(gflag), active=np.array(active, dtype=bool))
