@@ -43,7 +43,7 @@ extern "C" {
 typedef enum {
   DION_OK = 0,
   DION_ERR_INVALID_ARG = 1,  /* NULL pointer, bad size, r > min(m, n), unknown enum */
-  DION_ERR_UNSUPPORTED = 2,  /* valid request outside this build's limits (e.g. r > 512) */
+  DION_ERR_UNSUPPORTED = 2,  /* valid request outside the library's limits (e.g. r > 512) */
   DION_ERR_ALIGNMENT = 3,    /* pointer or leading dimension breaks the 16-byte rule */
   DION_ERR_CUDA = 4,         /* a CUDA runtime call failed (no device, launch error, OOM) */
   DION_ERR_BREAKDOWN = 5,    /* device: Cholesky pivot <= 0 or non-finite (rank-deficient P) */

@@ -128,7 +128,7 @@ const char *dion_status_string(dion_status s) {
   switch (s) {
     case DION_OK: return "DION_OK";
     case DION_ERR_INVALID_ARG: return "DION_ERR_INVALID_ARG: invalid argument";
-    case DION_ERR_UNSUPPORTED: return "DION_ERR_UNSUPPORTED: outside this build's limits";
+    case DION_ERR_UNSUPPORTED: return "DION_ERR_UNSUPPORTED: outside the library's limits";
     case DION_ERR_ALIGNMENT: return "DION_ERR_ALIGNMENT: pointer or leading dimension not 16-byte aligned";
     case DION_ERR_CUDA: return "DION_ERR_CUDA: CUDA runtime error";
     case DION_ERR_BREAKDOWN: return "DION_ERR_BREAKDOWN: Cholesky breakdown (rank-deficient P)";
