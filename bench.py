@@ -85,6 +85,8 @@ def kernel_work(name: str, w, prec: str):
         "tc_bq": ("hbm", mn * 2 + nr * 2 + mr * 8, "B"),  # Bh, bf16 Q; P and P^T fp32
         # buffer pass fused into B Q (bf16 G): read M, G; write Bh, P and P^T fp32
         "tc_form_bq": ("hbm", mn * (4 + gsz + 2) + mr * 8, "B"),
+        # gated modes: the norms pass read M, G (and the gate in its last block)
+        "norms_gate": ("hbm", mn * (4 + gsz), "B"),
         "tc_btp": ("hbm", mn * 2 + mr * 2 + nr * 6, "B"),  # Bh, bf16 P; R fp32 and bf16
         "tc_update": ("hbm", mn * (16 + (gsz if deferred else 0)), "B"),
         "tc_gram": ("tensor", 2 * mr2, "flop"),

@@ -79,6 +79,7 @@ struct StepArgs {
 };
 
 // Workspace shared by all kernels of a plan.
+constexpr int kScratchActive = 3;  // gate_scratch slot holding the count of Dion-branch layers
 struct Shared {
   DevLayer *layers;
   int32_t num_layers;
@@ -89,7 +90,10 @@ struct Shared {
   double *norm_b;        // [L]
   int32_t *status;       // [1] first device error
   uint8_t *orth_shifted; // [L] 1 = a Cholesky pass of this step needed the shift (third pass runs)
-  unsigned long long *gate_scratch;  // [2] the gate's running max of RMMC (ordered key), finished-block count
+  // [4]: the gate's running max of RMMC (ordered key), its finished-block count, the norms
+  // pass's finished-block count, and (written by the gate) the number of layers that take the
+  // Dion branch this step, which lets the later persistent kernels return at once when it is 0
+  unsigned long long *gate_scratch;
 };
 
 // A contraction C = op(A) op(B) for the CUDA-core path.
@@ -141,6 +145,7 @@ void launch_colnorm(const Shared &sh, const int4 *tiles, int32_t ntiles, float e
                     cudaStream_t s);
 void launch_update(const Shared &sh, const int4 *tiles, int32_t ntiles, float mu, float eta, float keep,
                    cudaStream_t s);
+void launch_norms_gate(const Shared &sh, const StepArgs &a, const int4 *tiles, int32_t ntiles, cudaStream_t s);
 void launch_local(const Shared &sh, const int4 *tiles, int32_t ntiles, float eta_local, float keep,
                   cudaStream_t s);
 void launch_finalize(const Shared &sh, const StepArgs &a, cudaStream_t s);

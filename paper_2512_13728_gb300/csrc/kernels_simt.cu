@@ -116,40 +116,71 @@ __device__ __forceinline__ double from_max_key(unsigned long long k) {
   return __longlong_as_double((long long)(k & ~(1ull << 63)));
 }
 
-// One warp per layer: ||B|| and ||M_{t-1}|| from the buffer pass's tile partials (fixed-order
-// fp64 sums), Algorithm 2's RMMC, prev_norm <- ||B||, the per-layer flag; the running maximum
-// of RMMC goes to an atomic max (order-independent, so deterministic).  The last block to
-// finish sets the global flag and the branch mask of every layer and resets the scratch.
+// Algorithm 2 for layer l, by one warp: ||B|| and ||M_{t-1}|| from the buffer pass's tile
+// partials (fixed-order fp64 sums), RMMC, prev_norm <- ||B||, the per-layer flag.  Returns
+// RMMC (in lane 0; +inf when not finite, which counts as above every threshold).
+__device__ double gate_layer(const Shared &sh, const StepArgs &a, int l, int lane) {
+  const DevLayer &Ly = sh.layers[l];
+  double sb = 0.0, sm = 0.0;
+  for (int k = lane; k < Ly.bpart_cnt; k += 32) {  // fixed lane/slot assignment
+    sb += __ldcg(&sh.bpart[2 * (Ly.bpart_off + k)]);
+    sm += __ldcg(&sh.bpart[2 * (Ly.bpart_off + k) + 1]);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    sb += __shfl_xor_sync(0xffffffffu, sb, o);
+    sm += __shfl_xor_sync(0xffffffffu, sm, o);
+  }
+  double rm = 0.0;
+  if (lane == 0) {
+    const double nb = sqrt(sb);
+    const double prev = a.prev_norm[l];
+    rm = fabs(nb - prev) / (prev + (double)a.eps_rmmc);
+    if (!isfinite(nb)) set_status(sh.status, ST_NONFINITE);
+    a.rmmc[l] = rm;
+    a.prev_norm[l] = nb;
+    a.flags[l] = above(rm, Ly.tau) ? 1 : 0;
+    sh.norm_b[l] = nb;
+    sh.norm_m_before[l] = sqrt(sm);
+  }
+  return isfinite(rm) ? rm : INFINITY;
+}
+
+// The gate mode's branch mask from the flags (all blocks' flags are written) and the global
+// flag; one block, all threads.  Also counts the Dion-branch layers into the scratch.
+__device__ void gate_finish(const Shared &sh, const StepArgs &a, int gflag, int *count_s) {
+  const int L = sh.num_layers;
+  if (threadIdx.x == 0) *count_s = 0;
+  __syncthreads();
+  int mine = 0;
+  for (int i = threadIdx.x; i < L; i += blockDim.x) {
+    int act;
+    switch (a.gate_mode) {
+      case GATE_ALWAYS: act = 1; break;
+      case GATE_GLOBAL: act = gflag; break;
+      case GATE_PER_LAYER: act = *reinterpret_cast<const volatile uint8_t *>(&a.flags[i]); break;  // other blocks'
+      default: act = (a.step % a.period) == 0; break;
+    }
+    sh.active[i] = (uint8_t)act;
+    mine += act;
+  }
+  atomicAdd(count_s, mine);
+  __syncthreads();
+  if (threadIdx.x == 0) sh.gate_scratch[kScratchActive] = (unsigned long long)*count_s;
+}
+
+// One warp per layer; the running maximum of RMMC goes to an atomic max (order-independent, so
+// deterministic).  The last block to finish sets the global flag and the branch mask of every
+// layer and resets the scratch.
 constexpr int kGateWarps = 8;
 __global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(Shared sh, StepArgs a) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int L = sh.num_layers;
   const int l = blockIdx.x * kGateWarps + warp;
-  __shared__ int last_s, gflag_s;
+  __shared__ int last_s, gflag_s, count_s;
   if (l < L) {
-    const DevLayer &Ly = sh.layers[l];
-    double sb = 0.0, sm = 0.0;
-    for (int k = lane; k < Ly.bpart_cnt; k += 32) {  // fixed lane/slot assignment
-      sb += sh.bpart[2 * (Ly.bpart_off + k)];
-      sm += sh.bpart[2 * (Ly.bpart_off + k) + 1];
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      sb += __shfl_xor_sync(0xffffffffu, sb, o);
-      sm += __shfl_xor_sync(0xffffffffu, sm, o);
-    }
-    if (lane == 0) {
-      const double nb = sqrt(sb);
-      const double prev = a.prev_norm[l];
-      const double rm = fabs(nb - prev) / (prev + (double)a.eps_rmmc);
-      if (!isfinite(nb)) set_status(sh.status, ST_NONFINITE);
-      a.rmmc[l] = rm;
-      a.prev_norm[l] = nb;
-      a.flags[l] = above(rm, Ly.tau) ? 1 : 0;
-      sh.norm_b[l] = nb;
-      sh.norm_m_before[l] = sqrt(sm);
-      atomicMax(&sh.gate_scratch[0], max_key(isfinite(rm) ? rm : INFINITY));
-    }
+    const double rm = gate_layer(sh, a, l, lane);
+    if (lane == 0) atomicMax(&sh.gate_scratch[0], max_key(rm));
   }
   __syncthreads();
   if (threadIdx.x == 0) {
@@ -168,20 +199,88 @@ __global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(Shared sh, StepAr
     sh.gate_scratch[1] = 0ull;
   }
   __syncthreads();
-  for (int i = threadIdx.x; i < L; i += kGateWarps * 32) {
-    int act;
-    switch (a.gate_mode) {
-      case GATE_ALWAYS: act = 1; break;
-      case GATE_GLOBAL: act = gflag_s; break;
-      case GATE_PER_LAYER: act = *reinterpret_cast<const volatile uint8_t *>(&a.flags[i]); break;  // other blocks'
-      default: act = (a.step % a.period) == 0; break;
-    }
-    sh.active[i] = (uint8_t)act;
-  }
+  gate_finish(sh, a, gflag_s, &count_s);
 }
 
 void launch_gate(const Shared &sh, const StepArgs &a, cudaStream_t s) {
   gate_kernel<<<std::max(1, (sh.num_layers + kGateWarps - 1) / kGateWarps), kGateWarps * 32, 0, s>>>(sh, a);
+}
+
+// ==================================================================== norms + gate ===
+// Gated modes with the fused buffer + B Q kernel: Algorithm 2 needs ||B|| before it knows which
+// layers take the Dion branch, so this pass reads M and G once more than the fused kernel would
+// (6 B/element) to form the sums of B^2 and M_{t-1}^2 per 128-row tile (the fused kernel's
+// slots), and the last block to finish runs the gate, so the fused kernel and everything after
+// it touch only the layers that sync.  Tile = {layer, 128-row block}.
+constexpr int kNormThreads = 256;
+template <int GT>
+__device__ void norms_tile(const DevLayer &L, int64_t row0, int64_t nrows, float sb[4], float sm[4]) {
+  const int64_t n = L.n, n4 = n >> 2;
+  for (int64_t rr = 0; rr < nrows; ++rr) {
+    const int64_t i = row0 + rr;
+    const float *Mrow = L.M + i * L.ldm;
+    const int64_t goff = i * L.ldg;
+    for (int64_t c4 = threadIdx.x; c4 < n4; c4 += kNormThreads) {
+      const float4 m = __ldcs(reinterpret_cast<const float4 *>(Mrow + 4 * c4));
+      float g[4];
+      load_g4<GT>(L.G, goff + 4 * c4, g);
+      const float b0 = m.x + g[0], b1 = m.y + g[1], b2 = m.z + g[2], b3 = m.w + g[3];
+      sm[0] = fmaf(m.x, m.x, sm[0]); sm[1] = fmaf(m.y, m.y, sm[1]);
+      sm[2] = fmaf(m.z, m.z, sm[2]); sm[3] = fmaf(m.w, m.w, sm[3]);
+      sb[0] = fmaf(b0, b0, sb[0]); sb[1] = fmaf(b1, b1, sb[1]);
+      sb[2] = fmaf(b2, b2, sb[2]); sb[3] = fmaf(b3, b3, sb[3]);
+    }
+    for (int64_t c = 4 * n4 + threadIdx.x; c < n; c += kNormThreads) {
+      const float mo = Mrow[c], b = mo + load_g1<GT>(L.G, goff + c);
+      sm[0] = fmaf(mo, mo, sm[0]);
+      sb[0] = fmaf(b, b, sb[0]);
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kNormThreads) norms_gate_kernel(Shared sh, StepArgs a, const int4 *tiles) {
+  __shared__ double red[kNormThreads / 32];
+  __shared__ int last_s, count_s;
+  __shared__ double max_s[kNormThreads / 32];
+  const int4 t = tiles[blockIdx.x];  // {layer, 128-row block}
+  const DevLayer &L = sh.layers[t.x];
+  const int64_t row0 = (int64_t)t.y * 128, nrows = min((int64_t)128, L.m - row0);
+  float sb[4] = {0.f, 0.f, 0.f, 0.f}, sm[4] = {0.f, 0.f, 0.f, 0.f};
+  if (L.g_dtype == DT_BF16) norms_tile<DT_BF16>(L, row0, nrows, sb, sm);
+  else norms_tile<DT_FP32>(L, row0, nrows, sb, sm);
+  const double b = block_sum<kNormThreads>(((double)sb[0] + sb[1]) + ((double)sb[2] + sb[3]), red);
+  const double mo = block_sum<kNormThreads>(((double)sm[0] + sm[1]) + ((double)sm[2] + sm[3]), red);
+  if (threadIdx.x == 0) {
+    const int slot = L.bpart_off + t.y;
+    sh.bpart[2 * slot] = b;
+    sh.bpart[2 * slot + 1] = mo;
+    __threadfence();  // this block's partials are visible before it is counted
+    last_s = atomicAdd(&sh.gate_scratch[2], 1ull) == (unsigned long long)(gridDim.x - 1);
+  }
+  __syncthreads();
+  if (!last_s) return;
+  __threadfence();
+  // the last block: Algorithm 2 for every layer, one warp per layer, and the maximum of RMMC
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  double mx = -1.0;
+  for (int l = warp; l < sh.num_layers; l += kNormThreads / 32) mx = fmax(mx, gate_layer(sh, a, l, lane));
+  if (lane == 0) max_s[warp] = mx;
+  __syncthreads();
+  __shared__ int gflag_s;
+  if (threadIdx.x == 0) {
+    double g = -1.0;
+    for (int w = 0; w < kNormThreads / 32; ++w) g = fmax(g, max_s[w]);
+    const int gf = (sh.num_layers > 0 && above(g, a.tau_global)) ? 1 : 0;
+    a.gflag[0] = (uint8_t)gf;
+    gflag_s = gf;
+    sh.gate_scratch[2] = 0ull;  // for the next step (kernel boundary orders it)
+  }
+  __syncthreads();
+  gate_finish(sh, a, gflag_s, &count_s);
+}
+
+void launch_norms_gate(const Shared &sh, const StepArgs &a, const int4 *tiles, int32_t ntiles, cudaStream_t s) {
+  if (ntiles > 0) norms_gate_kernel<<<ntiles, kNormThreads, 0, s>>>(sh, a, tiles);
 }
 
 // ==================================================================== grouped GEMM ===

@@ -217,7 +217,7 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
   const size_t o_nmb = cv.take<double>(std::max(num_layers, 1));
   const size_t o_nb = cv.take<double>(std::max(num_layers, 1));
   const size_t o_status = cv.take<int32_t>(1);
-  const size_t o_gate = cv.take<unsigned long long>(2);
+  const size_t o_gate = cv.take<unsigned long long>(4);
   const size_t o_bt = cv.take<int4>(std::max<size_t>(bt.size(), 1));
   const size_t o_ut = cv.take<int4>(std::max<size_t>(ut.size(), 1));
   const size_t o_ct = cv.take<int4>(std::max<size_t>(ct.size(), 1));
@@ -313,7 +313,7 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
     if (e == cudaSuccess) e = upload(p->gtiles[k], gt[k]);
   }
   if (e == cudaSuccess) e = cudaMemset(p->sh.status, 0, sizeof(int32_t));
-  if (e == cudaSuccess) e = cudaMemset(p->sh.gate_scratch, 0, 2 * sizeof(unsigned long long));  // key 0 < every RMMC
+  if (e == cudaSuccess) e = cudaMemset(p->sh.gate_scratch, 0, 4 * sizeof(unsigned long long));  // key 0 < every RMMC
   if (e == cudaSuccess && num_layers > 0) e = prepare_chol_inv(p->max_r, &p->chol_smem);
   if (e == cudaSuccess && precision != DION_PREC_FP32) {
     p->tcp.probs = p->probs;

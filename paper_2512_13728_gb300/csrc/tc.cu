@@ -47,6 +47,7 @@ constexpr uint32_t U_IDESC = idesc_bf16(128, 128, false, false);
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
     tc_update_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off, const LayerMaps *__restrict__ maps,
                      float mu, float eta, float keep) {
+  if (sh.gate_scratch[kScratchActive] == 0ull) return;  // no layer takes the Dion branch
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = align1024(smem_raw);
   uint8_t *stage = smem;
@@ -573,11 +574,17 @@ void refresh(const TcPlan &tp, const Shared &sh, cudaStream_t s) { launch_qn_ref
 
 void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, const int4 *btiles,
           int32_t n_btiles, const int4 *ctiles, int32_t n_ctiles, size_t chol_smem, cudaStream_t s) {
-  if (tp.fuse_buffer) {
-    launch_fused_bq(sh, tp, s);  // B = M + G, Bh, ||B||, ||M_{t-1}||, P = B Q_{t-1} (every layer)
+  if (tp.fuse_buffer && a.gate_mode == GATE_ALWAYS) {
+    launch_fused_bq(sh, tp, false, s);  // B = M + G, Bh, ||B||, ||M_{t-1}||, P = B Q_{t-1} (every layer)
     tick(p, s, "tc_form_bq");
     launch_gate(sh, a, s);
     tick(p, s, "gate");
+  } else if (tp.fuse_buffer) {
+    // gated modes: the norms and the gate first, then the fused kernel on the Dion-branch layers
+    launch_norms_gate(sh, a, tp.ftiles, tp.n_ftiles, s);
+    tick(p, s, "norms_gate");
+    launch_fused_bq(sh, tp, true, s);
+    tick(p, s, "tc_form_bq");
   } else {
     launch_form_b(sh, btiles, n_btiles, s);  // B = M + G (and its bf16 copy), ||B||, ||M_{t-1}||
     tick(p, s, "form_b");

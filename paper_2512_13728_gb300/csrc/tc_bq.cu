@@ -171,6 +171,7 @@ template <int KIND>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(R_THREADS, 1)
     tc_tma_gemm_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off,
                        const LayerMaps *__restrict__ maps, int nstages, uint32_t stage_bytes, uint32_t tmem_cols) {
+  if (sh.gate_scratch[kScratchActive] == 0ull) return;  // no layer takes the Dion branch
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = align1024(smem_raw);
   uint8_t *stg = smem + nstages * stage_bytes;
@@ -351,7 +352,10 @@ constexpr uint32_t FB_Q_OFF = FB_A_OFF + FB_ASTAGES * FB_GBOX;
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
     tc_form_bq_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off,
                       const LayerMaps *__restrict__ maps, uint32_t qstage_bytes, uint32_t qring_bytes,
-                      uint32_t tmem_cols) {
+                      uint32_t tmem_cols, int gated) {
+  // gated: the norms pass and the gate ran first; only Dion-branch layers are processed and the
+  // norm partials are not written again
+  if (gated && sh.gate_scratch[kScratchActive] == 0ull) return;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = align1024(smem_raw);
   uint8_t *aring = smem + FB_A_OFF;
@@ -409,6 +413,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
       bool ok = true;
       for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
+        if (gated && !sh.active[t.x]) continue;
         const DevLayer &L = sh.layers[t.x];
         const LayerMaps *mp = maps + t.x;
         const int kch = (int)((L.n + 63) / 64);
@@ -428,6 +433,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
     uint32_t it = 0;
     for (int ti = off[seg]; ti < off[seg + 1]; ++ti) {
       const int4 t = tiles[ti];
+      if (gated && !sh.active[t.x]) continue;
       const DevLayer &L = sh.layers[t.x];
       const int kch = (int)((L.n + 63) / 64);
       const int64_t row0 = (int64_t)(2 * t.y + (int)rank) * 128;
@@ -457,8 +463,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
     if (lane == 0) {
       uint32_t it = 0, tcount = 0;
       bool ok = true;
-      for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti, ++tcount) {
+      for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
+        if (gated && !sh.active[t.x]) continue;
         const DevLayer &L = sh.layers[t.x];
         const LayerMaps *mp = maps + t.x;
         const int kch = (int)((L.n + 63) / 64);
@@ -467,6 +474,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
         for (uint32_t part = 0; part < nparts; ++part) nbox += (half_cols(np, part) + 63) / 64;
         // the ring holds the previous tile's staged accumulator until its stores have read it
         if (tcount > 0 && !ab.wait(epi_free, (tcount - 1) & 1u, sh.status)) break;
+        ++tcount;
         for (int kc = 0; kc < kch; ++kc, ++it) {
           const uint32_t s = it % FB_QSTAGES, ph = (it / FB_QSTAGES) & 1u;
           if (!ab.wait(&qempty[s], ph ^ 1u, sh.status)) { ok = false; break; }
@@ -490,6 +498,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
       bool ok = true;
       for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
+        if (gated && !sh.active[t.x]) continue;
         const DevLayer &L = sh.layers[t.x];
         const int kch = (int)((L.n + 63) / 64);
         const int tr = 2 * t.y + (int)rank;
@@ -513,6 +522,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
       bool ok = true;
       for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
+        if (gated && !sh.active[t.x]) continue;
         const DevLayer &L = sh.layers[t.x];
         const int kch = (int)((L.n + 63) / 64);
         const uint32_t np = rpad16(L.r), nparts = (np + 255) / 256;
@@ -548,6 +558,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
     uint32_t tcount = 0, ecount = 0;
     for (int ti = off[seg]; ti < off[seg + 1]; ++ti) {
       const int4 t = tiles[ti];
+      if (gated && !sh.active[t.x]) continue;
       const DevLayer &L = sh.layers[t.x];
       const int tr = 2 * t.y + (int)rank;
       if (!named_and(1, 128, ab.wait(acc_full, tcount & 1u, sh.status))) break;
@@ -570,6 +581,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
     uint32_t it = 0;
     for (int ti = off[seg]; ti < off[seg + 1]; ++ti) {
       const int4 t = tiles[ti];
+      if (gated && !sh.active[t.x]) continue;
       const DevLayer &L = sh.layers[t.x];
       const int tr = 2 * t.y + (int)rank;
       const int kch = (int)((L.n + 63) / 64);
@@ -634,7 +646,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
         red_s[1][cw] = accm;
       }
       named_sync(2, 128);
-      if (ct == 0 && (int64_t)tr * 128 < L.m) {
+      if (ct == 0 && !gated && (int64_t)tr * 128 < L.m) {
         const int slot = L.bpart_off + tr;
         sh.bpart[2 * slot] = (red_s[0][0] + red_s[0][1]) + (red_s[0][2] + red_s[0][3]);
         sh.bpart[2 * slot + 1] = (red_s[1][0] + red_s[1][1]) + (red_s[1][2] + red_s[1][3]);
@@ -680,10 +692,11 @@ cudaError_t setup_fused_bq_kernel(uint32_t smem) {
   return cudaFuncSetAttribute(tc_form_bq_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
 }
 
-void launch_fused_bq(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
+void launch_fused_bq(const Shared &sh, const TcPlan &tp, bool gated, cudaStream_t s) {
   if (tp.d_bq.grid <= 0) return;
   tc_form_bq_kernel<<<2 * tp.d_bq.grid, FB_THREADS, tp.fb_smem, s>>>(
-      sh, tp.d_bq.tiles, tp.d_bq.off, tp.maps, tp.bq_boxes * BOX64, fused_bq_qring(tp.bq_boxes), tp.tmem_cols);
+      sh, tp.d_bq.tiles, tp.d_bq.off, tp.maps, tp.bq_boxes * BOX64, fused_bq_qring(tp.bq_boxes), tp.tmem_cols,
+      gated ? 1 : 0);
 }
 
 void launch_form_bq(const Shared &sh, const TcPlan &tp, cudaStream_t s) {

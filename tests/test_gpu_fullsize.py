@@ -44,13 +44,13 @@ def check_all_layer_flags(plan, taus, tau_global):
     assert bool(plan.global_flag[0].item()) == oc.above(gmax, float(np.float32(tau_global)))
 
 
-def run_sampled(w, precision, hp_kw, steps, tol, sample, check_steps=None):
+def run_sampled(w, precision, hp_kw, steps, tol, sample, check_steps=None, taus=None):
     """Runs `steps` steps of the whole stack; at the steps in `check_steps` (all by default) the
     oracle takes one step of the sampled layers from the device state and the results are
     compared.  Returns the worst errors seen."""
     import paper_2512_13728_gb300 as cd
 
-    st = gu.make_state(w)
+    st = gu.make_state(w, taus=taus)
     L = w.num_layers
     plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, precision)
     hpo = gu.oracle_hp(**hp_kw)
@@ -112,6 +112,21 @@ def test_gpt1p3b_stack_r512_bf16_blocks_0_and_23():
     sample = blocks(w, [0, 23])
     worst, _ = run_sampled(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_ALWAYS), 2, TOL_BF16, sample)
     print("1.3B stack sampled worst", worst)
+
+
+def test_gpt1p3b_stack_r512_bf16_per_layer_gate_mixed():
+    """The bench workload under the per-layer gate with every other layer forced local (tau
+    1e6) and the rest forced to sync (tau 1e-6): the norms pass + gate run first and the fused
+    buffer + B Q kernel and everything after it touch only the syncing layers.  Two steps;
+    blocks 0 and 23 checked against the oracle, every layer's flags against its RMMC."""
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.WORKLOADS["gpt1p3b_stack_r512"]
+    taus = [1e6 if l % 2 else 1e-6 for l in range(w.num_layers)]
+    sample = blocks(w, [0, 23])
+    worst, _ = run_sampled(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_PER_LAYER, tau_global=0.5), 2, TOL_BF16,
+                           sample, taus=taus)
+    print("1.3B stack per-layer mixed worst", worst)
 
 
 @pytest.mark.parametrize("name", ["gpt160m_stack_r192", "gpt160m_stack_r48"])
