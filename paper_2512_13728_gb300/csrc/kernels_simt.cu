@@ -216,25 +216,47 @@ constexpr int kNormThreads = 256;
 template <int GT>
 __device__ void norms_tile(const DevLayer &L, int64_t row0, int64_t nrows, float sb[4], float sm[4]) {
   const int64_t n = L.n, n4 = n >> 2;
-  for (int64_t rr = 0; rr < nrows; ++rr) {
+  // four rows at a time: each thread keeps four independent M and G loads in flight
+  int64_t rr = 0;
+  for (; rr + 4 <= nrows; rr += 4) {
     const int64_t i = row0 + rr;
-    const float *Mrow = L.M + i * L.ldm;
-    const int64_t goff = i * L.ldg;
     for (int64_t c4 = threadIdx.x; c4 < n4; c4 += kNormThreads) {
-      const float4 m = __ldcs(reinterpret_cast<const float4 *>(Mrow + 4 * c4));
+      float4 m[4];
+      float g[4][4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        m[u] = __ldcs(reinterpret_cast<const float4 *>(L.M + (i + u) * L.ldm + 4 * c4));
+        load_g4<GT>(L.G, (i + u) * L.ldg + 4 * c4, g[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float b0 = m[u].x + g[u][0], b1 = m[u].y + g[u][1], b2 = m[u].z + g[u][2], b3 = m[u].w + g[u][3];
+        sm[0] = fmaf(m[u].x, m[u].x, sm[0]); sm[1] = fmaf(m[u].y, m[u].y, sm[1]);
+        sm[2] = fmaf(m[u].z, m[u].z, sm[2]); sm[3] = fmaf(m[u].w, m[u].w, sm[3]);
+        sb[0] = fmaf(b0, b0, sb[0]); sb[1] = fmaf(b1, b1, sb[1]);
+        sb[2] = fmaf(b2, b2, sb[2]); sb[3] = fmaf(b3, b3, sb[3]);
+      }
+    }
+  }
+  for (; rr < nrows; ++rr) {
+    const int64_t i = row0 + rr;
+    for (int64_t c4 = threadIdx.x; c4 < n4; c4 += kNormThreads) {
+      const float4 m = __ldcs(reinterpret_cast<const float4 *>(L.M + i * L.ldm + 4 * c4));
       float g[4];
-      load_g4<GT>(L.G, goff + 4 * c4, g);
+      load_g4<GT>(L.G, i * L.ldg + 4 * c4, g);
       const float b0 = m.x + g[0], b1 = m.y + g[1], b2 = m.z + g[2], b3 = m.w + g[3];
       sm[0] = fmaf(m.x, m.x, sm[0]); sm[1] = fmaf(m.y, m.y, sm[1]);
       sm[2] = fmaf(m.z, m.z, sm[2]); sm[3] = fmaf(m.w, m.w, sm[3]);
       sb[0] = fmaf(b0, b0, sb[0]); sb[1] = fmaf(b1, b1, sb[1]);
       sb[2] = fmaf(b2, b2, sb[2]); sb[3] = fmaf(b3, b3, sb[3]);
     }
-    for (int64_t c = 4 * n4 + threadIdx.x; c < n; c += kNormThreads) {
-      const float mo = Mrow[c], b = mo + load_g1<GT>(L.G, goff + c);
-      sm[0] = fmaf(mo, mo, sm[0]);
-      sb[0] = fmaf(b, b, sb[0]);
-    }
+  }
+  // columns past the last multiple of 4
+  for (int64_t e = threadIdx.x; e < nrows * (n - 4 * n4); e += kNormThreads) {
+    const int64_t i = row0 + e / (n - 4 * n4), c = 4 * n4 + e % (n - 4 * n4);
+    const float mo = L.M[i * L.ldm + c], b = mo + load_g1<GT>(L.G, i * L.ldg + c);
+    sm[0] = fmaf(mo, mo, sm[0]);
+    sb[0] = fmaf(b, b, sb[0]);
   }
 }
 
