@@ -94,6 +94,10 @@ struct Shared {
   // pass's finished-block count, and (written by the gate) the number of layers that take the
   // Dion branch this step, which lets the later persistent kernels return at once when it is 0
   unsigned long long *gate_scratch;
+  // 1 when this step's norms pass has already written B = M + G into M (gated modes with bf16
+  // gradients): the fused kernel and the update then read B from M without G, and the local
+  // branch leaves M alone
+  int32_t b_in_m;
 };
 
 // A contraction C = op(A) op(B) for the CUDA-core path.

@@ -208,13 +208,15 @@ void launch_gate(const Shared &sh, const StepArgs &a, cudaStream_t s) {
 
 // ==================================================================== norms + gate ===
 // Gated modes with the fused buffer + B Q kernel: Algorithm 2 needs ||B|| before it knows which
-// layers take the Dion branch, so this pass reads M and G once more than the fused kernel would
-// (6 B/element) to form the sums of B^2 and M_{t-1}^2 per 128-row tile (the fused kernel's
-// slots), and the last block to finish runs the gate, so the fused kernel and everything after
-// it touch only the layers that sync.  Tile = {layer, 128-row block}.
+// layers take the Dion branch, so this pass forms B = M + G into M (read M, G; write M:
+// 10 B/element) with the sums of B^2 and M_{t-1}^2 per 128-row tile (the fused kernel's slots),
+// and the last block to finish runs the gate.  The fused kernel and everything after it touch
+// only the layers that sync and read B from M; the local branch then only updates X.
+// Tile = {layer, 128-row block}.
 constexpr int kNormThreads = 256;
 template <int GT>
 __device__ void norms_tile(const DevLayer &L, int64_t row0, int64_t nrows, float sb[4], float sm[4]) {
+  float *M = L.M;
   const int64_t n = L.n, n4 = n >> 2;
   // four rows at a time: each thread keeps four independent M and G loads in flight
   int64_t rr = 0;
@@ -235,6 +237,7 @@ __device__ void norms_tile(const DevLayer &L, int64_t row0, int64_t nrows, float
         sm[2] = fmaf(m[u].z, m[u].z, sm[2]); sm[3] = fmaf(m[u].w, m[u].w, sm[3]);
         sb[0] = fmaf(b0, b0, sb[0]); sb[1] = fmaf(b1, b1, sb[1]);
         sb[2] = fmaf(b2, b2, sb[2]); sb[3] = fmaf(b3, b3, sb[3]);
+        *reinterpret_cast<float4 *>(M + (i + u) * L.ldm + 4 * c4) = make_float4(b0, b1, b2, b3);
       }
     }
   }
@@ -249,14 +252,16 @@ __device__ void norms_tile(const DevLayer &L, int64_t row0, int64_t nrows, float
       sm[2] = fmaf(m.z, m.z, sm[2]); sm[3] = fmaf(m.w, m.w, sm[3]);
       sb[0] = fmaf(b0, b0, sb[0]); sb[1] = fmaf(b1, b1, sb[1]);
       sb[2] = fmaf(b2, b2, sb[2]); sb[3] = fmaf(b3, b3, sb[3]);
+      *reinterpret_cast<float4 *>(M + i * L.ldm + 4 * c4) = make_float4(b0, b1, b2, b3);
     }
   }
   // columns past the last multiple of 4
   for (int64_t e = threadIdx.x; e < nrows * (n - 4 * n4); e += kNormThreads) {
     const int64_t i = row0 + e / (n - 4 * n4), c = 4 * n4 + e % (n - 4 * n4);
-    const float mo = L.M[i * L.ldm + c], b = mo + load_g1<GT>(L.G, i * L.ldg + c);
+    const float mo = M[i * L.ldm + c], b = mo + load_g1<GT>(L.G, i * L.ldg + c);
     sm[0] = fmaf(mo, mo, sm[0]);
     sb[0] = fmaf(b, b, sb[0]);
+    M[i * L.ldm + c] = b;
   }
 }
 
@@ -908,9 +913,9 @@ void launch_update(const Shared &sh, const int4 *tiles, int32_t ntiles, float mu
 // keep = 1 - eta_local * weight_decay), and M = B = M + G (already in place unless the layer
 // defers B to the update).
 template <int GT>
-__device__ void local_tile(const DevLayer &L, int64_t row0, int64_t nrows, float eta_local, float keep) {
+__device__ void local_tile(const DevLayer &L, int64_t row0, int64_t nrows, float eta_local, float keep, bool b_in_m) {
   const int64_t n = L.n, n4 = n >> 2;
-  const bool form_m = L.b_deferred != 0;
+  const bool form_m = L.b_deferred != 0 && !b_in_m;
   for (int64_t rr = 0; rr < nrows; ++rr) {
     const int64_t i = row0 + rr;
     float *Xrow = L.X + i * L.ldx, *Mrow = L.M + i * L.ldm;
@@ -940,8 +945,8 @@ __global__ void __launch_bounds__(kRowThreads) local_kernel(Shared sh, const int
   const int4 t = tiles[blockIdx.x];
   if (sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
-  if (L.g_dtype == DT_BF16) local_tile<DT_BF16>(L, t.y, t.z, eta_local, keep);
-  else local_tile<DT_FP32>(L, t.y, t.z, eta_local, keep);
+  if (L.g_dtype == DT_BF16) local_tile<DT_BF16>(L, t.y, t.z, eta_local, keep, sh.b_in_m != 0);
+  else local_tile<DT_FP32>(L, t.y, t.z, eta_local, keep, sh.b_in_m != 0);
 }
 
 void launch_local(const Shared &sh, const int4 *tiles, int32_t ntiles, float eta_local, float keep, cudaStream_t s) {

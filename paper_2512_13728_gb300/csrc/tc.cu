@@ -182,7 +182,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
         if (issued >= U_EBUF) bulk_wait_read<1>();
         uint8_t *bs = epi + eb * U_EBUF2;
         const int r0 = (2 * t.y + (int)rank) * 128, x0 = t.z * 128 + lj * 16;
-        const bool defer = sh.layers[t.x].b_deferred != 0;  // B = M + G is formed here
+        const bool defer = sh.layers[t.x].b_deferred != 0 && !sh.b_in_m;  // B = M + G is formed here
         mbar_expect_tx(&epi_full[eb], 2u * U_EBOX + (defer ? U_GBOX : 0u));
         tma_load_2d(bs, &mp->Mf16, &epi_full[eb], x0, r0);
         tma_load_2d(bs + U_EBOX, &mp->Xf16, &epi_full[eb], x0, r0);
@@ -207,7 +207,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
       const int mb = 2 * t.y + (int)rank, r0 = mb * 128, c0 = t.z * 128;
       const int ntc = (int)((L.n + 127) / 128);
       const int ns = subs_of(t);
-      const bool defer = L.b_deferred != 0;
+      const bool defer = L.b_deferred != 0 && !sh.b_in_m;
       const uint32_t b = tcount & 1u, aph = (tcount >> 1) & 1u;
       if (!named_and(1, 128, ab.wait(&acc_full[b], aph, sh.status))) break;
       tc_fence_after();
@@ -572,8 +572,10 @@ int32_t launches_per_step(const TcPlan &tp) { return tp.launches; }
 
 void refresh(const TcPlan &tp, const Shared &sh, cudaStream_t s) { launch_qn_refresh(sh, tp, s); }
 
-void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, const int4 *btiles,
+void step(dion_plan *p, const TcPlan &tp, const Shared &sh_in, const StepArgs &a, const int4 *btiles,
           int32_t n_btiles, const int4 *ctiles, int32_t n_ctiles, size_t chol_smem, cudaStream_t s) {
+  Shared sh = sh_in;
+  sh.b_in_m = (tp.fuse_buffer && a.gate_mode != GATE_ALWAYS) ? 1 : 0;  // the norms pass writes B into M
   if (tp.fuse_buffer && a.gate_mode == GATE_ALWAYS) {
     launch_fused_bq(sh, tp, false, s);  // B = M + G, Bh, ||B||, ||M_{t-1}||, P = B Q_{t-1} (every layer)
     tick(p, s, "tc_form_bq");

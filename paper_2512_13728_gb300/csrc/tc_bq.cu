@@ -421,6 +421,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
         for (int kc = 0; kc < kch; ++kc, ++it) {
           const uint32_t sg = it % FB_ASTAGES, pg = (it / FB_ASTAGES) & 1u;
           if (!ab.wait(&gempty[sg], pg ^ 1u, sh.status)) { ok = false; break; }
+          if (gated) {  // B is already in M: the slot only receives the converted A box
+            mbar_arrive(&gfull[sg]);
+            continue;
+          }
           mbar_expect_tx(&gfull[sg], FB_GBOX);
           tma_load_2d(aring + sg * FB_GBOX, &mp->Gh64, &gfull[sg], kc * 64, tr * 128);
         }
@@ -602,7 +606,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
             const uint32_t e = (uint32_t)(i * 128 + ct);
             const uint32_t row = (e & 7u) + 8u * (e >> 6), c = (e >> 3) & 7u, sw = row & 7u;
             uint4 *ga = reinterpret_cast<uint4 *>(sG + row * 128u + ((c ^ sw) << 4));
-            const uint4 g = *ga;
+            const uint4 g = gated ? make_uint4(0u, 0u, 0u, 0u) : *ga;  // gated: B is in M, no G
             const uint8_t *mrow = sM + (c >> 2) * FB_MBOX + row * 128u;
             const uint32_t mc = 2u * (c & 3u);
             const float4 m0 = *reinterpret_cast<const float4 *>(mrow + ((mc ^ sw) << 4));
