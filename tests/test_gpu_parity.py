@@ -320,13 +320,18 @@ def test_deterministic_bitwise_bf16_mode(g_dtype):
         assert torch.equal(a, b)
 
 
-@pytest.mark.parametrize("prec,g_dtype", [("bf16", "bf16"), ("bf16", "fp32"), ("fp32", "bf16")])
-def test_step_host_matches_device_gradients(prec, g_dtype):
+@pytest.mark.parametrize("prec,g_dtype,mode", [("bf16", "bf16", "always"), ("bf16", "fp32", "always"),
+                                               ("fp32", "bf16", "always"), ("bf16", "bf16", "per_layer"),
+                                               ("bf16", "bf16", "global"), ("fp32", "fp32", "per_layer")])
+def test_step_host_matches_device_gradients(prec, g_dtype, mode):
     """dion_step_host (gradients copied from pinned host tensors into the plan's two alternating
     buffers) gives bit for bit the results of dion_step on the same gradients in device memory;
-    the host tensors of odd steps have a padded leading dimension (2-D copy)."""
+    the host tensors of odd steps have a padded leading dimension (2-D copy).  The gated cases
+    take local steps from step 3 on (RMMC falls below tau = 0.5), so the norms pass that writes
+    B into M runs on the host-gradient buffers too."""
     import paper_2512_13728_gb300 as cd
 
+    gm = {"always": cd.DION_GATE_ALWAYS, "per_layer": cd.DION_GATE_PER_LAYER, "global": cd.DION_GATE_GLOBAL}[mode]
     p = cd.DION_PREC_BF16 if prec == "bf16" else cd.DION_PREC_FP32
     w = wl.scaled(RAGGED, "ragged_host", RAGGED.shapes, g_dtype=g_dtype, steps=5)
     outs = []
@@ -348,10 +353,10 @@ def test_step_host_matches_device_gradients(prec, g_dtype):
                     buf[:, :n].copy_(g.cpu())
                     hg.append(buf[:, :n])
                     g.fill_(float("nan"))  # the device copies given at creation are not read
-                plan.step_host(cd.hparams(step=t), hg)
+                plan.step_host(cd.hparams(step=t, gate_mode=gm, tau_global=0.5), hg)
                 torch.cuda.synchronize()
             else:
-                plan.step(cd.hparams(step=t))
+                plan.step(cd.hparams(step=t, gate_mode=gm, tau_global=0.5))
             seq.append((plan.rmmc.clone(), plan.flags.clone(), plan.global_flag.clone()))
         torch.cuda.synchronize()
         assert plan.device_status() == 0
