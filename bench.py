@@ -44,12 +44,16 @@ def load_peaks():
     return dict(hbm=6800.0, bf16=1900.0, bf16_sust=1700.0, sm_mhz=2070.0, source="fallback")
 
 
-def csrc_hash() -> str:
+def sources_hash(names) -> str:
+    """Hash of the listed files under the package's csrc/ (the translation unit of one kernel and
+    its host-side schedule), so a stored ncu counter stays valid until that code changes."""
     h = hashlib.sha1()
     d = os.path.join(ROOT, "paper_2512_13728_gb300", "csrc")
-    for name in sorted(os.listdir(d)):
+    for name in sorted(names):
         with open(os.path.join(d, name), "rb") as f:
             h.update(name.encode() + f.read())
+    with open(os.path.join(ROOT, "include", "curvadion.h"), "rb") as f:
+        h.update(f.read())
     return h.hexdigest()[:12]
 
 
@@ -308,7 +312,7 @@ def run_ours(args, rank, world, local_rank):
             with open(tpath) as f:
                 tj = json.load(f)
             ent = tj.get(f"{args.workload}:{prec}:{dom['name']}")
-            if ent and ent.get("csrc") == csrc_hash():
+            if ent and ent.get("src_hash") == sources_hash(ent.get("sources", [])):
                 traffic = ent["bytes_per_launch"]
         roofline = {"kernel": dom["name"], "bound": dom["bound"], "achieved": round(achieved, 2), "peak": peak,
                     "unit": punit, "frac": round(achieved / peak, 4), "traffic": traffic,

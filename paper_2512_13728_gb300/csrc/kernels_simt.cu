@@ -718,13 +718,21 @@ __global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, in
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
   if (pass >= 1) {
-    // ||E||_F^2 from the lower triangle (E symmetric), fixed-order reduction
+    // ||E||_F^2 from the lower triangle (E symmetric), fixed-order reduction; 16-byte loads
+    // (a row's padding up to the next multiple of 4 columns lies inside ls and is masked)
     double fs = 0.0;
     for (int i = warp; i < r; i += kCholThreads / 32) {
       float a = 0.f;
-      for (int j = lane; j <= i; j += 32) {
-        const float e = S[(int64_t)i * ls + j] - (i == j ? 1.f : 0.f);
-        a = fmaf((j < i ? 2.f : 1.f) * e, e, a);
+#pragma unroll 4
+      for (int j4 = lane; 4 * j4 <= i; j4 += 32) {
+        const float4 v = *reinterpret_cast<const float4 *>(S + (int64_t)i * ls + 4 * j4);
+        const float ve[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const int j = 4 * j4 + c;
+          const float e = (j <= i) ? ve[c] - (i == j ? 1.f : 0.f) : 0.f;
+          a = fmaf((j < i ? 2.f : 1.f) * e, e, a);
+        }
       }
       fs += (double)a;
     }
@@ -737,11 +745,29 @@ __global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, in
       lam = power_norm_sym(S, r, ls, Y, ldy);
     }
     if (isfinite(lam) && 1.5f * lam < near_identity) {
-      for (int i = warp; i < r; i += kCholThreads / 32)
-        for (int j = lane; j < r; j += 32) {
-          const float sij = (j <= i) ? S[(int64_t)i * ls + j] : 0.f;
-          Li[(int64_t)i * ls + j] = (j < i) ? -sij : (j == i ? 1.f - 0.5f * (sij - 1.f) : 0.f);
+      // 16-byte loads and stores; a group that straddles column r is stored element-wise
+      const int r4 = (r + 3) / 4;
+      for (int i = warp; i < r; i += kCholThreads / 32) {
+#pragma unroll 4
+        for (int j4 = lane; j4 < r4; j4 += 32) {
+          float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+          if (4 * j4 <= i) v = *reinterpret_cast<const float4 *>(S + (int64_t)i * ls + 4 * j4);
+          float o[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            const int j = 4 * j4 + c;
+            o[c] = (j < i) ? -o[c] : (j == i ? 1.f - 0.5f * (o[c] - 1.f) : 0.f);
+          }
+          float *dst = Li + (int64_t)i * ls + 4 * j4;
+          if (4 * j4 + 4 <= r) {
+            *reinterpret_cast<float4 *>(dst) = make_float4(o[0], o[1], o[2], o[3]);
+          } else {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+              if (4 * j4 + c < r) dst[c] = o[c];
+          }
         }
+      }
       return;
     }
   }

@@ -68,3 +68,20 @@ def test_reference_arm_under_torchrun_world2():
     assert rec["impl"] == "reference" and rec["higher_is_better"] is False
     assert rec["value"] > 0 and rec["cpu_baseline"]["kind"] == "oracle"
     assert rec["e2e"]["h2d_bytes_per_step"] == 0
+
+
+def test_stored_traffic_entries_name_their_sources():
+    """Every stored per-launch DRAM figure names the sources of its kernel, and bench.py reports
+    it only while their hash matches (a changed kernel gets traffic null until re-captured)."""
+    sys.path.insert(0, ROOT)
+    import bench
+
+    with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+        tj = json.load(f)
+    assert tj
+    for key, ent in tj.items():
+        assert ent["sources"] and ent["bytes_per_launch"] > 0, key
+        for name in ent["sources"]:
+            assert os.path.exists(os.path.join(ROOT, "paper_2512_13728_gb300", "csrc", name)), (key, name)
+        assert len(ent["src_hash"]) == 12
+        assert bench.sources_hash(ent["sources"]) != bench.sources_hash(ent["sources"][:-1])
