@@ -59,24 +59,37 @@ def sources_hash(names) -> str:
 
 # ------------------------------------------------------------------ algorithmic work ---
 
-def kernel_work(name: str, w, prec: str):
-    """(bound, algorithmic units per launch, unit) for one kernel of the step, all layers active.
-    Bytes count each compulsory read and write once; flops count 2 per multiply-add."""
+def kernel_work(name: str, w, prec: str, gate: str = "always", wt=None):
+    """(bound, algorithmic units per launch, unit) for one kernel of the step.  wt[l] is the
+    fraction of the timed steps in which layer l took the Dion branch (all 1 with --gate always);
+    kernels that run only on syncing layers count those layers' work by it.  Bytes count each
+    compulsory read and write once; flops count 2 per multiply-add."""
     gsz = 2 if w.g_dtype == "bf16" else 4
     ranks = w.ranks()
-    mn = sum(m * n for m, n in w.shapes)
-    mnr = sum(m * n * r for (m, n), r in zip(w.shapes, ranks))
-    mr2 = sum(m * r * r for (m, n), r in zip(w.shapes, ranks))
-    r3 = sum(r ** 3 for r in ranks)
-    nr = sum(n * r for (m, n), r in zip(w.shapes, ranks))
-    mr = sum(m * r for (m, n), r in zip(w.shapes, ranks))
+    L = len(w.shapes)
+    wt = [1.0] * L if wt is None else list(wt)
+
+    def tot(f, act=True):  # sum over layers of f(m, n, r), weighted by activity
+        return sum(f(m, n, r) * (wt[l] if act else 1.0) for l, ((m, n), r) in enumerate(zip(w.shapes, ranks)))
+
+    mn_all = tot(lambda m, n, r: m * n, act=False)
+    mn = tot(lambda m, n, r: m * n)
+    mn_loc = mn_all - mn
+    mnr = tot(lambda m, n, r: m * n * r)
+    mr2 = tot(lambda m, n, r: m * r * r)
+    r3 = tot(lambda m, n, r: r ** 3)
+    nr = tot(lambda m, n, r: n * r)
+    mr = tot(lambda m, n, r: m * r)
     bh = 2 if prec == "bf16" else 0  # the bf16 copy of B the tensor-core contractions read
-    # tensor-core mode with bf16 G: the buffer pass leaves M_{t-1} in place and the update
-    # forms B = M + G itself (it reads G, the buffer pass does not write M)
-    deferred = prec == "bf16" and w.g_dtype == "bf16"
+    # tensor-core mode with bf16 G: in DION_GATE_ALWAYS the buffer pass leaves M_{t-1} in place
+    # and the update forms B = M + G itself (it reads G); in the gated modes the norms pass
+    # writes B into M first, and neither the fused B Q kernel nor the update reads G
+    fused = prec == "bf16" and w.g_dtype == "bf16"
+    b_in_m = fused and gate != "always"
+    deferred = fused and not b_in_m
     table = {
-        # CUDA-core path
-        "form_b": ("hbm", mn * (4 + gsz + (0 if deferred else 4) + bh), "B"),
+        # CUDA-core path (form_b runs on every layer before the gate)
+        "form_b": ("hbm", mn_all * (4 + gsz + (0 if fused else 4) + bh), "B"),
         "gemm_bq": ("alu", 2 * mnr, "flop"),
         "gemm_gram": ("alu", 2 * mr2, "flop"),
         "chol_inv": ("alu", 2 * r3 / 3, "flop"),
@@ -84,13 +97,16 @@ def kernel_work(name: str, w, prec: str):
         "gemm_btp": ("alu", 2 * mnr, "flop"),
         "colnorm": ("hbm", nr * 8, "B"),
         "update": ("alu", 4 * mnr, "flop") if prec == "fp32" else ("hbm", mn * 16, "B"),
-        "local": ("hbm", 0, "B"),
+        # local layers: read X, G; write X (M already holds B)
+        "local": ("hbm", mn_loc * (8 + gsz), "B"),
         # tensor-core path
         "tc_bq": ("hbm", mn * 2 + nr * 2 + mr * 8, "B"),  # Bh, bf16 Q; P and P^T fp32
-        # buffer pass fused into B Q (bf16 G): read M, G; write Bh, P and P^T fp32
-        "tc_form_bq": ("hbm", mn * (4 + gsz + 2) + mr * 8, "B"),
-        # gated modes: the norms pass read M, G (and the gate in its last block)
-        "norms_gate": ("hbm", mn * (4 + gsz), "B"),
+        # buffer pass fused into B Q (bf16 G): read M (and G unless B is already in M); write Bh,
+        # P and P^T fp32
+        "tc_form_bq": ("hbm", mn * (4 + (0 if b_in_m else gsz) + 2) + mr * 8, "B"),
+        # gated modes: the norms pass reads M, G and writes B into M on every layer (and runs
+        # the gate in its last block)
+        "norms_gate": ("hbm", mn_all * (4 + gsz + 4), "B"),
         "tc_btp": ("hbm", mn * 2 + mr * 2 + nr * 6, "B"),  # Bh, bf16 P; R fp32 and bf16
         "tc_update": ("hbm", mn * (16 + (gsz if deferred else 0)), "B"),
         "tc_gram": ("tensor", 2 * mr2, "flop"),
@@ -99,18 +115,79 @@ def kernel_work(name: str, w, prec: str):
     return table.get(name, ("latency", 0, ""))
 
 
-def step_bytes(w, prec):
-    """Bytes one synchronized step moves by design (the planned passes), and the compulsory floor."""
+def step_bytes(w, prec, gate: str = "always", wt=None):
+    """Bytes one step moves by design (the planned passes) and the compulsory floor (read M, G,
+    X; write M, X: 18 B/element with bf16 G, on either branch), with layer l syncing in a
+    fraction wt[l] of the steps."""
     gsz = 2 if w.g_dtype == "bf16" else 4
-    mn = sum(m * n for m, n in w.shapes)
-    if prec == "fp32":
-        planned = mn * ((4 + gsz + 4) + 4 + 4 + 16)
-    elif w.g_dtype == "bf16":  # buffer pass fused with B Q 8, the Bh read of B^T P 2, update 18
-        planned = mn * ((4 + gsz + 2) + 2 + (16 + gsz))
-    else:
-        planned = mn * ((4 + gsz + 4 + 2) + 2 + 2 + 16)
-    compulsory = mn * (4 + gsz + 4 + 4 + 4)  # read M, G, X; write M, X
+    L = len(w.shapes)
+    wt = [1.0] * L if wt is None else list(wt)
+    mn_all = sum(m * n for m, n in w.shapes)
+    mn = sum(m * n * wt[l] for l, (m, n) in enumerate(w.shapes))
+    mn_loc = mn_all - mn
+    fused = prec == "bf16" and w.g_dtype == "bf16"
+    if prec == "fp32":  # form_b 12 (+4 with fp32 G), B Q and B^T P read B 4 + 4, update 16
+        planned = mn_all * (4 + gsz + 4) + mn * (4 + 4 + 16)
+    elif fused and gate == "always":  # buffer pass fused with B Q 8, the Bh read of B^T P 2, update 18
+        planned = mn_all * ((4 + gsz + 2) + 2 + (16 + gsz))
+    elif fused:  # norms pass 10 on every layer; synced: fused B Q 6, Bh read 2, update 16
+        planned = mn_all * (4 + gsz + 4) + mn * (6 + 2 + 16)
+    else:  # form_b 14 with fp32 G, Bh read of B Q and B^T P 2 + 2, update 16
+        planned = mn_all * (4 + gsz + 4 + 2) + mn * (2 + 2 + 16)
+    planned += mn_loc * (8 + gsz)  # local branch: read X, G; write X
+    compulsory = mn_all * (4 + gsz + 4 + 4 + 4)  # read M, G, X; write M, X
     return planned, compulsory
+
+
+def make_gradient_sequence(wl, w, dtype, dev, steps):
+    """One flat device tensor per step t in `steps` holding every layer's G_t (row-major, layer
+    after layer)."""
+    import torch
+
+    out = []
+    for t in steps:
+        out.append(torch.cat([wl.gradient(w, l, t, dev).to(dtype).reshape(-1) for l in range(w.num_layers)]))
+    return out
+
+
+def layer_views(flat, w):
+    """Each layer's m x n gradient as a view of the flat buffer."""
+    views, off = [], 0
+    for m, n in w.shapes:
+        views.append(flat[off: off + m * n].view(m, n))
+        off += m * n
+    return views
+
+
+def replay_sync_pattern(cd, wl, w, prec_code, gate_code, tau, t0, warmup, steps, seq, dev):
+    """Which layers took the Dion branch in each timed step, from an untimed replay of the same
+    run (same seeded initial state, gradient sequence and hyper-parameters; a plan's steps are
+    deterministic, so it reaches the same decisions).  Returns per-layer fractions of the timed
+    steps and the number of syncing layers in each."""
+    X, M, Q = [], [], []
+    for l in range(w.num_layers):
+        x0, m0, q0 = wl.init_layer(w, l, dev)
+        X.append(x0); M.append(m0); Q.append(q0)
+    gflat = seq[0].clone()
+    L = w.num_layers
+    plan = cd.Plan(X, M, Q, layer_views(gflat, w), [tau] * L, prec_code)
+    counts, per_step = [0] * L, []
+    try:
+        for i in range(warmup + steps):
+            gflat.copy_(seq[i])
+            plan.step(cd.hparams(step=t0 + i, gate_mode=gate_code, tau_global=tau))
+            if i < warmup:
+                continue
+            if gate_code == cd.DION_GATE_GLOBAL:
+                act = [bool(plan.global_flag[0].item())] * L
+            else:
+                act = plan.flags[:L].cpu().numpy().astype(bool).tolist()
+            per_step.append(int(sum(act)))
+            for l in range(L):
+                counts[l] += int(act[l])
+    finally:
+        plan.close()
+    return [c / steps for c in counts], per_step
 
 
 # ---------------------------------------------------------------------------- clocks ---
@@ -193,23 +270,36 @@ def run_ours(args, rank, world, local_rank):
     prec = args.precision
     gdt = torch.bfloat16 if w.g_dtype == "bf16" else torch.float32
 
-    X, M, Q, G = [], [], [], []
+    # Gated runs follow the workload's gradient sequence G_t (the branch each layer takes depends
+    # on it); every layer's G is a view of one flat buffer, and step t's gradients are copied into
+    # it before the step, outside the step's timed interval.  With DION_GATE_ALWAYS every layer
+    # does the same work whatever G holds, so G_1 stays in place and the steps run back to back.
+    grad_seq = args.gate != "always"
+    X, M, Q = [], [], []
     for l in range(w.num_layers):
         x0, m0, q0 = wl.init_layer(w, l, dev)
         X.append(x0); M.append(m0); Q.append(q0)
-        G.append(wl.gradient(w, l, 1, dev))
+    seq = make_gradient_sequence(wl, w, gdt, dev, range(args.t0, args.t0 + (args.warmup + args.steps if grad_seq
+                                                                              else 1)))
+    gflat = seq[0].clone() if grad_seq else seq.pop()
+    G = layer_views(gflat, w)
     torch.cuda.synchronize()
     plan = cd.Plan(X, M, Q, G, [args.tau] * w.num_layers, PREC[prec])
     gate = {"always": cd.DION_GATE_ALWAYS, "global": cd.DION_GATE_GLOBAL, "per_layer": cd.DION_GATE_PER_LAYER}[args.gate]
     stream = torch.cuda.current_stream(dev)
-    t = 0
+    t = args.t0 - 1
 
     def one_step():
         nonlocal t
         t += 1
         plan.step(cd.hparams(step=t, gate_mode=gate, tau_global=args.tau), stream=stream.cuda_stream)
 
-    for _ in range(args.warmup):
+    def load_gradients(i):
+        if grad_seq:
+            gflat.copy_(seq[i], non_blocking=True)
+
+    for i in range(args.warmup):
+        load_gradients(i)
         one_step()
     torch.cuda.synchronize()
     if plan.device_status() != 0:
@@ -231,16 +321,24 @@ def run_ours(args, rank, world, local_rank):
 
         dist.barrier()
     torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        one_step()
-    e1.record(stream)
+    if grad_seq:  # one event pair per step; the gradient copies fall between them
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        for i in range(args.steps):
+            load_gradients(args.warmup + i)
+            evs[i][0].record(stream)
+            one_step()
+            evs[i][1].record(stream)
+    else:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            one_step()
+        e1.record(stream)
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
     clocks = sampler.stop() if sampler else None
-    ms_total = e0.elapsed_time(e1)
+    ms_total = sum(a.elapsed_time(b) for a, b in evs) if grad_seq else e0.elapsed_time(e1)
     nsteps_timed, ktimes = cd.native.dion_timing_read(plan.handle)
     cd.native.dion_timing_enable(plan.handle, 0)
     ms_total = max_over_ranks(ms_total, world, dev)
@@ -290,11 +388,17 @@ def run_ours(args, rank, world, local_rank):
     plan.close()
     if rank != 0:
         return None
+    wt, sync_per_step = None, None
+    if grad_seq:
+        del X, M, Q, G, gflat, host_G
+        torch.cuda.empty_cache()
+        wt, sync_per_step = replay_sync_pattern(cd, wl, w, PREC[prec], gate, args.tau, args.t0, args.warmup,
+                                                args.steps, seq, dev)
 
     peaks = load_peaks()
     kern = []
     for name, ms in ktimes:
-        bound, units, unit = kernel_work(name, w, prec)
+        bound, units, unit = kernel_work(name, w, prec, args.gate, wt)
         kern.append(dict(name=name, ms=ms, bound=bound, units=units, unit=unit))
     dom = max(kern, key=lambda k: k["ms"]) if kern else None
     roofline = None
@@ -317,7 +421,7 @@ def run_ours(args, rank, world, local_rank):
         roofline = {"kernel": dom["name"], "bound": dom["bound"], "achieved": round(achieved, 2), "peak": peak,
                     "unit": punit, "frac": round(achieved / peak, 4), "traffic": traffic,
                     "peak_source": f"{peaks['source']} ({'sustained bf16' if dom['bound'] == 'tensor' else 'copy' if dom['bound'] == 'hbm' else 'derived'})"}
-    planned, compulsory = step_bytes(w, prec)
+    planned, compulsory = step_bytes(w, prec, args.gate, wt)
     line = {
         "metric": METRIC, "value": round(ms_step, 4), "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_step, 4), "higher_is_better": False, "scaling": "weak",
@@ -326,12 +430,11 @@ def run_ours(args, rank, world, local_rank):
                    [list(s) for s in w.shapes[:6]], "gate_mode": args.gate, "precision": prec,
                    "l2": "no flush: each step streams far more than the 129 MB L2",
                    "matrices_per_s": round(world * w.num_layers / (ms_step * 1e-3), 1),
-                   # byte models of a step in which every layer syncs; a gated run takes the cheaper
-                   # local branch on most layers, so they are reported for --gate always only
-                   "step_hbm_frac_planned_bytes": round(planned / (ms_step * 1e-3) / 1e9 / peaks["hbm"], 4)
-                   if args.gate == "always" else None,
-                   "step_hbm_frac_compulsory_bytes": round(compulsory / (ms_step * 1e-3) / 1e9 / peaks["hbm"], 4)
-                   if args.gate == "always" else None,
+                   # byte models of the step with each layer's branch as taken in the timed steps
+                   "step_hbm_frac_planned_bytes": round(planned / (ms_step * 1e-3) / 1e9 / peaks["hbm"], 4),
+                   "step_hbm_frac_compulsory_bytes": round(compulsory / (ms_step * 1e-3) / 1e9 / peaks["hbm"], 4),
+                   "sync_rate": 1.0 if wt is None else round(sum(wt) / len(wt), 4),
+                   "synced_layers_per_step": sync_per_step,
                    "parallelism": f"replicas x{world}"},
         "roofline": roofline,
         "e2e": {"value": round(e2e_ms, 4), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
@@ -411,6 +514,8 @@ def main():
     ap.add_argument("--precision", default=None, choices=list(PREC))
     ap.add_argument("--gate", default="always", choices=["always", "global", "per_layer"])
     ap.add_argument("--tau", type=float, default=0.5)
+    ap.add_argument("--t0", type=int, default=1, help="index of the first (warm-up) step: gradients G_t and "
+                    "the step number t start there")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
