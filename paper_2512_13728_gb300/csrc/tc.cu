@@ -540,16 +540,20 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   const uint32_t o_parts = (uint32_t)std::max(1, ((lo.max_r + 15) / 16 * 16 + 255) / 256);
   const uint32_t ostage = 128u * 32u * 4u * (1u + o_parts);
   const int ostages = (int)std::min<uint32_t>(4u, budget / ostage);
-  if (stages < 2 || ostages < 2) return cudaErrorInvalidValue;
+  // TRSM: one 256-column part per sub-tile, so a stage holds the A box and one B box
+  const uint32_t tstage = 128u * 32u * 4u * 2u;
+  const int tstages = (int)std::min<uint32_t>(4u, budget / tstage);
+  if (stages < 2 || ostages < 2 || tstages < 2) return cudaErrorInvalidValue;
   tp->nb64 = nb64;
   tp->bq_boxes = bq_boxes;
   tp->nb128 = nb128;
   tp->o_parts = o_parts;
   tp->f_stages = tp->r_stages = stages;
   tp->o_stages = ostages;
+  tp->t_stages = tstages;
   tp->f_smem = form_bq_smem(stages, stage);
   tp->r_smem = btp_smem(stages, stage);
-  tp->o_smem = orth_smem(ostages, ostage);
+  tp->o_smem = std::max(orth_smem(ostages, ostage), orth_smem(tstages, tstage));
   uint32_t cols = 32;
   while (cols < (uint32_t)((lo.max_r + 15) / 16 * 16)) cols <<= 1;
   tp->tmem_cols = cols;

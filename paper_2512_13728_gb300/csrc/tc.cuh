@@ -83,7 +83,7 @@ struct TcPlan {
   int4 *trsm_tiles = nullptr;
   int32_t n_trsm_tiles = 0;
   int32_t max_r = 0;
-  int32_t f_stages = 0, r_stages = 0, o_stages = 0;
+  int32_t f_stages = 0, r_stages = 0, o_stages = 0, t_stages = 0;  // t: the TRSM's (A + one B box per stage)
   uint32_t f_smem = 0, r_smem = 0, o_smem = 0, nb64 = 0, nb128 = 0, bq_boxes = 0, o_parts = 0, tmem_cols = 0;
   int32_t num_sms = 0;
   int32_t precision = 0;

@@ -10,6 +10,10 @@
 //          (K-major), B = rows of L^{-1} (K-major, lower triangular: K chunks above a column
 //          part are skipped).  Epilogue stores Y (row-major) and Y^T (transposed boxes) for
 //          the next pass, or, in the pass that ends Orthogonalize, only the bf16 copy of Y.
+//          A tile runs as one sub-tile per 256-column part of N, each accumulated in one of two
+//          alternating 256-column TMEM slots, so the epilogue of one sub-tile (the stores that
+//          bound the solve) runs under the MMAs of the next; part 1 reads A chunks 0..7 a
+//          second time, from L2.
 //
 // Accuracy: tf32 products (10-bit mantissa) with fp32 accumulation give ~5e-4 relative
 // error in S and Y; the second CholeskyQR pass (on an already nearly orthonormal X) brings
@@ -90,7 +94,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
   uint8_t *stg = smem + nstages * stage_bytes;  // 2 x (row box 16 KB + 4 transposed boxes 16 KB)
   uint64_t *bars = reinterpret_cast<uint64_t *>(stg + 4 * O_BOX);
   uint64_t *full = bars, *empty = bars + nstages;
-  uint64_t *acc_full = bars + 2 * nstages, *acc_empty = acc_full + 1, *drain = acc_full + 2;
+  // two accumulator slots (the TRSM alternates them; the Gram uses slot 0)
+  uint64_t *acc_full = bars + 2 * nstages, *acc_empty = acc_full + 2, *drain = acc_full + 4;
   __shared__ uint32_t tmem_base_s;
   __shared__ int abort_s;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -102,8 +107,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
       mbar_init(&full[i], 1);   // used in CTA 0: its arm, both CTAs' bytes
       mbar_init(&empty[i], 1);  // pair commit after the stage's MMAs
     }
-    mbar_init(acc_full, 1);   // pair commit after the tile's MMAs
-    mbar_init(acc_empty, 2);  // used in CTA 0: one arrival per CTA's epilogue
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&acc_full[i], 1);   // pair commit after the (sub-)tile's MMAs
+      mbar_init(&acc_empty[i], 2);  // used in CTA 0: one arrival per CTA's epilogue
+    }
     mbar_init(drain, 1);
     abort_s = 0;
     fence_mbar_init();
@@ -136,6 +143,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
         const int kch = (int)((K + 31) / 32);
         const uint32_t nparts = (N + 255) / 256;
         const int tr = 2 * t.y + (int)rank;  // past the last tile: zero-filled, not stored
+        if constexpr (KIND == ORTH_TRSM) {
+          // sub-tile q: K chunks below 256 (q + 1); A chunk and part q's B box in each stage
+          for (uint32_t q = 0; q < nparts && ok; ++q) {
+            const int kq = min(kch, (int)(8u * (q + 1u)));
+            for (int kc = 0; kc < kq; ++kc, ++it) {
+              const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
+              if (!ab.wait(&empty[s], ph ^ 1u, sh.status)) { ok = false; break; }
+              uint8_t *sA = smem + s * stage_bytes, *sB = sA + O_BOX;
+              const uint32_t fb = cluster_addr(&full[s], 0);
+              if (rank == 0) mbar_expect_tx(&full[s], 2u * O_BOX * 2u);
+              tma_load_2d_pair(sA, om.A, fb, kc * 32, tr * 128);
+              tma_load_2d_pair(sB, om.B, fb, kc * 32, (int)(q * 256u + rank * half_rows(N, q)));
+            }
+          }
+          continue;
+        }
         const bool a_in_b = (KIND == ORTH_GRAM) && (uint32_t)t.y < nparts && half_rows(N, (uint32_t)t.y) == 128u;
         for (int kc = 0; kc < kch; ++kc, ++it) {
           const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
@@ -169,6 +192,30 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
         orth_dims<KIND>(L, t.y, N, K);
         const int kch = (int)((K + 31) / 32);
         const uint32_t nparts = (N + 255) / 256;
+        if constexpr (KIND == ORTH_TRSM) {
+          for (uint32_t q = 0; q < nparts && ok; ++q) {
+            const uint32_t slot = tcount & 1u;  // tcount counts sub-tiles here
+            if (!ab.wait(&acc_empty[slot], ((tcount >> 1) & 1u) ^ 1u, sh.status)) { ok = false; break; }
+            tc_fence_after();
+            const int kq = min(kch, (int)(8u * (q + 1u)));
+            for (int kc = 0; kc < kq; ++kc, ++it) {
+              const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
+              if (!ab.wait(&full[s], ph, sh.status)) { ok = false; break; }
+              tc_fence_after();
+              const uint32_t aB = smem_u32(smem + s * stage_bytes), bB = aB + O_BOX;
+#pragma unroll
+              for (int k8 = 0; k8 < 4; ++k8)
+                umma_pair_tf32(tmem + slot * 256u, smem_desc_sw128(aB + k8 * 32, 0, 1024),
+                               smem_desc_sw128(bB + k8 * 32, 0, 1024), idesc_tf32(256, 2u * half_rows(N, q), false, false),
+                               (kc | k8) ? 1u : 0u);
+              umma_pair_commit_mc(&empty[s], 0x3);  // the stage is free in both CTAs
+            }
+            if (!ok) break;
+            umma_pair_commit_mc(&acc_full[slot], 0x3);
+            ++tcount;
+          }
+          continue;
+        }
         const bool a_in_b = (KIND == ORTH_GRAM) && (uint32_t)t.y < nparts && half_rows(N, (uint32_t)t.y) == 128u;
         if (!ab.wait(acc_empty, (tcount & 1u) ^ 1u, sh.status)) break;
         tc_fence_after();
@@ -212,87 +259,102 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
       int64_t K;
       orth_dims<KIND>(L, t.y, N, K);
       const int tr = 2 * t.y + (int)rank;
-      if (!named_and(1, 128, ab.wait(acc_full, tcount & 1u, sh.status))) break;
-      tc_fence_after();
       const bool real = (int64_t)tr * 128 < (KIND == ORTH_GRAM ? L.r : L.m);  // not the pair's empty second tile
       const int nch = real ? (int)((min((int64_t)N, L.r) + 31) / 32) : 0;
       // The solve that ends Orthogonalize writes only the bf16 copy of P that R = B^T P and the
       // update read: pass 1 unless a shifted retry asked for pass 2, and pass 2 itself.
       const bool final_pass = (KIND == ORTH_TRSM) && (pass == 2 || (pass == 1 && !sh.orth_shifted[t.x]));
-      if (final_pass) {
-        for (int j = 0; j < nch; j += 2) {  // two 32-column chunks per 64-column bf16 box
-          const uint32_t eb = ecount & 1u;
-          uint8_t *hb = stg + eb * 2 * O_BOX;
-          if (leader) bulk_wait_read<1>();
-          named_sync(1, 128);
+      // the Gram drains its accumulator in one go; the TRSM one sub-tile (256-column part) at a
+      // time, from alternating slots (tcount counts sub-tiles there)
+      const uint32_t nsub = (KIND == ORTH_TRSM) ? (N + 255) / 256 : 1u;
+      bool stop = false;
+      for (uint32_t q = 0; q < nsub; ++q) {
+        const uint32_t slot = (KIND == ORTH_TRSM) ? (tcount & 1u) : 0u;
+        const uint32_t aph = (KIND == ORTH_TRSM) ? ((tcount >> 1) & 1u) : (tcount & 1u);
+        if (!named_and(1, 128, ab.wait(&acc_full[slot], aph, sh.status))) { stop = true; break; }
+        tc_fence_after();
+        // output chunks jb .. je - 1 (32 columns each); chunk j sits at TMEM column
+        // slot * 256 + 32 (j - jb)
+        const int jb = (KIND == ORTH_TRSM) ? (int)(8u * q) : 0;
+        const int je = (KIND == ORTH_TRSM) ? min(nch, jb + 8) : nch;
+        const uint32_t tcol = tmem + slot * 256u + (lg * 32u << 16);
+        if (final_pass) {
+          for (int j = jb; j < je; j += 2) {  // two 32-column chunks per 64-column bf16 box
+            const uint32_t eb = ecount & 1u;
+            uint8_t *hb = stg + eb * 2 * O_BOX;
+            if (leader) bulk_wait_read<1>();
+            named_sync(1, 128);
 #pragma unroll 1
-          for (int h = 0; h < 2; ++h) {
-            if (j + h < nch) {
-              uint32_t v[32];
-              tmem_ld32(tmem + (lg * 32u << 16) + (j + h) * 32, v);
-              tmem_ld_wait();
+            for (int h = 0; h < 2; ++h) {
+              if (j + h < je) {
+                uint32_t v[32];
+                tmem_ld32(tcol + (uint32_t)(j + h - jb) * 32u, v);
+                tmem_ld_wait();
 #pragma unroll
-              for (int q = 0; q < 8; ++q) {
-                const __nv_bfloat162 a = __floats2bfloat162_rn(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]));
-                const __nv_bfloat162 b =
-                    __floats2bfloat162_rn(__uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
-                uint2 hv;
-                hv.x = *reinterpret_cast<const uint32_t *>(&a);
-                hv.y = *reinterpret_cast<const uint32_t *>(&b);
-                *reinterpret_cast<uint2 *>(hb + sw128_offset(row, (uint32_t)(h * 4 + (q >> 1))) + (q & 1) * 8) = hv;
+                for (int c4 = 0; c4 < 8; ++c4) {
+                  const __nv_bfloat162 a =
+                      __floats2bfloat162_rn(__uint_as_float(v[4 * c4]), __uint_as_float(v[4 * c4 + 1]));
+                  const __nv_bfloat162 b =
+                      __floats2bfloat162_rn(__uint_as_float(v[4 * c4 + 2]), __uint_as_float(v[4 * c4 + 3]));
+                  uint2 hv;
+                  hv.x = *reinterpret_cast<const uint32_t *>(&a);
+                  hv.y = *reinterpret_cast<const uint32_t *>(&b);
+                  *reinterpret_cast<uint2 *>(hb + sw128_offset(row, (uint32_t)(h * 4 + (c4 >> 1))) + (c4 & 1) * 8) = hv;
+                }
+              } else {  // a lone last chunk: the other half of the box (clipped by the store)
+#pragma unroll
+                for (int c4 = 4; c4 < 8; ++c4) *reinterpret_cast<uint4 *>(hb + sw128_offset(row, c4)) = make_uint4(0, 0, 0, 0);
               }
-            } else {  // a lone last chunk: the other half of the box (clipped by the store)
-#pragma unroll
-              for (int q = 4; q < 8; ++q) *reinterpret_cast<uint4 *>(hb + sw128_offset(row, q)) = make_uint4(0, 0, 0, 0);
             }
+            fence_async_smem();
+            named_sync(1, 128);
+            if (leader) {
+              tma_store_2d(&maps[t.x].P_hi, hb, j * 32, tr * 128);
+              bulk_commit();
+            }
+            ++ecount;
           }
-          fence_async_smem();
-          named_sync(1, 128);
-          if (leader) {
-            tma_store_2d(&maps[t.x].P_hi, hb, j * 32, tr * 128);
-            bulk_commit();
-          }
-          ++ecount;
-        }
-      } else {
-        for (int j = 0; j < nch; ++j) {
-          const bool store_t = (KIND == ORTH_TRSM);  // transposed copy: the next Gram's operand
-          const uint32_t eb = ecount & 1u;
-          uint8_t *box = stg + eb * 2 * O_BOX, *tbox = box + O_BOX + lg * O_TBOX;
-          if (leader) bulk_wait_read<1>();
-          named_sync(1, 128);
-          uint32_t v[32];
-          tmem_ld32(tmem + (lg * 32u << 16) + j * 32, v);
-          tmem_ld_wait();
+        } else {
+          for (int j = jb; j < je; ++j) {
+            const bool store_t = (KIND == ORTH_TRSM);  // transposed copy: the next Gram's operand
+            const uint32_t eb = ecount & 1u;
+            uint8_t *box = stg + eb * 2 * O_BOX, *tbox = box + O_BOX + lg * O_TBOX;
+            if (leader) bulk_wait_read<1>();
+            named_sync(1, 128);
+            uint32_t v[32];
+            tmem_ld32(tcol + (uint32_t)(j - jb) * 32u, v);
+            tmem_ld_wait();
 #pragma unroll
-          for (int q = 0; q < 8; ++q)
-            *reinterpret_cast<float4 *>(box + sw128_f32(row, q)) =
-                make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]), __uint_as_float(v[4 * q + 2]),
-                            __uint_as_float(v[4 * q + 3]));
-          if (store_t) {
-            // transposed 32 x 32 box of this warp's rows: box row c = output column j*32 + c
+            for (int c4 = 0; c4 < 8; ++c4)
+              *reinterpret_cast<float4 *>(box + sw128_f32(row, c4)) =
+                  make_float4(__uint_as_float(v[4 * c4]), __uint_as_float(v[4 * c4 + 1]),
+                              __uint_as_float(v[4 * c4 + 2]), __uint_as_float(v[4 * c4 + 3]));
+            if (store_t) {
+              // transposed 32 x 32 box of this warp's rows: box row c = output column j*32 + c
 #pragma unroll
-            for (int c = 0; c < 32; ++c)
-              *reinterpret_cast<float *>(tbox + c * 128 + ((((uint32_t)lane >> 2) ^ (c & 7)) << 4) + (lane & 3) * 4) =
-                  __uint_as_float(v[c]);
+              for (int c = 0; c < 32; ++c)
+                *reinterpret_cast<float *>(tbox + c * 128 + ((((uint32_t)lane >> 2) ^ (c & 7)) << 4) + (lane & 3) * 4) =
+                    __uint_as_float(v[c]);
+            }
+            fence_async_smem();
+            named_sync(1, 128);
+            if (leader) {
+              tma_store_2d(om.out, box, j * 32, tr * 128);
+              if (store_t)
+                for (int w4 = 0; w4 < 4; ++w4)
+                  if ((int64_t)tr * 128 + w4 * 32 < L.m)
+                    tma_store_2d(om.out_t, stg + eb * 2 * O_BOX + O_BOX + w4 * O_TBOX, tr * 128 + w4 * 32, j * 32);
+              bulk_commit();
+            }
+            ++ecount;
           }
-          fence_async_smem();
-          named_sync(1, 128);
-          if (leader) {
-            tma_store_2d(om.out, box, j * 32, tr * 128);
-            if (store_t)
-              for (int w4 = 0; w4 < 4; ++w4)
-                if ((int64_t)tr * 128 + w4 * 32 < L.m)
-                  tma_store_2d(om.out_t, stg + eb * 2 * O_BOX + O_BOX + w4 * O_TBOX, tr * 128 + w4 * 32, j * 32);
-            bulk_commit();
-          }
-          ++ecount;
         }
+        tc_fence_before();
+        named_sync(1, 128);  // every thread's TMEM reads of this accumulator slot are done
+        if (leader) mbar_arrive_cluster(cluster_addr(&acc_empty[slot], 0));
+        ++tcount;
       }
-      tc_fence_before();
-      named_sync(1, 128);  // every thread's TMEM reads of this accumulator are done
-      if (leader) mbar_arrive_cluster(cluster_addr(acc_empty, 0));
-      ++tcount;
+      if (stop) break;
     }
     if (leader) bulk_wait<0>();
   }
@@ -303,6 +365,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
   if (warp == 1) tmem_dealloc_pair(tmem, tmem_cols);
 }
 
+// alignment slack + operand stages + 2 staging buffers + barriers (2 x stages + 5 words)
 uint32_t orth_smem(int nstages, uint32_t stage_bytes) { return 1024u + nstages * stage_bytes + 4u * O_BOX + 512u; }
 
 cudaError_t setup_orth_kernels(uint32_t smem) {
@@ -320,9 +383,9 @@ void launch_orth(const Shared &sh, const TcPlan &tp, bool gram, int pass, cudaSt
   if (gram)
     tc_orth_kernel<ORTH_GRAM><<<2 * d.grid, O_THREADS, tp.o_smem, s>>>(sh, d.tiles, d.off, tp.maps, pass,
                                                                          tp.o_stages, stage, tp.tmem_cols);
-  else
+  else  // two 256-column accumulator slots
     tc_orth_kernel<ORTH_TRSM><<<2 * d.grid, O_THREADS, tp.o_smem, s>>>(sh, d.tiles, d.off, tp.maps, pass,
-                                                                         tp.o_stages, stage, tp.tmem_cols);
+                                                                         tp.t_stages, 2u * O_BOX, 512u);
 }
 
 }  // namespace tc

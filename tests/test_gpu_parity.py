@@ -201,6 +201,18 @@ def test_gate_modes_bf16():
                      taus=[0.5, 0.3, 0.9])
 
 
+@pytest.mark.parametrize("pad", [0, 3])
+def test_ragged_shapes_bf16_per_layer_gate(pad):
+    """Ragged shapes with bf16 gradients under the per-layer gate, layers forced local (tau 1e6),
+    forced to sync (tau 1e-6) or gated at 0.5: the norms pass writes B into M over ragged row
+    tails (and, with pad, next to NaN-filled row padding), then the fused buffer + B Q kernel and
+    the update read B from M; every step against the oracle."""
+    import paper_2512_13728_gb300 as cd
+
+    run_per_step(RAGGED, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_PER_LAYER, tau_global=0.5), RAGGED.steps,
+                 TOL_BF16, pad=pad, taus=[1e6, 1e-6, 0.5, 0.5, 1e-6, 1e6])
+
+
 @pytest.mark.parametrize("prec", ["bf16", "fp32"])
 def test_weight_decay_both_branches(prec):
     """Decoupled weight decay (Section 4's 0.01, here 0.5 so that it is visible against the
