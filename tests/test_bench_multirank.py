@@ -40,7 +40,7 @@ def _rank_main(rank, world, port, values, out):
 def test_max_over_ranks_gloo_world2():
     world, port = 2, _free_port()
     values = [3.25, 7.5]
-    with mp.Manager() as mgr:
+    with mp.get_context("spawn").Manager() as mgr:  # no fork of a threaded process
         out = mgr.dict()
         mp.spawn(_rank_main, args=(world, port, values, out), nprocs=world, join=True)
         assert out[0] == out[1] == max(values)

@@ -91,7 +91,7 @@ def test_two_ranks_match_the_w_worker_emulation():
     import oracle.curvadion as oc
 
     world, port = 2, _free_port()
-    with mp.Manager() as mgr:
+    with mp.get_context("spawn").Manager() as mgr:  # no fork of a threaded process
         out = mgr.dict()
         mp.spawn(_rank_main, args=(world, port, out), nprocs=world, join=True)
         got = dict(out)
