@@ -189,6 +189,19 @@ def test_gpt160m_block_r192_bf16():
     print("bf16 block worst", worst)
 
 
+@pytest.mark.parametrize("rank", [300, 400])
+def test_rank_between_256_and_512_bf16(rank):
+    """256 < r < 512 in the tensor-core mode: the TRSM's second 256-column sub-tile is partial
+    (r = 400: 144 columns; r = 300, padded to 304: 48), and the Gram's second row block of S and
+    the B Q / B^T P accumulators are ragged too; ragged m and n over several tiles."""
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.scaled(wl.WORKLOADS["gpt160m_block_r192"], f"r{rank}", [(1200, 1100), (1100, 1200), (900, 700)],
+                  rank=rank, steps=3)
+    worst, _ = run_per_step(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_ALWAYS), w.steps, TOL_BF16)
+    print("rank", rank, "worst", worst)
+
+
 def test_gate_modes_bf16():
     """Gated modes on Gaussian gradients.  (The spiky low-rank stress workload makes kappa(P)
     reach ~1e2, where bf16 operands cannot meet 2e-2 on Q; it runs in the fp32-class modes.)"""
