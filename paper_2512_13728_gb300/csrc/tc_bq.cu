@@ -338,6 +338,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(R_THREADS, 1)
 //               wait until the staged stores have been read.
 // Separate rings keep each slot's turnaround short: an M slot waits for one load and one
 // conversion, an A slot for the load, conversion, MMA and store.
+// With `gated` (the gated modes) the norms pass has already written B into M, computed the
+// norms and run the gate: every role skips the layers that stay local, warp 0 loads no G (it
+// only marks the A slot full) and the converters round M itself and form no norms.
 constexpr int FB_MSTAGES = 3;  // M ring (2 x 16 KB per slot)
 constexpr int FB_ASTAGES = 4;  // G / A ring (16 KB per slot)
 constexpr int FB_QSTAGES = 2;  // Q ring (also the epilogue's staging)
