@@ -192,27 +192,47 @@ dion_status dion_timing_enable(dion_plan *plan, int32_t max_steps);
 dion_status dion_timing_read(dion_plan *plan, int32_t cap, float *ms_out, const char **names_out,
                              int32_t *count_out, int32_t *steps_out);
 
-/* Limits of dion_buffer_norms_noalloc (its fixed device scratch is ~1 MB per GPU). */
+/* Limits of dion_buffer_norms_noalloc.  Its fixed device scratch holds two doubles per tile,
+ * 1 MB per GPU; a tile is whole rows of about 64K elements of one layer. */
 #define DION_NOALLOC_MAX_LAYERS 256
 #define DION_NOALLOC_MAX_TILES 65536
 
-/* Buffer step without any allocation, for callers that cannot call cudaMalloc (a framework
- * whose allocator has reserved the device memory up front, or a latency-critical loop where
- * cudaMalloc/cudaFree would synchronize the device).  The paper has no counterpart: it is the
- * buffer line B = M + G (written back into M, as dion_step does) plus ||B|| and ||M_{t-1}||
- * per layer -- the inputs of Algorithm 2's RMMC -- without a plan.
- * Only m, n, M, ldm, G, ldg and g_dtype of each layer are used (same rules as dion_layer).
- * norm_b_out, norm_m_out: device double[num_layers], written.  Enqueued on `stream`.
- * Scratch: a fixed device array inside this library (layer table + per-tile partial sums),
- * held by every GPU that loads the library until the process exits.  Every call overwrites
- * what it reads, so nothing needs clearing, but calls that overlap on the GPU (two streams,
- * or two host threads) share that array and race: serialize them.  The first call on each
- * device looks up the array's device address (cudaGetSymbolAddress); make that first call
- * before any stream capture.  Allocates no device or host memory.
+/* The buffer step without any allocation.  The paper has no counterpart: this entry point is
+ * for callers that cannot call cudaMalloc -- a framework whose caching allocator has reserved
+ * the device memory up front and owns every byte of it, or a latency-critical loop in which a
+ * cudaMalloc or cudaFree would synchronize the device -- and so cannot hold a plan, whose
+ * workspace dion_plan_create allocates.
+ * For each layer it adds G into M in place (M = M + G, the buffer that dion_step forms) and
+ * writes two Frobenius norms: norm_b_out[l] = ||M + G|| (the new M) and norm_m_out[l] = ||M||
+ * (M as it was before the call).  Only m, n, M, ldm, G, ldg and g_dtype of each layer are used,
+ * with the same rules as in dion_layer.  norm_b_out, norm_m_out: device double[num_layers],
+ * written.  The work is enqueued on `stream` (a cudaStream_t; NULL = legacy default stream).
+ * Scratch: one fixed array of per-tile partial sums inside this library, in device memory,
+ * held by every GPU that loads the library until the process exits.  Every call shares it and
+ * it keeps the last call's contents; each call writes every slot it reads before reading it,
+ * so nothing needs clearing, but calls whose work overlaps on the GPU (two streams, or two host
+ * threads) race on it: serialize them.  The first call on a device (and the first after a
+ * cudaDeviceReset) looks up the array's device address with cudaGetSymbolAddress; make that
+ * first call before any stream capture.  The layer table is passed to the kernels as a kernel
+ * parameter, so no host-to-device copy is made.  No device or host memory is allocated.
  * Errors: INVALID_ARG, ALIGNMENT, UNSUPPORTED (num_layers > DION_NOALLOC_MAX_LAYERS, or the
- * layers need more than DION_NOALLOC_MAX_TILES tiles of ~64K elements), CUDA. */
+ * layers need more than DION_NOALLOC_MAX_TILES tiles; nothing is enqueued then), CUDA (the
+ * address lookup or a launch failed). */
 dion_status dion_buffer_norms_noalloc(const dion_layer *layers, int32_t num_layers, double *norm_b_out,
                                       double *norm_m_out, void *stream);
+
+/* Bounded device waits (failure detection; no counterpart in the paper).  Every wait of a
+ * tensor-core kernel on another role of the same CTA (a TMA load landing, an MMA finishing, an
+ * accumulator being drained) gives up after a limit, sets DION_ERR_TIMEOUT in the plan's status
+ * word and lets the kernel drain what it already issued and return; the step's later kernels
+ * still run, and the layers the kernel did not finish have unspecified outputs.
+ * dion_plan_set_wait_limit sets that limit, in nanoseconds, for the hand-off waits of the
+ * update kernel (error feedback and parameter update) of this plan; limit_ns <= 0 restores the
+ * default of 2 s.  The waits that drain copies and MMAs already in flight keep the default, so
+ * the kernel never exits with work in flight.  Meant for testing the timeout path: with a limit
+ * of a few nanoseconds the first wait that does not succeed at once gives up.  Host only;
+ * takes effect from the next dion_step.  Errors: INVALID_ARG (NULL plan). */
+dion_status dion_plan_set_wait_limit(dion_plan *plan, int64_t limit_ns);
 
 /* Frees the plan's workspace (synchronizes the device first).  NULL is a no-op. */
 void dion_plan_destroy(dion_plan *plan);

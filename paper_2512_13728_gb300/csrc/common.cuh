@@ -98,6 +98,8 @@ struct Shared {
   // gradients): the fused kernel and the update then read B from M without G, and the local
   // branch leaves M alone
   int32_t b_in_m;
+  // limit of the update kernel's hand-off waits between its roles (dion_plan_set_wait_limit)
+  uint64_t handoff_limit_ns;
 };
 
 // A contraction C = op(A) op(B) for the CUDA-core path.

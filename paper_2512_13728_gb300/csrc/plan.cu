@@ -79,6 +79,7 @@ void tick_end(dion_plan *p) {
 namespace {
 
 constexpr size_t kAlign = 256;
+constexpr uint64_t kDefaultWaitLimitNs = 2000000000ull;  // the bounded waits' default: 2 s
 
 struct Carver {
   size_t off = 0;
@@ -295,6 +296,7 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
   p->sh.status = reinterpret_cast<int32_t *>(base + o_status);
   p->sh.gate_scratch = reinterpret_cast<unsigned long long *>(base + o_gate);
   p->sh.orth_shifted = reinterpret_cast<uint8_t *>(base + o_shift);
+  p->sh.handoff_limit_ns = kDefaultWaitLimitNs;
   p->btiles = reinterpret_cast<int4 *>(base + o_bt);
   p->n_btiles = (int32_t)bt.size();
   p->utiles = reinterpret_cast<int4 *>(base + o_ut);
@@ -569,6 +571,12 @@ dion_status dion_get_device_status(dion_plan *p, int32_t clear, int32_t *code_ou
 }
 
 int32_t dion_step_launch_count(const dion_plan *p) { return p ? p->launches_per_step : 0; }
+
+dion_status dion_plan_set_wait_limit(dion_plan *p, int64_t limit_ns) {
+  if (!p) return DION_ERR_INVALID_ARG;
+  p->sh.handoff_limit_ns = limit_ns > 0 ? (uint64_t)limit_ns : kDefaultWaitLimitNs;
+  return DION_OK;
+}
 
 dion_status dion_plan_refresh(dion_plan *p, void *stream) {
   if (!p) return DION_ERR_INVALID_ARG;

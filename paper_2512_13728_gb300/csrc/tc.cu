@@ -3,8 +3,7 @@
 //
 // Error feedback + parameter update (Algorithm 1/2, sync branch):
 //   M = B - (1 - mu) P R^T,   X = X - eta sqrt(m/n) P Q_t^T
-// run as one persistent, warp-specialized kernel over 128 x 128 output tiles, in clusters of
-// two CTAs that share the R and Q_t chunks by multicast:
+// run as one persistent, warp-specialized kernel over 128 x 128 output tiles:
 //   warp 0      TMA producer: bf16 K-major chunks of P (A), R and Q_t (two B operands) into a
 //               3-stage shared-memory ring;
 //   warp 1      MMA issuer: two 128x128x16 tcgen05.mma per k-step into a double-buffered
@@ -27,10 +26,9 @@ void tick(dion_plan *p, cudaStream_t s, const char *name);
 namespace tc {
 
 // ============================================================ update (tcgen05) kernel ===
-// Clusters of two CTAs (one per SM) take row tiles 2 p and 2 p + 1 of the same column block:
-// the R and Q_t chunks are the same for both, so CTA 0 loads the R chunk and CTA 1 the Q_t
-// chunk and each multicasts it to the pair (half the L2 reads of those operands); each CTA's
-// MMA completion frees the stage in both CTAs.
+// CTAs 2 s and 2 s + 1 take row tiles 2 p and 2 p + 1 of the same column blocks in the same
+// order (schedule segment s), so the R and Q_t chunks one of them loads are usually still in L2
+// when the other asks for them.  Each CTA loads all three operand boxes of a stage itself.
 constexpr int U_STAGES = 3;
 constexpr uint32_t U_OPB = 128u * 64u * 2u;           // 128 x 64 bf16 operand box
 constexpr uint32_t U_STAGE = 3u * U_OPB;              // P, R, Q_t
@@ -44,7 +42,7 @@ constexpr int U_THREADS = 192;
 constexpr uint32_t U_IDESC = idesc_bf16(128, 128, false, false);
 
 // Tile = {layer, row-tile pair p, column tile, ||M_t|| slot of row tile 2 p}.
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
+__global__ void __launch_bounds__(U_THREADS, 1)
     tc_update_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off, const LayerMaps *__restrict__ maps,
                      float mu, float eta, float keep) {
   if (sh.gate_scratch[kScratchActive] == 0ull) return;  // no layer takes the Dion branch
@@ -60,14 +58,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
   __shared__ int abort_s;
   __shared__ double red_s[4];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const Abort ab{&abort_s};
-  const uint32_t rank = cluster_ctarank();
+  // hand-off waits between the roles use the plan's limit; the drains below keep the default
+  const Abort ab{&abort_s, sh.handoff_limit_ns};
+  const uint32_t rank = blockIdx.x & 1u;  // row tile 2 p + rank of the segment's tiles
   const int seg = blockIdx.x >> 1;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < U_STAGES; ++i) {
       mbar_init(&full[i], 1);
-      mbar_init(&empty[i], 2);  // the MMA commits of both CTAs of the pair
+      mbar_init(&empty[i], 1);  // this CTA's MMA commit
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
@@ -85,11 +84,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  cluster_sync();  // the peer's barriers are initialized before anything is multicast to them
   const uint32_t tmem = tmem_base_s;
 
   if (warp == 0) {
-    // ---------------------------------------------------------------- TMA producer (both CTAs)
+    // ---------------------------------------------------------------- TMA producer
     if (lane == 0) {
       uint32_t it = 0;
       bool ok = true;
@@ -105,16 +103,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
           uint8_t *sp = stage + s * U_STAGE;
           mbar_expect_tx(&full[s], U_STAGE);
           tma_load_2d(sp, &mp->P_hi, &full[s], kc * 64, mb * 128);
-          if (rank == 0) tma_load_2d_mc(sp + U_OPB, &mp->R_hi, &full[s], kc * 64, t.z * 128, 0x3);
-          else tma_load_2d_mc(sp + 2 * U_OPB, &mp->Qn_hi, &full[s], kc * 64, t.z * 128, 0x3);
+          tma_load_2d(sp + U_OPB, &mp->R_hi, &full[s], kc * 64, t.z * 128);
+          tma_load_2d(sp + 2 * U_OPB, &mp->Qn_hi, &full[s], kc * 64, t.z * 128);
         }
       }
-      // drain: every load into this CTA (its own and the peer's multicasts) has landed
+      // drain: every load this CTA issued has landed
       for (uint32_t k = (it > U_STAGES ? it - U_STAGES : 0); k < it; ++k)
         mbar_wait(&full[k % U_STAGES], (k / U_STAGES) & 1u, sh.status);
     }
   } else if (warp == 1) {
-    // ---------------------------------------------------------------- MMA issuer (each CTA)
+    // ---------------------------------------------------------------- MMA issuer
     if (lane == 0) {
       uint32_t it = 0, tcount = 0;
       bool ok = true;
@@ -140,7 +138,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
             umma_bf16(d1, ad, rd, U_IDESC, acc);
             umma_bf16(d2, ad, qd, U_IDESC, acc);
           }
-          umma_commit_mc(&empty[s], 0x3);  // the stage is free in both CTAs
+          umma_commit(&empty[s]);  // the stage is free once its MMAs have read it
         }
         if (!ok) break;
         umma_commit(&acc_full[b]);
@@ -197,6 +195,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
     };
     if (leader) issue_upto(U_EBUF - 1);
     uint32_t tcount = 0;
+    uint32_t waited = 0;  // sub-chunks whose load this role has waited for, in order
     bool ok = true;
     for (int ti = off[seg]; ti < tend && ok; ++ti) {
       const int4 t = tiles[ti];
@@ -226,6 +225,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
             ok = false;
             break;
           }
+          waited = k + 1;
           uint8_t *bs = epi + eb * U_EBUF2;
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
@@ -282,15 +282,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(U_THREADS, 1)
     }
     if (leader) {
       bulk_wait<0>();
-      // loads issued but not consumed (only after an abort)
-      for (uint32_t k = ecount; k < issued; ++k) mbar_wait(&epi_full[k % U_EBUF], (k / U_EBUF) & 1u, sh.status);
+      // loads issued but not waited for (only after an abort): at most U_EBUF - 1 of them, in
+      // distinct buffers, so each wait is for the latest phase of its buffer
+      for (uint32_t k = waited; k < issued; ++k) mbar_wait(&epi_full[k % U_EBUF], (k / U_EBUF) & 1u, sh.status);
     }
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem, 512);
-  cluster_sync();  // nothing more is multicast to, or arrives at, a CTA that has exited
 }
 
 // ========================================================================= host side ===
@@ -372,7 +372,7 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
   }
   // per-tile cost ~ K-loop length (+ a constant for the epilogue), LPT over the SMs
 
-  // update: row-tile pairs (one per cluster of two CTAs); w = ||M_t|| slot of the pair's first tile
+  // update: row-tile pairs (one per two consecutive CTAs); w = ||M_t|| slot of the pair's first tile
   std::vector<int4> upairs;
   for (size_t i = 0; i < lo.utiles.size(); ++i) {
     const int4 &u = lo.utiles[i];

@@ -120,15 +120,6 @@ __device__ __forceinline__ void umma_commit(uint64_t *bar) {
                : "memory");
 }
 
-// Arrival on the barrier at `bar`'s shared-memory offset in every CTA of `mask` (this
-// cluster) once the MMAs issued so far by this thread have completed.
-__device__ __forceinline__ void umma_commit_mc(uint64_t *bar, uint16_t mask) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
-                   smem_u32(bar)),
-               "h"(mask)
-               : "memory");
-}
-
 // ----------------------------------------------------------------- CTA pairs (2-SM MMA) ---
 // A cluster of two CTAs can issue one tcgen05.mma over both SMs (cta_group::2): the even CTA
 // issues it; A = 128 rows from each CTA's shared memory (M = 256), B = half of the N rows
@@ -203,17 +194,6 @@ __device__ __forceinline__ uint32_t cluster_ctarank() {
 __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
-// TMA tile load delivered to `dst`'s shared-memory offset in every CTA of `mask`; each of
-// those CTAs' barriers at `bar`'s offset receives the bytes that land there.
-__device__ __forceinline__ void tma_load_2d_mc(void *dst, const CUtensorMap *map, uint64_t *bar, int32_t c0,
-                                               int32_t c1, uint16_t mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster [%0], [%1, {%3, "
-      "%4}], [%2], %5;" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "h"(mask)
-      : "memory");
-}
-
 // 32 lanes x 32 consecutive 32-bit columns: thread t of the warp gets TMEM lane
 // (32 * (warp % 4) + t), columns [col, col + 32).
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
@@ -339,14 +319,18 @@ bool encode_f32_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t 
 // promptly so the CTA can drain its in-flight copies, free TMEM and exit.
 struct Abort {
   int *flag;
+  uint64_t limit_ns = kWaitLimitNs;
   __device__ bool wait(uint64_t *bar, uint32_t parity, int32_t *status) const {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
+    // the clock is read every 256 tries at the default limit (each try may suspend the thread
+    // for a while), and on every try under a shortened one
+    const uint32_t every = limit_ns < kWaitLimitNs ? 0u : 255u;
     for (uint32_t i = 1;; ++i) {
       if (mbar_try_wait(bar, parity)) return true;
-      if ((i & 255u) == 0) {
+      if ((i & every) == 0) {
         if (*(volatile int *)flag) return false;
-        if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        if (globaltimer_ns() - t0 > limit_ns) {
           set_status(status, ST_TIMEOUT);
           *(volatile int *)flag = 1;
           return false;

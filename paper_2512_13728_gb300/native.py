@@ -38,7 +38,7 @@ DION_MAX_RANK = 512
 EXPORTED = ("dion_plan_create", "dion_step", "dion_get_device_status", "dion_plan_refresh", "dion_step_launch_count",
             "dion_timing_enable", "dion_timing_read", "dion_buffer_norms_noalloc", "dion_plan_destroy",
             "dion_status_string", "dion_abi_version", "dion_plan_enable_host_gradients", "dion_step_host",
-            "dion_lr_schedule", "dion_rank_for")
+            "dion_lr_schedule", "dion_rank_for", "dion_plan_set_wait_limit")
 
 DION_ABI_VERSION = 2
 DION_NOALLOC_MAX_LAYERS = 256
@@ -109,6 +109,8 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     lib.dion_timing_read.restype = C.c_int
     lib.dion_buffer_norms_noalloc.argtypes = [C.POINTER(dion_layer), C.c_int32, P, P, P]
     lib.dion_buffer_norms_noalloc.restype = C.c_int
+    lib.dion_plan_set_wait_limit.argtypes = [P, C.c_int64]
+    lib.dion_plan_set_wait_limit.restype = C.c_int
     lib.dion_plan_destroy.argtypes = [P]
     lib.dion_plan_destroy.restype = None
     lib.dion_status_string.argtypes = [C.c_int]
@@ -223,6 +225,13 @@ def dion_buffer_norms_noalloc(layers, norm_b_out: int, norm_m_out: int, stream: 
                                           C.c_void_p(stream) if stream else None)
     if st != DION_OK:
         raise DionError(st, "dion_buffer_norms_noalloc")
+
+
+def dion_plan_set_wait_limit(plan: int, limit_ns: int) -> None:
+    """Limit of the update kernel's hand-off waits (<= 0: the default of 2 s); a test hook."""
+    st = load().dion_plan_set_wait_limit(C.c_void_p(plan), int(limit_ns))
+    if st != DION_OK:
+        raise DionError(st, "dion_plan_set_wait_limit")
 
 
 def dion_plan_destroy(plan: int) -> None:

@@ -148,3 +148,9 @@ def test_rank_for_rejects_bad_arguments(lib):
     assert native.dion_rank_for(0, 5, 0.1) == 0
     assert native.dion_rank_for(5, 5, 0.0) == 0
     assert native.dion_rank_for(5, 5, 1.5) == 0
+
+
+def test_wait_limit_rejects_null_plan(lib):
+    from paper_2512_13728_gb300 import native
+
+    assert lib.dion_plan_set_wait_limit(None, C.c_int64(5)) == native.DION_ERR_INVALID_ARG

@@ -17,7 +17,9 @@ import torch
 pytestmark = pytest.mark.gpu
 
 RTOL = 1e-5  # the RMMC tolerance of the parity tests (fp32 partial sums folded into fp64)
-SHAPES = [(200, 136, "bf16"), (136, 200, "fp32"), (67, 33, "bf16"), (1, 5, "bf16"), (300, 1024, "bf16")]
+# (2048, 4096) is 128 tiles of 16 rows, so the reduction's lanes take several tiles each
+SHAPES = [(200, 136, "bf16"), (136, 200, "fp32"), (67, 33, "bf16"), (1, 5, "bf16"), (300, 1024, "bf16"),
+          (2048, 4096, "bf16")]
 
 
 @pytest.fixture(scope="module")
@@ -93,3 +95,13 @@ def test_noalloc_rejects_sizes_beyond_its_scratch(cd):
     st = lib.dion_buffer_norms_noalloc(too_many, cd.native.DION_NOALLOC_MAX_LAYERS + 1, C.c_void_p(nb.data_ptr()),
                                        C.c_void_p(nb.data_ptr()), None)
     assert st == cd.native.DION_ERR_UNSUPPORTED
+    # more tiles than the scratch holds: a 70000 x 65536 layer is 70000 one-row tiles.  The sizes
+    # are checked before any device work, so the small buffer behind the pointers is never read.
+    big = cd.native.dion_layer(m=70000, n=65536, r=1, X=0, ldx=0, M=M[0].data_ptr(), ldm=65536, Q=0, ldq=0,
+                               G=G[0].data_ptr(), ldg=65536, g_dtype=cd.DION_DTYPE_BF16, tau=0.0)
+    before = M[0].clone()
+    st = lib.dion_buffer_norms_noalloc((cd.native.dion_layer * 1)(big), 1, C.c_void_p(nb.data_ptr()),
+                                       C.c_void_p(nb.data_ptr()), None)
+    assert st == cd.native.DION_ERR_UNSUPPORTED
+    torch.cuda.synchronize()
+    assert torch.equal(M[0], before)
