@@ -47,7 +47,8 @@ def check_all_layer_flags(plan, taus, tau_global):
 def run_sampled(w, precision, hp_kw, steps, tol, sample, check_steps=None, taus=None):
     """Runs `steps` steps of the whole stack; at the steps in `check_steps` (all by default) the
     oracle takes one step of the sampled layers from the device state and the results are
-    compared.  Returns the worst errors seen."""
+    compared.  Returns the worst errors seen, the flag margins at the checked steps and, per step,
+    the number of layers that took the Dion branch."""
     import paper_2512_13728_gb300 as cd
 
     st = gu.make_state(w, taus=taus)
@@ -55,7 +56,8 @@ def run_sampled(w, precision, hp_kw, steps, tol, sample, check_steps=None, taus=
     plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, precision)
     hpo = gu.oracle_hp(**hp_kw)
     worst = dict(M=0.0, X=0.0, Q=0.0, rmmc=0.0, eq1=0.0)
-    margins = []
+    margins, synced = [], []
+    gm = hp_kw.get("gate_mode", oc.GATE_ALWAYS)
     try:
         for t in range(1, steps + 1):
             gu.write_gradients(st, t)
@@ -69,6 +71,12 @@ def run_sampled(w, precision, hp_kw, steps, tol, sample, check_steps=None, taus=
             torch.cuda.synchronize()
             assert plan.device_status() == 0
             check_all_layer_flags(plan, st.taus, hp_kw.get("tau_global", 0.5))
+            if gm == oc.GATE_PER_LAYER:
+                synced.append(int(plan.flags[:L].sum().item()))
+            elif gm == oc.GATE_GLOBAL:
+                synced.append(L * int(plan.global_flag[0].item()))
+            else:
+                synced.append(L)
             if not check:
                 continue
             want = oc.curvadion_step(lay, grads, prev[sample], hpo, t)
@@ -85,16 +93,19 @@ def run_sampled(w, precision, hp_kw, steps, tol, sample, check_steps=None, taus=
             worst["eq1"] = max(worst["eq1"], float(np.max(np.abs(eq1 - want.rmmc_eq1) /
                                                           np.maximum(np.abs(want.rmmc_eq1), 1.0))))
             taus = np.array([lay_i.tau for lay_i in lay])
-            margin = float(np.min(np.abs(want.rmmc - taus) / np.abs(taus)))
+            rel = np.abs(want.rmmc - taus) / np.abs(taus)
+            margin = float(np.min(rel))
             margins.append(margin)
-            if margin > 1e-4:  # a flag at a near-tie is reported, not asserted
-                assert np.array_equal(flags, want.flags), (t, flags, want.flags)
+            tie = rel <= 1e-4  # a flag at a near-tie is reported, not asserted
+            for i in np.nonzero(tie)[0]:
+                print(f"near-tie: step {t} layer {sample[i]} RMMC {want.rmmc[i]:.9g} tau {taus[i]:.9g}")
+            assert np.array_equal(flags[~tie], want.flags[~tie]), (t, flags, want.flags)
             assert worst["M"] <= tol and worst["X"] <= tol and worst["Q"] <= tol, (t, worst)
             assert worst["rmmc"] <= RMMC_RTOL, (t, worst)
             assert worst["eq1"] <= max(RMMC_RTOL, tol), (t, worst)
     finally:
         plan.close()
-    return worst, margins
+    return worst, margins, synced
 
 
 def blocks(w, ids, per=6):
@@ -103,15 +114,19 @@ def blocks(w, ids, per=6):
     return [b * per + k for b in ids for k in range(per)]
 
 
-def test_gpt1p3b_stack_r512_bf16_blocks_0_and_23():
-    """The bench workload (144 matrices, r = 512, bf16 gradients, every layer syncs): two steps
-    of the whole stack; blocks 0 and 23 (12 matrices) checked against the oracle each step."""
+def test_gpt1p3b_stack_r512_bf16_50_steps():
+    """The bench workload (144 matrices, r = 512, bf16 gradients, every layer syncs) over its
+    stated 50 steps: every step checks every layer's flags against its RMMC; at t = 1, 2, 25
+    and 50 blocks 0 and 23 (12 matrices) take an oracle step from the device state.  The flag
+    margin at the checked steps stays above 1e-4 (no near-tie)."""
     import paper_2512_13728_gb300 as cd
 
     w = wl.WORKLOADS["gpt1p3b_stack_r512"]
     sample = blocks(w, [0, 23])
-    worst, _ = run_sampled(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_ALWAYS), 2, TOL_BF16, sample)
-    print("1.3B stack sampled worst", worst)
+    worst, margins, _ = run_sampled(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_ALWAYS), w.steps, TOL_BF16,
+                                    sample, check_steps={1, 2, 25, 50})
+    print("1.3B stack, 50 steps, sampled worst", worst, "min margin", min(margins))
+    assert min(margins) > 1e-4
 
 
 def test_gpt1p3b_stack_r512_bf16_per_layer_gate_mixed():
@@ -124,33 +139,50 @@ def test_gpt1p3b_stack_r512_bf16_per_layer_gate_mixed():
     w = wl.WORKLOADS["gpt1p3b_stack_r512"]
     taus = [1e6 if l % 2 else 1e-6 for l in range(w.num_layers)]
     sample = blocks(w, [0, 23])
-    worst, _ = run_sampled(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_PER_LAYER, tau_global=0.5), 2, TOL_BF16,
-                           sample, taus=taus)
+    worst, _, _ = run_sampled(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_PER_LAYER, tau_global=0.5), 2,
+                              TOL_BF16, sample, taus=taus)
     print("1.3B stack per-layer mixed worst", worst)
 
 
 @pytest.mark.parametrize("name", ["gpt160m_stack_r192", "gpt160m_stack_r48"])
-def test_gpt160m_stack_bf16_drift(name):
-    """The 160M-shaped stack (72 matrices) with the drifting rank-8 component, r in {192, 48}:
-    four steps; blocks 0, 5 and 11 checked against the oracle each step."""
+def test_gpt160m_stack_bf16_drift_100_steps(name):
+    """The 160M-shaped stack (72 matrices) with the drifting rank-8 component, r in {192, 48},
+    over its stated 100 steps: every layer's flags every step; at t = 1, 2, 50, 99 and 100
+    blocks 0, 5 and 11 take an oracle step from the device state."""
     import paper_2512_13728_gb300 as cd
 
     w = wl.WORKLOADS[name]
     sample = blocks(w, [0, 5, 11])
-    worst, _ = run_sampled(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_ALWAYS), 4, TOL_BF16, sample)
-    print(name, "sampled worst", worst)
+    worst, margins, _ = run_sampled(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_ALWAYS), w.steps, TOL_BF16,
+                                    sample, check_steps={1, 2, 50, 99, 100})
+    print(name, "100 steps, sampled worst", worst, "min margin", min(margins))
+    assert min(margins) > 1e-4
 
 
-def test_gpt350m_gate_stress_per_layer_flags_fp32():
-    """The gate-stress stack (144 matrices, r = 256, flat then spiky curvature phases of 50
-    steps), per-layer gate: 53 steps across the first phase change.  Every step checks every
-    layer's flags against its RMMC and the global flag; at steps 1, 2, 50, 51, 52, 53 blocks 0
-    and 23 take an oracle step from the device state (flags bit-exact, state to 1e-4)."""
+def phase_boundaries(w):
+    """t = 1, 2, the last step of every phase and the first step of the next (50, 51, 100, 101,
+    ...), and the last step of the run."""
+    out = {1, 2, w.steps}
+    for t0 in range(w.phase_len, w.steps + 1, w.phase_len):
+        out |= {t0, t0 + 1}
+    return {t for t in out if t <= w.steps}
+
+
+@pytest.mark.parametrize("mode", ["per_layer", "global"])
+def test_gpt350m_gate_stress_300_steps_fp32(mode):
+    """The gate-stress stack (144 matrices, r = 256, flat and spiky curvature phases of 50 steps)
+    over its stated 300 steps in both gated modes: every step checks every layer's flag against
+    its RMMC and the global flag against their maximum; at t = 1, 2 and the first two steps of
+    every phase (and t = 300) blocks 0 and 23 take an oracle step from the device state, with
+    flags bit-exact and state to 1e-4.  Both branches occur."""
     import paper_2512_13728_gb300 as cd
 
     w = wl.WORKLOADS["gpt350m_gate_stress_r256"]
+    gm = oc.GATE_PER_LAYER if mode == "per_layer" else oc.GATE_GLOBAL
     sample = blocks(w, [0, 23])
-    worst, margins = run_sampled(w, cd.DION_PREC_FP32,
-                                 dict(gate_mode=oc.GATE_PER_LAYER, tau_global=0.5), 53, TOL_FP32, sample,
-                                 check_steps={1, 2, 50, 51, 52, 53})
-    print("gate stress sampled worst", worst, "min margin", min(margins) if margins else math.inf)
+    worst, margins, synced = run_sampled(w, cd.DION_PREC_FP32, dict(gate_mode=gm, tau_global=0.5), w.steps,
+                                         TOL_FP32, sample, check_steps=phase_boundaries(w))
+    print("gate stress", mode, "300 steps, sampled worst", worst, "min margin", min(margins))
+    print("synced layers per step", synced)
+    assert min(margins) > 1e-4
+    assert any(synced) and min(synced) < w.num_layers  # both branches are taken

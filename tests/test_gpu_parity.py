@@ -55,6 +55,8 @@ def run_per_step(w, precision, hp_kw, steps, tol, taus=None, pad=0, min_margin=1
                 if c.margin > min_margin:
                     assert c.flags_equal, f"step {t}: flags differ (margin {c.margin:.2e})"
                     assert c.gflag_equal, f"step {t}: global flag differs"
+                else:  # a near-tie is reported, not asserted
+                    print(f"near-tie at step {t}: margin {c.margin:.3e}")
             assert c.err_M <= tol and c.err_X <= tol and c.err_Q <= tol, (t, c.err_M, c.err_X, c.err_Q)
             # Algorithm 2's RMMC comes from ||B|| (an exact fp32 add in every mode); Equation 1's
             # from ||M_t||, which carries the mode's error on M
@@ -72,6 +74,46 @@ def test_fp32_256x512_r16_all_modes(mode):
 
     w = wl.WORKLOADS["fp32_256x512_r16"]
     run_per_step(w, cd.DION_PREC_FP32, dict(gate_mode=mode, period=3, mu=0.95, eta=0.01), w.steps, TOL_FP32)
+
+
+def run_trajectory(w, precision, hp_kw, tol):
+    """`w.steps` library steps and `w.steps` oracle steps from the same initial state and the same
+    gradients, each side on its own state (end-of-run parity): the flag sequences bit for bit
+    and the final X, M, Q to `tol`.  The oracle's trajectory barely amplifies a perturbation of
+    its start on these workloads (a 6e-8 change of Q_0 grows to 2e-7 in 10 steps), so the
+    comparison measures the library's own per-step error."""
+    import paper_2512_13728_gb300 as cd
+
+    st = gu.make_state(w)
+    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, precision)
+    hpo = gu.oracle_hp(**hp_kw)
+    layers, _, _ = gu.snapshot(st)
+    prev = np.zeros(w.num_layers)
+    try:
+        for t in range(1, w.steps + 1):
+            gu.write_gradients(st, t)
+            grads = [oc.as_f64(g) for g in st.G]
+            want = oc.curvadion_step(layers, grads, prev, hpo, t)
+            layers, prev = want.layers, want.prev_norm
+            plan.step(cd.hparams(step=t, **hp_kw))
+            torch.cuda.synchronize()
+            assert plan.device_status() == 0
+            assert np.array_equal(plan.flags[: w.num_layers].cpu().numpy().astype(bool), want.flags), t
+            assert bool(plan.global_flag[0].item()) == want.global_flag, t
+        err = {k: max(gu.rel_fro(oc.as_f64(getattr(st, k)[l]), getattr(layers[l], k)) for l in range(w.num_layers))
+               for k in ("X", "M", "Q")}
+        print("end of run", err)
+        assert max(err.values()) <= tol, err
+    finally:
+        plan.close()
+
+
+def test_fp32_256x512_r16_trajectory():
+    """The single fp32 matrix over its stated 10 steps, end-of-run state against the oracle's own
+    10-step trajectory (fp32 arithmetic, 1e-4)."""
+    import paper_2512_13728_gb300 as cd
+
+    run_trajectory(wl.WORKLOADS["fp32_256x512_r16"], cd.DION_PREC_FP32, dict(gate_mode=oc.GATE_PER_LAYER), TOL_FP32)
 
 
 # ------------------------------------------------- ragged shapes, several tiles ---
@@ -180,13 +222,14 @@ def test_ragged_shapes_bf16_fp32_gradients():
     run_per_step(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_ALWAYS), w.steps, TOL_BF16, pad=1)
 
 
-def test_gpt160m_block_r192_bf16():
+def test_gpt160m_block_r192_bf16_50_steps():
+    """One GPT-160M-shaped block (six matrices, r = 192, bf16 gradients) over its stated 50 steps,
+    every step against an oracle step from the device state."""
     import paper_2512_13728_gb300 as cd
 
-    w = wl.scaled(wl.WORKLOADS["gpt160m_block_r192"], "block", wl.WORKLOADS["gpt160m_block_r192"].shapes,
-                  steps=4)
+    w = wl.WORKLOADS["gpt160m_block_r192"]
     worst, _ = run_per_step(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_ALWAYS), w.steps, TOL_BF16)
-    print("bf16 block worst", worst)
+    print("bf16 block, 50 steps, worst", worst)
 
 
 @pytest.mark.parametrize("rank", [300, 400])
