@@ -80,7 +80,9 @@ def kernel_work(name: str, w, prec: str, gate: str = "always", wt=None):
     r3 = tot(lambda m, n, r: r ** 3)
     nr = tot(lambda m, n, r: n * r)
     mr = tot(lambda m, n, r: m * r)
-    bh = 2 if prec == "bf16" else 0  # the bf16 copy of B the tensor-core contractions read
+    # the bf16 copy of B the tensor-core contractions read (its two halves with split operands)
+    bh = {"bf16": 2, "bf16x3": 4}.get(prec, 0)
+    hl = 2 if prec == "bf16x3" else 1  # bf16 copies of P, R, Q: one, or a high and a low half
     # tensor-core mode with bf16 G: in DION_GATE_ALWAYS the buffer pass leaves M_{t-1} in place
     # and the update forms B = M + G itself (it reads G); in the gated modes the norms pass
     # writes B into M first, and neither the fused B Q kernel nor the update reads G
@@ -100,14 +102,15 @@ def kernel_work(name: str, w, prec: str, gate: str = "always", wt=None):
         # local layers: read X, G; write X (M already holds B)
         "local": ("hbm", mn_loc * (8 + gsz), "B"),
         # tensor-core path
-        "tc_bq": ("hbm", mn * 2 + nr * 2 + mr * 8, "B"),  # Bh, bf16 Q; P and P^T fp32
+        "tc_bq": ("hbm", mn * bh + nr * 2 * hl + mr * 8, "B"),  # Bh (and Bl), bf16 Q; P and P^T fp32
         # buffer pass fused into B Q (bf16 G): read M (and G unless B is already in M); write Bh,
         # P and P^T fp32
         "tc_form_bq": ("hbm", mn * (4 + (0 if b_in_m else gsz) + 2) + mr * 8, "B"),
         # gated modes: the norms pass reads M, G and writes B into M on every layer (and runs
         # the gate in its last block)
         "norms_gate": ("hbm", mn_all * (4 + gsz + 4), "B"),
-        "tc_btp": ("hbm", mn * 2 + mr * 2 + nr * 6, "B"),  # Bh, bf16 P; R fp32 and bf16
+        "tc_btp": ("hbm", mn * bh + mr * 2 * hl + nr * (4 + 2 * hl), "B"),  # Bh (Bl), bf16 P; R fp32, bf16
+        "split_p": ("hbm", mr * 8, "B"),  # read P fp32; write its two bf16 halves
         "tc_update": ("hbm", mn * (16 + (gsz if deferred else 0)), "B"),
         "tc_gram": ("tensor", 2 * mr2, "flop"),
         "tc_trsm": ("tensor", 2 * mr2, "flop"),
@@ -128,6 +131,8 @@ def step_bytes(w, prec, gate: str = "always", wt=None):
     fused = prec == "bf16" and w.g_dtype == "bf16"
     if prec == "fp32":  # form_b 12 (+4 with fp32 G), B Q and B^T P read B 4 + 4, update 16
         planned = mn_all * (4 + gsz + 4) + mn * (4 + 4 + 16)
+    elif prec == "bf16x3":  # form_b writes M, Bh, Bl; B Q and B^T P read both halves 4 + 4, update 16
+        planned = mn_all * (4 + gsz + 4 + 4) + mn * (4 + 4 + 16)
     elif fused and gate == "always":  # buffer pass fused with B Q 8, the Bh read of B^T P 2, update 18
         planned = mn_all * ((4 + gsz + 2) + 2 + (16 + gsz))
     elif fused:  # norms pass 10 on every layer; synced: fused B Q 6, Bh read 2, update 16

@@ -65,9 +65,13 @@ enum { DION_DTYPE_FP32 = 0, DION_DTYPE_BF16 = 1 };
 /* Arithmetic of the contractions (B Q, Gram, triangular solve, B^T P, P R^T, P Q^T).
  * Every mode accumulates in fp32 and keeps M, X, Q in fp32.
  *   DION_PREC_FP32   : fp32 operands on CUDA cores (FFMA).
- *   DION_PREC_BF16   : bf16 operands on tcgen05 tensor cores, fp32 accumulators in TMEM.
- *   DION_PREC_BF16X3 : tcgen05 with each fp32 operand split as hi + lo bf16 and three
- *                      products (hi*hi + hi*lo + lo*hi): fp32-class accuracy. */
+ *   DION_PREC_BF16   : bf16 operands on tcgen05 tensor cores, fp32 accumulators in TMEM; the
+ *                      Gram and triangular solve of Orthogonalize as tf32 on tensor cores.
+ *   DION_PREC_BF16X3 : B Q, B^T P, P R^T and P Q^T on tcgen05 with each operand split as a high
+ *                      and a low bf16 half (x ~ hi + lo, |x - hi - lo| <= 2^-18 |x|) and three
+ *                      products per step (hi*hi + hi*lo + lo*hi); Orthogonalize in fp32 on CUDA
+ *                      cores: fp32-class accuracy for ill-conditioned P.  Ranks up to 256
+ *                      (dion_plan_create returns DION_ERR_UNSUPPORTED above). */
 enum { DION_PREC_FP32 = 0, DION_PREC_BF16 = 1, DION_PREC_BF16X3 = 2 };
 
 /* Largest supported rank r (one 128 x r fp32 accumulator fills the 512 TMEM columns). */

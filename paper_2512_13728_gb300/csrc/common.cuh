@@ -53,6 +53,9 @@ struct DevLayer {
   __nv_bfloat16 *Qn_hi;  // n x r : Q (Q_{t-1} when a step starts, Q_t after a sync step)
   __nv_bfloat16 *Bh;     // m x n, pitch ldbh : B rounded to bf16
   int64_t ldbh;
+  // BF16X3 low halves (x - bf16(x), rounded to bf16), same layouts as the copies above; null
+  // in the other modes
+  __nv_bfloat16 *Bl, *P_lo, *R_lo, *Qn_lo;
   float *PT_raw, *PT;    // r x m, pitch ldmt : transposed copies of P_raw and P (tensor-core Gram)
   int64_t ldmt;
   double *colsq;         // [row tiles of R][ldp]: per-tile column sums of squares of R

@@ -61,6 +61,15 @@ __device__ void form_b_tile(const DevLayer &L, int64_t row0, int64_t nrows, floa
         hv.x = *reinterpret_cast<const uint32_t *>(&h01);
         hv.y = *reinterpret_cast<const uint32_t *>(&h23);
         *reinterpret_cast<uint2 *>(L.Bh + i * L.ldbh + 4 * c4) = hv;
+        if (L.Bl != nullptr) {  // BF16X3: the low half B - bf16(B), rounded to bf16
+          const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+          const __nv_bfloat162 l01 = __floats2bfloat162_rn(m.x - f01.x, m.y - f01.y);
+          const __nv_bfloat162 l23 = __floats2bfloat162_rn(m.z - f23.x, m.w - f23.y);
+          uint2 lv;
+          lv.x = *reinterpret_cast<const uint32_t *>(&l01);
+          lv.y = *reinterpret_cast<const uint32_t *>(&l23);
+          *reinterpret_cast<uint2 *>(L.Bl + i * L.ldbh + 4 * c4) = lv;
+        }
       }
     }
     for (int64_t c = 4 * n4 + threadIdx.x; c < n; c += kRowThreads) {
@@ -69,7 +78,11 @@ __device__ void form_b_tile(const DevLayer &L, int64_t row0, int64_t nrows, floa
       sm[0] = fmaf(mo, mo, sm[0]);
       sb[0] = fmaf(b, b, sb[0]);
       if (!HAS_BH || !L.b_deferred) Mrow[c] = b;
-      if (HAS_BH) L.Bh[i * L.ldbh + c] = __float2bfloat16_rn(b);
+      if (HAS_BH) {
+        const __nv_bfloat16 h = __float2bfloat16_rn(b);
+        L.Bh[i * L.ldbh + c] = h;
+        if (L.Bl != nullptr) L.Bl[i * L.ldbh + c] = __float2bfloat16_rn(b - __bfloat162float(h));
+      }
     }
   }
 }

@@ -29,28 +29,42 @@ namespace tc {
 // CTAs 2 s and 2 s + 1 take row tiles 2 p and 2 p + 1 of the same column blocks in the same
 // order (schedule segment s), so the R and Q_t chunks one of them loads are usually still in L2
 // when the other asks for them.  Each CTA loads all three operand boxes of a stage itself.
-constexpr int U_STAGES = 3;
 constexpr uint32_t U_OPB = 128u * 64u * 2u;           // 128 x 64 bf16 operand box
-constexpr uint32_t U_STAGE = 3u * U_OPB;              // P, R, Q_t
 constexpr uint32_t U_EBOX = 128u * 16u * 4u;          // one 128 x 16 fp32 box (64-byte swizzle)
 constexpr uint32_t U_GBOX = 128u * 16u * 2u;          // one 128 x 16 bf16 box of G (32-byte swizzle)
 constexpr uint32_t U_EBUF2 = 2u * U_EBOX + U_GBOX;     // M, X and G of one 16-column sub-chunk (20 KB)
-constexpr int U_EBUF = 4;                             // sub-chunk buffers of the epilogue
 static_assert(U_EBUF2 % 1024u == 0, "every box of a sub-chunk buffer stays 1024-byte aligned");
-constexpr uint32_t U_SMEM = 1024u + U_STAGES * U_STAGE + U_EBUF * U_EBUF2 + 256u;
 constexpr int U_THREADS = 192;
 constexpr uint32_t U_IDESC = idesc_bf16(128, 128, false, false);
+// Ring depths.  BF16: 3 stages of {P, R, Q_t} and 4 epilogue sub-chunk buffers of M, X and G.
+// BF16X3: each stage also holds the low halves of P, R and Q_t (P R^T = Ph Rh^T + Ph Rl^T +
+// Pl Rh^T, the same for P Q_t^T), and B is already in M (no G box), so 2 stages of 6 boxes and
+// 2 epilogue buffers of M and X fit in shared memory.
+template <bool X3>
+struct UpdCfg {
+  static constexpr int STAGES = X3 ? 2 : 3;
+  static constexpr uint32_t STAGE = (X3 ? 6u : 3u) * U_OPB;  // P, R, Q_t [, P_lo, R_lo, Q_lo]
+  static constexpr int EBUF = X3 ? 2 : 4;
+  static constexpr uint32_t EBUF2 = X3 ? 2u * U_EBOX : U_EBUF2;  // bytes of one sub-chunk buffer
+  static constexpr uint32_t SMEM = 1024u + STAGES * STAGE + EBUF * EBUF2 + 256u;
+};
+static_assert(UpdCfg<true>::SMEM <= 227u * 1024u && UpdCfg<false>::SMEM <= 227u * 1024u, "update smem");
 
 // Tile = {layer, row-tile pair p, column tile, ||M_t|| slot of row tile 2 p}.
+template <bool X3>
 __global__ void __launch_bounds__(U_THREADS, 1)
     tc_update_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off, const LayerMaps *__restrict__ maps,
                      float mu, float eta, float keep) {
+  constexpr int U_STAGES = UpdCfg<X3>::STAGES;
+  constexpr uint32_t U_STAGE = UpdCfg<X3>::STAGE;
+  constexpr int U_EBUF = UpdCfg<X3>::EBUF;
+  constexpr uint32_t U_EBUFB = UpdCfg<X3>::EBUF2;
   if (sh.gate_scratch[kScratchActive] == 0ull) return;  // no layer takes the Dion branch
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = align1024(smem_raw);
   uint8_t *stage = smem;
   uint8_t *epi = smem + U_STAGES * U_STAGE;
-  uint64_t *bars = reinterpret_cast<uint64_t *>(epi + U_EBUF * U_EBUF2);
+  uint64_t *bars = reinterpret_cast<uint64_t *>(epi + U_EBUF * U_EBUFB);
   uint64_t *full = bars, *empty = bars + U_STAGES;
   uint64_t *acc_full = bars + 2 * U_STAGES, *acc_empty = acc_full + 2, *epi_full = acc_empty + 2;
   uint64_t *drain = epi_full + U_EBUF;
@@ -105,6 +119,11 @@ __global__ void __launch_bounds__(U_THREADS, 1)
           tma_load_2d(sp, &mp->P_hi, &full[s], kc * 64, mb * 128);
           tma_load_2d(sp + U_OPB, &mp->R_hi, &full[s], kc * 64, t.z * 128);
           tma_load_2d(sp + 2 * U_OPB, &mp->Qn_hi, &full[s], kc * 64, t.z * 128);
+          if (X3) {
+            tma_load_2d(sp + 3 * U_OPB, &mp->P_lo, &full[s], kc * 64, mb * 128);
+            tma_load_2d(sp + 4 * U_OPB, &mp->R_lo, &full[s], kc * 64, t.z * 128);
+            tma_load_2d(sp + 5 * U_OPB, &mp->Qn_lo, &full[s], kc * 64, t.z * 128);
+          }
         }
       }
       // drain: every load this CTA issued has landed
@@ -137,6 +156,13 @@ __global__ void __launch_bounds__(U_THREADS, 1)
             const uint32_t acc = (kc | k16) ? 1u : 0u;
             umma_bf16(d1, ad, rd, U_IDESC, acc);
             umma_bf16(d2, ad, qd, U_IDESC, acc);
+            if (X3) {  // P R^T = Ph Rh^T + Ph Rl^T + Pl Rh^T, P Q_t^T likewise
+              const uint64_t adl = smem_desc_sw128(base + 3 * U_OPB + k16 * 32, 0, 1024);
+              umma_bf16(d1, ad, smem_desc_sw128(base + 4 * U_OPB + k16 * 32, 0, 1024), U_IDESC, 1u);
+              umma_bf16(d1, adl, rd, U_IDESC, 1u);
+              umma_bf16(d2, ad, smem_desc_sw128(base + 5 * U_OPB + k16 * 32, 0, 1024), U_IDESC, 1u);
+              umma_bf16(d2, adl, qd, U_IDESC, 1u);
+            }
           }
           umma_commit(&empty[s]);  // the stage is free once its MMAs have read it
         }
@@ -178,7 +204,7 @@ __global__ void __launch_bounds__(U_THREADS, 1)
         // the buffer's previous sub-chunk (issued - U_EBUF) was stored at least one sub-chunk
         // ago: at most the latest store group may still be reading shared memory
         if (issued >= U_EBUF) bulk_wait_read<1>();
-        uint8_t *bs = epi + eb * U_EBUF2;
+        uint8_t *bs = epi + eb * U_EBUFB;
         const int r0 = (2 * t.y + (int)rank) * 128, x0 = t.z * 128 + lj * 16;
         const bool defer = sh.layers[t.x].b_deferred != 0 && !sh.b_in_m;  // B = M + G is formed here
         mbar_expect_tx(&epi_full[eb], 2u * U_EBOX + (defer ? U_GBOX : 0u));
@@ -226,7 +252,7 @@ __global__ void __launch_bounds__(U_THREADS, 1)
             break;
           }
           waited = k + 1;
-          uint8_t *bs = epi + eb * U_EBUF2;
+          uint8_t *bs = epi + eb * U_EBUFB;
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const uint32_t o = sw64_f32(row, q);
@@ -328,7 +354,11 @@ Schedule lpt(const std::vector<int4> &tiles, const std::vector<double> &cost, in
 
 dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int num_sms, size_t start,
                    TcLayout *out) {
-  if (precision != DION_PREC_BF16) return DION_ERR_UNSUPPORTED;
+  if (precision != DION_PREC_BF16 && precision != DION_PREC_BF16X3) return DION_ERR_UNSUPPORTED;
+  const bool x3 = precision == DION_PREC_BF16X3;
+  // BF16X3 stages hold the low halves too: its operand rings fit shared memory up to r = 256
+  for (int32_t l = 0; x3 && l < L; ++l)
+    if (layers[l].r > 256) return DION_ERR_UNSUPPORTED;
   TcLayout &lo = *out;
   lo.precision = precision;
   size_t off = start;
@@ -346,6 +376,10 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
   lo.o_pt.resize(L);
   lo.o_colsq.resize(L);
   lo.o_colinv.resize(L);
+  lo.o_bl.assign(L, 0);
+  lo.o_plo.assign(L, 0);
+  lo.o_rlo.assign(L, 0);
+  lo.o_qnlo.assign(L, 0);
   for (int32_t l = 0; l < L; ++l) {
     const dion_layer &ly = layers[l];
     const int64_t ldp = (ly.r + 7) / 8 * 8, ldbh = (ly.n + 7) / 8 * 8;
@@ -354,6 +388,12 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
     lo.o_rhi[l] = take(ly.n * ldp * 2);
     lo.o_qnhi[l] = take(ly.n * ldp * 2);
     lo.o_bh[l] = take(ly.m * ldbh * 2);
+    if (x3) {
+      lo.o_bl[l] = take(ly.m * ldbh * 2);
+      lo.o_plo[l] = take(ly.m * ldp * 2);
+      lo.o_rlo[l] = take(ly.n * ldp * 2);
+      lo.o_qnlo[l] = take(ly.n * ldp * 2);
+    }
     const int64_t ldmt = (ly.m + 7) / 8 * 8;
     lo.o_ptraw[l] = take(ly.r * ldmt * 4);
     lo.o_pt[l] = take(ly.r * ldmt * 4);
@@ -408,7 +448,7 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
   lo.o_qtiles = take(sizeof(int4) * std::max<size_t>(lo.qtiles.size(), 1));
   lo.o_gtiles = take(sizeof(int4) * std::max<size_t>(lo.gram_tiles.size(), 1));
   lo.o_ttiles = take(sizeof(int4) * std::max<size_t>(lo.trsm_tiles.size(), 1));
-  lo.fuse_buffer = L > 0;
+  lo.fuse_buffer = L > 0 && !x3;  // BF16X3 forms B and its two bf16 halves in the buffer pass
   for (int32_t l = 0; l < L; ++l) lo.fuse_buffer = lo.fuse_buffer && layers[l].g_dtype == DION_DTYPE_BF16;
   lo.end = off;
   (void)num_sms;
@@ -428,7 +468,14 @@ void bind(const TcLayout &lo, char *base, DevLayer *dl, int32_t L, TcPlan *tp) {
     dl[l].colsq = reinterpret_cast<double *>(base + lo.o_colsq[l]);
     dl[l].colinv = reinterpret_cast<float *>(base + lo.o_colinv[l]);
     dl[l].rtile_cnt = (int32_t)((dl[l].n + 127) / 128);
-    dl[l].b_deferred = (dl[l].g_dtype == DT_BF16) ? 1 : 0;  // the update forms B = M + G itself
+    // the update forms B = M + G itself (BF16 mode with bf16 G); BF16X3 writes B into M
+    dl[l].b_deferred = (dl[l].g_dtype == DT_BF16 && lo.precision == DION_PREC_BF16) ? 1 : 0;
+    if (lo.precision == DION_PREC_BF16X3) {
+      dl[l].Bl = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_bl[l]);
+      dl[l].P_lo = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_plo[l]);
+      dl[l].R_lo = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_rlo[l]);
+      dl[l].Qn_lo = reinterpret_cast<__nv_bfloat16 *>(base + lo.o_qnlo[l]);
+    }
     dl[l].upart_off = -1;
   }
   if (lo.fuse_buffer) {  // the fused kernel writes one ||B||^2 / ||M_{t-1}||^2 slot per 128-row tile
@@ -505,7 +552,15 @@ cudaError_t encode_maps(const DevLayer *dl, int32_t L, LayerMaps *dst) {
                     encode_f32_2d(&m.PTraw_t, d.PT_raw, d.m, d.r, (uint64_t)d.ldmt * 4, 32, 32) &&
                     encode_f32_2d(&m.PT_t, d.PT, d.m, d.r, (uint64_t)d.ldmt * 4, 32, 32) &&
                     encode_f32_2d(&m.Sst, d.S, d.r, d.r, p32, 32, 128) &&
-                    encode_f32_2d(&m.Linv, d.Linv, d.r, d.r, p32, 32, 128);
+                    encode_f32_2d(&m.Linv, d.Linv, d.r, d.r, p32, 32, 128) &&
+                    (d.P_lo == nullptr ||
+                     (encode_bf16_2d(&m.P_lo, d.P_lo, d.r, d.m, p16, 64, 128) &&
+                      encode_bf16_2d(&m.R_lo, d.R_lo, d.r, d.n, p16, 64, 128) &&
+                      encode_bf16_2d(&m.Qn_lo, d.Qn_lo, d.r, d.n, p16, 64, 128) &&
+                      encode_bf16_2d(&m.Qn_lo_mn, d.Qn_lo, d.r, d.n, p16, 64, 64) &&
+                      encode_bf16_2d(&m.P_lo_mn, d.P_lo, d.r, d.m, p16, 64, 64) &&
+                      encode_bf16_2d(&m.Bl_mn, d.Bl, d.n, d.m, (uint64_t)d.ldbh * 2, 64, 64) &&
+                      encode_bf16_2d(&m.Bl_k, d.Bl, d.n, d.m, (uint64_t)d.ldbh * 2, 64, 128)));
     if (!ok) return cudaErrorInvalidValue;
   }
   return cudaMemcpy(dst, maps.data(), sizeof(LayerMaps) * maps.size(), cudaMemcpyHostToDevice);
@@ -529,11 +584,14 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
       e = cudaMemcpy(base + sc->o_off, sc->off.data(), sizeof(int) * sc->off.size(), cudaMemcpyHostToDevice);
   }
   // shared-memory budget: operand stages + 2 staging buffers of (128 x 32 + 4 x 32 x 32) fp32
-  const uint32_t budget = 227u * 1024u - 1024u - 4u * 128u * 32u * 4u - 512u - 256u;
+  // and 1 KB of column partials
+  const uint32_t budget = 227u * 1024u - 1024u - 4u * 128u * 32u * 4u - 1024u - 512u - 256u;
+  const bool x3 = lo.precision == DION_PREC_BF16X3;
   const uint32_t nb64 = (uint32_t)std::max(1, (lo.max_r + 63) / 64);
   // B Q / B^T P (CTA pairs): A tile + per 256-column part of N, this CTA's half (two 64-column boxes)
   const uint32_t bq_boxes = 2u * (uint32_t)std::max(1, ((lo.max_r + 15) / 16 * 16 + 255) / 256);
-  const uint32_t stage = 128u * 64u * 2u + bq_boxes * 64u * 64u * 2u;
+  // BF16X3: the high and low halves of both operands
+  const uint32_t stage = (x3 ? 2u : 1u) * (128u * 64u * 2u + bq_boxes * 64u * 64u * 2u);
   const int stages = (int)std::min<uint32_t>(4u, budget / stage);
   const uint32_t nb128 = (uint32_t)std::max(1, (lo.max_r + 127) / 128);
   // Gram / TRSM (CTA pairs): A box + per 256-column part of N, this CTA's half (one 128-row box)
@@ -558,8 +616,12 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   while (cols < (uint32_t)((lo.max_r + 15) / 16 * 16)) cols <<= 1;
   tp->tmem_cols = cols;
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(tc_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)U_SMEM);
-  if (e == cudaSuccess) e = setup_bq_kernels(tp->f_smem, tp->r_smem);
+    e = tp->precision == DION_PREC_BF16X3
+            ? cudaFuncSetAttribute(tc_update_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   (int)UpdCfg<true>::SMEM)
+            : cudaFuncSetAttribute(tc_update_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   (int)UpdCfg<false>::SMEM);
+  if (e == cudaSuccess) e = setup_bq_kernels(tp->f_smem, tp->r_smem, x3);
   tp->fb_smem = fused_bq_smem(bq_boxes);
   if (tp->fuse_buffer && tp->fb_smem > 227u * 1024u) return cudaErrorInvalidValue;
   if (e == cudaSuccess && tp->fuse_buffer) e = setup_fused_bq_kernel(tp->fb_smem);
@@ -568,7 +630,7 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   tp->num_sms = sms;
-  tp->launches = tp->fuse_buffer ? 17 : 18;
+  tp->launches = x3 ? 19 : tp->fuse_buffer ? 17 : 18;
   return e;
 }
 
@@ -592,23 +654,39 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh_in, const StepArgs &a
     launch_fused_bq(sh, tp, true, s);
     tick(p, s, "tc_form_bq");
   } else {
-    launch_form_b(sh, btiles, n_btiles, s);  // B = M + G (and its bf16 copy), ||B||, ||M_{t-1}||
+    launch_form_b(sh, btiles, n_btiles, s);  // B = M + G (and its bf16 copy or halves), ||B||, ||M_{t-1}||
     tick(p, s, "form_b");
     launch_gate(sh, a, s);
     tick(p, s, "gate");
     launch_form_bq(sh, tp, s);  // P = B Q_{t-1} on the layers that take the Dion branch
     tick(p, s, "tc_bq");
   }
-  static const char *kGram[3] = {"tc_gram0", "tc_gram1", "tc_gram2"};
   static const char *kChol[3] = {"chol_inv0", "chol_inv1", "chol_inv2"};
-  static const char *kTrsm[3] = {"tc_trsm0", "tc_trsm1", "tc_trsm2"};
-  for (int pass = 0; pass < 3; ++pass) {  // CholeskyQR2; the third pass only after a shifted retry
-    launch_orth(sh, tp, true, pass, s);  // S = X^T X
-    tick(p, s, kGram[pass]);
-    launch_chol_inv(sh, chol_smem, pass, 6e-2f, s);  // L, L^{-1}
-    tick(p, s, kChol[pass]);
-    launch_orth(sh, tp, false, pass, s);  // X L^{-T} and its transpose, or its bf16 copy at the end
-    tick(p, s, kTrsm[pass]);
+  if (tp.precision == DION_PREC_BF16X3) {
+    // fp32-class Orthogonalize: the CUDA-core Gram and solve of the FP32 mode (sets 1..6)
+    static const char *kGram[3] = {"gemm_gram0", "gemm_gram1", "gemm_gram2"};
+    static const char *kTrsm[3] = {"gemm_trsm0", "gemm_trsm1", "gemm_trsm2"};
+    for (int pass = 0; pass < 3; ++pass) {
+      launch_gemm(sh, tp.probs[1 + pass], tp.gtiles[1 + pass], tp.n_gtiles[1 + pass], s);  // S = X^T X
+      tick(p, s, kGram[pass]);
+      launch_chol_inv(sh, chol_smem, pass, 1e-3f, s);  // L, L^{-1}
+      tick(p, s, kChol[pass]);
+      launch_gemm(sh, tp.probs[4 + pass], tp.gtiles[4 + pass], tp.n_gtiles[4 + pass], s);  // X L^{-T}
+      tick(p, s, kTrsm[pass]);
+    }
+    launch_split_p(sh, tp, s);  // the bf16 halves of the orthonormal P
+    tick(p, s, "split_p");
+  } else {
+    static const char *kGram[3] = {"tc_gram0", "tc_gram1", "tc_gram2"};
+    static const char *kTrsm[3] = {"tc_trsm0", "tc_trsm1", "tc_trsm2"};
+    for (int pass = 0; pass < 3; ++pass) {  // CholeskyQR2; the third pass only after a shifted retry
+      launch_orth(sh, tp, true, pass, s);  // S = X^T X
+      tick(p, s, kGram[pass]);
+      launch_chol_inv(sh, chol_smem, pass, 6e-2f, s);  // L, L^{-1}
+      tick(p, s, kChol[pass]);
+      launch_orth(sh, tp, false, pass, s);  // X L^{-T} and its transpose, or its bf16 copy at the end
+      tick(p, s, kTrsm[pass]);
+    }
   }
   launch_btp(sh, tp, s);  // R = B^T P
   tick(p, s, "tc_btp");
@@ -616,9 +694,14 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh_in, const StepArgs &a
   tick(p, s, "colnorm_reduce");
   launch_colnorm_scale(sh, tp, s);  // Q_t = R diag(...), its bf16 copy
   tick(p, s, "colnorm_scale");
-  if (tp.d_update.grid > 0)
-    tc_update_kernel<<<2 * tp.d_update.grid, U_THREADS, U_SMEM, s>>>(sh, tp.d_update.tiles, tp.d_update.off, tp.maps,
-                                                                      a.mu, a.eta, a.keep_sync);
+  if (tp.d_update.grid > 0) {
+    if (tp.precision == DION_PREC_BF16X3)
+      tc_update_kernel<true><<<2 * tp.d_update.grid, U_THREADS, UpdCfg<true>::SMEM, s>>>(
+          sh, tp.d_update.tiles, tp.d_update.off, tp.maps, a.mu, a.eta, a.keep_sync);
+    else
+      tc_update_kernel<false><<<2 * tp.d_update.grid, U_THREADS, UpdCfg<false>::SMEM, s>>>(
+          sh, tp.d_update.tiles, tp.d_update.off, tp.maps, a.mu, a.eta, a.keep_sync);
+  }
   tick(p, s, "tc_update");
   launch_local(sh, btiles, n_btiles, a.eta_local, a.keep_local, s);
   tick(p, s, "local");

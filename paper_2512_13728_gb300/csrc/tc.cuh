@@ -35,6 +35,10 @@ struct LayerMaps {
   CUtensorMap PT_t;     // r x m fp32: box {32, 32}  transposed output store
   CUtensorMap Sst;    // r x r fp32:  box {32, 128}  Gram output
   CUtensorMap Linv;   // r x r fp32:  box {32, 128}  TRSM B operand (rows of L^{-1})
+  // BF16X3: the low halves, boxes as their high counterparts (zeroed maps in the other modes)
+  CUtensorMap P_lo, R_lo, Qn_lo;  // K-major {64, 128}: update operands
+  CUtensorMap Qn_lo_mn, P_lo_mn, Bl_mn;  // MN-major {64, 64}: B Q / B^T P operands
+  CUtensorMap Bl_k;   // K-major {64, 128}: B Q A operand
 };
 
 // Tiles of one persistent kernel, reordered so that CTA b processes tiles [off[b], off[b+1]).
@@ -51,6 +55,7 @@ struct TcLayout {
   size_t o_maps = 0;
   size_t o_utiles = 0, o_ftiles = 0, o_rtiles = 0, o_qtiles = 0, o_gtiles = 0, o_ttiles = 0;
   std::vector<size_t> o_phi, o_rhi, o_qnhi, o_bh, o_ptraw, o_pt, o_colsq, o_colinv;
+  std::vector<size_t> o_bl, o_plo, o_rlo, o_qnlo;  // BF16X3 low halves
   std::vector<int4> gram_tiles, trsm_tiles;
   // update tiles {layer, m-block, n-block, slot}; P-convert tiles {layer, row0, rows, 0};
   // B Q tiles {layer, m-block, 0, slot}; B^T P tiles {layer, n-block, 0, 0}; Q-copy tiles

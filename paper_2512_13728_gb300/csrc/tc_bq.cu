@@ -23,6 +23,8 @@ namespace tc {
 constexpr uint32_t OPB_A = 128u * 64u * 2u;   // 128 x 64 bf16 A-operand tile (16 KB)
 constexpr uint32_t BOX64 = 64u * 64u * 2u;    // 64 x 64 bf16 MN-major box (8 KB)
 constexpr uint32_t EPI_BOX = 128u * 32u * 4u; // 128 x 32 fp32 output box (16 KB)
+// epilogue staging of the GEMM kernels: 4 boxes + 1 KB of column partials (R = B^T P)
+constexpr uint32_t STG_BYTES = 4u * EPI_BOX + 1024u;
 
 __device__ __forceinline__ uint32_t rpad16(int64_t r) { return (uint32_t)((r + 15) / 16 * 16); }
 
@@ -80,14 +82,16 @@ __device__ __forceinline__ void store_accumulator(uint32_t tmem, int warp, int l
 // Epilogue of R = B^T P for one 128-row tile of R: the fp32 rows of R and their bf16 copy
 // (TMA stores) and, per column, the tile's fp64 sum of squares for ColumnNormalize.
 // Two 32-column chunks are handled together so the bf16 box is one 64-column SW128 box.
+template <bool X3>
 __device__ __forceinline__ void store_r_tile(uint32_t tmem, int warp, int lane, bool leader, uint8_t *stg,
                                              const LayerMaps &mp, const DevLayer &L, int tile, uint32_t &ecount) {
   const uint32_t lg = (uint32_t)(warp & 3), row = 32u * lg + lane;
   const int et = (warp - 2) * 32 + lane;  // 0..127 within the epilogue warps (warps 2..5)
   const int nch = (int)((L.r + 31) / 32), row0 = tile * 128;
-  // staging: [fp32 box 16 KB][fp32 box 16 KB][bf16 box 16 KB] + column-partial scratch 4 x 64 floats
-  uint8_t *f0 = stg, *f1 = stg + EPI_BOX, *hb = stg + 2 * EPI_BOX;
-  float *red = reinterpret_cast<float *>(stg + 3 * EPI_BOX);
+  // staging: [fp32 box 16 KB][fp32 box 16 KB][bf16 box 16 KB][bf16 low-half box 16 KB (BF16X3)]
+  // + column-partial scratch 2 x 128 floats
+  uint8_t *f0 = stg, *f1 = stg + EPI_BOX, *hb = stg + 2 * EPI_BOX, *lb = stg + 3 * EPI_BOX;
+  float *red = reinterpret_cast<float *>(stg + 4 * EPI_BOX);
   for (int j = 0; j < nch; j += 2) {
     const bool two = (j + 1 < nch);
     if (leader) bulk_wait_read<0>();
@@ -109,12 +113,27 @@ __device__ __forceinline__ void store_r_tile(uint32_t tmem, int warp, int lane, 
         hv.x = *reinterpret_cast<const uint32_t *>(&a);
         hv.y = *reinterpret_cast<const uint32_t *>(&b);
         // bf16 64-column box: columns h*32 + 4q .. live in 16-byte chunk (h*4 + q/2)
-        *reinterpret_cast<uint2 *>(hb + sw128_offset(row, (uint32_t)(h * 4 + (q >> 1))) + (q & 1) * 8) = hv;
+        const uint32_t bo = sw128_offset(row, (uint32_t)(h * 4 + (q >> 1))) + (q & 1) * 8;
+        *reinterpret_cast<uint2 *>(hb + bo) = hv;
+        if (X3) {  // low halves: x - bf16(x), rounded to bf16
+          const float2 af = __bfloat1622float2(a), bf = __bfloat1622float2(b);
+          const __nv_bfloat162 al = __floats2bfloat162_rn(__uint_as_float(v[4 * q]) - af.x,
+                                                          __uint_as_float(v[4 * q + 1]) - af.y);
+          const __nv_bfloat162 bl = __floats2bfloat162_rn(__uint_as_float(v[4 * q + 2]) - bf.x,
+                                                          __uint_as_float(v[4 * q + 3]) - bf.y);
+          uint2 lv;
+          lv.x = *reinterpret_cast<const uint32_t *>(&al);
+          lv.y = *reinterpret_cast<const uint32_t *>(&bl);
+          *reinterpret_cast<uint2 *>(lb + bo) = lv;
+        }
       }
     }
     if (!two) {  // a lone last chunk: zero the unused half of the bf16 box (clipped by the store anyway)
 #pragma unroll
-      for (int q = 4; q < 8; ++q) *reinterpret_cast<uint4 *>(hb + sw128_offset(row, q)) = make_uint4(0, 0, 0, 0);
+      for (int q = 4; q < 8; ++q) {
+        *reinterpret_cast<uint4 *>(hb + sw128_offset(row, q)) = make_uint4(0, 0, 0, 0);
+        if (X3) *reinterpret_cast<uint4 *>(lb + sw128_offset(row, q)) = make_uint4(0, 0, 0, 0);
+      }
     }
     fence_async_smem();
     named_sync(1, 128);
@@ -122,6 +141,7 @@ __device__ __forceinline__ void store_r_tile(uint32_t tmem, int warp, int lane, 
       tma_store_2d(&mp.Rst, f0, j * 32, row0);
       if (two) tma_store_2d(&mp.Rst, f1, (j + 1) * 32, row0);
       tma_store_2d(&mp.R_hi, hb, j * 32, row0);
+      if (X3) tma_store_2d(&mp.R_lo, lb, j * 32, row0);
       bulk_commit();
     }
     // column sums of squares: thread et sums column (et % 32) of chunk j + h over rows (et / 32) * 32 ..
@@ -167,7 +187,10 @@ enum : int { GEMM_BQ = 0, GEMM_BTP = 1 };
 // to 256 columns, the half c of its B columns, and receives its 128 rows of the accumulator
 // in its own TMEM.  Per SM and k-chunk that is 16 KB of A and 32 KB of B (r = 512) instead of
 // 16 + 64 KB.  Tile = {layer, pair p}.
-template <int KIND>
+// X3 (DION_PREC_BF16X3): each operand comes as a high and a low bf16 half, a stage holds
+// [A hi][A lo][B hi boxes][B lo boxes], and every k-step issues A_hi B_hi + A_hi B_lo + A_lo B_hi
+// into the same accumulator (the A_lo B_lo term, 2^-18 relative, is left out).
+template <int KIND, bool X3>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(R_THREADS, 1)
     tc_tma_gemm_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off,
                        const LayerMaps *__restrict__ maps, int nstages, uint32_t stage_bytes, uint32_t tmem_cols) {
@@ -175,7 +198,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(R_THREADS, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = align1024(smem_raw);
   uint8_t *stg = smem + nstages * stage_bytes;
-  uint64_t *bars = reinterpret_cast<uint64_t *>(stg + 4 * EPI_BOX);
+  uint64_t *bars = reinterpret_cast<uint64_t *>(stg + STG_BYTES);
+  constexpr uint32_t A_BYTES = (X3 ? 2u : 1u) * OPB_A;  // the A halves of a stage
+  const uint32_t b_half = X3 ? (stage_bytes - A_BYTES) / 2u : 0u;  // offset of the B low boxes
   uint64_t *full = bars, *empty = bars + nstages;
   uint64_t *acc_full = bars + 2 * nstages, *acc_empty = acc_full + 1, *drain = acc_full + 2;
   __shared__ uint32_t tmem_base_s;
@@ -224,21 +249,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(R_THREADS, 1)
         for (int kc = 0; kc < kch; ++kc, ++it) {
           const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
           if (!ab.wait(&empty[s], ph ^ 1u, sh.status)) { ok = false; break; }
-          uint8_t *sA = smem + s * stage_bytes, *sB = sA + OPB_A;
+          uint8_t *sA = smem + s * stage_bytes, *sB = sA + A_BYTES;
           const uint32_t fb = cluster_addr(&full[s], 0);
-          if (rank == 0) mbar_expect_tx(&full[s], 2u * (OPB_A + nbox * BOX64));
-          if (KIND == GEMM_BQ) {
-            tma_load_2d_pair(sA, &mp->Bh_k, fb, kc * 64, tr * 128);
-          } else {
-            tma_load_2d_pair(sA, &mp->Bh_mn, fb, tr * 128, kc * 64);
-            tma_load_2d_pair(sA + BOX64, &mp->Bh_mn, fb, tr * 128 + 64, kc * 64);
-          }
-          const CUtensorMap *bmap = (KIND == GEMM_BQ) ? &mp->Qn_mn : &mp->P_mn;
-          for (uint32_t part = 0; part < nparts; ++part) {
-            const uint32_t hc = half_cols(np, part);
-            const int x0 = (int)(part * 256u + rank * hc);
-            for (uint32_t j = 0; j < (hc + 63) / 64; ++j)
-              tma_load_2d_pair(sB + (part * 2u + j) * BOX64, bmap, fb, x0 + (int)j * 64, kc * 64);
+          if (rank == 0) mbar_expect_tx(&full[s], 2u * (X3 ? 2u : 1u) * (OPB_A + nbox * BOX64));
+          for (int hl = 0; hl < (X3 ? 2 : 1); ++hl) {  // high half, then (BF16X3) low half
+            uint8_t *a = sA + hl * OPB_A;
+            if (KIND == GEMM_BQ) {
+              tma_load_2d_pair(a, hl ? &mp->Bl_k : &mp->Bh_k, fb, kc * 64, tr * 128);
+            } else {
+              const CUtensorMap *am = hl ? &mp->Bl_mn : &mp->Bh_mn;
+              tma_load_2d_pair(a, am, fb, tr * 128, kc * 64);
+              tma_load_2d_pair(a + BOX64, am, fb, tr * 128 + 64, kc * 64);
+            }
+            const CUtensorMap *bmap = (KIND == GEMM_BQ) ? (hl ? &mp->Qn_lo_mn : &mp->Qn_mn)
+                                                        : (hl ? &mp->P_lo_mn : &mp->P_mn);
+            uint8_t *b = sB + hl * b_half;
+            for (uint32_t part = 0; part < nparts; ++part) {
+              const uint32_t hc = half_cols(np, part);
+              const int x0 = (int)(part * 256u + rank * hc);
+              for (uint32_t j = 0; j < (hc + 63) / 64; ++j)
+                tma_load_2d_pair(b + (part * 2u + j) * BOX64, bmap, fb, x0 + (int)j * 64, kc * 64);
+            }
           }
         }
       }
@@ -262,17 +293,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(R_THREADS, 1)
           const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
           if (!ab.wait(&full[s], ph, sh.status)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t aB = smem_u32(smem + s * stage_bytes), bB = aB + OPB_A;
+          const uint32_t aB = smem_u32(smem + s * stage_bytes), bB = aB + A_BYTES;
 #pragma unroll
           for (int k16 = 0; k16 < 4; ++k16) {
             // A: K-major (B Q) advances 32 bytes per 16 k; MN-major (B^T P) two 8-row groups
-            const uint64_t ad = (KIND == GEMM_BQ) ? smem_desc_sw128(aB + k16 * 32, 0, 1024)
-                                                  : smem_desc_sw128(aB + k16 * 2048, BOX64, 1024);
+            const uint32_t ak = (KIND == GEMM_BQ) ? (uint32_t)k16 * 32u : (uint32_t)k16 * 2048u;
+            const uint32_t albo = (KIND == GEMM_BQ) ? 0u : BOX64;
+            const uint64_t ad = smem_desc_sw128(aB + ak, albo, 1024);
             for (uint32_t part = 0; part < nparts; ++part) {
               const uint32_t n_here = 2u * half_cols(np, part);
-              const uint64_t bd = smem_desc_sw128(bB + part * 2u * BOX64 + k16 * 2048, BOX64, 1024);
-              umma_pair_bf16(tmem + part * 256u, ad, bd, idesc_bf16(256, n_here, KIND == GEMM_BTP, true),
-                             (kc | k16) ? 1u : 0u);
+              const uint32_t idesc = idesc_bf16(256, n_here, KIND == GEMM_BTP, true);
+              const uint32_t bo = part * 2u * BOX64 + k16 * 2048;
+              const uint64_t bd = smem_desc_sw128(bB + bo, BOX64, 1024);
+              umma_pair_bf16(tmem + part * 256u, ad, bd, idesc, (kc | k16) ? 1u : 0u);
+              if (X3) {
+                umma_pair_bf16(tmem + part * 256u, ad, smem_desc_sw128(bB + b_half + bo, BOX64, 1024), idesc, 1u);
+                umma_pair_bf16(tmem + part * 256u, smem_desc_sw128(aB + OPB_A + ak, albo, 1024), bd, idesc, 1u);
+              }
             }
           }
           umma_pair_commit_mc(&empty[s], 0x3);  // the stage is free in both CTAs
@@ -299,7 +336,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(R_THREADS, 1)
           store_accumulator(tmem, warp, lane, leader, stg, &maps[t.x].Praw, &maps[t.x].PTraw_t, L.r, L.m, tr * 128,
                             ecount, 1, 0, 1);
         else
-          store_r_tile(tmem, warp, lane, leader, stg, maps[t.x], L, tr, ecount);
+          store_r_tile<X3>(tmem, warp, lane, leader, stg, maps[t.x], L, tr, ecount);
       }
       tc_fence_before();
       named_sync(1, 128);  // every thread's TMEM reads of this accumulator are done
@@ -674,24 +711,58 @@ __global__ void __launch_bounds__(256) qn_refresh_kernel(Shared sh, const int4 *
   const int64_t r = L.r, total = (int64_t)t.z * r;
   for (int64_t e = threadIdx.x; e < total; e += 256) {
     const int64_t i = t.y + e / r, j = e % r;
-    L.Qn_hi[i * L.ldp + j] = __float2bfloat16_rn(L.Q[i * L.ldq + j]);
+    const float q = L.Q[i * L.ldq + j];
+    const __nv_bfloat16 h = __float2bfloat16_rn(q);
+    L.Qn_hi[i * L.ldp + j] = h;
+    if (L.Qn_lo != nullptr) L.Qn_lo[i * L.ldp + j] = __float2bfloat16_rn(q - __bfloat162float(h));
+  }
+}
+
+// BF16X3: the bf16 halves of the orthonormal P (fp32, from the CUDA-core solve) for B^T P and
+// the update.  Tile = {layer, 128-row block}; a warp per row, 8-byte stores.
+__global__ void __launch_bounds__(256) split_p_kernel(Shared sh, const int4 *tiles) {
+  const int4 t = tiles[blockIdx.x];
+  if (!sh.active[t.x]) return;
+  const DevLayer &L = sh.layers[t.x];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t r4 = (L.r + 3) / 4, row_end = min((int64_t)t.y * 128 + 128, L.m);
+  for (int64_t i = (int64_t)t.y * 128 + warp; i < row_end; i += 8) {
+    for (int64_t c4 = lane; c4 < r4; c4 += 32) {
+      const float4 v = *reinterpret_cast<const float4 *>(L.P + i * L.ldp + 4 * c4);  // rows padded to 8
+      const __nv_bfloat162 h01 = __floats2bfloat162_rn(v.x, v.y), h23 = __floats2bfloat162_rn(v.z, v.w);
+      const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+      const __nv_bfloat162 l01 = __floats2bfloat162_rn(v.x - f01.x, v.y - f01.y);
+      const __nv_bfloat162 l23 = __floats2bfloat162_rn(v.z - f23.x, v.w - f23.y);
+      uint2 hv, lv;
+      hv.x = *reinterpret_cast<const uint32_t *>(&h01);
+      hv.y = *reinterpret_cast<const uint32_t *>(&h23);
+      lv.x = *reinterpret_cast<const uint32_t *>(&l01);
+      lv.y = *reinterpret_cast<const uint32_t *>(&l23);
+      *reinterpret_cast<uint2 *>(L.P_hi + i * L.ldp + 4 * c4) = hv;
+      *reinterpret_cast<uint2 *>(L.P_lo + i * L.ldp + 4 * c4) = lv;
+    }
   }
 }
 
 // ======================================================================= launchers ===
 uint32_t form_bq_smem(int nstages, uint32_t stage_bytes) {
-  return 1024u + nstages * stage_bytes + 4 * EPI_BOX + 512u;  // + barriers
+  return 1024u + nstages * stage_bytes + STG_BYTES + 512u;  // + barriers
 }
 uint32_t btp_smem(int nstages, uint32_t stage_bytes) { return form_bq_smem(nstages, stage_bytes); }
 // Q ring of the fused kernel: FB_QSTAGES Q chunks, at least the epilogue's 4 staging boxes
 uint32_t fused_bq_qring(uint32_t bq_boxes) { return std::max(FB_QSTAGES * bq_boxes * BOX64, 4u * EPI_BOX); }
 uint32_t fused_bq_smem(uint32_t bq_boxes) { return 1024u + FB_Q_OFF + fused_bq_qring(bq_boxes) + 512u; }
 
-cudaError_t setup_bq_kernels(uint32_t f_smem, uint32_t r_smem) {
-  cudaError_t e =
-      cudaFuncSetAttribute(tc_tma_gemm_kernel<GEMM_BQ>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)f_smem);
+cudaError_t setup_bq_kernels(uint32_t f_smem, uint32_t r_smem, bool x3) {
+  cudaError_t e = x3 ? cudaFuncSetAttribute(tc_tma_gemm_kernel<GEMM_BQ, true>,
+                                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)f_smem)
+                     : cudaFuncSetAttribute(tc_tma_gemm_kernel<GEMM_BQ, false>,
+                                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)f_smem);
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(tc_tma_gemm_kernel<GEMM_BTP>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)r_smem);
+    e = x3 ? cudaFuncSetAttribute(tc_tma_gemm_kernel<GEMM_BTP, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)r_smem)
+           : cudaFuncSetAttribute(tc_tma_gemm_kernel<GEMM_BTP, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)r_smem);
   return e;
 }
 
@@ -708,16 +779,30 @@ void launch_fused_bq(const Shared &sh, const TcPlan &tp, bool gated, cudaStream_
 
 void launch_form_bq(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
   if (tp.d_bq.grid <= 0) return;
-  const uint32_t stage = OPB_A + tp.bq_boxes * BOX64;
-  tc_tma_gemm_kernel<GEMM_BQ><<<2 * tp.d_bq.grid, R_THREADS, tp.f_smem, s>>>(sh, tp.d_bq.tiles, tp.d_bq.off,
-                                                                             tp.maps, tp.f_stages, stage, tp.tmem_cols);
+  const bool x3 = tp.precision == DION_PREC_BF16X3;
+  const uint32_t stage = (x3 ? 2u : 1u) * (OPB_A + tp.bq_boxes * BOX64);
+  if (x3)
+    tc_tma_gemm_kernel<GEMM_BQ, true><<<2 * tp.d_bq.grid, R_THREADS, tp.f_smem, s>>>(
+        sh, tp.d_bq.tiles, tp.d_bq.off, tp.maps, tp.f_stages, stage, tp.tmem_cols);
+  else
+    tc_tma_gemm_kernel<GEMM_BQ, false><<<2 * tp.d_bq.grid, R_THREADS, tp.f_smem, s>>>(
+        sh, tp.d_bq.tiles, tp.d_bq.off, tp.maps, tp.f_stages, stage, tp.tmem_cols);
 }
 
 void launch_btp(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
   if (tp.d_btp.grid <= 0) return;
-  const uint32_t stage = OPB_A + tp.bq_boxes * BOX64;
-  tc_tma_gemm_kernel<GEMM_BTP><<<2 * tp.d_btp.grid, R_THREADS, tp.r_smem, s>>>(sh, tp.d_btp.tiles, tp.d_btp.off,
-                                                                               tp.maps, tp.r_stages, stage, tp.tmem_cols);
+  const bool x3 = tp.precision == DION_PREC_BF16X3;
+  const uint32_t stage = (x3 ? 2u : 1u) * (OPB_A + tp.bq_boxes * BOX64);
+  if (x3)
+    tc_tma_gemm_kernel<GEMM_BTP, true><<<2 * tp.d_btp.grid, R_THREADS, tp.r_smem, s>>>(
+        sh, tp.d_btp.tiles, tp.d_btp.off, tp.maps, tp.r_stages, stage, tp.tmem_cols);
+  else
+    tc_tma_gemm_kernel<GEMM_BTP, false><<<2 * tp.d_btp.grid, R_THREADS, tp.r_smem, s>>>(
+        sh, tp.d_btp.tiles, tp.d_btp.off, tp.maps, tp.r_stages, stage, tp.tmem_cols);
+}
+
+void launch_split_p(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
+  if (tp.n_trsm_tiles > 0) split_p_kernel<<<tp.n_trsm_tiles, 256, 0, s>>>(sh, tp.trsm_tiles);
 }
 
 void launch_qn_refresh(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
@@ -778,6 +863,15 @@ __global__ void __launch_bounds__(kScaleThreads) colnorm_scale_kernel(Shared sh,
       hv.x = *reinterpret_cast<const uint32_t *>(&h01);
       hv.y = *reinterpret_cast<const uint32_t *>(&h23);
       *reinterpret_cast<uint2 *>(L.Qn_hi + i * L.ldp + 4 * c4) = hv;  // workspace rows: padded
+      if (L.Qn_lo != nullptr) {  // BF16X3: q - bf16(q), rounded to bf16
+        const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+        const __nv_bfloat162 l01 = __floats2bfloat162_rn(q.x - f01.x, q.y - f01.y);
+        const __nv_bfloat162 l23 = __floats2bfloat162_rn(q.z - f23.x, q.w - f23.y);
+        uint2 lv;
+        lv.x = *reinterpret_cast<const uint32_t *>(&l01);
+        lv.y = *reinterpret_cast<const uint32_t *>(&l23);
+        *reinterpret_cast<uint2 *>(L.Qn_lo + i * L.ldp + 4 * c4) = lv;
+      }
       float *Qrow = L.Q + i * L.ldq + 4 * c4;
       if (4 * c4 + 4 <= r) {
         *reinterpret_cast<float4 *>(Qrow) = q;

@@ -9,12 +9,13 @@ namespace tc {
 
 uint32_t form_bq_smem(int nstages, uint32_t stage_bytes);
 uint32_t btp_smem(int nstages, uint32_t stage_bytes);
-cudaError_t setup_bq_kernels(uint32_t f_smem, uint32_t r_smem);
+cudaError_t setup_bq_kernels(uint32_t f_smem, uint32_t r_smem, bool x3);
 void launch_form_bq(const Shared &sh, const TcPlan &tp, cudaStream_t s);
 uint32_t fused_bq_smem(uint32_t bq_boxes);
 cudaError_t setup_fused_bq_kernel(uint32_t smem);
 void launch_fused_bq(const Shared &sh, const TcPlan &tp, bool gated, cudaStream_t s);
 void launch_btp(const Shared &sh, const TcPlan &tp, cudaStream_t s);
+void launch_split_p(const Shared &sh, const TcPlan &tp, cudaStream_t s);
 void launch_qn_refresh(const Shared &sh, const TcPlan &tp, cudaStream_t s);
 void launch_colnorm_reduce(const Shared &sh, const int4 *ctiles, int32_t n_ctiles, float eps_col, cudaStream_t s);
 void launch_colnorm_scale(const Shared &sh, const TcPlan &tp, cudaStream_t s);

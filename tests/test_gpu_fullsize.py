@@ -168,21 +168,25 @@ def phase_boundaries(w):
     return {t for t in out if t <= w.steps}
 
 
+@pytest.mark.parametrize("prec", ["fp32", "bf16x3"])
 @pytest.mark.parametrize("mode", ["per_layer", "global"])
-def test_gpt350m_gate_stress_300_steps_fp32(mode):
+def test_gpt350m_gate_stress_300_steps(mode, prec):
     """The gate-stress stack (144 matrices, r = 256, flat and spiky curvature phases of 50 steps)
     over its stated 300 steps in both gated modes: every step checks every layer's flag against
-    its RMMC and the global flag against their maximum; at t = 1, 2 and the first two steps of
-    every phase (and t = 300) blocks 0 and 23 take an oracle step from the device state, with
-    flags bit-exact and state to 1e-4.  Both branches occur."""
+    its RMMC and the global flag against their maximum; at t = 1, 2, the last and first steps of
+    consecutive phases and t = 300, blocks 0 and 23 take an oracle step from the device state,
+    with flags bit-exact and the state to 1e-4, on CUDA cores (fp32) and on tensor cores with
+    split operands (bf16x3: fp32-class, well inside the 2e-2 of bf16 gradients).  Both branches
+    occur."""
     import paper_2512_13728_gb300 as cd
 
     w = wl.WORKLOADS["gpt350m_gate_stress_r256"]
     gm = oc.GATE_PER_LAYER if mode == "per_layer" else oc.GATE_GLOBAL
     sample = blocks(w, [0, 23])
-    worst, margins, synced = run_sampled(w, cd.DION_PREC_FP32, dict(gate_mode=gm, tau_global=0.5), w.steps,
-                                         TOL_FP32, sample, check_steps=phase_boundaries(w))
-    print("gate stress", mode, "300 steps, sampled worst", worst, "min margin", min(margins))
+    p, tol = (cd.DION_PREC_FP32, TOL_FP32) if prec == "fp32" else (cd.DION_PREC_BF16X3, TOL_FP32)
+    worst, margins, synced = run_sampled(w, p, dict(gate_mode=gm, tau_global=0.5), w.steps, tol, sample,
+                                         check_steps=phase_boundaries(w))
+    print("gate stress", mode, prec, "300 steps, sampled worst", worst, "min margin", min(margins))
     print("synced layers per step", synced)
     assert min(margins) > 1e-4
     assert any(synced) and min(synced) < w.num_layers  # both branches are taken

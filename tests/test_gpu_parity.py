@@ -20,6 +20,7 @@ pytestmark = pytest.mark.gpu
 
 TOL_FP32 = 1e-4
 TOL_BF16 = 2e-2
+PRECS = {"fp32": 0, "bf16": 1, "bf16x3": 2}  # DION_PREC_*
 RMMC_RTOL = 1e-5  # fp32 per-thread sums folded into fp64
 
 
@@ -68,12 +69,15 @@ def run_per_step(w, precision, hp_kw, steps, tol, taus=None, pad=0, min_margin=1
 
 # ------------------------------------------------------------- fp32 single matrix ---
 
+@pytest.mark.parametrize("prec", ["fp32", "bf16x3"])
 @pytest.mark.parametrize("mode", [oc.GATE_ALWAYS, oc.GATE_GLOBAL, oc.GATE_PER_LAYER, oc.GATE_SCHEDULED])
-def test_fp32_256x512_r16_all_modes(mode):
+def test_fp32_256x512_r16_all_modes(mode, prec):
+    """The single fp32 matrix at 1e-4 on CUDA cores and on tensor cores with split operands."""
     import paper_2512_13728_gb300 as cd
 
     w = wl.WORKLOADS["fp32_256x512_r16"]
-    run_per_step(w, cd.DION_PREC_FP32, dict(gate_mode=mode, period=3, mu=0.95, eta=0.01), w.steps, TOL_FP32)
+    p = cd.DION_PREC_FP32 if prec == "fp32" else cd.DION_PREC_BF16X3
+    run_per_step(w, p, dict(gate_mode=mode, period=3, mu=0.95, eta=0.01), w.steps, TOL_FP32)
 
 
 def run_trajectory(w, precision, hp_kw, tol):
@@ -108,12 +112,14 @@ def run_trajectory(w, precision, hp_kw, tol):
         plan.close()
 
 
-def test_fp32_256x512_r16_trajectory():
+@pytest.mark.parametrize("prec", ["fp32", "bf16x3"])
+def test_fp32_256x512_r16_trajectory(prec):
     """The single fp32 matrix over its stated 10 steps, end-of-run state against the oracle's own
-    10-step trajectory (fp32 arithmetic, 1e-4)."""
+    10-step trajectory (fp32-class arithmetic, 1e-4)."""
     import paper_2512_13728_gb300 as cd
 
-    run_trajectory(wl.WORKLOADS["fp32_256x512_r16"], cd.DION_PREC_FP32, dict(gate_mode=oc.GATE_PER_LAYER), TOL_FP32)
+    p = cd.DION_PREC_FP32 if prec == "fp32" else cd.DION_PREC_BF16X3
+    run_trajectory(wl.WORKLOADS["fp32_256x512_r16"], p, dict(gate_mode=oc.GATE_PER_LAYER), TOL_FP32)
 
 
 # ------------------------------------------------- ragged shapes, several tiles ---
@@ -127,6 +133,52 @@ def test_ragged_shapes_fp32(pad):
     import paper_2512_13728_gb300 as cd
 
     run_per_step(RAGGED, cd.DION_PREC_FP32, dict(gate_mode=oc.GATE_ALWAYS), RAGGED.steps, TOL_FP32, pad=pad)
+
+
+@pytest.mark.parametrize("g_dtype", ["bf16", "fp32"])
+@pytest.mark.parametrize("pad", [0, 1])
+def test_ragged_shapes_bf16x3(pad, g_dtype):
+    """Split-operand tensor-core mode on ragged shapes, several tiles and NaN-padded rows, at the
+    fp32 tolerance with either gradient dtype."""
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.scaled(RAGGED, "ragged_x3", RAGGED.shapes, g_dtype=g_dtype)
+    worst, _ = run_per_step(w, cd.DION_PREC_BF16X3, dict(gate_mode=oc.GATE_ALWAYS), w.steps, TOL_FP32, pad=pad)
+    print("bf16x3 ragged", g_dtype, worst)
+
+
+def test_bf16x3_full_rank_and_rank_256():
+    """r = min(m, n) and r = 256 (the mode's largest rank) with split operands, at 1e-4."""
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.scaled(wl.WORKLOADS["gpt160m_block_r192"], "x3rank", [(600, 256), (48, 40), (300, 520)], rank=256,
+                  steps=3, g_dtype="fp32")
+    st = gu.make_state(w)
+    _orthonormal_q0(st)
+    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_BF16X3)
+    hpo = gu.oracle_hp()
+    try:
+        for t in range(1, w.steps + 1):
+            gu.write_gradients(st, t)
+            layers, grads, prev = gu.snapshot(st, plan)
+            plan.step(cd.hparams(step=t))
+            torch.cuda.synchronize()
+            assert plan.device_status() == 0
+            c = gu.compare_step(st, plan, layers, grads, prev, hpo, t)
+            print(t, c.err_M, c.err_X, c.err_Q)
+            assert max(c.err_M, c.err_X, c.err_Q) <= TOL_FP32
+    finally:
+        plan.close()
+
+
+def test_bf16x3_rejects_rank_above_256():
+    import paper_2512_13728_gb300 as cd
+
+    w = wl.scaled(wl.WORKLOADS["gpt160m_block_r192"], "x3big", [(300, 300)], rank=257, steps=1)
+    st = gu.make_state(w)
+    with pytest.raises(cd.DionError) as e:
+        cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_BF16X3)
+    assert e.value.code == cd.native.DION_ERR_UNSUPPORTED
 
 
 def _orthonormal_q0(st):
@@ -314,7 +366,7 @@ def test_empty_plan_step():
 
 # ------------------------------------------------------------- device-side errors ---
 
-@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+@pytest.mark.parametrize("prec", ["fp32", "bf16", "bf16x3"])
 def test_breakdown_on_zero_buffer_sets_status_and_no_nan(prec):
     """B = 0 (rank-deficient P): DION_ERR_BREAKDOWN, L^{-1} = 0, so X is unchanged and nothing
     non-finite is written, in both the CUDA-core and the tensor-core path (fused buffer + B Q)."""
@@ -322,7 +374,7 @@ def test_breakdown_on_zero_buffer_sets_status_and_no_nan(prec):
 
     w = wl.scaled(RAGGED, "zero", [(64, 48), (256, 136)], rank=4, steps=1)
     st = gu.make_state(w)
-    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_FP32 if prec == "fp32" else cd.DION_PREC_BF16)
+    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, PRECS[prec])
     x0 = [x.clone() for x in st.X]
     plan.step(cd.hparams(step=1))  # G = 0 and M = 0: B = 0, P = 0, Gram = 0
     torch.cuda.synchronize()
@@ -334,7 +386,7 @@ def test_breakdown_on_zero_buffer_sets_status_and_no_nan(prec):
     plan.close()
 
 
-@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+@pytest.mark.parametrize("prec", ["fp32", "bf16", "bf16x3"])
 def test_nonfinite_gradient_sets_status_and_flags(prec):
     import paper_2512_13728_gb300 as cd
 
@@ -342,7 +394,7 @@ def test_nonfinite_gradient_sets_status_and_flags(prec):
     st = gu.make_state(w, taus=[1e9, 1e9])
     gu.write_gradients(st, 1)
     st.G[0][3, 5] = float("nan")
-    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_FP32 if prec == "fp32" else cd.DION_PREC_BF16)
+    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, PRECS[prec])
     plan.step(cd.hparams(step=1, gate_mode=cd.DION_GATE_PER_LAYER, tau_global=1e9))
     torch.cuda.synchronize()
     assert plan.device_status() == cd.native.DION_ERR_NONFINITE
@@ -367,16 +419,17 @@ def test_deterministic_bitwise():
         assert torch.equal(a, b)
 
 
+@pytest.mark.parametrize("prec", ["bf16", "bf16x3"])
 @pytest.mark.parametrize("g_dtype", ["bf16", "fp32"])
-def test_deterministic_bitwise_bf16_mode(g_dtype):
-    """The tensor-core mode repeats bit for bit (fixed-order norm and column reductions)."""
+def test_deterministic_bitwise_bf16_mode(g_dtype, prec):
+    """The tensor-core modes repeat bit for bit (fixed-order norm and column reductions)."""
     import paper_2512_13728_gb300 as cd
 
     w = wl.scaled(RAGGED, "ragged_det", RAGGED.shapes, g_dtype=g_dtype)
     outs = []
     for _ in range(2):
         st = gu.make_state(w)
-        plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_BF16)
+        plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, PRECS[prec])
         for t in range(1, 4):
             gu.write_gradients(st, t)
             plan.step(cd.hparams(step=t))
