@@ -38,7 +38,7 @@
 extern "C" {
 #endif
 
-#define DION_ABI_VERSION 2
+#define DION_ABI_VERSION 3
 
 typedef enum {
   DION_OK = 0,
@@ -131,6 +131,43 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
 dion_status dion_step(dion_plan *plan, const dion_hparams *hp, double *prev_norm,
                       double *rmmc_out, double *rmmc_eq1_out, uint8_t *sync_flags_out,
                       uint8_t *global_flag_out, void *stream);
+
+/* Data-parallel steps (Algorithm 2 with W workers, one plan per worker; no collective is
+ * issued by the library).  Algorithm 2 reduces across workers at three points: the maximum of
+ * RMMC before the branch (the AllReduce_max), P after PowerIter and R after it is formed from
+ * the orthonormal P (the AllReduce_DP lines, read as the mean over the workers).
+ * dion_step_phase runs one step as four phases, in order, on `stream`; between them the caller
+ * performs the reductions on device buffers (with NCCL, or any other means), on the same stream
+ * or ordered after it:
+ *   DION_PHASE_NORMS   B = M + G (written into M), ||B|| and this worker's RMMC_l into rmmc_out,
+ *                      prev_norm_l = ||B|| (each worker keeps its own prev_norm).
+ *                      Then: rmmc_out <- elementwise max over the workers.
+ *   DION_PHASE_POWER   sync flags, global flag and branch from the reduced rmmc_out (final
+ *                      values of those outputs), then P = B Q on the layers that synchronize.
+ *                      Then: the P range of dion_plan_exchange <- mean over the workers.
+ *   DION_PHASE_ORTHO   P = Orthogonalize(mean P), R = B^T P on the synchronizing layers.
+ *                      Then: the R range <- mean over the workers.
+ *   DION_PHASE_UPDATE  Q_t = ColumnNormalize(mean R), M = B - (1 - mu) P R^T (this worker's B),
+ *                      X = X - eta sqrt(m/n) P Q_t^T; local layers: X = X - eta_local G.
+ * Every phase takes the same hp and output pointers as dion_step.  A layer that stays local
+ * leaves stale values in its part of the exchange ranges; averaging them is harmless, and a
+ * caller that wants to skip the exchanges of a step with no synchronizing layer reads
+ * global_flag_out / sync_flags_out after DION_PHASE_POWER.  Workers' plans must have the same
+ * layer shapes and precision and the same Q at the start (as Algorithm 2's identical Q_t);
+ * their exchange ranges then line up element for element.  With one worker the reductions are
+ * the identity and the four phases compute what dion_step computes.  Errors: as dion_step, and
+ * INVALID_ARG for a phase out of order (dion_step and dion_step_host are refused while a phased
+ * step is unfinished). */
+enum { DION_PHASE_NORMS = 1, DION_PHASE_POWER = 2, DION_PHASE_ORTHO = 3, DION_PHASE_UPDATE = 4 };
+dion_status dion_step_phase(dion_plan *plan, int32_t phase, const dion_hparams *hp, double *prev_norm,
+                            double *rmmc_out, double *rmmc_eq1_out, uint8_t *sync_flags_out,
+                            uint8_t *global_flag_out, void *stream);
+/* The device range a worker reduces after `phase`: DION_PHASE_POWER gives P (every layer's m x r
+ * fp32 P, rows padded to a multiple of 8 floats, layers one after another with small zeroed
+ * gaps), DION_PHASE_ORTHO gives R (n x r per layer, the same layout).  *buf_out (device, owned
+ * by the plan) and *count_out (fp32 elements) are fixed for the plan's lifetime.  Errors:
+ * INVALID_ARG (NULL argument, other phase). */
+dion_status dion_plan_exchange(dion_plan *plan, int32_t phase, float **buf_out, int64_t *count_out);
 
 /* Gradients from host memory (no counterpart in the paper: it moves Algorithm 1's input G_t
  * onto the device).  dion_plan_enable_host_gradients allocates, once, two device gradient

@@ -10,8 +10,17 @@ from typing import Optional, Sequence
 
 from . import native
 from .native import (DION_DTYPE_BF16, DION_DTYPE_FP32, DION_GATE_ALWAYS, DION_GATE_GLOBAL,  # noqa: F401
-                     DION_GATE_PER_LAYER, DION_GATE_SCHEDULED, DION_PREC_BF16, DION_PREC_BF16X3,
+                     DION_GATE_PER_LAYER, DION_GATE_SCHEDULED, DION_PHASE_NORMS, DION_PHASE_ORTHO,
+                     DION_PHASE_POWER, DION_PHASE_UPDATE, DION_PREC_BF16, DION_PREC_BF16X3,
                      DION_PREC_FP32, DionError, dion_hparams, dion_layer)
+
+
+class _DeviceRange:
+    """A plan-owned fp32 device range exposed through __cuda_array_interface__, so that
+    torch.as_tensor views it without a copy (for a collective's in-place reduction)."""
+
+    def __init__(self, ptr: int, count: int):
+        self.__cuda_array_interface__ = {"shape": (count,), "typestr": "<f4", "data": (ptr, False), "version": 3}
 
 
 def _layer(X, M, Q, G, tau: float) -> dion_layer:
@@ -83,6 +92,26 @@ class Plan:
         native.dion_step(self.handle, hp, self.prev_norm.data_ptr(), self.rmmc.data_ptr(),
                          self.rmmc_eq1.data_ptr() if eq1 else None, self.flags.data_ptr(),
                          self.global_flag.data_ptr(), s)
+
+    def step_phase(self, phase: int, hp: dion_hparams, stream: Optional[int] = None, eq1: bool = True) -> None:
+        """One phase (DION_PHASE_*) of a data-parallel step; the caller reduces rmmc (max) after
+        NORMS and the exchange() ranges (mean) after POWER and ORTHO."""
+        import torch
+
+        s = torch.cuda.current_stream(self.device).cuda_stream if stream is None else stream
+        native.dion_step_phase(self.handle, phase, hp, self.prev_norm.data_ptr(), self.rmmc.data_ptr(),
+                               self.rmmc_eq1.data_ptr() if eq1 else None, self.flags.data_ptr(),
+                               self.global_flag.data_ptr(), s)
+
+    def exchange(self, phase: int):
+        """The plan's exchange range after `phase` (P after POWER, R after ORTHO) as a 1-D
+        float32 tensor sharing the plan's memory (valid while the plan lives)."""
+        import torch
+
+        ptr, count = native.dion_plan_exchange(self.handle, phase)
+        if count == 0:
+            return torch.empty(0, dtype=torch.float32, device=self.device)
+        return torch.as_tensor(_DeviceRange(ptr, count), device=self.device)
 
     def enable_host_gradients(self) -> None:
         """Lets step_host read each step's gradients from host memory (two device buffers per

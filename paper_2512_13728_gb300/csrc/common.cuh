@@ -145,6 +145,8 @@ __device__ __forceinline__ double block_sum(double v, double *red /* >= THREADS/
 // CUDA-core (fp32) kernels, kernels_simt.cu
 void launch_form_b(const Shared &sh, const int4 *tiles, int32_t ntiles, cudaStream_t s);
 void launch_gate(const Shared &sh, const StepArgs &a, cudaStream_t s);
+// the branch from RMMC values already in a.rmmc (reduced over data-parallel workers)
+void launch_gate_reduced(const Shared &sh, const StepArgs &a, cudaStream_t s);
 void launch_gemm(const Shared &sh, const GemmProblem *probs, const int4 *tiles, int32_t ntiles,
                  cudaStream_t s);
 cudaError_t prepare_chol_inv(int32_t max_r, size_t *smem_out);

@@ -219,6 +219,40 @@ void launch_gate(const Shared &sh, const StepArgs &a, cudaStream_t s) {
   gate_kernel<<<std::max(1, (sh.num_layers + kGateWarps - 1) / kGateWarps), kGateWarps * 32, 0, s>>>(sh, a);
 }
 
+// Data-parallel steps: Algorithm 2's branch from RMMC values the caller has already reduced
+// over the workers (AllReduce_max), in a.rmmc.  One block: every layer's flag, the maximum over
+// layers (a non-finite value counts as above every threshold) for the global flag, and the
+// branch mask of the gate mode.
+constexpr int kGateRedThreads = 256;
+__global__ void __launch_bounds__(kGateRedThreads) gate_reduced_kernel(Shared sh, StepArgs a) {
+  __shared__ double max_s[kGateRedThreads / 32];
+  __shared__ int gflag_s, count_s;
+  const int L = sh.num_layers, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  double mx = -1.0;
+  for (int l = threadIdx.x; l < L; l += kGateRedThreads) {
+    double v = a.rmmc[l];
+    if (!isfinite(v)) v = INFINITY;
+    a.flags[l] = above(v, sh.layers[l].tau) ? 1 : 0;
+    mx = fmax(mx, v);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mx = fmax(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  if (lane == 0) max_s[warp] = mx;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double g = -1.0;
+    for (int w = 0; w < kGateRedThreads / 32; ++w) g = fmax(g, max_s[w]);
+    gflag_s = (L > 0 && above(g, a.tau_global)) ? 1 : 0;
+    a.gflag[0] = (uint8_t)gflag_s;
+  }
+  __syncthreads();
+  gate_finish(sh, a, gflag_s, &count_s);
+}
+
+void launch_gate_reduced(const Shared &sh, const StepArgs &a, cudaStream_t s) {
+  gate_reduced_kernel<<<1, kGateRedThreads, 0, s>>>(sh, a);
+}
+
 // ==================================================================== norms + gate ===
 // Gated modes with the fused buffer + B Q kernel: Algorithm 2 needs ||B|| before it knows which
 // layers take the Dion branch, so this pass forms B = M + G into M (read M, G; write M:

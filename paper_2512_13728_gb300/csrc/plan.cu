@@ -34,6 +34,11 @@ struct dion_plan {
   size_t chol_smem = 0;
   tc::TcPlan tcp{};  // tensor-core path (BF16 / BF16X3)
   int32_t launches_per_step = 0;
+  // data-parallel phases (dion_step_phase): the exchange ranges (offsets into ws, fp32 counts)
+  // and the phase the next call must run
+  size_t xp_off = 0, xr_off = 0;
+  int64_t xp_count = 0, xr_count = 0;
+  int32_t next_phase = DION_PHASE_NORMS;
   // per-launch timing (dion_timing_enable)
   std::vector<cudaEvent_t> ev;  // [max_steps][launches + 1]
   std::vector<const char *> names;
@@ -167,6 +172,18 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
   std::vector<DevLayer> dl(num_layers);
   std::vector<size_t> o_Praw(num_layers), o_P(num_layers), o_R(num_layers), o_S(num_layers), o_Li(num_layers);
   std::vector<int4> bt, ut, ct;
+  // P_raw and R of all layers each in one contiguous range (256-byte gaps between layers): the
+  // buffers a data-parallel caller averages between the phases of dion_step_phase
+  for (int32_t l = 0; l < num_layers; ++l) o_Praw[l] = cv.take<float>(layers[l].m * ((layers[l].r + 7) / 8 * 8));
+  for (int32_t l = 0; l < num_layers; ++l) o_R[l] = cv.take<float>(layers[l].n * ((layers[l].r + 7) / 8 * 8));
+  if (num_layers > 0) {
+    const dion_layer &a = layers[num_layers - 1];
+    const int64_t lp = (a.r + 7) / 8 * 8;
+    p->xp_off = o_Praw[0];
+    p->xp_count = (int64_t)((o_Praw[num_layers - 1] - o_Praw[0]) / sizeof(float)) + a.m * lp;
+    p->xr_off = o_R[0];
+    p->xr_count = (int64_t)((o_R[num_layers - 1] - o_R[0]) / sizeof(float)) + a.n * lp;
+  }
   for (int32_t l = 0; l < num_layers; ++l) {
     const dion_layer &ly = layers[l];
     DevLayer &d = dl[l];
@@ -180,9 +197,7 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
     d.sqrt_m_over_n = (float)std::sqrt((double)ly.m / (double)ly.n);
     d.ldp = (int32_t)((ly.r + 7) / 8 * 8);
     p->max_r = std::max<int32_t>(p->max_r, (int32_t)ly.r);
-    o_Praw[l] = cv.take<float>(ly.m * d.ldp);
     o_P[l] = cv.take<float>(ly.m * d.ldp);
-    o_R[l] = cv.take<float>(ly.n * d.ldp);
     o_S[l] = cv.take<float>(ly.r * d.ldp);
     o_Li[l] = cv.take<float>(ly.r * d.ldp);
     // row tiles of about 64K elements for the buffer and local kernels
@@ -304,7 +319,8 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
   p->ctiles = reinterpret_cast<int4 *>(base + o_ct);
   p->n_ctiles = (int32_t)ct.size();
 
-  cudaError_t e = cudaSuccess;
+  // zeroed once, so the gaps and row padding inside the exchange ranges hold zeros
+  cudaError_t e = cudaMemset(p->ws, 0, cv.off);
   if (e == cudaSuccess) e = upload(p->sh.layers, dl);
   p->dl_host = dl;
   if (e == cudaSuccess) e = upload(p->btiles, bt);
@@ -359,9 +375,8 @@ dion_status check_step_args(const dion_plan *p, const dion_hparams *hp, const do
 // Enqueues the step's launch sequence on s with the given layer table and tensor maps (the
 // plan's own, or those of a host-gradient buffer).  The caller has checked the arguments and
 // made the plan's device current.
-void enqueue_step(dion_plan *p, const Shared &sh, const tc::TcPlan &tcp, const dion_hparams *hp, double *prev_norm,
-                  double *rmmc_out, double *rmmc_eq1_out, uint8_t *sync_flags_out, uint8_t *global_flag_out,
-                  cudaStream_t s) {
+StepArgs make_args(const dion_hparams *hp, double *prev_norm, double *rmmc_out, double *rmmc_eq1_out,
+                   uint8_t *sync_flags_out, uint8_t *global_flag_out) {
   StepArgs a{};
   a.mu = hp->mu; a.eta = hp->eta; a.eta_local = hp->eta_local;
   a.eps_rmmc = hp->eps_rmmc; a.eps_col = hp->eps_col; a.tau_global = hp->tau_global;
@@ -370,6 +385,13 @@ void enqueue_step(dion_plan *p, const Shared &sh, const tc::TcPlan &tcp, const d
   a.gate_mode = hp->gate_mode; a.period = hp->period < 1 ? 1 : hp->period; a.step = hp->step;
   a.prev_norm = prev_norm; a.rmmc = rmmc_out; a.eq1 = rmmc_eq1_out;
   a.flags = sync_flags_out; a.gflag = global_flag_out;
+  return a;
+}
+
+void enqueue_step(dion_plan *p, const Shared &sh, const tc::TcPlan &tcp, const dion_hparams *hp, double *prev_norm,
+                  double *rmmc_out, double *rmmc_eq1_out, uint8_t *sync_flags_out, uint8_t *global_flag_out,
+                  cudaStream_t s) {
+  const StepArgs a = make_args(hp, prev_norm, rmmc_out, rmmc_eq1_out, sync_flags_out, global_flag_out);
   tick_begin(p, s);
   if (p->precision == DION_PREC_FP32) {
     launch_form_b(sh, p->btiles, p->n_btiles, s);
@@ -405,6 +427,41 @@ void enqueue_step(dion_plan *p, const Shared &sh, const tc::TcPlan &tcp, const d
   tick_end(p);
 }
 
+// One phase of a data-parallel step (dion_step_phase).  The caller reduces rmmc (max) between
+// NORMS and POWER, the P range (mean) between POWER and ORTHO and the R range (mean) between
+// ORTHO and UPDATE.
+void enqueue_phase(dion_plan *p, const StepArgs &a, int32_t phase, cudaStream_t s) {
+  const Shared &sh = p->sh;
+  if (p->precision != DION_PREC_FP32) {
+    tc::step_phase(p->tcp, sh, a, phase, p->btiles, p->n_btiles, p->ctiles, p->n_ctiles, p->chol_smem, s);
+    return;
+  }
+  switch (phase) {
+    case DION_PHASE_NORMS:  // B = M + G, ||B||, this worker's RMMC, prev_norm <- ||B||
+      launch_form_b(sh, p->btiles, p->n_btiles, s);
+      launch_gate(sh, a, s);
+      break;
+    case DION_PHASE_POWER:  // the branch from the reduced RMMC, then P = B Q on the Dion layers
+      launch_gate_reduced(sh, a, s);
+      launch_gemm(sh, p->probs[0], p->gtiles[0], p->n_gtiles[0], s);
+      break;
+    case DION_PHASE_ORTHO:  // Orthogonalize the averaged P, then R = B^T P
+      for (int pass = 0; pass < 3; ++pass) {
+        launch_gemm(sh, p->probs[1 + pass], p->gtiles[1 + pass], p->n_gtiles[1 + pass], s);
+        launch_chol_inv(sh, p->chol_smem, pass, 1e-3f, s);
+        launch_gemm(sh, p->probs[4 + pass], p->gtiles[4 + pass], p->n_gtiles[4 + pass], s);
+      }
+      launch_gemm(sh, p->probs[7], p->gtiles[7], p->n_gtiles[7], s);
+      break;
+    default:  // UPDATE: Q_t from the averaged R, error feedback and parameter update, local branch
+      launch_colnorm(sh, p->ctiles, p->n_ctiles, a.eps_col, s);
+      launch_update(sh, p->utiles, p->n_utiles, a.mu, a.eta, a.keep_sync, s);
+      launch_local(sh, p->btiles, p->n_btiles, a.eta_local, a.keep_local, s);
+      launch_finalize(sh, a, s);
+      break;
+  }
+}
+
 // Makes the plan's device current for the duration of a call.
 struct DeviceGuard {
   int prev = -1;
@@ -426,11 +483,40 @@ dion_status dion_step(dion_plan *p, const dion_hparams *hp, double *prev_norm, d
                       void *stream) {
   const dion_status st = check_step_args(p, hp, prev_norm, rmmc_out, sync_flags_out, global_flag_out);
   if (st != DION_OK) return st;
+  if (p->next_phase != DION_PHASE_NORMS) return DION_ERR_INVALID_ARG;  // a phased step is unfinished
   DeviceGuard g(p->device);
   if (!g.ok) return DION_ERR_CUDA;
   enqueue_step(p, p->sh, p->tcp, hp, prev_norm, rmmc_out, rmmc_eq1_out, sync_flags_out, global_flag_out,
                static_cast<cudaStream_t>(stream));
   return cudaGetLastError() == cudaSuccess ? DION_OK : DION_ERR_CUDA;
+}
+
+dion_status dion_step_phase(dion_plan *p, int32_t phase, const dion_hparams *hp, double *prev_norm, double *rmmc_out,
+                            double *rmmc_eq1_out, uint8_t *sync_flags_out, uint8_t *global_flag_out, void *stream) {
+  const dion_status st = check_step_args(p, hp, prev_norm, rmmc_out, sync_flags_out, global_flag_out);
+  if (st != DION_OK) return st;
+  if (phase < DION_PHASE_NORMS || phase > DION_PHASE_UPDATE || phase != p->next_phase) return DION_ERR_INVALID_ARG;
+  DeviceGuard g(p->device);
+  if (!g.ok) return DION_ERR_CUDA;
+  const StepArgs a = make_args(hp, prev_norm, rmmc_out, rmmc_eq1_out, sync_flags_out, global_flag_out);
+  enqueue_phase(p, a, phase, static_cast<cudaStream_t>(stream));
+  if (cudaGetLastError() != cudaSuccess) return DION_ERR_CUDA;
+  p->next_phase = (phase == DION_PHASE_UPDATE) ? DION_PHASE_NORMS : phase + 1;
+  return DION_OK;
+}
+
+dion_status dion_plan_exchange(dion_plan *p, int32_t phase, float **buf_out, int64_t *count_out) {
+  if (!p || !buf_out || !count_out) return DION_ERR_INVALID_ARG;
+  if (phase == DION_PHASE_POWER) {
+    *buf_out = p->L > 0 ? reinterpret_cast<float *>(static_cast<char *>(p->ws) + p->xp_off) : nullptr;
+    *count_out = p->xp_count;
+  } else if (phase == DION_PHASE_ORTHO) {
+    *buf_out = p->L > 0 ? reinterpret_cast<float *>(static_cast<char *>(p->ws) + p->xr_off) : nullptr;
+    *count_out = p->xr_count;
+  } else {
+    return DION_ERR_INVALID_ARG;
+  }
+  return DION_OK;
 }
 
 dion_status dion_plan_enable_host_gradients(dion_plan *p) {
@@ -509,6 +595,7 @@ dion_status dion_step_host(dion_plan *p, const dion_hparams *hp, const void *con
   const dion_status st = check_step_args(p, hp, prev_norm, rmmc_out, sync_flags_out, global_flag_out);
   if (st != DION_OK) return st;
   if (!p->hg.on || (p->L > 0 && (!host_G || !host_ldg))) return DION_ERR_INVALID_ARG;
+  if (p->next_phase != DION_PHASE_NORMS) return DION_ERR_INVALID_ARG;  // a phased step is unfinished
   for (int32_t l = 0; l < p->L; ++l)
     if (!host_G[l] || host_ldg[l] < p->dl_host[l].n) return DION_ERR_INVALID_ARG;
   DeviceGuard g(p->device);

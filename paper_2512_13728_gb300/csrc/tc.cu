@@ -709,6 +709,63 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh_in, const StepArgs &a
   tick(p, s, "finalize");
 }
 
+void step_phase(const TcPlan &tp, const Shared &sh_in, const StepArgs &a, int32_t phase, const int4 *btiles,
+                int32_t n_btiles, const int4 *ctiles, int32_t n_ctiles, size_t chol_smem, cudaStream_t s) {
+  Shared sh = sh_in;
+  // with bf16 gradients the norms pass writes B into M before the branch is known (the flow
+  // of the gated modes), whatever the gate mode; the later phases read B from M
+  sh.b_in_m = tp.fuse_buffer ? 1 : 0;
+  const bool x3 = tp.precision == DION_PREC_BF16X3;
+  switch (phase) {
+    case DION_PHASE_NORMS:  // B = M + G, ||B||, this worker's RMMC, prev_norm <- ||B||
+      if (tp.fuse_buffer) {
+        launch_norms_gate(sh, a, tp.ftiles, tp.n_ftiles, s);
+      } else {
+        launch_form_b(sh, btiles, n_btiles, s);
+        launch_gate(sh, a, s);
+      }
+      break;
+    case DION_PHASE_POWER:  // the branch from the reduced RMMC, then P = B Q on the Dion layers
+      launch_gate_reduced(sh, a, s);
+      if (tp.fuse_buffer) launch_fused_bq(sh, tp, true, s);
+      else launch_form_bq(sh, tp, s);
+      break;
+    case DION_PHASE_ORTHO:  // Orthogonalize the averaged P, then R = B^T P
+      if (x3) {
+        for (int pass = 0; pass < 3; ++pass) {
+          launch_gemm(sh, tp.probs[1 + pass], tp.gtiles[1 + pass], tp.n_gtiles[1 + pass], s);
+          launch_chol_inv(sh, chol_smem, pass, 1e-3f, s);
+          launch_gemm(sh, tp.probs[4 + pass], tp.gtiles[4 + pass], tp.n_gtiles[4 + pass], s);
+        }
+        launch_split_p(sh, tp, s);
+      } else {
+        launch_transpose_praw(sh, tp, s);  // the first Gram reads P_raw^T
+        for (int pass = 0; pass < 3; ++pass) {
+          launch_orth(sh, tp, true, pass, s);
+          launch_chol_inv(sh, chol_smem, pass, 6e-2f, s);
+          launch_orth(sh, tp, false, pass, s);
+        }
+      }
+      launch_btp(sh, tp, s);
+      break;
+    default:  // UPDATE: Q_t from the averaged R, error feedback and parameter update, local branch
+      launch_r_refresh(sh, tp, s);
+      launch_colnorm_reduce(sh, ctiles, n_ctiles, a.eps_col, s);
+      launch_colnorm_scale(sh, tp, s);
+      if (tp.d_update.grid > 0) {
+        if (x3)
+          tc_update_kernel<true><<<2 * tp.d_update.grid, U_THREADS, UpdCfg<true>::SMEM, s>>>(
+              sh, tp.d_update.tiles, tp.d_update.off, tp.maps, a.mu, a.eta, a.keep_sync);
+        else
+          tc_update_kernel<false><<<2 * tp.d_update.grid, U_THREADS, UpdCfg<false>::SMEM, s>>>(
+              sh, tp.d_update.tiles, tp.d_update.off, tp.maps, a.mu, a.eta, a.keep_sync);
+      }
+      launch_local(sh, btiles, n_btiles, a.eta_local, a.keep_local, s);
+      launch_finalize(sh, a, s);
+      break;
+  }
+}
+
 void destroy(TcPlan *tp) { (void)tp; }
 
 }  // namespace tc

@@ -116,6 +116,9 @@ int32_t launches_per_step(const TcPlan &tp);
 // Enqueues one step.
 void step(dion_plan *p, const TcPlan &tp, const Shared &sh, const StepArgs &a, const int4 *btiles,
           int32_t n_btiles, const int4 *ctiles, int32_t n_ctiles, size_t chol_smem, cudaStream_t s);
+// Enqueues one phase of a data-parallel step (DION_PHASE_*).
+void step_phase(const TcPlan &tp, const Shared &sh, const StepArgs &a, int32_t phase, const int4 *btiles,
+                int32_t n_btiles, const int4 *ctiles, int32_t n_ctiles, size_t chol_smem, cudaStream_t s);
 void destroy(TcPlan *tp);
 // Re-derives the bf16 copy of every layer's Q from the caller's fp32 Q (plan creation and
 // dion_plan_refresh).

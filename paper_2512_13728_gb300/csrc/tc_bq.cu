@@ -801,6 +801,61 @@ void launch_btp(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
         sh, tp.d_btp.tiles, tp.d_btp.off, tp.maps, tp.r_stages, stage, tp.tmem_cols);
 }
 
+// Data-parallel phases.  P_raw^T (r x m, the first Gram's operand) from the averaged P_raw:
+// tile = {layer, 128-row block of P_raw}, 32 x 32 sub-tiles through shared memory.
+__global__ void __launch_bounds__(256) transpose_praw_kernel(Shared sh, const int4 *tiles) {
+  const int4 t = tiles[blockIdx.x];
+  if (!sh.active[t.x]) return;
+  const DevLayer &L = sh.layers[t.x];
+  __shared__ float tile[32][33];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t row_end = min((int64_t)t.y * 128 + 128, L.m);
+  for (int64_t r0 = (int64_t)t.y * 128; r0 < row_end; r0 += 32) {
+    for (int64_t c0 = 0; c0 < L.r; c0 += 32) {
+      for (int i = warp; i < 32; i += 8) {  // rows r0 + i, columns c0 + lane of P_raw
+        const int64_t row = r0 + i, col = c0 + lane;
+        tile[i][lane] = (row < row_end && col < L.r) ? L.P_raw[row * L.ldp + col] : 0.f;
+      }
+      __syncthreads();
+      for (int i = warp; i < 32; i += 8) {  // row c0 + i of P_raw^T, columns r0 + lane
+        const int64_t col = c0 + i, row = r0 + lane;
+        if (col < L.r && row < row_end) L.PT_raw[col * L.ldmt + row] = tile[lane][i];
+      }
+      __syncthreads();
+    }
+  }
+}
+
+// R's bf16 copy (and low half in BF16X3) and the per-tile column sums of squares that
+// ColumnNormalize reads, from the averaged R: tile = {layer, 128-row block of R}; thread j
+// takes columns j and j + 256, rows in order (fp32 over 32 rows, then fp64).
+__global__ void __launch_bounds__(256) r_refresh_kernel(Shared sh, const int4 *tiles) {
+  const int4 t = tiles[blockIdx.x];
+  if (!sh.active[t.x]) return;
+  const DevLayer &L = sh.layers[t.x];
+  const int64_t r0 = (int64_t)t.y * 128, r1 = min(r0 + 128, L.n);
+  for (int64_t c = threadIdx.x; c < L.r; c += 256) {
+    double acc = 0.0;
+    float f = 0.f;
+    for (int64_t i = r0; i < r1; ++i) {
+      const float v = L.R[i * L.ldp + c];
+      f = fmaf(v, v, f);
+      if (((i - r0) & 31) == 31) { acc += (double)f; f = 0.f; }
+      const __nv_bfloat16 h = __float2bfloat16_rn(v);
+      L.R_hi[i * L.ldp + c] = h;
+      if (L.R_lo != nullptr) L.R_lo[i * L.ldp + c] = __float2bfloat16_rn(v - __bfloat162float(h));
+    }
+    L.colsq[(int64_t)t.y * L.ldp + c] = acc + (double)f;
+  }
+}
+
+void launch_transpose_praw(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
+  if (tp.n_trsm_tiles > 0) transpose_praw_kernel<<<tp.n_trsm_tiles, 256, 0, s>>>(sh, tp.trsm_tiles);
+}
+void launch_r_refresh(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
+  if (tp.n_rtiles > 0) r_refresh_kernel<<<tp.n_rtiles, 256, 0, s>>>(sh, tp.rtiles);
+}
+
 void launch_split_p(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
   if (tp.n_trsm_tiles > 0) split_p_kernel<<<tp.n_trsm_tiles, 256, 0, s>>>(sh, tp.trsm_tiles);
 }

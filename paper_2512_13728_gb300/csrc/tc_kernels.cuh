@@ -16,6 +16,10 @@ cudaError_t setup_fused_bq_kernel(uint32_t smem);
 void launch_fused_bq(const Shared &sh, const TcPlan &tp, bool gated, cudaStream_t s);
 void launch_btp(const Shared &sh, const TcPlan &tp, cudaStream_t s);
 void launch_split_p(const Shared &sh, const TcPlan &tp, cudaStream_t s);
+// data-parallel phases: P_raw^T from the averaged P_raw; R's bf16 copies and column partials
+// from the averaged R
+void launch_transpose_praw(const Shared &sh, const TcPlan &tp, cudaStream_t s);
+void launch_r_refresh(const Shared &sh, const TcPlan &tp, cudaStream_t s);
 void launch_qn_refresh(const Shared &sh, const TcPlan &tp, cudaStream_t s);
 void launch_colnorm_reduce(const Shared &sh, const int4 *ctiles, int32_t n_ctiles, float eps_col, cudaStream_t s);
 void launch_colnorm_scale(const Shared &sh, const TcPlan &tp, cudaStream_t s);

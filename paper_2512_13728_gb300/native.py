@@ -34,13 +34,18 @@ DION_PREC_BF16X3 = 2
 
 DION_MAX_RANK = 512
 
+DION_PHASE_NORMS = 1
+DION_PHASE_POWER = 2
+DION_PHASE_ORTHO = 3
+DION_PHASE_UPDATE = 4
+
 # Every function declared in include/curvadion.h.
 EXPORTED = ("dion_plan_create", "dion_step", "dion_get_device_status", "dion_plan_refresh", "dion_step_launch_count",
             "dion_timing_enable", "dion_timing_read", "dion_buffer_norms_noalloc", "dion_plan_destroy",
             "dion_status_string", "dion_abi_version", "dion_plan_enable_host_gradients", "dion_step_host",
-            "dion_lr_schedule", "dion_rank_for", "dion_plan_set_wait_limit")
+            "dion_lr_schedule", "dion_rank_for", "dion_plan_set_wait_limit", "dion_step_phase", "dion_plan_exchange")
 
-DION_ABI_VERSION = 2
+DION_ABI_VERSION = 3
 DION_NOALLOC_MAX_LAYERS = 256
 DION_NOALLOC_MAX_TILES = 65536
 
@@ -109,6 +114,10 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     lib.dion_timing_read.restype = C.c_int
     lib.dion_buffer_norms_noalloc.argtypes = [C.POINTER(dion_layer), C.c_int32, P, P, P]
     lib.dion_buffer_norms_noalloc.restype = C.c_int
+    lib.dion_step_phase.argtypes = [P, C.c_int32, C.POINTER(dion_hparams), P, P, P, P, P, P]
+    lib.dion_step_phase.restype = C.c_int
+    lib.dion_plan_exchange.argtypes = [P, C.c_int32, C.POINTER(P), C.POINTER(C.c_int64)]
+    lib.dion_plan_exchange.restype = C.c_int
     lib.dion_plan_set_wait_limit.argtypes = [P, C.c_int64]
     lib.dion_plan_set_wait_limit.restype = C.c_int
     lib.dion_plan_destroy.argtypes = [P]
@@ -150,6 +159,25 @@ def dion_step(plan: int, hp: dion_hparams, prev_norm: int, rmmc_out: int, rmmc_e
                           C.c_void_p(global_flag_out), C.c_void_p(stream) if stream else None)
     if st != DION_OK:
         raise DionError(st, "dion_step")
+
+
+def dion_step_phase(plan: int, phase: int, hp: dion_hparams, prev_norm: int, rmmc_out: int, rmmc_eq1_out,
+                    sync_flags_out: int, global_flag_out: int, stream: int) -> None:
+    """One phase (DION_PHASE_*) of a data-parallel step; pointers as in dion_step."""
+    st = load().dion_step_phase(C.c_void_p(plan), int(phase), C.byref(hp), C.c_void_p(prev_norm), C.c_void_p(rmmc_out),
+                                C.c_void_p(rmmc_eq1_out) if rmmc_eq1_out else None, C.c_void_p(sync_flags_out),
+                                C.c_void_p(global_flag_out), C.c_void_p(stream) if stream else None)
+    if st != DION_OK:
+        raise DionError(st, "dion_step_phase")
+
+
+def dion_plan_exchange(plan: int, phase: int):
+    """(device address, fp32 element count) of the range a worker averages after `phase`."""
+    buf, cnt = C.c_void_p(), C.c_int64(0)
+    st = load().dion_plan_exchange(C.c_void_p(plan), int(phase), C.byref(buf), C.byref(cnt))
+    if st != DION_OK:
+        raise DionError(st, "dion_plan_exchange")
+    return buf.value or 0, int(cnt.value)
 
 
 def dion_lr_schedule(step: int, total_steps: int, base_lr: float, warmup_frac: float, warmdown_frac: float) -> float:

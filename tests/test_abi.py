@@ -45,7 +45,7 @@ def test_exported_symbols_via_nm(lib):
 def test_abi_version_and_status_strings(lib):
     from paper_2512_13728_gb300 import native
 
-    assert native.dion_abi_version() == native.DION_ABI_VERSION == 2
+    assert native.dion_abi_version() == native.DION_ABI_VERSION == 3
     for code in range(8):
         assert native.dion_status_string(code).startswith("DION_")
     assert "unknown" in native.dion_status_string(99)
@@ -154,3 +154,15 @@ def test_wait_limit_rejects_null_plan(lib):
     from paper_2512_13728_gb300 import native
 
     assert lib.dion_plan_set_wait_limit(None, C.c_int64(5)) == native.DION_ERR_INVALID_ARG
+
+
+def test_phase_entry_points_reject_bad_arguments(lib):
+    from paper_2512_13728_gb300 import native
+
+    hp = native.dion_hparams(mu=0.95, eta=0.01, eta_local=0.01, eps_rmmc=1e-8, eps_col=1e-8, tau_global=0.5,
+                             gate_mode=0, period=1, step=1)
+    assert lib.dion_step_phase(None, native.DION_PHASE_NORMS, C.byref(hp), None, None, None, None, None,
+                               None) == native.DION_ERR_INVALID_ARG
+    buf, cnt = C.c_void_p(), C.c_int64(0)
+    assert lib.dion_plan_exchange(None, native.DION_PHASE_POWER, C.byref(buf), C.byref(cnt)) == \
+        native.DION_ERR_INVALID_ARG
