@@ -44,6 +44,16 @@ def load_peaks():
     return dict(hbm=6800.0, bf16=1900.0, bf16_sust=1700.0, sm_mhz=2070.0, source="fallback")
 
 
+def load_tf32_peak():
+    """cuBLAS tf32 throughput measured on this machine's GB300 (`bench.py --tf32-peak`), else half of
+    the bf16 peak (the nominal ratio)."""
+    path = os.path.join(ROOT, "profiles", "tf32_peak.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            return float(json.load(f)["tf32_tflops"]), "measured"
+    return load_peaks()["bf16"] / 2, "half of bf16"
+
+
 def sources_hash(names) -> str:
     """Hash of the listed files under the package's csrc/ (the translation unit of one kernel and
     its host-side schedule), so a stored ncu counter stays valid until that code changes."""
@@ -77,6 +87,7 @@ def kernel_work(name: str, w, prec: str, gate: str = "always", wt=None):
     mn_loc = mn_all - mn
     mnr = tot(lambda m, n, r: m * n * r)
     mr2 = tot(lambda m, n, r: m * r * r)
+    mrr1 = tot(lambda m, n, r: m * r * (r + 1))  # a symmetric Gram or a triangular solve: 2 m r (r + 1) / 2
     r3 = tot(lambda m, n, r: r ** 3)
     nr = tot(lambda m, n, r: n * r)
     mr = tot(lambda m, n, r: m * r)
@@ -112,10 +123,17 @@ def kernel_work(name: str, w, prec: str, gate: str = "always", wt=None):
         "tc_btp": ("hbm", mn * bh + mr * 2 * hl + nr * (4 + 2 * hl), "B"),  # Bh (Bl), bf16 P; R fp32, bf16
         "split_p": ("hbm", mr * 8, "B"),  # read P fp32; write its two bf16 halves
         "tc_update": ("hbm", mn * (16 + (gsz if deferred else 0)), "B"),
-        "tc_gram": ("tensor", 2 * mr2, "flop"),
-        "tc_trsm": ("tensor", 2 * mr2, "flop"),
+        "tc_gram": ("tf32", mrr1, "flop"),
+        "tc_trsm": ("tf32", mrr1, "flop"),
     }
-    return table.get(name, ("latency", 0, ""))
+    # Orthogonalize's launches carry their pass: passes 0 and 1 run the Gram and the solve on
+    # every synchronizing layer; pass 1's factor is usually the first-order one and pass 2 runs
+    # only after a shifted retry, so those count as latency
+    base = name.rstrip("0123456789")
+    npass = int(name[len(base):]) if len(base) < len(name) else 0
+    if npass == 2 or (base == "chol_inv" and npass == 1):
+        return ("latency", 0, "")
+    return table.get(base, ("latency", 0, ""))
 
 
 def step_bytes(w, prec, gate: str = "always", wt=None):
@@ -254,6 +272,23 @@ def max_over_ranks(value: float, world: int, device) -> float:
     t = torch.tensor([float(value)], device=device, dtype=torch.float64)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def kernel_frac(k, peaks):
+    """{"bound", "frac"} of one kernel's measured time against its roofline (HBM copy, bf16 or
+    tf32 tensor throughput), or {} for latency-bound kernels."""
+    if k["ms"] <= 0 or not k["units"]:
+        return {}
+    rate = k["units"] / (k["ms"] * 1e-3)
+    if k["bound"] == "hbm":
+        return {"bound": "hbm", "frac": round(rate / 1e9 / peaks["hbm"], 4)}
+    if k["bound"] == "tensor":
+        return {"bound": "bf16", "frac": round(rate / 1e12 / peaks["bf16_sust"], 4)}
+    if k["bound"] == "tf32":
+        return {"bound": "tf32", "frac": round(rate / 1e12 / load_tf32_peak()[0], 4)}
+    if k["bound"] == "alu":
+        return {"bound": "fp32 FFMA", "frac": round(rate / 1e12 / (152 * 128 * 2 * peaks["sm_mhz"] * 1e6 / 1e12), 4)}
+    return {}
 
 
 def run_ours(args, rank, world, local_rank):
@@ -412,6 +447,8 @@ def run_ours(args, rank, world, local_rank):
             peak, punit, achieved = peaks["hbm"], "GB/s", dom["units"] / (dom["ms"] * 1e-3) / 1e9
         elif dom["bound"] == "tensor":
             peak, punit, achieved = peaks["bf16_sust"], "TFLOP/s", dom["units"] / (dom["ms"] * 1e-3) / 1e12
+        elif dom["bound"] == "tf32":
+            peak, punit, achieved = load_tf32_peak()[0], "TFLOP/s", dom["units"] / (dom["ms"] * 1e-3) / 1e12
         else:  # fp32 FFMA on CUDA cores: 152 SMs x 128 lanes x 2 flop x max SM clock
             peak = 152 * 128 * 2 * peaks["sm_mhz"] * 1e6 / 1e12
             punit, achieved = "TFLOP/s", dom["units"] / (dom["ms"] * 1e-3) / 1e12
@@ -445,7 +482,7 @@ def run_ours(args, rank, world, local_rank):
         "e2e": {"value": round(e2e_ms, 4), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": launches * args.steps,
         "clocks": clocks,
-        "kernels": [{"name": k["name"], "ms": round(k["ms"], 4)} for k in kern],
+        "kernels": [dict(name=k["name"], ms=round(k["ms"], 4), **kernel_frac(k, peaks)) for k in kern],
         "timed_steps_with_kernel_events": nsteps_timed,
     }
     return line
@@ -509,6 +546,29 @@ def run_reference(args, rank):
             "e2e": {"value": round(ms, 1), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
+def measure_tf32_peak():
+    """Dense tf32 throughput of cuBLAS on this GPU, measured the way the bf16 peak is: an
+    8192^3 fp32 GEMM with tf32 tensor cores allowed, best of 10 (CUDA events), 2 N^3 flops."""
+    import torch
+
+    torch.backends.cuda.matmul.allow_tf32 = True
+    n = 8192
+    a = torch.randn(n, n, device="cuda")
+    b = torch.randn(n, n, device="cuda")
+    for _ in range(3):
+        a @ b
+    best = math.inf
+    for _ in range(10):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        a @ b
+        e1.record()
+        torch.cuda.synchronize()
+        best = min(best, e0.elapsed_time(e1))
+    return {"tf32_tflops": round(2 * n ** 3 / (best * 1e-3) / 1e12, 1), "n": n, "best_ms": round(best, 4),
+            "how": "torch.matmul fp32 8192^3 with allow_tf32 (cuBLAS), best of 10, CUDA events"}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -522,7 +582,11 @@ def main():
     ap.add_argument("--t0", type=int, default=1, help="index of the first (warm-up) step: gradients G_t and "
                     "the step number t start there")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--tf32-peak", action="store_true", help="print the measured cuBLAS tf32 throughput and exit")
     args = ap.parse_args()
+    if args.tf32_peak:
+        print(json.dumps(measure_tf32_peak()), flush=True)
+        return
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.precision is None:
