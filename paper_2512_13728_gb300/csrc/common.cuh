@@ -152,6 +152,10 @@ void launch_gemm(const Shared &sh, const GemmProblem *probs, const int4 *tiles, 
 cudaError_t prepare_chol_inv(int32_t max_r, size_t *smem_out);
 // near_identity: Frobenius bound on S - I below which passes 1 and 2 use the first-order factor
 void launch_chol_inv(const Shared &sh, size_t smem, int32_t pass, float near_identity, cudaStream_t s);
+// the first CholeskyQR pass with the trailing update on tensor cores (chol_tc.cu, BF16 mode)
+cudaError_t prepare_chol_inv_tc(int32_t max_r, size_t *smem_out);
+namespace tc { struct LayerMaps; }
+void launch_chol_inv_tc(const Shared &sh, const tc::LayerMaps *maps, size_t smem, cudaStream_t s);
 void launch_colnorm(const Shared &sh, const int4 *tiles, int32_t ntiles, float eps_col,
                     cudaStream_t s);
 void launch_update(const Shared &sh, const int4 *tiles, int32_t ntiles, float mu, float eta, float keep,

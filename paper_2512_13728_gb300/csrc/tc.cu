@@ -553,6 +553,7 @@ cudaError_t encode_maps(const DevLayer *dl, int32_t L, LayerMaps *dst) {
                     encode_f32_2d(&m.PT_t, d.PT, d.m, d.r, (uint64_t)d.ldmt * 4, 32, 32) &&
                     encode_f32_2d(&m.Sst, d.S, d.r, d.r, p32, 32, 128) &&
                     encode_f32_2d(&m.Linv, d.Linv, d.r, d.r, p32, 32, 128) &&
+                    encode_f32_2d(&m.Linv32, d.Linv, d.r, d.r, p32, 32, 32) &&
                     (d.P_lo == nullptr ||
                      (encode_bf16_2d(&m.P_lo, d.P_lo, d.r, d.m, p16, 64, 128) &&
                       encode_bf16_2d(&m.R_lo, d.R_lo, d.r, d.n, p16, 64, 128) &&
@@ -626,6 +627,7 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   if (tp->fuse_buffer && tp->fb_smem > 227u * 1024u) return cudaErrorInvalidValue;
   if (e == cudaSuccess && tp->fuse_buffer) e = setup_fused_bq_kernel(tp->fb_smem);
   if (e == cudaSuccess) e = setup_orth_kernels(tp->o_smem);
+  if (e == cudaSuccess && !x3) e = prepare_chol_inv_tc(lo.max_r, &tp->chol_tc_smem);
   int dev = 0, sms = 0;
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -682,7 +684,8 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh_in, const StepArgs &a
     for (int pass = 0; pass < 3; ++pass) {  // CholeskyQR2; the third pass only after a shifted retry
       launch_orth(sh, tp, true, pass, s);  // S = X^T X
       tick(p, s, kGram[pass]);
-      launch_chol_inv(sh, chol_smem, pass, 6e-2f, s);  // L, L^{-1}
+      if (pass == 0) launch_chol_inv_tc(sh, tp.maps, tp.chol_tc_smem, s);  // L, L^{-1} (trailing update on tensor cores)
+      else launch_chol_inv(sh, chol_smem, pass, 6e-2f, s);        // usually the first-order factor
       tick(p, s, kChol[pass]);
       launch_orth(sh, tp, false, pass, s);  // X L^{-T} and its transpose, or its bf16 copy at the end
       tick(p, s, kTrsm[pass]);
@@ -742,7 +745,8 @@ void step_phase(const TcPlan &tp, const Shared &sh_in, const StepArgs &a, int32_
         launch_transpose_praw(sh, tp, s);  // the first Gram reads P_raw^T
         for (int pass = 0; pass < 3; ++pass) {
           launch_orth(sh, tp, true, pass, s);
-          launch_chol_inv(sh, chol_smem, pass, 6e-2f, s);
+          if (pass == 0) launch_chol_inv_tc(sh, tp.maps, tp.chol_tc_smem, s);
+          else launch_chol_inv(sh, chol_smem, pass, 6e-2f, s);
           launch_orth(sh, tp, false, pass, s);
         }
       }

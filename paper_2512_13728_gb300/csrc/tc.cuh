@@ -35,6 +35,7 @@ struct LayerMaps {
   CUtensorMap PT_t;     // r x m fp32: box {32, 32}  transposed output store
   CUtensorMap Sst;    // r x r fp32:  box {32, 128}  Gram output
   CUtensorMap Linv;   // r x r fp32:  box {32, 128}  TRSM B operand (rows of L^{-1})
+  CUtensorMap Linv32; // r x r fp32:  box {32, 32}   Cholesky trailing update (reduce-add)
   // BF16X3: the low halves, boxes as their high counterparts (zeroed maps in the other modes)
   CUtensorMap P_lo, R_lo, Qn_lo;  // K-major {64, 128}: update operands
   CUtensorMap Qn_lo_mn, P_lo_mn, Bl_mn;  // MN-major {64, 64}: B Q / B^T P operands
@@ -95,6 +96,7 @@ struct TcPlan {
   int32_t launches = 0;
   bool fuse_buffer = false;
   uint32_t fb_smem = 0;
+  size_t chol_tc_smem = 0;  // the first pass's Cholesky on tensor cores (BF16 mode)
   // CUDA-core pieces reused by this path (set by the plan)
   const GemmProblem *const *probs = nullptr;
   const int4 *const *gtiles = nullptr;

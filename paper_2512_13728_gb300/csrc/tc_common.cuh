@@ -258,6 +258,16 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, const void 
                : "memory");
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// Element-wise add of a shared-memory box into the tensor's box at {c0, c1} (fp32 add in L2;
+// out-of-range rows and columns are skipped), completed through the bulk async-group.
+__device__ __forceinline__ void tma_reduce_add_2d(const CUtensorMap *map, const void *src, int32_t c0, int32_t c1) {
+  asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(smem_u32(src)), "r"(c0), "r"(c1)
+               : "memory");
+}
+// Orders this thread's generic-proxy global accesses with async-proxy (TMA) accesses, both ways.
+__device__ __forceinline__ void fence_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
 
 // ------------------------------------------- per-thread async copies (load/store path) ---
 // 16-byte global -> shared copy through L2 (not L1); bytes past src_bytes (0..16) are zero.
