@@ -48,7 +48,9 @@ typedef enum {
   DION_ERR_CUDA = 4,         /* a CUDA runtime call failed (no device, launch error, OOM) */
   DION_ERR_BREAKDOWN = 5,    /* device: Cholesky pivot <= 0 or non-finite (rank-deficient P) */
   DION_ERR_NONFINITE = 6,    /* device: ||B|| is not finite for some layer */
-  DION_ERR_TIMEOUT = 7       /* device: a bounded wait gave up */
+  DION_ERR_TIMEOUT = 7,      /* device: a bounded wait gave up */
+  DION_ERR_CORRUPT = 8       /* device: a workspace guard was overwritten, or (debug build) a
+                              * kernel was given a tile outside its layer */
 } dion_status;
 
 /* Which layers run the synchronized Dion branch (Algorithm 1 body) in a step. */
@@ -274,6 +276,18 @@ dion_status dion_buffer_norms_noalloc(const dion_layer *layers, int32_t num_laye
  * of a few nanoseconds the first wait that does not succeed at once gives up.  Host only;
  * takes effect from the next dion_step.  Errors: INVALID_ARG (NULL plan). */
 dion_status dion_plan_set_wait_limit(dion_plan *plan, int64_t limit_ns);
+
+/* Workspace guards (memory-safety check; no counterpart in the paper).  Every region the plan
+ * carves from its workspace is followed by 64 guard words of a fixed pattern, written at
+ * creation.  dion_plan_check_guards synchronizes the device, counts the guard words that no
+ * longer hold their pattern into *damaged_out (0 when no kernel wrote past a region) and
+ * changes nothing.  Errors: INVALID_ARG (NULL argument), CUDA.
+ * A library built with DION_DEBUG_CHECKS (dion_debug_checks() returns 1; built as
+ * libcurvadion_debug.so) also checks the guards at the end of every step and checks every tile
+ * a kernel decodes against its layer's shape; either failure sets DION_ERR_CORRUPT in the
+ * status word, and a bad tile is skipped.  Such a step launches one more kernel. */
+dion_status dion_plan_check_guards(dion_plan *plan, int32_t *damaged_out);
+int32_t dion_debug_checks(void);
 
 /* Frees the plan's workspace (synchronizes the device first).  NULL is a no-op. */
 void dion_plan_destroy(dion_plan *plan);

@@ -146,6 +146,10 @@ class Plan:
     def device_status(self, clear: bool = True) -> int:
         return native.dion_get_device_status(self.handle, clear)
 
+    def check_guards(self) -> int:
+        """Damaged workspace guard words (synchronizes the device)."""
+        return native.dion_plan_check_guards(self.handle)
+
     def launches_per_step(self) -> int:
         return native.dion_step_launch_count(self.handle)
 

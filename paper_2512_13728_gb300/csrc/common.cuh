@@ -20,7 +20,32 @@ enum : int32_t {
   ST_BREAKDOWN = 5,
   ST_NONFINITE = 6,
   ST_TIMEOUT = 7,
+  ST_CORRUPT = 8,
 };
+
+// Workspace guards: every region carved from a plan's workspace is followed by kGuardWords
+// 32-bit words of a fixed pattern (guard_fill), checked by guard_check.
+constexpr int kGuardWords = 64;
+void launch_guard_fill(char *base, const uint64_t *offsets, int32_t n, cudaStream_t s);
+// Counts damaged guard words into *bad (device) and, when status is not null, sets ST_CORRUPT there.
+void launch_guard_check(const char *base, const uint64_t *offsets, int32_t n, int32_t *bad, int32_t *status,
+                        cudaStream_t s);
+
+// DION_DEBUG_CHECKS builds check every tile a kernel decodes against its layer's shape; a bad
+// tile sets ST_CORRUPT and the block returns.  Other builds compile the checks away.
+#ifdef DION_DEBUG_CHECKS
+#define DION_TILE_CHECK(cond, status)        \
+  do {                                       \
+    if (!(cond)) {                           \
+      atomicCAS((status), 0, (int32_t)ST_CORRUPT); \
+      return;                                \
+    }                                        \
+  } while (0)
+#else
+#define DION_TILE_CHECK(cond, status) \
+  do {                                \
+  } while (0)
+#endif
 
 enum : int32_t { GATE_ALWAYS = 0, GATE_GLOBAL = 1, GATE_PER_LAYER = 2, GATE_SCHEDULED = 3 };
 enum : int32_t { DT_FP32 = 0, DT_BF16 = 1 };

@@ -91,7 +91,9 @@ __device__ void form_b_tile(const DevLayer &L, int64_t row0, int64_t nrows, floa
 __global__ void __launch_bounds__(kRowThreads) form_b_kernel(Shared sh, const int4 *tiles) {
   __shared__ double red[kRowThreads / 32];
   const int4 t = tiles[blockIdx.x];
+  DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers, sh.status);
   const DevLayer &L = sh.layers[t.x];
+  DION_TILE_CHECK(t.y >= 0 && t.z >= 1 && (int64_t)t.y + t.z <= L.m, sh.status);
   float sb[4] = {0.f, 0.f, 0.f, 0.f}, sm[4] = {0.f, 0.f, 0.f, 0.f};
   if (L.Bh != nullptr) {
     if (L.g_dtype == DT_BF16) form_b_tile<DT_BF16, true>(L, t.y, t.z, sb, sm);
@@ -318,7 +320,9 @@ __global__ void __launch_bounds__(kNormThreads) norms_gate_kernel(Shared sh, Ste
   __shared__ int last_s, count_s;
   __shared__ double max_s[kNormThreads / 32];
   const int4 t = tiles[blockIdx.x];  // {layer, 128-row block}
+  DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers, sh.status);
   const DevLayer &L = sh.layers[t.x];
+  DION_TILE_CHECK(t.y >= 0 && (int64_t)t.y * 128 < L.m, sh.status);
   const int64_t row0 = (int64_t)t.y * 128, nrows = min((int64_t)128, L.m - row0);
   float sb[4] = {0.f, 0.f, 0.f, 0.f}, sm[4] = {0.f, 0.f, 0.f, 0.f};
   if (L.g_dtype == DT_BF16) norms_tile<DT_BF16>(L, row0, nrows, sb, sm);
@@ -367,6 +371,8 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_kernel(Shared sh, const Gem
                                                             const int4 *tiles) {
   const int4 t = tiles[blockIdx.x];
   const GemmProblem p = probs[t.x];
+  DION_TILE_CHECK(p.layer >= 0 && p.layer < sh.num_layers && t.y >= 0 && t.z >= 0 &&
+                      (int64_t)t.y * GBM < p.Mrows && (int64_t)t.z * GBN < p.Ncols, sh.status);
   if (!sh.active[p.layer]) return;
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
   const int64_t i0 = (int64_t)t.y * GBM, j0 = (int64_t)t.z * GBN;
@@ -799,6 +805,7 @@ constexpr int kColThreads = 256;
 
 __global__ void __launch_bounds__(kColThreads) colnorm_kernel(Shared sh, const int4 *tiles, float eps_col) {
   const int4 t = tiles[blockIdx.x];
+  DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers && t.y >= 0 && (int64_t)t.y * 32 < sh.layers[t.x].r, sh.status);
   if (!sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -854,6 +861,8 @@ __global__ void __launch_bounds__(kUpdThreads) update_kernel(Shared sh, const in
   __shared__ float Qs[UBK][UBN + 4];
   __shared__ double red[kUpdThreads / 32];
   const int4 t = tiles[blockIdx.x];
+  DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers && t.y >= 0 && t.z >= 0 &&
+                      (int64_t)t.y * UBM < sh.layers[t.x].m && (int64_t)t.z * UBN < sh.layers[t.x].n, sh.status);
   if (!sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
@@ -949,6 +958,8 @@ __device__ void local_tile(const DevLayer &L, int64_t row0, int64_t nrows, float
 
 __global__ void __launch_bounds__(kRowThreads) local_kernel(Shared sh, const int4 *tiles, float eta_local, float keep) {
   const int4 t = tiles[blockIdx.x];
+  DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers && t.y >= 0 && t.z >= 1 &&
+                      (int64_t)t.y + t.z <= sh.layers[t.x].m, sh.status);
   if (sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
   if (L.g_dtype == DT_BF16) local_tile<DT_BF16>(L, t.y, t.z, eta_local, keep, sh.b_in_m != 0);

@@ -39,6 +39,10 @@ struct dion_plan {
   size_t xp_off = 0, xr_off = 0;
   int64_t xp_count = 0, xr_count = 0;
   int32_t next_phase = DION_PHASE_NORMS;
+  // workspace guards (device list of offsets, damaged-word counter)
+  uint64_t *guard_off = nullptr;
+  int32_t *guard_bad = nullptr;
+  int32_t n_guards = 0;
   // per-launch timing (dion_timing_enable)
   std::vector<cudaEvent_t> ev;  // [max_steps][launches + 1]
   std::vector<const char *> names;
@@ -86,14 +90,23 @@ namespace {
 constexpr size_t kAlign = 256;
 constexpr uint64_t kDefaultWaitLimitNs = 2000000000ull;  // the bounded waits' default: 2 s
 
+// Carves the workspace: 256-byte aligned regions, each followed (unless guard = false) by
+// kGuardWords guard words whose offsets are recorded.
 struct Carver {
   size_t off = 0;
+  std::vector<uint64_t> guards;
   template <class T>
-  size_t take(size_t count) {
+  size_t take(size_t count, bool guard = true) {
     off = (off + kAlign - 1) / kAlign * kAlign;
     const size_t at = off;
     off += count * sizeof(T);
+    if (guard) add_guard();
     return at;
+  }
+  void add_guard() {
+    off = (off + 3) / 4 * 4;
+    guards.push_back(off);
+    off += kGuardWords * sizeof(uint32_t);
   }
 };
 
@@ -140,6 +153,7 @@ const char *dion_status_string(dion_status s) {
     case DION_ERR_BREAKDOWN: return "DION_ERR_BREAKDOWN: Cholesky breakdown (rank-deficient P)";
     case DION_ERR_NONFINITE: return "DION_ERR_NONFINITE: non-finite buffer norm";
     case DION_ERR_TIMEOUT: return "DION_ERR_TIMEOUT: bounded device wait gave up";
+    case DION_ERR_CORRUPT: return "DION_ERR_CORRUPT: workspace guard overwritten or tile out of range";
   }
   return "unknown dion_status";
 }
@@ -174,8 +188,13 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
   std::vector<int4> bt, ut, ct;
   // P_raw and R of all layers each in one contiguous range (256-byte gaps between layers): the
   // buffers a data-parallel caller averages between the phases of dion_step_phase
-  for (int32_t l = 0; l < num_layers; ++l) o_Praw[l] = cv.take<float>(layers[l].m * ((layers[l].r + 7) / 8 * 8));
-  for (int32_t l = 0; l < num_layers; ++l) o_R[l] = cv.take<float>(layers[l].n * ((layers[l].r + 7) / 8 * 8));
+  // (no guards inside them: a caller's average of equal words is exact, but not every reduction is)
+  for (int32_t l = 0; l < num_layers; ++l)
+    o_Praw[l] = cv.take<float>(layers[l].m * ((layers[l].r + 7) / 8 * 8), false);
+  if (num_layers > 0) cv.add_guard();
+  for (int32_t l = 0; l < num_layers; ++l)
+    o_R[l] = cv.take<float>(layers[l].n * ((layers[l].r + 7) / 8 * 8), false);
+  if (num_layers > 0) cv.add_guard();
   if (num_layers > 0) {
     const dion_layer &a = layers[num_layers - 1];
     const int64_t lp = (a.r + 7) / 8 * 8;
@@ -246,6 +265,7 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
       return st;
     }
     cv.off = tcl.end;
+    cv.guards.insert(cv.guards.end(), tcl.guards.begin(), tcl.guards.end());
   }
   const size_t o_shift = cv.take<uint8_t>(std::max(num_layers, 1));
   size_t o_gp[kSets], o_gt[kSets];
@@ -275,6 +295,10 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
     o_gt[k] = cv.take<int4>(std::max<size_t>(gt[k].size(), 1));
   }
 
+  // the guard list itself and the check's counter come last, unguarded
+  const size_t o_guards = cv.take<uint64_t>(std::max<size_t>(cv.guards.size(), 1), false);
+  const size_t o_gbad = cv.take<int32_t>(1, false);
+  p->n_guards = (int32_t)cv.guards.size();
   if (cudaMalloc(&p->ws, cv.off) != cudaSuccess) {
     delete p;
     return DION_ERR_CUDA;
@@ -321,6 +345,10 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
 
   // zeroed once, so the gaps and row padding inside the exchange ranges hold zeros
   cudaError_t e = cudaMemset(p->ws, 0, cv.off);
+  p->guard_off = reinterpret_cast<uint64_t *>(base + o_guards);
+  p->guard_bad = reinterpret_cast<int32_t *>(base + o_gbad);
+  if (e == cudaSuccess) e = upload(p->guard_off, cv.guards);
+  if (e == cudaSuccess) launch_guard_fill(base, p->guard_off, p->n_guards, nullptr);
   if (e == cudaSuccess) e = upload(p->sh.layers, dl);
   p->dl_host = dl;
   if (e == cudaSuccess) e = upload(p->btiles, bt);
@@ -350,6 +378,9 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
     return DION_ERR_CUDA;
   }
   p->launches_per_step = (precision == DION_PREC_FP32) ? 17 : tc::launches_per_step(p->tcp);
+#ifdef DION_DEBUG_CHECKS
+  p->launches_per_step += 1;  // the guard check at the end of every step
+#endif
   *out = p;
   return DION_OK;
 }
@@ -424,6 +455,10 @@ void enqueue_step(dion_plan *p, const Shared &sh, const tc::TcPlan &tcp, const d
   } else {
     tc::step(p, tcp, sh, a, p->btiles, p->n_btiles, p->ctiles, p->n_ctiles, p->chol_smem, s);
   }
+#ifdef DION_DEBUG_CHECKS
+  launch_guard_check(static_cast<const char *>(p->ws), p->guard_off, p->n_guards, p->guard_bad, sh.status, s);
+  tick(p, s, "guard_check");
+#endif
   tick_end(p);
 }
 
@@ -500,6 +535,11 @@ dion_status dion_step_phase(dion_plan *p, int32_t phase, const dion_hparams *hp,
   if (!g.ok) return DION_ERR_CUDA;
   const StepArgs a = make_args(hp, prev_norm, rmmc_out, rmmc_eq1_out, sync_flags_out, global_flag_out);
   enqueue_phase(p, a, phase, static_cast<cudaStream_t>(stream));
+#ifdef DION_DEBUG_CHECKS
+  if (phase == DION_PHASE_UPDATE)
+    launch_guard_check(static_cast<const char *>(p->ws), p->guard_off, p->n_guards, p->guard_bad, p->sh.status,
+                       static_cast<cudaStream_t>(stream));
+#endif
   if (cudaGetLastError() != cudaSuccess) return DION_ERR_CUDA;
   p->next_phase = (phase == DION_PHASE_UPDATE) ? DION_PHASE_NORMS : phase + 1;
   return DION_OK;
@@ -658,6 +698,28 @@ dion_status dion_get_device_status(dion_plan *p, int32_t clear, int32_t *code_ou
 }
 
 int32_t dion_step_launch_count(const dion_plan *p) { return p ? p->launches_per_step : 0; }
+
+dion_status dion_plan_check_guards(dion_plan *p, int32_t *damaged_out) {
+  if (!p || !damaged_out) return DION_ERR_INVALID_ARG;
+  DeviceGuard g(p->device);
+  if (!g.ok) return DION_ERR_CUDA;
+  if (cudaDeviceSynchronize() != cudaSuccess || cudaMemset(p->guard_bad, 0, sizeof(int32_t)) != cudaSuccess)
+    return DION_ERR_CUDA;
+  launch_guard_check(static_cast<const char *>(p->ws), p->guard_off, p->n_guards, p->guard_bad, nullptr, nullptr);
+  int32_t v = 0;
+  if (cudaGetLastError() != cudaSuccess || cudaMemcpy(&v, p->guard_bad, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return DION_ERR_CUDA;
+  *damaged_out = v;
+  return DION_OK;
+}
+
+int32_t dion_debug_checks(void) {
+#ifdef DION_DEBUG_CHECKS
+  return 1;
+#else
+  return 0;
+#endif
+}
 
 dion_status dion_plan_set_wait_limit(dion_plan *p, int64_t limit_ns) {
   if (!p) return DION_ERR_INVALID_ARG;

@@ -362,10 +362,13 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
   TcLayout &lo = *out;
   lo.precision = precision;
   size_t off = start;
-  auto take = [&](size_t bytes, size_t align = 256) {
+  auto take = [&](size_t bytes, size_t align = 256) {  // a region and its guard words
     off = (off + align - 1) / align * align;
     const size_t at = off;
     off += bytes;
+    off = (off + 3) / 4 * 4;
+    lo.guards.push_back(off);
+    off += kGuardWords * sizeof(uint32_t);
     return at;
   };
   lo.o_phi.resize(L);

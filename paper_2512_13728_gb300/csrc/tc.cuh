@@ -57,6 +57,7 @@ struct TcLayout {
   size_t o_utiles = 0, o_ftiles = 0, o_rtiles = 0, o_qtiles = 0, o_gtiles = 0, o_ttiles = 0;
   std::vector<size_t> o_phi, o_rhi, o_qnhi, o_bh, o_ptraw, o_pt, o_colsq, o_colinv;
   std::vector<size_t> o_bl, o_plo, o_rlo, o_qnlo;  // BF16X3 low halves
+  std::vector<uint64_t> guards;  // offsets of the guard words after each region
   std::vector<int4> gram_tiles, trsm_tiles;
   // update tiles {layer, m-block, n-block, slot}; P-convert tiles {layer, row0, rows, 0};
   // B Q tiles {layer, m-block, 0, slot}; B^T P tiles {layer, n-block, 0, 0}; Q-copy tiles

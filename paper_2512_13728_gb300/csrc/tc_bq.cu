@@ -707,6 +707,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(FB_THREADS, 1)
 // ================================================================== Q -> bf16 copy ===
 __global__ void __launch_bounds__(256) qn_refresh_kernel(Shared sh, const int4 *tiles) {
   const int4 t = tiles[blockIdx.x];  // {layer, first row, rows, 0}
+  DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers && t.y >= 0 && t.z >= 1 &&
+                      (int64_t)t.y + t.z <= sh.layers[t.x].n, sh.status);
   const DevLayer &L = sh.layers[t.x];
   const int64_t r = L.r, total = (int64_t)t.z * r;
   for (int64_t e = threadIdx.x; e < total; e += 256) {
@@ -722,6 +724,7 @@ __global__ void __launch_bounds__(256) qn_refresh_kernel(Shared sh, const int4 *
 // the update.  Tile = {layer, 128-row block}; a warp per row, 8-byte stores.
 __global__ void __launch_bounds__(256) split_p_kernel(Shared sh, const int4 *tiles) {
   const int4 t = tiles[blockIdx.x];
+  DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers && t.y >= 0 && (int64_t)t.y * 128 < sh.layers[t.x].m, sh.status);
   if (!sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -805,6 +808,7 @@ void launch_btp(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
 // tile = {layer, 128-row block of P_raw}, 32 x 32 sub-tiles through shared memory.
 __global__ void __launch_bounds__(256) transpose_praw_kernel(Shared sh, const int4 *tiles) {
   const int4 t = tiles[blockIdx.x];
+  DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers && t.y >= 0 && (int64_t)t.y * 128 < sh.layers[t.x].m, sh.status);
   if (!sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
   __shared__ float tile[32][33];
@@ -831,6 +835,7 @@ __global__ void __launch_bounds__(256) transpose_praw_kernel(Shared sh, const in
 // takes columns j and j + 256, rows in order (fp32 over 32 rows, then fp64).
 __global__ void __launch_bounds__(256) r_refresh_kernel(Shared sh, const int4 *tiles) {
   const int4 t = tiles[blockIdx.x];
+  DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers && t.y >= 0 && (int64_t)t.y * 128 < sh.layers[t.x].n, sh.status);
   if (!sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
   const int64_t r0 = (int64_t)t.y * 128, r1 = min(r0 + 128, L.n);
@@ -868,6 +873,7 @@ void launch_qn_refresh(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
 // fixed-order fp64 sum over the R tiles of the layer.  Grid: one block per (layer, 32 columns).
 __global__ void __launch_bounds__(256) colnorm_reduce_kernel(Shared sh, const int4 *ctiles, float eps_col) {
   const int4 t = ctiles[blockIdx.x];  // {layer, 32-column group, 0, 0}
+  DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers && t.y >= 0 && (int64_t)t.y * 32 < sh.layers[t.x].r, sh.status);
   if (!sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -891,6 +897,8 @@ __global__ void __launch_bounds__(256) colnorm_reduce_kernel(Shared sh, const in
 constexpr int kScaleThreads = 256;
 __global__ void __launch_bounds__(kScaleThreads) colnorm_scale_kernel(Shared sh, const int4 *tiles) {
   const int4 t = tiles[blockIdx.x];  // {layer, first row, rows, 0}
+  DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers && t.y >= 0 && t.z >= 1 &&
+                      (int64_t)t.y + t.z <= sh.layers[t.x].n, sh.status);
   if (!sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -946,4 +954,39 @@ void launch_colnorm_scale(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
 }
 
 }  // namespace tc
+
+// ====================================================================== workspace guards ===
+__device__ __forceinline__ uint32_t guard_word(int64_t g, int w) {
+  return 0xA5A5A5A5u ^ (uint32_t)(g * kGuardWords + w);
+}
+__global__ void guard_fill_kernel(char *base, const uint64_t *offsets, int32_t n) {
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < (int64_t)n * kGuardWords;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t g = e / kGuardWords;
+    const int w = (int)(e % kGuardWords);
+    reinterpret_cast<uint32_t *>(base + offsets[g])[w] = guard_word(g, w);
+  }
+}
+__global__ void guard_check_kernel(const char *base, const uint64_t *offsets, int32_t n, int32_t *bad,
+                                   int32_t *status) {
+  int mine = 0;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < (int64_t)n * kGuardWords;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t g = e / kGuardWords;
+    const int w = (int)(e % kGuardWords);
+    mine += reinterpret_cast<const uint32_t *>(base + offsets[g])[w] != guard_word(g, w);
+  }
+  if (mine) {
+    atomicAdd(bad, mine);
+    if (status != nullptr) set_status(status, ST_CORRUPT);
+  }
+}
+void launch_guard_fill(char *base, const uint64_t *offsets, int32_t n, cudaStream_t s) {
+  if (n > 0) guard_fill_kernel<<<std::min(1024, (n * kGuardWords + 255) / 256), 256, 0, s>>>(base, offsets, n);
+}
+void launch_guard_check(const char *base, const uint64_t *offsets, int32_t n, int32_t *bad, int32_t *status,
+                        cudaStream_t s) {
+  if (n > 0)
+    guard_check_kernel<<<std::min(1024, (n * kGuardWords + 255) / 256), 256, 0, s>>>(base, offsets, n, bad, status);
+}
 }  // namespace cd

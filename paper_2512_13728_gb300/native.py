@@ -9,7 +9,8 @@ import ctypes as C
 import os
 
 PKG = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(PKG, "libcurvadion.so")
+# CURVADION_LIB selects another build of the same library (e.g. libcurvadion_debug.so)
+LIB_PATH = os.environ.get("CURVADION_LIB") or os.path.join(PKG, "libcurvadion.so")
 
 DION_OK = 0
 DION_ERR_INVALID_ARG = 1
@@ -19,6 +20,7 @@ DION_ERR_CUDA = 4
 DION_ERR_BREAKDOWN = 5
 DION_ERR_NONFINITE = 6
 DION_ERR_TIMEOUT = 7
+DION_ERR_CORRUPT = 8
 
 DION_GATE_ALWAYS = 0
 DION_GATE_GLOBAL = 1
@@ -43,7 +45,8 @@ DION_PHASE_UPDATE = 4
 EXPORTED = ("dion_plan_create", "dion_step", "dion_get_device_status", "dion_plan_refresh", "dion_step_launch_count",
             "dion_timing_enable", "dion_timing_read", "dion_buffer_norms_noalloc", "dion_plan_destroy",
             "dion_status_string", "dion_abi_version", "dion_plan_enable_host_gradients", "dion_step_host",
-            "dion_lr_schedule", "dion_rank_for", "dion_plan_set_wait_limit", "dion_step_phase", "dion_plan_exchange")
+            "dion_lr_schedule", "dion_rank_for", "dion_plan_set_wait_limit", "dion_step_phase", "dion_plan_exchange",
+            "dion_plan_check_guards", "dion_debug_checks")
 
 DION_ABI_VERSION = 3
 DION_NOALLOC_MAX_LAYERS = 256
@@ -118,6 +121,10 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     lib.dion_step_phase.restype = C.c_int
     lib.dion_plan_exchange.argtypes = [P, C.c_int32, C.POINTER(P), C.POINTER(C.c_int64)]
     lib.dion_plan_exchange.restype = C.c_int
+    lib.dion_plan_check_guards.argtypes = [P, C.POINTER(C.c_int32)]
+    lib.dion_plan_check_guards.restype = C.c_int
+    lib.dion_debug_checks.argtypes = []
+    lib.dion_debug_checks.restype = C.c_int32
     lib.dion_plan_set_wait_limit.argtypes = [P, C.c_int64]
     lib.dion_plan_set_wait_limit.restype = C.c_int
     lib.dion_plan_destroy.argtypes = [P]
@@ -253,6 +260,19 @@ def dion_buffer_norms_noalloc(layers, norm_b_out: int, norm_m_out: int, stream: 
                                           C.c_void_p(stream) if stream else None)
     if st != DION_OK:
         raise DionError(st, "dion_buffer_norms_noalloc")
+
+
+def dion_plan_check_guards(plan: int) -> int:
+    """Number of damaged workspace guard words (0 when no kernel wrote past its region)."""
+    out = C.c_int32(0)
+    st = load().dion_plan_check_guards(C.c_void_p(plan), C.byref(out))
+    if st != DION_OK:
+        raise DionError(st, "dion_plan_check_guards")
+    return int(out.value)
+
+
+def dion_debug_checks() -> bool:
+    return bool(load().dion_debug_checks())
 
 
 def dion_plan_set_wait_limit(plan: int, limit_ns: int) -> None:

@@ -46,7 +46,7 @@ def test_abi_version_and_status_strings(lib):
     from paper_2512_13728_gb300 import native
 
     assert native.dion_abi_version() == native.DION_ABI_VERSION == 3
-    for code in range(8):
+    for code in range(9):
         assert native.dion_status_string(code).startswith("DION_")
     assert "unknown" in native.dion_status_string(99)
 
@@ -166,3 +166,26 @@ def test_phase_entry_points_reject_bad_arguments(lib):
     buf, cnt = C.c_void_p(), C.c_int64(0)
     assert lib.dion_plan_exchange(None, native.DION_PHASE_POWER, C.byref(buf), C.byref(cnt)) == \
         native.DION_ERR_INVALID_ARG
+
+
+def test_guard_entry_points(lib):
+    from paper_2512_13728_gb300 import native
+
+    out = C.c_int32(0)
+    assert lib.dion_plan_check_guards(None, C.byref(out)) == native.DION_ERR_INVALID_ARG
+    assert lib.dion_debug_checks() == 0  # the default build has no debug checks
+
+
+def test_debug_build_reports_its_checks():
+    """The DION_DEBUG_CHECKS variant builds from the same sources and says so (loaded in a child
+    process, so this process keeps the default library)."""
+    import subprocess
+    import sys
+
+    from paper_2512_13728_gb300 import build
+
+    path = build.build(debug=True)
+    code = ("import ctypes; l = ctypes.CDLL(%r); l.dion_debug_checks.restype = ctypes.c_int32; "
+            "print(l.dion_debug_checks())") % path
+    out = subprocess.run([sys.executable, "-c", code], stdout=subprocess.PIPE, text=True, check=True).stdout
+    assert out.strip() == "1"
