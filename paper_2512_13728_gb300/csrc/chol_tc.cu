@@ -311,7 +311,10 @@ __global__ void __launch_bounds__(kThreads, 1) chol_inv_tc_kernel(Shared sh, con
     res = (trace_s > 0.0 && isfinite(trace_s)) ? chol_inverse_tc(S, Li, r, ls, (float)sft, D, DI, rd, &bad, ts, sh.status)
                                                : 1;
   }
-  if (tid == 0) sh.orth_shifted[l] = shifted ? 1 : 0;
+  if (tid == 0) {
+    sh.orth_shifted[l] = shifted ? 1 : 0;
+    if (shifted) atomicAdd(&sh.gate_scratch[kScratchShifted], 1ull);
+  }
   if (res != 0) {
     if ((tid & 31) == 0) bulk_wait<0>();  // reduce-adds issued before the failure
     if (tid == 0) {

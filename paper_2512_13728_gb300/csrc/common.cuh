@@ -107,7 +107,9 @@ struct StepArgs {
 };
 
 // Workspace shared by all kernels of a plan.
-constexpr int kScratchActive = 3;  // gate_scratch slot holding the count of Dion-branch layers
+constexpr int kScratchActive = 3;   // gate_scratch slot holding the count of Dion-branch layers
+constexpr int kScratchShifted = 4;  // gate_scratch slot: layers whose Cholesky took the shifted retry
+constexpr int kScratchSlots = 8;
 struct Shared {
   DevLayer *layers;
   int32_t num_layers;
@@ -118,9 +120,11 @@ struct Shared {
   double *norm_b;        // [L]
   int32_t *status;       // [1] first device error
   uint8_t *orth_shifted; // [L] 1 = a Cholesky pass of this step needed the shift (third pass runs)
-  // [4]: the gate's running max of RMMC (ordered key), its finished-block count, the norms
-  // pass's finished-block count, and (written by the gate) the number of layers that take the
-  // Dion branch this step, which lets the later persistent kernels return at once when it is 0
+  // [kScratchSlots]: the gate's running max of RMMC (ordered key), its finished-block count, the
+  // norms pass's finished-block count, (written by the gate) the number of layers that take the
+  // Dion branch this step, which lets the later persistent kernels return at once when it is 0,
+  // and (reset by the gate, counted by the Cholesky kernels) the layers that took the shifted
+  // retry, which lets the third CholeskyQR pass return at once when it is 0
   unsigned long long *gate_scratch;
   // 1 when this step's norms pass has already written B = M + G into M (gated modes with bf16
   // gradients): the fused kernel and the update then read B from M without G, and the local

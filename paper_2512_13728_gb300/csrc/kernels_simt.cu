@@ -182,7 +182,10 @@ __device__ void gate_finish(const Shared &sh, const StepArgs &a, int gflag, int 
   }
   atomicAdd(count_s, mine);
   __syncthreads();
-  if (threadIdx.x == 0) sh.gate_scratch[kScratchActive] = (unsigned long long)*count_s;
+  if (threadIdx.x == 0) {
+    sh.gate_scratch[kScratchActive] = (unsigned long long)*count_s;
+    sh.gate_scratch[kScratchShifted] = 0ull;  // counted by this step's Cholesky kernels
+  }
 }
 
 // One warp per layer; the running maximum of RMMC goes to an atomic max (order-independent, so
@@ -371,6 +374,7 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_kernel(Shared sh, const Gem
                                                             const int4 *tiles) {
   const int4 t = tiles[blockIdx.x];
   const GemmProblem p = probs[t.x];
+  if (p.mode == GEMM_SHIFTED && sh.gate_scratch[kScratchShifted] == 0ull) return;  // no layer shifted
   DION_TILE_CHECK(p.layer >= 0 && p.layer < sh.num_layers && t.y >= 0 && t.z >= 0 &&
                       (int64_t)t.y * GBM < p.Mrows && (int64_t)t.z * GBN < p.Ncols, sh.status);
   if (!sh.active[p.layer]) return;
@@ -686,6 +690,7 @@ __device__ __noinline__ float power_norm_sym(const float *__restrict__ S, int r,
 // is small enough, else a power-iteration estimate of ||E||_2.
 __global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, int pass, float near_identity) {
   const int l = blockIdx.x;
+  if (pass == 2 && sh.gate_scratch[kScratchShifted] == 0ull) return;  // no layer took the shifted retry
   if (!sh.active[l]) return;
   if (pass == 2 && !sh.orth_shifted[l]) return;
   const DevLayer &Ly = sh.layers[l];
@@ -779,6 +784,7 @@ __global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, in
   if (tid == 0) {
     if (pass == 0) sh.orth_shifted[l] = shifted ? 1 : 0;
     else if (shifted) sh.orth_shifted[l] = 1;
+    if (shifted) atomicAdd(&sh.gate_scratch[kScratchShifted], 1ull);
   }
   if (!ok) {
     if (tid == 0) set_status(sh.status, ST_BREAKDOWN);

@@ -252,7 +252,7 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
   const size_t o_nmb = cv.take<double>(std::max(num_layers, 1));
   const size_t o_nb = cv.take<double>(std::max(num_layers, 1));
   const size_t o_status = cv.take<int32_t>(1);
-  const size_t o_gate = cv.take<unsigned long long>(4);
+  const size_t o_gate = cv.take<unsigned long long>(kScratchSlots);
   const size_t o_bt = cv.take<int4>(std::max<size_t>(bt.size(), 1));
   const size_t o_ut = cv.take<int4>(std::max<size_t>(ut.size(), 1));
   const size_t o_ct = cv.take<int4>(std::max<size_t>(ct.size(), 1));
@@ -282,7 +282,9 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
         q.mode = (k == 3) ? GEMM_SHIFTED : GEMM_ACTIVE;
       } else if (k <= 6) {
         q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.r; q.lda = ldp; q.ldb = ldp; q.ldc = ldp; q.transB = 1;
-        q.mode = (k == 6) ? GEMM_SHIFTED_OR_COPY : GEMM_ACTIVE;
+        // the third solve runs on shifted layers only; in DION_PREC_FP32 it also copies the second
+        // pass's result into P for the others (BF16X3's split_p reads it where it is)
+        q.mode = (k == 6) ? (precision == DION_PREC_BF16X3 ? GEMM_SHIFTED : GEMM_SHIFTED_OR_COPY) : GEMM_ACTIVE;
       } else {
         q.Mrows = ly.n; q.Ncols = ly.r; q.K = ly.m; q.lda = ly.ldm; q.ldb = ldp; q.ldc = ldp; q.transA = 1;
       }
@@ -359,7 +361,8 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
     if (e == cudaSuccess) e = upload(p->gtiles[k], gt[k]);
   }
   if (e == cudaSuccess) e = cudaMemset(p->sh.status, 0, sizeof(int32_t));
-  if (e == cudaSuccess) e = cudaMemset(p->sh.gate_scratch, 0, 4 * sizeof(unsigned long long));  // key 0 < every RMMC
+  if (e == cudaSuccess)
+    e = cudaMemset(p->sh.gate_scratch, 0, kScratchSlots * sizeof(unsigned long long));  // key 0 < every RMMC
   if (e == cudaSuccess && num_layers > 0) e = prepare_chol_inv(p->max_r, &p->chol_smem);
   if (e == cudaSuccess && precision != DION_PREC_FP32) {
     p->tcp.probs = p->probs;

@@ -89,6 +89,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
     tc_orth_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off, const LayerMaps *__restrict__ maps,
                    int pass, int nstages, uint32_t stage_bytes, uint32_t tmem_cols) {
   if (sh.gate_scratch[kScratchActive] == 0ull) return;  // no layer takes the Dion branch
+  if (pass == 2 && sh.gate_scratch[kScratchShifted] == 0ull) return;  // no layer took the shifted retry
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = align1024(smem_raw);
   uint8_t *stg = smem + nstages * stage_bytes;  // 2 x (row box 16 KB + 4 transposed boxes 16 KB)

@@ -215,11 +215,13 @@ def test_full_rank_and_max_rank_fp32():
         plan.close()
 
 
-def test_ill_conditioned_p_takes_shifted_pass():
+@pytest.mark.parametrize("prec", ["fp32", "bf16x3"])
+def test_ill_conditioned_p_takes_shifted_pass(prec):
     """Q_0 with two nearly parallel columns makes kappa(P) ~ 1e6: the fp32 Cholesky of P^T P
     breaks down, the shifted retry and third pass still give an orthonormal P (no breakdown
     status).  Column 2 of the Q factor is then only resolved to u * kappa by fp32 data, so
-    step 1 gets looser bounds."""
+    step 1 gets looser bounds.  In BF16X3 the third pass's result is read from the other
+    buffer than after two passes."""
     import paper_2512_13728_gb300 as cd
 
     w = wl.scaled(wl.WORKLOADS["gpt160m_block_r192"], "illcond", [(256, 192)], rank=16, steps=3)
@@ -229,7 +231,7 @@ def test_ill_conditioned_p_takes_shifted_pass():
     gen.manual_seed(5)
     q[:, 1] = q[:, 0] + 1e-6 * torch.randn(q.shape[0], device=q.device, generator=gen)
     q[:, 1] /= q[:, 1].norm()
-    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, cd.DION_PREC_FP32)
+    plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, PRECS[prec])
     hpo = gu.oracle_hp()
     try:
         for t in range(1, w.steps + 1):
@@ -241,8 +243,11 @@ def test_ill_conditioned_p_takes_shifted_pass():
             c = gu.compare_step(st, plan, layers, grads, prev, hpo, t)
             print(t, c.err_M, c.err_X, c.err_Q)
             # step 1: the ill-determined column (error ~ kappa u ~ 6e-2 in fp32 data) enters M and X
-            # through (1 - mu) P P^T B and P Q^T; later steps start from a well-conditioned Q_t.
-            assert c.err_M <= (1e-3 if t == 1 else TOL_FP32) and c.err_X <= (1e-3 if t == 1 else TOL_FP32)
+            # through (1 - mu) P P^T B and P Q^T (split bf16 operands resolve products to 2^-17, not
+            # fp32's 2^-24, so that column costs them a little more); later steps start from a
+            # well-conditioned Q_t.
+            first = 1e-3 if prec == "fp32" else 2e-3
+            assert c.err_M <= (first if t == 1 else TOL_FP32) and c.err_X <= (first if t == 1 else TOL_FP32)
             assert c.err_Q <= (0.1 if t == 1 else TOL_FP32)
     finally:
         plan.close()
