@@ -345,8 +345,18 @@ def run_ours(args, rank, world, local_rank):
     if plan.device_status() != 0:
         raise RuntimeError("device status after warm-up: " + cd.native.dion_status_string(plan.device_status()))
 
+    # --graph: one step captured into a CUDA graph (every kernel of dion_step is enqueued without
+    # a host sync or an allocation, so the call can be captured) and replayed in the timed region;
+    # the per-kernel breakdown then comes from eager steps timed after it
+    graph = None
+    if args.graph:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            plan.step(cd.hparams(step=t + 1, gate_mode=gate, tau_global=args.tau))
+        torch.cuda.synchronize()
     # ---- timed region (device-resident inputs) ----
-    cd.native.dion_timing_enable(plan.handle, args.steps)
+    if graph is None:
+        cd.native.dion_timing_enable(plan.handle, args.steps)
     sampler = None
     if rank == 0:
         props = torch.cuda.get_device_properties(dev)
@@ -368,6 +378,12 @@ def run_ours(args, rank, world, local_rank):
             evs[i][0].record(stream)
             one_step()
             evs[i][1].record(stream)
+    elif graph is not None:  # the same step replayed from a CUDA graph (launch overhead removed)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            graph.replay()
+        e1.record(stream)
     else:
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
@@ -379,6 +395,11 @@ def run_ours(args, rank, world, local_rank):
         dist.barrier()
     clocks = sampler.stop() if sampler else None
     ms_total = sum(a.elapsed_time(b) for a, b in evs) if grad_seq else e0.elapsed_time(e1)
+    if graph is not None:  # per-kernel times from eager steps
+        cd.native.dion_timing_enable(plan.handle, args.steps)
+        for _ in range(args.steps):
+            one_step()
+        torch.cuda.synchronize()
     nsteps_timed, ktimes = cd.native.dion_timing_read(plan.handle)
     cd.native.dion_timing_enable(plan.handle, 0)
     ms_total = max_over_ranks(ms_total, world, dev)
@@ -481,6 +502,7 @@ def run_ours(args, rank, world, local_rank):
         "roofline": roofline,
         "e2e": {"value": round(e2e_ms, 4), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": launches * args.steps,
+        "cuda_graph": bool(args.graph),
         "clocks": clocks,
         "kernels": [dict(name=k["name"], ms=round(k["ms"], 4), **kernel_frac(k, peaks)) for k in kern],
         "timed_steps_with_kernel_events": nsteps_timed,
@@ -583,7 +605,10 @@ def main():
                     "the step number t start there")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--tf32-peak", action="store_true", help="print the measured cuBLAS tf32 throughput and exit")
+    ap.add_argument("--graph", action="store_true", help="time steps replayed from a CUDA graph (--gate always only)")
     args = ap.parse_args()
+    if args.graph and args.gate != "always":
+        ap.error("--graph replays one captured step, which needs --gate always (no per-step gradients)")
     if args.tf32_peak:
         print(json.dumps(measure_tf32_peak()), flush=True)
         return

@@ -528,3 +528,33 @@ def test_checkpoint_resume_bitwise():
     for a, b in zip(got, ref):
         assert torch.equal(a, b)
     plan2.close()
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16", "bf16x3"])
+def test_cuda_graph_replay_matches_direct_steps(prec):
+    """dion_step only enqueues kernels (no host sync, no allocation), so a caller can capture it in
+    a CUDA graph: three replays of one captured step give the bits of three direct steps."""
+    import paper_2512_13728_gb300 as cd
+
+    outs = []
+    for use_graph in (False, True):
+        st = gu.make_state(RAGGED)
+        gu.write_gradients(st, 1)
+        plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, PRECS[prec])
+        torch.cuda.synchronize()
+        hp = cd.hparams(step=1)
+        if use_graph:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                plan.step(hp)
+            for _ in range(3):
+                g.replay()
+        else:
+            for _ in range(3):
+                plan.step(hp)
+        torch.cuda.synchronize()
+        assert plan.device_status() == 0
+        outs.append([x.clone() for x in st.X + st.M + st.Q] + [plan.rmmc.clone(), plan.prev_norm.clone()])
+        plan.close()
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
