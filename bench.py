@@ -121,10 +121,10 @@ def kernel_work(name: str, w, prec: str, gate: str = "always", wt=None):
         # the gate in its last block)
         "norms_gate": ("hbm", mn_all * (4 + gsz + 4), "B"),
         "tc_btp": ("hbm", mn * bh + mr * 2 * hl + nr * (4 + 2 * hl), "B"),  # Bh (Bl), bf16 P; R fp32, bf16
-        "split_p": ("hbm", mr * 8, "B"),  # read P fp32; write its two bf16 halves
         "tc_update": ("hbm", mn * (16 + (gsz if deferred else 0)), "B"),
-        "tc_gram": ("tf32", mrr1, "flop"),
-        "tc_trsm": ("tf32", mrr1, "flop"),
+        # tf32 tensor work: BF16X3 issues three products (hi.hi + hi.lo + lo.hi) per multiply-add
+        "tc_gram": ("tf32", mrr1 * (3 if prec == "bf16x3" else 1), "flop"),
+        "tc_trsm": ("tf32", mrr1 * (3 if prec == "bf16x3" else 1), "flop"),
     }
     # Orthogonalize's launches carry their pass: passes 0 and 1 run the Gram and the solve on
     # every synchronizing layer; pass 1's factor is usually the first-order one and pass 2 runs

@@ -282,9 +282,9 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
         q.mode = (k == 3) ? GEMM_SHIFTED : GEMM_ACTIVE;
       } else if (k <= 6) {
         q.Mrows = ly.m; q.Ncols = ly.r; q.K = ly.r; q.lda = ldp; q.ldb = ldp; q.ldc = ldp; q.transB = 1;
-        // the third solve runs on shifted layers only; in DION_PREC_FP32 it also copies the second
-        // pass's result into P for the others (BF16X3's split_p reads it where it is)
-        q.mode = (k == 6) ? (precision == DION_PREC_BF16X3 ? GEMM_SHIFTED : GEMM_SHIFTED_OR_COPY) : GEMM_ACTIVE;
+        // the third solve runs on shifted layers only; it also copies the second pass's result
+        // into P for the others
+        q.mode = (k == 6) ? GEMM_SHIFTED_OR_COPY : GEMM_ACTIVE;
       } else {
         q.Mrows = ly.n; q.Ncols = ly.r; q.K = ly.m; q.lda = ly.ldm; q.ldb = ldp; q.ldc = ldp; q.transA = 1;
       }

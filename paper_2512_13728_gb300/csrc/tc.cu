@@ -600,10 +600,11 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   const uint32_t nb128 = (uint32_t)std::max(1, (lo.max_r + 127) / 128);
   // Gram / TRSM (CTA pairs): A box + per 256-column part of N, this CTA's half (one 128-row box)
   const uint32_t o_parts = (uint32_t)std::max(1, ((lo.max_r + 15) / 16 * 16 + 255) / 256);
-  const uint32_t ostage = 128u * 32u * 4u * (1u + o_parts);
+  // BF16X3: every stage also holds the lo boxes its converters write
+  const uint32_t ostage = (x3 ? 2u : 1u) * 128u * 32u * 4u * (1u + o_parts);
   const int ostages = (int)std::min<uint32_t>(4u, budget / ostage);
   // TRSM: one 256-column part per sub-tile, so a stage holds the A box and one B box
-  const uint32_t tstage = 128u * 32u * 4u * 2u;
+  const uint32_t tstage = (x3 ? 2u : 1u) * 128u * 32u * 4u * 2u;
   const int tstages = (int)std::min<uint32_t>(4u, budget / tstage);
   if (stages < 2 || ostages < 2 || tstages < 2) return cudaErrorInvalidValue;
   tp->nb64 = nb64;
@@ -629,13 +630,13 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   tp->fb_smem = fused_bq_smem(bq_boxes);
   if (tp->fuse_buffer && tp->fb_smem > 227u * 1024u) return cudaErrorInvalidValue;
   if (e == cudaSuccess && tp->fuse_buffer) e = setup_fused_bq_kernel(tp->fb_smem);
-  if (e == cudaSuccess) e = setup_orth_kernels(tp->o_smem);
+  if (e == cudaSuccess) e = setup_orth_kernels(tp->o_smem, x3);
   if (e == cudaSuccess && !x3) e = prepare_chol_inv_tc(lo.max_r, &tp->chol_tc_smem);
   int dev = 0, sms = 0;
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   tp->num_sms = sms;
-  tp->launches = x3 ? 19 : tp->fuse_buffer ? 17 : 18;
+  tp->launches = tp->fuse_buffer ? 17 : 18;
   return e;
 }
 
@@ -667,32 +668,17 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh_in, const StepArgs &a
     tick(p, s, "tc_bq");
   }
   static const char *kChol[3] = {"chol_inv0", "chol_inv1", "chol_inv2"};
-  if (tp.precision == DION_PREC_BF16X3) {
-    // fp32-class Orthogonalize: the CUDA-core Gram and solve of the FP32 mode (sets 1..6)
-    static const char *kGram[3] = {"gemm_gram0", "gemm_gram1", "gemm_gram2"};
-    static const char *kTrsm[3] = {"gemm_trsm0", "gemm_trsm1", "gemm_trsm2"};
-    for (int pass = 0; pass < 3; ++pass) {
-      launch_gemm(sh, tp.probs[1 + pass], tp.gtiles[1 + pass], tp.n_gtiles[1 + pass], s);  // S = X^T X
-      tick(p, s, kGram[pass]);
-      launch_chol_inv(sh, chol_smem, pass, 1e-3f, s);  // L, L^{-1}
-      tick(p, s, kChol[pass]);
-      launch_gemm(sh, tp.probs[4 + pass], tp.gtiles[4 + pass], tp.n_gtiles[4 + pass], s);  // X L^{-T}
-      tick(p, s, kTrsm[pass]);
-    }
-    launch_split_p(sh, tp, s);  // the bf16 halves of the orthonormal P
-    tick(p, s, "split_p");
-  } else {
-    static const char *kGram[3] = {"tc_gram0", "tc_gram1", "tc_gram2"};
-    static const char *kTrsm[3] = {"tc_trsm0", "tc_trsm1", "tc_trsm2"};
-    for (int pass = 0; pass < 3; ++pass) {  // CholeskyQR2; the third pass only after a shifted retry
-      launch_orth(sh, tp, true, pass, s);  // S = X^T X
-      tick(p, s, kGram[pass]);
-      if (pass == 0) launch_chol_inv_tc(sh, tp.maps, tp.chol_tc_smem, s);  // L, L^{-1} (trailing update on tensor cores)
-      else launch_chol_inv(sh, chol_smem, pass, 6e-2f, s);        // usually the first-order factor
-      tick(p, s, kChol[pass]);
-      launch_orth(sh, tp, false, pass, s);  // X L^{-T} and its transpose, or its bf16 copy at the end
-      tick(p, s, kTrsm[pass]);
-    }
+  static const char *kGram[3] = {"tc_gram0", "tc_gram1", "tc_gram2"};
+  static const char *kTrsm[3] = {"tc_trsm0", "tc_trsm1", "tc_trsm2"};
+  const bool x3 = tp.precision == DION_PREC_BF16X3;
+  for (int pass = 0; pass < 3; ++pass) {  // CholeskyQR2; the third pass only after a shifted retry
+    launch_orth(sh, tp, true, pass, s);  // S = X^T X
+    tick(p, s, kGram[pass]);
+    if (pass == 0 && !x3) launch_chol_inv_tc(sh, tp.maps, tp.chol_tc_smem, s);  // trailing update on tensor cores
+    else launch_chol_inv(sh, chol_smem, pass, x3 ? 1e-3f : 6e-2f, s);  // passes 1-2: usually the first-order factor
+    tick(p, s, kChol[pass]);
+    launch_orth(sh, tp, false, pass, s);  // X L^{-T} and its transpose, or its bf16 copy (halves) at the end
+    tick(p, s, kTrsm[pass]);
   }
   launch_btp(sh, tp, s);  // R = B^T P
   tick(p, s, "tc_btp");
@@ -737,21 +723,12 @@ void step_phase(const TcPlan &tp, const Shared &sh_in, const StepArgs &a, int32_
       else launch_form_bq(sh, tp, s);
       break;
     case DION_PHASE_ORTHO:  // Orthogonalize the averaged P, then R = B^T P
-      if (x3) {
-        for (int pass = 0; pass < 3; ++pass) {
-          launch_gemm(sh, tp.probs[1 + pass], tp.gtiles[1 + pass], tp.n_gtiles[1 + pass], s);
-          launch_chol_inv(sh, chol_smem, pass, 1e-3f, s);
-          launch_gemm(sh, tp.probs[4 + pass], tp.gtiles[4 + pass], tp.n_gtiles[4 + pass], s);
-        }
-        launch_split_p(sh, tp, s);
-      } else {
-        launch_transpose_praw(sh, tp, s);  // the first Gram reads P_raw^T
-        for (int pass = 0; pass < 3; ++pass) {
-          launch_orth(sh, tp, true, pass, s);
-          if (pass == 0) launch_chol_inv_tc(sh, tp.maps, tp.chol_tc_smem, s);
-          else launch_chol_inv(sh, chol_smem, pass, 6e-2f, s);
-          launch_orth(sh, tp, false, pass, s);
-        }
+      launch_transpose_praw(sh, tp, s);  // the first Gram reads P_raw^T
+      for (int pass = 0; pass < 3; ++pass) {
+        launch_orth(sh, tp, true, pass, s);
+        if (pass == 0 && !x3) launch_chol_inv_tc(sh, tp.maps, tp.chol_tc_smem, s);
+        else launch_chol_inv(sh, chol_smem, pass, x3 ? 1e-3f : 6e-2f, s);
+        launch_orth(sh, tp, false, pass, s);
       }
       launch_btp(sh, tp, s);
       break;

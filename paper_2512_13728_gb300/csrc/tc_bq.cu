@@ -720,36 +720,6 @@ __global__ void __launch_bounds__(256) qn_refresh_kernel(Shared sh, const int4 *
   }
 }
 
-// BF16X3: the bf16 halves of the orthonormal P (fp32, from the CUDA-core solve) for B^T P and
-// the update.  The solves alternate between P_raw and P, so the result is in P_raw after two
-// passes and in P after a shifted third one.  Tile = {layer, 128-row block}; a warp per row,
-// 8-byte stores.
-__global__ void __launch_bounds__(256) split_p_kernel(Shared sh, const int4 *tiles) {
-  const int4 t = tiles[blockIdx.x];
-  DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers && t.y >= 0 && (int64_t)t.y * 128 < sh.layers[t.x].m, sh.status);
-  if (!sh.active[t.x]) return;
-  const DevLayer &L = sh.layers[t.x];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int64_t r4 = (L.r + 3) / 4, row_end = min((int64_t)t.y * 128 + 128, L.m);
-  const float *src = sh.orth_shifted[t.x] ? L.P : L.P_raw;
-  for (int64_t i = (int64_t)t.y * 128 + warp; i < row_end; i += 8) {
-    for (int64_t c4 = lane; c4 < r4; c4 += 32) {
-      const float4 v = *reinterpret_cast<const float4 *>(src + i * L.ldp + 4 * c4);  // rows padded to 8
-      const __nv_bfloat162 h01 = __floats2bfloat162_rn(v.x, v.y), h23 = __floats2bfloat162_rn(v.z, v.w);
-      const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
-      const __nv_bfloat162 l01 = __floats2bfloat162_rn(v.x - f01.x, v.y - f01.y);
-      const __nv_bfloat162 l23 = __floats2bfloat162_rn(v.z - f23.x, v.w - f23.y);
-      uint2 hv, lv;
-      hv.x = *reinterpret_cast<const uint32_t *>(&h01);
-      hv.y = *reinterpret_cast<const uint32_t *>(&h23);
-      lv.x = *reinterpret_cast<const uint32_t *>(&l01);
-      lv.y = *reinterpret_cast<const uint32_t *>(&l23);
-      *reinterpret_cast<uint2 *>(L.P_hi + i * L.ldp + 4 * c4) = hv;
-      *reinterpret_cast<uint2 *>(L.P_lo + i * L.ldp + 4 * c4) = lv;
-    }
-  }
-}
-
 // ======================================================================= launchers ===
 uint32_t form_bq_smem(int nstages, uint32_t stage_bytes) {
   return 1024u + nstages * stage_bytes + STG_BYTES + 512u;  // + barriers
@@ -862,10 +832,6 @@ void launch_transpose_praw(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
 }
 void launch_r_refresh(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
   if (tp.n_rtiles > 0) r_refresh_kernel<<<tp.n_rtiles, 256, 0, s>>>(sh, tp.rtiles);
-}
-
-void launch_split_p(const Shared &sh, const TcPlan &tp, cudaStream_t s) {
-  if (tp.n_trsm_tiles > 0) split_p_kernel<<<tp.n_trsm_tiles, 256, 0, s>>>(sh, tp.trsm_tiles);
 }
 
 void launch_qn_refresh(const Shared &sh, const TcPlan &tp, cudaStream_t s) {

@@ -1,5 +1,6 @@
-// Orthogonalize on tensor cores for DION_PREC_BF16: the Gram matrix and the triangular
-// solve of each CholeskyQR pass as kind::tf32 tcgen05 GEMMs on fp32 operands loaded by TMA.
+// Orthogonalize on tensor cores: the Gram matrix and the triangular solve of each
+// CholeskyQR pass as kind::tf32 tcgen05 GEMMs on fp32 operands loaded by TMA (DION_PREC_BF16),
+// or as three such products per k-step on split operands (DION_PREC_BF16X3, below).
 //
 //   Gram   S = X^T X (r x r).  Tile = 128 full rows of S; K loop over m.  B = all r rows of
 //          the transposed copy X^T (r x m, K-major), which the producing kernel (the B Q
@@ -20,6 +21,16 @@
 // P back to orthonormal to that level, below the bf16 rounding the following kernels apply.
 // Both run as pair MMAs over 256-row blocks (two CTAs on two SMs, cta_group::2), so each SM
 // receives half of the B operand.  Roles: warp 0 TMA, warp 1 MMA (even CTA), warps 2..5 epilogue.
+//
+// BF16X3 (fp32-class): every fp32 operand x is split as hi = x with the low 13 mantissa bits
+// cleared (exactly a tf32 value) and lo = x - hi (exact in fp32; its own tf32 rounding costs
+// ~2^-21 |x|), and each k-step issues hi.hi + hi.lo + lo.hi into the same accumulator (lo.lo,
+// ~2^-22 relative, is left out): the 3xTF32 scheme.  The split happens in shared memory, so the
+// bytes each SM receives do not change: four converter warps (6..9) wait for a stage's TMA
+// loads (counted on each CTA's own barrier), clear the low bits of every box in place, write
+// the lo boxes into the second half of the stage, and report the stage to the even CTA, whose
+// MMA warp waits for both CTAs' reports.  The solve that ends Orthogonalize writes the bf16
+// high and low halves of P that R = B^T P and the update read.
 #include "tc.cuh"
 #include "tc_common.cuh"
 #include "tc_kernels.cuh"
@@ -30,6 +41,7 @@ namespace tc {
 constexpr uint32_t O_BOX = 128u * 32u * 4u;  // one fp32 box: 128 rows x 32 (K) = 16 KB
 constexpr uint32_t O_TBOX = 32u * 32u * 4u;  // one transposed output box: 32 x 32 fp32 = 4 KB
 constexpr int O_THREADS = 6 * 32;
+constexpr int O_THREADS_X3 = 10 * 32;  // + four converter warps
 
 enum : int32_t { ORTH_GRAM = 0, ORTH_TRSM = 1 };
 
@@ -84,8 +96,8 @@ __device__ __forceinline__ bool part_needs(int kc, uint32_t part) {
 // each CTA receives its 128 rows of the accumulator in its own TMEM.  For the Gram with a
 // full 256-column part the tile's own rows of X^T are exactly the CTA's B half of part p,
 // so A is read in place.  Tile = {layer, pair p}.
-template <int KIND>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
+template <int KIND, bool X3>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(X3 ? O_THREADS_X3 : O_THREADS, 1)
     tc_orth_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off, const LayerMaps *__restrict__ maps,
                    int pass, int nstages, uint32_t stage_bytes, uint32_t tmem_cols) {
   if (sh.gate_scratch[kScratchActive] == 0ull) return;  // no layer takes the Dion branch
@@ -97,6 +109,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
   uint64_t *full = bars, *empty = bars + nstages;
   // two accumulator slots (the TRSM alternates them; the Gram uses slot 0)
   uint64_t *acc_full = bars + 2 * nstages, *acc_empty = acc_full + 2, *drain = acc_full + 4;
+  uint64_t *conv = drain + 1;  // BF16X3: a stage's boxes are split in both CTAs (used in CTA 0)
+  const uint32_t lo_off = X3 ? stage_bytes / 2u : 0u;  // BF16X3: lo boxes, same layout as the hi half
   __shared__ uint32_t tmem_base_s;
   __shared__ int abort_s;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -105,8 +119,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
   const int seg = blockIdx.x >> 1;
   if (threadIdx.x == 0) {
     for (int i = 0; i < nstages; ++i) {
-      mbar_init(&full[i], 1);   // used in CTA 0: its arm, both CTAs' bytes
+      mbar_init(&full[i], 1);   // BF16: used in CTA 0, its arm, both CTAs' bytes; BF16X3: this CTA's bytes
       mbar_init(&empty[i], 1);  // pair commit after the stage's MMAs
+      if (X3) mbar_init(&conv[i], 2);  // one arrival per CTA's converters
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&acc_full[i], 1);   // pair commit after the (sub-)tile's MMAs
@@ -128,6 +143,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
   auto skip = [&](int layer) { return !sh.active[layer] || (pass == 2 && !sh.orth_shifted[layer]); };
   // half of N part q held by each CTA (rows of the B operand)
   auto half_rows = [](uint32_t N, uint32_t q) { return min(256u, N - q * 256u) / 2u; };
+  // TMA load of one box of a stage: BF16 counts both CTAs' bytes on CTA 0's barrier, BF16X3
+  // each CTA's on its own (its converters wait for them)
+  auto load = [&](void *dst, const CUtensorMap *map, uint32_t s, int32_t c0, int32_t c1) {
+    if (X3) tma_load_2d(dst, map, &full[s], c0, c1);
+    else tma_load_2d_pair(dst, map, cluster_addr(&full[s], 0), c0, c1);
+  };
+  auto expect = [&](uint32_t s, uint32_t boxes) {
+    if (X3) mbar_expect_tx(&full[s], O_BOX * boxes);
+    else if (rank == 0) mbar_expect_tx(&full[s], 2u * O_BOX * boxes);
+  };
 
   if (warp == 0) {
     if (lane == 0) {
@@ -152,10 +177,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
               const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
               if (!ab.wait(&empty[s], ph ^ 1u, sh.status)) { ok = false; break; }
               uint8_t *sA = smem + s * stage_bytes, *sB = sA + O_BOX;
-              const uint32_t fb = cluster_addr(&full[s], 0);
-              if (rank == 0) mbar_expect_tx(&full[s], 2u * O_BOX * 2u);
-              tma_load_2d_pair(sA, om.A, fb, kc * 32, tr * 128);
-              tma_load_2d_pair(sB, om.B, fb, kc * 32, (int)(q * 256u + rank * half_rows(N, q)));
+              expect(s, 2u);
+              load(sA, om.A, s, kc * 32, tr * 128);
+              load(sB, om.B, s, kc * 32, (int)(q * 256u + rank * half_rows(N, q)));
             }
           }
           continue;
@@ -165,20 +189,80 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
           const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
           if (!ab.wait(&empty[s], ph ^ 1u, sh.status)) { ok = false; break; }
           uint8_t *sA = smem + s * stage_bytes, *sB = sA + O_BOX;
-          const uint32_t fb = cluster_addr(&full[s], 0);
           uint32_t nb = 0;  // B boxes this chunk feeds (all, or only the lower-triangular parts)
           for (uint32_t q = 0; q < nparts; ++q)
             if (part_needs<KIND>(kc, q)) ++nb;
-          if (rank == 0) mbar_expect_tx(&full[s], 2u * O_BOX * ((a_in_b ? 0u : 1u) + nb));
-          if (!a_in_b) tma_load_2d_pair(sA, om.A, fb, kc * 32, tr * 128);
+          expect(s, (a_in_b ? 0u : 1u) + nb);
+          if (!a_in_b) load(sA, om.A, s, kc * 32, tr * 128);
           for (uint32_t q = 0; q < nparts; ++q)
-            if (part_needs<KIND>(kc, q))
-              tma_load_2d_pair(sB + q * O_BOX, om.B, fb, kc * 32, (int)(q * 256u + rank * half_rows(N, q)));
+            if (part_needs<KIND>(kc, q)) load(sB + q * O_BOX, om.B, s, kc * 32, (int)(q * 256u + rank * half_rows(N, q)));
         }
       }
       // drain: the last stages' loads have landed and been consumed (their stage was freed)
       for (uint32_t k = (it > (uint32_t)nstages ? it - nstages : 0); k < it; ++k)
         mbar_wait(&empty[k % nstages], (k / nstages) & 1u, sh.status);
+    }
+  } else if (X3 && warp >= 6) {
+    // converters (BF16X3): split every box of a landed stage, in the order the producer loads
+    const int ct = threadIdx.x - 6 * 32;
+    auto split_box = [&](uint8_t *box) {
+#pragma unroll 4
+      for (int i = ct; i < (int)(O_BOX / 16u); i += 128) {
+        float4 *hp = reinterpret_cast<float4 *>(box + i * 16);
+        const float4 x = *hp;
+        float4 h, l;
+        h.x = __uint_as_float(__float_as_uint(x.x) & 0xFFFFE000u);
+        h.y = __uint_as_float(__float_as_uint(x.y) & 0xFFFFE000u);
+        h.z = __uint_as_float(__float_as_uint(x.z) & 0xFFFFE000u);
+        h.w = __uint_as_float(__float_as_uint(x.w) & 0xFFFFE000u);
+        l.x = x.x - h.x;
+        l.y = x.y - h.y;
+        l.z = x.z - h.z;
+        l.w = x.w - h.w;
+        *hp = h;
+        *reinterpret_cast<float4 *>(box + lo_off + i * 16) = l;
+      }
+    };
+    auto report = [&](uint32_t s) {
+      fence_async_smem();  // the converted boxes are visible to the tensor cores' reads
+      named_sync(2, 128);
+      if (ct == 0) mbar_arrive_cluster(cluster_addr(&conv[s], 0));
+    };
+    uint32_t it = 0;
+    bool ok = true;
+    for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
+      const int4 t = tiles[ti];
+      if (skip(t.x)) continue;
+      const DevLayer &L = sh.layers[t.x];
+      uint32_t N;
+      int64_t K;
+      orth_dims<KIND>(L, t.y, N, K);
+      const int kch = (int)((K + 31) / 32);
+      const uint32_t nparts = (N + 255) / 256;
+      if constexpr (KIND == ORTH_TRSM) {
+        for (uint32_t q = 0; q < nparts && ok; ++q) {
+          const int kq = min(kch, (int)(8u * (q + 1u)));
+          for (int kc = 0; kc < kq; ++kc, ++it) {
+            const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
+            if (!named_and(2, 128, ab.wait(&full[s], ph, sh.status))) { ok = false; break; }
+            uint8_t *sA = smem + s * stage_bytes;
+            split_box(sA);
+            split_box(sA + O_BOX);
+            report(s);
+          }
+        }
+        continue;
+      }
+      const bool a_in_b = (KIND == ORTH_GRAM) && (uint32_t)t.y < nparts && half_rows(N, (uint32_t)t.y) == 128u;
+      for (int kc = 0; kc < kch; ++kc, ++it) {
+        const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
+        if (!named_and(2, 128, ab.wait(&full[s], ph, sh.status))) { ok = false; break; }
+        uint8_t *sA = smem + s * stage_bytes, *sB = sA + O_BOX;
+        if (!a_in_b) split_box(sA);
+        for (uint32_t q = 0; q < nparts; ++q)
+          if (part_needs<KIND>(kc, q)) split_box(sB + q * O_BOX);
+        report(s);
+      }
     }
   } else if (warp == 1) {
     if (lane == 0 && rank == 0) {
@@ -199,16 +283,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
             if (!ab.wait(&acc_empty[slot], ((tcount >> 1) & 1u) ^ 1u, sh.status)) { ok = false; break; }
             tc_fence_after();
             const int kq = min(kch, (int)(8u * (q + 1u)));
+            const uint32_t idesc = idesc_tf32(256, 2u * half_rows(N, q), false, false);
             for (int kc = 0; kc < kq; ++kc, ++it) {
               const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
-              if (!ab.wait(&full[s], ph, sh.status)) { ok = false; break; }
+              if (!ab.wait(X3 ? &conv[s] : &full[s], ph, sh.status)) { ok = false; break; }
               tc_fence_after();
               const uint32_t aB = smem_u32(smem + s * stage_bytes), bB = aB + O_BOX;
 #pragma unroll
-              for (int k8 = 0; k8 < 4; ++k8)
-                umma_pair_tf32(tmem + slot * 256u, smem_desc_sw128(aB + k8 * 32, 0, 1024),
-                               smem_desc_sw128(bB + k8 * 32, 0, 1024), idesc_tf32(256, 2u * half_rows(N, q), false, false),
-                               (kc | k8) ? 1u : 0u);
+              for (int k8 = 0; k8 < 4; ++k8) {
+                const uint64_t ad = smem_desc_sw128(aB + k8 * 32, 0, 1024), bd = smem_desc_sw128(bB + k8 * 32, 0, 1024);
+                umma_pair_tf32(tmem + slot * 256u, ad, bd, idesc, (kc | k8) ? 1u : 0u);
+                if (X3) {  // hi.lo + lo.hi
+                  umma_pair_tf32(tmem + slot * 256u, ad, smem_desc_sw128(bB + lo_off + k8 * 32, 0, 1024), idesc, 1u);
+                  umma_pair_tf32(tmem + slot * 256u, smem_desc_sw128(aB + lo_off + k8 * 32, 0, 1024), bd, idesc, 1u);
+                }
+              }
               umma_pair_commit_mc(&empty[s], 0x3);  // the stage is free in both CTAs
             }
             if (!ok) break;
@@ -222,7 +311,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
         tc_fence_after();
         for (int kc = 0; kc < kch; ++kc, ++it) {
           const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
-          if (!ab.wait(&full[s], ph, sh.status)) { ok = false; break; }
+          if (!ab.wait(X3 ? &conv[s] : &full[s], ph, sh.status)) { ok = false; break; }
           tc_fence_after();
           const uint32_t aB = smem_u32(smem + s * stage_bytes), bB = aB + O_BOX;
           const uint32_t aSrc = a_in_b ? bB + (uint32_t)t.y * O_BOX : aB;
@@ -231,10 +320,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
             const uint64_t ad = smem_desc_sw128(aSrc + k8 * 32, 0, 1024);
             for (uint32_t q = 0; q < nparts; ++q) {
               if (!part_needs<KIND>(kc, q)) continue;
+              const uint32_t idesc = idesc_tf32(256, 2u * half_rows(N, q), false, false);
               const uint64_t bd = smem_desc_sw128(bB + q * O_BOX + k8 * 32, 0, 1024);
               // the first chunk that feeds a part starts its accumulation
-              umma_pair_tf32(tmem + q * 256u, ad, bd, idesc_tf32(256, 2u * half_rows(N, q), false, false),
-                             (kc | k8) ? 1u : 0u);
+              umma_pair_tf32(tmem + q * 256u, ad, bd, idesc, (kc | k8) ? 1u : 0u);
+              if (X3) {  // hi.lo + lo.hi
+                umma_pair_tf32(tmem + q * 256u, ad, smem_desc_sw128(bB + lo_off + q * O_BOX + k8 * 32, 0, 1024), idesc, 1u);
+                umma_pair_tf32(tmem + q * 256u, smem_desc_sw128(aSrc + lo_off + k8 * 32, 0, 1024), bd, idesc, 1u);
+              }
             }
           }
           umma_pair_commit_mc(&empty[s], 0x3);  // the stage is free in both CTAs
@@ -282,7 +375,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
         if (final_pass) {
           for (int j = jb; j < je; j += 2) {  // two 32-column chunks per 64-column bf16 box
             const uint32_t eb = ecount & 1u;
-            uint8_t *hb = stg + eb * 2 * O_BOX;
+            uint8_t *hb = stg + eb * 2 * O_BOX, *lb = hb + O_BOX;  // lb: BF16X3's low halves
             if (leader) bulk_wait_read<1>();
             named_sync(1, 128);
 #pragma unroll 1
@@ -300,17 +393,33 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
                   uint2 hv;
                   hv.x = *reinterpret_cast<const uint32_t *>(&a);
                   hv.y = *reinterpret_cast<const uint32_t *>(&b);
-                  *reinterpret_cast<uint2 *>(hb + sw128_offset(row, (uint32_t)(h * 4 + (c4 >> 1))) + (c4 & 1) * 8) = hv;
+                  const uint32_t bo = sw128_offset(row, (uint32_t)(h * 4 + (c4 >> 1))) + (c4 & 1) * 8;
+                  *reinterpret_cast<uint2 *>(hb + bo) = hv;
+                  if (X3) {  // low halves: x - bf16(x), rounded to bf16
+                    const float2 af = __bfloat1622float2(a), bf = __bfloat1622float2(b);
+                    const __nv_bfloat162 al = __floats2bfloat162_rn(__uint_as_float(v[4 * c4]) - af.x,
+                                                                    __uint_as_float(v[4 * c4 + 1]) - af.y);
+                    const __nv_bfloat162 bl = __floats2bfloat162_rn(__uint_as_float(v[4 * c4 + 2]) - bf.x,
+                                                                    __uint_as_float(v[4 * c4 + 3]) - bf.y);
+                    uint2 lv;
+                    lv.x = *reinterpret_cast<const uint32_t *>(&al);
+                    lv.y = *reinterpret_cast<const uint32_t *>(&bl);
+                    *reinterpret_cast<uint2 *>(lb + bo) = lv;
+                  }
                 }
               } else {  // a lone last chunk: the other half of the box (clipped by the store)
 #pragma unroll
-                for (int c4 = 4; c4 < 8; ++c4) *reinterpret_cast<uint4 *>(hb + sw128_offset(row, c4)) = make_uint4(0, 0, 0, 0);
+                for (int c4 = 4; c4 < 8; ++c4) {
+                  *reinterpret_cast<uint4 *>(hb + sw128_offset(row, c4)) = make_uint4(0, 0, 0, 0);
+                  if (X3) *reinterpret_cast<uint4 *>(lb + sw128_offset(row, c4)) = make_uint4(0, 0, 0, 0);
+                }
               }
             }
             fence_async_smem();
             named_sync(1, 128);
             if (leader) {
               tma_store_2d(&maps[t.x].P_hi, hb, j * 32, tr * 128);
+              if (X3) tma_store_2d(&maps[t.x].P_lo, lb, j * 32, tr * 128);
               bulk_commit();
             }
             ++ecount;
@@ -369,24 +478,36 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(O_THREADS, 1)
 // alignment slack + operand stages + 2 staging buffers + barriers (2 x stages + 5 words)
 uint32_t orth_smem(int nstages, uint32_t stage_bytes) { return 1024u + nstages * stage_bytes + 4u * O_BOX + 512u; }
 
-cudaError_t setup_orth_kernels(uint32_t smem) {
-  cudaError_t e =
-      cudaFuncSetAttribute(tc_orth_kernel<ORTH_GRAM>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+cudaError_t setup_orth_kernels(uint32_t smem, bool x3) {
+  const int sm = (int)smem;
+  const cudaFuncAttribute at = cudaFuncAttributeMaxDynamicSharedMemorySize;
+  cudaError_t e = x3 ? cudaFuncSetAttribute(tc_orth_kernel<ORTH_GRAM, true>, at, sm)
+                     : cudaFuncSetAttribute(tc_orth_kernel<ORTH_GRAM, false>, at, sm);
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(tc_orth_kernel<ORTH_TRSM>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    e = x3 ? cudaFuncSetAttribute(tc_orth_kernel<ORTH_TRSM, true>, at, sm)
+           : cudaFuncSetAttribute(tc_orth_kernel<ORTH_TRSM, false>, at, sm);
   return e;
 }
 
 void launch_orth(const Shared &sh, const TcPlan &tp, bool gram, int pass, cudaStream_t s) {
   const DevSchedule &d = gram ? tp.d_gram : tp.d_trsm;
   if (d.grid <= 0) return;
-  const uint32_t stage = O_BOX * (1 + tp.o_parts);
-  if (gram)
-    tc_orth_kernel<ORTH_GRAM><<<2 * d.grid, O_THREADS, tp.o_smem, s>>>(sh, d.tiles, d.off, tp.maps, pass,
-                                                                         tp.o_stages, stage, tp.tmem_cols);
-  else  // two 256-column accumulator slots
-    tc_orth_kernel<ORTH_TRSM><<<2 * d.grid, O_THREADS, tp.o_smem, s>>>(sh, d.tiles, d.off, tp.maps, pass,
-                                                                         tp.t_stages, 2u * O_BOX, 512u);
+  const bool x3 = tp.precision == DION_PREC_BF16X3;
+  const uint32_t f = x3 ? 2u : 1u;  // BF16X3 stages hold the lo boxes too
+  const uint32_t stage = f * O_BOX * (1 + tp.o_parts), tstage = f * 2u * O_BOX;  // TRSM: A box + one B box
+  const int g = 2 * d.grid;
+  if (gram && x3)
+    tc_orth_kernel<ORTH_GRAM, true><<<g, O_THREADS_X3, tp.o_smem, s>>>(sh, d.tiles, d.off, tp.maps, pass,
+                                                                        tp.o_stages, stage, tp.tmem_cols);
+  else if (gram)
+    tc_orth_kernel<ORTH_GRAM, false><<<g, O_THREADS, tp.o_smem, s>>>(sh, d.tiles, d.off, tp.maps, pass,
+                                                                      tp.o_stages, stage, tp.tmem_cols);
+  else if (x3)  // two 256-column accumulator slots
+    tc_orth_kernel<ORTH_TRSM, true><<<g, O_THREADS_X3, tp.o_smem, s>>>(sh, d.tiles, d.off, tp.maps, pass,
+                                                                        tp.t_stages, tstage, 512u);
+  else
+    tc_orth_kernel<ORTH_TRSM, false><<<g, O_THREADS, tp.o_smem, s>>>(sh, d.tiles, d.off, tp.maps, pass,
+                                                                      tp.t_stages, tstage, 512u);
 }
 
 }  // namespace tc
