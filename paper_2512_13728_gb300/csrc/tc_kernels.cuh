@@ -25,6 +25,8 @@ void launch_colnorm_scale(const Shared &sh, const TcPlan &tp, cudaStream_t s);
 uint32_t orth_smem(int nstages, uint32_t stage_bytes);
 cudaError_t setup_orth_kernels(uint32_t smem, bool x3);
 void launch_orth(const Shared &sh, const TcPlan &tp, bool gram, int pass, cudaStream_t s);
+cudaError_t setup_update_kernel(bool x3);
+void launch_update(const Shared &sh, const TcPlan &tp, float mu, float eta, float keep, cudaStream_t s);
 
 }  // namespace tc
 }  // namespace cd
