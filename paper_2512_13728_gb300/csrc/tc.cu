@@ -260,7 +260,13 @@ cudaError_t encode_maps(const DevLayer *dl, int32_t L, LayerMaps *dst) {
                       encode_bf16_2d(&m.Qn_lo_mn, d.Qn_lo, d.r, d.n, p16, 64, 64) &&
                       encode_bf16_2d(&m.P_lo_mn, d.P_lo, d.r, d.m, p16, 64, 64) &&
                       encode_bf16_2d(&m.Bl_mn, d.Bl, d.n, d.m, (uint64_t)d.ldbh * 2, 64, 64) &&
-                      encode_bf16_2d(&m.Bl_k, d.Bl, d.n, d.m, (uint64_t)d.ldbh * 2, 64, 128)));
+                      encode_bf16_2d(&m.Bl_k, d.Bl, d.n, d.m, (uint64_t)d.ldbh * 2, 64, 128) &&
+                      encode_bf16_2d(&m.P_hi32, d.P_hi, d.r, d.m, p16, 32, 128) &&
+                      encode_bf16_2d(&m.P_lo32, d.P_lo, d.r, d.m, p16, 32, 128) &&
+                      encode_bf16_2d(&m.R_hi32, d.R_hi, d.r, d.n, p16, 32, 128) &&
+                      encode_bf16_2d(&m.R_lo32, d.R_lo, d.r, d.n, p16, 32, 128) &&
+                      encode_bf16_2d(&m.Qn_hi32, d.Qn_hi, d.r, d.n, p16, 32, 128) &&
+                      encode_bf16_2d(&m.Qn_lo32, d.Qn_lo, d.r, d.n, p16, 32, 128)));
     if (!ok) return cudaErrorInvalidValue;
   }
   return cudaMemcpy(dst, maps.data(), sizeof(LayerMaps) * maps.size(), cudaMemcpyHostToDevice);

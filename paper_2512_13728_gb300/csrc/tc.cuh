@@ -40,6 +40,8 @@ struct LayerMaps {
   CUtensorMap P_lo, R_lo, Qn_lo;  // K-major {64, 128}: update operands
   CUtensorMap Qn_lo_mn, P_lo_mn, Bl_mn;  // MN-major {64, 64}: B Q / B^T P operands
   CUtensorMap Bl_k;   // K-major {64, 128}: B Q A operand
+  // BF16X3 update operands in 32-wide K chunks: K-major {32, 128}, 64-byte swizzle
+  CUtensorMap P_hi32, P_lo32, R_hi32, R_lo32, Qn_hi32, Qn_lo32;
 };
 
 // Tiles of one persistent kernel, reordered so that CTA b processes tiles [off[b], off[b+1]).

@@ -218,6 +218,13 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo
   return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
          ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | (1ull << 46) | (2ull << 61);
 }
+// The same with the 64-byte swizzle (TMA SWIZZLE_64B: the 16-byte chunk c of 64-byte row j of a
+// 512-byte atom sits at chunk c ^ ((j / 2) % 4)).  K-major operand with rows of 32 bf16 along
+// K: SBO = 512 (8-row group stride), LBO unused.
+__device__ __forceinline__ uint64_t smem_desc_sw64(uint32_t saddr, uint32_t sbo) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | (1ull << 46) |
+         (4ull << 61);
+}
 // Instruction descriptor of kind::f16 with bf16 A and B, fp32 D; a_mn / b_mn select
 // MN-major operands.  M = 128, N a multiple of 16 in [16, 256].
 __host__ __device__ constexpr uint32_t idesc_bf16(uint32_t M, uint32_t N, bool a_mn, bool b_mn) {

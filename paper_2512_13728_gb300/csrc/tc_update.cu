@@ -2,7 +2,7 @@
 //   M = B - (1 - mu) P R^T,   X = X - eta sqrt(m/n) P Q_t^T
 // run as one persistent, warp-specialized kernel over 128 x 128 output tiles:
 //   warp 0      TMA producer: bf16 K-major chunks of P (A), R and Q_t (two B operands) into a
-//               3-stage shared-memory ring;
+//               3-stage shared-memory ring (BF16X3: also their low halves);
 //   warp 1      MMA issuer: two 128x128x16 tcgen05.mma per k-step into a double-buffered
 //               pair of TMEM accumulators (U1 = P R^T, U2 = P Q_t^T; 4 x 128 = 512 columns);
 //   warps 2..5  epilogue (both CTAs): TMA-load 128 x 16 fp32 boxes of B (in the M buffer) and X,
@@ -21,22 +21,27 @@ namespace tc {
 // CTAs 2 s and 2 s + 1 take row tiles 2 p and 2 p + 1 of the same column blocks in the same
 // order (schedule segment s), so the R and Q_t chunks one of them loads are usually still in L2
 // when the other asks for them.  Each CTA loads all three operand boxes of a stage itself.
-constexpr uint32_t U_OPB = 128u * 64u * 2u;           // 128 x 64 bf16 operand box
+constexpr uint32_t U_OPB = 128u * 64u * 2u;           // 128 x 64 bf16 operand box (BF16: one per operand)
+constexpr uint32_t U_OPB32 = 128u * 32u * 2u;         // 128 x 32 bf16 operand box (BF16X3)
 constexpr uint32_t U_EBOX = 128u * 16u * 4u;          // one 128 x 16 fp32 box (64-byte swizzle)
 constexpr uint32_t U_GBOX = 128u * 16u * 2u;          // one 128 x 16 bf16 box of G (32-byte swizzle)
 constexpr uint32_t U_EBUF2 = 2u * U_EBOX + U_GBOX;     // M, X and G of one 16-column sub-chunk (20 KB)
 static_assert(U_EBUF2 % 1024u == 0, "every box of a sub-chunk buffer stays 1024-byte aligned");
 constexpr int U_THREADS = 192;
 constexpr uint32_t U_IDESC = idesc_bf16(128, 128, false, false);
-// Ring depths.  BF16: 3 stages of {P, R, Q_t} and 4 epilogue sub-chunk buffers of M, X and G.
-// BF16X3: each stage also holds the low halves of P, R and Q_t (P R^T = Ph Rh^T + Ph Rl^T +
-// Pl Rh^T, the same for P Q_t^T), and B is already in M (no G box), so 2 stages of 6 boxes and
-// 2 epilogue buffers of M and X fit in shared memory.
+// Ring depths.  BF16: 3 stages of {P, R, Q_t} in 64-wide K chunks (128-byte swizzle) and 4
+// epilogue sub-chunk buffers of M, X and G.  BF16X3: each stage also holds the low halves of P,
+// R and Q_t (P R^T = Ph Rh^T + Ph Rl^T + Pl Rh^T, the same for P Q_t^T), and B is already in M
+// (no G box); its stages take 32-wide K chunks (64-byte swizzle), so 3 stages of 6 boxes leave
+// room for 5 epilogue buffers of M and X (loads 4 sub-chunks ahead: with 2 buffers, one load in
+// flight, the epilogue waited on every sub-chunk).
 template <bool X3>
 struct UpdCfg {
-  static constexpr int STAGES = X3 ? 2 : 3;
-  static constexpr uint32_t STAGE = (X3 ? 6u : 3u) * U_OPB;  // P, R, Q_t [, P_lo, R_lo, Q_lo]
-  static constexpr int EBUF = X3 ? 2 : 4;
+  static constexpr uint32_t KW = X3 ? 32u : 64u;  // K chunk width (bf16 elements per operand row)
+  static constexpr uint32_t OPB = X3 ? U_OPB32 : U_OPB;
+  static constexpr int STAGES = 3;
+  static constexpr uint32_t STAGE = (X3 ? 6u : 3u) * OPB;  // P, R, Q_t [, P_lo, R_lo, Q_lo]
+  static constexpr int EBUF = X3 ? 5 : 4;
   static constexpr uint32_t EBUF2 = X3 ? 2u * U_EBOX : U_EBUF2;  // bytes of one sub-chunk buffer
   static constexpr uint32_t SMEM = 1024u + STAGES * STAGE + EBUF * EBUF2 + 256u;
 };
@@ -49,6 +54,7 @@ __global__ void __launch_bounds__(U_THREADS, 1)
                      float mu, float eta, float keep) {
   constexpr int U_STAGES = UpdCfg<X3>::STAGES;
   constexpr uint32_t U_STAGE = UpdCfg<X3>::STAGE;
+  constexpr uint32_t KW = UpdCfg<X3>::KW, OPB = UpdCfg<X3>::OPB;
   constexpr int U_EBUF = UpdCfg<X3>::EBUF;
   constexpr uint32_t U_EBUFB = UpdCfg<X3>::EBUF2;
   if (sh.gate_scratch[kScratchActive] == 0ull) return;  // no layer takes the Dion branch
@@ -101,20 +107,25 @@ __global__ void __launch_bounds__(U_THREADS, 1)
         const int4 t = tiles[ti];
         if (!sh.active[t.x]) continue;
         const LayerMaps *mp = maps + t.x;
-        const int kch = (int)((sh.layers[t.x].r + 63) / 64);
+        const int kch = (int)((sh.layers[t.x].r + KW - 1) / KW);
         const int mb = 2 * t.y + (int)rank;  // past the last row tile: zero-filled, not stored
         for (int kc = 0; kc < kch; ++kc, ++it) {
           const uint32_t s = it % U_STAGES, ph = (it / U_STAGES) & 1u;
           if (!ab.wait(&empty[s], ph ^ 1u, sh.status)) { ok = false; break; }
           uint8_t *sp = stage + s * U_STAGE;
           mbar_expect_tx(&full[s], U_STAGE);
-          tma_load_2d(sp, &mp->P_hi, &full[s], kc * 64, mb * 128);
-          tma_load_2d(sp + U_OPB, &mp->R_hi, &full[s], kc * 64, t.z * 128);
-          tma_load_2d(sp + 2 * U_OPB, &mp->Qn_hi, &full[s], kc * 64, t.z * 128);
+          const int k0 = kc * (int)KW;
           if (X3) {
-            tma_load_2d(sp + 3 * U_OPB, &mp->P_lo, &full[s], kc * 64, mb * 128);
-            tma_load_2d(sp + 4 * U_OPB, &mp->R_lo, &full[s], kc * 64, t.z * 128);
-            tma_load_2d(sp + 5 * U_OPB, &mp->Qn_lo, &full[s], kc * 64, t.z * 128);
+            tma_load_2d(sp, &mp->P_hi32, &full[s], k0, mb * 128);
+            tma_load_2d(sp + OPB, &mp->R_hi32, &full[s], k0, t.z * 128);
+            tma_load_2d(sp + 2 * OPB, &mp->Qn_hi32, &full[s], k0, t.z * 128);
+            tma_load_2d(sp + 3 * OPB, &mp->P_lo32, &full[s], k0, mb * 128);
+            tma_load_2d(sp + 4 * OPB, &mp->R_lo32, &full[s], k0, t.z * 128);
+            tma_load_2d(sp + 5 * OPB, &mp->Qn_lo32, &full[s], k0, t.z * 128);
+          } else {
+            tma_load_2d(sp, &mp->P_hi, &full[s], k0, mb * 128);
+            tma_load_2d(sp + OPB, &mp->R_hi, &full[s], k0, t.z * 128);
+            tma_load_2d(sp + 2 * OPB, &mp->Qn_hi, &full[s], k0, t.z * 128);
           }
         }
       }
@@ -130,7 +141,7 @@ __global__ void __launch_bounds__(U_THREADS, 1)
       for (int ti = off[seg]; ti < off[seg + 1] && ok; ++ti) {
         const int4 t = tiles[ti];
         if (!sh.active[t.x]) continue;
-        const int kch = (int)((sh.layers[t.x].r + 63) / 64);
+        const int kch = (int)((sh.layers[t.x].r + KW - 1) / KW);
         const uint32_t b = tcount & 1u, aph = (tcount >> 1) & 1u;
         if (!ab.wait(&acc_empty[b], aph ^ 1u, sh.status)) break;
         tc_fence_after();
@@ -140,19 +151,22 @@ __global__ void __launch_bounds__(U_THREADS, 1)
           if (!ab.wait(&full[s], ph, sh.status)) { ok = false; break; }
           tc_fence_after();
           const uint32_t base = smem_u32(stage + s * U_STAGE);
+          // K-major operand box o of the stage, advanced by k16 steps of 16 elements (32 bytes)
+          auto desc = [&](uint32_t o, int k16) {
+            const uint32_t a = base + o * OPB + (uint32_t)k16 * 32u;
+            return X3 ? smem_desc_sw64(a, 512) : smem_desc_sw128(a, 0, 1024);
+          };
 #pragma unroll
-          for (int k16 = 0; k16 < 4; ++k16) {
-            const uint64_t ad = smem_desc_sw128(base + k16 * 32, 0, 1024);
-            const uint64_t rd = smem_desc_sw128(base + U_OPB + k16 * 32, 0, 1024);
-            const uint64_t qd = smem_desc_sw128(base + 2 * U_OPB + k16 * 32, 0, 1024);
+          for (int k16 = 0; k16 < (int)(KW / 16u); ++k16) {
+            const uint64_t ad = desc(0, k16), rd = desc(1, k16), qd = desc(2, k16);
             const uint32_t acc = (kc | k16) ? 1u : 0u;
             umma_bf16(d1, ad, rd, U_IDESC, acc);
             umma_bf16(d2, ad, qd, U_IDESC, acc);
             if (X3) {  // P R^T = Ph Rh^T + Ph Rl^T + Pl Rh^T, P Q_t^T likewise
-              const uint64_t adl = smem_desc_sw128(base + 3 * U_OPB + k16 * 32, 0, 1024);
-              umma_bf16(d1, ad, smem_desc_sw128(base + 4 * U_OPB + k16 * 32, 0, 1024), U_IDESC, 1u);
+              const uint64_t adl = desc(3, k16);
+              umma_bf16(d1, ad, desc(4, k16), U_IDESC, 1u);
               umma_bf16(d1, adl, rd, U_IDESC, 1u);
-              umma_bf16(d2, ad, smem_desc_sw128(base + 5 * U_OPB + k16 * 32, 0, 1024), U_IDESC, 1u);
+              umma_bf16(d2, ad, desc(5, k16), U_IDESC, 1u);
               umma_bf16(d2, adl, qd, U_IDESC, 1u);
             }
           }
