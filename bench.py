@@ -100,9 +100,13 @@ def kernel_work(name: str, w, prec: str, gate: str = "always", wt=None):
     fused = prec == "bf16" and w.g_dtype == "bf16"
     b_in_m = fused and gate != "always"
     deferred = fused and not b_in_m
+    # BF16X3 in a gated mode: the buffer pass writes B alone; split_b writes the halves of the
+    # syncing layers' B after the gate
+    x3_split = prec == "bf16x3" and gate != "always"
     table = {
         # CUDA-core path (form_b runs on every layer before the gate)
-        "form_b": ("hbm", mn_all * (4 + gsz + (0 if fused else 4) + bh), "B"),
+        "form_b": ("hbm", mn_all * (4 + gsz + (0 if fused else 4) + (0 if x3_split else bh)), "B"),
+        "split_b": ("hbm", mn * 8, "B") if x3_split else ("latency", 0, ""),  # read B; write hi, lo
         "gemm_bq": ("alu", 2 * mnr, "flop"),
         "gemm_gram": ("alu", 2 * mr2, "flop"),
         "chol_inv": ("alu", 2 * r3 / 3, "flop"),
@@ -149,8 +153,10 @@ def step_bytes(w, prec, gate: str = "always", wt=None):
     fused = prec == "bf16" and w.g_dtype == "bf16"
     if prec == "fp32":  # form_b 12 (+4 with fp32 G), B Q and B^T P read B 4 + 4, update 16
         planned = mn_all * (4 + gsz + 4) + mn * (4 + 4 + 16)
-    elif prec == "bf16x3":  # form_b writes M, Bh, Bl; B Q and B^T P read both halves 4 + 4, update 16
+    elif prec == "bf16x3" and gate == "always":  # form_b writes M, Bh, Bl; B Q, B^T P read both halves, update 16
         planned = mn_all * (4 + gsz + 4 + 4) + mn * (4 + 4 + 16)
+    elif prec == "bf16x3":  # form_b writes M; synced: split_b 8, B Q and B^T P 4 + 4, update 16
+        planned = mn_all * (4 + gsz + 4) + mn * (8 + 4 + 4 + 16)
     elif fused and gate == "always":  # buffer pass fused with B Q 8, the Bh read of B^T P 2, update 18
         planned = mn_all * ((4 + gsz + 2) + 2 + (16 + gsz))
     elif fused:  # norms pass 10 on every layer; synced: fused B Q 6, Bh read 2, update 16

@@ -172,7 +172,8 @@ __device__ __forceinline__ double block_sum(double v, double *red /* >= THREADS/
 
 // ---------------------------------------------------------------- launch wrappers ---
 // CUDA-core (fp32) kernels, kernels_simt.cu
-void launch_form_b(const Shared &sh, const int4 *tiles, int32_t ntiles, cudaStream_t s);
+void launch_form_b(const Shared &sh, const int4 *tiles, int32_t ntiles, cudaStream_t s, bool halves = true);
+void launch_split_b(const Shared &sh, const int4 *tiles, int32_t ntiles, bool needed, cudaStream_t s);
 void launch_gate(const Shared &sh, const StepArgs &a, cudaStream_t s);
 // the branch from RMMC values already in a.rmmc (reduced over data-parallel workers)
 void launch_gate_reduced(const Shared &sh, const StepArgs &a, cudaStream_t s);

@@ -88,6 +88,10 @@ __device__ void form_b_tile(const DevLayer &L, int64_t row0, int64_t nrows, floa
   }
 }
 
+// HALVES: also write the layer's bf16 copy of B (or, in BF16X3, its two halves) where the plan
+// keeps one; without, only B (into M) and the norms, the halves following for the Dion-branch
+// layers alone once the gate has run (split_b_kernel).
+template <bool HALVES>
 __global__ void __launch_bounds__(kRowThreads) form_b_kernel(Shared sh, const int4 *tiles) {
   __shared__ double red[kRowThreads / 32];
   const int4 t = tiles[blockIdx.x];
@@ -95,7 +99,7 @@ __global__ void __launch_bounds__(kRowThreads) form_b_kernel(Shared sh, const in
   const DevLayer &L = sh.layers[t.x];
   DION_TILE_CHECK(t.y >= 0 && t.z >= 1 && (int64_t)t.y + t.z <= L.m, sh.status);
   float sb[4] = {0.f, 0.f, 0.f, 0.f}, sm[4] = {0.f, 0.f, 0.f, 0.f};
-  if (L.Bh != nullptr) {
+  if (HALVES && L.Bh != nullptr) {
     if (L.g_dtype == DT_BF16) form_b_tile<DT_BF16, true>(L, t.y, t.z, sb, sm);
     else form_b_tile<DT_FP32, true>(L, t.y, t.z, sb, sm);
   } else {
@@ -110,8 +114,53 @@ __global__ void __launch_bounds__(kRowThreads) form_b_kernel(Shared sh, const in
   }
 }
 
-void launch_form_b(const Shared &sh, const int4 *tiles, int32_t ntiles, cudaStream_t s) {
-  if (ntiles > 0) form_b_kernel<<<ntiles, kRowThreads, 0, s>>>(sh, tiles);
+void launch_form_b(const Shared &sh, const int4 *tiles, int32_t ntiles, cudaStream_t s, bool halves) {
+  if (ntiles <= 0) return;
+  if (halves) form_b_kernel<true><<<ntiles, kRowThreads, 0, s>>>(sh, tiles);
+  else form_b_kernel<false><<<ntiles, kRowThreads, 0, s>>>(sh, tiles);
+}
+
+// BF16X3, after the gate: the two bf16 halves of B (already in M) for the Dion-branch layers,
+// hi = bf16(B), lo = bf16(B - hi), the same roundings as form_b_tile.  Tile = a buffer-pass
+// row tile {layer, first row, rows, slot}.  `needed` false: the buffer pass already wrote them
+// (DION_GATE_ALWAYS), and every block returns at once.
+__global__ void __launch_bounds__(kRowThreads) split_b_kernel(Shared sh, const int4 *tiles, int needed) {
+  if (!needed) return;
+  const int4 t = tiles[blockIdx.x];
+  DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers, sh.status);
+  if (!sh.active[t.x]) return;
+  const DevLayer &L = sh.layers[t.x];
+  DION_TILE_CHECK(t.y >= 0 && t.z >= 1 && (int64_t)t.y + t.z <= L.m && L.Bh != nullptr && L.Bl != nullptr, sh.status);
+  const int64_t n = L.n, n4 = n >> 2;
+  for (int64_t rr = 0; rr < t.z; ++rr) {
+    const int64_t i = t.y + rr;
+    const float *Brow = L.M + i * L.ldm;
+    __nv_bfloat16 *hrow = L.Bh + i * L.ldbh, *lrow = L.Bl + i * L.ldbh;
+    for (int64_t c4 = threadIdx.x; c4 < n4; c4 += kRowThreads) {
+      const float4 b = *reinterpret_cast<const float4 *>(Brow + 4 * c4);
+      const __nv_bfloat162 h01 = __floats2bfloat162_rn(b.x, b.y), h23 = __floats2bfloat162_rn(b.z, b.w);
+      const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+      const __nv_bfloat162 l01 = __floats2bfloat162_rn(b.x - f01.x, b.y - f01.y);
+      const __nv_bfloat162 l23 = __floats2bfloat162_rn(b.z - f23.x, b.w - f23.y);
+      uint2 hv, lv;
+      hv.x = *reinterpret_cast<const uint32_t *>(&h01);
+      hv.y = *reinterpret_cast<const uint32_t *>(&h23);
+      lv.x = *reinterpret_cast<const uint32_t *>(&l01);
+      lv.y = *reinterpret_cast<const uint32_t *>(&l23);
+      *reinterpret_cast<uint2 *>(hrow + 4 * c4) = hv;
+      *reinterpret_cast<uint2 *>(lrow + 4 * c4) = lv;
+    }
+    for (int64_t c = 4 * n4 + threadIdx.x; c < n; c += kRowThreads) {
+      const float b = Brow[c];
+      const __nv_bfloat16 h = __float2bfloat16_rn(b);
+      hrow[c] = h;
+      lrow[c] = __float2bfloat16_rn(b - __bfloat162float(h));
+    }
+  }
+}
+
+void launch_split_b(const Shared &sh, const int4 *tiles, int32_t ntiles, bool needed, cudaStream_t s) {
+  if (ntiles > 0) split_b_kernel<<<ntiles, kRowThreads, 0, s>>>(sh, tiles, needed ? 1 : 0);
 }
 
 // =============================================================================== gate ===

@@ -333,7 +333,7 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   tp->num_sms = sms;
-  tp->launches = tp->fuse_buffer ? 17 : 18;
+  tp->launches = tp->fuse_buffer ? 17 : x3 ? 19 : 18;  // BF16X3: the split of B after the gate
   return e;
 }
 
@@ -357,10 +357,17 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh_in, const StepArgs &a
     launch_fused_bq(sh, tp, true, s);
     tick(p, s, "tc_form_bq");
   } else {
-    launch_form_b(sh, btiles, n_btiles, s);  // B = M + G (and its bf16 copy or halves), ||B||, ||M_{t-1}||
+    // BF16X3 in a gated mode writes the halves of B only for the Dion-branch layers, after the
+    // gate (a local layer needs B alone): 10 B/element on every layer, 8 more on syncing ones
+    const bool x3_split = tp.precision == DION_PREC_BF16X3 && a.gate_mode != GATE_ALWAYS;
+    launch_form_b(sh, btiles, n_btiles, s, !x3_split);  // B = M + G (its bf16 copy or halves), the norms
     tick(p, s, "form_b");
     launch_gate(sh, a, s);
     tick(p, s, "gate");
+    if (tp.precision == DION_PREC_BF16X3) {
+      launch_split_b(sh, btiles, n_btiles, x3_split, s);
+      tick(p, s, "split_b");
+    }
     launch_form_bq(sh, tp, s);  // P = B Q_{t-1} on the layers that take the Dion branch
     tick(p, s, "tc_bq");
   }
@@ -403,12 +410,13 @@ void step_phase(const TcPlan &tp, const Shared &sh_in, const StepArgs &a, int32_
       if (tp.fuse_buffer) {
         launch_norms_gate(sh, a, tp.ftiles, tp.n_ftiles, s);
       } else {
-        launch_form_b(sh, btiles, n_btiles, s);
+        launch_form_b(sh, btiles, n_btiles, s, !x3);  // BF16X3: the halves after the branch is known
         launch_gate(sh, a, s);
       }
       break;
     case DION_PHASE_POWER:  // the branch from the reduced RMMC, then P = B Q on the Dion layers
       launch_gate_reduced(sh, a, s);
+      if (x3) launch_split_b(sh, btiles, n_btiles, true, s);
       if (tp.fuse_buffer) launch_fused_bq(sh, tp, true, s);
       else launch_form_bq(sh, tp, s);
       break;

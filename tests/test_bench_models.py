@@ -56,6 +56,22 @@ def test_kernel_bytes_follow_branches(stack):
     assert bench.kernel_work("tc_update", stack, "bf16", "per_layer", wt)[1] == 16 * big
 
 
+def test_bf16x3_gated_splits_b_after_the_gate():
+    """BF16X3 with bf16 G: in DION_GATE_ALWAYS the buffer pass writes B and both halves (14 B per
+    element); in a gated mode it writes B alone (10) and split_b writes the halves of the syncing
+    layers (8 per synced element): 10 per element on a local step, 42 on a synced one."""
+    w = wl.WORKLOADS["gpt350m_gate_stress_r256"]
+    mn, L = _mn(w), w.num_layers
+    assert bench.kernel_work("form_b", w, "bf16x3")[1] == 14 * mn
+    assert bench.kernel_work("form_b", w, "bf16x3", "per_layer", [0.0] * L)[1] == 10 * mn
+    assert bench.kernel_work("split_b", w, "bf16x3", "per_layer", [0.0] * L)[1] == 0
+    assert bench.kernel_work("split_b", w, "bf16x3", "per_layer", [1.0] * L)[1] == 8 * mn
+    assert bench.kernel_work("split_b", w, "bf16x3")[0] == "latency"  # returns at once in ALWAYS
+    assert bench.step_bytes(w, "bf16x3")[0] == 14 * mn + 24 * mn
+    assert bench.step_bytes(w, "bf16x3", "per_layer", [1.0] * L)[0] == 10 * mn + 32 * mn
+    assert bench.step_bytes(w, "bf16x3", "per_layer", [0.0] * L)[0] == 10 * mn + 10 * mn
+
+
 def test_flat_gradient_views_match_layers():
     w = wl.WORKLOADS["gpt160m_block_r192"]
     seq = bench.make_gradient_sequence(wl, w, torch.bfloat16, "cpu", range(3, 5))
