@@ -69,11 +69,31 @@ def sources_hash(names) -> str:
 
 # ------------------------------------------------------------------ algorithmic work ---
 
-def kernel_work(name: str, w, prec: str, gate: str = "always", wt=None):
+def kernel_work(name: str, w, prec: str, gate: str = "always", wt=None, peaks=None):
     """(bound, algorithmic units per launch, unit) for one kernel of the step.  wt[l] is the
     fraction of the timed steps in which layer l took the Dion branch (all 1 with --gate always);
     kernels that run only on syncing layers count those layers' work by it.  Bytes count each
-    compulsory read and write once; flops count 2 per multiply-add."""
+    compulsory read and write once; flops count 2 per multiply-add.  With `peaks`, a bf16
+    contraction (B Q, B^T P, the update) is held to whichever of its two rooflines takes longer:
+    its bytes at the HBM copy rate or its tensor flops at the sustained bf16 rate (BF16X3 issues
+    three products per multiply-add)."""
+    base_work = _kernel_work(name, w, prec, gate, wt)
+    if peaks is None or base_work[0] != "hbm":
+        return base_work
+    base = name.rstrip("0123456789")
+    ranks = w.ranks()
+    wts = [1.0] * len(w.shapes) if wt is None else list(wt)
+    mnr = sum(m * n * r * wts[l] for l, ((m, n), r) in enumerate(zip(w.shapes, ranks)))
+    prods = 3 if prec == "bf16x3" else 1
+    flops = {"tc_bq": 2 * mnr, "tc_form_bq": 2 * mnr, "tc_btp": 2 * mnr, "tc_update": 4 * mnr}.get(base)
+    if flops is None:
+        return base_work
+    t_hbm = base_work[1] / (peaks["hbm"] * 1e9)
+    t_tensor = prods * flops / (peaks["bf16_sust"] * 1e12)
+    return ("tensor", prods * flops, "flop") if t_tensor > t_hbm else base_work
+
+
+def _kernel_work(name: str, w, prec: str, gate: str = "always", wt=None):
     gsz = 2 if w.g_dtype == "bf16" else 4
     ranks = w.ranks()
     L = len(w.shapes)
@@ -465,7 +485,7 @@ def run_ours(args, rank, world, local_rank):
     peaks = load_peaks()
     kern = []
     for name, ms in ktimes:
-        bound, units, unit = kernel_work(name, w, prec, args.gate, wt)
+        bound, units, unit = kernel_work(name, w, prec, args.gate, wt, peaks)
         kern.append(dict(name=name, ms=ms, bound=bound, units=units, unit=unit))
     dom = max(kern, key=lambda k: k["ms"]) if kern else None
     roofline = None
