@@ -73,7 +73,8 @@ enum { DION_DTYPE_FP32 = 0, DION_DTYPE_BF16 = 1 };
  *                      and a low bf16 half (x ~ hi + lo, |x - hi - lo| <= 2^-18 |x|) and three
  *                      products per step (hi*hi + hi*lo + lo*hi); Orthogonalize's Gram and
  *                      triangular solves on tcgen05 kind::tf32 with fp32 operands split the same
- *                      way into tf32 halves (3xTF32), its Cholesky in fp32 on CUDA cores:
+ *                      way into tf32 halves (3xTF32), the first Cholesky's trailing update
+ *                      likewise, the rest of the Cholesky in fp32 on CUDA cores:
  *                      fp32-class accuracy for ill-conditioned P.  Ranks up to 256
  *                      (dion_plan_create returns DION_ERR_UNSUPPORTED above). */
 enum { DION_PREC_FP32 = 0, DION_PREC_BF16 = 1, DION_PREC_BF16X3 = 2 };

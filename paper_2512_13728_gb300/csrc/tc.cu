@@ -328,7 +328,7 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   if (tp->fuse_buffer && tp->fb_smem > 227u * 1024u) return cudaErrorInvalidValue;
   if (e == cudaSuccess && tp->fuse_buffer) e = setup_fused_bq_kernel(tp->fb_smem);
   if (e == cudaSuccess) e = setup_orth_kernels(tp->o_smem, x3);
-  if (e == cudaSuccess && !x3) e = prepare_chol_inv_tc(lo.max_r, &tp->chol_tc_smem);
+  if (e == cudaSuccess) e = prepare_chol_inv_tc(lo.max_r, &tp->chol_tc_smem);
   int dev = 0, sms = 0;
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -378,7 +378,7 @@ void step(dion_plan *p, const TcPlan &tp, const Shared &sh_in, const StepArgs &a
   for (int pass = 0; pass < 3; ++pass) {  // CholeskyQR2; the third pass only after a shifted retry
     launch_orth(sh, tp, true, pass, s);  // S = X^T X
     tick(p, s, kGram[pass]);
-    if (pass == 0 && !x3) launch_chol_inv_tc(sh, tp.maps, tp.chol_tc_smem, s);  // trailing update on tensor cores
+    if (pass == 0) launch_chol_inv_tc(sh, tp.maps, tp.chol_tc_smem, s);  // trailing update on tensor cores (3xTF32)
     else launch_chol_inv(sh, chol_smem, pass, x3 ? 1e-3f : 6e-2f, s);  // passes 1-2: usually the first-order factor
     tick(p, s, kChol[pass]);
     launch_orth(sh, tp, false, pass, s);  // X L^{-T} and its transpose, or its bf16 copy (halves) at the end
@@ -424,7 +424,7 @@ void step_phase(const TcPlan &tp, const Shared &sh_in, const StepArgs &a, int32_
       launch_transpose_praw(sh, tp, s);  // the first Gram reads P_raw^T
       for (int pass = 0; pass < 3; ++pass) {
         launch_orth(sh, tp, true, pass, s);
-        if (pass == 0 && !x3) launch_chol_inv_tc(sh, tp.maps, tp.chol_tc_smem, s);
+        if (pass == 0) launch_chol_inv_tc(sh, tp.maps, tp.chol_tc_smem, s);
         else launch_chol_inv(sh, chol_smem, pass, x3 ? 1e-3f : 6e-2f, s);
         launch_orth(sh, tp, false, pass, s);
       }
