@@ -525,6 +525,7 @@ void launch_gemm(const Shared &sh, const GemmProblem *probs, const int4 *tiles, 
 // is set and L^{-1} = 0 for the layer, so its P, R and Q become 0, M becomes B and X is
 // unchanged (no NaN written).
 constexpr int kCholThreads = 512;
+constexpr int kFoBatch = 8;  // 16-byte groups each thread has in flight in the first-order factor
 
 // Column c of Y lives at ysw(c): bit 2 flips when bit 5 is set, so the two 16-byte halves of
 // an 8-column group swap in every other 32-column stretch.  Eight consecutive groups read by
@@ -758,19 +759,33 @@ __global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, in
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
   if (pass >= 1) {
-    // ||E||_F^2 from the lower triangle (E symmetric), fixed-order reduction; 16-byte loads
-    // (a row's padding up to the next multiple of 4 columns lies inside ls and is masked)
+    // ||E||_F^2 from the lower triangle (E symmetric), fixed-order reduction.  The 16-byte
+    // groups (i, j4) of the r x ceil(r / 4) grid are taken in a flat order, consecutive threads
+    // on consecutive groups of a row, kFoBatch groups per thread in flight (a row's padding up to
+    // the next multiple of 4 columns lies inside ls and is masked; groups above the diagonal are
+    // not loaded)
+    const int r4 = (r + 3) / 4;
+    const int64_t groups = (int64_t)r * r4;
     double fs = 0.0;
-    for (int i = warp; i < r; i += kCholThreads / 32) {
+    for (int64_t g0 = tid; g0 < groups; g0 += (int64_t)kCholThreads * kFoBatch) {
+      float4 v[kFoBatch];
+#pragma unroll
+      for (int u = 0; u < kFoBatch; ++u) {
+        const int64_t g = g0 + (int64_t)u * kCholThreads;
+        const int i = (int)(g / r4), j4 = (int)(g % r4);
+        v[u] = (g < groups && 4 * j4 <= i) ? *reinterpret_cast<const float4 *>(S + (int64_t)i * ls + 4 * j4)
+                                           : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
       float a = 0.f;
-#pragma unroll 4
-      for (int j4 = lane; 4 * j4 <= i; j4 += 32) {
-        const float4 v = *reinterpret_cast<const float4 *>(S + (int64_t)i * ls + 4 * j4);
-        const float ve[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+      for (int u = 0; u < kFoBatch; ++u) {
+        const int64_t g = g0 + (int64_t)u * kCholThreads;
+        const int i = (int)(g / r4), j4 = (int)(g % r4);
+        const float ve[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
           const int j = 4 * j4 + c;
-          const float e = (j <= i) ? ve[c] - (i == j ? 1.f : 0.f) : 0.f;
+          const float e = (g < groups && j <= i) ? ve[c] - (i == j ? 1.f : 0.f) : 0.f;
           a = fmaf((j < i ? 2.f : 1.f) * e, e, a);
         }
       }
@@ -785,14 +800,23 @@ __global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, in
       lam = power_norm_sym(S, r, ls, Y, ldy);
     }
     if (isfinite(lam) && 1.5f * lam < near_identity) {
-      // 16-byte loads and stores; a group that straddles column r is stored element-wise
-      const int r4 = (r + 3) / 4;
-      for (int i = warp; i < r; i += kCholThreads / 32) {
-#pragma unroll 4
-        for (int j4 = lane; j4 < r4; j4 += 32) {
-          float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-          if (4 * j4 <= i) v = *reinterpret_cast<const float4 *>(S + (int64_t)i * ls + 4 * j4);
-          float o[4] = {v.x, v.y, v.z, v.w};
+      // the same flat order over the groups of every row; 16-byte loads and stores (a group
+      // that straddles column r is stored element-wise)
+      for (int64_t g0 = tid; g0 < groups; g0 += (int64_t)kCholThreads * kFoBatch) {
+        float4 v[kFoBatch];
+#pragma unroll
+        for (int u = 0; u < kFoBatch; ++u) {
+          const int64_t g = g0 + (int64_t)u * kCholThreads;
+          const int i = (int)(g / r4), j4 = (int)(g % r4);
+          v[u] = (g < groups && 4 * j4 <= i) ? *reinterpret_cast<const float4 *>(S + (int64_t)i * ls + 4 * j4)
+                                             : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int u = 0; u < kFoBatch; ++u) {
+          const int64_t g = g0 + (int64_t)u * kCholThreads;
+          if (g >= groups) break;
+          const int i = (int)(g / r4), j4 = (int)(g % r4);
+          float o[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
 #pragma unroll
           for (int c = 0; c < 4; ++c) {
             const int j = 4 * j4 + c;
