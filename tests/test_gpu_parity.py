@@ -135,16 +135,21 @@ def test_ragged_shapes_fp32(pad):
     run_per_step(RAGGED, cd.DION_PREC_FP32, dict(gate_mode=oc.GATE_ALWAYS), RAGGED.steps, TOL_FP32, pad=pad)
 
 
+@pytest.mark.parametrize("gate", ["always", "per_layer"])
 @pytest.mark.parametrize("g_dtype", ["bf16", "fp32"])
 @pytest.mark.parametrize("pad", [0, 1])
-def test_ragged_shapes_bf16x3(pad, g_dtype):
+def test_ragged_shapes_bf16x3(pad, g_dtype, gate):
     """Split-operand tensor-core mode on ragged shapes, several tiles and NaN-padded rows, at the
-    fp32 tolerance with either gradient dtype."""
+    fp32 tolerance with either gradient dtype.  Under the per-layer gate the buffer pass writes B
+    alone and the halves of B follow for the syncing layers after the gate (their column tails
+    included: n = 33, 5, 1)."""
     import paper_2512_13728_gb300 as cd
 
     w = wl.scaled(RAGGED, "ragged_x3", RAGGED.shapes, g_dtype=g_dtype)
-    worst, _ = run_per_step(w, cd.DION_PREC_BF16X3, dict(gate_mode=oc.GATE_ALWAYS), w.steps, TOL_FP32, pad=pad)
-    print("bf16x3 ragged", g_dtype, worst)
+    gm = oc.GATE_ALWAYS if gate == "always" else oc.GATE_PER_LAYER
+    taus = [0.5, 1e6, 0.5, 1e6, 0.5, 0.5] if gate == "per_layer" else None  # two layers stay local
+    worst, _ = run_per_step(w, cd.DION_PREC_BF16X3, dict(gate_mode=gm), w.steps, TOL_FP32, pad=pad, taus=taus)
+    print("bf16x3 ragged", g_dtype, gate, worst)
 
 
 def test_bf16x3_full_rank_and_rank_256():
