@@ -535,19 +535,23 @@ def test_checkpoint_resume_bitwise():
     plan2.close()
 
 
+@pytest.mark.parametrize("gate", ["always", "per_layer"])
 @pytest.mark.parametrize("prec", ["fp32", "bf16", "bf16x3"])
-def test_cuda_graph_replay_matches_direct_steps(prec):
+def test_cuda_graph_replay_matches_direct_steps(prec, gate):
     """dion_step only enqueues kernels (no host sync, no allocation), so a caller can capture it in
-    a CUDA graph: three replays of one captured step give the bits of three direct steps."""
+    a CUDA graph: three replays of one captured step give the bits of three direct steps.  Under
+    the per-layer gate the branch is decided on the device each replay (two layers' thresholds
+    keep them local after the first step)."""
     import paper_2512_13728_gb300 as cd
 
     outs = []
     for use_graph in (False, True):
-        st = gu.make_state(RAGGED)
+        taus = [0.5, 1e6, 0.5, 1e6, 0.5, 0.5] if gate == "per_layer" else None
+        st = gu.make_state(RAGGED, taus=taus)
         gu.write_gradients(st, 1)
         plan = cd.Plan(st.X, st.M, st.Q, st.G, st.taus, PRECS[prec])
         torch.cuda.synchronize()
-        hp = cd.hparams(step=1)
+        hp = cd.hparams(step=1, gate_mode=cd.DION_GATE_ALWAYS if gate == "always" else cd.DION_GATE_PER_LAYER)
         if use_graph:
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g):
@@ -559,7 +563,8 @@ def test_cuda_graph_replay_matches_direct_steps(prec):
                 plan.step(hp)
         torch.cuda.synchronize()
         assert plan.device_status() == 0
-        outs.append([x.clone() for x in st.X + st.M + st.Q] + [plan.rmmc.clone(), plan.prev_norm.clone()])
+        outs.append([x.clone() for x in st.X + st.M + st.Q] + [plan.rmmc.clone(), plan.prev_norm.clone(),
+                                                                plan.flags.clone()])
         plan.close()
     for a, b in zip(*outs):
         assert torch.equal(a, b)
