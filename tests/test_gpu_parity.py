@@ -331,7 +331,7 @@ def test_ragged_shapes_bf16_per_layer_gate(pad):
                  TOL_BF16, pad=pad, taus=[1e6, 1e-6, 0.5, 0.5, 1e-6, 1e6])
 
 
-@pytest.mark.parametrize("prec", ["bf16", "fp32"])
+@pytest.mark.parametrize("prec", ["bf16", "fp32", "bf16x3"])
 def test_weight_decay_both_branches(prec):
     """Decoupled weight decay (Section 4's 0.01, here 0.5 so that it is visible against the
     tolerance) in the Dion branch and the local branch: a per-layer gate with one layer that
@@ -339,7 +339,7 @@ def test_weight_decay_both_branches(prec):
     against the oracle step by step."""
     import paper_2512_13728_gb300 as cd
 
-    p = cd.DION_PREC_BF16 if prec == "bf16" else cd.DION_PREC_FP32
+    p = PRECS[prec]
     w = wl.scaled(wl.WORKLOADS["gpt350m_gate_stress_r256"], "wd", [(128, 192), (192, 128), (64, 64)],
                   rank=16, steps=6, kind="gaussian")
     run_per_step(w, p, dict(gate_mode=oc.GATE_PER_LAYER, tau_global=0.5, eta=0.05, eta_local=0.03,
@@ -453,7 +453,8 @@ def test_deterministic_bitwise_bf16_mode(g_dtype, prec):
 
 @pytest.mark.parametrize("prec,g_dtype,mode", [("bf16", "bf16", "always"), ("bf16", "fp32", "always"),
                                                ("fp32", "bf16", "always"), ("bf16", "bf16", "per_layer"),
-                                               ("bf16", "bf16", "global"), ("fp32", "fp32", "per_layer")])
+                                               ("bf16", "bf16", "global"), ("fp32", "fp32", "per_layer"),
+                                               ("bf16x3", "bf16", "always"), ("bf16x3", "bf16", "per_layer")])
 def test_step_host_matches_device_gradients(prec, g_dtype, mode):
     """dion_step_host (gradients copied from pinned host tensors into the plan's two alternating
     buffers) gives bit for bit the results of dion_step on the same gradients in device memory;
@@ -463,7 +464,7 @@ def test_step_host_matches_device_gradients(prec, g_dtype, mode):
     import paper_2512_13728_gb300 as cd
 
     gm = {"always": cd.DION_GATE_ALWAYS, "per_layer": cd.DION_GATE_PER_LAYER, "global": cd.DION_GATE_GLOBAL}[mode]
-    p = cd.DION_PREC_BF16 if prec == "bf16" else cd.DION_PREC_FP32
+    p = PRECS[prec]
     w = wl.scaled(RAGGED, "ragged_host", RAGGED.shapes, g_dtype=g_dtype, steps=5)
     outs = []
     for host in (False, True):
