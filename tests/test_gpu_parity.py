@@ -284,14 +284,15 @@ def test_ragged_shapes_bf16_fp32_gradients():
     run_per_step(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_ALWAYS), w.steps, TOL_BF16, pad=1)
 
 
-def test_gpt160m_block_r192_bf16_50_steps():
+@pytest.mark.parametrize("prec", ["bf16", "bf16x3"])
+def test_gpt160m_block_r192_bf16_50_steps(prec):
     """One GPT-160M-shaped block (six matrices, r = 192, bf16 gradients) over its stated 50 steps,
-    every step against an oracle step from the device state."""
-    import paper_2512_13728_gb300 as cd
-
+    every step against an oracle step from the device state (bf16 operands at 2e-2, split
+    operands at 1e-4)."""
     w = wl.WORKLOADS["gpt160m_block_r192"]
-    worst, _ = run_per_step(w, cd.DION_PREC_BF16, dict(gate_mode=oc.GATE_ALWAYS), w.steps, TOL_BF16)
-    print("bf16 block, 50 steps, worst", worst)
+    worst, _ = run_per_step(w, PRECS[prec], dict(gate_mode=oc.GATE_ALWAYS), w.steps,
+                            TOL_BF16 if prec == "bf16" else TOL_FP32)
+    print(prec, "block, 50 steps, worst", worst)
 
 
 @pytest.mark.parametrize("rank", [300, 400])
