@@ -638,8 +638,9 @@ def main():
     if args.tf32_peak:
         print(json.dumps(measure_tf32_peak()), flush=True)
         return
-    if args.warmup < 3:
-        ap.error("--warmup must be >= 3")
+    if args.warmup < 3:  # the timing rules ask for at least 3 warm-up steps; the line reports 3
+        print(f"bench.py: --warmup {args.warmup} raised to 3", file=sys.stderr)
+        args.warmup = 3
     if args.precision is None:
         args.precision = os.environ.get("CURVADION_BENCH_PRECISION", "bf16")
 
