@@ -140,6 +140,8 @@ struct Shared {
 // mode: GEMM_ACTIVE runs on active layers; GEMM_SHIFTED only where orth_shifted is set;
 // GEMM_SHIFTED_OR_COPY multiplies where orth_shifted is set and copies A to C elsewhere.
 enum : int32_t { GEMM_ACTIVE = 0, GEMM_SHIFTED = 1, GEMM_SHIFTED_OR_COPY = 2 };
+constexpr int kGemmTile = 128;  // output tile edge of the CUDA-core grouped GEMM
+constexpr int kUpdTileM = 128, kUpdTileN = 64;  // output tile of the CUDA-core update (FP32 mode)
 struct GemmProblem {
   const float *A;
   const float *B;

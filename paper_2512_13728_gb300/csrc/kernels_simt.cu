@@ -415,9 +415,26 @@ void launch_norms_gate(const Shared &sh, const StepArgs &a, const int4 *tiles, i
 }
 
 // ==================================================================== grouped GEMM ===
-// C = op(A) op(B) over a list of problems; 64 x 64 output tiles, 16-deep k slices staged in
-// shared memory, 4 x 4 register tile per thread.  Tile = {problem, tile row, tile col}.
-constexpr int GBM = 64, GBN = 64, GBK = 16, kGemmThreads = 256;
+// C = op(A) op(B) over a list of problems (the FP32 mode's contractions) on CUDA cores: 128 x 128
+// output tiles, 8-deep k slices through two shared-memory buffers (the next slice's global loads
+// are in flight while the current one is multiplied), 8 x 8 outputs per thread as 2 x 2 blocks
+// of 4 x 4 that lie 64 rows / columns apart, so each k step reads 16 bytes per operand block per
+// thread without bank conflicts.  Global loads are 16 bytes along whichever dimension of an
+// operand is contiguous (zero outside the matrix).  Tile = {problem, tile row, tile col}.
+constexpr int GBM = kGemmTile, GBN = kGemmTile, GBK = 8, kGemmThreads = 256;
+
+// Elements (row, col .. col + 3) of a row-major matrix (col a multiple of 4, rows 16-byte
+// aligned), zero outside it.
+__device__ __forceinline__ float4 ld4_rows(const float *base, int64_t row, int64_t col, int64_t rows, int64_t cols,
+                                           int64_t ld) {
+  if (row >= rows || col >= cols) return make_float4(0.f, 0.f, 0.f, 0.f);
+  const float *p = base + row * ld + col;
+  if (col + 4 <= cols) return *reinterpret_cast<const float4 *>(p);
+  float v[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int e = 0; e < 4; ++e)
+    if (col + e < cols) v[e] = p[e];
+  return make_float4(v[0], v[1], v[2], v[3]);
+}
 
 __global__ void __launch_bounds__(kGemmThreads) gemm_kernel(Shared sh, const GemmProblem *probs,
                                                             const int4 *tiles) {
@@ -438,53 +455,74 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_kernel(Shared sh, const Gem
     }
     return;
   }
-  __shared__ float As[GBK][GBM + 4];
-  __shared__ float Bs[GBK][GBN + 4];
-  float acc[4][4] = {};
+  __shared__ __align__(16) float As[2][GBK][GBM + 4];
+  __shared__ __align__(16) float Bs[2][GBK][GBN + 4];
+  // this thread's 16-byte share of a k slice of A (128 x 8) and of B (8 x 128): along the
+  // contiguous dimension, 4 consecutive elements of one row / column
+  const int a_r = p.transA ? (tid >> 5) : (tid >> 1), a_c = p.transA ? (tid & 31) * 4 : (tid & 1) * 4;
+  const int b_r = p.transB ? (tid >> 1) : (tid >> 5), b_c = p.transB ? (tid & 1) * 4 : (tid & 31) * 4;
+  auto load = [&](int64_t k0, float4 &av, float4 &bv) {
+    av = p.transA ? ld4_rows(p.A, k0 + a_r, i0 + a_c, p.K, p.Mrows, p.lda)   // A^T stored K x M
+                  : ld4_rows(p.A, i0 + a_r, k0 + a_c, p.Mrows, p.K, p.lda);  // A stored M x K
+    bv = p.transB ? ld4_rows(p.B, j0 + b_r, k0 + b_c, p.Ncols, p.K, p.ldb)   // B^T stored N x K
+                  : ld4_rows(p.B, k0 + b_r, j0 + b_c, p.K, p.Ncols, p.ldb);  // B stored K x N
+  };
+  auto store = [&](int buf, const float4 &av, const float4 &bv) {
+    if (p.transA) {
+      *reinterpret_cast<float4 *>(&As[buf][a_r][a_c]) = av;
+    } else {
+      As[buf][a_c + 0][a_r] = av.x; As[buf][a_c + 1][a_r] = av.y;
+      As[buf][a_c + 2][a_r] = av.z; As[buf][a_c + 3][a_r] = av.w;
+    }
+    if (p.transB) {
+      Bs[buf][b_c + 0][b_r] = bv.x; Bs[buf][b_c + 1][b_r] = bv.y;
+      Bs[buf][b_c + 2][b_r] = bv.z; Bs[buf][b_c + 3][b_r] = bv.w;
+    } else {
+      *reinterpret_cast<float4 *>(&Bs[buf][b_r][b_c]) = bv;
+    }
+  };
+  float acc[8][8] = {};
+  float4 av, bv;
+  load(0, av, bv);
+  store(0, av, bv);
+  __syncthreads();
+  int cur = 0;
   for (int64_t k0 = 0; k0 < p.K; k0 += GBK) {
-#pragma unroll
-    for (int s = 0; s < (GBM * GBK) / kGemmThreads; ++s) {
-      const int idx = tid + s * kGemmThreads;
-      int ii, kk;
-      if (p.transA) { ii = idx % GBM; kk = idx / GBM; } else { kk = idx % GBK; ii = idx / GBK; }
-      const int64_t gi = i0 + ii, gk = k0 + kk;
-      float v = 0.f;
-      if (gi < p.Mrows && gk < p.K) v = p.transA ? p.A[gk * p.lda + gi] : p.A[gi * p.lda + gk];
-      As[kk][ii] = v;
-    }
-#pragma unroll
-    for (int s = 0; s < (GBN * GBK) / kGemmThreads; ++s) {
-      const int idx = tid + s * kGemmThreads;
-      int jj, kk;
-      if (p.transB) { kk = idx % GBK; jj = idx / GBK; } else { jj = idx % GBN; kk = idx / GBN; }
-      const int64_t gj = j0 + jj, gk = k0 + kk;
-      float v = 0.f;
-      if (gj < p.Ncols && gk < p.K) v = p.transB ? p.B[gj * p.ldb + gk] : p.B[gk * p.ldb + gj];
-      Bs[kk][jj] = v;
-    }
-    __syncthreads();
+    const bool more = k0 + GBK < p.K;
+    if (more) load(k0 + GBK, av, bv);  // in flight during this slice's products
 #pragma unroll
     for (int kk = 0; kk < GBK; ++kk) {
-      float av[4], bv[4];
+      const float4 a0 = *reinterpret_cast<const float4 *>(&As[cur][kk][ty * 4]);
+      const float4 a1 = *reinterpret_cast<const float4 *>(&As[cur][kk][64 + ty * 4]);
+      const float4 b0 = *reinterpret_cast<const float4 *>(&Bs[cur][kk][tx * 4]);
+      const float4 b1 = *reinterpret_cast<const float4 *>(&Bs[cur][kk][64 + tx * 4]);
+      const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+      const float b[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
-      for (int i = 0; i < 4; ++i) av[i] = As[kk][ty * 4 + i];
+      for (int i = 0; i < 8; ++i)
 #pragma unroll
-      for (int j = 0; j < 4; ++j) bv[j] = Bs[kk][tx * 4 + j];
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+        for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
     }
+    if (more) store(cur ^ 1, av, bv);
     __syncthreads();
+    cur ^= 1;
   }
+  // output rows ty*4 + (0..3) and 64 + ty*4 + (0..3), columns likewise with tx
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int64_t gi = i0 + ty * 4 + i;
+  for (int i = 0; i < 8; ++i) {
+    const int64_t gi = i0 + (i < 4 ? ty * 4 + i : 64 + ty * 4 + (i - 4));
     if (gi >= p.Mrows) continue;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int64_t gj = j0 + tx * 4 + j;
-      if (gj < p.Ncols) p.C[gi * p.ldc + gj] = acc[i][j];
+    for (int h = 0; h < 2; ++h) {
+      const int64_t gj = j0 + h * 64 + tx * 4;
+      float *c = p.C + gi * p.ldc + gj;
+      if (gj + 4 <= p.Ncols) {
+        *reinterpret_cast<float4 *>(c) = make_float4(acc[i][4 * h], acc[i][4 * h + 1], acc[i][4 * h + 2], acc[i][4 * h + 3]);
+      } else {
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          if (gj + e < p.Ncols) c[e] = acc[i][4 * h + e];
+      }
     }
   }
 }
@@ -929,15 +967,19 @@ void launch_colnorm(const Shared &sh, const int4 *tiles, int32_t ntiles, float e
 
 // =============================================================== error feedback + update ===
 // M = B - (1 - mu) P R^T and X = X - eta sqrt(m/n) P Q_t^T in one pass over the tile, plus the
-// fp64 partial of ||M_t||^2 for Equation 1.  Tile = {layer, tile row, tile col, slot}.
-constexpr int UBM = 64, UBN = 64, UBK = 16, kUpdThreads = 256;
+// fp64 partial of ||M_t||^2 for Equation 1.  128 x 64 tiles, 8-deep k slices through two
+// shared-memory buffers (the next slice's 16-byte loads in flight during this one's products),
+// 8 x 4 outputs of each product per thread (rows 64 apart, so the 16-byte shared reads are
+// conflict-free); the epilogue reads and writes M and X 16 bytes at a time.
+// Tile = {layer, tile row, tile col, slot}.
+constexpr int UBM = kUpdTileM, UBN = kUpdTileN, UBK = 8, kUpdThreads = 256;
 
-__global__ void __launch_bounds__(kUpdThreads) update_kernel(Shared sh, const int4 *tiles, float mu, float eta,
+__global__ void __launch_bounds__(kUpdThreads, 2) update_kernel(Shared sh, const int4 *tiles, float mu, float eta,
                                                              float keep) {
-  // P, R: ld ldp; Q: ld ldq
-  __shared__ float As[UBK][UBM + 4];
-  __shared__ float Rs[UBK][UBN + 4];
-  __shared__ float Qs[UBK][UBN + 4];
+  // P, R: ld ldp; Q: ld ldq; k slices stored transposed (K-th row = one k of every tile row)
+  __shared__ __align__(16) float As[2][UBK][UBM + 4];
+  __shared__ __align__(16) float Rs[2][UBK][UBN + 4];
+  __shared__ __align__(16) float Qs[2][UBK][UBN + 4];
   __shared__ double red[kUpdThreads / 32];
   const int4 t = tiles[blockIdx.x];
   DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers && t.y >= 0 && t.z >= 0 &&
@@ -946,51 +988,77 @@ __global__ void __launch_bounds__(kUpdThreads) update_kernel(Shared sh, const in
   const DevLayer &L = sh.layers[t.x];
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
   const int64_t i0 = (int64_t)t.y * UBM, j0 = (int64_t)t.z * UBN, r = L.r, ldp = L.ldp;
-  float u1[4][4] = {}, u2[4][4] = {};
+  // this thread's share of a k slice: 4 consecutive k of one row of P, and of one row of R
+  // (threads 0..127) or of Q_t (threads 128..255)
+  const int pr = tid >> 1, kq = (tid & 1) * 4, br = (tid & 127) >> 1;
+  const bool is_q = tid >= 128;
+  auto load = [&](int64_t k0, float4 &pv, float4 &bv) {
+    pv = ld4_rows(L.P, i0 + pr, k0 + kq, L.m, r, ldp);
+    bv = is_q ? ld4_rows(L.Q, j0 + br, k0 + kq, L.n, r, L.ldq) : ld4_rows(L.R, j0 + br, k0 + kq, L.n, r, ldp);
+  };
+  auto store = [&](int buf, const float4 &pv, const float4 &bv) {
+    As[buf][kq + 0][pr] = pv.x; As[buf][kq + 1][pr] = pv.y;
+    As[buf][kq + 2][pr] = pv.z; As[buf][kq + 3][pr] = pv.w;
+    float(*Bd)[UBN + 4] = is_q ? Qs[buf] : Rs[buf];
+    Bd[kq + 0][br] = bv.x; Bd[kq + 1][br] = bv.y;
+    Bd[kq + 2][br] = bv.z; Bd[kq + 3][br] = bv.w;
+  };
+  float u1[8][4] = {}, u2[8][4] = {};
+  float4 pv, bv;
+  load(0, pv, bv);
+  store(0, pv, bv);
+  __syncthreads();
+  int cur = 0;
   for (int64_t k0 = 0; k0 < r; k0 += UBK) {
-#pragma unroll
-    for (int s = 0; s < (UBM * UBK) / kUpdThreads; ++s) {
-      const int idx = tid + s * kUpdThreads;
-      const int kk = idx % UBK, ii = idx / UBK;
-      const int64_t gk = k0 + kk, gi = i0 + ii, gj = j0 + ii;
-      As[kk][ii] = (gi < L.m && gk < r) ? L.P[gi * ldp + gk] : 0.f;
-      Rs[kk][ii] = (gj < L.n && gk < r) ? L.R[gj * ldp + gk] : 0.f;
-      Qs[kk][ii] = (gj < L.n && gk < r) ? L.Q[gj * L.ldq + gk] : 0.f;
-    }
-    __syncthreads();
+    const bool more = k0 + UBK < r;
+    if (more) load(k0 + UBK, pv, bv);
 #pragma unroll
     for (int kk = 0; kk < UBK; ++kk) {
-      float a[4], b[4], q[4];
+      const float4 a0 = *reinterpret_cast<const float4 *>(&As[cur][kk][ty * 4]);
+      const float4 a1 = *reinterpret_cast<const float4 *>(&As[cur][kk][64 + ty * 4]);
+      const float4 b4 = *reinterpret_cast<const float4 *>(&Rs[cur][kk][tx * 4]);
+      const float4 q4 = *reinterpret_cast<const float4 *>(&Qs[cur][kk][tx * 4]);
+      const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+      const float b[4] = {b4.x, b4.y, b4.z, b4.w}, q[4] = {q4.x, q4.y, q4.z, q4.w};
 #pragma unroll
-      for (int i = 0; i < 4; ++i) a[i] = As[kk][ty * 4 + i];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) { b[j] = Rs[kk][tx * 4 + j]; q[j] = Qs[kk][tx * 4 + j]; }
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
+      for (int i = 0; i < 8; ++i)
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           u1[i][j] = fmaf(a[i], b[j], u1[i][j]);
           u2[i][j] = fmaf(a[i], q[j], u2[i][j]);
         }
     }
+    if (more) store(cur ^ 1, pv, bv);
     __syncthreads();
+    cur ^= 1;
   }
   const float dec = 1.f - mu, c = eta * L.sqrt_m_over_n;
   float ss = 0.f;
+  const int64_t gj = j0 + tx * 4;
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int64_t gi = i0 + ty * 4 + i;
-    if (gi >= L.m) continue;
+  for (int i = 0; i < 8; ++i) {
+    const int64_t gi = i0 + (i < 4 ? ty * 4 + i : 64 + ty * 4 + (i - 4));
+    if (gi >= L.m || gj >= L.n) continue;
+    float *mp = L.M + gi * L.ldm + gj, *xp = L.X + gi * L.ldx + gj;
+    if (gj + 4 <= L.n) {
+      float4 mv = *reinterpret_cast<float4 *>(mp), xv = *reinterpret_cast<float4 *>(xp);
+      mv.x = fmaf(-dec, u1[i][0], mv.x); mv.y = fmaf(-dec, u1[i][1], mv.y);
+      mv.z = fmaf(-dec, u1[i][2], mv.z); mv.w = fmaf(-dec, u1[i][3], mv.w);
+      xv.x = fmaf(-c, u2[i][0], xv.x * keep); xv.y = fmaf(-c, u2[i][1], xv.y * keep);
+      xv.z = fmaf(-c, u2[i][2], xv.z * keep); xv.w = fmaf(-c, u2[i][3], xv.w * keep);
+      *reinterpret_cast<float4 *>(mp) = mv;
+      *reinterpret_cast<float4 *>(xp) = xv;
+      ss = fmaf(mv.x, mv.x, ss); ss = fmaf(mv.y, mv.y, ss);
+      ss = fmaf(mv.z, mv.z, ss); ss = fmaf(mv.w, mv.w, ss);
+    } else {
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int64_t gj = j0 + tx * 4 + j;
-      if (gj >= L.n) continue;
-      float *mp = L.M + gi * L.ldm + gj;
-      const float mn = fmaf(-dec, u1[i][j], *mp);
-      *mp = mn;
-      float *xp = L.X + gi * L.ldx + gj;
-      *xp = fmaf(-c, u2[i][j], *xp * keep);
-      ss = fmaf(mn, mn, ss);
+      for (int j = 0; j < 4; ++j) {
+        if (gj + j >= L.n) continue;
+        const float mn = fmaf(-dec, u1[i][j], mp[j]);
+        mp[j] = mn;
+        xp[j] = fmaf(-c, u2[i][j], xp[j] * keep);
+        ss = fmaf(mn, mn, ss);
+      }
     }
   }
   const double tot = block_sum<kUpdThreads>((double)ss, red);

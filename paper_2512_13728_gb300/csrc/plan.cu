@@ -225,10 +225,10 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
     for (int64_t r0 = 0; r0 < ly.m; r0 += rows)
       bt.push_back(make_int4(l, (int)r0, (int)std::min(rows, ly.m - r0), (int)bt.size()));
     d.bpart_cnt = (int32_t)bt.size() - d.bpart_off;
-    // 64 x 64 update tiles
+    // update tiles of the CUDA-core update kernel (FP32 mode)
     d.upart_off = (int32_t)ut.size();
-    for (int64_t ti = 0; ti < (ly.m + 63) / 64; ++ti)
-      for (int64_t tj = 0; tj < (ly.n + 63) / 64; ++tj)
+    for (int64_t ti = 0; ti < (ly.m + kUpdTileM - 1) / kUpdTileM; ++ti)
+      for (int64_t tj = 0; tj < (ly.n + kUpdTileN - 1) / kUpdTileN; ++tj)
         ut.push_back(make_int4(l, (int)ti, (int)tj, (int)ut.size()));
     d.upart_cnt = (int32_t)ut.size() - d.upart_off;
     for (int64_t cg = 0; cg < (ly.r + 31) / 32; ++cg) ct.push_back(make_int4(l, (int)cg, 0, 0));
@@ -290,8 +290,9 @@ dion_status dion_plan_create(const dion_layer *layers, int32_t num_layers, int32
       }
       const int32_t pi = (int32_t)gp[k].size();
       gp[k].push_back(q);
-      for (int64_t ti = 0; ti < (q.Mrows + 63) / 64; ++ti)
-        for (int64_t tj = 0; tj < (q.Ncols + 63) / 64; ++tj) gt[k].push_back(make_int4(pi, (int)ti, (int)tj, 0));
+      for (int64_t ti = 0; ti < (q.Mrows + kGemmTile - 1) / kGemmTile; ++ti)
+        for (int64_t tj = 0; tj < (q.Ncols + kGemmTile - 1) / kGemmTile; ++tj)
+          gt[k].push_back(make_int4(pi, (int)ti, (int)tj, 0));
     }
     o_gp[k] = cv.take<GemmProblem>(std::max<size_t>(gp[k].size(), 1));
     o_gt[k] = cv.take<int4>(std::max<size_t>(gt[k].size(), 1));
