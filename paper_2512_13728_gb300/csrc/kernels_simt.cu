@@ -916,46 +916,84 @@ void launch_chol_inv(const Shared &sh, size_t smem, int32_t pass, float near_ide
 }
 
 // ===================================================================== ColumnNormalize ===
-// Q_t[:, j] = R[:, j] / (||R[:, j]||_2 + eps_col).  Tile = {layer, 32-column group}; lane =
-// column, warps stride over rows; fp32 sums of 16 rows folded into fp64 in a fixed order.
-constexpr int kColThreads = 256;
+// Q_t[:, j] = R[:, j] / (||R[:, j]||_2 + eps_col).  Tile = {layer, 32-column group}.  A thread
+// owns 4 adjacent columns of every 32nd row (8 threads span the group's 128 bytes of a row, so a
+// warp reads 4 full row segments per instruction) and keeps 4 rows' 16-byte loads in flight;
+// fp32 sums of 16 rows folded into fp64, the 32 row-group partials added in a fixed order.
+constexpr int kColThreads = 256, kColRowGroups = kColThreads / 8, kColUnroll = 4;
 
 __global__ void __launch_bounds__(kColThreads) colnorm_kernel(Shared sh, const int4 *tiles, float eps_col) {
   const int4 t = tiles[blockIdx.x];
   DION_TILE_CHECK(t.x >= 0 && t.x < sh.num_layers && t.y >= 0 && (int64_t)t.y * 32 < sh.layers[t.x].r, sh.status);
   if (!sh.active[t.x]) return;
   const DevLayer &L = sh.layers[t.x];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int64_t j = (int64_t)t.y * 32 + lane, n = L.n, r = L.r, ldp = L.ldp;
-  __shared__ double part[kColThreads / 32][32];
+  const int quad = threadIdx.x & 7, rg = threadIdx.x >> 3;
+  const int64_t n = L.n, r = L.r, ldp = L.ldp, ldq = L.ldq;
+  const int64_t j = (int64_t)t.y * 32 + 4 * quad;  // first of this thread's columns
+  const int nc = r - j >= 4 ? 4 : r - j > 0 ? (int)(r - j) : 0;  // columns of this thread in range
+  // R rows are 16-byte aligned (ldp a multiple of 8, the workspace 256-byte aligned); Q is the
+  // caller's and takes 16-byte stores only when its base and stride allow them
+  const bool q_vec = nc == 4 && ((reinterpret_cast<uintptr_t>(L.Q) | (uintptr_t)(ldq * 4)) & 15) == 0;
+  const float *R = L.R + j;
+  auto load = [&](int64_t i) -> float4 {
+    if (i >= n || nc == 0) return make_float4(0.f, 0.f, 0.f, 0.f);
+    if (nc == 4) return *reinterpret_cast<const float4 *>(R + i * ldp);
+    const float *p = R + i * ldp;
+    return make_float4(p[0], nc > 1 ? p[1] : 0.f, nc > 2 ? p[2] : 0.f, 0.f);
+  };
+  __shared__ double part[kColRowGroups][33];
   __shared__ float inv[32];
-  double acc = 0.0;
-  if (j < r) {
-    float f = 0.f;
-    int cnt = 0;
-    for (int64_t i = warp; i < n; i += kColThreads / 32) {
-      const float v = L.R[i * ldp + j];
-      f = fmaf(v, v, f);
-      if (++cnt == 16) { acc += f; f = 0.f; cnt = 0; }
+  double a0 = 0.0, a1 = 0.0, a2 = 0.0, a3 = 0.0;
+  float f0 = 0.f, f1 = 0.f, f2 = 0.f, f3 = 0.f;
+  int cnt = 0;
+  for (int64_t i = rg; i < n; i += kColRowGroups * kColUnroll) {
+    float4 v[kColUnroll];
+#pragma unroll
+    for (int u = 0; u < kColUnroll; ++u) v[u] = load(i + (int64_t)u * kColRowGroups);
+#pragma unroll
+    for (int u = 0; u < kColUnroll; ++u) {
+      f0 = fmaf(v[u].x, v[u].x, f0);
+      f1 = fmaf(v[u].y, v[u].y, f1);
+      f2 = fmaf(v[u].z, v[u].z, f2);
+      f3 = fmaf(v[u].w, v[u].w, f3);
     }
-    acc += f;
+    if (++cnt == 16 / kColUnroll) {
+      a0 += f0; a1 += f1; a2 += f2; a3 += f3;
+      f0 = f1 = f2 = f3 = 0.f;
+      cnt = 0;
+    }
   }
-  part[warp][lane] = acc;
+  part[rg][4 * quad + 0] = a0 + f0;
+  part[rg][4 * quad + 1] = a1 + f1;
+  part[rg][4 * quad + 2] = a2 + f2;
+  part[rg][4 * quad + 3] = a3 + f3;
   __syncthreads();
-  if (warp == 0) {
+  if (threadIdx.x < 32) {
     double s = 0.0;
-    for (int w = 0; w < kColThreads / 32; ++w) s += part[w][lane];
-    inv[lane] = (float)(1.0 / (sqrt(s) + (double)eps_col));
+    for (int g = 0; g < kColRowGroups; ++g) s += part[g][threadIdx.x];
+    inv[threadIdx.x] = (float)(1.0 / (sqrt(s) + (double)eps_col));
   }
   __syncthreads();
-  if (j < r) {
-    const float c = inv[lane];
-    for (int64_t i = warp; i < n; i += kColThreads / 32) {
-      const float rv = L.R[i * ldp + j], q = rv * c;
-      L.Q[i * L.ldq + j] = q;
-      if (L.R_hi != nullptr) {  // bf16 operands of the tensor-core update (rounded to nearest)
-        L.R_hi[i * ldp + j] = __float2bfloat16_rn(rv);
-        L.Qn_hi[i * ldp + j] = __float2bfloat16_rn(q);
+  if (nc == 0) return;
+  const float c0 = inv[4 * quad], c1 = inv[4 * quad + 1], c2 = inv[4 * quad + 2], c3 = inv[4 * quad + 3];
+  float *Q = L.Q + j;
+  for (int64_t i = rg; i < n; i += kColRowGroups * kColUnroll) {
+    float4 v[kColUnroll];
+#pragma unroll
+    for (int u = 0; u < kColUnroll; ++u) v[u] = load(i + (int64_t)u * kColRowGroups);
+#pragma unroll
+    for (int u = 0; u < kColUnroll; ++u) {
+      const int64_t ii = i + (int64_t)u * kColRowGroups;
+      if (ii >= n) break;
+      const float4 q = make_float4(v[u].x * c0, v[u].y * c1, v[u].z * c2, v[u].w * c3);
+      float *dst = Q + ii * ldq;
+      if (q_vec) {
+        *reinterpret_cast<float4 *>(dst) = q;
+      } else {
+        dst[0] = q.x;
+        if (nc > 1) dst[1] = q.y;
+        if (nc > 2) dst[2] = q.z;
+        if (nc > 3) dst[3] = q.w;
       }
     }
   }
