@@ -931,9 +931,8 @@ __global__ void __launch_bounds__(kColThreads) colnorm_kernel(Shared sh, const i
   const int64_t n = L.n, r = L.r, ldp = L.ldp, ldq = L.ldq;
   const int64_t j = (int64_t)t.y * 32 + 4 * quad;  // first of this thread's columns
   const int nc = r - j >= 4 ? 4 : r - j > 0 ? (int)(r - j) : 0;  // columns of this thread in range
-  // R rows are 16-byte aligned (ldp a multiple of 8, the workspace 256-byte aligned); Q is the
-  // caller's and takes 16-byte stores only when its base and stride allow them
-  const bool q_vec = nc == 4 && ((reinterpret_cast<uintptr_t>(L.Q) | (uintptr_t)(ldq * 4)) & 15) == 0;
+  // rows of R (ldp a multiple of 8, the workspace 256-byte aligned) and of Q (the plan checks
+  // the caller's base and ldq against the 16-byte rule) start on 16-byte boundaries
   const float *R = L.R + j;
   auto load = [&](int64_t i) -> float4 {
     if (i >= n || nc == 0) return make_float4(0.f, 0.f, 0.f, 0.f);
@@ -987,7 +986,7 @@ __global__ void __launch_bounds__(kColThreads) colnorm_kernel(Shared sh, const i
       if (ii >= n) break;
       const float4 q = make_float4(v[u].x * c0, v[u].y * c1, v[u].z * c2, v[u].w * c3);
       float *dst = Q + ii * ldq;
-      if (q_vec) {
+      if (nc == 4) {
         *reinterpret_cast<float4 *>(dst) = q;
       } else {
         dst[0] = q.x;

@@ -135,6 +135,20 @@ def test_ragged_shapes_fp32(pad):
     run_per_step(RAGGED, cd.DION_PREC_FP32, dict(gate_mode=oc.GATE_ALWAYS), RAGGED.steps, TOL_FP32, pad=pad)
 
 
+# ranks whose last group of four columns is partial (r mod 4 = 3, 1, 2, 3) over one to three
+# 32-column groups: the FP32 ColumnNormalize's 16-byte and element-wise column paths
+QUADS = wl.scaled(wl.WORKLOADS["gpt160m_block_r192"], "quads", [(96, 70), (45, 130), (6, 40), (40, 7)],
+                  rank=67, steps=3)
+
+
+@pytest.mark.parametrize("pad", [0, 1])
+def test_partial_column_quads_fp32(pad):
+    import paper_2512_13728_gb300 as cd
+
+    assert QUADS.ranks() == [67, 45, 6, 7]
+    run_per_step(QUADS, cd.DION_PREC_FP32, dict(gate_mode=oc.GATE_ALWAYS), QUADS.steps, TOL_FP32, pad=pad)
+
+
 @pytest.mark.parametrize("gate", ["always", "per_layer"])
 @pytest.mark.parametrize("g_dtype", ["bf16", "fp32"])
 @pytest.mark.parametrize("pad", [0, 1])
