@@ -132,8 +132,8 @@ dion_status layout(const dion_layer *layers, int32_t L, int32_t precision, int n
   };
   lo.s_bq = pair_sched(pairs_of(lo.ftiles), [&](const int4 &t) { return (double)layers[t.x].n + 2.0 * layers[t.x].r; });
   lo.s_btp = pair_sched(pairs_of(lo.rtiles), [&](const int4 &t) { return (double)layers[t.x].m + 2.0 * layers[t.x].r; });
-  // equal cost for every tile of a layer, so that they run side by side and stream the layer's
-  // X^T from DRAM about once (the lower-triangle tiles of the first pair finish early)
+  // equal cost for every tile of a layer (at r > 256 both load two boxes per chunk), so that
+  // they run side by side and stream the layer's X^T from DRAM about once
   lo.s_gram = pair_sched(pairs_of(lo.gram_tiles), [&](const int4 &t) { return (double)layers[t.x].m * layers[t.x].r; });
   lo.s_trsm = pair_sched(pairs_of(lo.trsm_tiles), [&](const int4 &t) { return 3.0 * layers[t.x].r + 64.0; });
   for (Schedule *sc : {&lo.s_update, &lo.s_bq, &lo.s_btp, &lo.s_gram, &lo.s_trsm}) {

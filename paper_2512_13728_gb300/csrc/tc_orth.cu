@@ -2,11 +2,12 @@
 // CholeskyQR pass as kind::tf32 tcgen05 GEMMs on fp32 operands loaded by TMA (DION_PREC_BF16),
 // or as three such products per k-step on split operands (DION_PREC_BF16X3, below).
 //
-//   Gram   S = X^T X (r x r).  Tile = 128 full rows of S; K loop over m.  B = all r rows of
-//          the transposed copy X^T (r x m, K-major), which the producing kernel (the B Q
-//          epilogue or the previous TRSM) writes next to X; A = the tile's own 128 rows, read
-//          in place from B's boxes.  Every tile of a layer costs the same and streams the same
-//          X^T, so the layer's tiles run side by side and read X^T from DRAM about once.
+//   Gram   S = X^T X (r x r), lower block triangle; K loop over m.  Operands are rows of the
+//          transposed copy X^T (r x m, K-major), which the producing kernel (the B Q epilogue or
+//          the previous TRSM) writes next to X.  r <= 256: one pair tile.  r > 256: one tile for
+//          the two diagonal 256 x 256 blocks, whose A operands are read in place from their B
+//          boxes, and one for the block below the first; each loads two boxes per chunk, so a
+//          layer's tiles cost the same, run side by side and read X^T from DRAM about once.
 //   TRSM   Y = X L^{-T} (m x r).  Tile = 128 rows of X; K loop over r.  A = rows of X
 //          (K-major), B = rows of L^{-1} (K-major, lower triangular: K chunks above a column
 //          part are skipped).  Epilogue stores Y (row-major) and Y^T (transposed boxes) for
@@ -70,32 +71,69 @@ __device__ __forceinline__ OrthMaps orth_maps(const LayerMaps &mp, int pass) {
   return o;
 }
 
-// Per tile: M-dim rows [row0, row0 + 128), N columns, K extent, and whether K chunk kc
-// feeds N part p (TRSM: L^{-1} is lower triangular, so column part p needs k < 256 (p + 1)).
+// Per tile: N columns and the K extent (the Gram's parts are those of gram_tile below), and
+// whether K chunk kc feeds N part p (TRSM: L^{-1} is lower triangular, so column part p needs
+// k < 256 (p + 1)).
 template <int KIND>
 __device__ __forceinline__ void orth_dims(const DevLayer &L, int blk, uint32_t &N, int64_t &K) {
-  if (KIND == ORTH_GRAM) {
-    // rows 256 blk .. 256 blk + 255 of S: only columns below 256 (blk + 1) are read (the
-    // Cholesky and the orthogonality bound use the lower triangle of S)
-    N = min(pad16(L.r), 256u * (uint32_t)(blk + 1));
-    K = L.m;
-  } else {
-    N = pad16(L.r);
-    K = L.r;
+  (void)blk;
+  N = pad16(L.r);
+  K = (KIND == ORTH_GRAM) ? L.m : L.r;
+}
+
+// A Gram pair tile.  Part q is an accumulator of N[q] <= 256 columns at TMEM column 256 q and
+// S column 256 q (the first part of tile 1 at r > 256: column 0), fed by the B rows b_row[q] ..
+// of X^T (CTA c holds N[q] / 2 of them from b_row[q] + c N[q] / 2) and by the A rows of its 128
+// output rows: in place in B's box a_box[q], or the separate A box (rows a_row + 128 c).  Its
+// rows of S are the 128-row tile o_row[q] + c.  Output chunk j (32 columns) belongs to part j / 8.
+struct GramTile {
+  uint32_t nparts, N[2], b_row[2];
+  int a_box[2], o_row[2], a_row, nch;
+  bool sep_a;
+};
+
+__device__ __forceinline__ GramTile gram_tile(int64_t r, int p) {
+  GramTile g{};
+  const uint32_t np = pad16(r);
+  g.nch = (int)((r + 31) / 32);
+  if (np <= 256u) {  // rows and columns 0 .. r
+    g.nparts = 1;
+    g.N[0] = np;
+    g.sep_a = np != 256u;
+    g.a_box[0] = g.sep_a ? -1 : 0;
+  } else if (p == 0) {  // the diagonal blocks: rows and columns 0..255, then 256 .. r
+    g.nparts = 2;
+    g.N[0] = 256u;
+    g.N[1] = np - 256u;
+    g.b_row[1] = 256u;
+    g.o_row[1] = 2;
+    g.a_box[0] = 0;
+    g.sep_a = g.N[1] != 256u;
+    g.a_box[1] = g.sep_a ? -1 : 1;
+    g.a_row = 256;
+  } else {  // the block below the first: rows 256 .. r, columns 0..255
+    g.nparts = 1;
+    g.N[0] = 256u;
+    g.o_row[0] = 2;
+    g.sep_a = true;
+    g.a_box[0] = -1;
+    g.a_row = 256;
+    g.nch = 8;
   }
+  return g;
 }
 
 template <int KIND>
 __device__ __forceinline__ bool part_needs(int kc, uint32_t part) {
-  return KIND == ORTH_GRAM || (uint32_t)kc * 32u < 256u * (part + 1u);
+  return (uint32_t)kc * 32u < 256u * (part + 1u);
 }
 
 // Run in clusters of two CTAs with pair MMAs (cta_group::2, M = 256): CTA c of the pair owns
-// 128-row tile 2 p + c (rows of S for the Gram, rows of X for the TRSM), its A chunk, and of
-// every N part of up to 256 columns the half c of the B rows; the even CTA issues the MMAs and
-// each CTA receives its 128 rows of the accumulator in its own TMEM.  For the Gram with a
-// full 256-column part the tile's own rows of X^T are exactly the CTA's B half of part p,
-// so A is read in place.  Tile = {layer, pair p}.
+// 128 rows of each accumulator part (the TRSM: 128-row tile 2 p + c of X; the Gram: as
+// gram_tile says), its A chunk, and of every N part of up to 256 columns the half c of the B
+// rows; the even CTA issues the MMAs and each CTA receives its 128 rows of the accumulator in
+// its own TMEM.  For a diagonal block of S with a full 256-column part, the CTA's own rows of
+// X^T are exactly its B half, so A is read in place.  Tile = {layer, pair p}.
 template <int KIND, bool X3>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(X3 ? O_THREADS_X3 : O_THREADS, 1)
     tc_orth_kernel(Shared sh, const int4 *__restrict__ tiles, const int *__restrict__ off, const LayerMaps *__restrict__ maps,
@@ -184,18 +222,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(X3 ? O_THREADS_X3 : 
           }
           continue;
         }
-        const bool a_in_b = (KIND == ORTH_GRAM) && (uint32_t)t.y < nparts && half_rows(N, (uint32_t)t.y) == 128u;
+        const GramTile g = gram_tile(L.r, t.y);
         for (int kc = 0; kc < kch; ++kc, ++it) {
           const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
           if (!ab.wait(&empty[s], ph ^ 1u, sh.status)) { ok = false; break; }
           uint8_t *sA = smem + s * stage_bytes, *sB = sA + O_BOX;
-          uint32_t nb = 0;  // B boxes this chunk feeds (all, or only the lower-triangular parts)
-          for (uint32_t q = 0; q < nparts; ++q)
-            if (part_needs<KIND>(kc, q)) ++nb;
-          expect(s, (a_in_b ? 0u : 1u) + nb);
-          if (!a_in_b) load(sA, om.A, s, kc * 32, tr * 128);
-          for (uint32_t q = 0; q < nparts; ++q)
-            if (part_needs<KIND>(kc, q)) load(sB + q * O_BOX, om.B, s, kc * 32, (int)(q * 256u + rank * half_rows(N, q)));
+          expect(s, (g.sep_a ? 1u : 0u) + g.nparts);
+          if (g.sep_a) load(sA, om.A, s, kc * 32, g.a_row + (int)rank * 128);
+#pragma unroll
+          for (uint32_t q = 0; q < 2u; ++q)
+            if (q < g.nparts) load(sB + q * O_BOX, om.B, s, kc * 32, (int)(g.b_row[q] + rank * (g.N[q] / 2u)));
         }
       }
       // drain: the last stages' loads have landed and been consumed (their stage was freed)
@@ -253,14 +289,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(X3 ? O_THREADS_X3 : 
         }
         continue;
       }
-      const bool a_in_b = (KIND == ORTH_GRAM) && (uint32_t)t.y < nparts && half_rows(N, (uint32_t)t.y) == 128u;
+      const GramTile g = gram_tile(L.r, t.y);
       for (int kc = 0; kc < kch; ++kc, ++it) {
         const uint32_t s = it % nstages, ph = (it / nstages) & 1u;
         if (!named_and(2, 128, ab.wait(&full[s], ph, sh.status))) { ok = false; break; }
         uint8_t *sA = smem + s * stage_bytes, *sB = sA + O_BOX;
-        if (!a_in_b) split_box(sA);
-        for (uint32_t q = 0; q < nparts; ++q)
-          if (part_needs<KIND>(kc, q)) split_box(sB + q * O_BOX);
+        if (g.sep_a) split_box(sA);
+#pragma unroll
+        for (uint32_t q = 0; q < 2u; ++q)
+          if (q < g.nparts) split_box(sB + q * O_BOX);
         report(s);
       }
     }
@@ -306,7 +343,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(X3 ? O_THREADS_X3 : 
           }
           continue;
         }
-        const bool a_in_b = (KIND == ORTH_GRAM) && (uint32_t)t.y < nparts && half_rows(N, (uint32_t)t.y) == 128u;
+        const GramTile g = gram_tile(L.r, t.y);
         if (!ab.wait(acc_empty, (tcount & 1u) ^ 1u, sh.status)) break;
         tc_fence_after();
         for (int kc = 0; kc < kch; ++kc, ++it) {
@@ -314,13 +351,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(X3 ? O_THREADS_X3 : 
           if (!ab.wait(X3 ? &conv[s] : &full[s], ph, sh.status)) { ok = false; break; }
           tc_fence_after();
           const uint32_t aB = smem_u32(smem + s * stage_bytes), bB = aB + O_BOX;
-          const uint32_t aSrc = a_in_b ? bB + (uint32_t)t.y * O_BOX : aB;
 #pragma unroll
           for (int k8 = 0; k8 < 4; ++k8) {
-            const uint64_t ad = smem_desc_sw128(aSrc + k8 * 32, 0, 1024);
-            for (uint32_t q = 0; q < nparts; ++q) {
-              if (!part_needs<KIND>(kc, q)) continue;
-              const uint32_t idesc = idesc_tf32(256, 2u * half_rows(N, q), false, false);
+#pragma unroll
+            for (uint32_t q = 0; q < 2u; ++q) {
+              if (q >= g.nparts) break;
+              const uint32_t aSrc = g.a_box[q] >= 0 ? bB + (uint32_t)g.a_box[q] * O_BOX : aB;
+              const uint64_t ad = smem_desc_sw128(aSrc + k8 * 32, 0, 1024);
+              const uint32_t idesc = idesc_tf32(256, g.N[q], false, false);
               const uint64_t bd = smem_desc_sw128(bB + q * O_BOX + k8 * 32, 0, 1024);
               // the first chunk that feeds a part starts its accumulation
               umma_pair_tf32(tmem + q * 256u, ad, bd, idesc, (kc | k8) ? 1u : 0u);
@@ -353,8 +391,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(X3 ? O_THREADS_X3 : 
       int64_t K;
       orth_dims<KIND>(L, t.y, N, K);
       const int tr = 2 * t.y + (int)rank;
-      const bool real = (int64_t)tr * 128 < (KIND == ORTH_GRAM ? L.r : L.m);  // not the pair's empty second tile
-      const int nch = real ? (int)((min((int64_t)N, L.r) + 31) / 32) : 0;
+      const bool real = (int64_t)tr * 128 < L.m;  // TRSM: not the pair's empty second tile
+      const GramTile g = gram_tile(L.r, KIND == ORTH_GRAM ? t.y : 0);
+      const int nch = (KIND == ORTH_GRAM) ? g.nch : real ? (int)((min((int64_t)N, L.r) + 31) / 32) : 0;
       // The solve that ends Orthogonalize writes only the bf16 copy of P that R = B^T P and the
       // update read: pass 1 unless a shifted retry asked for pass 2, and pass 2 itself.
       const bool final_pass = (KIND == ORTH_TRSM) && (pass == 2 || (pass == 1 && !sh.orth_shifted[t.x]));
@@ -426,6 +465,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(X3 ? O_THREADS_X3 : 
           }
         } else {
           for (int j = jb; j < je; ++j) {
+            // the Gram's chunk j belongs to part j / 8, rows of S from tile o_row + rank; the
+            // rows of a CTA past r are not stored (the same for every epilogue thread)
+            const int otr = (KIND == ORTH_GRAM) ? (j >= 8 ? g.o_row[1] : g.o_row[0]) + (int)rank : tr;
+            if (KIND == ORTH_GRAM && (int64_t)otr * 128 >= L.r) continue;
             const bool store_t = (KIND == ORTH_TRSM);  // transposed copy: the next Gram's operand
             const uint32_t eb = ecount & 1u;
             uint8_t *box = stg + eb * 2 * O_BOX, *tbox = box + O_BOX + lg * O_TBOX;
@@ -449,7 +492,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(X3 ? O_THREADS_X3 : 
             fence_async_smem();
             named_sync(1, 128);
             if (leader) {
-              tma_store_2d(om.out, box, j * 32, tr * 128);
+              tma_store_2d(om.out, box, j * 32, otr * 128);
               if (store_t)
                 for (int w4 = 0; w4 < 4; ++w4)
                   if ((int64_t)tr * 128 + w4 * 32 < L.m)
