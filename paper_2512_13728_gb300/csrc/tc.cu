@@ -305,9 +305,11 @@ cudaError_t init(const TcLayout &lo, char *base, const DevLayer *dl, int32_t L, 
   // BF16X3: every stage also holds the lo boxes its converters write
   const uint32_t ostage = (x3 ? 2u : 1u) * 128u * 32u * 4u * (1u + o_parts);
   const int ostages = (int)std::min<uint32_t>(4u, budget / ostage);
-  // TRSM: one 256-column part per sub-tile, so a stage holds the A box and one B box
+  // TRSM: one 256-column part per sub-tile, so a stage holds the A box and one B box; up to 5
+  // stages (the solve gains from the bytes in flight: the final pass 0.294 -> 0.279 ms on the
+  // 1.3B stack with 5 against 4)
   const uint32_t tstage = (x3 ? 2u : 1u) * 128u * 32u * 4u * 2u;
-  const int tstages = (int)std::min<uint32_t>(4u, budget / tstage);
+  const int tstages = (int)std::min<uint32_t>(5u, budget / tstage);
   if (stages < 2 || ostages < 2 || tstages < 2) return cudaErrorInvalidValue;
   tp->nb64 = nb64;
   tp->bq_boxes = bq_boxes;
