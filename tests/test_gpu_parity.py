@@ -309,11 +309,12 @@ def test_gpt160m_block_r192_bf16_50_steps(prec):
     print(prec, "block, 50 steps, worst", worst)
 
 
-@pytest.mark.parametrize("rank", [300, 400])
+@pytest.mark.parametrize("rank", [260, 300, 400, 500])
 def test_rank_between_256_and_512_bf16(rank):
     """256 < r < 512 in the tensor-core mode: the TRSM's second 256-column sub-tile is partial
-    (r = 400: 144 columns; r = 300, padded to 304: 48), and the Gram's second row block of S and
-    the B Q / B^T P accumulators are ragged too; ragged m and n over several tiles."""
+    (r = 400: 144 columns; r = 300, padded to 304: 48; r = 260: 16), the Gram's second diagonal
+    block is ragged (its A operand from its own box below r = 497, read in place from the B box at
+    r = 500), and so are the B Q / B^T P accumulators; ragged m and n over several tiles."""
     import paper_2512_13728_gb300 as cd
 
     w = wl.scaled(wl.WORKLOADS["gpt160m_block_r192"], f"r{rank}", [(1200, 1100), (1100, 1200), (900, 700)],
