@@ -565,6 +565,14 @@ void launch_gemm(const Shared &sh, const GemmProblem *probs, const int4 *tiles, 
 constexpr int kCholThreads = 512;
 constexpr int kFoBatch = 8;  // 16-byte groups each thread has in flight in the first-order factor
 
+// Row i and 16-byte column group j4 of flat group g of an r x r4 grid (g < 2^32: a 32-bit
+// division, several times cheaper than the 64-bit one, which dominated the loops below).
+__device__ __forceinline__ void fo_group(int64_t g, int r4, int &i, int &j4) {
+  const uint32_t gu = (uint32_t)g, q = gu / (uint32_t)r4;
+  i = (int)q;
+  j4 = (int)(gu - q * (uint32_t)r4);
+}
+
 // Column c of Y lives at ysw(c): bit 2 flips when bit 5 is set, so the two 16-byte halves of
 // an 8-column group swap in every other 32-column stretch.  Eight consecutive groups read by
 // one quarter-warp then fall on distinct banks.
@@ -810,7 +818,8 @@ __global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, in
 #pragma unroll
       for (int u = 0; u < kFoBatch; ++u) {
         const int64_t g = g0 + (int64_t)u * kCholThreads;
-        const int i = (int)(g / r4), j4 = (int)(g % r4);
+        int i, j4;
+        fo_group(g, r4, i, j4);
         v[u] = (g < groups && 4 * j4 <= i) ? *reinterpret_cast<const float4 *>(S + (int64_t)i * ls + 4 * j4)
                                            : make_float4(0.f, 0.f, 0.f, 0.f);
       }
@@ -818,7 +827,8 @@ __global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, in
 #pragma unroll
       for (int u = 0; u < kFoBatch; ++u) {
         const int64_t g = g0 + (int64_t)u * kCholThreads;
-        const int i = (int)(g / r4), j4 = (int)(g % r4);
+        int i, j4;
+        fo_group(g, r4, i, j4);
         const float ve[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
@@ -845,7 +855,8 @@ __global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, in
 #pragma unroll
         for (int u = 0; u < kFoBatch; ++u) {
           const int64_t g = g0 + (int64_t)u * kCholThreads;
-          const int i = (int)(g / r4), j4 = (int)(g % r4);
+          int i, j4;
+        fo_group(g, r4, i, j4);
           v[u] = (g < groups && 4 * j4 <= i) ? *reinterpret_cast<const float4 *>(S + (int64_t)i * ls + 4 * j4)
                                              : make_float4(0.f, 0.f, 0.f, 0.f);
         }
@@ -853,7 +864,8 @@ __global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, in
         for (int u = 0; u < kFoBatch; ++u) {
           const int64_t g = g0 + (int64_t)u * kCholThreads;
           if (g >= groups) break;
-          const int i = (int)(g / r4), j4 = (int)(g % r4);
+          int i, j4;
+        fo_group(g, r4, i, j4);
           float o[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
 #pragma unroll
           for (int c = 0; c < 4; ++c) {
