@@ -565,12 +565,17 @@ void launch_gemm(const Shared &sh, const GemmProblem *probs, const int4 *tiles, 
 constexpr int kCholThreads = 512;
 constexpr int kFoBatch = 8;  // 16-byte groups each thread has in flight in the first-order factor
 
-// Row i and 16-byte column group j4 of flat group g of an r x r4 grid (g < 2^32: a 32-bit
-// division, several times cheaper than the 64-bit one, which dominated the loops below).
-__device__ __forceinline__ void fo_group(int64_t g, int r4, int &i, int &j4) {
-  const uint32_t gu = (uint32_t)g, q = gu / (uint32_t)r4;
-  i = (int)q;
-  j4 = (int)(gu - q * (uint32_t)r4);
+// Row i and 16-byte column group j4 (4 j4 <= i) of flat group p of a lower triangle whose rows
+// 4 b .. 4 b + 3 hold b + 1 groups each, 2 b (b + 1) groups before them (p < 2^24: the fp32
+// estimate of b is off by at most one, corrected in integers; 32-bit division).
+__device__ __forceinline__ void lower_group(int64_t p, int &i, int &j4) {
+  const uint32_t pu = (uint32_t)p;
+  uint32_t b = (uint32_t)((sqrtf(2.f * (float)pu + 1.f) - 1.f) * 0.5f);
+  while (2u * (b + 1u) * (b + 2u) <= pu) ++b;
+  while (b > 0u && 2u * b * (b + 1u) > pu) --b;
+  const uint32_t off = pu - 2u * b * (b + 1u), q = off / (b + 1u);
+  i = (int)(4u * b + q);
+  j4 = (int)(off - q * (b + 1u));
 }
 
 // Column c of Y lives at ysw(c): bit 2 flips when bit 5 is set, so the two 16-byte halves of
@@ -806,34 +811,33 @@ __global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, in
 
   if (pass >= 1) {
     // ||E||_F^2 from the lower triangle (E symmetric), fixed-order reduction.  The 16-byte
-    // groups (i, j4) of the r x ceil(r / 4) grid are taken in a flat order, consecutive threads
-    // on consecutive groups of a row, kFoBatch groups per thread in flight (a row's padding up to
-    // the next multiple of 4 columns lies inside ls and is masked; groups above the diagonal are
-    // not loaded)
-    const int r4 = (r + 3) / 4;
-    const int64_t groups = (int64_t)r * r4;
+    // groups (i, j4) on or below the diagonal (4 j4 <= i) are taken in a flat order (rows 4 b ..
+    // 4 b + 3 hold b + 1 groups each), consecutive threads on consecutive groups, kFoBatch
+    // groups per thread in flight, every one of them a load (a group's columns past the
+    // diagonal are masked)
+    const int r4 = (r + 3) / 4, nb4 = r / 4;
+    const int64_t lgroups = 2ll * nb4 * (nb4 + 1) + (int64_t)(r % 4) * (nb4 + 1);
     double fs = 0.0;
-    for (int64_t g0 = tid; g0 < groups; g0 += (int64_t)kCholThreads * kFoBatch) {
+    for (int64_t g0 = tid; g0 < lgroups; g0 += (int64_t)kCholThreads * kFoBatch) {
       float4 v[kFoBatch];
+      int gi[kFoBatch], gj[kFoBatch];
 #pragma unroll
       for (int u = 0; u < kFoBatch; ++u) {
         const int64_t g = g0 + (int64_t)u * kCholThreads;
-        int i, j4;
-        fo_group(g, r4, i, j4);
-        v[u] = (g < groups && 4 * j4 <= i) ? *reinterpret_cast<const float4 *>(S + (int64_t)i * ls + 4 * j4)
-                                           : make_float4(0.f, 0.f, 0.f, 0.f);
+        lower_group(g, gi[u], gj[u]);
+        v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (g < lgroups) v[u] = *reinterpret_cast<const float4 *>(S + (int64_t)gi[u] * ls + 4 * gj[u]);
+        else gi[u] = -1;  // past the last group: every column masked below
       }
       float a = 0.f;
 #pragma unroll
       for (int u = 0; u < kFoBatch; ++u) {
-        const int64_t g = g0 + (int64_t)u * kCholThreads;
-        int i, j4;
-        fo_group(g, r4, i, j4);
+        const int i = gi[u];
         const float ve[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
-          const int j = 4 * j4 + c;
-          const float e = (g < groups && j <= i) ? ve[c] - (i == j ? 1.f : 0.f) : 0.f;
+          const int j = 4 * gj[u] + c;
+          const float e = (j <= i) ? ve[c] - (i == j ? 1.f : 0.f) : 0.f;
           a = fmaf((j < i ? 2.f : 1.f) * e, e, a);
         }
       }
@@ -848,24 +852,22 @@ __global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, in
       lam = power_norm_sym(S, r, ls, Y, ldy);
     }
     if (isfinite(lam) && 1.5f * lam < near_identity) {
-      // the same flat order over the groups of every row; 16-byte loads and stores (a group
-      // that straddles column r is stored element-wise)
-      for (int64_t g0 = tid; g0 < groups; g0 += (int64_t)kCholThreads * kFoBatch) {
+      // the groups on or below the diagonal in the same order, 16-byte loads and stores (a group
+      // that straddles column r is stored element-wise), then zeros above them, a warp per row
+      for (int64_t g0 = tid; g0 < lgroups; g0 += (int64_t)kCholThreads * kFoBatch) {
         float4 v[kFoBatch];
+        int gi[kFoBatch], gj[kFoBatch];
 #pragma unroll
         for (int u = 0; u < kFoBatch; ++u) {
           const int64_t g = g0 + (int64_t)u * kCholThreads;
-          int i, j4;
-        fo_group(g, r4, i, j4);
-          v[u] = (g < groups && 4 * j4 <= i) ? *reinterpret_cast<const float4 *>(S + (int64_t)i * ls + 4 * j4)
-                                             : make_float4(0.f, 0.f, 0.f, 0.f);
+          lower_group(g, gi[u], gj[u]);
+          v[u] = g < lgroups ? *reinterpret_cast<const float4 *>(S + (int64_t)gi[u] * ls + 4 * gj[u])
+                             : make_float4(0.f, 0.f, 0.f, 0.f);
         }
 #pragma unroll
         for (int u = 0; u < kFoBatch; ++u) {
-          const int64_t g = g0 + (int64_t)u * kCholThreads;
-          if (g >= groups) break;
-          int i, j4;
-        fo_group(g, r4, i, j4);
+          if (g0 + (int64_t)u * kCholThreads >= lgroups) break;
+          const int i = gi[u], j4 = gj[u];
           float o[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
 #pragma unroll
           for (int c = 0; c < 4; ++c) {
@@ -879,6 +881,16 @@ __global__ void __launch_bounds__(kCholThreads, 1) chol_inv_kernel(Shared sh, in
 #pragma unroll
             for (int c = 0; c < 4; ++c)
               if (4 * j4 + c < r) dst[c] = o[c];
+          }
+        }
+      }
+      for (int i = warp; i < r; i += kCholThreads / 32) {
+        for (int j4 = i / 4 + 1 + lane; j4 < r4; j4 += 32) {
+          float *dst = Li + (int64_t)i * ls + 4 * j4;
+          if (4 * j4 + 4 <= r) {
+            *reinterpret_cast<float4 *>(dst) = make_float4(0.f, 0.f, 0.f, 0.f);
+          } else {
+            for (int c = 0; 4 * j4 + c < r; ++c) dst[c] = 0.f;
           }
         }
       }
