@@ -7,7 +7,6 @@ DION_GATE_PER_LAYER the layers are independent, so a sampled step is exact).  Ev
 still checked for the properties that hold at any size: each flag is RMMC_l > tau_l and the
 global flag is max_l RMMC_l > tau_0, bit for bit.
 """
-import math
 
 import numpy as np
 import pytest

@@ -6,7 +6,6 @@ are compared: sync flags and the global flag bit-exact, RMMC to fp32-accumulatio
 M, X, Q by relative Frobenius error (1e-4 for fp32 arithmetic; 2e-2 where bf16 operands
 are used, the tolerances the design states for fp32 and bf16 inputs).
 """
-import math
 
 import numpy as np
 import pytest

@@ -7,7 +7,6 @@ tolerance, RMMC to 1e-5), and the device's RMMC is checked against Theorem 1's d
 the exact momentum-norm ratio |sqrt((1 - B_t - eta kappa)^2 + rho^2) - 1| (to the mode's
 accuracy) and |eta kappa + B_t| within the perpendicular-gradient term.
 """
-import numpy as np
 import pytest
 import torch
 
